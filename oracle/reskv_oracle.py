@@ -1,0 +1,463 @@
+"""fp64 CPU oracle for ResKV construction and shared-softmax decode.
+
+TEST INFRASTRUCTURE ONLY.  This module is a plain, slow, obviously-correct
+restatement of the paper "ResKV: Reconstructing Omitted Attention
+Contributions for Fixed-Budget KV Cache Compression" in numpy float64.  Only
+``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` / reference
+leg of ``bench.py`` may import it.  It shares no code with the CUDA library
+(``paper_2607_29591_gb300``) and imports nothing from it; the product path
+never calls it.
+
+Every function follows one passage of the paper, named in its docstring
+(section, equation label or algorithm).  Inputs arrive as bf16 values that are
+upcast exactly to float64; all arithmetic is float64.  Where the paper is
+silent the reading taken is stated at the function (the same list is kept in
+the project's design notes):
+
+* observation queries: the caller supplies ``n_obs`` rows per query head, the
+  first ``n_fit`` are the fit part and the last ``n_val`` the validation part
+  (Sec. 5.5.1), and every observation query attends to all ``s`` tokens;
+* SnapKV scores: per fit query and head, softmax over all tokens; the weights
+  are averaged over the GQA group and summed over fit queries, then average
+  pooled with a zero-padded window of ``pool`` (5) tokens (App. B.2);
+* query-free scoring (no observation window): ``s_p = ||k_p||^2`` -- a build
+  choice, the paper defines no such rule;
+* ranking ties go to the lower token index; Lloyd assignment ties go to the
+  lower centre index; an empty cluster keeps its centre and ends with count 0
+  (log-count ``-inf``: the slot contributes nothing);
+* candidate budgets ``r = floor(ratio * b)`` over the ratio grid, duplicates
+  and zero dropped; ``argmin`` ties go to the smaller ``r``; the residual is
+  enabled only on a strict improvement (Eq. valproxy);
+* stored residual entries are rounded to bf16 (round-to-nearest-even); the
+  validation loss is evaluated on the stored (rounded) entries;
+* the validation loss averages over validation queries and the G query heads
+  of the KV head.
+
+Parity status: every function here is pinned by ``tests/test_oracle_pins.py``
+against closed forms, fixed points or hand-computed fixtures; none is
+"parity unpinned".  The end-to-end accuracy numbers of the paper (RULER,
+LongBench) are not reproducible here (no model weights or benchmark data).
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import Optional, Sequence
+
+import numpy as np
+
+# ---------------------------------------------------------------------------
+# Hyper-parameters (App. B, "ResKV Construction Settings")
+# ---------------------------------------------------------------------------
+
+GATE_DYNAMIC = 0
+GATE_FIXED = 1
+
+SCORE_OBS_POOL = 0
+SCORE_KEYNORM = 1
+
+
+@dataclass
+class OracleConfig:
+    """Construction / decode settings for one (layer, KV head) unit.
+
+    Defaults are the paper's (App. B "ResKV Construction Settings"; App. B.2
+    SnapKV: window protection 64, pooling kernel 5).
+    """
+
+    budget: int                      # b, slots per (layer, KV head)   (Sec. 3.2)
+    recent_window: int = 64          # |P|, protected recent tokens   (Eq. main_selection)
+    n_fit: int = 96                  # fitting queries                 (Sec. 5.5.1)
+    n_val: int = 32                  # validation queries              (Sec. 5.5.1)
+    pool_kernel: int = 5             # SnapKV average pooling          (App. B.2)
+    score_mode: int = SCORE_OBS_POOL
+    grid_ratios: Sequence[float] = (0.0, 0.05, 0.10, 0.15, 0.20)  # App. B
+    lloyd_iters: int = 4             # App. B
+    delta: float = 0.01              # Eq. valproxy margin
+    beta: float = 1.0                # count exponent in the residual logit (App. B)
+    residual_override: Optional[int] = None  # fixed r, bypasses the proxy
+    gate_mode: int = GATE_DYNAMIC
+    tau: float = 0.25                # Eq. gate threshold (App. B)
+    alpha: float = 12.0              # sigmoid slope = 1/T_g (App. B)
+    g_min: float = 0.0               # minimum gate (App. B)
+    g_fixed: float = 1.0             # gate value when gate_mode == GATE_FIXED
+
+
+# ---------------------------------------------------------------------------
+# bf16 helpers (storage format of the cache; not part of the method)
+# ---------------------------------------------------------------------------
+
+def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Exact upcast of bf16 bit patterns (uint16) to float64."""
+    b = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << 16
+    return b.view(np.float32).astype(np.float64)
+
+
+def round_to_bf16(x: np.ndarray) -> np.ndarray:
+    """Round float64 values to the nearest bf16 value, ties to even.
+
+    Direct rounding from float64 (8 significant bits kept), written with
+    frexp/ldexp so that no float32 double rounding occurs.  Zero stays zero;
+    the values rounded here (cluster means of bf16 inputs) lie far inside the
+    bf16 normal range.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    mant, expo = np.frexp(x)                 # x = mant * 2**expo, 0.5 <= |mant| < 1
+    scaled = np.ldexp(mant, 8)               # 8 significant bits in the integer part
+    rounded = np.rint(scaled)                # numpy rint: round half to even
+    return np.ldexp(rounded, expo - 8)
+
+
+# ---------------------------------------------------------------------------
+# Attention statistics (Sec. 3.1, Sec. 4.2)
+# ---------------------------------------------------------------------------
+
+def logits(q: np.ndarray, K: np.ndarray) -> np.ndarray:
+    """a_p(q) = <q, k_p> / sqrt(d)  (Sec. 4.1, Eq. expand; Sec. 5.4)."""
+    d = K.shape[-1]
+    return (K @ q) / np.sqrt(d)
+
+
+def attention_full(q: np.ndarray, K: np.ndarray, V: np.ndarray) -> np.ndarray:
+    """o_S(q) = softmax(q K^T / sqrt(d)) V over all rows  (Eq. attn)."""
+    a = logits(q, K)
+    w = np.exp(a - a.max())
+    return (w @ V) / w.sum()
+
+
+def zn_stats(q: np.ndarray, K: np.ndarray, V: np.ndarray, shift: float = 0.0):
+    """Unnormalised statistics Z_T(q), N_T(q) of a token set  (Eq. zn).
+
+    Returned as e^{-shift} Z and e^{-shift} N so that callers can keep a common
+    scale between several sets without overflow.
+    """
+    a = logits(q, K)
+    e = np.exp(a - shift)
+    return e.sum(), e @ V
+
+
+# ---------------------------------------------------------------------------
+# Token scoring (App. B.2 SnapKV rule; Alg. 1 step 2)
+# ---------------------------------------------------------------------------
+
+def scores_obs_pool(K: np.ndarray, Qfit: np.ndarray, pool: int) -> np.ndarray:
+    """SnapKV-style token scores from the fit observation queries.
+
+    ``K``: [s, d]; ``Qfit``: [G, n_fit, d] (the fit rows of the G query heads
+    that share this KV head).  For every fit query and head the attention
+    weights over all s tokens are formed; they are averaged over the G heads
+    (GQA: one score per KV head, App. B) and summed over fit queries; the sum
+    is average pooled with a zero-padded window of ``pool`` tokens.
+    """
+    G, n_fit, d = Qfit.shape
+    s = K.shape[0]
+    if pool < 1 or pool % 2 == 0:
+        raise ValueError("pool kernel must be a positive odd integer")
+    acc = np.zeros(s, dtype=np.float64)
+    for g in range(G):
+        for t in range(n_fit):
+            a = logits(Qfit[g, t], K)
+            w = np.exp(a - a.max())
+            acc += (w / w.sum()) / G
+    half = pool // 2
+    padded = np.concatenate([np.zeros(half), acc, np.zeros(half)])
+    pooled = np.zeros(s, dtype=np.float64)
+    for j in range(pool):                      # (A_{p-h} + ... + A_{p+h}) / pool
+        pooled += padded[j:j + s]
+    return pooled / pool
+
+
+def scores_keynorm(K: np.ndarray) -> np.ndarray:
+    """Query-free score s_p = ||k_p||^2 (a build choice; the paper has none)."""
+    return np.sum(K * K, axis=1)
+
+
+# ---------------------------------------------------------------------------
+# Main-cache selection (Sec. 5.2, Eq. main_selection)
+# ---------------------------------------------------------------------------
+
+def rank_evictable(scores: np.ndarray, recent: int) -> np.ndarray:
+    """Positions of S \\ P ordered by score, highest first; ties -> lower index.
+
+    P is the protected window of the last ``recent`` positions.
+    """
+    s = scores.shape[0]
+    n = max(s - recent, 0)
+    pos = np.arange(n)
+    # lexsort sorts by the last key first: primary = -score, secondary = index
+    order = np.lexsort((pos, -scores[:n]))
+    return pos[order]
+
+
+def select_main(ranked: np.ndarray, s: int, recent: int, m: int):
+    """M = P u Top_{m-|P|}(s), E = S \\ M  (Eq. main_selection).
+
+    Returns (M as ascending positions, E in rank order).  E in rank order is
+    what Lloyd initialisation needs (App. B: initial centres are the evicted
+    keys with the highest scores).
+    """
+    n_p = min(recent, s)
+    take = m - n_p
+    if take < 0:
+        raise ValueError("main budget smaller than the protected window")
+    P = np.arange(s - n_p, s)
+    top = ranked[:take]
+    M = np.sort(np.concatenate([top, P]))
+    E = ranked[take:]
+    return M, E
+
+
+def candidate_budgets(budget: int, ratios: Sequence[float]) -> list:
+    """Residual candidates r = floor(ratio * b) > 0, distinct, ascending (App. B)."""
+    rs = set()
+    for ratio in ratios:
+        r = int(np.floor(float(np.float32(ratio)) * budget))
+        if r > 0:
+            rs.add(r)
+    return sorted(rs)
+
+
+# ---------------------------------------------------------------------------
+# Residual construction (Sec. 5.3, Eq. summary, Eq. residual_partition)
+# ---------------------------------------------------------------------------
+
+def lloyd_assign(KE: np.ndarray, centers: np.ndarray) -> np.ndarray:
+    """argmin_j ||k_p - c_j||^2 for every row of KE; ties -> lowest j.
+
+    The squared distance is evaluated as ||c_j||^2 - 2<k_p, c_j> (+ ||k_p||^2,
+    the same for every j and omitted) with one float64 matrix product.  A
+    centre that is bit-identical to an earlier one can never win (exact ties
+    go to the lower index), so such duplicates are excluded explicitly.
+    """
+    cn = np.sum(centers * centers, axis=1)
+    dist = cn[None, :] - 2.0 * (KE @ centers.T)
+    r = centers.shape[0]
+    if r > 1:
+        _, first = np.unique(centers, axis=0, return_index=True)
+        dup = np.ones(r, dtype=bool)
+        dup[first] = False
+        if dup.any():
+            dist[:, dup] = np.inf
+    return np.argmin(dist, axis=1)             # first minimum = lowest index
+
+
+def lloyd_residual(K: np.ndarray, V: np.ndarray, E: np.ndarray, r: int, iters: int):
+    """Residual entries of E by Lloyd's algorithm (Sec. 5.3; App. B).
+
+    ``E`` lists the evicted positions in rank order; the initial centres are
+    the keys of its first ``r`` entries (the highest-scored evicted tokens).
+    ``iters`` rounds of (assign every evicted key to its nearest centre, move
+    each non-empty centre to the mean of its members).  An empty cluster keeps
+    its centre.  Returns the unrounded entries (k_bar, v_bar, c) of Eq. summary
+    for the final assignment: k_bar_j = mean key, v_bar_j = mean value,
+    c_j = member count.
+    """
+    if r <= 0:
+        d = K.shape[1]
+        return np.zeros((0, d)), np.zeros((0, V.shape[1])), np.zeros(0, dtype=np.int64)
+    if E.shape[0] < r:
+        raise ValueError("fewer evicted tokens than residual entries")
+    if iters < 1:
+        raise ValueError("at least one Lloyd iteration is required")
+    KE = K[E]
+    VE = V[E]
+    centers = KE[:r].copy()
+    for _ in range(iters):
+        assign = lloyd_assign(KE, centers)
+        for j in range(r):
+            members = assign == j
+            if members.any():
+                centers[j] = KE[members].mean(axis=0)
+    counts = np.bincount(assign, minlength=r).astype(np.int64)
+    vbar = np.zeros((r, V.shape[1]))
+    for j in range(r):
+        members = assign == j
+        if members.any():
+            vbar[j] = VE[members].mean(axis=0)
+    return centers, vbar, counts
+
+
+def log_counts(counts: np.ndarray, beta: float) -> np.ndarray:
+    """beta * log c_j, with log 0 = -inf (an empty entry carries no mass)."""
+    out = np.full(counts.shape, -np.inf)
+    nz = counts > 0
+    out[nz] = beta * np.log(counts[nz].astype(np.float64))
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Dynamic gate (Sec. 5.5.2, Eq. gate) and shared-softmax decode (Sec. 5.4)
+# ---------------------------------------------------------------------------
+
+def sigmoid(x: float) -> float:
+    return 1.0 / (1.0 + np.exp(-x))
+
+
+def dynamic_gate(p_max: float, tau: float, alpha: float, g_min: float) -> float:
+    """g = max(g_min, sigmoid((tau - p_max) / T_g)) with T_g = 1/alpha (Eq. gate)."""
+    return max(g_min, sigmoid(alpha * (tau - p_max)))
+
+
+def shared_softmax_decode(q, Kmain, Vmain, Kres, Vres, logc, cfg: OracleConfig,
+                          return_stats: bool = False):
+    """One decode query of one query head (Alg. 2; Eqs. residual_logit, reskv_den,
+    reskv_num, reskv; Eq. gate).
+
+    a_p = <q,k_p>/sqrt(d) over the main cache; p_max = max_p softmax_M(a)_p;
+    g = gate(p_max); residual logits a~_j = <q, k_bar_j>/sqrt(d) + log c_j + log g;
+    Z^ = sum_M e^{a_p} + sum_R e^{a~_j};  N^ = sum_M e^{a_p} v_p + sum_R e^{a~_j} v_bar_j;
+    o^ = N^ / Z^.  With R empty (or g = 0) this is eviction attention (Eq. evict).
+    """
+    a = logits(q, Kmain)
+    mu_m = a.max()
+    e_main = np.exp(a - mu_m)
+    p_max = 1.0 / e_main.sum()                 # largest main-only weight: e^0 / sum
+    if cfg.gate_mode == GATE_DYNAMIC:
+        g = dynamic_gate(p_max, cfg.tau, cfg.alpha, cfg.g_min)
+    else:
+        g = cfg.g_fixed
+    log_g = np.log(g) if g > 0 else -np.inf
+    if Kres.shape[0] > 0:
+        at = logits(q, Kres) + logc + log_g
+    else:
+        at = np.zeros(0)
+    finite = at[np.isfinite(at)]
+    mu = max(mu_m, finite.max()) if finite.size else mu_m
+    w_main = np.exp(a - mu)
+    w_res = np.exp(at - mu)                    # -inf logits (c = 0 or g = 0) give 0
+    Z = w_main.sum() + w_res.sum()
+    N = w_main @ Vmain + (w_res @ Vres if Kres.shape[0] > 0 else 0.0)
+    out = N / Z
+    if return_stats:
+        return out, dict(p_max=p_max, g=g, Z=Z, N=N, shift=mu)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Construction (Alg. 1) with the validation proxy (Sec. 5.5.1)
+# ---------------------------------------------------------------------------
+
+@dataclass
+class UnitCache:
+    """The compressed cache of one (layer, KV head) unit."""
+
+    main_pos: np.ndarray          # [m] ascending original positions
+    kmain: np.ndarray             # [m, d] exact keys
+    vmain: np.ndarray             # [m, d] exact values
+    kbar: np.ndarray              # [r, d] stored (bf16-rounded) mean keys
+    vbar: np.ndarray              # [r, d] stored (bf16-rounded) mean values
+    counts: np.ndarray            # [r] populations c_j
+    logc: np.ndarray              # [r] beta * log c_j
+    r: int
+    # diagnostics for tests
+    scores: Optional[np.ndarray] = None
+    ranked: Optional[np.ndarray] = None
+    losses: dict = field(default_factory=dict)
+    init_order: Optional[np.ndarray] = None   # E of the chosen r in rank order
+
+
+def build_candidate(K, V, ranked, cfg: OracleConfig, r: int) -> UnitCache:
+    """Main cache M_r and residual entries for one candidate r (Alg. 1 steps 5-6)."""
+    s = K.shape[0]
+    m = min(cfg.budget - r, s)
+    if r == 0:
+        m = min(cfg.budget, s)
+    M, E = select_main(ranked, s, cfg.recent_window, m)
+    kbar, vbar, counts = lloyd_residual(K, V, E, r, cfg.lloyd_iters)
+    kbar_s = round_to_bf16(kbar)
+    vbar_s = round_to_bf16(vbar)
+    return UnitCache(main_pos=M, kmain=K[M], vmain=V[M], kbar=kbar_s, vbar=vbar_s,
+                     counts=counts, logc=log_counts(counts, cfg.beta), r=r,
+                     init_order=E)
+
+
+def candidate_valid(s: int, cfg: OracleConfig, r: int) -> bool:
+    """A candidate needs room for P in the main cache and r evicted tokens."""
+    m = cfg.budget - r
+    if m < min(cfg.recent_window, s):
+        return False
+    n_evicted = s - m
+    return r <= n_evicted
+
+
+def decode_unit(cache: UnitCache, Q: np.ndarray, cfg: OracleConfig) -> np.ndarray:
+    """Decode the G query heads of one KV head (GQA sharing, App. B): [G, d]."""
+    return np.stack([shared_softmax_decode(q, cache.kmain, cache.vmain, cache.kbar,
+                                           cache.vbar, cache.logc, cfg) for q in Q])
+
+
+def validation_loss(cache: UnitCache, Qval: np.ndarray, O_full: np.ndarray,
+                    cfg: OracleConfig) -> float:
+    """L_r = mean over validation queries (and the G heads) of ||o^(r) - o_S||^2
+    (Eq. valloss), with the decode rule of Sec. 5.4 including the gate."""
+    G, n_val, _ = Qval.shape
+    total = 0.0
+    for g in range(G):
+        for t in range(n_val):
+            o = shared_softmax_decode(Qval[g, t], cache.kmain, cache.vmain, cache.kbar,
+                                      cache.vbar, cache.logc, cfg)
+            diff = o - O_full[g, t]
+            total += float(diff @ diff)
+    return total / (G * n_val)
+
+
+def choose_r(L0: float, rs: Sequence[int], losses: Sequence[float], delta: float) -> int:
+    """r* = argmin_{r>0} L_r (ties -> smaller r); keep r* only if
+    L_{r*} < (1 - delta) L_0, else r = 0  (Eq. valproxy; Alg. 1 steps 9-14)."""
+    if len(rs) == 0:
+        return 0
+    order = sorted(range(len(rs)), key=lambda i: (losses[i], rs[i]))
+    best = order[0]
+    return rs[best] if losses[best] < (1.0 - delta) * L0 else 0
+
+
+def build_unit(K: np.ndarray, V: np.ndarray, Qobs: Optional[np.ndarray],
+               cfg: OracleConfig) -> UnitCache:
+    """Alg. 1 for one (layer, KV head).
+
+    ``K``, ``V``: [s, d] float64 (exact bf16 values).  ``Qobs``: [G, n_obs, d]
+    observation queries of the G query heads (fit rows first), or None with the
+    query-free score.
+    """
+    s = K.shape[0]
+    # step 2: token scores on the fit queries; recent protection P
+    if cfg.score_mode == SCORE_OBS_POOL:
+        scores = scores_obs_pool(K, Qobs[:, :cfg.n_fit], cfg.pool_kernel)
+    elif cfg.score_mode == SCORE_KEYNORM:
+        scores = scores_keynorm(K)
+    else:
+        raise ValueError("unknown score mode")
+    ranked = rank_evictable(scores, cfg.recent_window)
+
+    if cfg.budget >= s:                        # the budget covers every token: M = S
+        out = build_candidate(K, V, ranked, cfg, 0)
+        out.scores, out.ranked = scores, ranked
+        return out
+
+    if cfg.residual_override is not None:      # fixed r: the proxy is bypassed
+        r = int(cfg.residual_override)
+        if r > 0 and not candidate_valid(s, cfg, r):
+            raise ValueError("residual override does not fit the budget")
+        out = build_candidate(K, V, ranked, cfg, r)
+        out.scores, out.ranked = scores, ranked
+        return out
+
+    # step 1: validation part of the observation window; its full-cache outputs
+    Qval = Qobs[:, Qobs.shape[1] - cfg.n_val:]
+    G = Qval.shape[0]
+    O_full = np.stack([np.stack([attention_full(Qval[g, t], K, V)
+                                 for t in range(cfg.n_val)]) for g in range(G)])
+    # step 3: pure-main cache and L_0
+    c0 = build_candidate(K, V, ranked, cfg, 0)
+    L0 = validation_loss(c0, Qval, O_full, cfg)
+    losses = {0: L0}
+    # steps 4-8: every candidate r > 0
+    rs = [r for r in candidate_budgets(cfg.budget, cfg.grid_ratios) if candidate_valid(s, cfg, r)]
+    built = {}
+    for r in rs:
+        built[r] = build_candidate(K, V, ranked, cfg, r)
+        losses[r] = validation_loss(built[r], Qval, O_full, cfg)
+    # steps 9-14: r* and the margin test; step 15: the cache for the chosen r
+    r_star = choose_r(L0, rs, [losses[r] for r in rs], cfg.delta)
+    out = built[r_star] if r_star > 0 else c0
+    out.scores, out.ranked, out.losses = scores, ranked, losses
+    return out

@@ -1,0 +1,486 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+Each test names the passage it follows.  None of them re-derives the oracle's
+own formula: they use closed forms (App. A.1, A.2), fixed points the paper
+states (Sec. 5.4: R empty gives eviction; Sec. 4.2: adding the exact residual
+recovers full attention; Sec. 5.3: c_j = 1 gives an exact token), textbook
+softmax through scipy (which the oracle does not call), explicit scalar loops
+and hand-computed fixtures under ``tests/golden``.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+from scipy.special import softmax
+
+import oracle as orc
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def golden(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def bf16ish(rng, shape, scale=1.0):
+    """Random values that are exact bf16 numbers (8 significant bits)."""
+    return orc.round_to_bf16(rng.standard_normal(shape) * scale)
+
+
+def textbook_attention(q, K, V):
+    """softmax(q K^T / sqrt(d)) V through scipy (Eq. attn / Eq. evict)."""
+    w = softmax(K @ q / math.sqrt(K.shape[1]))
+    return w @ V
+
+
+# ---------------------------------------------------------------------------
+# storage helpers
+# ---------------------------------------------------------------------------
+
+def test_bf16_rounding_fixture():
+    g = golden("bf16_rounding.json")
+    for c in g["cases"]:
+        assert orc.round_to_bf16(np.array([c["x"]]))[0] == c["rounded"], c["note"]
+    for c in g["bits"]:
+        assert orc.bf16_bits_to_f64(np.array([c["bits"]], dtype=np.uint16))[0] == c["value"]
+
+
+def test_bf16_rounding_is_idempotent_on_bf16_values():
+    bits = np.arange(0, 1 << 16, 7, dtype=np.uint16)
+    bits = bits[((bits >> 7) & 0xFF) != 0xFF]          # drop inf / NaN patterns
+    vals = orc.bf16_bits_to_f64(bits)
+    vals = vals[np.isfinite(vals) & (np.abs(vals) > 1e-30) & (np.abs(vals) < 1e30)]
+    assert np.array_equal(orc.round_to_bf16(vals), vals)
+
+
+# ---------------------------------------------------------------------------
+# Decode (Alg. 2) fixed points and closed forms
+# ---------------------------------------------------------------------------
+
+def _cfg(**kw):
+    base = dict(budget=8)
+    base.update(kw)
+    return orc.OracleConfig(**base)
+
+
+def test_decode_empty_residual_is_eviction_attention():
+    """Sec. 5.4: with R empty the shared softmax is eviction attention (Eq. evict)."""
+    rng = np.random.default_rng(1)
+    d, m = 16, 37
+    K, V, q = bf16ish(rng, (m, d)), bf16ish(rng, (m, d)), bf16ish(rng, d, 2.0)
+    out = orc.shared_softmax_decode(q, K, V, np.zeros((0, d)), np.zeros((0, d)),
+                                    np.zeros(0), _cfg())
+    np.testing.assert_allclose(out, textbook_attention(q, K, V), rtol=1e-12, atol=1e-13)
+
+
+def test_decode_gate_zero_is_main_only():
+    """Gate fixed to 0: log g = -inf removes every residual term (Eq. residual_logit)."""
+    rng = np.random.default_rng(2)
+    d, m, r = 16, 20, 6
+    K, V, q = bf16ish(rng, (m, d)), bf16ish(rng, (m, d)), bf16ish(rng, d, 2.0)
+    Kr, Vr = bf16ish(rng, (r, d)), bf16ish(rng, (r, d), 5.0)
+    logc = np.log(rng.integers(1, 50, r).astype(float))
+    out = orc.shared_softmax_decode(q, K, V, Kr, Vr, logc,
+                                    _cfg(gate_mode=orc.GATE_FIXED, g_fixed=0.0))
+    np.testing.assert_allclose(out, textbook_attention(q, K, V), rtol=1e-12, atol=1e-13)
+
+
+def test_decode_exact_residual_encoding_recovers_full_attention():
+    """Sec. 4.2, Eq. residual: adding (N_E, Z_E) back recovers o_S exactly.
+
+    One residual entry whose logit carries log Z_E(q) and whose value is
+    N_E/Z_E encodes the omitted statistics of q exactly; with g = 1 the shared
+    softmax (Eqs. reskv_den, reskv_num) must equal full attention.  Z_E and N_E
+    are summed here with explicit scalar loops.
+    """
+    rng = np.random.default_rng(3)
+    d, s, m = 8, 40, 12
+    K, V, q = bf16ish(rng, (s, d)), bf16ish(rng, (s, d)), bf16ish(rng, d, 1.5)
+    M, E = np.arange(m), np.arange(m, s)
+    ZE, NE = 0.0, np.zeros(d)
+    for p in E:
+        a = sum(q[i] * K[p, i] for i in range(d)) / math.sqrt(d)
+        ZE += math.exp(a)
+        NE += math.exp(a) * V[p]
+    kbar = bf16ish(rng, (1, d))
+    a_bar = float(kbar[0] @ q) / math.sqrt(d)
+    logc = np.array([math.log(ZE) - a_bar])
+    out = orc.shared_softmax_decode(q, K[M], V[M], kbar, (NE / ZE)[None, :], logc,
+                                    _cfg(gate_mode=orc.GATE_FIXED, g_fixed=1.0))
+    np.testing.assert_allclose(out, textbook_attention(q, K, V), rtol=1e-11, atol=1e-12)
+
+
+def test_decode_weights_sum_to_one():
+    """o^ = N^/Z^ is a convex combination: constant values come back unchanged."""
+    rng = np.random.default_rng(4)
+    d, m, r = 8, 10, 5
+    c = bf16ish(rng, d)
+    K, q = bf16ish(rng, (m, d)), bf16ish(rng, d)
+    Kr = bf16ish(rng, (r, d))
+    logc = np.log(np.arange(1, r + 1, dtype=float) * 3)
+    out = orc.shared_softmax_decode(q, K, np.tile(c, (m, 1)), Kr, np.tile(c, (r, 1)), logc, _cfg())
+    np.testing.assert_allclose(out, c, rtol=1e-13, atol=1e-14)
+
+
+def test_decode_residual_mass_enters_both_numerator_and_denominator():
+    """Eqs. reskv_den/reskv_num on a hand-sized case: one main token, one entry.
+
+    Main: a_1 = 0, v = 0.  Entry: <q,k_bar>/sqrt(d) = 0, c = 3, g = 1, v_bar = 1:
+    o^ = 3 * 1 / (1 + 3) = 0.75.
+    """
+    d = 4
+    q = np.zeros(d)
+    out = orc.shared_softmax_decode(q, np.zeros((1, d)), np.zeros((1, d)), np.zeros((1, d)),
+                                    np.ones((1, d)), np.log([3.0]),
+                                    _cfg(gate_mode=orc.GATE_FIXED, g_fixed=1.0))
+    np.testing.assert_allclose(out, 0.75, rtol=1e-15)
+    # the dynamic gate with a single main token: p_max = 1 -> g = sigmoid(-9)
+    out2, st = orc.shared_softmax_decode(q, np.zeros((1, d)), np.zeros((1, d)), np.zeros((1, d)),
+                                         np.ones((1, d)), np.log([3.0]), _cfg(), return_stats=True)
+    g = 1.0 / (1.0 + math.exp(9.0))
+    assert st["p_max"] == 1.0
+    np.testing.assert_allclose(st["g"], g, rtol=1e-15)
+    np.testing.assert_allclose(out2, 3 * g / (1 + 3 * g), rtol=1e-14)
+
+
+def test_gate_closed_forms():
+    """Eq. gate with the paper's tau = 0.25, alpha = 12 (App. B), via uniform main caches."""
+    gc = golden("gate_closed_forms.json")
+    for c in gc["cases"]:
+        assert orc.dynamic_gate(c["p_max"], 0.25, 12.0, 0.0) == pytest.approx(c["g"], rel=1e-14)
+    cm = gc["g_min_case"]
+    assert orc.dynamic_gate(cm["p_max"], 0.25, 12.0, cm["g_min"]) == cm["g"]
+    # through the decode path: m identical keys give p_max = 1/m
+    d = 4
+    q = np.ones(d)
+    for m, case in ((4, 0), (1, 1), (8, 2), (2, 3)):
+        K = np.tile(np.array([0.5, -1.0, 0.25, 2.0]), (m, 1))
+        _, st = orc.shared_softmax_decode(q, K, np.zeros((m, d)), np.zeros((1, d)), np.zeros((1, d)),
+                                          np.zeros(1), _cfg(), return_stats=True)
+        assert st["p_max"] == pytest.approx(1.0 / m, rel=1e-15)
+        assert st["g"] == pytest.approx(gc["cases"][case]["g"], rel=1e-13)
+
+
+def test_eviction_error_closed_form():
+    """App. A.1, Eq. app_evict_error: o_S - o_M = (Z_M N_E - Z_E N_M) / (Z_M (Z_M + Z_E))."""
+    rng = np.random.default_rng(5)
+    d, s, m = 8, 50, 15
+    K, V, q = bf16ish(rng, (s, d)), bf16ish(rng, (s, d)), bf16ish(rng, d, 1.5)
+    M, E = np.arange(m), np.arange(m, s)
+    ZM = sum(math.exp(float(K[p] @ q) / math.sqrt(d)) for p in M)
+    NM = sum(math.exp(float(K[p] @ q) / math.sqrt(d)) * V[p] for p in M)
+    ZE = sum(math.exp(float(K[p] @ q) / math.sqrt(d)) for p in E)
+    NE = sum(math.exp(float(K[p] @ q) / math.sqrt(d)) * V[p] for p in E)
+    closed = (ZM * NE - ZE * NM) / (ZM * (ZM + ZE))
+    o_S = orc.attention_full(q, K, V)
+    o_M = orc.shared_softmax_decode(q, K[M], V[M], np.zeros((0, d)), np.zeros((0, d)),
+                                    np.zeros(0), _cfg())
+    np.testing.assert_allclose(o_S - o_M, closed, rtol=1e-10, atol=1e-13)
+
+
+def test_entry_error_bound():
+    """App. A.2: |Z_j - c_j e^{a_bar}| <= c_j e^{a_bar} (e^eta - 1) and the
+    numerator bound with V = max ||v_p||, for the entry the oracle builds."""
+    rng = np.random.default_rng(6)
+    d, c = 16, 30
+    centre = bf16ish(rng, d)
+    for spread in (0.01, 0.1, 0.5):
+        KC = centre + spread * rng.standard_normal((c, d))
+        VC = rng.standard_normal((c, d))
+        q = rng.standard_normal(d)
+        E = np.arange(c)
+        kbar, vbar, counts = orc.lloyd_residual(KC, VC, E, 1, 4)
+        assert counts[0] == c
+        # the entry's reconstructed statistics, read from the shared softmax
+        main_k = np.zeros((1, d))
+        _, st = orc.shared_softmax_decode(q, main_k, np.zeros((1, d)), kbar, vbar,
+                                          orc.log_counts(counts, 1.0),
+                                          _cfg(gate_mode=orc.GATE_FIXED, g_fixed=1.0),
+                                          return_stats=True)
+        Z_hat = st["Z"] * math.exp(st["shift"]) - 1.0          # minus the main token's e^0
+        N_hat = st["N"] * math.exp(st["shift"])                 # main value is 0
+        a = KC @ q / math.sqrt(d)
+        a_bar = float(kbar[0] @ q) / math.sqrt(d)
+        eta = float(np.max(np.abs(a - a_bar)))
+        Zj = float(np.sum(np.exp(a)))
+        Nj = np.exp(a) @ VC
+        bound_z = c * math.exp(a_bar) * (math.exp(eta) - 1)
+        Vmax = float(np.max(np.linalg.norm(VC, axis=1)))
+        np.testing.assert_allclose(Z_hat, c * math.exp(a_bar), rtol=1e-12)
+        assert abs(Zj - Z_hat) <= bound_z * (1 + 1e-12)
+        assert np.linalg.norm(Nj - N_hat) <= bound_z * Vmax * (1 + 1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Selection (Sec. 5.2) and candidate budgets (App. B)
+# ---------------------------------------------------------------------------
+
+def test_ranking_and_selection_fixture():
+    g = golden("ranking_ties.json")
+    ranked = orc.rank_evictable(np.array(g["scores"]), g["recent"])
+    assert ranked.tolist() == g["ranked"]
+    M, E = orc.select_main(ranked, len(g["scores"]), g["recent"], g["m"])
+    assert M.tolist() == g["M"]
+    assert E.tolist() == g["E_rank_order"]
+
+
+def test_ranking_matches_brute_force_order():
+    """Brute force: a scalar insertion sort by (score desc, index asc)."""
+    rng = np.random.default_rng(7)
+    for trial in range(20):
+        s = int(rng.integers(1, 30))
+        recent = int(rng.integers(0, 6))
+        scores = rng.integers(0, 5, s).astype(float)     # many exact ties
+        ranked = orc.rank_evictable(scores, recent)
+        out = []
+        for p in range(max(s - recent, 0)):
+            i = 0
+            while i < len(out) and (scores[out[i]] > scores[p] or
+                                    (scores[out[i]] == scores[p] and out[i] < p)):
+                i += 1
+            out.insert(i, p)
+        assert ranked.tolist() == out
+
+
+def test_candidate_budgets_fixture():
+    g = golden("candidate_budgets.json")
+    for b, rs in g["cases"].items():
+        assert orc.candidate_budgets(int(b), g["ratios"]) == rs
+
+
+def test_choose_r_rules():
+    """Eq. valproxy: argmin over r > 0 (ties -> smaller r), strict margin test."""
+    rs = [25, 51, 76, 102]
+    assert orc.choose_r(1.0, rs, [0.5, 0.4, 0.4, 0.6], 0.01) == 51
+    assert orc.choose_r(1.0, rs, [0.995] * 4, 0.01) == 0
+    assert orc.choose_r(1.0, rs, [0.99, 1.0, 1.1, 1.2], 0.01) == 0   # equality is not enough
+    assert orc.choose_r(1.0, rs, [0.98, 1.0, 1.1, 1.2], 0.01) == 25
+    assert orc.choose_r(0.0, rs, [0.0] * 4, 0.01) == 0
+    assert orc.choose_r(1.0, [], [], 0.01) == 0
+
+
+# ---------------------------------------------------------------------------
+# Residual construction (Sec. 5.3)
+# ---------------------------------------------------------------------------
+
+def test_lloyd_hand_traces():
+    g = golden("lloyd_traces.json")
+    for c in g["cases"]:
+        K = np.array(c["keys"], dtype=float)[:, None]
+        V = 2 * K + 1
+        kbar, vbar, counts = orc.lloyd_residual(K, V, np.array(c["E"]), c["r"], c["iters"])
+        np.testing.assert_allclose(kbar[:, 0], c["kbar"], rtol=1e-15, err_msg=c["name"])
+        assert counts.tolist() == c["counts"], c["name"]
+        for j in range(c["r"]):
+            if counts[j] > 0:
+                assert vbar[j, 0] == pytest.approx(2 * kbar[j, 0] + 1, rel=1e-14), c["name"]
+            else:
+                assert vbar[j, 0] == 0.0
+
+
+def test_lloyd_single_entry_is_global_mean():
+    rng = np.random.default_rng(8)
+    K, V = rng.standard_normal((57, 6)), rng.standard_normal((57, 6))
+    E = rng.permutation(57)[:40]
+    kbar, vbar, counts = orc.lloyd_residual(K, V, E, 1, 4)
+    np.testing.assert_allclose(kbar[0], K[E].mean(axis=0), rtol=1e-13)
+    np.testing.assert_allclose(vbar[0], V[E].mean(axis=0), rtol=1e-13)
+    assert counts.tolist() == [40]
+
+
+def test_lloyd_separated_clusters_converge_to_true_means():
+    rng = np.random.default_rng(9)
+    d, per = 8, 25
+    centres = 50.0 * np.eye(d)[:3]
+    K = np.concatenate([c + rng.standard_normal((per, d)) for c in centres])
+    V = rng.standard_normal((3 * per, d))
+    E = np.array([0, per, 2 * per] + [p for p in range(3 * per) if p % per])
+    kbar, vbar, counts = orc.lloyd_residual(K, V, E, 3, 4)
+    for j in range(3):
+        np.testing.assert_allclose(kbar[j], K[j * per:(j + 1) * per].mean(axis=0), rtol=1e-12)
+        np.testing.assert_allclose(vbar[j], V[j * per:(j + 1) * per].mean(axis=0), rtol=1e-12)
+    assert counts.tolist() == [per] * 3
+
+
+def test_lloyd_assign_matches_direct_distances():
+    """The matrix-product form of the distance picks the same centre as a
+    direct sum of squared differences (scalar loops)."""
+    rng = np.random.default_rng(10)
+    KE = bf16ish(rng, (60, 5))
+    C = bf16ish(rng, (7, 5))
+    got = orc.lloyd_assign(KE, C)
+    for p in range(KE.shape[0]):
+        best, bd = 0, None
+        for j in range(C.shape[0]):
+            dd = sum((KE[p, i] - C[j, i]) ** 2 for i in range(5))
+            if bd is None or dd < bd:
+                best, bd = j, dd
+        assert got[p] == best
+
+
+def test_exact_groups_reproduce_full_attention():
+    """Sec. 5.3 / App. A.2 with eta = 0: an entry with c_j = 1 is an exact token,
+    and a group of c_j identical tokens is reconstructed exactly (c_j e^{a_bar}
+    equals the group's sum).  With every evicted group exact and g = 1 the
+    shared softmax is full attention over S."""
+    rng = np.random.default_rng(11)
+    d, m = 16, 20
+    # singletons: r = |E|, every key distinct
+    K, V = bf16ish(rng, (m + 12, d)), bf16ish(rng, (m + 12, d))
+    E = np.arange(m, m + 12)[::-1]
+    kbar, vbar, counts = orc.lloyd_residual(K, V, E, len(E), 4)
+    assert counts.tolist() == [1] * len(E)
+    np.testing.assert_array_equal(kbar, K[E])
+    cfg = orc.OracleConfig(budget=m + 12, gate_mode=orc.GATE_FIXED, g_fixed=1.0)
+    for _ in range(4):
+        q = bf16ish(rng, d, 1.5)
+        out = orc.shared_softmax_decode(q, K[:m], V[:m], kbar, vbar, orc.log_counts(counts, 1.0), cfg)
+        np.testing.assert_allclose(out, textbook_attention(q, K, V), rtol=1e-11, atol=1e-12)
+    # groups of identical tokens: 5 prototypes repeated 1..5 times
+    protos_k, protos_v = bf16ish(rng, (5, d)), bf16ish(rng, (5, d))
+    reps = [3, 1, 5, 2, 4]
+    KE = np.concatenate([np.tile(protos_k[i], (reps[i], 1)) for i in range(5)])
+    VE = np.concatenate([np.tile(protos_v[i], (reps[i], 1)) for i in range(5)])
+    K2 = np.concatenate([K[:m], KE])
+    V2 = np.concatenate([V[:m], VE])
+    firsts = np.cumsum([0] + reps[:-1]) + m
+    rest = [p for p in range(m, m + sum(reps)) if p not in set(firsts.tolist())]
+    E2 = np.concatenate([firsts, rest])                 # one of each prototype first
+    kbar, vbar, counts = orc.lloyd_residual(K2, V2, E2, 5, 4)
+    assert counts.tolist() == reps
+    for _ in range(4):
+        q = bf16ish(rng, d, 1.5)
+        out = orc.shared_softmax_decode(q, K2[:m], V2[:m], kbar, vbar,
+                                        orc.log_counts(counts, 1.0), cfg)
+        np.testing.assert_allclose(out, textbook_attention(q, K2, V2), rtol=1e-11, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Scoring (App. B.2)
+# ---------------------------------------------------------------------------
+
+def test_scores_uniform_keys():
+    """Identical keys give uniform weights 1/s per query and head; the sum over
+    n_fit queries is n_fit/s, and the zero-padded pool of width 5 keeps 3/5 and
+    4/5 of it at the two ends."""
+    s, d, G, n_fit = 20, 4, 3, 7
+    K = np.tile(np.array([0.5, 1.0, -2.0, 0.25]), (s, 1))
+    Q = np.random.default_rng(12).standard_normal((G, n_fit, d))
+    sc = orc.scores_obs_pool(K, Q, 5)
+    base = n_fit / s
+    expect = np.full(s, base)
+    expect[[0, -1]] = base * 3 / 5
+    expect[[1, -2]] = base * 4 / 5
+    np.testing.assert_allclose(sc, expect, rtol=1e-13)
+
+
+def test_scores_single_peak_pooling_and_head_average():
+    """One key with logit L (others 0) per head: weight e^L/(e^L + s - 1) at
+    that token.  Two heads peaked at different tokens average with 1/G, fit
+    queries sum, and the pool spreads each peak over 5 neighbours.  The
+    validation rows (not passed) play no part."""
+    s, d = 30, 2
+    K = np.zeros((s, d))
+    K[10, 0] = 4.0
+    K[20, 1] = 6.0
+    n_fit = 3
+    Q = np.zeros((2, n_fit, d))
+    Q[0, :, 0] = 2.0
+    Q[1, :, 1] = 1.0
+    L0, L1 = 4.0 * 2.0 / math.sqrt(2), 6.0 * 1.0 / math.sqrt(2)
+    w0 = math.exp(L0) / (math.exp(L0) + s - 1)
+    w1 = math.exp(L1) / (math.exp(L1) + s - 1)
+    A = np.zeros(s)
+    A += n_fit * 0.5 * np.where(np.arange(s) == 10, w0, (1 - w0) / (s - 1))
+    A += n_fit * 0.5 * np.where(np.arange(s) == 20, w1, (1 - w1) / (s - 1))
+    expect = np.array([sum(A[p + j] for j in range(-2, 3) if 0 <= p + j < s) / 5 for p in range(s)])
+    np.testing.assert_allclose(orc.scores_obs_pool(K, Q, 5), expect, rtol=1e-12)
+
+
+def test_build_uses_only_fit_rows_for_scores():
+    rng = np.random.default_rng(13)
+    s, d = 64, 8
+    K, V = bf16ish(rng, (s, d)), bf16ish(rng, (s, d))
+    Q = bf16ish(rng, (2, 10, d))
+    cfg = orc.OracleConfig(budget=24, recent_window=4, n_fit=7, n_val=3, residual_override=4)
+    a = orc.build_unit(K, V, Q, cfg)
+    Q2 = Q.copy()
+    Q2[:, 7:] = bf16ish(rng, (2, 3, d), 3.0)
+    b = orc.build_unit(K, V, Q2, cfg)
+    np.testing.assert_array_equal(a.scores, b.scores)
+    np.testing.assert_array_equal(a.main_pos, b.main_pos)
+
+
+def test_keynorm_scores():
+    K = np.array([[1.0, 2.0], [3.0, -1.0], [0.0, 0.5]])
+    np.testing.assert_array_equal(orc.scores_keynorm(K), [5.0, 10.0, 0.25])
+
+
+# ---------------------------------------------------------------------------
+# Construction (Alg. 1) and the validation proxy (Sec. 5.5.1)
+# ---------------------------------------------------------------------------
+
+def test_budget_covering_every_token_is_full_attention():
+    """b >= s: M = S, E empty, r = 0, and decode is full attention (Eq. attn)."""
+    rng = np.random.default_rng(14)
+    s, d = 30, 8
+    K, V = bf16ish(rng, (s, d)), bf16ish(rng, (s, d))
+    Q = bf16ish(rng, (4, 12, d))
+    cfg = orc.OracleConfig(budget=32, recent_window=4, n_fit=8, n_val=4)
+    cache = orc.build_unit(K, V, Q, cfg)
+    assert cache.r == 0 and cache.main_pos.tolist() == list(range(s))
+    q = bf16ish(rng, d)
+    np.testing.assert_allclose(orc.decode_unit(cache, q[None], cfg)[0],
+                               textbook_attention(q, K, V), rtol=1e-12, atol=1e-13)
+
+
+def test_validation_loss_r0_matches_eviction_closed_form():
+    """L_0 (Eq. valloss on the pure-main cache) equals the mean of ||o_S - o_M||^2
+    written with the App. A.1 closed form."""
+    rng = np.random.default_rng(15)
+    s, d, G = 80, 8, 2
+    K, V = bf16ish(rng, (s, d)), bf16ish(rng, (s, d))
+    Q = bf16ish(rng, (G, 10, d), 1.5)
+    cfg = orc.OracleConfig(budget=20, recent_window=4, n_fit=6, n_val=4)
+    cache = orc.build_unit(K, V, Q, cfg)
+    c0 = orc.build_candidate(K, V, cache.ranked, cfg, 0)
+    M = c0.main_pos
+    E = np.setdiff1d(np.arange(s), M)
+    tot = 0.0
+    for g in range(G):
+        for t in range(6, 10):
+            q = Q[g, t]
+            e = np.exp(K @ q / math.sqrt(d))
+            ZM, ZE = e[M].sum(), e[E].sum()
+            NM, NE = e[M] @ V[M], e[E] @ V[E]
+            diff = (ZM * NE - ZE * NM) / (ZM * (ZM + ZE))
+            tot += float(diff @ diff)
+    assert cache.losses[0] == pytest.approx(tot / (G * 4), rel=1e-10)
+
+
+def test_validation_proxy_enables_residual_on_clusterable_diffuse_attention():
+    """Evicted keys that form a few tight clusters under diffuse attention are
+    reconstructed well, so L_r* beats L_0 by more than delta and r* > 0."""
+    rng = np.random.default_rng(16)
+    d, s = 8, 400
+    protos = bf16ish(rng, (4, d), 0.6)
+    K = np.concatenate([protos[i % 4] + 0.0 for i in range(s)]).reshape(s, d)
+    V = np.concatenate([np.full(d, float(i % 4)) for i in range(s)]).reshape(s, d)
+    K[: s // 2] = bf16ish(rng, (s // 2, d), 0.6)      # unclustered half, scored high
+    Q = bf16ish(rng, (2, 16, d), 0.3)
+    cfg = orc.OracleConfig(budget=100, recent_window=8, n_fit=12, n_val=4)
+    cache = orc.build_unit(K, V, Q, cfg)
+    assert cache.r > 0
+    assert cache.losses[cache.r] < (1 - cfg.delta) * cache.losses[0]
+
+
+def test_validation_proxy_falls_back_when_nothing_is_evicted():
+    rng = np.random.default_rng(17)
+    s, d = 24, 4
+    K, V = bf16ish(rng, (s, d)), bf16ish(rng, (s, d))
+    Q = bf16ish(rng, (1, 8, d))
+    cache = orc.build_unit(K, V, Q, orc.OracleConfig(budget=24, recent_window=4, n_fit=6, n_val=2))
+    assert cache.r == 0 and len(cache.main_pos) == s
