@@ -1,0 +1,204 @@
+/*
+ * reskv.h -- C ABI of the GB300 (sm_103a) ResKV decode library.
+ *
+ * ResKV ("Reconstructing Omitted Attention Contributions for Fixed-Budget KV
+ * Cache Compression") keeps, per (layer, KV head), a fixed budget of b cache
+ * slots split as b = m + r (Sec. 5.1): m exact main-cache tokens (Sec. 5.2,
+ * Eq. main_selection) and r residual entries (k_bar_j, v_bar_j, c_j) that
+ * summarise the evicted tokens (Sec. 5.3, Eq. summary).  Decoding attends with
+ * one shared softmax over both (Sec. 5.4, Eqs. residual_logit, reskv_den,
+ * reskv_num, reskv) with the residual logits shifted by log g(q), the dynamic
+ * gate of Sec. 5.5.2 (Eq. gate).  r is chosen per (layer, KV head) by the
+ * validation proxy of Sec. 5.5.1 (Eqs. valloss, valproxy).  Alg. 1 is the
+ * construction, Alg. 2 the decode step.
+ *
+ * Conventions for every entry point:
+ *  - Pointers named "device" are CUDA device pointers of the current device;
+ *    "host" pointers are ordinary host memory.  The library never takes
+ *    ownership of caller buffers.
+ *  - `stream` is a cudaStream_t (NULL = legacy default stream).  Work is
+ *    enqueued asynchronously on it; callers must not free inputs before the
+ *    stream has passed the call.
+ *  - Every function returns a status; nothing aborts or throws across the ABI.
+ *    On error the output handle is left untouched and reskv_last_error()
+ *    returns a message (thread-local, valid until the next call on the thread).
+ *  - Arguments are validated on the host before any launch.
+ *  - Calls that share one cache handle must be ordered (same stream, or
+ *    synchronised): the handle's decode workspace is reused by every call.
+ */
+#ifndef RESKV_H
+#define RESKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  RESKV_OK = 0,
+  RESKV_ERR_INVALID_ARG = 1,   /* bad pointer, size or configuration        */
+  RESKV_ERR_UNSUPPORTED = 2,   /* valid but outside what the kernels cover   */
+  RESKV_ERR_OOM = 3,           /* cudaMalloc failed                          */
+  RESKV_ERR_CUDA = 4,          /* a CUDA runtime call or launch failed       */
+  RESKV_ERR_DEVICE_STATUS = 5  /* a kernel reported a fault (bounded wait
+                                  timed out or an index left its range)      */
+} reskv_status;
+
+enum { RESKV_SCORE_OBS_POOL = 0, RESKV_SCORE_KEYNORM = 1 };
+enum { RESKV_GATE_DYNAMIC = 0, RESKV_GATE_FIXED = 1 };
+
+#define RESKV_MAX_GRID 8
+
+/*
+ * Construction and decode settings.  reskv_config_default() fills the paper's
+ * values (App. B, "ResKV Construction Settings"; App. B.2 SnapKV): recent
+ * window 64, pooling kernel 5, 96 fit + 32 validation queries, ratio grid
+ * {0, .05, .10, .15, .20}, 4 Lloyd iterations, delta 0.01, beta 1.0,
+ * tau 0.25, alpha (= 1/T_g) 12, g_min 0.
+ */
+typedef struct reskv_config {
+  int32_t batch;           /* B                                              */
+  int32_t n_layers;        /* L                                              */
+  int32_t n_kv_heads;      /* H_kv                                           */
+  int32_t group;           /* G query heads per KV head (GQA); 1, 2 or 4     */
+  int32_t head_dim;        /* d; must be 128                                 */
+  int64_t seq_len;         /* s, cached tokens per (batch, layer, KV head)   */
+  int32_t budget;          /* b slots per (layer, KV head) (Sec. 3.2)        */
+  int32_t recent_window;   /* |P|, always kept (Eq. main_selection)          */
+  int32_t n_obs;           /* observation queries per query head             */
+  int32_t n_fit;           /* first n_fit rows score tokens (Sec. 5.5.1)     */
+  int32_t n_val;           /* last n_val rows validate (Sec. 5.5.1)          */
+  int32_t pool_kernel;     /* SnapKV average-pooling width, odd (App. B.2)   */
+  int32_t score_mode;      /* RESKV_SCORE_*                                  */
+  int32_t n_grid;          /* entries used in grid_ratios                    */
+  float grid_ratios[RESKV_MAX_GRID]; /* candidates r = floor(ratio * b)      */
+  int32_t lloyd_iters;     /* T rounds of (assign, update) (App. B)          */
+  float delta;             /* margin of Eq. valproxy                         */
+  float beta;              /* count exponent: logit term beta * log c_j      */
+  const int32_t* residual_override; /* host [L*B*H_kv] fixed r per unit, or
+                              NULL to run the validation proxy               */
+  int32_t gate_mode;       /* RESKV_GATE_DYNAMIC (Eq. gate) or _FIXED        */
+  float tau;               /* gate threshold                                 */
+  float alpha;             /* gate slope 1/T_g                               */
+  float g_min;             /* gate floor                                     */
+  float g_fixed;           /* gate value for RESKV_GATE_FIXED (0 = main-only,
+                              1 = the paper's "w/o dynamic gate" ablation)   */
+  int32_t keep_debug;      /* nonzero: keep construction intermediates for
+                              reskv_export_debug (scores, ranking, losses)   */
+  int32_t decode_warps;    /* 0: automatic.  Otherwise the number of equal
+                              pieces (one warp each) a decode call cuts its
+                              slot range into, capped at 8 warps per SM; the
+                              result does not depend on it beyond rounding   */
+} reskv_config;
+
+/* Fill *cfg with the paper's defaults; shape fields are zeroed. */
+void reskv_config_default(reskv_config* cfg);
+
+/* Opaque handle; owns every device buffer of the compressed cache. */
+typedef struct reskv_cache reskv_cache;
+
+/*
+ * Alg. 1 for every (layer, batch, KV head) unit: token scores (App. B.2 rule
+ * from the fit observation queries, or the query-free key-norm score), main
+ * selection (Eq. main_selection), Lloyd residual entries (Eqs.
+ * residual_partition, summary), validation proxy (Eqs. valloss, valproxy) and
+ * packing into the ragged main+residual layout.
+ *
+ *   K_layers[l], V_layers[l] : device bf16 [B, H_kv, s, d] (row-major)
+ *   Qobs_layers[l]           : device bf16 [B, H_kv*G, n_obs, d], or the
+ *                              array itself NULL with RESKV_SCORE_KEYNORM and
+ *                              residual_override set
+ *   out                      : receives a new handle on success
+ *
+ * Inputs may be freed once the stream has passed the call.  The call
+ * allocates the handle's device memory (cudaMalloc) and temporary workspace.
+ */
+reskv_status reskv_build_cache(const reskv_config* cfg, const void* const* K_layers,
+                               const void* const* V_layers, const void* const* Qobs_layers,
+                               void* stream, reskv_cache** out);
+
+/*
+ * Alg. 2 (shared-softmax decode with the dynamic gate) for one decode query
+ * per query head.
+ *
+ *   layer in [0, L) : Q device bf16 [B, H_kv*G, d], O device fp32 [B, H_kv*G, d]
+ *   layer == -1     : all layers in one launch, Q [L, B, H_kv*G, d], O likewise
+ *
+ * Query head hq attends with KV head hq / G.  O must not alias Q.
+ */
+reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* Q, void* O,
+                               void* stream);
+
+/* Release every device buffer of the handle (synchronises the device). NULL-safe. */
+void reskv_free(reskv_cache* c);
+
+/* Message of the last failing call on this thread ("" if none). */
+const char* reskv_last_error(void);
+
+/* Read the kernels' device status word; RESKV_ERR_DEVICE_STATUS if a kernel
+ * reported a fault since the handle was made (synchronises the device). */
+reskv_status reskv_check_status(const reskv_cache* c);
+
+/* Shape of a handle's cache. */
+typedef struct reskv_cache_info {
+  int64_t n_units;         /* U = L*B*H_kv, unit u = (l*B + b)*H_kv + h      */
+  int32_t budget;          /* slot stride per unit                           */
+  int32_t head_dim;
+  int64_t slot_bytes;      /* bytes of one K row + one V row                 */
+  int64_t cache_bytes;     /* device bytes of K/V slots + log-counts         */
+} reskv_cache_info;
+
+reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info);
+
+/*
+ * Host-side view of a cache layout, used by reskv_import_cache (read) and
+ * reskv_export_cache (written).  Unit u owns slots [u*b, u*b + b); its first
+ * n_main[u] slots are main-cache tokens, the next n_res[u] residual entries.
+ *   n_main, n_res : int32 [U]
+ *   kslots, vslots: bf16 bit patterns, uint16 [U, b, d]
+ *   logc          : fp32 [U, b]; beta*log c_j at residual slots (-inf for an
+ *                   empty entry), ignored at main slots
+ *   slot_pos      : int32 [U, b]; original token position of main slots,
+ *                   -1 at residual slots (may be NULL on import)
+ *   counts        : int32 [U, b]; c_j at residual slots, 0 at main slots
+ *                   (may be NULL on import)
+ */
+typedef struct reskv_host_cache {
+  int32_t* n_main;
+  int32_t* n_res;
+  uint16_t* kslots;
+  uint16_t* vslots;
+  float* logc;
+  int32_t* slot_pos;
+  int32_t* counts;
+} reskv_host_cache;
+
+/* Build a handle from host arrays (an externally constructed cache; only the
+ * shape, gate and budget fields of cfg are used).  Requires 1 <= n_main[u] and
+ * n_main[u] + n_res[u] <= budget. */
+reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache* h,
+                                void* stream, reskv_cache** out);
+
+/* Copy the handle's layout to host arrays (every pointer non-NULL, sized as
+ * above).  Synchronises `stream`. */
+reskv_status reskv_export_cache(const reskv_cache* c, reskv_host_cache* h, void* stream);
+
+enum {
+  RESKV_DEBUG_SCORES = 0,  /* fp64 [U, s]: token scores                      */
+  RESKV_DEBUG_RANKED = 1,  /* int32 [U, b - |P|]: top of the ranking of S\P  */
+  RESKV_DEBUG_LOSSES = 2,  /* fp64 [U, 1 + n_cand]: L_0 then L_r per candidate */
+  RESKV_DEBUG_CANDIDATES = 3 /* int32 [n_cand]: candidate r values, ascending */
+};
+
+/* Copy a construction intermediate (cfg.keep_debug was set) to host memory.
+ * `bytes` must equal the size of the array.  Synchronises the device. */
+reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_dst,
+                                size_t bytes);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RESKV_H */

@@ -1,0 +1,80 @@
+// Internal declarations shared by the host ABI and the kernels.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "reskv.h"
+
+namespace reskv {
+
+constexpr int kHeadDim = 128;          // d (only 128 is built)
+constexpr int kSlotRowBytes = kHeadDim * 2;
+constexpr float kLog2e = 1.4426950408889634f;
+
+// Decode split: every launch streams the concatenated slot range of its units
+// ("flat" index x = local_unit * budget + j) and cuts it into n_warps equal
+// contiguous pieces, one per warp.  A unit covered by one warp is finished by
+// that warp; a unit cut between warps is finished by the last of them to
+// arrive, from per-(unit, warp) partial records.
+struct DecodeParams {
+  const __nv_bfloat16* kslots;  // [U, budget, d] whole cache
+  const __nv_bfloat16* vslots;  // [U, budget, d]
+  const float* logc;            // [U, budget]  beta*ln c at residual slots
+  const int32_t* n_main;        // [U]
+  const int32_t* n_res;         // [U]
+  const __nv_bfloat16* Q;       // [n_units / H_kv, H_kv*G, d] for this launch
+  float* O;                     // same shape as Q, fp32
+  float* partials;              // [(n_units + n_warps) * 2 * G * (d + 2)]
+  int32_t* tickets;             // [U], zero between launches
+  uint32_t* status;             // device status word
+  int64_t unit0;                // first unit of the launch
+  int64_t total_slots;          // n_units * budget
+  int32_t n_units;
+  int32_t budget;
+  int32_t n_kv_heads;
+  int32_t n_warps;              // W
+  int32_t gate_mode;
+  float tau, alpha, g_min, g_fixed;
+};
+
+constexpr int kDecodeWarpsPerCta = 8;
+
+// Launch the decode kernel for `group` (1, 2 or 4) query heads per KV head.
+cudaError_t launch_decode(const DecodeParams& p, int group, int n_ctas, cudaStream_t stream);
+size_t decode_partials_floats(int64_t n_units, int n_warps, int group);
+
+void set_error(const std::string& msg);
+
+}  // namespace reskv
+
+// The opaque handle of the C ABI.
+struct reskv_cache {
+  reskv_config cfg;             // residual_override cleared
+  int device = 0;
+  int num_sms = 0;
+  int64_t n_units = 0;
+  int32_t budget = 0;
+  // layout (device)
+  __nv_bfloat16* kslots = nullptr;
+  __nv_bfloat16* vslots = nullptr;
+  float* logc = nullptr;
+  int32_t* slot_pos = nullptr;
+  int32_t* counts = nullptr;
+  int32_t* n_main = nullptr;
+  int32_t* n_res = nullptr;
+  // decode workspace (device)
+  float* partials = nullptr;
+  int32_t* tickets = nullptr;
+  uint32_t* status = nullptr;
+  int max_warps = 0;
+  // construction intermediates kept for reskv_export_debug (device)
+  double* dbg_scores = nullptr;
+  int32_t* dbg_ranked = nullptr;
+  double* dbg_losses = nullptr;
+  int64_t dbg_n_top = 0;
+  std::vector<int32_t> candidates;
+};

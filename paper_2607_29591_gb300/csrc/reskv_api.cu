@@ -1,0 +1,363 @@
+// Host side of the C ABI declared in include/reskv.h: argument validation,
+// ownership of the device layout, import/export, and decode launches.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "internal.h"
+#include "reskv.h"
+
+namespace reskv {
+
+static thread_local std::string g_last_error;
+
+void set_error(const std::string& msg) { g_last_error = msg; }
+
+// construction (construct.cu)
+reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
+                              const int32_t* override_host, const void* const* K,
+                              const void* const* V, const void* const* Qobs,
+                              cudaStream_t stream);
+
+namespace {
+
+reskv_status fail(reskv_status st, const std::string& msg) {
+  set_error(msg);
+  return st;
+}
+
+reskv_status cuda_fail(cudaError_t err, const char* what) {
+  return fail(err == cudaErrorMemoryAllocation ? RESKV_ERR_OOM : RESKV_ERR_CUDA,
+              std::string(what) + ": " + cudaGetErrorString(err));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Shape and gate fields shared by build and import.
+reskv_status validate_shape(const reskv_config* cfg) {
+  if (!cfg) return fail(RESKV_ERR_INVALID_ARG, "cfg is NULL");
+  if (cfg->batch < 1 || cfg->n_layers < 1 || cfg->n_kv_heads < 1)
+    return fail(RESKV_ERR_INVALID_ARG, "batch, n_layers and n_kv_heads must be >= 1");
+  if (cfg->group != 1 && cfg->group != 2 && cfg->group != 4)
+    return fail(RESKV_ERR_UNSUPPORTED, "group (query heads per KV head) must be 1, 2 or 4");
+  if (cfg->head_dim != kHeadDim) return fail(RESKV_ERR_UNSUPPORTED, "head_dim must be 128");
+  if (cfg->seq_len < 1 || cfg->seq_len > (int64_t(1) << 30))
+    return fail(RESKV_ERR_INVALID_ARG, "seq_len must be in [1, 2^30]");
+  if (cfg->budget < 1 || cfg->budget > (1 << 20))
+    return fail(RESKV_ERR_INVALID_ARG, "budget must be in [1, 2^20]");
+  if (cfg->decode_warps < 0) return fail(RESKV_ERR_INVALID_ARG, "decode_warps must be >= 0");
+  if (cfg->gate_mode != RESKV_GATE_DYNAMIC && cfg->gate_mode != RESKV_GATE_FIXED)
+    return fail(RESKV_ERR_INVALID_ARG, "unknown gate_mode");
+  if (!std::isfinite(cfg->tau) || !std::isfinite(cfg->alpha) || !(cfg->g_min >= 0.f) ||
+      !(cfg->g_min <= 1.f) || !(cfg->g_fixed >= 0.f) || !(cfg->g_fixed <= 1.f))
+    return fail(RESKV_ERR_INVALID_ARG, "gate parameters out of range (g_min, g_fixed in [0,1])");
+  const double units = double(cfg->n_layers) * cfg->batch * cfg->n_kv_heads;
+  if (units * cfg->budget > double(int64_t(1) << 40))
+    return fail(RESKV_ERR_INVALID_ARG, "cache too large");
+  return RESKV_OK;
+}
+
+template <typename T>
+reskv_status dalloc(T** p, size_t count, const char* what) {
+  *p = nullptr;
+  if (count == 0) count = 1;
+  cudaError_t err = cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T));
+  if (err != cudaSuccess) {
+    *p = nullptr;
+    cudaGetLastError();
+    return cuda_fail(err, what);
+  }
+  return RESKV_OK;
+}
+
+void free_handle(reskv_cache* c) {
+  if (!c) return;
+  cudaFree(c->kslots);
+  cudaFree(c->vslots);
+  cudaFree(c->logc);
+  cudaFree(c->slot_pos);
+  cudaFree(c->counts);
+  cudaFree(c->n_main);
+  cudaFree(c->n_res);
+  cudaFree(c->partials);
+  cudaFree(c->tickets);
+  cudaFree(c->status);
+  cudaFree(c->dbg_scores);
+  cudaFree(c->dbg_ranked);
+  cudaFree(c->dbg_losses);
+  delete c;
+}
+
+}  // namespace
+
+// Allocate a zeroed layout and decode workspace for cfg's shape.
+reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_cache** out) {
+  reskv_cache* c = new (std::nothrow) reskv_cache();
+  if (!c) return fail(RESKV_ERR_OOM, "host allocation failed");
+  c->cfg = cfg;
+  c->cfg.residual_override = nullptr;
+  cudaError_t err = cudaGetDevice(&c->device);
+  if (err == cudaSuccess)
+    err = cudaDeviceGetAttribute(&c->num_sms, cudaDevAttrMultiProcessorCount, c->device);
+  if (err != cudaSuccess) {
+    delete c;
+    return cuda_fail(err, "device query");
+  }
+  c->n_units = int64_t(cfg.n_layers) * cfg.batch * cfg.n_kv_heads;
+  c->budget = cfg.budget;
+  c->max_warps = c->num_sms * kDecodeWarpsPerCta;
+  const size_t slots = size_t(c->n_units) * cfg.budget;
+  reskv_status st = RESKV_OK;
+  if ((st = dalloc(&c->kslots, slots * kHeadDim, "cache keys")) != RESKV_OK ||
+      (st = dalloc(&c->vslots, slots * kHeadDim, "cache values")) != RESKV_OK ||
+      (st = dalloc(&c->logc, slots, "log counts")) != RESKV_OK ||
+      (st = dalloc(&c->slot_pos, slots, "slot positions")) != RESKV_OK ||
+      (st = dalloc(&c->counts, slots, "slot counts")) != RESKV_OK ||
+      (st = dalloc(&c->n_main, size_t(c->n_units), "n_main")) != RESKV_OK ||
+      (st = dalloc(&c->n_res, size_t(c->n_units), "n_res")) != RESKV_OK ||
+      (st = dalloc(&c->partials, decode_partials_floats(c->n_units, c->max_warps, cfg.group),
+                   "decode workspace")) != RESKV_OK ||
+      (st = dalloc(&c->tickets, size_t(c->n_units), "decode tickets")) != RESKV_OK ||
+      (st = dalloc(&c->status, 1, "status word")) != RESKV_OK) {
+    free_handle(c);
+    return st;
+  }
+  err = cudaMemsetAsync(c->kslots, 0, slots * kHeadDim * 2, stream);
+  if (err == cudaSuccess) err = cudaMemsetAsync(c->vslots, 0, slots * kHeadDim * 2, stream);
+  if (err == cudaSuccess) err = cudaMemsetAsync(c->logc, 0, slots * 4, stream);
+  if (err == cudaSuccess) err = cudaMemsetAsync(c->slot_pos, 0xff, slots * 4, stream);
+  if (err == cudaSuccess) err = cudaMemsetAsync(c->counts, 0, slots * 4, stream);
+  if (err == cudaSuccess) err = cudaMemsetAsync(c->tickets, 0, size_t(c->n_units) * 4, stream);
+  if (err == cudaSuccess) err = cudaMemsetAsync(c->status, 0, 4, stream);
+  if (err != cudaSuccess) {
+    free_handle(c);
+    return cuda_fail(err, "initialising the cache");
+  }
+  *out = c;
+  return RESKV_OK;
+}
+
+void release_handle(reskv_cache* c) { free_handle(c); }
+
+}  // namespace reskv
+
+using namespace reskv;
+
+extern "C" {
+
+void reskv_config_default(reskv_config* cfg) {
+  if (!cfg) return;
+  std::memset(cfg, 0, sizeof(*cfg));
+  cfg->head_dim = kHeadDim;
+  cfg->group = 4;
+  cfg->recent_window = 64;
+  cfg->n_obs = 128;
+  cfg->n_fit = 96;
+  cfg->n_val = 32;
+  cfg->pool_kernel = 5;
+  cfg->score_mode = RESKV_SCORE_OBS_POOL;
+  cfg->n_grid = 5;
+  const float grid[5] = {0.0f, 0.05f, 0.10f, 0.15f, 0.20f};
+  for (int i = 0; i < 5; ++i) cfg->grid_ratios[i] = grid[i];
+  cfg->lloyd_iters = 4;
+  cfg->delta = 0.01f;
+  cfg->beta = 1.0f;
+  cfg->residual_override = nullptr;
+  cfg->gate_mode = RESKV_GATE_DYNAMIC;
+  cfg->tau = 0.25f;
+  cfg->alpha = 12.0f;
+  cfg->g_min = 0.0f;
+  cfg->g_fixed = 1.0f;
+  cfg->keep_debug = 0;
+}
+
+const char* reskv_last_error(void) { return g_last_error.c_str(); }
+
+reskv_status reskv_build_cache(const reskv_config* cfg, const void* const* K_layers,
+                               const void* const* V_layers, const void* const* Qobs_layers,
+                               void* stream, reskv_cache** out) {
+  g_last_error.clear();
+  reskv_status st = validate_shape(cfg);
+  if (st != RESKV_OK) return st;
+  if (!out || !K_layers || !V_layers) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  reskv_cache* c = nullptr;
+  st = build_all_layers(&c, *cfg, cfg->residual_override, K_layers, V_layers, Qobs_layers,
+                        static_cast<cudaStream_t>(stream));
+  if (st == RESKV_OK) *out = c;
+  return st;
+}
+
+reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache* h, void* stream,
+                                reskv_cache** out) {
+  g_last_error.clear();
+  reskv_status st = validate_shape(cfg);
+  if (st != RESKV_OK) return st;
+  if (!h || !out || !h->n_main || !h->n_res || !h->kslots || !h->vslots || !h->logc)
+    return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  const int64_t U = int64_t(cfg->n_layers) * cfg->batch * cfg->n_kv_heads;
+  for (int64_t u = 0; u < U; ++u) {
+    if (h->n_main[u] < 1 || h->n_res[u] < 0 ||
+        int64_t(h->n_main[u]) + h->n_res[u] > cfg->budget)
+      return fail(RESKV_ERR_INVALID_ARG,
+                  "unit " + std::to_string(u) + ": need 1 <= n_main and n_main + n_res <= budget");
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  reskv_cache* c = nullptr;
+  if ((st = alloc_handle(*cfg, s, &c)) != RESKV_OK) return st;
+  const size_t slots = size_t(U) * cfg->budget;
+  cudaError_t err = cudaMemcpyAsync(c->kslots, h->kslots, slots * kHeadDim * 2,
+                                    cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess)
+    err = cudaMemcpyAsync(c->vslots, h->vslots, slots * kHeadDim * 2, cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess)
+    err = cudaMemcpyAsync(c->logc, h->logc, slots * 4, cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess)
+    err = cudaMemcpyAsync(c->n_main, h->n_main, size_t(U) * 4, cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess)
+    err = cudaMemcpyAsync(c->n_res, h->n_res, size_t(U) * 4, cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess && h->slot_pos)
+    err = cudaMemcpyAsync(c->slot_pos, h->slot_pos, slots * 4, cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess && h->counts)
+    err = cudaMemcpyAsync(c->counts, h->counts, slots * 4, cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+  if (err != cudaSuccess) {
+    release_handle(c);
+    return cuda_fail(err, "importing the cache");
+  }
+  *out = c;
+  return RESKV_OK;
+}
+
+reskv_status reskv_export_cache(const reskv_cache* c, reskv_host_cache* h, void* stream) {
+  g_last_error.clear();
+  if (!c || !h || !h->n_main || !h->n_res || !h->kslots || !h->vslots || !h->logc ||
+      !h->slot_pos || !h->counts)
+    return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t U = size_t(c->n_units), slots = U * c->budget;
+  cudaError_t err = cudaMemcpyAsync(h->kslots, c->kslots, slots * kHeadDim * 2,
+                                    cudaMemcpyDeviceToHost, s);
+  if (err == cudaSuccess)
+    err = cudaMemcpyAsync(h->vslots, c->vslots, slots * kHeadDim * 2, cudaMemcpyDeviceToHost, s);
+  if (err == cudaSuccess) err = cudaMemcpyAsync(h->logc, c->logc, slots * 4, cudaMemcpyDeviceToHost, s);
+  if (err == cudaSuccess)
+    err = cudaMemcpyAsync(h->slot_pos, c->slot_pos, slots * 4, cudaMemcpyDeviceToHost, s);
+  if (err == cudaSuccess)
+    err = cudaMemcpyAsync(h->counts, c->counts, slots * 4, cudaMemcpyDeviceToHost, s);
+  if (err == cudaSuccess) err = cudaMemcpyAsync(h->n_main, c->n_main, U * 4, cudaMemcpyDeviceToHost, s);
+  if (err == cudaSuccess) err = cudaMemcpyAsync(h->n_res, c->n_res, U * 4, cudaMemcpyDeviceToHost, s);
+  if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+  if (err != cudaSuccess) return cuda_fail(err, "exporting the cache");
+  return RESKV_OK;
+}
+
+reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* Q, void* O,
+                               void* stream) {
+  if (!c || !Q || !O) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  const reskv_config& cfg = c->cfg;
+  if (layer < -1 || layer >= cfg.n_layers)
+    return fail(RESKV_ERR_INVALID_ARG, "layer must be -1 or in [0, n_layers)");
+  if (!aligned16(Q) || !aligned16(O))
+    return fail(RESKV_ERR_INVALID_ARG, "Q and O must be 16-byte aligned");
+  const int64_t per_layer = int64_t(cfg.batch) * cfg.n_kv_heads;
+  DecodeParams p{};
+  p.kslots = c->kslots;
+  p.vslots = c->vslots;
+  p.logc = c->logc;
+  p.n_main = c->n_main;
+  p.n_res = c->n_res;
+  p.Q = static_cast<const __nv_bfloat16*>(Q);
+  p.O = static_cast<float*>(O);
+  p.partials = c->partials;
+  p.tickets = c->tickets;
+  p.status = c->status;
+  p.unit0 = layer < 0 ? 0 : int64_t(layer) * per_layer;
+  p.n_units = int32_t(layer < 0 ? c->n_units : per_layer);
+  p.budget = c->budget;
+  p.n_kv_heads = cfg.n_kv_heads;
+  p.total_slots = int64_t(p.n_units) * c->budget;
+  // one warp per >= 32 slots, at most a full wave of 8 warps per SM
+  int64_t W = cfg.decode_warps > 0 ? cfg.decode_warps : p.total_slots / 32;
+  if (W > p.total_slots) W = p.total_slots;
+  if (W < 1) W = 1;
+  if (W > c->max_warps) W = c->max_warps;
+  p.n_warps = int32_t(W);
+  p.gate_mode = cfg.gate_mode;
+  p.tau = cfg.tau;
+  p.alpha = cfg.alpha;
+  p.g_min = cfg.g_min;
+  p.g_fixed = cfg.g_fixed;
+  const int n_ctas = int((W + kDecodeWarpsPerCta - 1) / kDecodeWarpsPerCta);
+  cudaError_t err = launch_decode(p, cfg.group, n_ctas, static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return cuda_fail(err, "decode launch");
+  return RESKV_OK;
+}
+
+void reskv_free(reskv_cache* c) {
+  if (!c) return;
+  cudaDeviceSynchronize();
+  free_handle(c);
+}
+
+reskv_status reskv_check_status(const reskv_cache* c) {
+  if (!c) return fail(RESKV_ERR_INVALID_ARG, "NULL handle");
+  uint32_t word = 0;
+  cudaError_t err = cudaDeviceSynchronize();
+  if (err == cudaSuccess) err = cudaMemcpy(&word, c->status, 4, cudaMemcpyDeviceToHost);
+  if (err != cudaSuccess) return cuda_fail(err, "reading the status word");
+  if (word != 0)
+    return fail(RESKV_ERR_DEVICE_STATUS, "kernel status word " + std::to_string(word) +
+                                             " (1 = bounded wait timed out, 2 = index out of range)");
+  return RESKV_OK;
+}
+
+reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info) {
+  if (!c || !info) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  info->n_units = c->n_units;
+  info->budget = c->budget;
+  info->head_dim = kHeadDim;
+  info->slot_bytes = 2 * kSlotRowBytes;
+  info->cache_bytes = c->n_units * int64_t(c->budget) * (2 * kSlotRowBytes + 4);
+  return RESKV_OK;
+}
+
+reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_dst, size_t bytes) {
+  if (!c || !host_dst) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  const void* src = nullptr;
+  size_t need = 0;
+  const size_t U = size_t(c->n_units);
+  const size_t ncand = c->candidates.size();
+  switch (what) {
+    case RESKV_DEBUG_SCORES:
+      src = c->dbg_scores;
+      need = U * size_t(c->cfg.seq_len) * 8;
+      break;
+    case RESKV_DEBUG_RANKED:
+      src = c->dbg_ranked;
+      need = U * size_t(c->dbg_n_top) * 4;
+      break;
+    case RESKV_DEBUG_LOSSES:
+      src = c->dbg_losses;
+      need = U * (1 + ncand) * 8;
+      break;
+    case RESKV_DEBUG_CANDIDATES:
+      if (bytes != ncand * 4) return fail(RESKV_ERR_INVALID_ARG, "size mismatch");
+      if (ncand) std::memcpy(host_dst, c->candidates.data(), bytes);
+      return RESKV_OK;
+    default:
+      return fail(RESKV_ERR_INVALID_ARG, "unknown debug array");
+  }
+  if (!src) return fail(RESKV_ERR_INVALID_ARG, "intermediate not kept (keep_debug was 0)");
+  if (bytes != need)
+    return fail(RESKV_ERR_INVALID_ARG, "size mismatch: need " + std::to_string(need) + " bytes");
+  cudaError_t err = cudaDeviceSynchronize();
+  if (err == cudaSuccess) err = cudaMemcpy(host_dst, src, bytes, cudaMemcpyDeviceToHost);
+  if (err != cudaSuccess) return cuda_fail(err, "exporting an intermediate");
+  return RESKV_OK;
+}
+
+}  // extern "C"

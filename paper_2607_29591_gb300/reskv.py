@@ -1,0 +1,284 @@
+"""Python binding of the ResKV C ABI (include/reskv.h).
+
+Argument marshalling only: every step of construction and decode runs in the
+CUDA library ``libreskv.so``.  Tensors are passed by ``data_ptr()``; streams
+default to torch's current stream.  Importing this module does not load the
+library; the first call does, and fails loudly if it has not been built.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libreskv.so")
+
+RESKV_OK = 0
+STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "OOM", 4: "CUDA",
+                5: "DEVICE_STATUS"}
+RESKV_SCORE_OBS_POOL, RESKV_SCORE_KEYNORM = 0, 1
+RESKV_GATE_DYNAMIC, RESKV_GATE_FIXED = 0, 1
+RESKV_DEBUG_SCORES, RESKV_DEBUG_RANKED, RESKV_DEBUG_LOSSES, RESKV_DEBUG_CANDIDATES = 0, 1, 2, 3
+MAX_GRID = 8
+
+
+class ReskvError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"reskv status {STATUS_NAMES.get(status, status)}: {msg}")
+        self.status = status
+
+
+class reskv_config(ctypes.Structure):
+    _fields_ = [
+        ("batch", ctypes.c_int32), ("n_layers", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+        ("group", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("seq_len", ctypes.c_int64),
+        ("budget", ctypes.c_int32), ("recent_window", ctypes.c_int32), ("n_obs", ctypes.c_int32),
+        ("n_fit", ctypes.c_int32), ("n_val", ctypes.c_int32), ("pool_kernel", ctypes.c_int32),
+        ("score_mode", ctypes.c_int32), ("n_grid", ctypes.c_int32),
+        ("grid_ratios", ctypes.c_float * MAX_GRID), ("lloyd_iters", ctypes.c_int32),
+        ("delta", ctypes.c_float), ("beta", ctypes.c_float),
+        ("residual_override", ctypes.POINTER(ctypes.c_int32)),
+        ("gate_mode", ctypes.c_int32), ("tau", ctypes.c_float), ("alpha", ctypes.c_float),
+        ("g_min", ctypes.c_float), ("g_fixed", ctypes.c_float), ("keep_debug", ctypes.c_int32),
+        ("decode_warps", ctypes.c_int32),
+    ]
+
+
+class reskv_host_cache(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in
+                ("n_main", "n_res", "kslots", "vslots", "logc", "slot_pos", "counts")]
+
+
+class reskv_cache_info(ctypes.Structure):
+    _fields_ = [("n_units", ctypes.c_int64), ("budget", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("slot_bytes", ctypes.c_int64),
+                ("cache_bytes", ctypes.c_int64)]
+
+
+_lib = None
+
+
+def load_library():
+    """Load libreskv.so (built in-tree by ``paper_2607_29591_gb300.build``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                           "`python -m paper_2607_29591_gb300.build` (there is no fallback)")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+    cfgp = ctypes.POINTER(reskv_config)
+    lib.reskv_config_default.argtypes = [cfgp]
+    lib.reskv_config_default.restype = None
+    lib.reskv_build_cache.argtypes = [cfgp, ctypes.POINTER(vp), ctypes.POINTER(vp),
+                                      ctypes.POINTER(vp), vp, ctypes.POINTER(vp)]
+    lib.reskv_build_cache.restype = i32
+    lib.reskv_decode_attn.argtypes = [vp, i32, vp, vp, vp]
+    lib.reskv_decode_attn.restype = i32
+    lib.reskv_free.argtypes = [vp]
+    lib.reskv_free.restype = None
+    lib.reskv_last_error.argtypes = []
+    lib.reskv_last_error.restype = ctypes.c_char_p
+    lib.reskv_check_status.argtypes = [vp]
+    lib.reskv_check_status.restype = i32
+    lib.reskv_get_info.argtypes = [vp, ctypes.POINTER(reskv_cache_info)]
+    lib.reskv_get_info.restype = i32
+    lib.reskv_import_cache.argtypes = [cfgp, ctypes.POINTER(reskv_host_cache), vp,
+                                       ctypes.POINTER(vp)]
+    lib.reskv_import_cache.restype = i32
+    lib.reskv_export_cache.argtypes = [vp, ctypes.POINTER(reskv_host_cache), vp]
+    lib.reskv_export_cache.restype = i32
+    lib.reskv_export_debug.argtypes = [vp, i32, vp, sz]
+    lib.reskv_export_debug.restype = i32
+    _lib = lib
+    return lib
+
+
+def _check(status: int):
+    if status != RESKV_OK:
+        raise ReskvError(status, load_library().reskv_last_error().decode())
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dptr(t, dtype_name: str, what: str):
+    """Device pointer of a contiguous CUDA tensor of the expected dtype."""
+    if not t.is_cuda:
+        raise ValueError(f"{what} must be a CUDA tensor")
+    if str(t.dtype) != dtype_name:
+        raise ValueError(f"{what} must be {dtype_name}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{what} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+class Cache:
+    """Owning wrapper of a reskv_cache* handle (freed with reskv_free)."""
+
+    def __init__(self, handle: ctypes.c_void_p, cfg: reskv_config):
+        self.handle = handle
+        self.cfg = cfg
+
+    def free(self):
+        if self.handle:
+            load_library().reskv_free(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def reskv_config_default(**fields) -> reskv_config:
+    """reskv_config with the paper's defaults, then ``fields`` applied.
+
+    ``grid_ratios`` may be a sequence (sets n_grid); ``residual_override`` a
+    numpy int32 array of per-unit r (kept alive on the returned struct).
+    """
+    cfg = reskv_config()
+    load_library().reskv_config_default(ctypes.byref(cfg))
+    for k, v in fields.items():
+        if k == "grid_ratios":
+            vals = list(v)
+            cfg.n_grid = len(vals)
+            for i in range(MAX_GRID):
+                cfg.grid_ratios[i] = vals[i] if i < len(vals) else 0.0
+        elif k == "residual_override":
+            if v is None:
+                cfg.residual_override = None
+                cfg._override_keepalive = None
+            else:
+                arr = np.ascontiguousarray(v, dtype=np.int32)
+                cfg._override_keepalive = arr
+                cfg.residual_override = arr.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
+        else:
+            setattr(cfg, k, v)
+    return cfg
+
+
+def reskv_last_error() -> str:
+    return load_library().reskv_last_error().decode()
+
+
+def reskv_build_cache(cfg: reskv_config, K_layers: Sequence, V_layers: Sequence,
+                      Qobs_layers: Optional[Sequence] = None, stream=None) -> Cache:
+    """Alg. 1 on the GPU.  K_layers[l], V_layers[l]: bf16 [B, H_kv, s, d] CUDA
+    tensors; Qobs_layers[l]: bf16 [B, H_kv*G, n_obs, d] or None."""
+    L = cfg.n_layers
+    if len(K_layers) != L or len(V_layers) != L:
+        raise ValueError("one K and one V tensor per layer")
+    kp = (ctypes.c_void_p * L)(*[_dptr(k, "torch.bfloat16", "K").value for k in K_layers])
+    vp = (ctypes.c_void_p * L)(*[_dptr(v, "torch.bfloat16", "V").value for v in V_layers])
+    qp = None
+    if Qobs_layers is not None:
+        if len(Qobs_layers) != L:
+            raise ValueError("one Qobs tensor per layer")
+        qp = (ctypes.c_void_p * L)(*[_dptr(q, "torch.bfloat16", "Qobs").value
+                                     for q in Qobs_layers])
+    out = ctypes.c_void_p()
+    _check(load_library().reskv_build_cache(ctypes.byref(cfg), kp, vp, qp, _stream(stream),
+                                            ctypes.byref(out)))
+    return Cache(out, cfg)
+
+
+def reskv_decode_attn(cache: Cache, layer: int, Q, O, stream=None) -> None:
+    """Alg. 2.  layer >= 0: Q bf16 [B, H_q, d], O fp32 [B, H_q, d]; layer == -1:
+    every layer, Q [L, B, H_q, d] and O likewise."""
+    _check(load_library().reskv_decode_attn(cache.handle, int(layer),
+                                            _dptr(Q, "torch.bfloat16", "Q"),
+                                            _dptr(O, "torch.float32", "O"), _stream(stream)))
+
+
+def reskv_free(cache: Cache) -> None:
+    cache.free()
+
+
+def reskv_check_status(cache: Cache) -> None:
+    _check(load_library().reskv_check_status(cache.handle))
+
+
+def reskv_get_info(cache: Cache) -> dict:
+    info = reskv_cache_info()
+    _check(load_library().reskv_get_info(cache.handle, ctypes.byref(info)))
+    return {f: getattr(info, f) for f, _ in info._fields_}
+
+
+def _host_view(arrs: dict) -> reskv_host_cache:
+    h = reskv_host_cache()
+    for k, _ in h._fields_:
+        a = arrs.get(k)
+        setattr(h, k, None if a is None else a.ctypes.data)
+    return h
+
+
+def reskv_import_cache(cfg: reskv_config, n_main, n_res, kslots, vslots, logc,
+                       slot_pos=None, counts=None, stream=None) -> Cache:
+    """Build a handle from host numpy arrays (layout as in include/reskv.h):
+    kslots/vslots uint16 bf16 bits [U, b, d], logc float32 [U, b]."""
+    arrs = dict(n_main=np.ascontiguousarray(n_main, np.int32),
+                n_res=np.ascontiguousarray(n_res, np.int32),
+                kslots=np.ascontiguousarray(kslots, np.uint16),
+                vslots=np.ascontiguousarray(vslots, np.uint16),
+                logc=np.ascontiguousarray(logc, np.float32),
+                slot_pos=None if slot_pos is None else np.ascontiguousarray(slot_pos, np.int32),
+                counts=None if counts is None else np.ascontiguousarray(counts, np.int32))
+    U = cfg.n_layers * cfg.batch * cfg.n_kv_heads
+    b, d = cfg.budget, cfg.head_dim
+    for k, shape in (("n_main", (U,)), ("n_res", (U,)), ("kslots", (U, b, d)),
+                     ("vslots", (U, b, d)), ("logc", (U, b)), ("slot_pos", (U, b)),
+                     ("counts", (U, b))):
+        if arrs[k] is not None and arrs[k].shape != shape:
+            raise ValueError(f"{k} must have shape {shape}, got {arrs[k].shape}")
+    h = _host_view(arrs)
+    out = ctypes.c_void_p()
+    _check(load_library().reskv_import_cache(ctypes.byref(cfg), ctypes.byref(h), _stream(stream),
+                                             ctypes.byref(out)))
+    return Cache(out, cfg)
+
+
+def reskv_export_cache(cache: Cache, stream=None) -> dict:
+    """Copy the cache layout to host numpy arrays."""
+    cfg = cache.cfg
+    U = cfg.n_layers * cfg.batch * cfg.n_kv_heads
+    b, d = cfg.budget, cfg.head_dim
+    arrs = dict(n_main=np.zeros(U, np.int32), n_res=np.zeros(U, np.int32),
+                kslots=np.zeros((U, b, d), np.uint16), vslots=np.zeros((U, b, d), np.uint16),
+                logc=np.zeros((U, b), np.float32), slot_pos=np.zeros((U, b), np.int32),
+                counts=np.zeros((U, b), np.int32))
+    h = _host_view(arrs)
+    _check(load_library().reskv_export_cache(cache.handle, ctypes.byref(h), _stream(stream)))
+    return arrs
+
+
+def reskv_export_debug(cache: Cache, what: int, n_cand: Optional[int] = None) -> np.ndarray:
+    """Construction intermediates (cfg.keep_debug must have been set)."""
+    cfg = cache.cfg
+    U = cfg.n_layers * cfg.batch * cfg.n_kv_heads
+    s, b = cfg.seq_len, cfg.budget
+    n_top = max(min(b, s) - min(cfg.recent_window, s), 0)
+    if what == RESKV_DEBUG_CANDIDATES:
+        out = np.zeros(n_cand if n_cand is not None else 0, np.int32)
+    elif what == RESKV_DEBUG_SCORES:
+        out = np.zeros((U, s), np.float64)
+    elif what == RESKV_DEBUG_RANKED:
+        out = np.zeros((U, n_top), np.int32)
+    elif what == RESKV_DEBUG_LOSSES:
+        out = np.zeros((U, 1 + (n_cand or 0)), np.float64)
+    else:
+        raise ValueError("unknown debug array")
+    _check(load_library().reskv_export_debug(cache.handle, int(what),
+                                             ctypes.c_void_p(out.ctypes.data), out.nbytes))
+    return out

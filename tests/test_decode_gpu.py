@@ -1,0 +1,260 @@
+"""GPU decode (Alg. 2) through the C ABI against the fp64 oracle.
+
+Caches are imported through reskv_import_cache: either built by the oracle
+(Alg. 1 in fp64) or assembled from seeded synthetic rows with ragged
+main/residual splits, so that the decode kernel is checked on its own.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+from scipy.special import softmax
+
+import oracle as orc
+from paper_2607_29591_gb300 import build as B
+from paper_2607_29591_gb300 import reskv as R
+from paper_2607_29591_gb300 import workloads as wl
+
+from helpers import (assert_north_star, bf16_bits, bf16_to_f64, empty_layout, errors,
+                     put_unit, unit_from_layout)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    B.build()
+    return R.load_library()
+
+
+def ocfg_from(cfg):
+    return orc.OracleConfig(budget=cfg.budget, gate_mode=cfg.gate_mode, tau=cfg.tau,
+                            alpha=cfg.alpha, g_min=cfg.g_min, g_fixed=cfg.g_fixed)
+
+
+def synthetic_layout(L, Bt, H, b, splits, seed_layer=0, s=None):
+    """Units filled with generator rows: main = first m rows, residual = next r
+    rows, counts drawn from the hash (some zero)."""
+    U = L * Bt * H
+    s = s or (b + 64)
+    w = wl.Workload("synthetic", L, Bt, H, 4, 128, s, b, 0, 0, 0, 0, "fixed:0", 1)
+    lay = empty_layout(U, b)
+    rng = np.random.default_rng(1234)
+    for u in range(U):
+        m, r = splits[u]
+        l, rem = divmod(u, Bt * H)
+        bb, h = divmod(rem, H)
+        K, V = wl.unit_kv(w, l + seed_layer, bb, h)
+        lay["n_main"][u], lay["n_res"][u] = m, r
+        lay["kslots"][u, :m + r] = bf16_bits(K[:m + r])
+        lay["vslots"][u, :m + r] = bf16_bits(V[:m + r])
+        lay["slot_pos"][u, :m] = np.arange(m)
+        if r:
+            c = rng.integers(0, 200, r)
+            c[rng.random(r) < 0.1] = 0
+            lay["counts"][u, m:m + r] = c
+            with np.errstate(divide="ignore"):
+                lay["logc"][u, m:m + r] = np.log(c.astype(np.float64)).astype(np.float32)
+    return w, lay
+
+
+def queries_for(w, L, Bt, H, G, lay_K_source_rows=None, step=0):
+    """Decode queries [L, B, H*G, d] aimed at the units' first rows."""
+    Q = torch.empty((L, Bt, H * G, 128), dtype=torch.bfloat16)
+    for l in range(L):
+        for bb in range(Bt):
+            for h in range(H):
+                K, _ = wl.unit_kv(w, l, bb, h)
+                q = wl.unit_decode_queries(w, l, bb, h, K, step + 1)[:, step]
+                Q[l, bb, h * G:(h + 1) * G] = q[:G]
+    return Q
+
+
+def oracle_decode_all(lay, Q, cfg):
+    L, Bt, Hq, d = Q.shape
+    H = cfg.n_kv_heads
+    G = Hq // H
+    qf = bf16_to_f64(Q)
+    out = np.zeros((L, Bt, Hq, d))
+    oc = ocfg_from(cfg)
+    for l in range(L):
+        for bb in range(Bt):
+            for h in range(H):
+                u = (l * Bt + bb) * H + h
+                uc = unit_from_layout(lay, u)
+                out[l, bb, h * G:(h + 1) * G] = orc.decode_unit(uc, qf[l, bb, h * G:(h + 1) * G], oc)
+    return out
+
+
+def run_decode(cache, Q, layer=-1):
+    Qd = Q.cuda().contiguous()
+    O = torch.full(Qd.shape, float("nan"), dtype=torch.float32, device="cuda")
+    R.reskv_decode_attn(cache, layer, Qd, O)
+    torch.cuda.synchronize()
+    return O
+
+
+def test_tiny_oracle_built_cache():
+    """Tiny workload: s = 4096, b = 256 = 224 main + 32 residual (fixed), 16 decode queries."""
+    w = wl.WORKLOADS["tiny"]
+    K, V = wl.unit_kv(w, 0, 0, 0)
+    Qo = wl.unit_obs_queries(w, 0, 0, 0, K)
+    Qd = wl.unit_decode_queries(w, 0, 0, 0, K, w.steps)
+    oc = orc.OracleConfig(budget=w.budget, residual_override=32)
+    cache = orc.build_unit(bf16_to_f64(K), bf16_to_f64(V), bf16_to_f64(Qo), oc)
+    assert cache.r == 32 and len(cache.main_pos) == 224
+    lay = empty_layout(1, w.budget)
+    put_unit(lay, 0, cache)
+    cfg = R.reskv_config_default(batch=1, n_layers=1, n_kv_heads=1, group=4, seq_len=w.seq_len,
+                                 budget=w.budget)
+    h = R.reskv_import_cache(cfg, **lay)
+    qf = bf16_to_f64(Qd)
+    worst = (0.0, 0.0)
+    for t in range(w.steps):
+        q = Qd[:, t].reshape(1, 4, 128).contiguous()
+        O = run_decode(h, q, layer=0).cpu().numpy()[0]
+        ref = orc.decode_unit(cache, qf[:, t], oc)
+        mx, rel = assert_north_star(O, ref, f"step {t}")
+        worst = (max(worst[0], mx), max(worst[1], rel))
+    assert worst[1] < 1e-4          # fp32 accumulation lands far inside the bar
+    R.reskv_check_status(h)
+    h.free()
+
+
+SPLITS = [(1, 0), (300, 0), (250, 50), (100, 7), (17, 1), (200, 60), (64, 12), (299, 1),
+          (150, 150), (33, 0), (5, 200), (260, 40)]
+
+
+@pytest.mark.parametrize("decode_warps", [0, 1, 3, 17, 64, 5000])
+def test_ragged_layout_all_layers(decode_warps):
+    """12 units (2 layers x 3 batch x 2 KV heads), b = 300 (rows straddle the
+    8-slot stages), ragged main/residual splits with empty entries and unused
+    tail slots; one all-layer launch cut into various warp counts."""
+    L, Bt, H, G, b = 2, 3, 2, 4, 300
+    w, lay = synthetic_layout(L, Bt, H, b, SPLITS)
+    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+                                 budget=b, decode_warps=decode_warps)
+    h = R.reskv_import_cache(cfg, **lay)
+    Q = queries_for(w, L, Bt, H, G)
+    O = run_decode(h, Q).cpu().numpy()
+    ref = oracle_decode_all(lay, Q, cfg)
+    assert not np.isnan(O).any()
+    mx, rel = assert_north_star(O, ref, f"warps {decode_warps}")
+    assert rel < 1e-4
+    R.reskv_check_status(h)
+
+
+def test_per_layer_calls_match_all_layer_call():
+    L, Bt, H, G, b = 2, 3, 2, 4, 300
+    w, lay = synthetic_layout(L, Bt, H, b, SPLITS)
+    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+                                 budget=b)
+    h = R.reskv_import_cache(cfg, **lay)
+    Q = queries_for(w, L, Bt, H, G)
+    O_all = run_decode(h, Q).cpu().numpy()
+    for l in range(L):
+        O_l = run_decode(h, Q[l].contiguous(), layer=l).cpu().numpy()
+        mx, rel = errors(O_l, O_all[l].astype(np.float64))
+        assert rel < 1e-6
+
+
+def test_determinism_and_split_invariance():
+    L, Bt, H, G, b = 2, 3, 2, 4, 300
+    w, lay = synthetic_layout(L, Bt, H, b, SPLITS)
+    Q = queries_for(w, L, Bt, H, G)
+    outs = []
+    for dw in (1, 2, 4, 16, 0):
+        cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G,
+                                     seq_len=w.seq_len, budget=b, decode_warps=dw)
+        h = R.reskv_import_cache(cfg, **lay)
+        o1 = run_decode(h, Q)
+        o2 = run_decode(h, Q)
+        assert torch.equal(o1, o2), "decode must be bitwise deterministic"
+        outs.append(o1.cpu().numpy().astype(np.float64))
+    for o in outs[1:]:
+        assert errors(o, outs[0])[1] < 1e-6
+
+
+@pytest.mark.parametrize("G", [1, 2])
+def test_group_sizes(G):
+    L, Bt, H, b = 1, 2, 3, 256
+    splits = [(200, 56), (256, 0), (10, 100), (128, 64), (1, 255), (100, 3)]
+    w, lay = synthetic_layout(L, Bt, H, b, splits)
+    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+                                 budget=b)
+    h = R.reskv_import_cache(cfg, **lay)
+    Q = queries_for(w, L, Bt, H, G)
+    O = run_decode(h, Q).cpu().numpy()
+    assert_north_star(O, oracle_decode_all(lay, Q, cfg), f"G={G}")
+
+
+def _textbook(q, K, V):
+    return softmax(K @ q / math.sqrt(K.shape[1])) @ V
+
+
+def test_fixed_point_empty_residual_is_eviction():
+    """Sec. 5.4: R empty gives eviction attention over M (Eq. evict)."""
+    L, Bt, H, G, b = 1, 2, 2, 4, 512
+    splits = [(512, 0), (300, 0), (77, 0), (1, 0)]
+    w, lay = synthetic_layout(L, Bt, H, b, splits)
+    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+                                 budget=b)
+    h = R.reskv_import_cache(cfg, **lay)
+    Q = queries_for(w, L, Bt, H, G)
+    O = run_decode(h, Q).cpu().numpy()
+    qf = bf16_to_f64(Q)
+    for u, (m, _) in enumerate(splits):
+        bb, hh = divmod(u, H)
+        Km = orc.bf16_bits_to_f64(lay["kslots"][u, :m])
+        Vm = orc.bf16_bits_to_f64(lay["vslots"][u, :m])
+        for g in range(G):
+            ref = _textbook(qf[0, bb, hh * G + g], Km, Vm)
+            assert_north_star(O[0, bb, hh * G + g], ref, "eviction")
+
+
+def test_fixed_point_gate_zero_is_main_only():
+    L, Bt, H, G, b = 1, 1, 3, 4, 400
+    splits = [(300, 100), (50, 350), (399, 1)]
+    w, lay = synthetic_layout(L, Bt, H, b, splits)
+    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+                                 budget=b, gate_mode=R.RESKV_GATE_FIXED, g_fixed=0.0)
+    h = R.reskv_import_cache(cfg, **lay)
+    Q = queries_for(w, L, Bt, H, G)
+    O = run_decode(h, Q).cpu().numpy()
+    qf = bf16_to_f64(Q)
+    for u, (m, _) in enumerate(splits):
+        Km = orc.bf16_bits_to_f64(lay["kslots"][u, :m])
+        Vm = orc.bf16_bits_to_f64(lay["vslots"][u, :m])
+        for g in range(G):
+            assert_north_star(O[0, 0, u * G + g], _textbook(qf[0, 0, u * G + g], Km, Vm), "g=0")
+
+
+def test_fixed_point_exact_residual_encoding_is_full_attention():
+    """Sec. 4.2, Eq. residual: one entry carrying log Z_E(q) and N_E/Z_E of the
+    evicted tokens for the query of each head (G = 1) recovers o_S; the only
+    error left is the bf16 storage of the entry's value."""
+    s, m, d = 2048, 300, 128
+    w = wl.scaled(wl.WORKLOADS["tiny"], seq_len=s)
+    K, V = wl.unit_kv(w, 0, 0, 0)
+    Qd = wl.unit_decode_queries(w, 0, 0, 0, K, 1)[0, 0]
+    Kf, Vf, q = bf16_to_f64(K), bf16_to_f64(V), bf16_to_f64(Qd)
+    a = Kf[m:] @ q / math.sqrt(d)
+    ZE = np.exp(a).sum()
+    NE = np.exp(a) @ Vf[m:]
+    lay = empty_layout(1, m + 1)
+    lay["n_main"][0], lay["n_res"][0] = m, 1
+    lay["kslots"][0, :m] = bf16_bits(K[:m])
+    lay["vslots"][0, :m] = bf16_bits(V[:m])
+    vbar = orc.round_to_bf16(NE / ZE)
+    lay["vslots"][0, m] = (vbar.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
+    lay["logc"][0, m] = np.float32(np.log(ZE))          # k_bar = 0, so <q, k_bar> = 0
+    cfg = R.reskv_config_default(batch=1, n_layers=1, n_kv_heads=1, group=1, seq_len=s,
+                                 budget=m + 1, gate_mode=R.RESKV_GATE_FIXED, g_fixed=1.0)
+    h = R.reskv_import_cache(cfg, **lay)
+    O = run_decode(h, Qd.reshape(1, 1, 1, d)).cpu().numpy()[0, 0, 0]
+    full = _textbook(q, Kf, Vf)
+    assert_north_star(O, full, "exact encoding")
+    # the residual's share of the output carries only bf16 rounding of v_bar
+    assert errors(O, full)[1] < 4e-3 * ZE / (ZE + np.exp(Kf[:m] @ q / math.sqrt(d)).sum()) + 1e-5
