@@ -1,17 +1,346 @@
-// Construction (Alg. 1) -- kernels follow.
+// Construction of the compressed cache (Alg. 1), layer by layer, on the
+// caller's stream.  Every step is a kernel of construct_kernels.cuh; the host
+// only validates, sizes the scratch buffers and sequences the launches.
 #include <cuda_runtime.h>
 
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "construct_kernels.cuh"
 #include "internal.h"
 
 namespace reskv {
 
+reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_cache** out);
+void release_handle(reskv_cache* c);
+
+namespace {
+
+using namespace build;
+
+reskv_status fail(reskv_status st, const std::string& msg) {
+  set_error(msg);
+  return st;
+}
+
+struct Scratch {
+  std::vector<void*> ptrs;
+  ~Scratch() {
+    for (void* p : ptrs) cudaFree(p);
+  }
+  template <typename T>
+  bool get(T** p, size_t count) {
+    *p = nullptr;
+    if (count == 0) count = 1;
+    if (cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T)) != cudaSuccess) {
+      cudaGetLastError();
+      *p = nullptr;
+      return false;
+    }
+    ptrs.push_back(*p);
+    return true;
+  }
+};
+
+#define RESKV_LAUNCH_CHECK(what)                                                      \
+  do {                                                                               \
+    cudaError_t e_ = cudaGetLastError();                                             \
+    if (e_ != cudaSuccess)                                                           \
+      return fail(RESKV_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e_)); \
+  } while (0)
+
+template <typename K>
+cudaError_t set_smem(K kernel, size_t bytes) {
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(bytes));
+}
+
+int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+}  // namespace
+
 reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
-                              const int32_t* override_host, const void* const* K,
-                              const void* const* V, const void* const* Qobs,
-                              cudaStream_t stream) {
-  (void)out; (void)cfg; (void)override_host; (void)K; (void)V; (void)Qobs; (void)stream;
-  set_error("construction not built yet");
-  return RESKV_ERR_UNSUPPORTED;
+                              const int32_t* override_host, const void* const* Kl,
+                              const void* const* Vl, const void* const* Ql, cudaStream_t stream) {
+  // ---------------- validation ----------------
+  const int64_t s = cfg.seq_len;
+  const int b = cfg.budget;
+  if (cfg.recent_window < 0) return fail(RESKV_ERR_INVALID_ARG, "recent_window must be >= 0");
+  const int P = int(std::min<int64_t>(cfg.recent_window, s));
+  const int n_top = int(std::min<int64_t>(b, s)) - P;
+  if (n_top > kTopMax)
+    return fail(RESKV_ERR_UNSUPPORTED, "budget - recent_window must be <= 8192");
+  const bool all_main = int64_t(b) >= s;
+  const bool proxy = override_host == nullptr && !all_main;
+  const int UL = cfg.batch * cfg.n_kv_heads;
+  const int G = cfg.group;
+  if (cfg.score_mode != RESKV_SCORE_OBS_POOL && cfg.score_mode != RESKV_SCORE_KEYNORM)
+    return fail(RESKV_ERR_INVALID_ARG, "unknown score_mode");
+  if (cfg.pool_kernel < 1 || cfg.pool_kernel % 2 == 0)
+    return fail(RESKV_ERR_INVALID_ARG, "pool_kernel must be a positive odd number");
+  const bool need_q = cfg.score_mode == RESKV_SCORE_OBS_POOL || proxy;
+  if (need_q) {
+    if (!Ql) return fail(RESKV_ERR_INVALID_ARG, "observation queries are required");
+    for (int l = 0; l < cfg.n_layers; ++l)
+      if (!Ql[l]) return fail(RESKV_ERR_INVALID_ARG, "NULL observation-query layer");
+    if (cfg.score_mode == RESKV_SCORE_OBS_POOL && (cfg.n_fit < 1 || cfg.n_fit > cfg.n_obs))
+      return fail(RESKV_ERR_INVALID_ARG, "need 1 <= n_fit <= n_obs");
+    if (proxy) {
+      const int used_fit = cfg.score_mode == RESKV_SCORE_OBS_POOL ? cfg.n_fit : 0;
+      if (cfg.n_val < 1 || used_fit + cfg.n_val > cfg.n_obs)
+        return fail(RESKV_ERR_INVALID_ARG, "need n_val >= 1 and n_fit + n_val <= n_obs");
+    }
+  }
+  for (int l = 0; l < cfg.n_layers; ++l)
+    if (!Kl[l] || !Vl[l]) return fail(RESKV_ERR_INVALID_ARG, "NULL K or V layer");
+  if (cfg.lloyd_iters < 1 || cfg.lloyd_iters > 64)
+    return fail(RESKV_ERR_INVALID_ARG, "lloyd_iters must be in [1, 64]");
+  if (cfg.n_grid < 0 || cfg.n_grid > RESKV_MAX_GRID)
+    return fail(RESKV_ERR_INVALID_ARG, "n_grid must be in [0, 8]");
+  if (!(cfg.delta >= 0.f && cfg.delta < 1.f) || !std::isfinite(cfg.beta))
+    return fail(RESKV_ERR_INVALID_ARG, "delta must be in [0, 1) and beta finite");
+
+  // candidate budgets r = floor(ratio * b) > 0, distinct, ascending (App. B)
+  std::vector<int32_t> cands;
+  if (proxy) {
+    for (int i = 0; i < cfg.n_grid; ++i) {
+      const float ratio = cfg.grid_ratios[i];
+      if (!(ratio >= 0.f && ratio <= 1.f))
+        return fail(RESKV_ERR_INVALID_ARG, "grid ratios must be in [0, 1]");
+      const int r = int(std::floor(double(ratio) * double(b)));
+      if (r > 0 && b - r >= P && std::find(cands.begin(), cands.end(), r) == cands.end())
+        cands.push_back(r);
+    }
+    std::sort(cands.begin(), cands.end());
+  }
+  std::vector<int32_t> ovr;
+  int rmax = 0;
+  if (override_host) {
+    const int64_t U = int64_t(cfg.n_layers) * UL;
+    ovr.assign(override_host, override_host + U);
+    for (int64_t u = 0; u < U; ++u) {
+      const int r = ovr[u];
+      if (r < 0 || r >= b) return fail(RESKV_ERR_INVALID_ARG, "residual_override out of [0, budget)");
+      if (r > 0 && (all_main || b - r < P))
+        return fail(RESKV_ERR_INVALID_ARG,
+                    "residual_override needs budget <= seq_len and budget - r >= recent_window");
+      rmax = std::max(rmax, r);
+    }
+  }
+  for (int32_t r : cands) rmax = std::max(rmax, r);
+  if (rmax > kMaxR) return fail(RESKV_ERR_UNSUPPORTED, "residual entries per unit must be <= 8192");
+
+  // ---------------- handle and scratch ----------------
+  reskv_cache* c = nullptr;
+  reskv_status st = alloc_handle(cfg, stream, &c);
+  if (st != RESKV_OK) return st;
+  c->candidates = cands;
+  const int ncol = 1 + int(cands.size());            // run 0 = pure-main cache
+  const int ntiles = int(cdiv(s, kTile));
+  const int n_fit_rows = cfg.score_mode == RESKV_SCORE_OBS_POOL ? G * cfg.n_fit : 0;
+  const int n_val_rows = proxy ? G * cfg.n_val : 0;
+  const int nchunks = int(cdiv(s, int64_t(kTile) * kValChunkTiles));
+  // entry storage: one slice per run with r > 0
+  std::vector<int32_t> run_off(std::max(ncol, 2), 0);
+  int64_t ent_stride = 0;
+  if (proxy) {
+    for (int i = 0; i < int(cands.size()); ++i) {
+      run_off[1 + i] = int32_t(ent_stride);
+      ent_stride += cands[i];
+    }
+  } else {
+    ent_stride = rmax;
+  }
+
+  Scratch S;
+  double* scores = nullptr;
+  float* A = nullptr;
+  float2* tstats = nullptr;
+  float2* rstats = nullptr;
+  int32_t *top = nullptr, *rank_pos = nullptr, *assign = nullptr, *hist = nullptr;
+  int32_t *ccount = nullptr, *cbase = nullptr, *members = nullptr, *ecount = nullptr;
+  int32_t *r_runs = nullptr, *r_final = nullptr, *chosen = nullptr, *run_off_d = nullptr;
+  int32_t *cand_r_d = nullptr;
+  float *centersT = nullptr, *cnorm = nullptr, *vpart = nullptr, *oS = nullptr;
+  __nv_bfloat16 *kbar = nullptr, *vbar = nullptr;
+  double *rowerr = nullptr, *losses = nullptr;
+  const size_t US = size_t(UL) * size_t(s);
+  const int nruns = proxy ? ncol : 2;
+  bool ok = S.get(&scores, US) && S.get(&top, size_t(UL) * std::max(n_top, 1)) &&
+            S.get(&rank_pos, US) && S.get(&r_runs, size_t(nruns) * UL) &&
+            S.get(&r_final, UL) && S.get(&chosen, UL) && S.get(&run_off_d, run_off.size());
+  if (ok && n_fit_rows > 0)
+    ok = S.get(&A, US) && S.get(&tstats, size_t(UL) * n_fit_rows * ntiles) &&
+         S.get(&rstats, size_t(UL) * n_fit_rows);
+  if (ok && rmax > 0)
+    ok = S.get(&assign, US) && S.get(&hist, size_t(UL) * ntiles * rmax) &&
+         S.get(&ccount, size_t(UL) * rmax) && S.get(&cbase, size_t(UL) * rmax) &&
+         S.get(&members, US) && S.get(&centersT, size_t(UL) * kHeadDim * rmax) &&
+         S.get(&cnorm, size_t(UL) * rmax) && S.get(&kbar, size_t(UL) * ent_stride * kHeadDim) &&
+         S.get(&vbar, size_t(UL) * ent_stride * kHeadDim) &&
+         S.get(&ecount, size_t(UL) * ent_stride);
+  if (ok && proxy)
+    ok = S.get(&vpart, size_t(UL) * n_val_rows * nchunks * kValRec) &&
+         S.get(&oS, size_t(UL) * n_val_rows * kHeadDim) &&
+         S.get(&rowerr, size_t(UL) * n_val_rows) && S.get(&losses, size_t(UL) * ncol) &&
+         S.get(&cand_r_d, ncol);
+  if (ok && cfg.keep_debug) {
+    const size_t U = size_t(c->n_units);
+    cudaError_t e = cudaMalloc(&c->dbg_scores, U * size_t(s) * 8);
+    if (e == cudaSuccess) e = cudaMalloc(&c->dbg_ranked, U * std::max(n_top, 1) * 4);
+    if (e == cudaSuccess) e = cudaMalloc(&c->dbg_losses, U * ncol * 8);
+    if (e == cudaSuccess) e = cudaMemsetAsync(c->dbg_losses, 0, U * ncol * 8, stream);
+    ok = e == cudaSuccess;
+    c->dbg_n_top = n_top;
+  }
+  if (!ok) {
+    cudaGetLastError();
+    release_handle(c);
+    return fail(RESKV_ERR_OOM, "construction scratch allocation failed");
+  }
+
+  auto cleanup_fail = [&](reskv_status e) {
+    release_handle(c);
+    return e;
+  };
+
+  // per-run r arrays (proxy: uniform per run; override: filled per layer)
+  std::vector<int32_t> hr(size_t(nruns) * UL, 0);
+  if (proxy)
+    for (int i = 0; i < int(cands.size()); ++i)
+      std::fill(hr.begin() + size_t(1 + i) * UL, hr.begin() + size_t(2 + i) * UL, cands[i]);
+  std::vector<int32_t> cand_col(ncol, 0);
+  for (int i = 0; i < int(cands.size()); ++i) cand_col[1 + i] = cands[i];
+  if (cudaMemcpyAsync(run_off_d, run_off.data(), run_off.size() * 4, cudaMemcpyHostToDevice,
+                      stream) != cudaSuccess ||
+      (proxy && cudaMemcpyAsync(cand_r_d, cand_col.data(), ncol * 4, cudaMemcpyHostToDevice,
+                                stream) != cudaSuccess))
+    return cleanup_fail(fail(RESKV_ERR_CUDA, "copying run tables"));
+
+  // kernel attributes
+  const size_t sm_obs1 = size_t(kHeadDim) * (kTile + kRowBlk) * 4;
+  const size_t sm_obs2 = sm_obs1 + size_t(8) * kTile * 4;
+  const size_t sm_top = size_t(kTopMax) * 12 + (256 + 32 + 4) * 4;
+  const size_t sm_assign = (size_t(kHeadDim) * (kTile + kRowBlk) + kRowBlk + 8 * kTile) * 4 +
+                           size_t(8) * kTile * 4 + size_t(std::max(rmax, 1)) * 4;
+  const size_t sm_val = size_t(kHeadDim) * (2 * kTile + 2 * kRowBlk) * 4;
+  if (set_smem(k_obs_pass1, sm_obs1) != cudaSuccess || set_smem(k_obs_pass2, sm_obs2) != cudaSuccess ||
+      set_smem(k_topk, sm_top) != cudaSuccess || set_smem(k_lloyd_assign, sm_assign) != cudaSuccess ||
+      set_smem(k_val_full, sm_val) != cudaSuccess)
+    return cleanup_fail(fail(RESKV_ERR_CUDA, "setting kernel shared-memory limits"));
+
+  const double one_minus_delta = 1.0 - double(cfg.delta);
+
+  for (int l = 0; l < cfg.n_layers; ++l) {
+    const __nv_bfloat16* K = static_cast<const __nv_bfloat16*>(Kl[l]);
+    const __nv_bfloat16* V = static_cast<const __nv_bfloat16*>(Vl[l]);
+    const __nv_bfloat16* Q = Ql ? static_cast<const __nv_bfloat16*>(Ql[l]) : nullptr;
+
+    // ---- step 2: token scores ----
+    if (cfg.score_mode == RESKV_SCORE_OBS_POOL) {
+      ObsArgs oa{K, Q, s, G, cfg.n_obs, n_fit_rows, cfg.n_fit, ntiles, tstats, rstats, A};
+      k_obs_pass1<<<dim3(ntiles, UL), kThreads, sm_obs1, stream>>>(oa);
+      k_obs_rowstats<<<unsigned(cdiv(int64_t(UL) * n_fit_rows, 256)), 256, 0, stream>>>(oa, UL);
+      k_obs_pass2<<<dim3(ntiles, UL), kThreads, sm_obs2, stream>>>(oa);
+      k_pool<<<unsigned(cdiv(int64_t(US), 256)), 256, 0, stream>>>(A, scores, s, UL, cfg.pool_kernel);
+    } else {
+      k_score_keynorm<<<unsigned(cdiv(int64_t(US), 256)), 256, 0, stream>>>(K, scores, int64_t(US));
+    }
+    RESKV_LAUNCH_CHECK("scoring");
+    TopArgs ta{scores, s, P, n_top, top, rank_pos, c->status};
+    k_topk<<<UL, kTopThreads, sm_top, stream>>>(ta);
+    RESKV_LAUNCH_CHECK("ranking");
+
+    LloydArgs la{K, V, s, P, n_top, b, ntiles, rmax, top, rank_pos, nullptr, centersT, cnorm,
+                 assign, hist, ccount, cbase, members, kbar, vbar, ecount, ent_stride, 0,
+                 c->status};
+    auto lloyd_run = [&](const int32_t* r_unit, int ent_off) -> reskv_status {
+      la.r_unit = r_unit;
+      la.ent_off = ent_off;
+      k_lloyd_init<<<dim3(rmax, UL), kHeadDim, 0, stream>>>(la);
+      for (int it = 0; it < cfg.lloyd_iters; ++it) {
+        k_lloyd_assign<<<dim3(ntiles, UL), kThreads, sm_assign, stream>>>(la);
+        k_lloyd_scan<<<UL, 256, 0, stream>>>(la);
+        k_lloyd_scatter<<<dim3(ntiles, UL), kTile, 0, stream>>>(la);
+        k_lloyd_update<<<dim3(rmax, UL), kThreads, 0, stream>>>(la, it == cfg.lloyd_iters - 1);
+      }
+      RESKV_LAUNCH_CHECK("residual entries");
+      return RESKV_OK;
+    };
+
+    if (proxy) {
+      // ---- steps 1, 3-14: validation targets, candidates, choice ----
+      ValArgs va{K, V, Q, s, G, cfg.n_obs, cfg.n_val, n_val_rows, nchunks, vpart, oS};
+      k_val_full<<<dim3(nchunks, unsigned(cdiv(n_val_rows, kRowBlk)), UL), kThreads, sm_val, stream>>>(va);
+      k_val_combine<<<dim3(n_val_rows, UL), kHeadDim, 0, stream>>>(va);
+      RESKV_LAUNCH_CHECK("validation targets");
+      if (l == 0 &&
+          cudaMemcpyAsync(r_runs, hr.data(), hr.size() * 4, cudaMemcpyHostToDevice, stream) != cudaSuccess)
+        return cleanup_fail(fail(RESKV_ERR_CUDA, "copying candidate budgets"));
+      for (int run = 0; run < ncol; ++run) {
+        const int32_t* r_unit = r_runs + size_t(run) * UL;
+        if (run > 0) {
+          st = lloyd_run(r_unit, run_off[run]);
+          if (st != RESKV_OK) return cleanup_fail(st);
+        }
+        LossArgs lo{K, V, Q, s, G, cfg.n_obs, cfg.n_val, n_val_rows, P, n_top, b, top, r_unit,
+                    kbar, vbar, ecount, ent_stride, run_off[run], cfg.beta, cfg.gate_mode,
+                    cfg.tau, cfg.alpha, cfg.g_min, cfg.g_fixed, oS, rowerr};
+        k_val_loss<<<dim3(unsigned(cdiv(n_val_rows, 8)), UL), kThreads, 0, stream>>>(lo);
+        k_loss_reduce<<<unsigned(cdiv(UL, 128)), 128, 0, stream>>>(rowerr, losses, n_val_rows, UL,
+                                                                  ncol, run);
+        RESKV_LAUNCH_CHECK("validation loss");
+      }
+      k_choose<<<unsigned(cdiv(UL, 128)), 128, 0, stream>>>(losses, ncol, cand_r_d, UL,
+                                                           one_minus_delta, r_final, chosen);
+      RESKV_LAUNCH_CHECK("choosing r");
+    } else {
+      // fixed r per unit (or the budget covers every token: r = 0)
+      std::vector<int32_t> rl(UL, 0), ch(UL, 0);
+      bool any = false;
+      if (!ovr.empty())
+        for (int i = 0; i < UL; ++i) {
+          rl[i] = ovr[size_t(l) * UL + i];
+          ch[i] = rl[i] > 0 ? 1 : 0;
+          any |= rl[i] > 0;
+        }
+      if (cudaMemcpyAsync(r_final, rl.data(), UL * 4, cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+          cudaMemcpyAsync(chosen, ch.data(), UL * 4, cudaMemcpyHostToDevice, stream) != cudaSuccess ||
+          cudaStreamSynchronize(stream) != cudaSuccess)
+        return cleanup_fail(fail(RESKV_ERR_CUDA, "copying residual counts"));
+      if (any) {
+        st = lloyd_run(r_final, 0);
+        if (st != RESKV_OK) return cleanup_fail(st);
+      }
+    }
+
+    // ---- step 15: pack the chosen cache ----
+    PackArgs pa{K, V, s, P, b, rank_pos, r_final, chosen, run_off_d, kbar, vbar, ecount,
+                ent_stride, cfg.beta, int64_t(l) * UL, c->kslots, c->vslots, c->logc,
+                c->slot_pos, c->counts, c->n_main, c->n_res};
+    k_pack<<<UL, 1024, 0, stream>>>(pa);
+    RESKV_LAUNCH_CHECK("packing");
+
+    if (cfg.keep_debug) {
+      cudaError_t e = cudaMemcpyAsync(c->dbg_scores + size_t(l) * US, scores, US * 8,
+                                      cudaMemcpyDeviceToDevice, stream);
+      if (e == cudaSuccess && n_top > 0)
+        e = cudaMemcpyAsync(c->dbg_ranked + size_t(l) * UL * n_top, top, size_t(UL) * n_top * 4,
+                            cudaMemcpyDeviceToDevice, stream);
+      if (e == cudaSuccess && proxy)
+        e = cudaMemcpyAsync(c->dbg_losses + size_t(l) * UL * ncol, losses, size_t(UL) * ncol * 8,
+                            cudaMemcpyDeviceToDevice, stream);
+      if (e != cudaSuccess) return cleanup_fail(fail(RESKV_ERR_CUDA, "keeping intermediates"));
+    }
+  }
+  // scratch is freed (cudaFree synchronises) when S leaves scope
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cleanup_fail(fail(RESKV_ERR_CUDA, std::string("construction: ") +
+                                                                   cudaGetErrorString(e)));
+  *out = c;
+  return RESKV_OK;
 }
 
 }  // namespace reskv

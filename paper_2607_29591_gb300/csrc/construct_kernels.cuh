@@ -400,5 +400,639 @@ __global__ void __launch_bounds__(kTopThreads, 1) k_topk(TopArgs p) {
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// Residual entries by Lloyd's algorithm (Sec. 5.3, Eqs. residual_partition,
+// summary; App. B: 4 iterations, initial centres = the highest-scored evicted
+// keys).  One "run" builds r_unit[ul] entries for every unit of the layer.
+// E = S \ M_r = { p < s - |P| : rank_pos[p] >= m - |P| },  m = b - r.
+// Deterministic: assignments by (distance, centre index); member sums in
+// fp64 in token order (stable counting sort); no float atomics.
+// ---------------------------------------------------------------------------
+
+constexpr int kMaxR = 8192;
+
+struct LloydArgs {
+  const __nv_bfloat16* K;      // layer keys [UL, s, d]
+  const __nv_bfloat16* V;      // layer values
+  int64_t s;
+  int32_t recent;              // |P| (already clamped to s)
+  int32_t n_top;
+  int32_t budget;
+  int32_t ntiles;
+  int32_t rmax;
+  const int32_t* top;          // [UL, n_top]
+  const int32_t* rank_pos;     // [UL, s]
+  const int32_t* r_unit;       // [UL]
+  float* centersT;             // [UL, d, rmax]  (dim-major)
+  float* cnorm;                // [UL, rmax]
+  int32_t* assign;             // [UL, s] centre index, -1 outside E
+  int32_t* hist;               // [UL, ntiles, rmax] per-tile counts, then offsets
+  int32_t* ccount;             // [UL, rmax] members per centre
+  int32_t* cbase;              // [UL, rmax] first member slot per centre
+  int32_t* members;            // [UL, s] token positions grouped by centre
+  __nv_bfloat16* kbar;         // [UL, ent_stride, d] entries of this run at ent_off
+  __nv_bfloat16* vbar;
+  int32_t* ecount;             // [UL, ent_stride]
+  int64_t ent_stride;
+  int32_t ent_off;
+  uint32_t* status;
+};
+
+__device__ __forceinline__ bool in_evicted(const LloydArgs& p, int ul, int64_t pos, int r) {
+  const int32_t rk = p.rank_pos[int64_t(ul) * p.s + pos];
+  const int32_t keep = p.budget - r - p.recent;           // ranked tokens kept as main
+  return rk >= 0 && rk >= keep;
+}
+
+// centre j = key of the (m - |P| + j)-th ranked token
+__global__ void k_lloyd_init(LloydArgs p) {
+  __shared__ float red[kHeadDim];
+  const int j = blockIdx.x, ul = blockIdx.y, d = threadIdx.x;
+  const int r = p.r_unit[ul];
+  if (j >= r) return;
+  const int32_t keep = p.budget - r - p.recent;
+  const int32_t pos = p.top[int64_t(ul) * p.n_top + keep + j];
+  const float c = __bfloat162float(p.K[(int64_t(ul) * p.s + pos) * kHeadDim + d]);
+  p.centersT[(int64_t(ul) * kHeadDim + d) * p.rmax + j] = c;
+  red[d] = c * c;
+  __syncthreads();
+  if (d == 0) {
+    float n = 0.f;
+    for (int i = 0; i < kHeadDim; ++i) n += red[i];
+    p.cnorm[int64_t(ul) * p.rmax + j] = n;
+  }
+}
+
+// nearest centre of every evicted token of a 128-token tile; per-tile counts
+__global__ void __launch_bounds__(kThreads, 2) k_lloyd_assign(LloydArgs p) {
+  extern __shared__ __align__(16) float sm[];
+  float* Kt = sm;                                   // [128][128]
+  float* Ct = Kt + kHeadDim * kTile;                // [128][32]
+  float* cn = Ct + kHeadDim * kRowBlk;              // [32]
+  float* bd = cn + kRowBlk;                         // [8][128] best distance per warp
+  int* bj = reinterpret_cast<int*>(bd + 8 * kTile); // [8][128] best centre per warp
+  int* cnt = bj + 8 * kTile;                        // [rmax] tile histogram
+  const int tile = blockIdx.x, ul = blockIdx.y;
+  const int r = p.r_unit[ul];
+  if (r == 0) return;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t tok0 = int64_t(tile) * kTile;
+  load_kt(Kt, p.K + int64_t(ul) * p.s * kHeadDim, p.s, tok0);
+  for (int i = threadIdx.x; i < r; i += blockDim.x) cnt[i] = 0;
+  float best[4];
+  int bidx[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    best[j] = INFINITY;
+    bidx[j] = 0x7fffffff;
+  }
+  for (int cb = 0; cb < r; cb += kRowBlk) {
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < kHeadDim * kRowBlk; idx += blockDim.x) {
+      const int k = idx / kRowBlk, c = idx % kRowBlk;
+      Ct[idx] = (cb + c < r) ? p.centersT[(int64_t(ul) * kHeadDim + k) * p.rmax + cb + c] : 0.f;
+    }
+    if (threadIdx.x < kRowBlk)
+      cn[threadIdx.x] = (cb + threadIdx.x < r) ? p.cnorm[int64_t(ul) * p.rmax + cb + threadIdx.x] : 0.f;
+    __syncthreads();
+    float S[4][4];
+    tile_logits(Ct, Kt, S);                         // <c_i, k_j> for centres 4w+i
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int c = cb + 4 * w + i;
+      if (c >= r) continue;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float dist = cn[4 * w + i] - 2.0f * S[i][j];   // ||c||^2 - 2<c,k> (+||k||^2)
+        if (dist < best[j]) {                                 // strict: lower index kept
+          best[j] = dist;
+          bidx[j] = c;
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    bd[w * kTile + 4 * lane + j] = best[j];
+    bj[w * kTile + 4 * lane + j] = bidx[j];
+  }
+  __syncthreads();
+  if (threadIdx.x < kTile) {
+    const int t = threadIdx.x;
+    float b0 = bd[t];
+    int j0 = bj[t];
+    for (int ww = 1; ww < 8; ++ww) {
+      const float b1 = bd[ww * kTile + t];
+      const int j1 = bj[ww * kTile + t];
+      if (b1 < b0 || (b1 == b0 && j1 < j0)) {
+        b0 = b1;
+        j0 = j1;
+      }
+    }
+    const int64_t pos = tok0 + t;
+    if (pos < p.s) {
+      bool ev = in_evicted(p, ul, pos, r);
+      if (ev && (j0 < 0 || j0 >= r)) {        // only a NaN distance gets here
+        report_status(p.status, kStatusBadIndex);
+        j0 = 0;
+      }
+      p.assign[int64_t(ul) * p.s + pos] = ev ? j0 : -1;
+      if (ev) atomicAdd(&cnt[j0], 1);
+    }
+  }
+  __syncthreads();
+  int32_t* h = p.hist + (int64_t(ul) * p.ntiles + tile) * p.rmax;
+  for (int i = threadIdx.x; i < r; i += blockDim.x) h[i] = cnt[i];
+}
+
+// per centre: counts, per-tile offsets (in place) and member bases
+__global__ void k_lloyd_scan(LloydArgs p) {
+  __shared__ int warp_sums[32];
+  const int ul = blockIdx.x;
+  const int r = p.r_unit[ul];
+  if (r == 0) return;
+  const int per = (r + blockDim.x - 1) / blockDim.x;      // centres per thread (contiguous)
+  int total_mine = 0;
+  for (int q = 0; q < per; ++q) {
+    const int j = threadIdx.x * per + q;
+    if (j >= r) break;
+    int run = 0;
+    for (int t = 0; t < p.ntiles; ++t) {
+      int32_t* h = p.hist + (int64_t(ul) * p.ntiles + t) * p.rmax + j;
+      const int c = *h;
+      *h = run;
+      run += c;
+    }
+    p.ccount[int64_t(ul) * p.rmax + j] = run;
+    total_mine += run;
+  }
+  int base = block_exclusive_scan(total_mine, warp_sums, nullptr);
+  for (int q = 0; q < per; ++q) {
+    const int j = threadIdx.x * per + q;
+    if (j >= r) break;
+    p.cbase[int64_t(ul) * p.rmax + j] = base;
+    base += p.ccount[int64_t(ul) * p.rmax + j];
+  }
+}
+
+// stable scatter of evicted tokens into per-centre member lists
+__global__ void k_lloyd_scatter(LloydArgs p) {
+  __shared__ int a_s[kTile];
+  const int tile = blockIdx.x, ul = blockIdx.y;
+  const int r = p.r_unit[ul];
+  if (r == 0) return;
+  const int t = threadIdx.x;
+  const int64_t pos = int64_t(tile) * kTile + t;
+  const int a = pos < p.s ? p.assign[int64_t(ul) * p.s + pos] : -1;
+  a_s[t] = a;
+  __syncthreads();
+  if (a < 0) return;
+  int rank = 0;
+  for (int i = 0; i < t; ++i) rank += (a_s[i] == a);
+  const int64_t off = p.cbase[int64_t(ul) * p.rmax + a] +
+                      p.hist[(int64_t(ul) * p.ntiles + tile) * p.rmax + a] + rank;
+  p.members[int64_t(ul) * p.s + off] = int32_t(pos);
+}
+
+// new centre = mean key of its members (fp64 sums in member order); on the
+// last iteration also the mean value, and the stored bf16 entry
+__global__ void __launch_bounds__(kThreads) k_lloyd_update(LloydArgs p, int final_pass) {
+  __shared__ double redk[8][kHeadDim];
+  __shared__ double redv[8][kHeadDim];
+  __shared__ float nrm[kHeadDim];
+  const int j = blockIdx.x, ul = blockIdx.y;
+  const int r = p.r_unit[ul];
+  if (j >= r) return;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int cnt = p.ccount[int64_t(ul) * p.rmax + j];
+  const int base = p.cbase[int64_t(ul) * p.rmax + j];
+  const int per = (cnt + 7) / 8;
+  const int lo = w * per, hi = min(cnt, lo + per);
+  const int32_t* mem = p.members + int64_t(ul) * p.s + base;
+  const __nv_bfloat16* Kb = p.K + int64_t(ul) * p.s * kHeadDim + 4 * lane;
+  const __nv_bfloat16* Vb = p.V + int64_t(ul) * p.s * kHeadDim + 4 * lane;
+  double sk[4] = {0, 0, 0, 0}, sv[4] = {0, 0, 0, 0};
+  for (int i = lo; i < hi; i += 4) {
+    uint2 kw[4], vw[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (i + q < hi) {
+        const int64_t pos = mem[i + q];
+        kw[q] = __ldg(reinterpret_cast<const uint2*>(Kb + pos * kHeadDim));
+        if (final_pass) vw[q] = __ldg(reinterpret_cast<const uint2*>(Vb + pos * kHeadDim));
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (i + q < hi) {
+        const float2 a = bf16x2_to_float2(kw[q].x), b = bf16x2_to_float2(kw[q].y);
+        sk[0] += a.x; sk[1] += a.y; sk[2] += b.x; sk[3] += b.y;
+        if (final_pass) {
+          const float2 c = bf16x2_to_float2(vw[q].x), d = bf16x2_to_float2(vw[q].y);
+          sv[0] += c.x; sv[1] += c.y; sv[2] += d.x; sv[3] += d.y;
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    redk[w][4 * lane + q] = sk[q];
+    redv[w][4 * lane + q] = sv[q];
+  }
+  __syncthreads();
+  if (threadIdx.x < kHeadDim) {
+    const int d = threadIdx.x;
+    double tk = 0.0, tv = 0.0;
+    for (int ww = 0; ww < 8; ++ww) {
+      tk += redk[ww][d];
+      tv += redv[ww][d];
+    }
+    float* cptr = p.centersT + (int64_t(ul) * kHeadDim + d) * p.rmax + j;
+    double mk;
+    if (cnt > 0) {
+      mk = tk / double(cnt);
+      *cptr = float(mk);
+    } else {
+      mk = double(*cptr);              // an empty cluster keeps its centre
+    }
+    const float c = *cptr;
+    nrm[d] = c * c;
+    if (final_pass) {
+      const int64_t e = int64_t(ul) * p.ent_stride + p.ent_off + j;
+      p.kbar[e * kHeadDim + d] = __double2bfloat16(mk);
+      p.vbar[e * kHeadDim + d] = __double2bfloat16(cnt > 0 ? tv / double(cnt) : 0.0);
+      if (d == 0) p.ecount[e] = cnt;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float n = 0.f;
+    for (int i = 0; i < kHeadDim; ++i) n += nrm[i];
+    p.cnorm[int64_t(ul) * p.rmax + j] = n;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Validation proxy (Sec. 5.5.1, Eqs. valloss, valproxy; Alg. 1 steps 3-14)
+// ---------------------------------------------------------------------------
+
+constexpr int kValChunkTiles = 16;           // 2048 tokens per CTA
+constexpr int kValRec = kHeadDim + 4;        // m, l, 2 pad, acc[d]: acc 16-byte aligned
+
+struct ValArgs {
+  const __nv_bfloat16* K;
+  const __nv_bfloat16* V;
+  const __nv_bfloat16* Qobs;   // [UL*G, n_obs, d]
+  int64_t s;
+  int32_t G, n_obs, n_val, n_rows;     // n_rows = G * n_val, row = g * n_val + t
+  int32_t nchunks;
+  float* part;                 // [UL, n_rows, nchunks, kValRec]  (m, l, pad, acc)
+  float* oS;                   // [UL, n_rows, d]
+};
+
+__device__ __forceinline__ const __nv_bfloat16* val_row(const ValArgs& p, int ul, int row) {
+  const int g = row / p.n_val, t = row % p.n_val;
+  return p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + (p.n_obs - p.n_val) + t) * kHeadDim;
+}
+
+// o_S(q) over all s tokens for the validation queries (Eq. attn), per chunk
+__global__ void __launch_bounds__(kThreads, 1) k_val_full(ValArgs p) {
+  extern __shared__ __align__(16) float sm[];
+  float* Kt = sm;                               // [128][128] swizzled
+  float* Vs = Kt + kHeadDim * kTile;            // [128 tok][128 d]
+  float* Qt = Vs + kHeadDim * kTile;            // [128][32]
+  float* Pt = Qt + kHeadDim * kRowBlk;          // [128 tok][32 rows] swizzled
+  const int chunk = blockIdx.x, rb = blockIdx.y * kRowBlk, ul = blockIdx.z;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float scale = kLog2e * rsqrtf(float(kHeadDim));
+  load_qt(Qt, min(kRowBlk, p.n_rows - rb), scale, [&](int r) { return val_row(p, ul, rb + r); });
+  float m[4], l[4], acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    m[i] = -INFINITY;
+    l[i] = 0.f;
+#pragma unroll
+    for (int d = 0; d < 4; ++d) acc[i][d] = 0.f;
+  }
+  const __nv_bfloat16* Ku = p.K + int64_t(ul) * p.s * kHeadDim;
+  const __nv_bfloat16* Vu = p.V + int64_t(ul) * p.s * kHeadDim;
+  for (int tt = 0; tt < kValChunkTiles; ++tt) {
+    const int64_t tok0 = (int64_t(chunk) * kValChunkTiles + tt) * kTile;
+    if (tok0 >= p.s) break;
+    __syncthreads();
+    load_kt(Kt, Ku, p.s, tok0);
+    for (int it = 0; it < 8; ++it) {
+      const int idx = it * kThreads + threadIdx.x;
+      const int tok = idx >> 4, dc = idx & 15;
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (tok0 + tok < p.s) v = __ldg(reinterpret_cast<const uint4*>(Vu + (tok0 + tok) * kHeadDim) + dc);
+      const float2 a = bf16x2_to_float2(v.x), b = bf16x2_to_float2(v.y);
+      const float2 c = bf16x2_to_float2(v.z), d = bf16x2_to_float2(v.w);
+      *reinterpret_cast<float4*>(Vs + tok * kHeadDim + 8 * dc) = make_float4(a.x, a.y, b.x, b.y);
+      *reinterpret_cast<float4*>(Vs + tok * kHeadDim + 8 * dc + 4) = make_float4(c.x, c.y, d.x, d.y);
+    }
+    __syncthreads();
+    float S[4][4];
+    tile_logits(Qt, Kt, S);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float tmax = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (tok0 + 4 * lane + j >= p.s) S[i][j] = -INFINITY;
+        tmax = fmaxf(tmax, S[i][j]);
+      }
+      tmax = warp_max(tmax);
+      const float mn = fmaxf(m[i], tmax);
+      const float sc = exp2f(m[i] - mn);
+      l[i] *= sc;
+#pragma unroll
+      for (int d = 0; d < 4; ++d) acc[i][d] *= sc;
+      m[i] = mn;
+      float ps = 0.f;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        S[i][j] = exp2f(S[i][j] - mn);
+        ps += S[i][j];
+      }
+      l[i] += warp_sum(ps);
+    }
+    // P^T into shared memory: Pt[tok][rows], float4 column swizzled by (tok / 4)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int tok = 4 * lane + j;
+      *reinterpret_cast<float4*>(Pt + tok * kRowBlk + ((w ^ (lane & 7)) << 2)) =
+          make_float4(S[0][j], S[1][j], S[2][j], S[3][j]);
+    }
+    __syncthreads();
+#pragma unroll 4
+    for (int tok = 0; tok < kTile; ++tok) {
+      const float4 pp = *reinterpret_cast<const float4*>(Pt + tok * kRowBlk + ((w ^ ((tok >> 2) & 7)) << 2));
+      const float4 vv = *reinterpret_cast<const float4*>(Vs + tok * kHeadDim + 4 * lane);
+      const float pa[4] = {pp.x, pp.y, pp.z, pp.w};
+      const float va[4] = {vv.x, vv.y, vv.z, vv.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int d = 0; d < 4; ++d) acc[i][d] = fmaf(pa[i], va[d], acc[i][d]);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int row = rb + 4 * w + i;
+    if (row >= p.n_rows) continue;
+    float* out = p.part + ((int64_t(ul) * p.n_rows + row) * p.nchunks + chunk) * kValRec;
+    if (lane == 0) {
+      out[0] = m[i];
+      out[1] = l[i];
+    }
+    *reinterpret_cast<float4*>(out + 4 + 4 * lane) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+  }
+}
+
+__global__ void k_val_combine(ValArgs p) {
+  const int row = blockIdx.x, ul = blockIdx.y, d = threadIdx.x;
+  const float* base = p.part + (int64_t(ul) * p.n_rows + row) * p.nchunks * kValRec;
+  float m = -INFINITY, l = 0.f, a = 0.f;
+  for (int c = 0; c < p.nchunks; ++c) {
+    const float* q = base + int64_t(c) * kValRec;
+    const float cm = q[0], cl = q[1];
+    if (cl <= 0.f) continue;
+    const float mn = fmaxf(m, cm);
+    const float s0 = exp2f(m - mn), s1 = exp2f(cm - mn);
+    l = l * s0 + cl * s1;
+    a = a * s0 + q[4 + d] * s1;
+    m = mn;
+  }
+  p.oS[(int64_t(ul) * p.n_rows + row) * kHeadDim + d] = a / l;
+}
+
+struct LossArgs {
+  const __nv_bfloat16* K;
+  const __nv_bfloat16* V;
+  const __nv_bfloat16* Qobs;
+  int64_t s;
+  int32_t G, n_obs, n_val, n_rows;
+  int32_t recent, n_top, budget;
+  const int32_t* top;          // [UL, n_top]
+  const int32_t* r_unit;       // [UL]
+  const __nv_bfloat16* kbar;   // [UL, ent_stride, d]
+  const __nv_bfloat16* vbar;
+  const int32_t* ecount;
+  int64_t ent_stride;
+  int32_t ent_off;
+  float beta;
+  int32_t gate_mode;
+  float tau, alpha, g_min, g_fixed;
+  const float* oS;             // [UL, n_rows, d]
+  double* rowerr;              // [UL, n_rows]
+};
+
+// ||o^(r)(q) - o_S(q)||^2 per validation query, with the decode rule of
+// Sec. 5.4 and the gate (one warp per query, 4 dims per lane)
+__global__ void __launch_bounds__(kThreads) k_val_loss(LossArgs p) {
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = blockIdx.x * 8 + w, ul = blockIdx.y;
+  if (row >= p.n_rows) return;
+  const int r = p.r_unit[ul];
+  const int64_t m = r == 0 ? (p.budget < p.s ? p.budget : p.s) : p.budget - r;
+  const int64_t keep = m - p.recent;
+  const int g = row / p.n_val, t = row % p.n_val;
+  const __nv_bfloat16* qp = p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + (p.n_obs - p.n_val) + t) * kHeadDim;
+  const float scale = kLog2e * rsqrtf(float(kHeadDim));
+  const uint2 qw = __ldg(reinterpret_cast<const uint2*>(qp + 4 * lane));
+  const float2 q01 = bf16x2_to_float2(qw.x), q23 = bf16x2_to_float2(qw.y);
+  const float q[4] = {q01.x * scale, q01.y * scale, q23.x * scale, q23.y * scale};
+  const __nv_bfloat16* Ku = p.K + int64_t(ul) * p.s * kHeadDim + 4 * lane;
+  const __nv_bfloat16* Vu = p.V + int64_t(ul) * p.s * kHeadDim + 4 * lane;
+  const int32_t* top = p.top + int64_t(ul) * p.n_top;
+  // main cache
+  float mM = -INFINITY, lM = 0.f, aM[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int64_t j0 = 0; j0 < m; j0 += 4) {
+    uint2 kw[4], vw[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t j = j0 + u;
+      if (j < m) {
+        const int64_t pos = j < keep ? top[j] : (p.s - p.recent) + (j - keep);
+        kw[u] = __ldg(reinterpret_cast<const uint2*>(Ku + pos * kHeadDim));
+        vw[u] = __ldg(reinterpret_cast<const uint2*>(Vu + pos * kHeadDim));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (j0 + u >= m) break;
+      const float2 k01 = bf16x2_to_float2(kw[u].x), k23 = bf16x2_to_float2(kw[u].y);
+      const float a = warp_sum(q[0] * k01.x + q[1] * k01.y + q[2] * k23.x + q[3] * k23.y);
+      const float mn = fmaxf(mM, a);
+      const float sc = exp2f(mM - mn), pr = exp2f(a - mn);
+      const float2 v01 = bf16x2_to_float2(vw[u].x), v23 = bf16x2_to_float2(vw[u].y);
+      lM = lM * sc + pr;
+      aM[0] = aM[0] * sc + pr * v01.x;
+      aM[1] = aM[1] * sc + pr * v01.y;
+      aM[2] = aM[2] * sc + pr * v23.x;
+      aM[3] = aM[3] * sc + pr * v23.y;
+      mM = mn;
+    }
+  }
+  // residual entries: logit + beta*log c (log2 units); gate applied below
+  float mR = -INFINITY, lR = 0.f, aR[4] = {0.f, 0.f, 0.f, 0.f};
+  const int64_t e0 = int64_t(ul) * p.ent_stride + p.ent_off;
+  for (int j = 0; j < r; ++j) {
+    const int c = p.ecount[e0 + j];
+    if (c <= 0) continue;
+    const uint2 kw = *reinterpret_cast<const uint2*>(p.kbar + (e0 + j) * kHeadDim + 4 * lane);
+    const uint2 vw = *reinterpret_cast<const uint2*>(p.vbar + (e0 + j) * kHeadDim + 4 * lane);
+    const float2 k01 = bf16x2_to_float2(kw.x), k23 = bf16x2_to_float2(kw.y);
+    const float a = warp_sum(q[0] * k01.x + q[1] * k01.y + q[2] * k23.x + q[3] * k23.y) +
+                    p.beta * logf(float(c)) * kLog2e;
+    const float mn = fmaxf(mR, a);
+    const float sc = exp2f(mR - mn), pr = exp2f(a - mn);
+    const float2 v01 = bf16x2_to_float2(vw.x), v23 = bf16x2_to_float2(vw.y);
+    lR = lR * sc + pr;
+    aR[0] = aR[0] * sc + pr * v01.x;
+    aR[1] = aR[1] * sc + pr * v01.y;
+    aR[2] = aR[2] * sc + pr * v23.x;
+    aR[3] = aR[3] * sc + pr * v23.y;
+    mR = mn;
+  }
+  float g_val = p.g_fixed;
+  if (p.gate_mode == RESKV_GATE_DYNAMIC) {
+    const float pmax = 1.0f / lM;
+    g_val = fmaxf(p.g_min, 1.0f / (1.0f + expf(-p.alpha * (p.tau - pmax))));
+  }
+  float wM = 1.f, wR = 0.f;
+  if (lR > 0.f && g_val > 0.f) {
+    const float mx = fmaxf(mM, mR);
+    wM = exp2f(mM - mx);
+    wR = g_val * exp2f(mR - mx);
+  }
+  const float inv = 1.0f / (wM * lM + wR * lR);
+  const float* os = p.oS + (int64_t(ul) * p.n_rows + row) * kHeadDim + 4 * lane;
+  float e = 0.f;
+#pragma unroll
+  for (int d = 0; d < 4; ++d) {
+    const float o = (wM * aM[d] + wR * aR[d]) * inv;
+    const float df = o - os[d];
+    e += df * df;
+  }
+  e = warp_sum(e);
+  if (lane == 0) p.rowerr[int64_t(ul) * p.n_rows + row] = double(e);
+}
+
+// L_r = mean of the per-query errors (rows in order, fp64)
+__global__ void k_loss_reduce(const double* rowerr, double* losses, int n_rows, int UL, int ncol,
+                              int col) {
+  const int ul = blockIdx.x * blockDim.x + threadIdx.x;
+  if (ul >= UL) return;
+  double acc = 0.0;
+  for (int i = 0; i < n_rows; ++i) acc += rowerr[int64_t(ul) * n_rows + i];
+  losses[int64_t(ul) * ncol + col] = acc / double(n_rows);
+}
+
+// r* = argmin_{r>0} L_r (ties -> smaller r); keep it only if L_r* < (1 - delta) L_0
+__global__ void k_choose(const double* losses, int ncol, const int32_t* cand_r, int UL,
+                         double one_minus_delta, int32_t* r_final, int32_t* chosen) {
+  const int ul = blockIdx.x * blockDim.x + threadIdx.x;
+  if (ul >= UL) return;
+  const double* L = losses + int64_t(ul) * ncol;
+  int best = 0;
+  for (int c = 1; c < ncol; ++c)
+    if (best == 0 || L[c] < L[best]) best = c;
+  const bool use = best > 0 && L[best] < one_minus_delta * L[0];
+  r_final[ul] = use ? cand_r[best] : 0;
+  chosen[ul] = use ? best : 0;
+}
+
+// ---------------------------------------------------------------------------
+// Packing into the ragged layout (Alg. 1 step 15): main rows in position
+// order, then the chosen run's residual entries.
+// ---------------------------------------------------------------------------
+
+struct PackArgs {
+  const __nv_bfloat16* K;
+  const __nv_bfloat16* V;
+  int64_t s;
+  int32_t recent, budget;
+  const int32_t* rank_pos;     // [UL, s]
+  const int32_t* r_final;      // [UL]
+  const int32_t* chosen;       // [UL] run index of the chosen entries (0 = none)
+  const int32_t* run_off;      // [n_runs] entry offset of each run
+  const __nv_bfloat16* kbar;
+  const __nv_bfloat16* vbar;
+  const int32_t* ecount;
+  int64_t ent_stride;
+  float beta;
+  int64_t unit0;               // global unit index of ul = 0
+  __nv_bfloat16* kslots;
+  __nv_bfloat16* vslots;
+  float* logc;
+  int32_t* slot_pos;
+  int32_t* counts;
+  int32_t* n_main;
+  int32_t* n_res;
+};
+
+__global__ void __launch_bounds__(1024) k_pack(PackArgs p) {
+  __shared__ int warp_sums[32];
+  const int ul = blockIdx.x;
+  const int64_t u = p.unit0 + ul;
+  const int r = p.r_final[ul];
+  const int64_t m = r == 0 ? (p.budget < p.s ? p.budget : p.s) : p.budget - r;
+  const int64_t keep = m - p.recent;
+  const int32_t* rp = p.rank_pos + int64_t(ul) * p.s;
+  int32_t* spos = p.slot_pos + u * p.budget;
+  const int64_t chunk = (p.s + blockDim.x - 1) / blockDim.x;
+  const int64_t lo = int64_t(threadIdx.x) * chunk, hi = lo + chunk < p.s ? lo + chunk : p.s;
+  int mine = 0;
+  for (int64_t i = lo; i < hi; ++i) {
+    const int32_t rk = rp[i];
+    mine += (rk < 0 || rk < keep);
+  }
+  int out = block_exclusive_scan(mine, warp_sums, nullptr);
+  for (int64_t i = lo; i < hi; ++i) {
+    const int32_t rk = rp[i];
+    if (rk < 0 || rk < keep) {
+      if (out < m) spos[out] = int32_t(i);
+      ++out;
+    }
+  }
+  __syncthreads();
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  const __nv_bfloat16* Ku = p.K + int64_t(ul) * p.s * kHeadDim;
+  const __nv_bfloat16* Vu = p.V + int64_t(ul) * p.s * kHeadDim;
+  for (int64_t j = w; j < m; j += nw) {
+    const int64_t pos = spos[j];
+    const uint2 kw = __ldg(reinterpret_cast<const uint2*>(Ku + pos * kHeadDim) + lane);
+    const uint2 vw = __ldg(reinterpret_cast<const uint2*>(Vu + pos * kHeadDim) + lane);
+    reinterpret_cast<uint2*>(p.kslots + (u * p.budget + j) * kHeadDim)[lane] = kw;
+    reinterpret_cast<uint2*>(p.vslots + (u * p.budget + j) * kHeadDim)[lane] = vw;
+    if (lane == 0) {
+      p.counts[u * p.budget + j] = 0;
+      p.logc[u * p.budget + j] = 0.f;
+    }
+  }
+  const int c = p.chosen[ul];
+  for (int j = w; j < r; j += nw) {
+    const int64_t e = int64_t(ul) * p.ent_stride + p.run_off[c] + j;
+    const int64_t slot = u * p.budget + m + j;
+    reinterpret_cast<uint2*>(p.kslots + slot * kHeadDim)[lane] =
+        reinterpret_cast<const uint2*>(p.kbar + e * kHeadDim)[lane];
+    reinterpret_cast<uint2*>(p.vslots + slot * kHeadDim)[lane] =
+        reinterpret_cast<const uint2*>(p.vbar + e * kHeadDim)[lane];
+    if (lane == 0) {
+      const int cnt = p.ecount[e];
+      p.counts[slot] = cnt;
+      p.logc[slot] = cnt > 0 ? p.beta * logf(float(cnt)) : -INFINITY;
+      spos[m + j] = -1;
+    }
+  }
+  if (threadIdx.x == 0) {
+    p.n_main[u] = int32_t(m);
+    p.n_res[u] = r;
+  }
+}
+
 }  // namespace build
 }  // namespace reskv

@@ -1,0 +1,237 @@
+"""GPU construction (Alg. 1) through the C ABI against the fp64 oracle.
+
+Stage-wise protocol (float32 on the GPU, float64 in the oracle):
+  scores     relative error <= 1e-4;
+  ranking    bit-exact when the oracle ranks the GPU's own scores; against the
+             oracle's fp64 scores, two positions may only trade places if their
+             fp64 scores differ by < 1e-5 relative (a near tie);
+  key-norm   scores and selection bit-exact (both sides sum the same bf16 squares
+             in fp64 in the same order);
+  entries    given the GPU's evicted set in the GPU's rank order, the oracle's
+             Lloyd gives the same counts and the same bf16 entries (up to one
+             bf16 ulp where the fp32 centres left a near tie);
+  r choice   equal unless the oracle's deciding margin is < 1e-3 relative;
+  decode     of the GPU-built cache within max abs 1e-2, rel L2 2e-3 of the
+             oracle's decode of the oracle-built cache.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as orc
+from paper_2607_29591_gb300 import build as B
+from paper_2607_29591_gb300 import reskv as R
+from paper_2607_29591_gb300 import workloads as wl
+
+from helpers import assert_north_star, bf16_to_f64, errors, unit_from_layout
+
+pytestmark = pytest.mark.gpu
+
+NEAR_TIE = 1e-5
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    B.build()
+    return R.load_library()
+
+
+def make_inputs(w):
+    """Inputs drawn on the CPU (the oracle's copies) and uploaded for the library."""
+    Ks, Vs, Qs = [], [], []
+    for l in range(w.n_layers):
+        K, V, Qo, _ = wl.layer_inputs(w, l, "cpu")
+        Ks.append(K)
+        Vs.append(V)
+        Qs.append(Qo)
+    up = lambda ts: [None if t is None else t.cuda() for t in ts]
+    return (Ks, Vs, Qs), (up(Ks), up(Vs), up(Qs))
+
+
+def lib_config(w, **kw):
+    ovr = w.residual_override()
+    return R.reskv_config_default(batch=w.batch, n_layers=w.n_layers, n_kv_heads=w.n_kv_heads,
+                                  group=w.group, seq_len=w.seq_len, budget=w.budget,
+                                  recent_window=w.recent_window, n_obs=w.n_obs, n_fit=w.n_fit,
+                                  n_val=w.n_val, score_mode=w.score_mode,
+                                  residual_override=ovr, keep_debug=1, **kw)
+
+
+def oracle_config(w, cfg):
+    ovr = w.residual_override()
+    return lambda u: orc.OracleConfig(
+        budget=w.budget, recent_window=w.recent_window, n_fit=w.n_fit, n_val=w.n_val,
+        score_mode=w.score_mode, residual_override=None if ovr is None else int(ovr[u]),
+        delta=float(np.float32(cfg.delta)), gate_mode=cfg.gate_mode, tau=cfg.tau,
+        alpha=cfg.alpha, g_min=cfg.g_min, g_fixed=cfg.g_fixed)
+
+
+def unit_inputs(Ks, Vs, Qs, w, u):
+    l, rem = divmod(u, w.batch * w.n_kv_heads)
+    b, h = divmod(rem, w.n_kv_heads)
+    K = bf16_to_f64(Ks[l][b, h])
+    V = bf16_to_f64(Vs[l][b, h])
+    Q = None if Qs[l] is None else bf16_to_f64(Qs[l][b, h * w.group:(h + 1) * w.group])
+    return K, V, Q
+
+
+def check_ranking(gpu_scores, gpu_top, ref_scores, recent, keynorm):
+    """Ranking protocol for one unit; returns the number of near-tie swaps."""
+    n_top = len(gpu_top)
+    own = orc.rank_evictable(gpu_scores, recent)[:n_top]
+    assert np.array_equal(own, gpu_top), "GPU ranking differs from ranking its own scores"
+    ref = orc.rank_evictable(ref_scores, recent)[:n_top]
+    if keynorm:
+        assert np.array_equal(gpu_scores, ref_scores)
+        assert np.array_equal(ref, gpu_top)
+        return 0
+    np.testing.assert_allclose(gpu_scores, ref_scores, rtol=1e-4, atol=0)
+    swaps = 0
+    for i in np.nonzero(ref != gpu_top)[0]:
+        a, b = ref_scores[ref[i]], ref_scores[gpu_top[i]]
+        assert abs(a - b) <= NEAR_TIE * max(abs(a), abs(b)), f"rank {i}: not a near tie"
+        swaps += 1
+    return swaps
+
+
+def check_entries(gpu_unit, K, V, gpu_top, recent, s, b, iters):
+    """Oracle Lloyd on the GPU's evicted set (GPU rank order) vs GPU entries."""
+    r = gpu_unit.r
+    if r == 0:
+        return
+    m = b - r
+    keep = m - recent
+    main = set(gpu_unit.main_pos.tolist())
+    assert len(main) == m
+    rest = [p for p in range(s - recent) if p not in set(gpu_top[:keep].tolist())]
+    in_top = set(gpu_top.tolist())
+    E = np.array(list(gpu_top[keep:]) + [p for p in rest if p not in in_top])
+    assert not (set(E.tolist()) & main) and len(E) == s - m
+    kbar, vbar, counts = orc.lloyd_residual(K, V, E, r, iters)
+    kb, vb = orc.round_to_bf16(kbar), orc.round_to_bf16(vbar)
+    diff_c = np.nonzero(counts != gpu_unit.counts)[0]
+    assert len(diff_c) <= max(1, r // 50), f"{len(diff_c)} of {r} entry counts differ"
+    same = np.setdiff1d(np.arange(r), diff_c)
+    ulp = np.abs(kb[same]) * 2.0 ** -7 + 1e-30
+    assert np.all(np.abs(kb[same] - gpu_unit.kbar[same]) <= ulp)
+    ulpv = np.abs(vb[same]) * 2.0 ** -7 + 1e-30
+    assert np.all(np.abs(vb[same] - gpu_unit.vbar[same]) <= ulpv)
+    exact = np.mean(np.all(kb[same] == gpu_unit.kbar[same], axis=1))
+    assert exact > 0.9, f"only {exact:.2f} of the entries are bit-identical"
+
+
+def decode_parity(cache, lay, ref_units, Ks, Qd, w, ocfg_of):
+    """GPU decode of the GPU-built cache vs oracle decode of the oracle cache."""
+    L, Bt, H, G = w.n_layers, w.batch, w.n_kv_heads, w.group
+    O = torch.empty(Qd.shape, dtype=torch.float32, device="cuda")
+    R.reskv_decode_attn(cache, -1, Qd, O)
+    torch.cuda.synchronize()
+    O = O.cpu().numpy()
+    qf = bf16_to_f64(Qd)
+    worst = 0.0
+    for u, ref in ref_units.items():
+        l, rem = divmod(u, Bt * H)
+        b, h = divmod(rem, H)
+        q = qf[l, b, h * G:(h + 1) * G]
+        ref_o = orc.decode_unit(ref, q, ocfg_of(u))
+        mx, rel = assert_north_star(O[l, b, h * G:(h + 1) * G], ref_o, f"unit {u}")
+        # the kernel alone: oracle decode of the GPU's own cache
+        own = orc.decode_unit(unit_from_layout(lay, u), q, ocfg_of(u))
+        assert errors(O[l, b, h * G:(h + 1) * G], own)[1] < 1e-4
+        worst = max(worst, rel)
+    return worst
+
+
+def decode_queries(w, Ks):
+    Q = torch.empty((w.n_layers, w.batch, w.n_q_heads, w.head_dim), dtype=torch.bfloat16)
+    for l in range(w.n_layers):
+        for b in range(w.batch):
+            for h in range(w.n_kv_heads):
+                k = Ks[l][b, h]
+                Q[l, b, h * w.group:(h + 1) * w.group] = \
+                    wl.unit_decode_queries(w, l, b, h, k, 1)[:, 0]
+    return Q.cuda()
+
+
+def run_case(w, units=None, **cfg_kw):
+    (Ks, Vs, Qs), (Kd, Vd, Qdv) = make_inputs(w)
+    cfg = lib_config(w, **cfg_kw)
+    Qarg = Qdv if w.n_obs > 0 else None
+    cache = R.reskv_build_cache(cfg, Kd, Vd, Qarg)
+    R.reskv_check_status(cache)
+    lay = R.reskv_export_cache(cache)
+    scores = R.reskv_export_debug(cache, R.RESKV_DEBUG_SCORES)
+    top = R.reskv_export_debug(cache, R.RESKV_DEBUG_RANKED)
+    proxy = w.residual == "proxy" and w.budget < w.seq_len
+    P = min(w.recent_window, w.seq_len)
+    expect = [r for r in orc.candidate_budgets(w.budget, orc.OracleConfig(budget=1).grid_ratios)
+              if w.budget - r >= P] if proxy else []
+    cands = R.reskv_export_debug(cache, R.RESKV_DEBUG_CANDIDATES, n_cand=len(expect))
+    assert cands.tolist() == expect
+    ocfg_of = oracle_config(w, cfg)
+    units = range(w.n_units) if units is None else units
+    ref_units, swaps, margins = {}, 0, []
+    for u in units:
+        K, V, Q = unit_inputs(Ks, Vs, Qs, w, u)
+        oc = ocfg_of(u)
+        ref = orc.build_unit(K, V, Q, oc)
+        ref_units[u] = ref
+        swaps += check_ranking(scores[u], top[u], ref.scores, P, w.score_mode == 1)
+        gu = unit_from_layout(lay, u)
+        if proxy:
+            L = ref.losses
+            rs = sorted(k for k in L if k > 0)
+            best = min(rs, key=lambda r: (L[r], r))
+            margin = abs(L[best] / L[0] - (1 - oc.delta)) if L[0] > 0 else 1.0
+            second = sorted(L[r] for r in rs)
+            gap = (second[1] - second[0]) / second[0] if len(second) > 1 else 1.0
+            margins.append(min(margin, gap))
+            if min(margin, gap) > 1e-3:
+                assert gu.r == ref.r, f"unit {u}: r {gu.r} vs oracle {ref.r}"
+            gl = R.reskv_export_debug(cache, R.RESKV_DEBUG_LOSSES, n_cand=len(cands))[u]
+            np.testing.assert_allclose(gl, [L[0]] + [L[r] for r in cands], rtol=2e-3)
+        else:
+            assert gu.r == ref.r
+        if gu.r == ref.r and set(gu.main_pos.tolist()) != set(ref.main_pos.tolist()):
+            # only near-tie swaps may move a token across the boundary
+            assert swaps > 0
+        check_entries(gu, K, V, top[u], P, w.seq_len, w.budget, 4)
+    worst = decode_parity(cache, lay, ref_units, Ks, decode_queries(w, Ks), w, ocfg_of)
+    cache.free()
+    return dict(swaps=swaps, worst_rel=worst, margins=margins)
+
+
+def test_tiny_fixed_residual():
+    """Tiny workload: s = 4096, b = 256 with r = 32 fixed, SnapKV scores."""
+    out = run_case(wl.WORKLOADS["tiny"])
+    assert out["worst_rel"] < 2e-3
+
+
+def test_proxy_two_heads():
+    """Validation proxy (Sec. 5.5.1) on 2 batch x 2 KV heads, s = 2048, b = 256."""
+    w = wl.scaled(wl.WORKLOADS["llama8b_layer_32k"], seq_len=2048, budget=256, batch=2,
+                  n_kv_heads=2)
+    run_case(w)
+
+
+def test_proxy_short_window_drift_needles():
+    """32-token observation window (24 fit / 8 val) on drifting keys with needles."""
+    w = wl.scaled(wl.WORKLOADS["long_128k_b4"], seq_len=4096, budget=512, batch=1, n_layers=2,
+                  n_kv_heads=2, n_obs=32, n_fit=24, n_val=8)
+    run_case(w)
+
+
+def test_keynorm_drawn_residual():
+    """Query-free scores, per-(layer, head) drawn r (some 0), s = 2048, b = 128."""
+    w = wl.scaled(wl.WORKLOADS["small_budget_b64"], seq_len=2048, batch=3, n_layers=2,
+                  n_kv_heads=3)
+    run_case(w)
+
+
+def test_budget_covering_every_token():
+    """b >= s: M = S, r = 0, decode = full attention (Eq. attn)."""
+    w = wl.scaled(wl.WORKLOADS["llama8b_layer_32k"], seq_len=600, budget=640, batch=1,
+                  n_kv_heads=2)
+    out = run_case(w)
+    assert out["swaps"] == 0
