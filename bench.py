@@ -1,0 +1,449 @@
+"""Decode benchmark of the ResKV library on synthetic long-context workloads.
+
+One step = one shared-softmax decode (Alg. 2) of every (layer, batch, KV head)
+unit of the workload for one fresh decode query per query head, through the
+C ABI (reskv_decode_attn with layer = -1: one launch covers all layers).  The
+compressed cache is built first by reskv_build_cache (Alg. 1, timed on its
+own).  Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   (the fp64 CPU oracle on host cores)
+
+Under torchrun (N > 1) every rank runs an independent replica on its own GPU
+(the path has no exchange step); rank 0 prints the aggregate.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2607_29591_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "compressed-decode attn tokens/s and achieved HBM GB/s (% of peak), 1 GB300"
+DEFAULT_WORKLOAD = "llama8b_32l_32k_b8"
+SLOT_BYTES = 2 * 128 * 2            # one K row + one V row, bf16
+PROFILE = os.path.join(ROOT, "profiles", "decode_kernel_llama8b_32l_32k_b8.md")
+KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_29591_gb300", "csrc", f)
+                  for f in ("decode_kernel.cu", "device_utils.cuh")]
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["reskv", "reference"], default="reskv")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(wl.WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-per-layer", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="use only this many layers (smaller profiling case)")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (replicas only)
+# ---------------------------------------------------------------------------
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def reduce_max(x: float, world: int, device) -> float:
+    """Max over ranks of a per-rank time (the job's time is the slowest rank)."""
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate(per_rank_units: float, max_seconds: float, world: int) -> float:
+    """Whole-job throughput: units of every rank over the slowest rank's time."""
+    return per_rank_units * world / max_seconds
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.3)
+        except FileNotFoundError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = float(parts[1])
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# roofline bookkeeping
+# ---------------------------------------------------------------------------
+
+def measured_peak_gbs():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def kernel_hash():
+    h = hashlib.sha256()
+    for p in KERNEL_SOURCES:
+        with open(p, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(units_per_launch: int):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel
+    source has not changed since it was captured (else None)."""
+    if not os.path.exists(PROFILE):
+        return None
+    text = open(PROFILE).read()
+    m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", text)
+    m_bpu = re.search(r"dram_bytes_per_unit:\s*([0-9.]+)", text)
+    if not m_hash or not m_bpu or m_hash.group(1) != kernel_hash():
+        return None
+    return int(float(m_bpu.group(1)) * units_per_launch)
+
+
+def algorithmic_bytes(n_main: np.ndarray, n_res: np.ndarray) -> int:
+    """Bytes the method must read per decode step: every main and residual
+    K/V row (512 B) plus the residual log-counts (4 B)."""
+    return int((n_main.astype(np.int64) + n_res).sum()) * SLOT_BYTES + int(n_res.sum()) * 4
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the fp64 oracle on host cores
+# ---------------------------------------------------------------------------
+
+def oracle_sample_units(w: wl.Workload, n_units: int, seed_step: int = 0):
+    """Units shaped like the workload's compressed cache, for timing the
+    oracle: rows from the seeded generator, r from the candidate grid."""
+    import oracle as orc
+    rng = np.random.default_rng(42)
+    grid = [0] + orc.candidate_budgets(w.budget, (0.05, 0.10, 0.15, 0.20))
+    units = []
+    sample = rng.choice(w.n_units, size=min(n_units, w.n_units), replace=False)
+    ws = wl.scaled(w, seq_len=max(w.budget, 64))
+    hidx = wl.counter_hash(2 * ws.seq_len * ws.head_dim, "cpu")
+    for u in sample:
+        l, rem = divmod(int(u), w.batch * w.n_kv_heads)
+        b, h = divmod(rem, w.n_kv_heads)
+        K, V = wl.unit_kv(ws, l, b, h, "cpu", hidx)
+        r = int(rng.choice(grid)) if w.residual != "drawn" else int(w.residual_override()[u])
+        m = w.budget - r
+        Kf, Vf = K.double().numpy(), V.double().numpy()
+        cnt = rng.integers(1, 300, r)
+        units.append((orc.UnitCache(main_pos=np.arange(m), kmain=Kf[:m], vmain=Vf[:m],
+                                    kbar=Kf[m:m + r], vbar=Vf[m:m + r], counts=cnt,
+                                    logc=np.log(cnt.astype(np.float64)), r=r),
+                      wl.unit_decode_queries(ws, l, b, h, K, 1)[:, 0].double().numpy()))
+    return units
+
+
+def time_oracle(units, cores: int, reps: int = 1):
+    import concurrent.futures
+    import oracle as orc
+    cfg = orc.OracleConfig(budget=1)
+    t0 = time.perf_counter()
+    with concurrent.futures.ThreadPoolExecutor(cores) as ex:
+        for _ in range(reps):
+            list(ex.map(lambda uq: orc.decode_unit(uq[0], uq[1], cfg), units))
+    return (time.perf_counter() - t0) / reps
+
+
+def cpu_baseline(w: wl.Workload, target_s: float = 15.0):
+    cores = os.cpu_count() or 1
+    units = oracle_sample_units(w, 256)
+    per = time_oracle(units, cores)
+    reps = max(1, int(target_s / max(per, 1e-3)))
+    per = time_oracle(units, cores, reps)
+    step_s = per * w.n_units / len(units)
+    return {"value": w.batch / step_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"fp64 oracle decode of {len(units)} seeded units x {reps} repetitions "
+                      f"(G={w.group} heads each, b={w.budget}), extrapolated to all "
+                      f"{w.n_units} units of one step"}
+
+
+def run_reference(args, world, rank):
+    """The reference arm: the fp64 oracle, as it stands, on the host cores."""
+    if rank != 0:
+        return
+    w = wl.WORKLOADS[args.workload]
+    cores = os.cpu_count() or 1
+    units = oracle_sample_units(w, 16)
+    for _ in range(args.warmup):
+        time_oracle(units, cores)
+    t = 0.0
+    for _ in range(args.steps):
+        t += time_oracle(units, cores)
+    step_s = (t / args.steps) * w.n_units / len(units)
+    value = w.batch / step_s
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"each step: fp64 oracle decode of {len(units)} seeded "
+                                       f"units, extrapolated to {w.n_units} units"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+
+def build_workload(w: wl.Workload, n_q: int, device):
+    """Generate inputs layer by layer; build the compressed cache (timed)."""
+    from paper_2607_29591_gb300 import reskv as R
+    Ks, Vs, Qs = [], [], []
+    Qdec = torch.empty((n_q, w.n_layers, w.batch, w.n_q_heads, w.head_dim),
+                       dtype=torch.bfloat16, device=device)
+    for l in range(w.n_layers):
+        K, V, Qo, Qd = wl.layer_inputs(w, l, device, n_dec_steps=n_q)
+        Ks.append(K)
+        Vs.append(V)
+        Qs.append(Qo)
+        Qdec[:, l] = Qd
+    cfg = R.reskv_config_default(batch=w.batch, n_layers=w.n_layers, n_kv_heads=w.n_kv_heads,
+                                 group=w.group, seq_len=w.seq_len, budget=w.budget,
+                                 recent_window=w.recent_window, n_obs=w.n_obs, n_fit=w.n_fit,
+                                 n_val=w.n_val, score_mode=w.score_mode,
+                                 residual_override=w.residual_override())
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    cache = R.reskv_build_cache(cfg, Ks, Vs, Qs if w.n_obs > 0 else None)
+    e1.record()
+    torch.cuda.synchronize()
+    build_s = e0.elapsed_time(e1) / 1e3
+    R.reskv_check_status(cache)
+    del Ks, Vs, Qs
+    torch.cuda.empty_cache()
+    return cache, Qdec, build_s
+
+
+def main():
+    args = parse_args()
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+        return
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+    from paper_2607_29591_gb300 import build as B
+    from paper_2607_29591_gb300 import reskv as R
+    B.build()
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    w = wl.WORKLOADS[args.workload]
+    if args.layers:
+        w = wl.scaled(w, n_layers=args.layers, name=f"{w.name}_{args.layers}l")
+    n_q = args.steps + args.warmup
+    cache, Qdec, build_s = build_workload(w, n_q, device)
+    lay_meta = R.reskv_export_cache(cache)
+    alg = algorithmic_bytes(lay_meta["n_main"], lay_meta["n_res"])
+    r_counts = lay_meta["n_res"]
+    del lay_meta
+    O = torch.empty((w.n_layers, w.batch, w.n_q_heads, w.head_dim), dtype=torch.float32,
+                    device=device)
+    stream = torch.cuda.current_stream(device)
+
+    # ---- device-resident timing: K steps, one launch each ----
+    for i in range(args.warmup):
+        R.reskv_decode_attn(cache, -1, Qdec[i], O)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        barrier(world)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for i in range(args.steps):
+            R.reskv_decode_attn(cache, -1, Qdec[args.warmup + i], O)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+    t_local = e0.elapsed_time(e1) / 1e3
+    t = reduce_max(t_local, world, device)
+    R.reskv_check_status(cache)
+    ms_step = t * 1e3 / args.steps
+    value = aggregate(w.batch * args.steps, t, world)
+    launch_s = t_local / args.steps                      # one launch per step
+    peak, peak_kind = measured_peak_gbs()
+    achieved = alg / launch_s / 1e9
+
+    # ---- per-layer calls (one launch per layer) captured in a CUDA graph ----
+    per_layer = None
+    if not args.no_per_layer:
+        Ql = [Qdec[0, l].contiguous() for l in range(w.n_layers)]
+        Ol = [O[l] for l in range(w.n_layers)]
+        g_stream = torch.cuda.Stream(device)
+        g_stream.wait_stream(stream)
+        with torch.cuda.stream(g_stream):
+            for l in range(w.n_layers):                      # warm, outside capture
+                R.reskv_decode_attn(cache, l, Ql[l], Ol[l], stream=g_stream)
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=g_stream):
+                for l in range(w.n_layers):
+                    R.reskv_decode_attn(cache, l, Ql[l], Ol[l], stream=g_stream)
+        stream.wait_stream(g_stream)
+        for _ in range(args.warmup):
+            graph.replay()
+        torch.cuda.synchronize()
+        reps = max(10, args.steps // 4)
+        e0.record(stream)
+        for _ in range(reps):
+            graph.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        tg = e0.elapsed_time(e1) / 1e3 / reps
+        per_layer = {"us_per_step": tg * 1e6, "us_per_layer_step": tg * 1e6 / w.n_layers,
+                     "tokens_per_s": w.batch / tg, "gbs": alg / tg / 1e9,
+                     "frac_of_peak": alg / tg / 1e9 / peak,
+                     "how": f"{w.n_layers} per-layer reskv_decode_attn launches replayed as one "
+                            f"CUDA graph, {reps} replays"}
+        del graph
+
+    # ---- end to end through the C ABI with host buffers ----
+    Qh = Qdec[:min(n_q, 64)].cpu().pin_memory()
+    Oh = torch.empty(O.shape, dtype=torch.float32).pin_memory()
+    Qd_buf = torch.empty_like(Qdec[0])
+    e2e_steps = min(args.steps, 64)
+    for i in range(3):
+        Qd_buf.copy_(Qh[i % Qh.shape[0]], non_blocking=True)
+        R.reskv_decode_attn(cache, -1, Qd_buf, O)
+        Oh.copy_(O, non_blocking=True)
+    torch.cuda.synchronize()
+    barrier(world)
+    t0 = time.perf_counter()
+    for i in range(e2e_steps):
+        Qd_buf.copy_(Qh[i % Qh.shape[0]], non_blocking=True)
+        R.reskv_decode_attn(cache, -1, Qd_buf, O)
+        Oh.copy_(O, non_blocking=True)
+        torch.cuda.synchronize()
+    te = reduce_max(time.perf_counter() - t0, world, device)
+    e2e = {"value": aggregate(w.batch * e2e_steps, te, world), "unit": "tokens/s",
+           "h2d_bytes_per_step": int(Qd_buf.numel() * 2), "d2h_bytes_per_step": int(O.numel() * 4),
+           "how": "pinned host Q -> device, reskv_decode_attn, O -> pinned host, synchronised "
+                  "every step"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w)
+
+    if rank == 0:
+        units_launch = w.n_units
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": w.name, "layers": w.n_layers, "batch": w.batch,
+                       "kv_heads": w.n_kv_heads, "q_heads": w.n_q_heads, "head_dim": w.head_dim,
+                       "seq_len": w.seq_len, "budget": w.budget, "residual": w.residual,
+                       "mean_r": float(np.mean(r_counts)),
+                       "units_with_residual": float(np.mean(r_counts > 0)),
+                       "launch": "one reskv_decode_attn(layer=-1) launch per step",
+                       "l2": f"inputs larger than L2: {alg / 1e9:.2f} GB of cache read per step",
+                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "hbm_gbs": achieved, "frac_of_peak": achieved / peak,
+            "frac_of_nominal_8tbs": achieved / 8000.0,
+            "us_per_layer_step": ms_step * 1e3 / w.n_layers,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": profiled_traffic(units_launch),
+                         "peak_kind": f"{peak_kind} (burst copy)",
+                         "algorithmic_bytes_per_launch": alg},
+            "per_layer_graph": per_layer,
+            "construction_s": build_s,
+            "e2e": e2e,
+            "clocks": clk.summary(),
+            "gpu_launches": args.steps,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    cache.free()
+
+
+if __name__ == "__main__":
+    main()

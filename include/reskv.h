@@ -48,6 +48,7 @@ typedef enum {
 
 enum { RESKV_SCORE_OBS_POOL = 0, RESKV_SCORE_KEYNORM = 1 };
 enum { RESKV_GATE_DYNAMIC = 0, RESKV_GATE_FIXED = 1 };
+enum { RESKV_DECODE_AUTO = 0, RESKV_DECODE_FMA = 1, RESKV_DECODE_MMA = 2 };
 
 #define RESKV_MAX_GRID 8
 
@@ -91,6 +92,8 @@ typedef struct reskv_config {
                               pieces (one warp each) a decode call cuts its
                               slot range into, capped at 8 warps per SM; the
                               result does not depend on it beyond rounding   */
+  int32_t decode_kernel;   /* RESKV_DECODE_*: 0 automatic (tensor cores),
+                              1 CUDA-core fp32x2 FMA, 2 tensor-core mma.sync  */
 } reskv_config;
 
 /* Fill *cfg with the paper's defaults; shape fields are zeroed. */

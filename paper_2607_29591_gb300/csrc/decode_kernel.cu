@@ -26,6 +26,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 
@@ -420,10 +421,20 @@ size_t decode_partials_floats(int64_t n_units, int n_warps, int group) {
 
 template <int G>
 static cudaError_t launch_g(const DecodeParams& p, int n_ctas, cudaStream_t stream) {
+  // the shared-memory opt-in is set once per device, so that launches made
+  // during CUDA-graph capture issue nothing but the launch itself
+  static std::atomic<unsigned long long> configured{0};
   const int smem = kDecodeWarpsPerCta * kWarpSmem;
-  cudaError_t err = cudaFuncSetAttribute(reskv_decode_kernel<G>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (!(configured.load() & bit)) {
+    err = cudaFuncSetAttribute(reskv_decode_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               smem);
+    if (err != cudaSuccess) return err;
+    configured.fetch_or(bit);
+  }
   reskv_decode_kernel<G><<<n_ctas, kDecodeWarpsPerCta * 32, smem, stream>>>(p);
   return cudaGetLastError();
 }

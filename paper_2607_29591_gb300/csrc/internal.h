@@ -1,5 +1,6 @@
 // Internal declarations shared by the host ABI and the kernels.
 #pragma once
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -43,9 +44,15 @@ struct DecodeParams {
 
 constexpr int kDecodeWarpsPerCta = 8;
 
-// Launch the decode kernel for `group` (1, 2 or 4) query heads per KV head.
+// Launch the CUDA-core decode kernel for `group` (1, 2 or 4) query heads per KV head.
 cudaError_t launch_decode(const DecodeParams& p, int group, int n_ctas, cudaStream_t stream);
 size_t decode_partials_floats(int64_t n_units, int n_warps, int group);
+// Launch the tensor-core decode kernel (K/V rows through the given TMA maps).
+cudaError_t launch_decode_mma(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
+                              int group, int n_ctas, cudaStream_t stream);
+size_t decode_mma_partials_floats(int64_t n_units, int n_warps, int group);
+// Slots of zero padding after the log-count array (16-slot chunk copies).
+constexpr int kLogcPad = 16;
 
 void set_error(const std::string& msg);
 
@@ -71,6 +78,10 @@ struct reskv_cache {
   int32_t* tickets = nullptr;
   uint32_t* status = nullptr;
   int max_warps = 0;
+  // 2-D TMA maps of kslots / vslots: [U * budget rows, 128 dims], boxes of
+  // 16 rows x 64 dims with the 128-byte swizzle
+  CUtensorMap tmap_k;
+  CUtensorMap tmap_v;
   // construction intermediates kept for reskv_export_debug (device)
   double* dbg_scores = nullptr;
   int32_t* dbg_ranked = nullptr;

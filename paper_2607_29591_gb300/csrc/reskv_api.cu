@@ -1,7 +1,10 @@
 // Host side of the C ABI declared in include/reskv.h: argument validation,
 // ownership of the device layout, import/export, and decode launches.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -50,6 +53,11 @@ reskv_status validate_shape(const reskv_config* cfg) {
   if (cfg->budget < 1 || cfg->budget > (1 << 20))
     return fail(RESKV_ERR_INVALID_ARG, "budget must be in [1, 2^20]");
   if (cfg->decode_warps < 0) return fail(RESKV_ERR_INVALID_ARG, "decode_warps must be >= 0");
+  if (cfg->decode_kernel < RESKV_DECODE_AUTO || cfg->decode_kernel > RESKV_DECODE_MMA)
+    return fail(RESKV_ERR_INVALID_ARG, "unknown decode_kernel");
+  if (double(cfg->n_layers) * cfg->batch * cfg->n_kv_heads * cfg->budget + kLogcPad >=
+      double(int64_t(1) << 31))
+    return fail(RESKV_ERR_UNSUPPORTED, "at most 2^31 cache slots");
   if (cfg->gate_mode != RESKV_GATE_DYNAMIC && cfg->gate_mode != RESKV_GATE_FIXED)
     return fail(RESKV_ERR_INVALID_ARG, "unknown gate_mode");
   if (!std::isfinite(cfg->tau) || !std::isfinite(cfg->alpha) || !(cfg->g_min >= 0.f) ||
@@ -72,6 +80,33 @@ reskv_status dalloc(T** p, size_t count, const char* what) {
     return cuda_fail(err, what);
   }
   return RESKV_OK;
+}
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no -lcuda)
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+// [rows, 128] bf16 row-major -> TMA map with boxes of 16 rows x 64 dims, 128B swizzle
+bool encode_rows(CUtensorMap* map, void* base, uint64_t rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {cuuint64_t(kHeadDim), cuuint64_t(rows)};
+  const cuuint64_t strides[1] = {cuuint64_t(kSlotRowBytes)};
+  const cuuint32_t box[2] = {64, 16};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 void free_handle(reskv_cache* c) {
@@ -114,12 +149,14 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
   reskv_status st = RESKV_OK;
   if ((st = dalloc(&c->kslots, slots * kHeadDim, "cache keys")) != RESKV_OK ||
       (st = dalloc(&c->vslots, slots * kHeadDim, "cache values")) != RESKV_OK ||
-      (st = dalloc(&c->logc, slots, "log counts")) != RESKV_OK ||
+      (st = dalloc(&c->logc, slots + kLogcPad, "log counts")) != RESKV_OK ||
       (st = dalloc(&c->slot_pos, slots, "slot positions")) != RESKV_OK ||
       (st = dalloc(&c->counts, slots, "slot counts")) != RESKV_OK ||
       (st = dalloc(&c->n_main, size_t(c->n_units), "n_main")) != RESKV_OK ||
       (st = dalloc(&c->n_res, size_t(c->n_units), "n_res")) != RESKV_OK ||
-      (st = dalloc(&c->partials, decode_partials_floats(c->n_units, c->max_warps, cfg.group),
+      (st = dalloc(&c->partials,
+                   std::max(decode_partials_floats(c->n_units, c->max_warps, cfg.group),
+                            decode_mma_partials_floats(c->n_units, c->max_warps, cfg.group)),
                    "decode workspace")) != RESKV_OK ||
       (st = dalloc(&c->tickets, size_t(c->n_units), "decode tickets")) != RESKV_OK ||
       (st = dalloc(&c->status, 1, "status word")) != RESKV_OK) {
@@ -128,7 +165,7 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
   }
   err = cudaMemsetAsync(c->kslots, 0, slots * kHeadDim * 2, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->vslots, 0, slots * kHeadDim * 2, stream);
-  if (err == cudaSuccess) err = cudaMemsetAsync(c->logc, 0, slots * 4, stream);
+  if (err == cudaSuccess) err = cudaMemsetAsync(c->logc, 0, (slots + kLogcPad) * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->slot_pos, 0xff, slots * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->counts, 0, slots * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->tickets, 0, size_t(c->n_units) * 4, stream);
@@ -136,6 +173,10 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
   if (err != cudaSuccess) {
     free_handle(c);
     return cuda_fail(err, "initialising the cache");
+  }
+  if (!encode_rows(&c->tmap_k, c->kslots, slots) || !encode_rows(&c->tmap_v, c->vslots, slots)) {
+    free_handle(c);
+    return fail(RESKV_ERR_CUDA, "creating the TMA tensor maps of the cache");
   }
   *out = c;
   return RESKV_OK;
@@ -292,7 +333,11 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   p.g_min = cfg.g_min;
   p.g_fixed = cfg.g_fixed;
   const int n_ctas = int((W + kDecodeWarpsPerCta - 1) / kDecodeWarpsPerCta);
-  cudaError_t err = launch_decode(p, cfg.group, n_ctas, static_cast<cudaStream_t>(stream));
+  cudaError_t err =
+      cfg.decode_kernel == RESKV_DECODE_FMA
+          ? launch_decode(p, cfg.group, n_ctas, static_cast<cudaStream_t>(stream))
+          : launch_decode_mma(p, c->tmap_k, c->tmap_v, cfg.group, n_ctas,
+                              static_cast<cudaStream_t>(stream));
   if (err != cudaSuccess) return cuda_fail(err, "decode launch");
   return RESKV_OK;
 }

@@ -21,6 +21,7 @@ STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "OOM", 4: "CUDA"
                 5: "DEVICE_STATUS"}
 RESKV_SCORE_OBS_POOL, RESKV_SCORE_KEYNORM = 0, 1
 RESKV_GATE_DYNAMIC, RESKV_GATE_FIXED = 0, 1
+RESKV_DECODE_AUTO, RESKV_DECODE_FMA, RESKV_DECODE_MMA = 0, 1, 2
 RESKV_DEBUG_SCORES, RESKV_DEBUG_RANKED, RESKV_DEBUG_LOSSES, RESKV_DEBUG_CANDIDATES = 0, 1, 2, 3
 MAX_GRID = 8
 
@@ -43,7 +44,7 @@ class reskv_config(ctypes.Structure):
         ("residual_override", ctypes.POINTER(ctypes.c_int32)),
         ("gate_mode", ctypes.c_int32), ("tau", ctypes.c_float), ("alpha", ctypes.c_float),
         ("g_min", ctypes.c_float), ("g_fixed", ctypes.c_float), ("keep_debug", ctypes.c_int32),
-        ("decode_warps", ctypes.c_int32),
+        ("decode_warps", ctypes.c_int32), ("decode_kernel", ctypes.c_int32),
     ]
 
 

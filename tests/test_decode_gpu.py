@@ -29,6 +29,20 @@ def lib():
     return R.load_library()
 
 
+KERNEL = {"id": R.RESKV_DECODE_MMA}
+
+
+@pytest.fixture(autouse=True, params=[R.RESKV_DECODE_FMA, R.RESKV_DECODE_MMA], ids=["fma", "mma"])
+def decode_kernel(request):
+    """Every decode test runs on both kernels: CUDA-core FMA and tensor-core mma."""
+    KERNEL["id"] = request.param
+    yield request.param
+
+
+def mkcfg(**kw):
+    return R.reskv_config_default(decode_kernel=KERNEL["id"], **kw)
+
+
 def ocfg_from(cfg):
     return orc.OracleConfig(budget=cfg.budget, gate_mode=cfg.gate_mode, tau=cfg.tau,
                             alpha=cfg.alpha, g_min=cfg.g_min, g_fixed=cfg.g_fixed)
@@ -107,7 +121,7 @@ def test_tiny_oracle_built_cache():
     assert cache.r == 32 and len(cache.main_pos) == 224
     lay = empty_layout(1, w.budget)
     put_unit(lay, 0, cache)
-    cfg = R.reskv_config_default(batch=1, n_layers=1, n_kv_heads=1, group=4, seq_len=w.seq_len,
+    cfg = mkcfg(batch=1, n_layers=1, n_kv_heads=1, group=4, seq_len=w.seq_len,
                                  budget=w.budget)
     h = R.reskv_import_cache(cfg, **lay)
     qf = bf16_to_f64(Qd)
@@ -134,7 +148,7 @@ def test_ragged_layout_all_layers(decode_warps):
     tail slots; one all-layer launch cut into various warp counts."""
     L, Bt, H, G, b = 2, 3, 2, 4, 300
     w, lay = synthetic_layout(L, Bt, H, b, SPLITS)
-    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
                                  budget=b, decode_warps=decode_warps)
     h = R.reskv_import_cache(cfg, **lay)
     Q = queries_for(w, L, Bt, H, G)
@@ -149,7 +163,7 @@ def test_ragged_layout_all_layers(decode_warps):
 def test_per_layer_calls_match_all_layer_call():
     L, Bt, H, G, b = 2, 3, 2, 4, 300
     w, lay = synthetic_layout(L, Bt, H, b, SPLITS)
-    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
                                  budget=b)
     h = R.reskv_import_cache(cfg, **lay)
     Q = queries_for(w, L, Bt, H, G)
@@ -166,7 +180,7 @@ def test_determinism_and_split_invariance():
     Q = queries_for(w, L, Bt, H, G)
     outs = []
     for dw in (1, 2, 4, 16, 0):
-        cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G,
+        cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G,
                                      seq_len=w.seq_len, budget=b, decode_warps=dw)
         h = R.reskv_import_cache(cfg, **lay)
         o1 = run_decode(h, Q)
@@ -182,7 +196,7 @@ def test_group_sizes(G):
     L, Bt, H, b = 1, 2, 3, 256
     splits = [(200, 56), (256, 0), (10, 100), (128, 64), (1, 255), (100, 3)]
     w, lay = synthetic_layout(L, Bt, H, b, splits)
-    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
                                  budget=b)
     h = R.reskv_import_cache(cfg, **lay)
     Q = queries_for(w, L, Bt, H, G)
@@ -199,7 +213,7 @@ def test_fixed_point_empty_residual_is_eviction():
     L, Bt, H, G, b = 1, 2, 2, 4, 512
     splits = [(512, 0), (300, 0), (77, 0), (1, 0)]
     w, lay = synthetic_layout(L, Bt, H, b, splits)
-    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
                                  budget=b)
     h = R.reskv_import_cache(cfg, **lay)
     Q = queries_for(w, L, Bt, H, G)
@@ -218,7 +232,7 @@ def test_fixed_point_gate_zero_is_main_only():
     L, Bt, H, G, b = 1, 1, 3, 4, 400
     splits = [(300, 100), (50, 350), (399, 1)]
     w, lay = synthetic_layout(L, Bt, H, b, splits)
-    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
                                  budget=b, gate_mode=R.RESKV_GATE_FIXED, g_fixed=0.0)
     h = R.reskv_import_cache(cfg, **lay)
     Q = queries_for(w, L, Bt, H, G)
@@ -250,7 +264,7 @@ def test_fixed_point_exact_residual_encoding_is_full_attention():
     vbar = orc.round_to_bf16(NE / ZE)
     lay["vslots"][0, m] = (vbar.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)
     lay["logc"][0, m] = np.float32(np.log(ZE))          # k_bar = 0, so <q, k_bar> = 0
-    cfg = R.reskv_config_default(batch=1, n_layers=1, n_kv_heads=1, group=1, seq_len=s,
+    cfg = mkcfg(batch=1, n_layers=1, n_kv_heads=1, group=1, seq_len=s,
                                  budget=m + 1, gate_mode=R.RESKV_GATE_FIXED, g_fixed=1.0)
     h = R.reskv_import_cache(cfg, **lay)
     O = run_decode(h, Qd.reshape(1, 1, 1, d)).cpu().numpy()[0, 0, 0]
