@@ -136,7 +136,7 @@ def zn_stats(q: np.ndarray, K: np.ndarray, V: np.ndarray, shift: float = 0.0):
 
 
 # ---------------------------------------------------------------------------
-# Token scoring (App. B.2 SnapKV rule; Alg. 1 step 2)
+# Token scoring (App. B.2 SnapKV rule; Alg. 1)
 # ---------------------------------------------------------------------------
 
 def scores_obs_pool(K: np.ndarray, Qfit: np.ndarray, pool: int) -> np.ndarray:
@@ -356,7 +356,7 @@ class UnitCache:
 
 
 def build_candidate(K, V, ranked, cfg: OracleConfig, r: int) -> UnitCache:
-    """Main cache M_r and residual entries for one candidate r (Alg. 1 steps 5-6)."""
+    """Main cache M_r and residual entries for one candidate r (Alg. 1, candidate loop)."""
     s = K.shape[0]
     m = min(cfg.budget - r, s)
     if r == 0:
@@ -402,7 +402,7 @@ def validation_loss(cache: UnitCache, Qval: np.ndarray, O_full: np.ndarray,
 
 def choose_r(L0: float, rs: Sequence[int], losses: Sequence[float], delta: float) -> int:
     """r* = argmin_{r>0} L_r (ties -> smaller r); keep r* only if
-    L_{r*} < (1 - delta) L_0, else r = 0  (Eq. valproxy; Alg. 1 steps 9-14)."""
+    L_{r*} < (1 - delta) L_0, else r = 0  (Eq. valproxy; Alg. 1, choice of r)."""
     if len(rs) == 0:
         return 0
     order = sorted(range(len(rs)), key=lambda i: (losses[i], rs[i]))
@@ -419,7 +419,7 @@ def build_unit(K: np.ndarray, V: np.ndarray, Qobs: Optional[np.ndarray],
     query-free score.
     """
     s = K.shape[0]
-    # step 2: token scores on the fit queries; recent protection P
+    # token scores on the fit queries; recent protection P
     if cfg.score_mode == SCORE_OBS_POOL:
         scores = scores_obs_pool(K, Qobs[:, :cfg.n_fit], cfg.pool_kernel)
     elif cfg.score_mode == SCORE_KEYNORM:
@@ -441,22 +441,22 @@ def build_unit(K: np.ndarray, V: np.ndarray, Qobs: Optional[np.ndarray],
         out.scores, out.ranked = scores, ranked
         return out
 
-    # step 1: validation part of the observation window; its full-cache outputs
+    # validation part of the observation window; its full-cache outputs
     Qval = Qobs[:, Qobs.shape[1] - cfg.n_val:]
     G = Qval.shape[0]
     O_full = np.stack([np.stack([attention_full(Qval[g, t], K, V)
                                  for t in range(cfg.n_val)]) for g in range(G)])
-    # step 3: pure-main cache and L_0
+    # pure-main cache and L_0
     c0 = build_candidate(K, V, ranked, cfg, 0)
     L0 = validation_loss(c0, Qval, O_full, cfg)
     losses = {0: L0}
-    # steps 4-8: every candidate r > 0
+    # Alg. 1, candidate loop: every candidate r > 0
     rs = [r for r in candidate_budgets(cfg.budget, cfg.grid_ratios) if candidate_valid(s, cfg, r)]
     built = {}
     for r in rs:
         built[r] = build_candidate(K, V, ranked, cfg, r)
         losses[r] = validation_loss(built[r], Qval, O_full, cfg)
-    # steps 9-14: r* and the margin test; step 15: the cache for the chosen r
+    # Alg. 1: r* and the margin test, then the cache for the chosen r
     r_star = choose_r(L0, rs, [losses[r] for r in rs], cfg.delta)
     out = built[r_star] if r_star > 0 else c0
     out.scores, out.ranked, out.losses = scores, ranked, losses

@@ -238,7 +238,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     const __nv_bfloat16* V = static_cast<const __nv_bfloat16*>(Vl[l]);
     const __nv_bfloat16* Q = Ql ? static_cast<const __nv_bfloat16*>(Ql[l]) : nullptr;
 
-    // ---- step 2: token scores ----
+    // ---- token scores ----
     if (cfg.score_mode == RESKV_SCORE_OBS_POOL) {
       ObsArgs oa{K, Q, s, G, cfg.n_obs, n_fit_rows, cfg.n_fit, ntiles, tstats, rstats, A};
       k_obs_pass1<<<dim3(ntiles, UL), kThreads, sm_obs1, stream>>>(oa);
@@ -271,7 +271,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     };
 
     if (proxy) {
-      // ---- steps 1, 3-14: validation targets, candidates, choice ----
+      // ---- validation targets, candidates, choice of r ----
       ValArgs va{K, V, Q, s, G, cfg.n_obs, cfg.n_val, n_val_rows, nchunks, vpart, oS};
       k_val_full<<<dim3(nchunks, unsigned(cdiv(n_val_rows, kRowBlk)), UL), kThreads, sm_val, stream>>>(va);
       k_val_combine<<<dim3(n_val_rows, UL), kHeadDim, 0, stream>>>(va);
@@ -316,7 +316,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       }
     }
 
-    // ---- step 15: pack the chosen cache ----
+    // ---- pack the chosen cache ----
     PackArgs pa{K, V, s, P, b, rank_pos, r_final, chosen, run_off_d, kbar, vbar, ecount,
                 ent_stride, cfg.beta, int64_t(l) * UL, c->kslots, c->vslots, c->logc,
                 c->slot_pos, c->counts, c->n_main, c->n_res};

@@ -96,7 +96,7 @@ __device__ __forceinline__ float warp_sum(float v) {
 }
 
 // ---------------------------------------------------------------------------
-// Token scores (App. B.2 SnapKV rule; Alg. 1 step 2)
+// Token scores (App. B.2 SnapKV rule; Alg. 1)
 // ---------------------------------------------------------------------------
 
 struct ObsArgs {
@@ -674,7 +674,7 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_update(LloydArgs p, int fina
 }
 
 // ---------------------------------------------------------------------------
-// Validation proxy (Sec. 5.5.1, Eqs. valloss, valproxy; Alg. 1 steps 3-14)
+// Validation proxy (Sec. 5.5.1, Eqs. valloss, valproxy; Alg. 1)
 // ---------------------------------------------------------------------------
 
 constexpr int kValChunkTiles = 16;           // 2048 tokens per CTA
@@ -946,7 +946,7 @@ __global__ void k_choose(const double* losses, int ncol, const int32_t* cand_r, 
 }
 
 // ---------------------------------------------------------------------------
-// Packing into the ragged layout (Alg. 1 step 15): main rows in position
+// Packing into the ragged layout (end of Alg. 1): main rows in position
 // order, then the chosen run's residual entries.
 // ---------------------------------------------------------------------------
 

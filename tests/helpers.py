@@ -64,7 +64,7 @@ def errors(out: np.ndarray, ref: np.ndarray):
     return float(np.max(np.abs(diff))), float(np.linalg.norm(diff) / np.linalg.norm(ref))
 
 
-def assert_north_star(out, ref, what=""):
+def assert_output_parity(out, ref, what=""):
     mx, rel = errors(out, ref)
     assert mx <= MAX_ABS and rel <= REL_L2, f"{what}: max abs {mx:.3g}, rel L2 {rel:.3g}"
     return mx, rel

@@ -23,7 +23,7 @@ from paper_2607_29591_gb300 import build as B
 from paper_2607_29591_gb300 import reskv as R
 from paper_2607_29591_gb300 import workloads as wl
 
-from helpers import assert_north_star, bf16_to_f64, errors, unit_from_layout
+from helpers import assert_output_parity, bf16_to_f64, errors, unit_from_layout
 
 pytestmark = pytest.mark.gpu
 
@@ -135,7 +135,7 @@ def decode_parity(cache, lay, ref_units, Ks, Qd, w, ocfg_of):
         b, h = divmod(rem, H)
         q = qf[l, b, h * G:(h + 1) * G]
         ref_o = orc.decode_unit(ref, q, ocfg_of(u))
-        mx, rel = assert_north_star(O[l, b, h * G:(h + 1) * G], ref_o, f"unit {u}")
+        mx, rel = assert_output_parity(O[l, b, h * G:(h + 1) * G], ref_o, f"unit {u}")
         # the kernel alone: oracle decode of the GPU's own cache
         own = orc.decode_unit(unit_from_layout(lay, u), q, ocfg_of(u))
         assert errors(O[l, b, h * G:(h + 1) * G], own)[1] < 1e-4

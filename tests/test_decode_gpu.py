@@ -16,7 +16,7 @@ from paper_2607_29591_gb300 import build as B
 from paper_2607_29591_gb300 import reskv as R
 from paper_2607_29591_gb300 import workloads as wl
 
-from helpers import (assert_north_star, bf16_bits, bf16_to_f64, empty_layout, errors,
+from helpers import (assert_output_parity, bf16_bits, bf16_to_f64, empty_layout, errors,
                      put_unit, unit_from_layout)
 
 pytestmark = pytest.mark.gpu
@@ -130,7 +130,7 @@ def test_tiny_oracle_built_cache():
         q = Qd[:, t].reshape(1, 4, 128).contiguous()
         O = run_decode(h, q, layer=0).cpu().numpy()[0]
         ref = orc.decode_unit(cache, qf[:, t], oc)
-        mx, rel = assert_north_star(O, ref, f"step {t}")
+        mx, rel = assert_output_parity(O, ref, f"step {t}")
         worst = (max(worst[0], mx), max(worst[1], rel))
     assert worst[1] < 1e-4          # fp32 accumulation lands far inside the bar
     R.reskv_check_status(h)
@@ -155,7 +155,7 @@ def test_ragged_layout_all_layers(decode_warps):
     O = run_decode(h, Q).cpu().numpy()
     ref = oracle_decode_all(lay, Q, cfg)
     assert not np.isnan(O).any()
-    mx, rel = assert_north_star(O, ref, f"warps {decode_warps}")
+    mx, rel = assert_output_parity(O, ref, f"warps {decode_warps}")
     assert rel < 1e-4
     R.reskv_check_status(h)
 
@@ -201,7 +201,7 @@ def test_group_sizes(G):
     h = R.reskv_import_cache(cfg, **lay)
     Q = queries_for(w, L, Bt, H, G)
     O = run_decode(h, Q).cpu().numpy()
-    assert_north_star(O, oracle_decode_all(lay, Q, cfg), f"G={G}")
+    assert_output_parity(O, oracle_decode_all(lay, Q, cfg), f"G={G}")
 
 
 def _textbook(q, K, V):
@@ -225,7 +225,7 @@ def test_fixed_point_empty_residual_is_eviction():
         Vm = orc.bf16_bits_to_f64(lay["vslots"][u, :m])
         for g in range(G):
             ref = _textbook(qf[0, bb, hh * G + g], Km, Vm)
-            assert_north_star(O[0, bb, hh * G + g], ref, "eviction")
+            assert_output_parity(O[0, bb, hh * G + g], ref, "eviction")
 
 
 def test_fixed_point_gate_zero_is_main_only():
@@ -242,7 +242,7 @@ def test_fixed_point_gate_zero_is_main_only():
         Km = orc.bf16_bits_to_f64(lay["kslots"][u, :m])
         Vm = orc.bf16_bits_to_f64(lay["vslots"][u, :m])
         for g in range(G):
-            assert_north_star(O[0, 0, u * G + g], _textbook(qf[0, 0, u * G + g], Km, Vm), "g=0")
+            assert_output_parity(O[0, 0, u * G + g], _textbook(qf[0, 0, u * G + g], Km, Vm), "g=0")
 
 
 def test_fixed_point_exact_residual_encoding_is_full_attention():
@@ -269,6 +269,6 @@ def test_fixed_point_exact_residual_encoding_is_full_attention():
     h = R.reskv_import_cache(cfg, **lay)
     O = run_decode(h, Qd.reshape(1, 1, 1, d)).cpu().numpy()[0, 0, 0]
     full = _textbook(q, Kf, Vf)
-    assert_north_star(O, full, "exact encoding")
+    assert_output_parity(O, full, "exact encoding")
     # the residual's share of the output carries only bf16 rounding of v_bar
     assert errors(O, full)[1] < 4e-3 * ZE / (ZE + np.exp(Kf[:m] @ q / math.sqrt(d)).sum()) + 1e-5
