@@ -167,8 +167,12 @@ def scores_obs_pool(K: np.ndarray, Qfit: np.ndarray, pool: int) -> np.ndarray:
 
 
 def scores_keynorm(K: np.ndarray) -> np.ndarray:
-    """Query-free score s_p = ||k_p||^2 (a build choice; the paper has none)."""
-    return np.sum(K * K, axis=1)
+    """Query-free score s_p = ||k_p||^2 (a build choice; the paper has none),
+    summed over the dimensions in order (k_1^2 + k_2^2 + ...)."""
+    acc = np.zeros(K.shape[0], dtype=np.float64)
+    for i in range(K.shape[1]):
+        acc = acc + K[:, i] * K[:, i]
+    return acc
 
 
 # ---------------------------------------------------------------------------
