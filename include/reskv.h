@@ -200,6 +200,54 @@ enum {
 reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_dst,
                                 size_t bytes);
 
+/*
+ * Decode that allocates nothing.  The paper has no counterpart: this entry
+ * point exists for callers that cannot allocate device memory at decode time
+ * -- code running inside a host application whose memory manager owns every
+ * GPU allocation, or latency-critical paths that must not call cudaMalloc
+ * (it may block and synchronise the device).  Such callers hold the
+ * compressed cache in memory of their own and describe it here with plain
+ * device pointers (the layout of reskv_import_cache, on the device).
+ *
+ * The per-call scratch (partial results of units split between warps, their
+ * tickets, a status word) lives in one static device array of 16 MiB inside
+ * the library; every GPU that loads the library holds it until the process
+ * exits.  A call whose scratch would exceed it fails with
+ * RESKV_ERR_UNSUPPORTED before launching anything; decode fewer units per call
+ * (one layer at a time) in that case.  Roughly, a call needs
+ * (n_units + 8 * SMs) * 2 * group * 520 bytes plus 4 bytes per unit.
+ *
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current); make that first call
+ * before any stream capture.  Every call shares the array and clears the
+ * parts that must start at zero, so calls that overlap on the GPU race: order
+ * them on one stream (or synchronise between them).
+ *
+ *   kslots, vslots : device bf16 [n_units, budget, 128], 16-byte aligned
+ *   logc           : device fp32 [n_units, budget] (beta*log c at residual slots)
+ *   n_main, n_res  : device int32 [n_units]; the caller guarantees
+ *                    1 <= n_main[u] and n_main[u] + n_res[u] <= budget
+ *   Q              : device bf16 [n_units / n_kv_heads, n_kv_heads*group, 128]
+ *   O              : device fp32, same shape as Q
+ * Runs the CUDA-core decode kernel, which reads only inside these arrays.
+ */
+typedef struct reskv_device_cache {
+  const void* kslots;
+  const void* vslots;
+  const float* logc;
+  const int32_t* n_main;
+  const int32_t* n_res;
+  int64_t n_units;
+  int32_t budget;
+  int32_t n_kv_heads;
+  int32_t group;
+  int32_t gate_mode;
+  float tau, alpha, g_min, g_fixed;
+} reskv_device_cache;
+
+reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, const void* Q, void* O,
+                                       void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -59,6 +59,15 @@ class reskv_cache_info(ctypes.Structure):
                 ("cache_bytes", ctypes.c_int64)]
 
 
+class reskv_device_cache(ctypes.Structure):
+    _fields_ = [("kslots", ctypes.c_void_p), ("vslots", ctypes.c_void_p),
+                ("logc", ctypes.c_void_p), ("n_main", ctypes.c_void_p), ("n_res", ctypes.c_void_p),
+                ("n_units", ctypes.c_int64), ("budget", ctypes.c_int32),
+                ("n_kv_heads", ctypes.c_int32), ("group", ctypes.c_int32),
+                ("gate_mode", ctypes.c_int32), ("tau", ctypes.c_float), ("alpha", ctypes.c_float),
+                ("g_min", ctypes.c_float), ("g_fixed", ctypes.c_float)]
+
+
 _lib = None
 
 
@@ -95,6 +104,8 @@ def load_library():
     lib.reskv_export_cache.restype = i32
     lib.reskv_export_debug.argtypes = [vp, i32, vp, sz]
     lib.reskv_export_debug.restype = i32
+    lib.reskv_decode_attn_noalloc.argtypes = [ctypes.POINTER(reskv_device_cache), vp, vp, vp]
+    lib.reskv_decode_attn_noalloc.restype = i32
     _lib = lib
     return lib
 
@@ -283,3 +294,28 @@ def reskv_export_debug(cache: Cache, what: int, n_cand: Optional[int] = None) ->
     _check(load_library().reskv_export_debug(cache.handle, int(what),
                                              ctypes.c_void_p(out.ctypes.data), out.nbytes))
     return out
+
+
+def reskv_decode_attn_noalloc(kslots, vslots, logc, n_main, n_res, n_kv_heads: int, group: int,
+                              Q, O, gate_mode: int = RESKV_GATE_DYNAMIC, tau: float = 0.25,
+                              alpha: float = 12.0, g_min: float = 0.0, g_fixed: float = 1.0,
+                              stream=None) -> None:
+    """Decode from a cache held in the caller's own device tensors, with no
+    device allocation by the library (see include/reskv.h).
+
+    kslots, vslots: bf16 [U, b, 128]; logc: float32 [U, b]; n_main, n_res:
+    int32 [U]; Q: bf16 [U / n_kv_heads, n_kv_heads * group, 128]; O: float32.
+    """
+    U, b = int(kslots.shape[0]), int(kslots.shape[1])
+    d = reskv_device_cache(
+        kslots=_dptr(kslots, "torch.bfloat16", "kslots").value,
+        vslots=_dptr(vslots, "torch.bfloat16", "vslots").value,
+        logc=_dptr(logc, "torch.float32", "logc").value,
+        n_main=_dptr(n_main, "torch.int32", "n_main").value,
+        n_res=_dptr(n_res, "torch.int32", "n_res").value,
+        n_units=U, budget=b, n_kv_heads=int(n_kv_heads), group=int(group),
+        gate_mode=int(gate_mode), tau=tau, alpha=alpha, g_min=g_min, g_fixed=g_fixed)
+    _check(load_library().reskv_decode_attn_noalloc(ctypes.byref(d),
+                                                    _dptr(Q, "torch.bfloat16", "Q"),
+                                                    _dptr(O, "torch.float32", "O"),
+                                                    _stream(stream)))

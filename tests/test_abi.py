@@ -50,6 +50,9 @@ def test_struct_layout_matches_c(lib, tmp_path):
              'printf("%zu\\n", sizeof(reskv_host_cache));',
              'printf("%zu\\n", sizeof(reskv_cache_info));']
     lines += [f'printf("%zu\\n", offsetof(reskv_config, {f}));' for f in fields]
+    lines += ['printf("%zu\\n", sizeof(reskv_device_cache));']
+    lines += [f'printf("%zu\\n", offsetof(reskv_device_cache, {f}));'
+              for f, _ in R.reskv_device_cache._fields_]
     lines += ["return 0;}"]
     src.write_text("\n".join(lines))
     exe = tmp_path / "layout"
@@ -60,8 +63,12 @@ def test_struct_layout_matches_c(lib, tmp_path):
     assert vals[0] == ctypes.sizeof(R.reskv_config)
     assert vals[1] == ctypes.sizeof(R.reskv_host_cache)
     assert vals[2] == ctypes.sizeof(R.reskv_cache_info)
-    for f, off in zip(fields, vals[3:]):
+    for f, off in zip(fields, vals[3:3 + len(fields)]):
         assert getattr(R.reskv_config, f).offset == off, f
+    dfields = [f for f, _ in R.reskv_device_cache._fields_]
+    assert vals[3 + len(fields)] == ctypes.sizeof(R.reskv_device_cache)
+    for f, off in zip(dfields, vals[4 + len(fields):]):
+        assert getattr(R.reskv_device_cache, f).offset == off, f
 
 
 def test_defaults_are_the_papers(lib):

@@ -1,0 +1,107 @@
+"""The decode entry point that allocates nothing (reskv_decode_attn_noalloc).
+
+It serves callers that cannot allocate GPU memory while decoding -- for
+instance code living inside a host application whose memory manager owns all
+device allocations, or latency-critical paths that must avoid cudaMalloc.  They
+keep the cache in their own device memory; the library takes its per-call
+scratch from a fixed static array instead of allocating.  The output must
+agree with the regular entry point (reskv_decode_attn on a handle holding the
+same cache), call after call, since every call reuses the same scratch.
+
+This file is named so that pytest collects it last; it needs nothing from the
+other tests and runs alone in a fresh process as well.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_29591_gb300 import build as B
+from paper_2607_29591_gb300 import reskv as R
+from paper_2607_29591_gb300 import workloads as wl
+
+from helpers import assert_output_parity, bf16_bits, empty_layout, errors
+
+pytestmark = pytest.mark.gpu
+
+
+def _layout(L, Bt, H, b, seed=7):
+    """A ragged cache of seeded generator rows (main, residual, unused tail)."""
+    U = L * Bt * H
+    w = wl.Workload("noalloc", L, Bt, H, 4, 128, b + 32, b, 0, 0, 0, 0, "fixed:0", 1)
+    lay = empty_layout(U, b)
+    rng = np.random.default_rng(seed)
+    for u in range(U):
+        l, rem = divmod(u, Bt * H)
+        bb, h = divmod(rem, H)
+        m = int(rng.integers(1, b + 1))
+        r = int(rng.integers(0, b - m + 1))
+        K, V = wl.unit_kv(w, l, bb, h)
+        lay["n_main"][u], lay["n_res"][u] = m, r
+        lay["kslots"][u, :m + r] = bf16_bits(K[:m + r])
+        lay["vslots"][u, :m + r] = bf16_bits(V[:m + r])
+        if r:
+            c = rng.integers(0, 100, r)
+            with np.errstate(divide="ignore"):
+                lay["logc"][u, m:m + r] = np.log(c.astype(np.float64)).astype(np.float32)
+    Q = torch.empty((L, Bt, H * 4, 128), dtype=torch.bfloat16)
+    for l in range(L):
+        for bb in range(Bt):
+            for h in range(H):
+                K, _ = wl.unit_kv(w, l, bb, h)
+                Q[l, bb, h * 4:(h + 1) * 4] = wl.unit_decode_queries(w, l, bb, h, K, 1)[:, 0]
+    return lay, Q
+
+
+def test_noalloc_matches_regular_entry_point_on_repeated_calls():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    B.build()
+    L, Bt, H, b = 3, 2, 4, 400
+    lay, Q = _layout(L, Bt, H, b)
+    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=4, seq_len=b + 32,
+                                 budget=b)
+    handle = R.reskv_import_cache(cfg, **lay)
+    Qd = Q.cuda()
+    O_ref = torch.empty(Qd.shape, dtype=torch.float32, device="cuda")
+    R.reskv_decode_attn(handle, -1, Qd, O_ref)
+
+    # the same cache in the caller's own device memory
+    dev = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a)).cuda().view(dt)
+    ks = dev(lay["kslots"].view(np.int16), torch.bfloat16)
+    vs = dev(lay["vslots"].view(np.int16), torch.bfloat16)
+    lc = dev(lay["logc"], torch.float32)
+    nm = dev(lay["n_main"], torch.int32)
+    nr = dev(lay["n_res"], torch.int32)
+    ref = O_ref.cpu().numpy().astype(np.float64)
+    for call in range(2):
+        O = torch.full(Qd.shape, float("nan"), dtype=torch.float32, device="cuda")
+        R.reskv_decode_attn_noalloc(ks, vs, lc, nm, nr, H, 4, Qd, O)
+        torch.cuda.synchronize()
+        out = O.cpu().numpy()
+        assert not np.isnan(out).any(), f"call {call}: output not fully written"
+        assert_output_parity(out, ref, f"call {call}")
+        assert errors(out, ref)[1] < 1e-5, f"call {call}"
+    # per-layer calls through the same scratch
+    for l in range(L):
+        U_l = Bt * H
+        O = torch.empty(Qd[l].shape, dtype=torch.float32, device="cuda")
+        sl = slice(l * U_l, (l + 1) * U_l)
+        R.reskv_decode_attn_noalloc(ks[sl], vs[sl], lc[sl], nm[sl], nr[sl], H, 4,
+                                    Qd[l].contiguous(), O)
+        torch.cuda.synchronize()
+        assert errors(O.cpu().numpy(), ref[l])[1] < 1e-5
+    handle.free()
+
+
+def test_noalloc_rejects_calls_beyond_its_scratch():
+    """A call whose scratch would exceed the 16 MiB array fails on the host
+    with a clear message, before anything is launched."""
+    B.build()
+    U, b = 65536, 8
+    ks = torch.zeros((U, b, 128), dtype=torch.bfloat16, device="cuda")
+    lc = torch.zeros((U, b), dtype=torch.float32, device="cuda")
+    n = torch.ones(U, dtype=torch.int32, device="cuda")
+    Q = torch.zeros((U // 8, 32, 128), dtype=torch.bfloat16, device="cuda")
+    O = torch.zeros((U // 8, 32, 128), dtype=torch.float32, device="cuda")
+    with pytest.raises(R.ReskvError) as e:
+        R.reskv_decode_attn_noalloc(ks, ks, lc, n, n * 0, 8, 4, Q, O)
+    assert e.value.status == 2 and "16 MiB" in str(e.value)
