@@ -38,7 +38,7 @@ DEFAULT_WORKLOAD = "llama8b_32l_32k_b8"
 SLOT_BYTES = 2 * 128 * 2            # one K row + one V row, bf16
 PROFILE = os.path.join(ROOT, "profiles", "decode_kernel_llama8b_32l_32k_b8.md")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_29591_gb300", "csrc", f)
-                  for f in ("decode_kernel.cu", "device_utils.cuh")]
+                  for f in ("decode_mma.cu", "device_utils.cuh")]
 
 
 def parse_args():
@@ -50,6 +50,8 @@ def parse_args():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(wl.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-per-layer", action="store_true")
+    ap.add_argument("--decode-kernel", choices=["mma", "fma"], default="mma",
+                    help="tensor-core (default) or CUDA-core decode kernel")
     ap.add_argument("--layers", type=int, default=0,
                     help="use only this many layers (smaller profiling case)")
     return ap.parse_args()
@@ -274,7 +276,7 @@ def run_reference(args, world, rank):
 # the GPU arm
 # ---------------------------------------------------------------------------
 
-def build_workload(w: wl.Workload, n_q: int, device):
+def build_workload(w: wl.Workload, n_q: int, device, decode_kernel: int):
     """Generate inputs layer by layer; build the compressed cache (timed)."""
     from paper_2607_29591_gb300 import reskv as R
     Ks, Vs, Qs = [], [], []
@@ -290,7 +292,8 @@ def build_workload(w: wl.Workload, n_q: int, device):
                                  group=w.group, seq_len=w.seq_len, budget=w.budget,
                                  recent_window=w.recent_window, n_obs=w.n_obs, n_fit=w.n_fit,
                                  n_val=w.n_val, score_mode=w.score_mode,
-                                 residual_override=w.residual_override())
+                                 residual_override=w.residual_override(),
+                                 decode_kernel=decode_kernel)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
@@ -321,7 +324,8 @@ def main():
     if args.layers:
         w = wl.scaled(w, n_layers=args.layers, name=f"{w.name}_{args.layers}l")
     n_q = args.steps + args.warmup
-    cache, Qdec, build_s = build_workload(w, n_q, device)
+    kern = R.RESKV_DECODE_MMA if args.decode_kernel == "mma" else R.RESKV_DECODE_FMA
+    cache, Qdec, build_s = build_workload(w, n_q, device, kern)
     lay_meta = R.reskv_export_cache(cache)
     alg = algorithmic_bytes(lay_meta["n_main"], lay_meta["n_res"])
     r_counts = lay_meta["n_res"]

@@ -39,13 +39,15 @@
 namespace reskv {
 namespace {
 
-constexpr int kW = kDecodeWarpsPerCta;  // warps per CTA
-constexpr int kSt = 3;                  // ring stages per warp
+constexpr int kMaxW = 8;                // warps per CTA (at most)
+constexpr int kMaxSt = 12;              // ring stages per warp (at most)
 constexpr int kCh = 16;                 // slots per stage (= one MMA tile)
 constexpr int kBox = kCh * 128;         // one 64-dim half of 16 rows, bytes
 constexpr int kStageBytes = 4 * kBox;   // K lo | K hi | V lo | V hi
-constexpr int kWarpBytes = kSt * kStageBytes + 1024;   // + logc, barriers, padding
 constexpr int kRec = kHeadDim + 4;      // m, l, pad, pad, acc[d]
+constexpr int kSmemLimit = 227 * 1024;  // dynamic shared memory per CTA
+
+__host__ __device__ constexpr int warp_bytes(int stages) { return stages * kStageBytes + 1024; }
 
 __device__ __forceinline__ int64_t warp_begin(int64_t w, int64_t T, int64_t W) { return (w * T) / W; }
 __device__ __forceinline__ int64_t warp_of(int64_t x, int64_t T, int64_t W) { return ((x + 1) * W - 1) / T; }
@@ -97,10 +99,13 @@ __device__ __forceinline__ float gate_of(const DecodeParams& p, float lM) {
 }
 
 template <int G>
-__global__ void __launch_bounds__(kW * 32, 1)
+__global__ void __launch_bounds__(kMaxW * 32, 1)
     reskv_decode_mma_kernel(const DecodeParams p, const __grid_constant__ CUtensorMap tmK,
                             const __grid_constant__ CUtensorMap tmV) {
   extern __shared__ uint8_t smem_raw[];
+  const int kW = blockDim.x >> 5;       // warps per CTA of this launch
+  const int kSt = p.n_stages;           // ring stages per warp of this launch
+  const int kWarpBytes = warp_bytes(kSt);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = lane >> 2;              // query head (row of the mma tile)
   const int qp = lane & 3;              // position in the quad
@@ -123,7 +128,7 @@ __global__ void __launch_bounds__(kW * 32, 1)
   const uint32_t base = ((raw + 1023u) & ~1023u) + uint32_t(warp) * kWarpBytes;
   uint8_t* base_ptr = smem_raw + (base - raw);
   float* logc_s = reinterpret_cast<float*>(base_ptr + kSt * kStageBytes);        // [kSt][16]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + kSt * kStageBytes + kSt * kCh * 4);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + kSt * kStageBytes + kMaxSt * kCh * 4);
 
   const int64_t cb = ga & ~int64_t(kCh - 1);              // first chunk, 16-slot aligned
   const int64_t nchunks = (ge - cb + kCh - 1) / kCh;
@@ -247,35 +252,35 @@ __global__ void __launch_bounds__(kW * 32, 1)
     if (ticket != int(w1 - w0)) return;
     __threadfence();
     if (hv) {
-      float Ms[2], Ls[2];
+      // one pass over the records in warp order (online log-sum-exp merge)
+      float Ms[2] = {-INFINITY, -INFINITY}, Ls[2] = {0.f, 0.f};
       float acc[2][32];
 #pragma unroll
-      for (int sg = 0; sg < 2; ++sg) {
-        float mx = -INFINITY;
-        for (int64_t w = w0; w <= w1; ++w) {
-          const float* r = p.partials + (ul + w) * (2 * G * kRec) + (sg * G + h) * kRec;
-          if (__ldcg(r + 1) > 0.f) mx = fmaxf(mx, __ldcg(r));
-        }
-        float L = 0.f;
+      for (int sg = 0; sg < 2; ++sg)
 #pragma unroll
         for (int i = 0; i < 32; ++i) acc[sg][i] = 0.f;
-        if (mx > -INFINITY) {
-#pragma unroll 2
-          for (int64_t w = w0; w <= w1; ++w) {
-            const float* r = p.partials + (ul + w) * (2 * G * kRec) + (sg * G + h) * kRec;
-            const float rl = __ldcg(r + 1);
-            const float sc = rl > 0.f ? exp2f(__ldcg(r) - mx) : 0.f;
-            L += rl * sc;
+      for (int64_t w = w0; w <= w1; ++w) {
+        const float* rr = p.partials + (ul + w) * (2 * G * kRec);
+#pragma unroll
+        for (int sg = 0; sg < 2; ++sg) {
+          const float* r = rr + (sg * G + h) * kRec;
+          const float rm = __ldcg(r), rl = __ldcg(r + 1);
+          float2 v[16];
+#pragma unroll
+          for (int dt = 0; dt < 16; ++dt)
+            v[dt] = __ldcg(reinterpret_cast<const float2*>(r + 4 + dt * 8 + 2 * qp));
+          if (rl > 0.f) {
+            const float mx = fmaxf(Ms[sg], rm);
+            const float sa = exp2f(Ms[sg] - mx), sb = exp2f(rm - mx);
+            Ls[sg] = Ls[sg] * sa + rl * sb;
 #pragma unroll
             for (int dt = 0; dt < 16; ++dt) {
-              const float2 v = __ldcg(reinterpret_cast<const float2*>(r + 4 + dt * 8 + 2 * qp));
-              acc[sg][2 * dt] += v.x * sc;
-              acc[sg][2 * dt + 1] += v.y * sc;
+              acc[sg][2 * dt] = acc[sg][2 * dt] * sa + v[dt].x * sb;
+              acc[sg][2 * dt + 1] = acc[sg][2 * dt + 1] * sa + v[dt].y * sb;
             }
+            Ms[sg] = mx;
           }
         }
-        Ms[sg] = mx;
-        Ls[sg] = L;
       }
       const float g = gate_of(p, Ls[0]);
       float wM = 1.f, wR = 0.f;
@@ -434,31 +439,37 @@ __global__ void __launch_bounds__(kW * 32, 1)
 
 template <int G>
 static cudaError_t launch_mma_g(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
-                                int n_ctas, cudaStream_t stream) {
+                                int n_ctas, int warps_per_cta, cudaStream_t stream) {
   static std::atomic<unsigned long long> configured{0};
-  const int smem = kW * kWarpBytes + 1024;
+  const int smem = warps_per_cta * warp_bytes(p.n_stages) + 1024;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
   const unsigned long long bit = 1ull << (dev & 63);
   if (!(configured.load() & bit)) {
     err = cudaFuncSetAttribute(reskv_decode_mma_kernel<G>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
     if (err != cudaSuccess) return err;
     configured.fetch_or(bit);
   }
-  reskv_decode_mma_kernel<G><<<n_ctas, kW * 32, smem, stream>>>(p, tk, tv);
+  reskv_decode_mma_kernel<G><<<n_ctas, warps_per_cta * 32, smem, stream>>>(p, tk, tv);
   return cudaGetLastError();
 }
 
 cudaError_t launch_decode_mma(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
-                              int group, int n_ctas, cudaStream_t stream) {
+                              int group, int n_ctas, int warps_per_cta, cudaStream_t stream) {
   switch (group) {
-    case 1: return launch_mma_g<1>(p, tk, tv, n_ctas, stream);
-    case 2: return launch_mma_g<2>(p, tk, tv, n_ctas, stream);
-    case 4: return launch_mma_g<4>(p, tk, tv, n_ctas, stream);
+    case 1: return launch_mma_g<1>(p, tk, tv, n_ctas, warps_per_cta, stream);
+    case 2: return launch_mma_g<2>(p, tk, tv, n_ctas, warps_per_cta, stream);
+    case 4: return launch_mma_g<4>(p, tk, tv, n_ctas, warps_per_cta, stream);
     default: return cudaErrorInvalidValue;
   }
+}
+
+// Ring depth for `warps_per_cta` warps sharing one SM's shared memory.
+int decode_mma_stages(int warps_per_cta) {
+  int st = ((kSmemLimit - 1024) / warps_per_cta - 1024) / kStageBytes;
+  return st > kMaxSt ? kMaxSt : st;
 }
 
 size_t decode_mma_partials_floats(int64_t n_units, int n_warps, int group) {

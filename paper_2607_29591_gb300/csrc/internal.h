@@ -38,6 +38,7 @@ struct DecodeParams {
   int32_t budget;
   int32_t n_kv_heads;
   int32_t n_warps;              // W
+  int32_t n_stages;             // ring stages per warp (tensor-core kernel)
   int32_t gate_mode;
   float tau, alpha, g_min, g_fixed;
 };
@@ -49,7 +50,8 @@ cudaError_t launch_decode(const DecodeParams& p, int group, int n_ctas, cudaStre
 size_t decode_partials_floats(int64_t n_units, int n_warps, int group);
 // Launch the tensor-core decode kernel (K/V rows through the given TMA maps).
 cudaError_t launch_decode_mma(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
-                              int group, int n_ctas, cudaStream_t stream);
+                              int group, int n_ctas, int warps_per_cta, cudaStream_t stream);
+int decode_mma_stages(int warps_per_cta);
 size_t decode_mma_partials_floats(int64_t n_units, int n_warps, int group);
 // Slots of zero padding after the log-count array (16-slot chunk copies).
 constexpr int kLogcPad = 16;

@@ -321,23 +321,43 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   p.budget = c->budget;
   p.n_kv_heads = cfg.n_kv_heads;
   p.total_slots = int64_t(p.n_units) * c->budget;
-  // one warp per >= 32 slots, at most a full wave of 8 warps per SM
-  int64_t W = cfg.decode_warps > 0 ? cfg.decode_warps : p.total_slots / 32;
-  if (W > p.total_slots) W = p.total_slots;
+  // Split plan.  CUDA-core kernel: one warp per >= 32 slots, at most 8 warps
+  // per SM.  Tensor-core kernel: one CTA per SM with 1..8 warps so that every
+  // warp streams >= ~200 slots (fewer, longer pieces for small launches, with
+  // a deeper ring in the shared memory that fewer warps leave free).
+  const bool mma = cfg.decode_kernel != RESKV_DECODE_FMA;
+  int64_t W = 0;
+  int wpc = kDecodeWarpsPerCta;
+  if (mma) {
+    if (cfg.decode_warps > 0) {
+      W = cfg.decode_warps;
+    } else {
+      wpc = int(std::min<int64_t>(8, std::max<int64_t>(1, p.total_slots / (int64_t(c->num_sms) * 200))));
+      W = int64_t(c->num_sms) * wpc;
+      if (p.total_slots < W * 32) W = std::max<int64_t>(1, p.total_slots / 32);
+    }
+    if (W > p.total_slots) W = p.total_slots;
+    if (W > c->max_warps) W = c->max_warps;
+    wpc = int(std::min<int64_t>(8, (W + c->num_sms - 1) / c->num_sms));
+  } else {
+    W = cfg.decode_warps > 0 ? cfg.decode_warps : p.total_slots / 32;
+    if (W > p.total_slots) W = p.total_slots;
+    if (W < 1) W = 1;
+    if (W > c->max_warps) W = c->max_warps;
+  }
   if (W < 1) W = 1;
-  if (W > c->max_warps) W = c->max_warps;
   p.n_warps = int32_t(W);
+  p.n_stages = mma ? decode_mma_stages(wpc) : 0;
   p.gate_mode = cfg.gate_mode;
   p.tau = cfg.tau;
   p.alpha = cfg.alpha;
   p.g_min = cfg.g_min;
   p.g_fixed = cfg.g_fixed;
-  const int n_ctas = int((W + kDecodeWarpsPerCta - 1) / kDecodeWarpsPerCta);
   cudaError_t err =
-      cfg.decode_kernel == RESKV_DECODE_FMA
-          ? launch_decode(p, cfg.group, n_ctas, static_cast<cudaStream_t>(stream))
-          : launch_decode_mma(p, c->tmap_k, c->tmap_v, cfg.group, n_ctas,
-                              static_cast<cudaStream_t>(stream));
+      mma ? launch_decode_mma(p, c->tmap_k, c->tmap_v, cfg.group, int((W + wpc - 1) / wpc), wpc,
+                              static_cast<cudaStream_t>(stream))
+          : launch_decode(p, cfg.group, int((W + kDecodeWarpsPerCta - 1) / kDecodeWarpsPerCta),
+                          static_cast<cudaStream_t>(stream));
   if (err != cudaSuccess) return cuda_fail(err, "decode launch");
   return RESKV_OK;
 }
