@@ -164,6 +164,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   int32_t *r_runs = nullptr, *r_final = nullptr, *chosen = nullptr, *run_off_d = nullptr;
   int32_t *cand_r_d = nullptr;
   float *centersT = nullptr, *cnorm = nullptr, *vpart = nullptr, *oS = nullptr;
+  double* centers64 = nullptr;
   __nv_bfloat16 *kbar = nullptr, *vbar = nullptr;
   double *rowerr = nullptr, *losses = nullptr;
   const size_t US = size_t(UL) * size_t(s);
@@ -178,6 +179,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     ok = S.get(&assign, US) && S.get(&hist, size_t(UL) * ntiles * rmax) &&
          S.get(&ccount, size_t(UL) * rmax) && S.get(&cbase, size_t(UL) * rmax) &&
          S.get(&members, US) && S.get(&centersT, size_t(UL) * kHeadDim * rmax) &&
+         S.get(&centers64, size_t(UL) * kHeadDim * rmax) &&
          S.get(&cnorm, size_t(UL) * rmax) && S.get(&kbar, size_t(UL) * ent_stride * kHeadDim) &&
          S.get(&vbar, size_t(UL) * ent_stride * kHeadDim) &&
          S.get(&ecount, size_t(UL) * ent_stride);
@@ -223,8 +225,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   const size_t sm_obs1 = size_t(kHeadDim) * (kTile + kRowBlk) * 4;
   const size_t sm_obs2 = sm_obs1 + size_t(8) * kTile * 4;
   const size_t sm_top = size_t(kTopMax) * 12 + (256 + 32 + 4) * 4;
-  const size_t sm_assign = (size_t(kHeadDim) * (kTile + kRowBlk) + kRowBlk + 8 * kTile) * 4 +
-                           size_t(8) * kTile * 4 + size_t(std::max(rmax, 1)) * 4;
+  const size_t sm_assign = (size_t(kHeadDim) * (kTile + kRowBlk) + kRowBlk + kTile) * 4 +
+                           size_t(8) * kTile * 3 * 4 + size_t(std::max(rmax, 1)) * 4;
   const size_t sm_val = size_t(kHeadDim) * (2 * kTile + 2 * kRowBlk) * 4;
   if (set_smem(k_obs_pass1, sm_obs1) != cudaSuccess || set_smem(k_obs_pass2, sm_obs2) != cudaSuccess ||
       set_smem(k_topk, sm_top) != cudaSuccess || set_smem(k_lloyd_assign, sm_assign) != cudaSuccess ||
@@ -254,8 +256,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     RESKV_LAUNCH_CHECK("ranking");
 
     LloydArgs la{K, V, s, P, n_top, b, ntiles, rmax, top, rank_pos, nullptr, centersT, cnorm,
-                 assign, hist, ccount, cbase, members, kbar, vbar, ecount, ent_stride, 0,
-                 c->status};
+                 centers64, assign, hist, ccount, cbase, members, kbar, vbar, ecount,
+                 ent_stride, 0, c->status};
     auto lloyd_run = [&](const int32_t* r_unit, int ent_off) -> reskv_status {
       la.r_unit = r_unit;
       la.ent_off = ent_off;

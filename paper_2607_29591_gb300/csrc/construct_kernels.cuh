@@ -424,8 +424,9 @@ struct LloydArgs {
   const int32_t* top;          // [UL, n_top]
   const int32_t* rank_pos;     // [UL, s]
   const int32_t* r_unit;       // [UL]
-  float* centersT;             // [UL, d, rmax]  (dim-major)
-  float* cnorm;                // [UL, rmax]
+  float* centersT;             // [UL, d, rmax]  fp32 copy (dim-major) for the fast path
+  float* cnorm;                // [UL, rmax]     ||c||^2 of the fp32 copy
+  double* centers64;           // [UL, rmax, d]  the centres (fp64 means)
   int32_t* assign;             // [UL, s] centre index, -1 outside E
   int32_t* hist;               // [UL, ntiles, rmax] per-tile counts, then offsets
   int32_t* ccount;             // [UL, rmax] members per centre
@@ -455,6 +456,7 @@ __global__ void k_lloyd_init(LloydArgs p) {
   const int32_t pos = p.top[int64_t(ul) * p.n_top + keep + j];
   const float c = __bfloat162float(p.K[(int64_t(ul) * p.s + pos) * kHeadDim + d]);
   p.centersT[(int64_t(ul) * kHeadDim + d) * p.rmax + j] = c;
+  p.centers64[(int64_t(ul) * p.rmax + j) * kHeadDim + d] = double(c);
   red[d] = c * c;
   __syncthreads();
   if (d == 0) {
@@ -464,15 +466,53 @@ __global__ void k_lloyd_init(LloydArgs p) {
   }
 }
 
-// nearest centre of every evicted token of a 128-token tile; per-tile counts
+// Nearest centre of every evicted token of a 128-token tile; per-tile counts.
+//
+// The choice is certified in fp64: distances are first evaluated in fp32
+// (||c||^2 - 2<c,k>, the ||k||^2 term being common) keeping the three best
+// centres per token; a rigorous bound on the fp32 error of each distance
+// (dot products of 128 terms with fused multiply-adds, fp32-rounded centres)
+// decides whether the runner-up could in truth be nearer.  Only then are the
+// candidates re-evaluated as sum_i (k_i - c_i)^2 in fp64 against the fp64
+// centres -- all centres if even the third is within the bound.  Ties go to the
+// lower centre index.
+struct Cand {
+  float d;
+  int j;
+};
+
+__device__ __forceinline__ void cand_insert(Cand* t, float d, int j) {
+  // keeps t[0..2] sorted by (d, j); centres arrive in increasing j per thread
+  if (d < t[2].d || (d == t[2].d && j < t[2].j)) {
+    t[2] = Cand{d, j};
+    if (t[2].d < t[1].d || (t[2].d == t[1].d && t[2].j < t[1].j)) {
+      Cand x = t[1]; t[1] = t[2]; t[2] = x;
+      if (t[1].d < t[0].d || (t[1].d == t[0].d && t[1].j < t[0].j)) {
+        x = t[0]; t[0] = t[1]; t[1] = x;
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ double dist64(const float* Kt, int tok, const double* c) {
+  double acc = 0.0;
+  for (int i = 0; i < kHeadDim; ++i) {
+    const double df = double(Kt[kt_index(i, tok)]) - c[i];
+    acc = fma(df, df, acc);
+  }
+  return acc;
+}
+
 __global__ void __launch_bounds__(kThreads, 2) k_lloyd_assign(LloydArgs p) {
   extern __shared__ __align__(16) float sm[];
   float* Kt = sm;                                   // [128][128]
-  float* Ct = Kt + kHeadDim * kTile;                // [128][32]
+  float* Ct = Kt + kHeadDim * kTile;                // [128][32]; later candidate distances
   float* cn = Ct + kHeadDim * kRowBlk;              // [32]
-  float* bd = cn + kRowBlk;                         // [8][128] best distance per warp
-  int* bj = reinterpret_cast<int*>(bd + 8 * kTile); // [8][128] best centre per warp
-  int* cnt = bj + 8 * kTile;                        // [rmax] tile histogram
+  float* knrm = cn + kRowBlk;                       // [128] ||k|| per token
+  int* cj = reinterpret_cast<int*>(knrm + kTile);   // [8][128][3] candidate centres
+  int* cnt = cj + 8 * kTile * 3;                    // [rmax] tile histogram
+  float* cd = Ct;                                   // [8][128][3] candidate distances
+  __shared__ unsigned int cnmax_bits;               // max ||c||^2 over the unit's centres
   const int tile = blockIdx.x, ul = blockIdx.y;
   const int r = p.r_unit[ul];
   if (r == 0) return;
@@ -480,21 +520,23 @@ __global__ void __launch_bounds__(kThreads, 2) k_lloyd_assign(LloydArgs p) {
   const int64_t tok0 = int64_t(tile) * kTile;
   load_kt(Kt, p.K + int64_t(ul) * p.s * kHeadDim, p.s, tok0);
   for (int i = threadIdx.x; i < r; i += blockDim.x) cnt[i] = 0;
-  float best[4];
-  int bidx[4];
+  if (threadIdx.x == 0) cnmax_bits = 0u;
+  Cand best[4][3];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    best[j] = INFINITY;
-    bidx[j] = 0x7fffffff;
-  }
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int q = 0; q < 3; ++q) best[j][q] = Cand{INFINITY, 0x7fffffff};
   for (int cb = 0; cb < r; cb += kRowBlk) {
     __syncthreads();
     for (int idx = threadIdx.x; idx < kHeadDim * kRowBlk; idx += blockDim.x) {
       const int k = idx / kRowBlk, c = idx % kRowBlk;
       Ct[idx] = (cb + c < r) ? p.centersT[(int64_t(ul) * kHeadDim + k) * p.rmax + cb + c] : 0.f;
     }
-    if (threadIdx.x < kRowBlk)
-      cn[threadIdx.x] = (cb + threadIdx.x < r) ? p.cnorm[int64_t(ul) * p.rmax + cb + threadIdx.x] : 0.f;
+    if (threadIdx.x < kRowBlk) {
+      const float v = (cb + threadIdx.x < r) ? p.cnorm[int64_t(ul) * p.rmax + cb + threadIdx.x] : 0.f;
+      cn[threadIdx.x] = v;
+      atomicMax(&cnmax_bits, __float_as_uint(v));   // non-negative: bit order = value order
+    }
     __syncthreads();
     float S[4][4];
     tile_logits(Ct, Kt, S);                         // <c_i, k_j> for centres 4w+i
@@ -503,42 +545,85 @@ __global__ void __launch_bounds__(kThreads, 2) k_lloyd_assign(LloydArgs p) {
       const int c = cb + 4 * w + i;
       if (c >= r) continue;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float dist = cn[4 * w + i] - 2.0f * S[i][j];   // ||c||^2 - 2<c,k> (+||k||^2)
-        if (dist < best[j]) {                                 // strict: lower index kept
-          best[j] = dist;
-          bidx[j] = c;
-        }
-      }
+      for (int j = 0; j < 4; ++j) cand_insert(best[j], cn[4 * w + i] - 2.0f * S[i][j], c);
     }
   }
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    bd[w * kTile + 4 * lane + j] = best[j];
-    bj[w * kTile + 4 * lane + j] = bidx[j];
+  __syncthreads();                                  // Ct is reused for the candidates
+  if (threadIdx.x < kTile) {                        // ||k|| of token threadIdx.x
+    float n = 0.f;
+    for (int i = 0; i < kHeadDim; ++i) {
+      const float x = Kt[kt_index(i, threadIdx.x)];
+      n = fmaf(x, x, n);
+    }
+    knrm[threadIdx.x] = sqrtf(n);
   }
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+      const int o = (w * kTile + 4 * lane + j) * 3 + q;
+      cd[o] = best[j][q].d;
+      cj[o] = best[j][q].j;
+    }
   __syncthreads();
   if (threadIdx.x < kTile) {
     const int t = threadIdx.x;
-    float b0 = bd[t];
-    int j0 = bj[t];
-    for (int ww = 1; ww < 8; ++ww) {
-      const float b1 = bd[ww * kTile + t];
-      const int j1 = bj[ww * kTile + t];
-      if (b1 < b0 || (b1 == b0 && j1 < j0)) {
-        b0 = b1;
-        j0 = j1;
-      }
-    }
     const int64_t pos = tok0 + t;
-    if (pos < p.s) {
-      bool ev = in_evicted(p, ul, pos, r);
-      if (ev && (j0 < 0 || j0 >= r)) {        // only a NaN distance gets here
+    if (pos < p.s && in_evicted(p, ul, pos, r)) {
+      Cand top[3] = {{INFINITY, 0x7fffffff}, {INFINITY, 0x7fffffff}, {INFINITY, 0x7fffffff}};
+      for (int ww = 0; ww < 8; ++ww)
+        for (int q = 0; q < 3; ++q) {
+          const int o = (ww * kTile + t) * 3 + q;
+          if (cj[o] < r) cand_insert(top, cd[o], cj[o]);
+        }
+      // Bound on the fp32 error of d_j = ||c_j||^2 - 2<c_j, k> for any centre:
+      // 128-term fused dot product (gamma ~ 130 u), fp32 rounding of the fp64
+      // centre (u per coordinate), the norm sum and the final subtraction,
+      // with ||c_j|| <= max ||c||, times a safety factor 2.  A centre outside
+      // the fp32 top three lies at least d_3 - d_1 above the best in fp32.
+      const float gam = 130.0f * 5.9604645e-8f, u = 5.9604645e-8f;
+      const float kn = knrm[t];
+      const float cm = sqrtf(__uint_as_float(cnmax_bits));
+      float err[3];
+      int n_amb = 1;
+#pragma unroll
+      for (int q = 0; q < 3; ++q)
+        err[q] = 2.0f * (2.0f * gam * cm * kn + 2.0f * gam * cm * cm + 4.0f * u * kn * cm +
+                         2.0f * u * fabsf(top[q].d));
+      for (int q = 1; q < 3; ++q)
+        if (top[q].j < r && top[q].d - top[0].d <= err[0] + err[q]) n_amb = q + 1;
+      int j0 = top[0].j;
+      if (j0 >= r) {                                  // only a NaN distance gets here
         report_status(p.status, kStatusBadIndex);
         j0 = 0;
+      } else if (n_amb > 1) {
+        const double* c64 = p.centers64 + int64_t(ul) * p.rmax * kHeadDim;
+        double bd = INFINITY;
+        int bj = j0;
+        if (n_amb < 3) {
+          for (int q = 0; q < n_amb; ++q) {
+            const int j = top[q].j;
+            const double dd = dist64(Kt, t, c64 + int64_t(j) * kHeadDim);
+            if (dd < bd || (dd == bd && j < bj)) {
+              bd = dd;
+              bj = j;
+            }
+          }
+        } else {                                      // three or more within the bound
+          for (int j = 0; j < r; ++j) {
+            const double dd = dist64(Kt, t, c64 + int64_t(j) * kHeadDim);
+            if (dd < bd) {
+              bd = dd;
+              bj = j;
+            }
+          }
+        }
+        j0 = bj;
       }
-      p.assign[int64_t(ul) * p.s + pos] = ev ? j0 : -1;
-      if (ev) atomicAdd(&cnt[j0], 1);
+      p.assign[int64_t(ul) * p.s + pos] = j0;
+      atomicAdd(&cnt[j0], 1);
+    } else if (pos < p.s) {
+      p.assign[int64_t(ul) * p.s + pos] = -1;
     }
   }
   __syncthreads();
@@ -649,12 +734,14 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_update(LloydArgs p, int fina
       tv += redv[ww][d];
     }
     float* cptr = p.centersT + (int64_t(ul) * kHeadDim + d) * p.rmax + j;
+    double* c64 = p.centers64 + (int64_t(ul) * p.rmax + j) * kHeadDim + d;
     double mk;
     if (cnt > 0) {
       mk = tk / double(cnt);
+      *c64 = mk;
       *cptr = float(mk);
     } else {
-      mk = double(*cptr);              // an empty cluster keeps its centre
+      mk = *c64;                        // an empty cluster keeps its centre
     }
     const float c = *cptr;
     nrm[d] = c * c;
