@@ -309,10 +309,11 @@ def build_workload(w: wl.Workload, n_q: int, device, decode_kernel: int):
 
 def main():
     args = parse_args()
-    world, rank, local = dist_setup()
     if args.impl == "reference":
-        run_reference(args, world, rank)
+        # the CPU oracle needs no process group: rank 0 runs, the others exit
+        run_reference(args, int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")))
         return
+    world, rank, local = dist_setup()
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")
     from paper_2607_29591_gb300 import build as B
