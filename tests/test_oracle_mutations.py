@@ -1,0 +1,228 @@
+"""Plant plausible mistakes in the oracle (on the CPU) and check that the pins
+of tests/test_oracle_pins.py catch every one of them.
+
+Each mutant replaces one oracle function with a version carrying a single
+mistake of the kind that slips into a restatement of the paper: a dropped
+term, a wrong sign, scale or index, a tie broken the other way, a missing
+normalisation.  A mutant survives if every pin still passes; none may.
+"""
+import contextlib
+import inspect
+
+import numpy as np
+import pytest
+
+import oracle
+import oracle.reskv_oracle as core
+import test_oracle_pins as pins
+
+
+@contextlib.contextmanager
+def patched(name, fn):
+    """Replace `name` in the oracle module and in the package re-export."""
+    old = getattr(core, name)
+    setattr(core, name, fn)
+    setattr(oracle, name, fn)
+    try:
+        yield
+    finally:
+        setattr(core, name, old)
+        setattr(oracle, name, old)
+
+
+def pin_functions():
+    return [f for n, f in inspect.getmembers(pins, inspect.isfunction)
+            if n.startswith("test_") and not inspect.signature(f).parameters]
+
+
+def caught(name, fn):
+    """True if at least one pin's assertion fails with the mutant in place
+    (an error of another kind would not show that the pin checks anything)."""
+    with patched(name, fn):
+        for f in pin_functions():
+            try:
+                with np.errstate(all="ignore"):
+                    f()
+            except AssertionError:
+                return True
+    return False
+
+
+_orig = {n: getattr(core, n) for n in dir(core) if not n.startswith("_")}
+
+
+def _logits_over_d(q, K):
+    return (K @ q) / K.shape[-1]
+
+
+def _decode_drop_logc(q, Km, Vm, Kr, Vr, logc, cfg, return_stats=False):
+    return _orig["shared_softmax_decode"](q, Km, Vm, Kr, Vr, np.zeros_like(logc), cfg, return_stats)
+
+
+def _gate_wrong_sign(p_max, tau, alpha, g_min):
+    return max(g_min, core.sigmoid(alpha * (p_max - tau)))
+
+
+def _gate_temperature(p_max, tau, alpha, g_min):
+    return max(g_min, core.sigmoid((tau - p_max) / alpha))
+
+
+def _decode_residual_numerator_only(q, Km, Vm, Kr, Vr, logc, cfg, return_stats=False):
+    a = core.logits(q, Km)
+    mu = a.max()
+    e = np.exp(a - mu)
+    p_max = 1.0 / e.sum()
+    g = core.dynamic_gate(p_max, cfg.tau, cfg.alpha, cfg.g_min) if cfg.gate_mode == 0 else cfg.g_fixed
+    at = core.logits(q, Kr) + logc + (np.log(g) if g > 0 else -np.inf) if Kr.shape[0] else np.zeros(0)
+    wr = np.exp(at - mu)
+    out = (e @ Vm + (wr @ Vr if Kr.shape[0] else 0.0)) / e.sum()       # Z^ misses the residual
+    if return_stats:
+        return out, dict(p_max=p_max, g=g, Z=e.sum(), N=e @ Vm, shift=mu)
+    return out
+
+
+def _decode_gate_on_main(q, Km, Vm, Kr, Vr, logc, cfg, return_stats=False):
+    # the gate applied to the main branch instead of the residual one
+    a = core.logits(q, Km)
+    mu = a.max()
+    p_max = 1.0 / np.exp(a - mu).sum()
+    g = core.dynamic_gate(p_max, cfg.tau, cfg.alpha, cfg.g_min) if cfg.gate_mode == 0 else cfg.g_fixed
+    lg = np.log(g) if g > 0 else -np.inf
+    at = core.logits(q, Kr) + logc if Kr.shape[0] else np.zeros(0)
+    allv = np.concatenate([a + lg, at])
+    m = np.max(allv[np.isfinite(allv)])
+    w = np.exp(allv - m)
+    V = np.concatenate([Vm, Vr]) if Kr.shape[0] else Vm
+    out = (w @ V) / w.sum()
+    if return_stats:
+        return out, dict(p_max=p_max, g=g, Z=w.sum(), N=w @ V, shift=m)
+    return out
+
+
+def _scores_no_head_average(K, Qfit, pool):
+    return _orig["scores_obs_pool"](K, Qfit, pool) * Qfit.shape[0]
+
+
+def _scores_edge_normalised(K, Qfit, pool):
+    out = _orig["scores_obs_pool"](K, Qfit, pool)
+    s, h = K.shape[0], pool // 2
+    n = np.array([min(p + h, s - 1) - max(p - h, 0) + 1 for p in range(s)], dtype=float)
+    return out * pool / n
+
+
+def _scores_no_softmax(K, Qfit, pool):
+    G, n_fit, _ = Qfit.shape
+    acc = np.zeros(K.shape[0])
+    for g in range(G):
+        for t in range(n_fit):
+            acc += np.exp(core.logits(Qfit[g, t], K)) / G
+    padded = np.concatenate([np.zeros(pool // 2), acc, np.zeros(pool // 2)])
+    return sum(padded[j:j + K.shape[0]] for j in range(pool)) / pool
+
+
+def _rank_ties_high(scores, recent):
+    n = max(scores.shape[0] - recent, 0)
+    pos = np.arange(n)
+    return pos[np.lexsort((-pos, -scores[:n]))]
+
+
+def _rank_includes_recent(scores, recent):
+    return _orig["rank_evictable"](scores, 0)[: max(scores.shape[0] - recent, 0)]
+
+
+def _select_off_by_one(ranked, s, recent, m):
+    M, E = _orig["select_main"](ranked, s, recent, m + 1)
+    return M, E
+
+
+def _lloyd_init_low(K, V, E, r, iters):
+    return _orig["lloyd_residual"](K, V, np.concatenate([E[r:], E[:r]]) if len(E) > r else E, r, iters)
+
+
+def _lloyd_one_iteration(K, V, E, r, iters):
+    return _orig["lloyd_residual"](K, V, E, r, 1)
+
+
+def _assign_ties_high(KE, centers):
+    d = np.sum(centers * centers, axis=1)[None, :] - 2.0 * (KE @ centers.T)
+    return centers.shape[0] - 1 - np.argmin(d[:, ::-1], axis=1)
+
+
+def _assign_no_norm(KE, centers):
+    return np.argmax(KE @ centers.T, axis=1)
+
+
+def _choose_r_non_strict(L0, rs, losses, delta):
+    if len(rs) == 0:
+        return 0
+    i = int(np.argmin(losses))
+    return rs[i] if losses[i] <= (1.0 - delta) * L0 else 0
+
+
+def _choose_r_largest_on_tie(L0, rs, losses, delta):
+    if len(rs) == 0:
+        return 0
+    order = sorted(range(len(rs)), key=lambda i: (losses[i], -rs[i]))
+    best = order[0]
+    return rs[best] if losses[best] < (1.0 - delta) * L0 else 0
+
+
+def _round_truncate(x):
+    x = np.asarray(x, dtype=np.float64)
+    mant, expo = np.frexp(x)
+    return np.ldexp(np.trunc(np.ldexp(mant, 8)), expo - 8)
+
+
+def _logc_plus_one(counts, beta):
+    return beta * np.log(counts.astype(np.float64) + 1.0)
+
+
+def _keynorm_abs(K):
+    return np.sum(np.abs(K), axis=1)
+
+
+def _val_loss_no_mean(cache, Qval, O_full, cfg):
+    return _orig["validation_loss"](cache, Qval, O_full, cfg) * Qval.shape[0] * Qval.shape[1]
+
+
+def _attention_full_no_shift(q, K, V):
+    a = core.logits(q, K)
+    w = np.exp(a)
+    return (w @ V) / (w.sum() + 1.0)
+
+
+MUTANTS = [
+    ("logits", _logits_over_d),
+    ("shared_softmax_decode", _decode_drop_logc),
+    ("shared_softmax_decode", _decode_residual_numerator_only),
+    ("shared_softmax_decode", _decode_gate_on_main),
+    ("dynamic_gate", _gate_wrong_sign),
+    ("dynamic_gate", _gate_temperature),
+    ("scores_obs_pool", _scores_no_head_average),
+    ("scores_obs_pool", _scores_edge_normalised),
+    ("scores_obs_pool", _scores_no_softmax),
+    ("rank_evictable", _rank_ties_high),
+    ("rank_evictable", _rank_includes_recent),
+    ("select_main", _select_off_by_one),
+    ("lloyd_residual", _lloyd_init_low),
+    ("lloyd_residual", _lloyd_one_iteration),
+    ("lloyd_assign", _assign_ties_high),
+    ("lloyd_assign", _assign_no_norm),
+    ("choose_r", _choose_r_non_strict),
+    ("choose_r", _choose_r_largest_on_tie),
+    ("round_to_bf16", _round_truncate),
+    ("log_counts", _logc_plus_one),
+    ("scores_keynorm", _keynorm_abs),
+    ("validation_loss", _val_loss_no_mean),
+    ("attention_full", _attention_full_no_shift),
+]
+
+
+@pytest.mark.parametrize("name,fn", MUTANTS, ids=[f"{n}:{f.__name__}" for n, f in MUTANTS])
+def test_pins_catch_planted_mistake(name, fn):
+    assert caught(name, fn), f"no pin fails when {name} carries the mistake {fn.__name__}"
+
+
+def test_unmutated_oracle_passes_every_pin():
+    for f in pin_functions():
+        f()
