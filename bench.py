@@ -50,8 +50,9 @@ def parse_args():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(wl.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-per-layer", action="store_true")
-    ap.add_argument("--decode-kernel", choices=["mma", "fma"], default="mma",
-                    help="tensor-core (default) or CUDA-core decode kernel")
+    ap.add_argument("--decode-kernel", choices=["auto", "mma", "cluster", "fma"], default="auto",
+                    help="automatic plan (default: cluster kernel for launches whose units "
+                         "fit on the device at once, else tensor-core stream-K), or one kernel")
     ap.add_argument("--layers", type=int, default=0,
                     help="use only this many layers (smaller profiling case)")
     return ap.parse_args()
@@ -325,8 +326,18 @@ def main():
     if args.layers:
         w = wl.scaled(w, n_layers=args.layers, name=f"{w.name}_{args.layers}l")
     n_q = args.steps + args.warmup
-    kern = R.RESKV_DECODE_MMA if args.decode_kernel == "mma" else R.RESKV_DECODE_FMA
+    kern = {"auto": R.RESKV_DECODE_AUTO, "mma": R.RESKV_DECODE_MMA,
+            "cluster": R.RESKV_DECODE_CLUSTER, "fma": R.RESKV_DECODE_FMA}[args.decode_kernel]
     cache, Qdec, build_s = build_workload(w, n_q, device, kern)
+    info = R.reskv_get_info(cache)
+
+    def plan_name(cs, wpc):
+        if cs == 0:
+            return "fma" if kern == R.RESKV_DECODE_FMA else "tensor-core stream-K"
+        return f"tensor-core cluster: {cs} CTA(s) x {wpc} warps per unit"
+
+    decode_plan = {"all_layer": plan_name(info["all_cluster"], info["all_cluster_warps"]),
+                   "per_layer": plan_name(info["layer_cluster"], info["layer_cluster_warps"])}
     lay_meta = R.reskv_export_cache(cache)
     alg = algorithmic_bytes(lay_meta["n_main"], lay_meta["n_res"])
     r_counts = lay_meta["n_res"]
@@ -430,6 +441,7 @@ def main():
                        "mean_r": float(np.mean(r_counts)),
                        "units_with_residual": float(np.mean(r_counts > 0)),
                        "launch": "one reskv_decode_attn(layer=-1) launch per step",
+                       "decode_plan": decode_plan,
                        "l2": f"inputs larger than L2: {alg / 1e9:.2f} GB of cache read per step",
                        "parallelism": "replicas" if world > 1 else "single GPU"},
             "hbm_gbs": achieved, "frac_of_peak": achieved / peak,

@@ -48,7 +48,7 @@ typedef enum {
 
 enum { RESKV_SCORE_OBS_POOL = 0, RESKV_SCORE_KEYNORM = 1 };
 enum { RESKV_GATE_DYNAMIC = 0, RESKV_GATE_FIXED = 1 };
-enum { RESKV_DECODE_AUTO = 0, RESKV_DECODE_FMA = 1, RESKV_DECODE_MMA = 2 };
+enum { RESKV_DECODE_AUTO = 0, RESKV_DECODE_FMA = 1, RESKV_DECODE_MMA = 2, RESKV_DECODE_CLUSTER = 3 };
 
 #define RESKV_MAX_GRID 8
 
@@ -92,8 +92,13 @@ typedef struct reskv_config {
                               pieces (one warp each) a decode call cuts its
                               slot range into, capped at 8 warps per SM; the
                               result does not depend on it beyond rounding   */
-  int32_t decode_kernel;   /* RESKV_DECODE_*: 0 automatic (tensor cores),
-                              1 CUDA-core fp32x2 FMA, 2 tensor-core mma.sync  */
+  int32_t decode_kernel;   /* RESKV_DECODE_*: 0 automatic (tensor cores:
+                              cluster kernel when a launch's units fit on the
+                              device in one wave and decode_warps is 0, else
+                              stream-K), 1 CUDA-core fp32x2 FMA, 2 tensor-core
+                              stream-K over the launch's slot range, 3
+                              tensor-core with one thread-block cluster of 1..8
+                              CTAs per unit (decode_warps ignored)           */
 } reskv_config;
 
 /* Fill *cfg with the paper's defaults; shape fields are zeroed. */
@@ -151,6 +156,11 @@ typedef struct reskv_cache_info {
   int32_t head_dim;
   int64_t slot_bytes;      /* bytes of one K row + one V row                 */
   int64_t cache_bytes;     /* device bytes of K/V slots + log-counts         */
+  int32_t layer_cluster;   /* CTAs per unit of an automatic one-layer decode
+                              launch (cluster kernel); 0: stream-K kernel     */
+  int32_t layer_cluster_warps; /* warps per CTA of that cluster launch       */
+  int32_t all_cluster;     /* the same for an all-layer launch (layer = -1)  */
+  int32_t all_cluster_warps;
 } reskv_cache_info;
 
 reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info);

@@ -1,0 +1,429 @@
+// Shared-softmax residual decode (Alg. 2; Sec. 5.4 Eqs. residual_logit,
+// reskv_den, reskv_num, reskv; Sec. 5.5.2 Eq. gate) on the tensor cores, one
+// thread-block cluster per unit.
+//
+// The stream-K kernel (decode_mma.cu) cuts a launch's whole slot range into
+// equal warp pieces.  When a launch holds few units -- one layer of a decode
+// step, a few dozen (batch, KV head) units -- nearly every unit is then cut
+// between many warps, and merging their partial results through global
+// records and an arrival ticket costs more than streaming the unit.  Here a
+// unit is given to a cluster of CS CTAs (CS = 1..8) on as many SMs; the
+// cluster's CS x kW warps each stream an equal run of the unit's 16-slot
+// chunks with the tile step of mma_tile.cuh, and the partial results never
+// leave the chip:
+//
+//   1. every warp writes its record (per query head and branch: running max,
+//      sum, numerator) into its own, drained, ring buffer;
+//   2. after a CTA barrier, the CTA's threads merge its warps' records in
+//      warp order and store the CTA record into rank 0's shared memory
+//      (distributed shared memory, slot = rank);
+//   3. after one cluster barrier, rank 0 merges the CS CTA records in rank
+//      order, applies the gate and writes o^; the other CTAs are done.
+//
+// A cluster barrier phase opened at the start (arrive) and closed before the
+// first remote store (wait) makes sure rank 0 is running before it is written.
+// Launches are programmatic dependent launches: a kernel streams its first
+// ring of cache chunks while the previous kernel on the stream finishes, and
+// waits for it before touching Q or O.
+// The result does not depend on timing: both merges run in a fixed order.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cmath>
+#include <cstdint>
+
+#include "device_utils.cuh"
+#include "internal.h"
+#include "mma_tile.cuh"
+
+namespace reskv {
+namespace {
+
+constexpr int kMaxCluster = 8;                              // portable cluster size
+constexpr int kCtaRecFloats = 2 * 4 * kRec;                // 2 branches x G <= 4 heads
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_size() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+
+// Every thread of every CTA of the cluster arrives; shared-memory writes
+// before it are visible to every thread of the cluster after it.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile(
+      "barrier.cluster.arrive.release.aligned;\n\t"
+      "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// The two halves of a cluster barrier phase with no memory ordering: after
+// the wait, every CTA of the cluster has started.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+}
+
+// Store into the shared memory of CTA `rank` of the cluster, at the address
+// that `local` has in this CTA.
+__device__ __forceinline__ uint32_t map_rank(uint32_t local, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(rank));
+  return remote;
+}
+
+__device__ __forceinline__ void st_cluster(uint32_t local, uint32_t rank, float4 v) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(map_rank(local, rank)),
+               "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
+
+__device__ __forceinline__ void st_cluster(uint32_t local, uint32_t rank, float2 v) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(map_rank(local, rank)), "f"(v.x),
+               "f"(v.y)
+               : "memory");
+}
+
+template <int G>
+__global__ void __launch_bounds__(kMmaMaxW * 32, 1)
+    reskv_decode_cluster_kernel(const DecodeParams p, const __grid_constant__ CUtensorMap tmK,
+                                const __grid_constant__ CUtensorMap tmV) {
+  extern __shared__ uint8_t smem_raw[];
+  const int kW = blockDim.x >> 5;       // warps per CTA of this launch
+  const int kSt = p.n_stages;           // ring stages per warp of this launch
+  const int kWarpBytes = warp_bytes(kSt);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = lane >> 2;              // query head (row of the mma tile)
+  const int qp = lane & 3;              // position in the quad
+  const bool hv = h < G;
+  const uint32_t cs = cluster_size(), rank = cluster_rank();
+
+  // this cluster's unit, slots [ub, ub + b).  Slot indices fit in 32 bits
+  // (a cache holds fewer than 2^31 slots), so no 64-bit division is needed.
+  const int ul = int(blockIdx.x / cs);
+  const int u = int(p.unit0) + ul;
+  const int b = p.budget;
+  const int ub = u * b;
+  // the 16-slot chunks (aligned to 16 global slots) of the unit's whole slot
+  // range, split evenly over the cluster's warps.  The split does not wait for
+  // n_main / n_res: the first copies are in flight before those loads return
+  // (unused tail slots, present only when s < b, are streamed and masked).
+  const int cb = ub & ~(kCh - 1);
+  const int nch = (ub + b - cb + kCh - 1) / kCh;
+  const int NW = int(cs) * kW, iw = int(rank) * kW + warp;
+  const int k0 = (iw * nch) / NW, k1 = ((iw + 1) * nch) / NW;
+  const int nchunks = k1 - k0;
+  const int wcb = cb + k0 * kCh;                           // first row of this warp's run
+
+  // per-warp shared memory, 1024-byte aligned for the 128-byte swizzle
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t abase = (raw + 1023u) & ~1023u;
+  uint8_t* abase_ptr = smem_raw + (abase - raw);
+  const uint32_t base = abase + uint32_t(warp) * kWarpBytes;
+  uint8_t* base_ptr = abase_ptr + warp * kWarpBytes;
+  float* logc_s = reinterpret_cast<float*>(base_ptr + warp_logc_offset(kSt));   // [kSt][16]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + warp_bars_offset(kSt));
+  // CTA records [cs][2][G][kRec] after the rings (read only in rank 0)
+  float* crec = reinterpret_cast<float*>(abase_ptr + kW * kWarpBytes);
+  const uint32_t crec_s = abase + uint32_t(kW * kWarpBytes);
+
+  cluster_arrive_relaxed();             // closed by cluster_wait() before step 2
+  if (lane == 0) {
+    for (int s = 0; s < kSt; ++s) mbar_init(&bars[s], 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+
+  auto issue = [&](int k, int s) {     // lane 0: chunk k into stage s
+    const int row = wcb + k * kCh;
+    const uint32_t st = base + s * kStageBytes;
+    mbar_arrive_expect_tx(&bars[s], kStageBytes + kCh * 4);
+    tma_load_2d(st, &tmK, 0, row, &bars[s]);
+    tma_load_2d(st + kBox, &tmK, 64, row, &bars[s]);
+    tma_load_2d(st + 2 * kBox, &tmV, 0, row, &bars[s]);
+    tma_load_2d(st + 3 * kBox, &tmV, 64, row, &bars[s]);
+    bulk_g2s(logc_s + s * kCh, p.logc + row, kCh * 4, &bars[s]);
+  };
+  const int issued0 = nchunks < kSt ? nchunks : kSt;
+  if (lane == 0)
+    for (int k = 0; k < issued0; ++k) issue(k, k);
+  // Programmatic dependent launch: the next kernel on the stream may start
+  // now (its own prologue and cache copies overlap this kernel's tail) ...
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+  const int nm = p.n_main[u], nr = p.n_res[u];
+  const int ue = ub + nm + nr;                             // used slots [ub, ue)
+  uint32_t off_qk[4], off_pv[8];
+  tile_offsets(lane, off_qk, off_pv);
+  const float qscale = kLog2e * rsqrtf(float(kHeadDim));
+  const int64_t orow0 = int64_t(ul / p.n_kv_heads) * p.n_kv_heads * G + (ul % p.n_kv_heads) * G;
+  uint32_t qa[16];
+  // ... and this kernel reads Q and writes O only after the previous kernel
+  // has completed and its memory is visible.  Before this point it reads
+  // only the cache (K, V, log-counts, n_main, n_res), which no kernel that
+  // may run concurrently writes.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  load_q_frag(p.Q, orow0 + h, hv, qp, qa);
+
+  TileState S;
+  S.reset();
+  int issued = issued0;                 // chunks [0, issued) requested
+  int waited = 0;                       // chunks [0, waited) completed
+  int s = 0;                            // stage of chunk k
+  uint32_t phase = 0;                   // parity of its current use
+  for (int k = 0; k < nchunks; ++k) {
+    if (!mbar_wait_bounded(&bars[s], phase)) {
+      if (lane == 0) report_status(p.status, kStatusWaitTimeout);
+      break;
+    }
+    waited = k + 1;
+    tile_update(S, base + s * kStageBytes, logc_s + s * kCh, wcb + k * kCh, ub, ub + nm, ub + nm,
+                ue, qa, off_qk, off_pv, qscale, hv, qp);
+    __syncwarp();
+    if (k + kSt < nchunks) {
+      if (lane == 0) {
+        fence_proxy_async_smem();
+        issue(k + kSt, s);
+      }
+      issued = k + kSt + 1;
+    }
+    if (++s == kSt) {
+      s = 0;
+      phase ^= 1u;
+    }
+  }
+  // never reuse the ring while a copy is in flight into it (bounded waits)
+  for (int kk = waited; kk < issued; ++kk)
+    mbar_wait_bounded(&bars[kk % kSt], uint32_t((kk / kSt) & 1));
+  __syncwarp();
+
+  // 1. this warp's record, in the first bytes of its own ring
+  float lMt = S.lM + __shfl_xor_sync(0xffffffffu, S.lM, 1);
+  lMt += __shfl_xor_sync(0xffffffffu, lMt, 2);
+  float lRt = S.lR + __shfl_xor_sync(0xffffffffu, S.lR, 1);
+  lRt += __shfl_xor_sync(0xffffffffu, lRt, 2);
+  if (hv) {
+    float* rm = reinterpret_cast<float*>(base_ptr) + (0 * G + h) * kRec;
+    float* rr = reinterpret_cast<float*>(base_ptr) + (1 * G + h) * kRec;
+    if (qp == 0) {
+      rm[0] = S.mM;
+      rm[1] = lMt;
+      rr[0] = S.mR;
+      rr[1] = lRt;
+    }
+#pragma unroll
+    for (int dt = 0; dt < 16; ++dt) {
+      *reinterpret_cast<float2*>(rm + 4 + dt * 8 + 2 * qp) = make_float2(S.O[dt][0], S.O[dt][1]);
+      *reinterpret_cast<float2*>(rr + 4 + dt * 8 + 2 * qp) = make_float2(S.O[dt][2], S.O[dt][3]);
+    }
+  }
+  __syncthreads();
+  cluster_wait();                        // every CTA of the cluster is running
+
+  // 2. CTA record: merge the kW warp records in warp order; a thread takes
+  //    four dims of one (branch, head) record and issues all of its loads
+  //    before the first use.  The record goes straight into slot `rank` of
+  //    rank 0's CTA records (distributed shared memory).
+  for (int idx = threadIdx.x; idx < 2 * G * (kHeadDim / 4); idx += blockDim.x) {
+    const int rec = idx / (kHeadDim / 4), d4 = 4 * (idx % (kHeadDim / 4));
+    float2 ml[kMmaMaxW];
+    float4 ac[kMmaMaxW];
+#pragma unroll
+    for (int w = 0; w < kMmaMaxW; ++w) {
+      const int ws = w < kW ? w : 0;           // in-range address; weight masked below
+      const float* r = reinterpret_cast<const float*>(abase_ptr + ws * kWarpBytes) + rec * kRec;
+      ml[w] = *reinterpret_cast<const float2*>(r);
+      ac[w] = *reinterpret_cast<const float4*>(r + 4 + d4);
+    }
+    float mx = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kMmaMaxW; ++w)
+      if (w < kW && ml[w].y > 0.f) mx = fmaxf(mx, ml[w].x);
+    float l = 0.f;
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int w = 0; w < kMmaMaxW; ++w)
+      if (w < kW && ml[w].y > 0.f) {
+        const float sc = exp2f(ml[w].x - mx);
+        l += ml[w].y * sc;
+        a.x += ac[w].x * sc;
+        a.y += ac[w].y * sc;
+        a.z += ac[w].z * sc;
+        a.w += ac[w].w * sc;
+      }
+    const uint32_t dst = crec_s + uint32_t(rank * kCtaRecFloats + rec * kRec) * 4u;
+    st_cluster(dst + uint32_t(4 + d4) * 4u, 0, a);
+    if (d4 == 0) st_cluster(dst, 0, make_float2(mx, l));
+  }
+  cluster_sync();
+  if (rank != 0) return;                 // nobody reads this CTA's shared memory
+
+  // 3. rank 0: merge the CS CTA records in rank order, gate, write o^
+  for (int idx = threadIdx.x; idx < G * (kHeadDim / 4); idx += blockDim.x) {
+    const int hh = idx / (kHeadDim / 4), d4 = 4 * (idx % (kHeadDim / 4));
+    float2 ml[2][kMaxCluster];
+    float4 ac[2][kMaxCluster];
+#pragma unroll
+    for (int sg = 0; sg < 2; ++sg)
+#pragma unroll
+      for (int c = 0; c < kMaxCluster; ++c) {
+        const int cc = c < int(cs) ? c : 0;
+        const float* r = crec + cc * kCtaRecFloats + (sg * G + hh) * kRec;
+        ml[sg][c] = *reinterpret_cast<const float2*>(r);
+        ac[sg][c] = *reinterpret_cast<const float4*>(r + 4 + d4);
+      }
+    float Ms[2], Ls[2];
+    float4 As[2];
+#pragma unroll
+    for (int sg = 0; sg < 2; ++sg) {
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < kMaxCluster; ++c)
+        if (c < int(cs) && ml[sg][c].y > 0.f) mx = fmaxf(mx, ml[sg][c].x);
+      float l = 0.f;
+      float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int c = 0; c < kMaxCluster; ++c)
+        if (c < int(cs) && ml[sg][c].y > 0.f) {
+          const float sc = exp2f(ml[sg][c].x - mx);
+          l += ml[sg][c].y * sc;
+          a.x += ac[sg][c].x * sc;
+          a.y += ac[sg][c].y * sc;
+          a.z += ac[sg][c].z * sc;
+          a.w += ac[sg][c].w * sc;
+        }
+      Ms[sg] = mx;
+      Ls[sg] = l;
+      As[sg] = a;
+    }
+    const float g = gate_of(p, Ls[0]);
+    float wM = 1.f, wR = 0.f;
+    if (Ls[1] > 0.f && g > 0.f) {
+      const float mx = fmaxf(Ms[0], Ms[1]);
+      wM = exp2f(Ms[0] - mx);
+      wR = g * exp2f(Ms[1] - mx);
+    }
+    const float inv = 1.0f / (wM * Ls[0] + wR * Ls[1]);
+    *reinterpret_cast<float4*>(p.O + (orow0 + hh) * kHeadDim + d4) =
+        make_float4((wM * As[0].x + wR * As[1].x) * inv, (wM * As[0].y + wR * As[1].y) * inv,
+                    (wM * As[0].z + wR * As[1].z) * inv, (wM * As[0].w + wR * As[1].w) * inv);
+  }
+}
+
+}  // namespace
+
+template <int G>
+static cudaError_t configure_cluster_g() {
+  static std::atomic<unsigned long long> configured{0};
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (!(configured.load() & bit)) {
+    err = cudaFuncSetAttribute(reskv_decode_cluster_kernel<G>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
+    if (err != cudaSuccess) return err;
+    configured.fetch_or(bit);
+  }
+  return cudaSuccess;
+}
+
+template <int G>
+static cudaLaunchConfig_t cluster_config(int64_t n_units, int cluster, int warps_per_cta,
+                                         cudaStream_t stream, cudaLaunchAttribute* attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(n_units) * unsigned(cluster), 1, 1);
+  cfg.blockDim = dim3(unsigned(warps_per_cta) * 32u, 1, 1);
+  cfg.dynamicSmemBytes =
+      size_t(decode_cluster_smem_bytes(warps_per_cta, decode_cluster_stages(warps_per_cta, cluster),
+                                       cluster));
+  cfg.stream = stream;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = unsigned(cluster);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
+template <int G>
+static int max_active_g(int cluster, int warps_per_cta) {
+  if (configure_cluster_g<G>() != cudaSuccess) return -1;
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = cluster_config<G>(cluster, cluster, warps_per_cta, nullptr, attr);
+  int n = 0;
+  const cudaError_t err =
+      cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(reskv_decode_cluster_kernel<G>), &cfg);
+  if (err != cudaSuccess) {
+    (void)cudaGetLastError();
+    return 0;                          // this shape cannot be launched at all
+  }
+  return n;
+}
+
+template <int G>
+static cudaError_t launch_cluster_g(const DecodeParams& p, const CUtensorMap& tk,
+                                    const CUtensorMap& tv, int cluster, int warps_per_cta,
+                                    cudaStream_t stream) {
+  cudaError_t err = configure_cluster_g<G>();
+  if (err != cudaSuccess) return err;
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = cluster_config<G>(p.n_units, cluster, warps_per_cta, stream, attr);
+  cfg.dynamicSmemBytes = size_t(decode_cluster_smem_bytes(warps_per_cta, p.n_stages, cluster));
+  // may start before the previous kernel on the stream has finished (see
+  // griddepcontrol.wait in the kernel)
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.numAttrs = 2;
+  err = cudaLaunchKernelEx(&cfg, reskv_decode_cluster_kernel<G>, p, tk, tv);
+  if (err != cudaSuccess) return err;
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decode_cluster(const DecodeParams& p, const CUtensorMap& tk,
+                                  const CUtensorMap& tv, int group, int cluster,
+                                  int warps_per_cta, cudaStream_t stream) {
+  if (cluster < 1 || cluster > kMaxCluster || warps_per_cta < 1 || warps_per_cta > kMmaMaxW ||
+      p.n_stages < 1 || p.n_stages > decode_cluster_stages(warps_per_cta, cluster))
+    return cudaErrorInvalidValue;
+  switch (group) {
+    case 1: return launch_cluster_g<1>(p, tk, tv, cluster, warps_per_cta, stream);
+    case 2: return launch_cluster_g<2>(p, tk, tv, cluster, warps_per_cta, stream);
+    case 4: return launch_cluster_g<4>(p, tk, tv, cluster, warps_per_cta, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+int decode_cluster_max_active(int group, int cluster, int warps_per_cta) {
+  if (cluster < 1 || cluster > kMaxCluster || warps_per_cta < 1 || warps_per_cta > kMmaMaxW)
+    return 0;
+  switch (group) {
+    case 1: return max_active_g<1>(cluster, warps_per_cta);
+    case 2: return max_active_g<2>(cluster, warps_per_cta);
+    case 4: return max_active_g<4>(cluster, warps_per_cta);
+    default: return 0;
+  }
+}
+
+// Ring depth for `warps_per_cta` warps next to `cluster` CTA records.
+int decode_cluster_stages(int warps_per_cta, int cluster) {
+  int st = ((kSmemLimit - 1024 - cluster * kCtaRecFloats * 4) / warps_per_cta - 1024) / kStageBytes;
+  return st > kMmaMaxSt ? kMmaMaxSt : st;
+}
+
+int decode_cluster_smem_bytes(int warps_per_cta, int stages, int cluster) {
+  return warps_per_cta * warp_bytes(stages) + 1024 + cluster * kCtaRecFloats * 4;
+}
+
+}  // namespace reskv

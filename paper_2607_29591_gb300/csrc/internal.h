@@ -53,6 +53,17 @@ cudaError_t launch_decode_mma(const DecodeParams& p, const CUtensorMap& tk, cons
                               int group, int n_ctas, int warps_per_cta, cudaStream_t stream);
 int decode_mma_stages(int warps_per_cta);
 size_t decode_mma_partials_floats(int64_t n_units, int n_warps, int group);
+// Launch the cluster decode kernel: one cluster of `cluster` CTAs (1..8) of
+// `warps_per_cta` warps per unit, p.n_stages <= decode_cluster_stages(warps, cluster).
+cudaError_t launch_decode_cluster(const DecodeParams& p, const CUtensorMap& tk,
+                                  const CUtensorMap& tv, int group, int cluster,
+                                  int warps_per_cta, cudaStream_t stream);
+int decode_cluster_stages(int warps_per_cta, int cluster);
+int decode_cluster_smem_bytes(int warps_per_cta, int stages, int cluster);
+// How many clusters of that shape the current device holds at once (0: none).
+int decode_cluster_max_active(int group, int cluster, int warps_per_cta);
+// Slots per tensor-core tile and per TMA chunk of the decode kernels.
+constexpr int kDecodeChunk = 16;
 // Slots of zero padding after the log-count array (16-slot chunk copies).
 constexpr int kLogcPad = 16;
 
@@ -80,6 +91,12 @@ struct reskv_cache {
   int32_t* tickets = nullptr;
   uint32_t* status = nullptr;
   int max_warps = 0;
+  // cluster decode shape for one-layer and all-layer launches; cluster = 0
+  // when the launch's units do not fit on the device in one wave
+  struct ClusterPlan {
+    int cluster = 0;
+    int warps_per_cta = 0;
+  } cplan_layer, cplan_all;
   // 2-D TMA maps of kslots / vslots: [U * budget rows, 128 dims], boxes of
   // 16 rows x 64 dims with the 128-byte swizzle
   CUtensorMap tmap_k;

@@ -53,7 +53,7 @@ reskv_status validate_shape(const reskv_config* cfg) {
   if (cfg->budget < 1 || cfg->budget > (1 << 20))
     return fail(RESKV_ERR_INVALID_ARG, "budget must be in [1, 2^20]");
   if (cfg->decode_warps < 0) return fail(RESKV_ERR_INVALID_ARG, "decode_warps must be >= 0");
-  if (cfg->decode_kernel < RESKV_DECODE_AUTO || cfg->decode_kernel > RESKV_DECODE_MMA)
+  if (cfg->decode_kernel < RESKV_DECODE_AUTO || cfg->decode_kernel > RESKV_DECODE_CLUSTER)
     return fail(RESKV_ERR_INVALID_ARG, "unknown decode_kernel");
   if (double(cfg->n_layers) * cfg->batch * cfg->n_kv_heads * cfg->budget + kLogcPad >=
       double(int64_t(1) << 31))
@@ -127,6 +127,33 @@ void free_handle(reskv_cache* c) {
   delete c;
 }
 
+// Warps per CTA of the cluster kernel for clusters of `cluster` CTAs: 8, or
+// fewer when the unit has less than one 16-slot chunk per warp.
+int cluster_warps(int64_t budget, int cluster) {
+  const int64_t chunks = (budget + kDecodeChunk - 1) / kDecodeChunk + 1;
+  return int(std::min<int64_t>(kDecodeWarpsPerCta,
+                               std::max<int64_t>(1, (chunks + cluster - 1) / cluster)));
+}
+
+// Cluster decode shape for launches of `units` units: the largest cluster
+// (at most 8 CTAs, at most SMs / units) at which all of the launch's clusters
+// are resident at once; cluster = 0 if not even single-CTA clusters are.
+reskv_status plan_cluster(const reskv_cache* c, int64_t units, reskv_cache::ClusterPlan* out) {
+  *out = reskv_cache::ClusterPlan{};
+  if (units > c->num_sms) return RESKV_OK;
+  for (int cs = int(std::min<int64_t>(8, c->num_sms / units)); cs >= 1; --cs) {
+    const int wpc = cluster_warps(c->budget, cs);
+    const int fit = decode_cluster_max_active(c->cfg.group, cs, wpc);
+    if (fit < 0) return fail(RESKV_ERR_CUDA, "querying cluster occupancy of the decode kernel");
+    if (fit >= units) {
+      out->cluster = cs;
+      out->warps_per_cta = wpc;
+      return RESKV_OK;
+    }
+  }
+  return RESKV_OK;
+}
+
 }  // namespace
 
 // Allocate a zeroed layout and decode workspace for cfg's shape.
@@ -177,6 +204,12 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
   if (!encode_rows(&c->tmap_k, c->kslots, slots) || !encode_rows(&c->tmap_v, c->vslots, slots)) {
     free_handle(c);
     return fail(RESKV_ERR_CUDA, "creating the TMA tensor maps of the cache");
+  }
+  const int64_t per_layer = int64_t(cfg.batch) * cfg.n_kv_heads;
+  if ((st = plan_cluster(c, per_layer, &c->cplan_layer)) != RESKV_OK ||
+      (st = plan_cluster(c, c->n_units, &c->cplan_all)) != RESKV_OK) {
+    free_handle(c);
+    return st;
   }
   *out = c;
   return RESKV_OK;
@@ -321,20 +354,47 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   p.budget = c->budget;
   p.n_kv_heads = cfg.n_kv_heads;
   p.total_slots = int64_t(p.n_units) * c->budget;
+  p.gate_mode = cfg.gate_mode;
+  p.tau = cfg.tau;
+  p.alpha = cfg.alpha;
+  p.g_min = cfg.g_min;
+  p.g_fixed = cfg.g_fixed;
+  const reskv_cache::ClusterPlan& cp = layer < 0 ? c->cplan_all : c->cplan_layer;
+  int kernel = cfg.decode_kernel;
+  if (kernel == RESKV_DECODE_AUTO)
+    kernel = (cp.cluster > 0 && cfg.decode_warps == 0) ? RESKV_DECODE_CLUSTER : RESKV_DECODE_MMA;
+  if (kernel == RESKV_DECODE_CLUSTER) {
+    // one cluster per unit; a launch too large for one wave runs single-CTA
+    // clusters in several waves
+    const int cs = cp.cluster > 0 ? cp.cluster : 1;
+    const int wpc = cp.cluster > 0 ? cp.warps_per_cta : cluster_warps(c->budget, 1);
+    p.n_warps = int32_t(int64_t(cs) * wpc);
+    p.n_stages = decode_cluster_stages(wpc, cs);
+    cudaError_t err = launch_decode_cluster(p, c->tmap_k, c->tmap_v, cfg.group, cs, wpc,
+                                            static_cast<cudaStream_t>(stream));
+    if (err != cudaSuccess) return cuda_fail(err, "decode launch");
+    return RESKV_OK;
+  }
   // Split plan.  CUDA-core kernel: one warp per >= 32 slots, at most 8 warps
-  // per SM.  Tensor-core kernel: one CTA per SM with 1..8 warps so that every
-  // warp streams >= ~200 slots (fewer, longer pieces for small launches, with
-  // a deeper ring in the shared memory that fewer warps leave free).
-  const bool mma = cfg.decode_kernel != RESKV_DECODE_FMA;
+  // per SM.  Tensor-core stream-K kernel: one warp per unit when the launch
+  // has between 1 and 4 units per SM; otherwise one CTA per SM with 1..8
+  // warps so that every warp streams >= ~200 slots (fewer, longer pieces for
+  // small launches, with a deeper ring in the shared memory that fewer warps
+  // leave free).
+  const bool mma = kernel == RESKV_DECODE_MMA;
   int64_t W = 0;
   int wpc = kDecodeWarpsPerCta;
   if (mma) {
     if (cfg.decode_warps > 0) {
       W = cfg.decode_warps;
     } else {
-      wpc = int(std::min<int64_t>(8, std::max<int64_t>(1, p.total_slots / (int64_t(c->num_sms) * 200))));
-      W = int64_t(c->num_sms) * wpc;
-      if (p.total_slots < W * 32) W = std::max<int64_t>(1, p.total_slots / 32);
+      if (p.n_units >= c->num_sms && p.n_units <= 4 * int64_t(c->num_sms)) {
+        W = p.n_units;                // one warp per unit: no partial records at all
+      } else {
+        wpc = int(std::min<int64_t>(8, std::max<int64_t>(1, p.total_slots / (int64_t(c->num_sms) * 200))));
+        W = int64_t(c->num_sms) * wpc;
+        if (p.total_slots < W * 32) W = std::max<int64_t>(1, p.total_slots / 32);
+      }
     }
     if (W > p.total_slots) W = p.total_slots;
     if (W > c->max_warps) W = c->max_warps;
@@ -348,11 +408,6 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   if (W < 1) W = 1;
   p.n_warps = int32_t(W);
   p.n_stages = mma ? decode_mma_stages(wpc) : 0;
-  p.gate_mode = cfg.gate_mode;
-  p.tau = cfg.tau;
-  p.alpha = cfg.alpha;
-  p.g_min = cfg.g_min;
-  p.g_fixed = cfg.g_fixed;
   cudaError_t err =
       mma ? launch_decode_mma(p, c->tmap_k, c->tmap_v, cfg.group, int((W + wpc - 1) / wpc), wpc,
                               static_cast<cudaStream_t>(stream))
@@ -387,6 +442,20 @@ reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info) {
   info->head_dim = kHeadDim;
   info->slot_bytes = 2 * kSlotRowBytes;
   info->cache_bytes = c->n_units * int64_t(c->budget) * (2 * kSlotRowBytes + 4);
+  const bool auto_plan = c->cfg.decode_kernel == RESKV_DECODE_AUTO && c->cfg.decode_warps == 0;
+  const bool cluster = c->cfg.decode_kernel == RESKV_DECODE_CLUSTER;
+  info->layer_cluster = auto_plan ? c->cplan_layer.cluster
+                                  : cluster ? std::max(1, c->cplan_layer.cluster) : 0;
+  info->layer_cluster_warps =
+      info->layer_cluster ? (c->cplan_layer.cluster ? c->cplan_layer.warps_per_cta
+                                                    : cluster_warps(c->budget, 1))
+                          : 0;
+  info->all_cluster = auto_plan ? c->cplan_all.cluster
+                                : cluster ? std::max(1, c->cplan_all.cluster) : 0;
+  info->all_cluster_warps =
+      info->all_cluster ? (c->cplan_all.cluster ? c->cplan_all.warps_per_cta
+                                                : cluster_warps(c->budget, 1))
+                        : 0;
   return RESKV_OK;
 }
 

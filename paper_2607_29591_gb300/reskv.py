@@ -21,7 +21,7 @@ STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "OOM", 4: "CUDA"
                 5: "DEVICE_STATUS"}
 RESKV_SCORE_OBS_POOL, RESKV_SCORE_KEYNORM = 0, 1
 RESKV_GATE_DYNAMIC, RESKV_GATE_FIXED = 0, 1
-RESKV_DECODE_AUTO, RESKV_DECODE_FMA, RESKV_DECODE_MMA = 0, 1, 2
+RESKV_DECODE_AUTO, RESKV_DECODE_FMA, RESKV_DECODE_MMA, RESKV_DECODE_CLUSTER = 0, 1, 2, 3
 RESKV_DEBUG_SCORES, RESKV_DEBUG_RANKED, RESKV_DEBUG_LOSSES, RESKV_DEBUG_CANDIDATES = 0, 1, 2, 3
 MAX_GRID = 8
 
@@ -56,7 +56,9 @@ class reskv_host_cache(ctypes.Structure):
 class reskv_cache_info(ctypes.Structure):
     _fields_ = [("n_units", ctypes.c_int64), ("budget", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("slot_bytes", ctypes.c_int64),
-                ("cache_bytes", ctypes.c_int64)]
+                ("cache_bytes", ctypes.c_int64), ("layer_cluster", ctypes.c_int32),
+                ("layer_cluster_warps", ctypes.c_int32), ("all_cluster", ctypes.c_int32),
+                ("all_cluster_warps", ctypes.c_int32)]
 
 
 class reskv_device_cache(ctypes.Structure):
@@ -209,6 +211,11 @@ def reskv_build_cache(cfg: reskv_config, K_layers: Sequence, V_layers: Sequence,
 def reskv_decode_attn(cache: Cache, layer: int, Q, O, stream=None) -> None:
     """Alg. 2.  layer >= 0: Q bf16 [B, H_q, d], O fp32 [B, H_q, d]; layer == -1:
     every layer, Q [L, B, H_q, d] and O likewise."""
+    c = cache.cfg
+    need = (c.n_layers if layer == -1 else 1) * c.batch * c.n_kv_heads * c.group * c.head_dim
+    for name, t in (("Q", Q), ("O", O)):
+        if t.numel() != need:
+            raise ValueError(f"{name} holds {t.numel()} elements; this call needs {need}")
     _check(load_library().reskv_decode_attn(cache.handle, int(layer),
                                             _dptr(Q, "torch.bfloat16", "Q"),
                                             _dptr(O, "torch.float32", "O"), _stream(stream)))

@@ -32,9 +32,11 @@ def lib():
 KERNEL = {"id": R.RESKV_DECODE_MMA}
 
 
-@pytest.fixture(autouse=True, params=[R.RESKV_DECODE_FMA, R.RESKV_DECODE_MMA], ids=["fma", "mma"])
+@pytest.fixture(autouse=True, params=[R.RESKV_DECODE_FMA, R.RESKV_DECODE_MMA, R.RESKV_DECODE_CLUSTER],
+                ids=["fma", "mma", "cluster"])
 def decode_kernel(request):
-    """Every decode test runs on both kernels: CUDA-core FMA and tensor-core mma."""
+    """Every decode test runs on the three kernels: CUDA-core FMA, tensor-core
+    stream-K and tensor-core one-cluster-per-unit."""
     KERNEL["id"] = request.param
     yield request.param
 
@@ -272,3 +274,30 @@ def test_fixed_point_exact_residual_encoding_is_full_attention():
     assert_output_parity(O, full, "exact encoding")
     # the residual's share of the output carries only bf16 rounding of v_bar
     assert errors(O, full)[1] < 4e-3 * ZE / (ZE + np.exp(Kf[:m] @ q / math.sqrt(d)).sum()) + 1e-5
+
+
+@pytest.mark.parametrize("L,Bt,H", [(1, 1, 1), (1, 3, 4), (2, 4, 8), (1, 25, 4), (2, 20, 8)])
+def test_launch_sizes(L, Bt, H):
+    """Launches of 1 to 320 units with b = 200 (chunks straddle units): the
+    automatic plan moves from clusters of 8 CTAs per unit through smaller ones
+    to the stream-K split (and, for the cluster kernel chosen explicitly,
+    single-CTA clusters in several waves); per-layer and all-layer calls."""
+    G, b = 4, 200
+    U = L * Bt * H
+    rng = np.random.default_rng(U)
+    splits = []
+    for _ in range(U):
+        n = int(rng.integers(1, b + 1))
+        m = int(rng.integers(1, n + 1))
+        splits.append((m, n - m))
+    w, lay = synthetic_layout(L, Bt, H, b, splits)
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len, budget=b)
+    h = R.reskv_import_cache(cfg, **lay)
+    Q = queries_for(w, L, Bt, H, G)
+    ref = oracle_decode_all(lay, Q, cfg)
+    O = run_decode(h, Q).cpu().numpy()
+    assert_output_parity(O, ref, f"all layers, {U} units")
+    for l in range(L):
+        O_l = run_decode(h, Q[l].contiguous(), layer=l).cpu().numpy()
+        assert_output_parity(O_l, ref[l], f"layer {l}, {Bt * H} units")
+    R.reskv_check_status(h)

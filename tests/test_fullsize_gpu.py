@@ -1,5 +1,6 @@
-"""Parity at the workloads' full sizes, in the launch configuration that
-bench.py times (one all-layer reskv_decode_attn launch after reskv_build_cache).
+"""Parity at the workloads' full sizes, in the launch configurations that
+bench.py times (one all-layer reskv_decode_attn launch after reskv_build_cache,
+and one launch per layer).
 
 The inputs are generated on the GPU by the same generator as the benchmark;
 for a seeded sample of units they are regenerated on the CPU (and checked to be
@@ -70,6 +71,14 @@ def run_full(name, n_sample):
     R.reskv_decode_attn(cache, -1, Qd, O)
     torch.cuda.synchronize()
     R.reskv_check_status(cache)
+    # one launch per layer (the plan a decode step uses layer by layer)
+    O_layers = torch.full(Qd.shape, float("nan"), dtype=torch.float32, device="cuda")
+    for l in range(L):
+        R.reskv_decode_attn(cache, l, Qd[l], O_layers[l])
+    torch.cuda.synchronize()
+    R.reskv_check_status(cache)
+    assert errors(O_layers.cpu().numpy(), O.cpu().numpy().astype(np.float64))[1] < 1e-5
+    del O_layers
     lay = R.reskv_export_cache(cache)
     scores = R.reskv_export_debug(cache, R.RESKV_DEBUG_SCORES)
     top = R.reskv_export_debug(cache, R.RESKV_DEBUG_RANKED)
