@@ -36,9 +36,14 @@ from paper_2607_29591_gb300 import workloads as wl  # noqa: E402
 METRIC = "compressed-decode attn tokens/s and achieved HBM GB/s (% of peak), 1 GB300"
 DEFAULT_WORKLOAD = "llama8b_32l_32k_b8"
 SLOT_BYTES = 2 * 128 * 2            # one K row + one V row, bf16
+CSRC = os.path.join(ROOT, "paper_2607_29591_gb300", "csrc")
+# ncu summaries of the two tensor-core decode kernels on the default workload,
+# and the sources each summary's counters were taken from
 PROFILE = os.path.join(ROOT, "profiles", "decode_kernel_llama8b_32l_32k_b8.md")
-KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_29591_gb300", "csrc", f)
-                  for f in ("decode_mma.cu", "device_utils.cuh")]
+KERNEL_SOURCES = [os.path.join(CSRC, f) for f in ("decode_mma.cu", "mma_tile.cuh", "device_utils.cuh")]
+PROFILE_LAYER = os.path.join(ROOT, "profiles", "decode_cluster_llama8b_32l_32k_b8_per_layer.md")
+KERNEL_SOURCES_LAYER = [os.path.join(CSRC, f)
+                        for f in ("decode_cluster.cu", "mma_tile.cuh", "device_utils.cuh")]
 
 
 def parse_args():
@@ -166,23 +171,24 @@ def measured_peak_gbs():
     return 6800.0, "fallback"
 
 
-def kernel_hash():
+def kernel_hash(sources=None):
     h = hashlib.sha256()
-    for p in KERNEL_SOURCES:
+    for p in sources or KERNEL_SOURCES:
         with open(p, "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(units_per_launch: int):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel
+def profiled_traffic(units_per_launch: int, profile=None, sources=None):
+    """DRAM bytes per launch from a committed ncu summary, if the kernel
     source has not changed since it was captured (else None)."""
-    if not os.path.exists(PROFILE):
+    profile = profile or PROFILE
+    if not os.path.exists(profile):
         return None
-    text = open(PROFILE).read()
+    text = open(profile).read()
     m_hash = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", text)
     m_bpu = re.search(r"dram_bytes_per_unit:\s*([0-9.]+)", text)
-    if not m_hash or not m_bpu or m_hash.group(1) != kernel_hash():
+    if not m_hash or not m_bpu or m_hash.group(1) != kernel_hash(sources):
         return None
     return int(float(m_bpu.group(1)) * units_per_launch)
 
@@ -399,6 +405,13 @@ def main():
                      "frac_of_peak": alg / tg / 1e9 / peak,
                      "how": f"{w.n_layers} per-layer reskv_decode_attn launches replayed as one "
                             f"CUDA graph, {reps} replays"}
+        units_layer = w.batch * w.n_kv_heads
+        per_layer["roofline"] = {
+            "bound": "hbm", "achieved": alg / tg / 1e9, "peak": peak, "unit": "GB/s",
+            "frac": alg / tg / 1e9 / peak, "kernel": decode_plan["per_layer"],
+            "traffic": (profiled_traffic(units_layer, PROFILE_LAYER, KERNEL_SOURCES_LAYER)
+                        if info["layer_cluster"] > 0 else None),
+            "algorithmic_bytes_per_launch": alg // w.n_layers}
         del graph
 
     # ---- end to end through the C ABI with host buffers ----

@@ -377,7 +377,9 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   }
   // Split plan.  CUDA-core kernel: one warp per >= 32 slots, at most 8 warps
   // per SM.  Tensor-core stream-K kernel: one warp per unit when the launch
-  // has between 1 and 4 units per SM; otherwise one CTA per SM with 1..8
+  // has between 1 and 4 short units (at most 16 tiles of 16 slots) per SM, so
+  // that no unit is cut; otherwise (a lone warp on a long unit is bound by
+  // the latency of its tile chain) one CTA per SM with 1..8
   // warps so that every warp streams >= ~200 slots (fewer, longer pieces for
   // small launches, with a deeper ring in the shared memory that fewer warps
   // leave free).
@@ -388,7 +390,7 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
     if (cfg.decode_warps > 0) {
       W = cfg.decode_warps;
     } else {
-      if (p.n_units >= c->num_sms && p.n_units <= 4 * int64_t(c->num_sms)) {
+      if (p.n_units >= c->num_sms && p.n_units <= 4 * int64_t(c->num_sms) && c->budget <= 256) {
         W = p.n_units;                // one warp per unit: no partial records at all
       } else {
         wpc = int(std::min<int64_t>(8, std::max<int64_t>(1, p.total_slots / (int64_t(c->num_sms) * 200))));
