@@ -6,4 +6,4 @@ library and imports nothing from it.
 """
 from .reskv_oracle import *  # noqa: F401,F403
 from .reskv_oracle import (OracleConfig, UnitCache, GATE_DYNAMIC, GATE_FIXED,  # noqa: F401
-                           SCORE_OBS_POOL, SCORE_KEYNORM)
+                           SCORE_OBS_POOL, SCORE_KEYNORM, SOFTMAX_SHARED, SOFTMAX_SEPARATE)

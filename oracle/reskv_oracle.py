@@ -55,6 +55,9 @@ GATE_FIXED = 1
 SCORE_OBS_POOL = 0
 SCORE_KEYNORM = 1
 
+SOFTMAX_SHARED = 0        # Eq. reskv: one softmax over main and residual entries
+SOFTMAX_SEPARATE = 1      # "w/o shared softmax" ablation (Table ablation_main)
+
 
 @dataclass
 class OracleConfig:
@@ -80,6 +83,7 @@ class OracleConfig:
     alpha: float = 12.0              # sigmoid slope = 1/T_g (App. B)
     g_min: float = 0.0               # minimum gate (App. B)
     g_fixed: float = 1.0             # gate value when gate_mode == GATE_FIXED
+    softmax_mode: int = SOFTMAX_SHARED
 
 
 # ---------------------------------------------------------------------------
@@ -336,6 +340,51 @@ def shared_softmax_decode(q, Kmain, Vmain, Kres, Vres, logc, cfg: OracleConfig,
     return out
 
 
+def separate_softmax_decode(q, Kmain, Vmain, Kres, Vres, logc, cfg: OracleConfig,
+                            return_stats: bool = False):
+    """One decode query with separate main and residual normalisations, the
+    "w/o shared softmax" ablation (Sec. 7 ablations, Table ablation_main).
+
+    The paper names the variant but prints no combination rule; the reading
+    taken here keeps every other part of the method and mixes the two
+    normalised branches with the gate:
+
+      o_M = sum_M softmax_M(a)_p v_p,          a_p = <q,k_p>/sqrt(d)
+      o_R = sum_R softmax_R(a')_j v_bar_j,     a'_j = <q,k_bar_j>/sqrt(d) + log c_j
+      o^  = (1 - g) o_M + g o_R,               g = gate(p_max) as in Eq. gate
+
+    Without residual mass (R empty or every c_j = 0) or with g = 0, o^ = o_M.
+    """
+    a = logits(q, Kmain)
+    e_main = np.exp(a - a.max())
+    Z_M = e_main.sum()
+    p_max = 1.0 / Z_M
+    if cfg.gate_mode == GATE_DYNAMIC:
+        g = dynamic_gate(p_max, cfg.tau, cfg.alpha, cfg.g_min)
+    else:
+        g = cfg.g_fixed
+    o_main = (e_main @ Vmain) / Z_M
+    ar = logits(q, Kres) + logc if Kres.shape[0] > 0 else np.zeros(0)
+    finite = ar[np.isfinite(ar)]
+    if finite.size == 0 or g == 0:
+        out = o_main
+    else:
+        e_res = np.exp(ar - finite.max())      # log c_j = -inf (c = 0) gives 0
+        o_res = (e_res @ Vres) / e_res.sum()
+        out = (1.0 - g) * o_main + g * o_res
+    if return_stats:
+        return out, dict(p_max=p_max, g=g)
+    return out
+
+
+def decode_query(q, Kmain, Vmain, Kres, Vres, logc, cfg: OracleConfig):
+    """The decode rule that cfg selects: Eq. reskv (shared softmax, the method)
+    or the separate-normalisation ablation."""
+    if cfg.softmax_mode == SOFTMAX_SEPARATE:
+        return separate_softmax_decode(q, Kmain, Vmain, Kres, Vres, logc, cfg)
+    return shared_softmax_decode(q, Kmain, Vmain, Kres, Vres, logc, cfg)
+
+
 # ---------------------------------------------------------------------------
 # Construction (Alg. 1) with the validation proxy (Sec. 5.5.1)
 # ---------------------------------------------------------------------------
@@ -385,20 +434,21 @@ def candidate_valid(s: int, cfg: OracleConfig, r: int) -> bool:
 
 def decode_unit(cache: UnitCache, Q: np.ndarray, cfg: OracleConfig) -> np.ndarray:
     """Decode the G query heads of one KV head (GQA sharing, App. B): [G, d]."""
-    return np.stack([shared_softmax_decode(q, cache.kmain, cache.vmain, cache.kbar,
-                                           cache.vbar, cache.logc, cfg) for q in Q])
+    return np.stack([decode_query(q, cache.kmain, cache.vmain, cache.kbar, cache.vbar,
+                                  cache.logc, cfg) for q in Q])
 
 
 def validation_loss(cache: UnitCache, Qval: np.ndarray, O_full: np.ndarray,
                     cfg: OracleConfig) -> float:
     """L_r = mean over validation queries (and the G heads) of ||o^(r) - o_S||^2
-    (Eq. valloss), with the decode rule of Sec. 5.4 including the gate."""
+    (Eq. valloss), with the decode rule of Sec. 5.4 including the gate (or the
+    ablation's rule, when cfg selects it)."""
     G, n_val, _ = Qval.shape
     total = 0.0
     for g in range(G):
         for t in range(n_val):
-            o = shared_softmax_decode(Qval[g, t], cache.kmain, cache.vmain, cache.kbar,
-                                      cache.vbar, cache.logc, cfg)
+            o = decode_query(Qval[g, t], cache.kmain, cache.vmain, cache.kbar, cache.vbar,
+                             cache.logc, cfg)
             diff = o - O_full[g, t]
             total += float(diff @ diff)
     return total / (G * n_val)

@@ -185,6 +185,18 @@ def _val_loss_no_mean(cache, Qval, O_full, cfg):
     return _orig["validation_loss"](cache, Qval, O_full, cfg) * Qval.shape[0] * Qval.shape[1]
 
 
+def _separate_additive(q, Kmain, Vmain, Kres, Vres, logc, cfg, return_stats=False):
+    out, st = _orig["separate_softmax_decode"](q, Kmain, Vmain, Kres, Vres, logc, cfg, True)
+    o_main = _orig["separate_softmax_decode"](q, Kmain, Vmain, Kres[:0], Vres[:0], logc[:0], cfg)
+    g = st["g"]
+    return o_main + (out - (1 - g) * o_main)          # o_M + g o_R instead of a mixture
+
+
+def _separate_drop_logc(q, Kmain, Vmain, Kres, Vres, logc, cfg, return_stats=False):
+    lc = np.where(np.isfinite(logc), 0.0, logc)
+    return _orig["separate_softmax_decode"](q, Kmain, Vmain, Kres, Vres, lc, cfg, return_stats)
+
+
 def _attention_full_no_shift(q, K, V):
     a = core.logits(q, K)
     w = np.exp(a)
@@ -215,6 +227,8 @@ MUTANTS = [
     ("scores_keynorm", _keynorm_abs),
     ("validation_loss", _val_loss_no_mean),
     ("attention_full", _attention_full_no_shift),
+    ("separate_softmax_decode", _separate_additive),
+    ("separate_softmax_decode", _separate_drop_logc),
 ]
 
 

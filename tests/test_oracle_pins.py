@@ -146,6 +146,51 @@ def test_decode_residual_mass_enters_both_numerator_and_denominator():
     np.testing.assert_allclose(out2, 3 * g / (1 + 3 * g), rtol=1e-14)
 
 
+def test_separate_softmax_hand_sized():
+    """"w/o shared softmax" ablation (Table ablation_main), reading o^ = (1-g) o_M + g o_R.
+
+    Main: one token with v = 0; one entry with v_bar = 1 and c = 3.  Each branch
+    is normalised on its own, so o_R = 1 whatever c is, and o^ = g."""
+    d = 4
+    q = np.zeros(d)
+    args = (q, np.zeros((1, d)), np.zeros((1, d)), np.zeros((1, d)), np.ones((1, d)), np.log([3.0]))
+    for gf in (0.0, 0.3, 1.0):
+        out = orc.separate_softmax_decode(*args, _cfg(gate_mode=orc.GATE_FIXED, g_fixed=gf,
+                                                      softmax_mode=orc.SOFTMAX_SEPARATE))
+        np.testing.assert_allclose(out, gf, rtol=1e-15, atol=0)
+    out = orc.separate_softmax_decode(*args, _cfg(softmax_mode=orc.SOFTMAX_SEPARATE))
+    np.testing.assert_allclose(out, 1.0 / (1.0 + math.exp(9.0)), rtol=1e-14)   # p_max = 1
+
+
+def test_separate_softmax_single_entry_and_count_weighting():
+    """Separate normalisations on random data: a single entry gives o_R = v_bar,
+    so o^ = (1-g) o_M + g v_bar with the gate of the main logits; two entries
+    with one key weigh their values by their counts (log c_j in the logit)."""
+    rng = np.random.default_rng(21)
+    d, m = 16, 30
+    K, V, q = bf16ish(rng, (m, d)), bf16ish(rng, (m, d)), bf16ish(rng, d, 2.0)
+    cfg = _cfg(softmax_mode=orc.SOFTMAX_SEPARATE)
+    # gate by hand: p_max = largest main softmax weight
+    a = [sum(q[i] * K[p, i] for i in range(d)) / math.sqrt(d) for p in range(m)]
+    p_max = 1.0 / sum(math.exp(x - max(a)) for x in a)
+    g = max(0.0, 1.0 / (1.0 + math.exp(-12.0 * (0.25 - p_max))))
+    kb, vb = bf16ish(rng, (1, d)), bf16ish(rng, (1, d), 3.0)
+    out = orc.separate_softmax_decode(q, K, V, kb, vb, np.log([7.0]), cfg)
+    np.testing.assert_allclose(out, (1 - g) * textbook_attention(q, K, V) + g * vb[0],
+                               rtol=1e-12, atol=1e-13)
+    kb2 = np.vstack([kb, kb])
+    vb2 = bf16ish(rng, (2, d), 3.0)
+    out2 = orc.separate_softmax_decode(q, K, V, kb2, vb2, np.log([2.0, 6.0]), cfg)
+    o_r = (2.0 * vb2[0] + 6.0 * vb2[1]) / 8.0
+    np.testing.assert_allclose(out2, (1 - g) * textbook_attention(q, K, V) + g * o_r,
+                               rtol=1e-12, atol=1e-13)
+    # no residual mass (every c = 0): main-only, whatever g
+    out3 = orc.separate_softmax_decode(q, K, V, kb2, vb2, np.array([-np.inf, -np.inf]), cfg)
+    np.testing.assert_allclose(out3, textbook_attention(q, K, V), rtol=1e-12, atol=1e-13)
+    # the dispatcher routes by softmax_mode
+    np.testing.assert_allclose(orc.decode_query(q, K, V, kb, vb, np.log([7.0]), cfg), out, rtol=0)
+
+
 def test_gate_closed_forms():
     """Eq. gate with the paper's tau = 0.25, alpha = 12 (App. B), via uniform main caches."""
     gc = golden("gate_closed_forms.json")
