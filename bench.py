@@ -466,6 +466,9 @@ def main():
                          "algorithmic_bytes_per_launch": alg},
             "per_layer_graph": per_layer,
             "construction_s": build_s,
+            "construction_stages_ms": dict(zip(
+                ["scores", "ranking", "validation_targets", "lloyd", "validation_loss_and_choice",
+                 "pack"], [round(x, 3) for x in info["build_ms"]])),
             "e2e": e2e,
             "clocks": clk.summary(),
             "gpu_launches": args.steps,

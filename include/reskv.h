@@ -48,6 +48,13 @@ typedef enum {
 
 enum { RESKV_SCORE_OBS_POOL = 0, RESKV_SCORE_KEYNORM = 1 };
 enum { RESKV_GATE_DYNAMIC = 0, RESKV_GATE_FIXED = 1 };
+/* RESKV_SOFTMAX_SHARED: Eq. reskv, one softmax over main and residual entries
+ * (the method).  RESKV_SOFTMAX_SEPARATE: the "w/o shared softmax" ablation
+ * (Table ablation_main); the paper prints no combination rule, and the one
+ * built is o^ = (1 - g) o_M + g o_R with each branch normalised on its own
+ * (o^ = o_M without residual mass).  It applies to decode and to the
+ * validation proxy of reskv_build_cache. */
+enum { RESKV_SOFTMAX_SHARED = 0, RESKV_SOFTMAX_SEPARATE = 1 };
 enum { RESKV_DECODE_AUTO = 0, RESKV_DECODE_FMA = 1, RESKV_DECODE_MMA = 2, RESKV_DECODE_CLUSTER = 3 };
 
 #define RESKV_MAX_GRID 8
@@ -99,6 +106,7 @@ typedef struct reskv_config {
                               stream-K over the launch's slot range, 3
                               tensor-core with one thread-block cluster of 1..8
                               CTAs per unit (decode_warps ignored)           */
+  int32_t softmax_mode;    /* RESKV_SOFTMAX_*                                */
 } reskv_config;
 
 /* Fill *cfg with the paper's defaults; shape fields are zeroed. */
@@ -161,6 +169,11 @@ typedef struct reskv_cache_info {
   int32_t layer_cluster_warps; /* warps per CTA of that cluster launch       */
   int32_t all_cluster;     /* the same for an all-layer launch (layer = -1)  */
   int32_t all_cluster_warps;
+  float build_ms[6];       /* device time of reskv_build_cache per stage of
+                              Alg. 1, summed over layers (ms): token scores,
+                              ranking, validation targets o_S, Lloyd residual
+                              entries, validation losses + choice of r,
+                              packing; zero for an imported cache          */
 } reskv_cache_info;
 
 reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info);

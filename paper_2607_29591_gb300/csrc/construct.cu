@@ -59,6 +59,48 @@ cudaError_t set_smem(K kernel, size_t bytes) {
 
 int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+// Device time per construction stage: an event is recorded on the stream at
+// every stage boundary of a layer; at the end of the layer the intervals are
+// added to their stages (events are reused from layer to layer).
+class StageTimer {
+ public:
+  explicit StageTimer(cudaStream_t s) : stream_(s) {}
+  ~StageTimer() {
+    for (cudaEvent_t e : pool_) cudaEventDestroy(e);
+  }
+  // the interval that starts now belongs to `stage` (-1: not timed)
+  bool mark(int stage) {
+    if (n_ == pool_.size()) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) return false;
+      pool_.push_back(e);
+    }
+    stage_.resize(n_ + 1);
+    stage_[n_] = stage;
+    return cudaEventRecord(pool_[n_++], stream_) == cudaSuccess;
+  }
+  // close the layer: wait for its last event, accumulate, start over
+  bool flush(float* ms) {
+    if (n_ == 0) return true;
+    if (cudaEventSynchronize(pool_[n_ - 1]) != cudaSuccess) return false;
+    for (size_t i = 0; i + 1 < n_; ++i) {
+      float t = 0.f;
+      if (cudaEventElapsedTime(&t, pool_[i], pool_[i + 1]) != cudaSuccess) return false;
+      if (stage_[i] >= 0) ms[stage_[i]] += t;
+    }
+    n_ = 0;
+    return true;
+  }
+
+ private:
+  cudaStream_t stream_;
+  std::vector<cudaEvent_t> pool_;
+  std::vector<int> stage_;
+  size_t n_ = 0;
+};
+
+enum { kStScore = 0, kStRank, kStValTargets, kStLloyd, kStValLoss, kStPack };
+
 }  // namespace
 
 reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
@@ -234,6 +276,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     return cleanup_fail(fail(RESKV_ERR_CUDA, "setting kernel shared-memory limits"));
 
   const double one_minus_delta = 1.0 - double(cfg.delta);
+  StageTimer timer(stream);
+  bool timing_ok = true;
 
   for (int l = 0; l < cfg.n_layers; ++l) {
     const __nv_bfloat16* K = static_cast<const __nv_bfloat16*>(Kl[l]);
@@ -241,6 +285,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     const __nv_bfloat16* Q = Ql ? static_cast<const __nv_bfloat16*>(Ql[l]) : nullptr;
 
     // ---- token scores ----
+    timing_ok &= timer.mark(kStScore);
     if (cfg.score_mode == RESKV_SCORE_OBS_POOL) {
       ObsArgs oa{K, Q, s, G, cfg.n_obs, n_fit_rows, cfg.n_fit, ntiles, tstats, rstats, A};
       k_obs_pass1<<<dim3(ntiles, UL), kThreads, sm_obs1, stream>>>(oa);
@@ -251,6 +296,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       k_score_keynorm<<<unsigned(cdiv(int64_t(US), 256)), 256, 0, stream>>>(K, scores, int64_t(US));
     }
     RESKV_LAUNCH_CHECK("scoring");
+    timing_ok &= timer.mark(kStRank);
     TopArgs ta{scores, s, P, n_top, top, rank_pos, c->status};
     k_topk<<<UL, kTopThreads, sm_top, stream>>>(ta);
     RESKV_LAUNCH_CHECK("ranking");
@@ -261,6 +307,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     auto lloyd_run = [&](const int32_t* r_unit, int ent_off) -> reskv_status {
       la.r_unit = r_unit;
       la.ent_off = ent_off;
+      timing_ok &= timer.mark(kStLloyd);
       k_lloyd_init<<<dim3(rmax, UL), kHeadDim, 0, stream>>>(la);
       for (int it = 0; it < cfg.lloyd_iters; ++it) {
         k_lloyd_assign<<<dim3(ntiles, UL), kThreads, sm_assign, stream>>>(la);
@@ -274,6 +321,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
 
     if (proxy) {
       // ---- validation targets, candidates, choice of r ----
+      timing_ok &= timer.mark(kStValTargets);
       ValArgs va{K, V, Q, s, G, cfg.n_obs, cfg.n_val, n_val_rows, nchunks, vpart, oS};
       k_val_full<<<dim3(nchunks, unsigned(cdiv(n_val_rows, kRowBlk)), UL), kThreads, sm_val, stream>>>(va);
       k_val_combine<<<dim3(n_val_rows, UL), kHeadDim, 0, stream>>>(va);
@@ -287,9 +335,10 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
           st = lloyd_run(r_unit, run_off[run]);
           if (st != RESKV_OK) return cleanup_fail(st);
         }
+        timing_ok &= timer.mark(kStValLoss);
         LossArgs lo{K, V, Q, s, G, cfg.n_obs, cfg.n_val, n_val_rows, P, n_top, b, top, r_unit,
                     kbar, vbar, ecount, ent_stride, run_off[run], cfg.beta, cfg.gate_mode,
-                    cfg.tau, cfg.alpha, cfg.g_min, cfg.g_fixed, oS, rowerr};
+                    cfg.tau, cfg.alpha, cfg.g_min, cfg.g_fixed, oS, rowerr, cfg.softmax_mode};
         k_val_loss<<<dim3(unsigned(cdiv(n_val_rows, 8)), UL), kThreads, 0, stream>>>(lo);
         k_loss_reduce<<<unsigned(cdiv(UL, 128)), 128, 0, stream>>>(rowerr, losses, n_val_rows, UL,
                                                                   ncol, run);
@@ -300,6 +349,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       RESKV_LAUNCH_CHECK("choosing r");
     } else {
       // fixed r per unit (or the budget covers every token: r = 0)
+      timing_ok &= timer.mark(-1);
       std::vector<int32_t> rl(UL, 0), ch(UL, 0);
       bool any = false;
       if (!ovr.empty())
@@ -319,11 +369,14 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     }
 
     // ---- pack the chosen cache ----
+    timing_ok &= timer.mark(kStPack);
     PackArgs pa{K, V, s, P, b, rank_pos, r_final, chosen, run_off_d, kbar, vbar, ecount,
                 ent_stride, cfg.beta, int64_t(l) * UL, c->kslots, c->vslots, c->logc,
                 c->slot_pos, c->counts, c->n_main, c->n_res};
     k_pack<<<UL, 1024, 0, stream>>>(pa);
     RESKV_LAUNCH_CHECK("packing");
+    timing_ok &= timer.mark(-1);
+    timing_ok &= timer.flush(c->build_ms);
 
     if (cfg.keep_debug) {
       cudaError_t e = cudaMemcpyAsync(c->dbg_scores + size_t(l) * US, scores, US * 8,
@@ -337,6 +390,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       if (e != cudaSuccess) return cleanup_fail(fail(RESKV_ERR_CUDA, "keeping intermediates"));
     }
   }
+  if (!timing_ok)                        // timing is reported, not needed: clear it
+    for (float& t : c->build_ms) t = 0.f;
   // scratch is freed (cudaFree synchronises) when S leaves scope
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return cleanup_fail(fail(RESKV_ERR_CUDA, std::string("construction: ") +

@@ -914,6 +914,7 @@ struct LossArgs {
   float tau, alpha, g_min, g_fixed;
   const float* oS;             // [UL, n_rows, d]
   double* rowerr;              // [UL, n_rows]
+  int32_t softmax_mode;        // decode rule of the losses (RESKV_SOFTMAX_*)
 };
 
 // ||o^(r)(q) - o_S(q)||^2 per validation query, with the decode rule of
@@ -989,18 +990,12 @@ __global__ void __launch_bounds__(kThreads) k_val_loss(LossArgs p) {
     const float pmax = 1.0f / lM;
     g_val = fmaxf(p.g_min, 1.0f / (1.0f + expf(-p.alpha * (p.tau - pmax))));
   }
-  float wM = 1.f, wR = 0.f;
-  if (lR > 0.f && g_val > 0.f) {
-    const float mx = fmaxf(mM, mR);
-    wM = exp2f(mM - mx);
-    wR = g_val * exp2f(mR - mx);
-  }
-  const float inv = 1.0f / (wM * lM + wR * lR);
+  const float2 coef = branch_coefs(p.softmax_mode, g_val, mM, lM, mR, lR);
   const float* os = p.oS + (int64_t(ul) * p.n_rows + row) * kHeadDim + 4 * lane;
   float e = 0.f;
 #pragma unroll
   for (int d = 0; d < 4; ++d) {
-    const float o = (wM * aM[d] + wR * aR[d]) * inv;
+    const float o = coef.x * aM[d] + coef.y * aR[d];
     const float df = o - os[d];
     e += df * df;
   }

@@ -306,17 +306,10 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
       Ls[sg] = l;
       As[sg] = a;
     }
-    const float g = gate_of(p, Ls[0]);
-    float wM = 1.f, wR = 0.f;
-    if (Ls[1] > 0.f && g > 0.f) {
-      const float mx = fmaxf(Ms[0], Ms[1]);
-      wM = exp2f(Ms[0] - mx);
-      wR = g * exp2f(Ms[1] - mx);
-    }
-    const float inv = 1.0f / (wM * Ls[0] + wR * Ls[1]);
+    const float2 w = branch_coefs(p.softmax_mode, gate_of(p, Ls[0]), Ms[0], Ls[0], Ms[1], Ls[1]);
     *reinterpret_cast<float4*>(p.O + (orow0 + hh) * kHeadDim + d4) =
-        make_float4((wM * As[0].x + wR * As[1].x) * inv, (wM * As[0].y + wR * As[1].y) * inv,
-                    (wM * As[0].z + wR * As[1].z) * inv, (wM * As[0].w + wR * As[1].w) * inv);
+        make_float4(w.x * As[0].x + w.y * As[1].x, w.x * As[0].y + w.y * As[1].y,
+                    w.x * As[0].z + w.y * As[1].z, w.x * As[0].w + w.y * As[1].w);
   }
 }
 

@@ -66,16 +66,9 @@ __device__ __forceinline__ float gate_value(const DecodeParams& p, float lM) {
 // o^ for one head over this lane's 16 dims from the main and residual states.
 __device__ __forceinline__ void finalize(const DecodeParams& p, const SegState& M,
                                          const SegState& R, float* out16) {
-  const float g = gate_value(p, M.l);
-  float wM = 1.0f, wR = 0.0f;
-  if (R.l > 0.0f && g > 0.0f) {
-    const float mx = fmaxf(M.m, R.m);
-    wM = exp2f(M.m - mx);
-    wR = g * exp2f(R.m - mx);
-  }
-  const float inv = 1.0f / (wM * M.l + wR * R.l);
+  const float2 w = branch_coefs(p.softmax_mode, gate_value(p, M.l), M.m, M.l, R.m, R.l);
 #pragma unroll
-  for (int i = 0; i < 16; ++i) out16[i] = (wM * M.acc[i] + wR * R.acc[i]) * inv;
+  for (int i = 0; i < 16; ++i) out16[i] = w.x * M.acc[i] + w.y * R.acc[i];
 }
 
 // Combine state b into a (both in the log2 domain).

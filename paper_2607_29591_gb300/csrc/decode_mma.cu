@@ -134,19 +134,12 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     const int64_t orow = (ul / p.n_kv_heads) * int64_t(p.n_kv_heads) * G + (ul % p.n_kv_heads) * G + h;
     if (ga <= ubase && ge >= uend) {
       if (hv) {
-        const float g = gate_of(p, lMt);
-        float wM = 1.f, wR = 0.f;
-        if (lRt > 0.f && g > 0.f) {
-          const float mx = fmaxf(mM, mR);
-          wM = exp2f(mM - mx);
-          wR = g * exp2f(mR - mx);
-        }
-        const float inv = 1.0f / (wM * lMt + wR * lRt);
+        const float2 w = branch_coefs(p.softmax_mode, gate_of(p, lMt), mM, lMt, mR, lRt);
         float* op = p.O + orow * kHeadDim + 2 * qp;
 #pragma unroll
         for (int dt = 0; dt < 16; ++dt)
           *reinterpret_cast<float2*>(op + dt * 8) =
-              make_float2((wM * O[dt][0] + wR * O[dt][2]) * inv, (wM * O[dt][1] + wR * O[dt][3]) * inv);
+              make_float2(w.x * O[dt][0] + w.y * O[dt][2], w.x * O[dt][1] + w.y * O[dt][3]);
       }
       return;
     }
@@ -206,20 +199,13 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
           }
         }
       }
-      const float g = gate_of(p, Ls[0]);
-      float wM = 1.f, wR = 0.f;
-      if (Ls[1] > 0.f && g > 0.f) {
-        const float mx = fmaxf(Ms[0], Ms[1]);
-        wM = exp2f(Ms[0] - mx);
-        wR = g * exp2f(Ms[1] - mx);
-      }
-      const float inv = 1.0f / (wM * Ls[0] + wR * Ls[1]);
+      const float2 w = branch_coefs(p.softmax_mode, gate_of(p, Ls[0]), Ms[0], Ls[0], Ms[1], Ls[1]);
       float* op = p.O + orow * kHeadDim + 2 * qp;
 #pragma unroll
       for (int dt = 0; dt < 16; ++dt)
         *reinterpret_cast<float2*>(op + dt * 8) =
-            make_float2((wM * acc[0][2 * dt] + wR * acc[1][2 * dt]) * inv,
-                        (wM * acc[0][2 * dt + 1] + wR * acc[1][2 * dt + 1]) * inv);
+            make_float2(w.x * acc[0][2 * dt] + w.y * acc[1][2 * dt],
+                        w.x * acc[0][2 * dt + 1] + w.y * acc[1][2 * dt + 1]);
     }
     __syncwarp();
     if (lane == 0) p.tickets[uu] = 0;

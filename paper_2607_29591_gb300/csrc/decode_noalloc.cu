@@ -145,6 +145,7 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
   p.total_slots = total;
   p.n_warps = int32_t(W);
   p.gate_mode = c->gate_mode;
+  p.softmax_mode = RESKV_SOFTMAX_SHARED;
   p.tau = c->tau;
   p.alpha = c->alpha;
   p.g_min = c->g_min;

@@ -4,6 +4,8 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
+#include "reskv.h"
+
 namespace reskv {
 
 // Device status word codes (written with atomicOr, read by reskv_check_status).
@@ -92,6 +94,23 @@ __device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
   unsigned long long rd;
   asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(rd) : "l"(ra), "l"(rb));
   return *reinterpret_cast<float2*>(&rd);
+}
+
+// Coefficients (a, c) of o^ = a * acc_M + c * acc_R from the two branch
+// states (m: running max in log2 units, l: sum of 2^(logit - m), acc: sum of
+// 2^(logit - m) v) and the gate value g.
+//   RESKV_SOFTMAX_SHARED (Eq. reskv): x = max(mM, mR), wM = 2^(mM - x),
+//     wR = g 2^(mR - x), a = wM / den, c = wR / den, den = wM lM + wR lR;
+//   RESKV_SOFTMAX_SEPARATE (ablation): a = (1 - g) / lM, c = g / lR.
+// Without residual mass (lR = 0) or with g = 0 both are main-only: a = 1 / lM.
+__device__ __forceinline__ float2 branch_coefs(int32_t softmax_mode, float g, float mM, float lM,
+                                               float mR, float lR) {
+  if (!(lR > 0.f) || !(g > 0.f)) return make_float2(1.0f / lM, 0.f);
+  if (softmax_mode == RESKV_SOFTMAX_SEPARATE) return make_float2((1.0f - g) / lM, g / lR);
+  const float x = fmaxf(mM, mR);
+  const float wM = exp2f(mM - x), wR = g * exp2f(mR - x);
+  const float inv = 1.0f / (wM * lM + wR * lR);
+  return make_float2(wM * inv, wR * inv);
 }
 
 __device__ __forceinline__ void report_status(uint32_t* status, uint32_t code) {

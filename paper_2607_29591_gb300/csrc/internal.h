@@ -40,6 +40,7 @@ struct DecodeParams {
   int32_t n_warps;              // W
   int32_t n_stages;             // ring stages per warp (tensor-core kernel)
   int32_t gate_mode;
+  int32_t softmax_mode;         // RESKV_SOFTMAX_*
   float tau, alpha, g_min, g_fixed;
 };
 
@@ -107,4 +108,7 @@ struct reskv_cache {
   double* dbg_losses = nullptr;
   int64_t dbg_n_top = 0;
   std::vector<int32_t> candidates;
+  // device time of the construction stages (ms): scores, ranking, validation
+  // targets, Lloyd, validation losses + choice of r, packing
+  float build_ms[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 };

@@ -55,6 +55,8 @@ reskv_status validate_shape(const reskv_config* cfg) {
   if (cfg->decode_warps < 0) return fail(RESKV_ERR_INVALID_ARG, "decode_warps must be >= 0");
   if (cfg->decode_kernel < RESKV_DECODE_AUTO || cfg->decode_kernel > RESKV_DECODE_CLUSTER)
     return fail(RESKV_ERR_INVALID_ARG, "unknown decode_kernel");
+  if (cfg->softmax_mode != RESKV_SOFTMAX_SHARED && cfg->softmax_mode != RESKV_SOFTMAX_SEPARATE)
+    return fail(RESKV_ERR_INVALID_ARG, "unknown softmax_mode");
   if (double(cfg->n_layers) * cfg->batch * cfg->n_kv_heads * cfg->budget + kLogcPad >=
       double(int64_t(1) << 31))
     return fail(RESKV_ERR_UNSUPPORTED, "at most 2^31 cache slots");
@@ -355,6 +357,7 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   p.n_kv_heads = cfg.n_kv_heads;
   p.total_slots = int64_t(p.n_units) * c->budget;
   p.gate_mode = cfg.gate_mode;
+  p.softmax_mode = cfg.softmax_mode;
   p.tau = cfg.tau;
   p.alpha = cfg.alpha;
   p.g_min = cfg.g_min;
@@ -454,6 +457,7 @@ reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info) {
                           : 0;
   info->all_cluster = auto_plan ? c->cplan_all.cluster
                                 : cluster ? std::max(1, c->cplan_all.cluster) : 0;
+  for (int i = 0; i < 6; ++i) info->build_ms[i] = c->build_ms[i];
   info->all_cluster_warps =
       info->all_cluster ? (c->cplan_all.cluster ? c->cplan_all.warps_per_cta
                                                 : cluster_warps(c->budget, 1))

@@ -22,6 +22,7 @@ STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "OOM", 4: "CUDA"
 RESKV_SCORE_OBS_POOL, RESKV_SCORE_KEYNORM = 0, 1
 RESKV_GATE_DYNAMIC, RESKV_GATE_FIXED = 0, 1
 RESKV_DECODE_AUTO, RESKV_DECODE_FMA, RESKV_DECODE_MMA, RESKV_DECODE_CLUSTER = 0, 1, 2, 3
+RESKV_SOFTMAX_SHARED, RESKV_SOFTMAX_SEPARATE = 0, 1
 RESKV_DEBUG_SCORES, RESKV_DEBUG_RANKED, RESKV_DEBUG_LOSSES, RESKV_DEBUG_CANDIDATES = 0, 1, 2, 3
 MAX_GRID = 8
 
@@ -45,6 +46,7 @@ class reskv_config(ctypes.Structure):
         ("gate_mode", ctypes.c_int32), ("tau", ctypes.c_float), ("alpha", ctypes.c_float),
         ("g_min", ctypes.c_float), ("g_fixed", ctypes.c_float), ("keep_debug", ctypes.c_int32),
         ("decode_warps", ctypes.c_int32), ("decode_kernel", ctypes.c_int32),
+        ("softmax_mode", ctypes.c_int32),
     ]
 
 
@@ -58,7 +60,7 @@ class reskv_cache_info(ctypes.Structure):
                 ("head_dim", ctypes.c_int32), ("slot_bytes", ctypes.c_int64),
                 ("cache_bytes", ctypes.c_int64), ("layer_cluster", ctypes.c_int32),
                 ("layer_cluster_warps", ctypes.c_int32), ("all_cluster", ctypes.c_int32),
-                ("all_cluster_warps", ctypes.c_int32)]
+                ("all_cluster_warps", ctypes.c_int32), ("build_ms", ctypes.c_float * 6)]
 
 
 class reskv_device_cache(ctypes.Structure):
@@ -232,7 +234,9 @@ def reskv_check_status(cache: Cache) -> None:
 def reskv_get_info(cache: Cache) -> dict:
     info = reskv_cache_info()
     _check(load_library().reskv_get_info(cache.handle, ctypes.byref(info)))
-    return {f: getattr(info, f) for f, _ in info._fields_}
+    out = {f: getattr(info, f) for f, _ in info._fields_}
+    out["build_ms"] = list(out["build_ms"])
+    return out
 
 
 def _host_view(arrs: dict) -> reskv_host_cache:

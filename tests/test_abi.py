@@ -78,6 +78,7 @@ def test_defaults_are_the_papers(lib):
     assert cfg.delta == pytest.approx(0.01) and cfg.beta == 1.0
     assert cfg.tau == 0.25 and cfg.alpha == 12.0 and cfg.g_min == 0.0
     assert cfg.gate_mode == R.RESKV_GATE_DYNAMIC and cfg.head_dim == 128
+    assert cfg.softmax_mode == R.RESKV_SOFTMAX_SHARED and cfg.decode_kernel == R.RESKV_DECODE_AUTO
 
 
 def test_host_validation_errors(lib):
@@ -94,4 +95,12 @@ def test_host_validation_errors(lib):
     st = lib.reskv_build_cache(ctypes.byref(cfg), (ctypes.c_void_p * 1)(1), (ctypes.c_void_p * 1)(1),
                                None, None, ctypes.byref(out))
     assert st == 2 and out.value is None
+    cfg.group = 4
+    for field, bad, word in (("softmax_mode", 2, "softmax_mode"), ("decode_kernel", 4, "decode_kernel"),
+                             ("decode_warps", -1, "decode_warps")):
+        setattr(cfg, field, bad)
+        st = lib.reskv_build_cache(ctypes.byref(cfg), (ctypes.c_void_p * 1)(1),
+                                   (ctypes.c_void_p * 1)(1), None, None, ctypes.byref(out))
+        assert st == 1 and word in R.reskv_last_error() and out.value is None, field
+        setattr(cfg, field, 0)
     lib.reskv_free(None)                       # NULL-safe

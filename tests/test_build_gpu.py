@@ -63,7 +63,7 @@ def oracle_config(w, cfg):
         budget=w.budget, recent_window=w.recent_window, n_fit=w.n_fit, n_val=w.n_val,
         score_mode=w.score_mode, residual_override=None if ovr is None else int(ovr[u]),
         delta=float(np.float32(cfg.delta)), gate_mode=cfg.gate_mode, tau=cfg.tau,
-        alpha=cfg.alpha, g_min=cfg.g_min, g_fixed=cfg.g_fixed)
+        alpha=cfg.alpha, g_min=cfg.g_min, g_fixed=cfg.g_fixed, softmax_mode=cfg.softmax_mode)
 
 
 def unit_inputs(Ks, Vs, Qs, w, u):
@@ -92,6 +92,12 @@ def run_case(w, units=None, **cfg_kw):
     Qarg = Qdv if w.n_obs > 0 else None
     cache = R.reskv_build_cache(cfg, Kd, Vd, Qarg)
     R.reskv_check_status(cache)
+    # per-stage device times: scores, ranking and packing always run; the
+    # validation stages exactly when the proxy decides r
+    ms = R.reskv_get_info(cache)["build_ms"]
+    proxy_run = w.residual == "proxy" and w.budget < w.seq_len
+    assert ms[0] > 0 and ms[1] > 0 and ms[5] > 0
+    assert (ms[2] > 0) == proxy_run and (ms[4] > 0) == proxy_run
     lay = R.reskv_export_cache(cache)
     scores = R.reskv_export_debug(cache, R.RESKV_DEBUG_SCORES)
     top = R.reskv_export_debug(cache, R.RESKV_DEBUG_RANKED)
@@ -152,6 +158,15 @@ def test_proxy_short_window_drift_needles():
     w = wl.scaled(wl.WORKLOADS["long_128k_b4"], seq_len=4096, budget=512, batch=1, n_layers=2,
                   n_kv_heads=2, n_obs=32, n_fit=24, n_val=8)
     run_case(w)
+
+
+def test_proxy_separate_softmax_ablation():
+    """The "w/o shared softmax" ablation end to end: the validation proxy scores
+    candidates and decode mixes the separately normalised branches."""
+    w = wl.scaled(wl.WORKLOADS["llama8b_layer_32k"], seq_len=2048, budget=256, batch=2,
+                  n_kv_heads=2)
+    out = run_case(w, softmax_mode=R.RESKV_SOFTMAX_SEPARATE)
+    assert out["worst_rel"] < 2e-3
 
 
 def test_keynorm_drawn_residual():

@@ -47,7 +47,8 @@ def mkcfg(**kw):
 
 def ocfg_from(cfg):
     return orc.OracleConfig(budget=cfg.budget, gate_mode=cfg.gate_mode, tau=cfg.tau,
-                            alpha=cfg.alpha, g_min=cfg.g_min, g_fixed=cfg.g_fixed)
+                            alpha=cfg.alpha, g_min=cfg.g_min, g_fixed=cfg.g_fixed,
+                            softmax_mode=cfg.softmax_mode)
 
 
 def synthetic_layout(L, Bt, H, b, splits, seed_layer=0, s=None):
@@ -300,4 +301,29 @@ def test_launch_sizes(L, Bt, H):
     for l in range(L):
         O_l = run_decode(h, Q[l].contiguous(), layer=l).cpu().numpy()
         assert_output_parity(O_l, ref[l], f"layer {l}, {Bt * H} units")
+    R.reskv_check_status(h)
+
+
+@pytest.mark.parametrize("gate", ["dynamic", "fixed_0.4", "fixed_1"])
+def test_separate_softmax_ablation(gate):
+    """The "w/o shared softmax" ablation (separately normalised branches mixed by
+    the gate) on the ragged 12-unit layout, all-layer and per-layer calls."""
+    L, Bt, H, G, b = 2, 3, 2, 4, 300
+    w, lay = synthetic_layout(L, Bt, H, b, SPLITS)
+    kw = {} if gate == "dynamic" else dict(gate_mode=R.RESKV_GATE_FIXED,
+                                           g_fixed=float(gate.split("_")[1]))
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len, budget=b,
+                softmax_mode=R.RESKV_SOFTMAX_SEPARATE, **kw)
+    h = R.reskv_import_cache(cfg, **lay)
+    Q = queries_for(w, L, Bt, H, G)
+    ref = oracle_decode_all(lay, Q, cfg)
+    O = run_decode(h, Q).cpu().numpy()
+    assert_output_parity(O, ref, f"separate softmax, gate {gate}")
+    for l in range(L):
+        O_l = run_decode(h, Q[l].contiguous(), layer=l).cpu().numpy()
+        assert_output_parity(O_l, ref[l], f"separate softmax, gate {gate}, layer {l}")
+    # the ablation differs from the method where residual mass is present
+    shared = oracle_decode_all(lay, Q, mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G,
+                                             seq_len=w.seq_len, budget=b, **kw))
+    assert errors(ref, shared)[1] > 1e-3
     R.reskv_check_status(h)
