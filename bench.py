@@ -55,9 +55,12 @@ def parse_args():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(wl.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-per-layer", action="store_true")
-    ap.add_argument("--decode-kernel", choices=["auto", "mma", "cluster", "fma"], default="auto",
+    ap.add_argument("--decode-kernel", choices=["auto", "mma", "cluster", "fma", "lse"],
+                    default="auto",
                     help="automatic plan (default: cluster kernel for launches whose units "
-                         "fit on the device at once, else tensor-core stream-K), or one kernel")
+                         "fit on the device at once, else tensor-core stream-K), one kernel, "
+                         "or the paper-style comparison path (lse: main and residual passes "
+                         "merged through log-sum-exp statistics)")
     ap.add_argument("--layers", type=int, default=0,
                     help="use only this many layers (smaller profiling case)")
     return ap.parse_args()
@@ -333,11 +336,14 @@ def main():
         w = wl.scaled(w, n_layers=args.layers, name=f"{w.name}_{args.layers}l")
     n_q = args.steps + args.warmup
     kern = {"auto": R.RESKV_DECODE_AUTO, "mma": R.RESKV_DECODE_MMA,
-            "cluster": R.RESKV_DECODE_CLUSTER, "fma": R.RESKV_DECODE_FMA}[args.decode_kernel]
+            "cluster": R.RESKV_DECODE_CLUSTER, "fma": R.RESKV_DECODE_FMA,
+            "lse": R.RESKV_DECODE_LSE_MERGE}[args.decode_kernel]
     cache, Qdec, build_s = build_workload(w, n_q, device, kern)
     info = R.reskv_get_info(cache)
 
     def plan_name(cs, wpc):
+        if kern == R.RESKV_DECODE_LSE_MERGE:
+            return "paper-style: main pass + residual pass + log-sum-exp merge (3 launches)"
         if cs == 0:
             return "fma" if kern == R.RESKV_DECODE_FMA else "tensor-core stream-K"
         return f"tensor-core cluster: {cs} CTA(s) x {wpc} warps per unit"
@@ -471,7 +477,7 @@ def main():
                  "pack"], [round(x, 3) for x in info["build_ms"]])),
             "e2e": e2e,
             "clocks": clk.summary(),
-            "gpu_launches": args.steps,
+            "gpu_launches": args.steps * (3 if kern == R.RESKV_DECODE_LSE_MERGE else 1),
             "cpu_baseline": cpu,
         }
         print(json.dumps(line), flush=True)

@@ -55,7 +55,8 @@ enum { RESKV_GATE_DYNAMIC = 0, RESKV_GATE_FIXED = 1 };
  * (o^ = o_M without residual mass).  It applies to decode and to the
  * validation proxy of reskv_build_cache. */
 enum { RESKV_SOFTMAX_SHARED = 0, RESKV_SOFTMAX_SEPARATE = 1 };
-enum { RESKV_DECODE_AUTO = 0, RESKV_DECODE_FMA = 1, RESKV_DECODE_MMA = 2, RESKV_DECODE_CLUSTER = 3 };
+enum { RESKV_DECODE_AUTO = 0, RESKV_DECODE_FMA = 1, RESKV_DECODE_MMA = 2, RESKV_DECODE_CLUSTER = 3,
+       RESKV_DECODE_LSE_MERGE = 4 };
 
 #define RESKV_MAX_GRID 8
 
@@ -105,7 +106,11 @@ typedef struct reskv_config {
                               stream-K), 1 CUDA-core fp32x2 FMA, 2 tensor-core
                               stream-K over the launch's slot range, 3
                               tensor-core with one thread-block cluster of 1..8
-                              CTAs per unit (decode_warps ignored)           */
+                              CTAs per unit (decode_warps ignored), 4 the
+                              paper's decode structure for comparison (Sec.
+                              6.1, App. B): main-cache pass and residual pass
+                              merged through log-sum-exp statistics, three
+                              launches (decode_warps ignored)                */
   int32_t softmax_mode;    /* RESKV_SOFTMAX_*                                */
 } reskv_config;
 

@@ -26,6 +26,12 @@
 // ring of cache chunks while the previous kernel on the stream finishes, and
 // waits for it before touching Q or O.
 // The result does not depend on timing: both merges run in a fixed order.
+//
+// The same kernel, instantiated per branch, also gives the paper's own
+// decode structure as a measured comparison (launch_decode_lse): main-cache
+// attention and the residual branch as two passes that write (max, sum,
+// normalised output) per query row, and a merge kernel that combines them
+// through those log-sum-exp statistics and the gate.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -94,7 +100,15 @@ __device__ __forceinline__ void st_cluster(uint32_t local, uint32_t rank, float2
                : "memory");
 }
 
-template <int G>
+// What one launch computes: the fused decode (o^ of Eq. reskv, the library's
+// path), or one branch of the paper-style comparison path (Sec. 6.1, App. B:
+// main-cache attention and residual branch as separate passes merged through
+// log-sum-exp statistics), which writes per query row the branch's running
+// max m, sum l and normalised output o = acc / l to a branch record.
+enum : int { kFused = 0, kMainBranch = 1, kResBranch = 2 };
+constexpr int kBrRec = kHeadDim + 4;    // branch record: m, l, pad, pad, o[d]
+
+template <int G, int kMode>
 __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
     reskv_decode_cluster_kernel(const DecodeParams p, const __grid_constant__ CUtensorMap tmK,
                                 const __grid_constant__ CUtensorMap tmV) {
@@ -115,11 +129,19 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   const int b = p.budget;
   const int ub = u * b;
   // the 16-slot chunks (aligned to 16 global slots) of the unit's whole slot
-  // range, split evenly over the cluster's warps.  The split does not wait for
-  // n_main / n_res: the first copies are in flight before those loads return
-  // (unused tail slots, present only when s < b, are streamed and masked).
-  const int cb = ub & ~(kCh - 1);
-  const int nch = (ub + b - cb + kCh - 1) / kCh;
+  // range, split evenly over the cluster's warps.  The fused split does not
+  // wait for n_main / n_res: the first copies are in flight before those loads
+  // return (unused tail slots, present only when s < b, are streamed and
+  // masked).  A branch pass streams only its own rows.
+  int nm = 0, nr = 0, lo = ub, hi = ub + b;
+  if constexpr (kMode != kFused) {
+    nm = p.n_main[u];
+    nr = p.n_res[u];
+    lo = kMode == kMainBranch ? ub : ub + nm;
+    hi = kMode == kMainBranch ? ub + nm : ub + nm + nr;
+  }
+  const int cb = lo & ~(kCh - 1);
+  const int nch = hi > lo ? (hi - cb + kCh - 1) / kCh : 0;
   const int NW = int(cs) * kW, iw = int(rank) * kW + warp;
   const int k0 = (iw * nch) / NW, k1 = ((iw + 1) * nch) / NW;
   const int nchunks = k1 - k0;
@@ -161,8 +183,15 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   // now (its own prologue and cache copies overlap this kernel's tail) ...
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  const int nm = p.n_main[u], nr = p.n_res[u];
+  if constexpr (kMode == kFused) {
+    nm = p.n_main[u];
+    nr = p.n_res[u];
+  }
   const int ue = ub + nm + nr;                             // used slots [ub, ue)
+  // rows of each branch that this launch folds in (the other branch's range
+  // is empty in a branch pass)
+  const int m_lo = kMode == kResBranch ? 0 : ub, m_hi = kMode == kResBranch ? 0 : ub + nm;
+  const int r_lo = kMode == kMainBranch ? 0 : ub + nm, r_hi = kMode == kMainBranch ? 0 : ue;
   uint32_t off_qk[4], off_pv[8];
   tile_offsets(lane, off_qk, off_pv);
   const float qscale = kLog2e * rsqrtf(float(kHeadDim));
@@ -187,8 +216,8 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
       break;
     }
     waited = k + 1;
-    tile_update(S, base + s * kStageBytes, logc_s + s * kCh, wcb + k * kCh, ub, ub + nm, ub + nm,
-                ue, qa, off_qk, off_pv, qscale, hv, qp);
+    tile_update(S, base + s * kStageBytes, logc_s + s * kCh, wcb + k * kCh, m_lo, m_hi, r_lo,
+                r_hi, qa, off_qk, off_pv, qscale, hv, qp);
     __syncwarp();
     if (k + kSt < nchunks) {
       if (lane == 0) {
@@ -306,16 +335,48 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
       Ls[sg] = l;
       As[sg] = a;
     }
-    const float2 w = branch_coefs(p.softmax_mode, gate_of(p, Ls[0]), Ms[0], Ls[0], Ms[1], Ls[1]);
-    *reinterpret_cast<float4*>(p.O + (orow0 + hh) * kHeadDim + d4) =
-        make_float4(w.x * As[0].x + w.y * As[1].x, w.x * As[0].y + w.y * As[1].y,
-                    w.x * As[0].z + w.y * As[1].z, w.x * As[0].w + w.y * As[1].w);
+    if constexpr (kMode == kFused) {
+      const float2 w = branch_coefs(p.softmax_mode, gate_of(p, Ls[0]), Ms[0], Ls[0], Ms[1], Ls[1]);
+      *reinterpret_cast<float4*>(p.O + (orow0 + hh) * kHeadDim + d4) =
+          make_float4(w.x * As[0].x + w.y * As[1].x, w.x * As[0].y + w.y * As[1].y,
+                      w.x * As[0].z + w.y * As[1].z, w.x * As[0].w + w.y * As[1].w);
+    } else {
+      constexpr int sg = kMode == kMainBranch ? 0 : 1;
+      const float inv = Ls[sg] > 0.f ? 1.0f / Ls[sg] : 0.f;
+      float* br = p.partials + (orow0 + hh) * kBrRec;
+      *reinterpret_cast<float4*>(br + 4 + d4) =
+          make_float4(As[sg].x * inv, As[sg].y * inv, As[sg].z * inv, As[sg].w * inv);
+      if (d4 == 0) *reinterpret_cast<float2*>(br) = make_float2(Ms[sg], Ls[sg]);
+    }
   }
+}
+
+// Paper-style path, last step: merge the two branch records of every query
+// row through their log-sum-exp statistics and the gate.  With the branch
+// states (m, l, o = acc / l), o^ = a l_M o_M + c l_R o_R for the coefficients
+// (a, c) of branch_coefs: Eq. reskv, or the ablation's rule.  Four rows per
+// 128-thread block, four dims per thread.
+__global__ void __launch_bounds__(128) reskv_lse_merge_kernel(const DecodeParams p,
+                                                              int64_t n_rows) {
+  const int64_t row = int64_t(blockIdx.x) * 4 + (threadIdx.x >> 5);
+  if (row >= n_rows) return;
+  const int d4 = 4 * (threadIdx.x & 31);
+  const float* bm = p.partials + row * kBrRec;
+  const float* br = p.partials + (n_rows + row) * kBrRec;
+  const float2 sm = *reinterpret_cast<const float2*>(bm);
+  const float2 sr = *reinterpret_cast<const float2*>(br);
+  const float4 om = *reinterpret_cast<const float4*>(bm + 4 + d4);
+  const float4 orr = *reinterpret_cast<const float4*>(br + 4 + d4);
+  const float2 w = branch_coefs(p.softmax_mode, gate_of(p, sm.y), sm.x, sm.y, sr.x, sr.y);
+  const float a = w.x * sm.y, c = w.y * sr.y;
+  *reinterpret_cast<float4*>(p.O + row * kHeadDim + d4) =
+      make_float4(a * om.x + c * orr.x, a * om.y + c * orr.y, a * om.z + c * orr.z,
+                  a * om.w + c * orr.w);
 }
 
 }  // namespace
 
-template <int G>
+template <int G, int kMode>
 static cudaError_t configure_cluster_g() {
   static std::atomic<unsigned long long> configured{0};
   int dev = 0;
@@ -323,7 +384,7 @@ static cudaError_t configure_cluster_g() {
   if (err != cudaSuccess) return err;
   const unsigned long long bit = 1ull << (dev & 63);
   if (!(configured.load() & bit)) {
-    err = cudaFuncSetAttribute(reskv_decode_cluster_kernel<G>,
+    err = cudaFuncSetAttribute(reskv_decode_cluster_kernel<G, kMode>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
     if (err != cudaSuccess) return err;
     configured.fetch_or(bit);
@@ -331,7 +392,6 @@ static cudaError_t configure_cluster_g() {
   return cudaSuccess;
 }
 
-template <int G>
 static cudaLaunchConfig_t cluster_config(int64_t n_units, int cluster, int warps_per_cta,
                                          cudaStream_t stream, cudaLaunchAttribute* attr) {
   cudaLaunchConfig_t cfg = {};
@@ -350,14 +410,14 @@ static cudaLaunchConfig_t cluster_config(int64_t n_units, int cluster, int warps
   return cfg;
 }
 
-template <int G>
+template <int G, int kMode>
 static int max_active_g(int cluster, int warps_per_cta) {
-  if (configure_cluster_g<G>() != cudaSuccess) return -1;
+  if (configure_cluster_g<G, kMode>() != cudaSuccess) return -1;
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = cluster_config<G>(cluster, cluster, warps_per_cta, nullptr, attr);
+  cudaLaunchConfig_t cfg = cluster_config(cluster, cluster, warps_per_cta, nullptr, attr);
   int n = 0;
   const cudaError_t err =
-      cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(reskv_decode_cluster_kernel<G>), &cfg);
+      cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(reskv_decode_cluster_kernel<G, kMode>), &cfg);
   if (err != cudaSuccess) {
     (void)cudaGetLastError();
     return 0;                          // this shape cannot be launched at all
@@ -365,21 +425,21 @@ static int max_active_g(int cluster, int warps_per_cta) {
   return n;
 }
 
-template <int G>
+template <int G, int kMode>
 static cudaError_t launch_cluster_g(const DecodeParams& p, const CUtensorMap& tk,
                                     const CUtensorMap& tv, int cluster, int warps_per_cta,
                                     cudaStream_t stream) {
-  cudaError_t err = configure_cluster_g<G>();
+  cudaError_t err = configure_cluster_g<G, kMode>();
   if (err != cudaSuccess) return err;
   cudaLaunchAttribute attr[2];
-  cudaLaunchConfig_t cfg = cluster_config<G>(p.n_units, cluster, warps_per_cta, stream, attr);
+  cudaLaunchConfig_t cfg = cluster_config(p.n_units, cluster, warps_per_cta, stream, attr);
   cfg.dynamicSmemBytes = size_t(decode_cluster_smem_bytes(warps_per_cta, p.n_stages, cluster));
   // may start before the previous kernel on the stream has finished (see
   // griddepcontrol.wait in the kernel)
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.numAttrs = 2;
-  err = cudaLaunchKernelEx(&cfg, reskv_decode_cluster_kernel<G>, p, tk, tv);
+  err = cudaLaunchKernelEx(&cfg, reskv_decode_cluster_kernel<G, kMode>, p, tk, tv);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
@@ -391,9 +451,9 @@ cudaError_t launch_decode_cluster(const DecodeParams& p, const CUtensorMap& tk,
       p.n_stages < 1 || p.n_stages > decode_cluster_stages(warps_per_cta, cluster))
     return cudaErrorInvalidValue;
   switch (group) {
-    case 1: return launch_cluster_g<1>(p, tk, tv, cluster, warps_per_cta, stream);
-    case 2: return launch_cluster_g<2>(p, tk, tv, cluster, warps_per_cta, stream);
-    case 4: return launch_cluster_g<4>(p, tk, tv, cluster, warps_per_cta, stream);
+    case 1: return launch_cluster_g<1, kFused>(p, tk, tv, cluster, warps_per_cta, stream);
+    case 2: return launch_cluster_g<2, kFused>(p, tk, tv, cluster, warps_per_cta, stream);
+    case 4: return launch_cluster_g<4, kFused>(p, tk, tv, cluster, warps_per_cta, stream);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -402,11 +462,43 @@ int decode_cluster_max_active(int group, int cluster, int warps_per_cta) {
   if (cluster < 1 || cluster > kMaxCluster || warps_per_cta < 1 || warps_per_cta > kMmaMaxW)
     return 0;
   switch (group) {
-    case 1: return max_active_g<1>(cluster, warps_per_cta);
-    case 2: return max_active_g<2>(cluster, warps_per_cta);
-    case 4: return max_active_g<4>(cluster, warps_per_cta);
+    case 1: return max_active_g<1, kFused>(cluster, warps_per_cta);
+    case 2: return max_active_g<2, kFused>(cluster, warps_per_cta);
+    case 4: return max_active_g<4, kFused>(cluster, warps_per_cta);
     default: return 0;
   }
+}
+
+template <int G>
+static cudaError_t launch_lse_g(const DecodeParams& p, const CUtensorMap& tk,
+                                const CUtensorMap& tv, int cluster, int warps_per_cta,
+                                cudaStream_t stream) {
+  const int64_t n_rows = int64_t(p.n_units) * G;
+  DecodeParams pr = p;
+  pr.partials = p.partials + n_rows * kBrRec;
+  cudaError_t err = launch_cluster_g<G, kMainBranch>(p, tk, tv, cluster, warps_per_cta, stream);
+  if (err == cudaSuccess)
+    err = launch_cluster_g<G, kResBranch>(pr, tk, tv, cluster, warps_per_cta, stream);
+  if (err != cudaSuccess) return err;
+  reskv_lse_merge_kernel<<<unsigned((n_rows + 3) / 4), 128, 0, stream>>>(p, n_rows);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decode_lse(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
+                              int group, int cluster, int warps_per_cta, cudaStream_t stream) {
+  if (cluster < 1 || cluster > kMaxCluster || warps_per_cta < 1 || warps_per_cta > kMmaMaxW ||
+      p.n_stages < 1 || p.n_stages > decode_cluster_stages(warps_per_cta, cluster))
+    return cudaErrorInvalidValue;
+  switch (group) {
+    case 1: return launch_lse_g<1>(p, tk, tv, cluster, warps_per_cta, stream);
+    case 2: return launch_lse_g<2>(p, tk, tv, cluster, warps_per_cta, stream);
+    case 4: return launch_lse_g<4>(p, tk, tv, cluster, warps_per_cta, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+size_t decode_lse_scratch_floats(int64_t n_units, int group) {
+  return size_t(2) * size_t(n_units) * size_t(group) * kBrRec;
 }
 
 // Ring depth for `warps_per_cta` warps next to `cluster` CTA records.

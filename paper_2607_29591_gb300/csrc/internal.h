@@ -61,6 +61,12 @@ cudaError_t launch_decode_cluster(const DecodeParams& p, const CUtensorMap& tk,
                                   int warps_per_cta, cudaStream_t stream);
 int decode_cluster_stages(int warps_per_cta, int cluster);
 int decode_cluster_smem_bytes(int warps_per_cta, int stages, int cluster);
+// The paper-style comparison path: main-branch pass, residual-branch pass (both
+// the cluster kernel on one branch's rows) and a log-sum-exp merge kernel; the
+// branch records go to p.partials, which must hold decode_lse_scratch_floats().
+cudaError_t launch_decode_lse(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
+                              int group, int cluster, int warps_per_cta, cudaStream_t stream);
+size_t decode_lse_scratch_floats(int64_t n_units, int group);
 // How many clusters of that shape the current device holds at once (0: none).
 int decode_cluster_max_active(int group, int cluster, int warps_per_cta);
 // Slots per tensor-core tile and per TMA chunk of the decode kernels.

@@ -53,7 +53,7 @@ reskv_status validate_shape(const reskv_config* cfg) {
   if (cfg->budget < 1 || cfg->budget > (1 << 20))
     return fail(RESKV_ERR_INVALID_ARG, "budget must be in [1, 2^20]");
   if (cfg->decode_warps < 0) return fail(RESKV_ERR_INVALID_ARG, "decode_warps must be >= 0");
-  if (cfg->decode_kernel < RESKV_DECODE_AUTO || cfg->decode_kernel > RESKV_DECODE_CLUSTER)
+  if (cfg->decode_kernel < RESKV_DECODE_AUTO || cfg->decode_kernel > RESKV_DECODE_LSE_MERGE)
     return fail(RESKV_ERR_INVALID_ARG, "unknown decode_kernel");
   if (cfg->softmax_mode != RESKV_SOFTMAX_SHARED && cfg->softmax_mode != RESKV_SOFTMAX_SEPARATE)
     return fail(RESKV_ERR_INVALID_ARG, "unknown softmax_mode");
@@ -184,8 +184,9 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
       (st = dalloc(&c->n_main, size_t(c->n_units), "n_main")) != RESKV_OK ||
       (st = dalloc(&c->n_res, size_t(c->n_units), "n_res")) != RESKV_OK ||
       (st = dalloc(&c->partials,
-                   std::max(decode_partials_floats(c->n_units, c->max_warps, cfg.group),
-                            decode_mma_partials_floats(c->n_units, c->max_warps, cfg.group)),
+                   std::max({decode_partials_floats(c->n_units, c->max_warps, cfg.group),
+                             decode_mma_partials_floats(c->n_units, c->max_warps, cfg.group),
+                             decode_lse_scratch_floats(c->n_units, cfg.group)}),
                    "decode workspace")) != RESKV_OK ||
       (st = dalloc(&c->tickets, size_t(c->n_units), "decode tickets")) != RESKV_OK ||
       (st = dalloc(&c->status, 1, "status word")) != RESKV_OK) {
@@ -366,15 +367,19 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   int kernel = cfg.decode_kernel;
   if (kernel == RESKV_DECODE_AUTO)
     kernel = (cp.cluster > 0 && cfg.decode_warps == 0) ? RESKV_DECODE_CLUSTER : RESKV_DECODE_MMA;
-  if (kernel == RESKV_DECODE_CLUSTER) {
+  if (kernel == RESKV_DECODE_CLUSTER || kernel == RESKV_DECODE_LSE_MERGE) {
     // one cluster per unit; a launch too large for one wave runs single-CTA
     // clusters in several waves
     const int cs = cp.cluster > 0 ? cp.cluster : 1;
     const int wpc = cp.cluster > 0 ? cp.warps_per_cta : cluster_warps(c->budget, 1);
     p.n_warps = int32_t(int64_t(cs) * wpc);
     p.n_stages = decode_cluster_stages(wpc, cs);
-    cudaError_t err = launch_decode_cluster(p, c->tmap_k, c->tmap_v, cfg.group, cs, wpc,
-                                            static_cast<cudaStream_t>(stream));
+    cudaError_t err =
+        kernel == RESKV_DECODE_CLUSTER
+            ? launch_decode_cluster(p, c->tmap_k, c->tmap_v, cfg.group, cs, wpc,
+                                    static_cast<cudaStream_t>(stream))
+            : launch_decode_lse(p, c->tmap_k, c->tmap_v, cfg.group, cs, wpc,
+                                static_cast<cudaStream_t>(stream));
     if (err != cudaSuccess) return cuda_fail(err, "decode launch");
     return RESKV_OK;
   }

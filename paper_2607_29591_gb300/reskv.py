@@ -22,6 +22,7 @@ STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "OOM", 4: "CUDA"
 RESKV_SCORE_OBS_POOL, RESKV_SCORE_KEYNORM = 0, 1
 RESKV_GATE_DYNAMIC, RESKV_GATE_FIXED = 0, 1
 RESKV_DECODE_AUTO, RESKV_DECODE_FMA, RESKV_DECODE_MMA, RESKV_DECODE_CLUSTER = 0, 1, 2, 3
+RESKV_DECODE_LSE_MERGE = 4
 RESKV_SOFTMAX_SHARED, RESKV_SOFTMAX_SEPARATE = 0, 1
 RESKV_DEBUG_SCORES, RESKV_DEBUG_RANKED, RESKV_DEBUG_LOSSES, RESKV_DEBUG_CANDIDATES = 0, 1, 2, 3
 MAX_GRID = 8

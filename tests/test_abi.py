@@ -96,7 +96,7 @@ def test_host_validation_errors(lib):
                                None, None, ctypes.byref(out))
     assert st == 2 and out.value is None
     cfg.group = 4
-    for field, bad, word in (("softmax_mode", 2, "softmax_mode"), ("decode_kernel", 4, "decode_kernel"),
+    for field, bad, word in (("softmax_mode", 2, "softmax_mode"), ("decode_kernel", 5, "decode_kernel"),
                              ("decode_warps", -1, "decode_warps")):
         setattr(cfg, field, bad)
         st = lib.reskv_build_cache(ctypes.byref(cfg), (ctypes.c_void_p * 1)(1),

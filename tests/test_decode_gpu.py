@@ -32,11 +32,13 @@ def lib():
 KERNEL = {"id": R.RESKV_DECODE_MMA}
 
 
-@pytest.fixture(autouse=True, params=[R.RESKV_DECODE_FMA, R.RESKV_DECODE_MMA, R.RESKV_DECODE_CLUSTER],
-                ids=["fma", "mma", "cluster"])
+@pytest.fixture(autouse=True, params=[R.RESKV_DECODE_FMA, R.RESKV_DECODE_MMA, R.RESKV_DECODE_CLUSTER,
+                                      R.RESKV_DECODE_LSE_MERGE],
+                ids=["fma", "mma", "cluster", "lse"])
 def decode_kernel(request):
-    """Every decode test runs on the three kernels: CUDA-core FMA, tensor-core
-    stream-K and tensor-core one-cluster-per-unit."""
+    """Every decode test runs on the four decode paths: CUDA-core FMA,
+    tensor-core stream-K, tensor-core one-cluster-per-unit, and the paper-style
+    comparison path (branch passes merged through log-sum-exp statistics)."""
     KERNEL["id"] = request.param
     yield request.param
 
