@@ -343,7 +343,7 @@ def shared_softmax_decode(q, Kmain, Vmain, Kres, Vres, logc, cfg: OracleConfig,
 def separate_softmax_decode(q, Kmain, Vmain, Kres, Vres, logc, cfg: OracleConfig,
                             return_stats: bool = False):
     """One decode query with separate main and residual normalisations, the
-    "w/o shared softmax" ablation (Sec. 7 ablations, Table ablation_main).
+    "w/o shared softmax" ablation (Sec. 6 ablation study, Table ablation_main).
 
     The paper names the variant but prints no combination rule; the reading
     taken here keeps every other part of the method and mixes the two
@@ -430,6 +430,18 @@ def candidate_valid(s: int, cfg: OracleConfig, r: int) -> bool:
         return False
     n_evicted = s - m
     return r <= n_evicted
+
+
+def append_tokens(cache: UnitCache, k_new: np.ndarray, v_new: np.ndarray,
+                  positions: np.ndarray) -> UnitCache:
+    """Decode-time growth (Sec. 3.1: each decode step appends the new token's
+    key and value): the new tokens join the exact main cache M, so every later
+    decode attends to them exactly and counts them in p_max of the gate.  The
+    residual entries stay as built (no refresh)."""
+    return UnitCache(main_pos=np.concatenate([cache.main_pos, positions]),
+                     kmain=np.vstack([cache.kmain, k_new]), vmain=np.vstack([cache.vmain, v_new]),
+                     kbar=cache.kbar, vbar=cache.vbar, counts=cache.counts, logc=cache.logc,
+                     r=cache.r, losses=cache.losses, scores=cache.scores)
 
 
 def decode_unit(cache: UnitCache, Q: np.ndarray, cfg: OracleConfig) -> np.ndarray:

@@ -197,6 +197,26 @@ def _separate_drop_logc(q, Kmain, Vmain, Kres, Vres, logc, cfg, return_stats=Fal
     return _orig["separate_softmax_decode"](q, Kmain, Vmain, Kres, Vres, lc, cfg, return_stats)
 
 
+def _append_replaces_last_main(cache, k_new, v_new, positions):
+    n = len(positions)
+    return _orig["append_tokens"](orc_unit_drop_last(cache, n), k_new, v_new, positions)
+
+
+def orc_unit_drop_last(cache, n):
+    return core.UnitCache(main_pos=cache.main_pos[:len(cache.main_pos) - n],
+                          kmain=cache.kmain[:len(cache.kmain) - n],
+                          vmain=cache.vmain[:len(cache.vmain) - n], kbar=cache.kbar,
+                          vbar=cache.vbar, counts=cache.counts, logc=cache.logc, r=cache.r)
+
+
+def _append_as_residual(cache, k_new, v_new, positions):
+    return core.UnitCache(main_pos=cache.main_pos, kmain=cache.kmain, vmain=cache.vmain,
+                          kbar=np.vstack([cache.kbar, k_new]), vbar=np.vstack([cache.vbar, v_new]),
+                          counts=np.concatenate([cache.counts, np.ones(len(positions), int)]),
+                          logc=np.concatenate([cache.logc, np.zeros(len(positions))]),
+                          r=cache.r + len(positions))
+
+
 def _attention_full_no_shift(q, K, V):
     a = core.logits(q, K)
     w = np.exp(a)
@@ -229,6 +249,8 @@ MUTANTS = [
     ("attention_full", _attention_full_no_shift),
     ("separate_softmax_decode", _separate_additive),
     ("separate_softmax_decode", _separate_drop_logc),
+    ("append_tokens", _append_replaces_last_main),
+    ("append_tokens", _append_as_residual),
 ]
 
 

@@ -191,6 +191,50 @@ def test_separate_softmax_single_entry_and_count_weighting():
     np.testing.assert_allclose(orc.decode_query(q, K, V, kb, vb, np.log([7.0]), cfg), out, rtol=0)
 
 
+def test_append_without_residual_is_attention_over_main_and_new_tokens():
+    """Sec. 3.1 decode growth: tokens appended to a residual-free cache are
+    attended exactly, so decode is textbook softmax attention over M plus the
+    new tokens (Eq. attn on the grown cache)."""
+    rng = np.random.default_rng(31)
+    d, m, n = 16, 25, 3
+    K, V = bf16ish(rng, (m + n, d)), bf16ish(rng, (m + n, d))
+    q = bf16ish(rng, d, 2.0)
+    base = orc.UnitCache(main_pos=np.arange(m), kmain=K[:m], vmain=V[:m], kbar=np.zeros((0, d)),
+                         vbar=np.zeros((0, d)), counts=np.zeros(0, int), logc=np.zeros(0), r=0)
+    grown = orc.append_tokens(base, K[m:], V[m:], np.arange(100, 100 + n))
+    assert grown.main_pos.tolist() == list(range(m)) + [100, 101, 102]
+    out = orc.decode_unit(grown, q[None, :], _cfg())[0]
+    np.testing.assert_allclose(out, textbook_attention(q, K, V), rtol=1e-12, atol=1e-13)
+
+
+def test_append_counts_in_the_gate_and_keeps_residual_entries():
+    """An appended token with a dominant logit takes all main mass: p_max -> 1,
+    so the dynamic gate falls to sigmoid(alpha (tau - 1)) (Eq. gate) and the
+    residual entries, unchanged by the append, weigh in with that gate."""
+    d = 4
+    q = np.zeros(d)
+    q[0] = 40.0
+    Km = np.zeros((3, d))                        # three main tokens with logit 0
+    Vm = np.zeros((3, d))
+    kb, vb = np.zeros((1, d)), np.ones((1, d))   # one entry, logit log 5
+    base = orc.UnitCache(main_pos=np.arange(3), kmain=Km, vmain=Vm, kbar=kb, vbar=vb,
+                         counts=np.array([5]), logc=np.log([5.0]), r=1)
+    k_new = np.zeros((1, d))
+    k_new[0, 0] = 1.0                            # <q, k_new>/sqrt(d) = 20
+    v_new = np.full((1, d), 2.0)
+    grown = orc.append_tokens(base, k_new, v_new, np.array([7]))
+    assert grown.r == 1 and np.array_equal(grown.kbar, kb) and grown.logc[0] == math.log(5.0)
+    out, st = orc.shared_softmax_decode(q, grown.kmain, grown.vmain, grown.kbar, grown.vbar,
+                                        grown.logc, _cfg(), return_stats=True)
+    e20 = math.exp(20.0)
+    p_max = e20 / (3.0 + e20)
+    g = 1.0 / (1.0 + math.exp(-12.0 * (0.25 - p_max)))
+    np.testing.assert_allclose(st["p_max"], p_max, rtol=1e-15)
+    np.testing.assert_allclose(st["g"], g, rtol=1e-12)
+    expect = (e20 * 2.0 + 5.0 * g * 1.0) / (3.0 + e20 + 5.0 * g)
+    np.testing.assert_allclose(out, expect, rtol=1e-14)
+
+
 def test_gate_closed_forms():
     """Eq. gate with the paper's tau = 0.25, alpha = 12 (App. B), via uniform main caches."""
     gc = golden("gate_closed_forms.json")
