@@ -112,6 +112,9 @@ typedef struct reskv_config {
                               merged through log-sum-exp statistics, three
                               launches (decode_warps ignored)                */
   int32_t softmax_mode;    /* RESKV_SOFTMAX_*                                */
+  int32_t append_capacity; /* A >= 0: slots per unit reserved for tokens
+                              appended at decode time (reskv_append); the
+                              unit stride of the layout is budget + A        */
 } reskv_config;
 
 /* Fill *cfg with the paper's defaults; shape fields are zeroed. */
@@ -165,7 +168,7 @@ reskv_status reskv_check_status(const reskv_cache* c);
 /* Shape of a handle's cache. */
 typedef struct reskv_cache_info {
   int64_t n_units;         /* U = L*B*H_kv, unit u = (l*B + b)*H_kv + h      */
-  int32_t budget;          /* slot stride per unit                           */
+  int32_t budget;          /* b, main + residual slots per unit              */
   int32_t head_dim;
   int64_t slot_bytes;      /* bytes of one K row + one V row                 */
   int64_t cache_bytes;     /* device bytes of K/V slots + log-counts         */
@@ -179,22 +182,30 @@ typedef struct reskv_cache_info {
                               ranking, validation targets o_S, Lloyd residual
                               entries, validation losses + choice of r,
                               packing; zero for an imported cache          */
+  int32_t append_capacity; /* A, slots per unit for appended tokens          */
+  int32_t stride;          /* b + A, slots per unit in the layout            */
+  int32_t max_appended;    /* most tokens appended to any unit so far        */
+  int32_t pad0;
 } reskv_cache_info;
 
 reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info);
 
 /*
  * Host-side view of a cache layout, used by reskv_import_cache (read) and
- * reskv_export_cache (written).  Unit u owns slots [u*b, u*b + b); its first
- * n_main[u] slots are main-cache tokens, the next n_res[u] residual entries.
+ * reskv_export_cache (written).  With stride S = budget + append_capacity,
+ * unit u owns slots [u*S, u*S + S): its first n_main[u] slots are main-cache
+ * tokens, the next n_res[u] residual entries, the next n_app[u] tokens
+ * appended at decode time (exact main rows, reskv_append); the rest is unused.
  *   n_main, n_res : int32 [U]
- *   kslots, vslots: bf16 bit patterns, uint16 [U, b, d]
- *   logc          : fp32 [U, b]; beta*log c_j at residual slots (-inf for an
+ *   kslots, vslots: bf16 bit patterns, uint16 [U, S, d]
+ *   logc          : fp32 [U, S]; beta*log c_j at residual slots (-inf for an
  *                   empty entry), ignored at main slots
- *   slot_pos      : int32 [U, b]; original token position of main slots,
- *                   -1 at residual slots (may be NULL on import)
- *   counts        : int32 [U, b]; c_j at residual slots, 0 at main slots
+ *   slot_pos      : int32 [U, S]; original token position of main slots
+ *                   (appended tokens: s, s+1, ...), -1 at residual slots (may
+ *                   be NULL on import)
+ *   counts        : int32 [U, S]; c_j at residual slots, 0 at main slots
  *                   (may be NULL on import)
+ *   n_app         : int32 [U] (may be NULL on import: none appended)
  */
 typedef struct reskv_host_cache {
   int32_t* n_main;
@@ -204,17 +215,38 @@ typedef struct reskv_host_cache {
   float* logc;
   int32_t* slot_pos;
   int32_t* counts;
+  int32_t* n_app;
 } reskv_host_cache;
 
 /* Build a handle from host arrays (an externally constructed cache; only the
- * shape, gate and budget fields of cfg are used).  Requires 1 <= n_main[u] and
- * n_main[u] + n_res[u] <= budget. */
+ * shape, gate, budget and append_capacity fields of cfg are used).  Requires
+ * 1 <= n_main[u], n_main[u] + n_res[u] <= budget and 0 <= n_app[u] <=
+ * append_capacity. */
 reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache* h,
                                 void* stream, reskv_cache** out);
 
 /* Copy the handle's layout to host arrays (every pointer non-NULL, sized as
  * above).  Synchronises `stream`. */
 reskv_status reskv_export_cache(const reskv_cache* c, reskv_host_cache* h, void* stream);
+
+/*
+ * Append the newest decoded token to the cache: one exact K row and V row per
+ * (batch, KV head) unit of `layer`, after the unit's main and residual slots
+ * (Sec. 3.1: each decode step appends the new token's key and value; Alg. 2
+ * attends over the cache as it stands).  Appended tokens are main-cache tokens
+ * for every later decode: exact rows in the shared softmax, counted in p_max of
+ * the gate.  Residual entries are not refreshed (the paper leaves residual
+ * updates during generation to future work, App. E).
+ *
+ *   layer in [0, L) : K_new, V_new device bf16 [B, H_kv, d]
+ *   layer == -1     : every layer, K_new, V_new [L, B, H_kv, d]
+ *
+ * RESKV_ERR_UNSUPPORTED (nothing written) when a unit of the call has
+ * append_capacity tokens already.  The rows are complete when the stream
+ * reaches the next call on it.
+ */
+reskv_status reskv_append(reskv_cache* c, int32_t layer, const void* K_new, const void* V_new,
+                          void* stream);
 
 enum {
   RESKV_DEBUG_SCORES = 0,  /* fp64 [U, s]: token scores                      */
@@ -251,6 +283,7 @@ reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_d
  * parts that must start at zero, so calls that overlap on the GPU race: order
  * them on one stream (or synchronise between them).
  *
+ * The cache has no appended tokens (budget here is the unit stride).
  *   kslots, vslots : device bf16 [n_units, budget, 128], 16-byte aligned
  *   logc           : device fp32 [n_units, budget] (beta*log c at residual slots)
  *   n_main, n_res  : device int32 [n_units]; the caller guarantees

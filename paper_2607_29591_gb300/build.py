@@ -17,7 +17,7 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libreskv.so")
 SOURCES = ["reskv_api.cu", "decode_kernel.cu", "decode_mma.cu", "decode_cluster.cu",
-           "construct.cu", "decode_noalloc.cu"]
+           "construct.cu", "decode_noalloc.cu", "append.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + INCLUDE,
                 "-I" + CSRC]

@@ -370,7 +370,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
 
     // ---- pack the chosen cache ----
     timing_ok &= timer.mark(kStPack);
-    PackArgs pa{K, V, s, P, b, rank_pos, r_final, chosen, run_off_d, kbar, vbar, ecount,
+    PackArgs pa{K, V, s, P, b, c->stride, rank_pos, r_final, chosen, run_off_d, kbar, vbar, ecount,
                 ent_stride, cfg.beta, int64_t(l) * UL, c->kslots, c->vslots, c->logc,
                 c->slot_pos, c->counts, c->n_main, c->n_res};
     k_pack<<<UL, 1024, 0, stream>>>(pa);

@@ -1037,6 +1037,7 @@ struct PackArgs {
   const __nv_bfloat16* V;
   int64_t s;
   int32_t recent, budget;
+  int32_t stride;              // slots per unit in the cache (budget + append capacity)
   const int32_t* rank_pos;     // [UL, s]
   const int32_t* r_final;      // [UL]
   const int32_t* chosen;       // [UL] run index of the chosen entries (0 = none)
@@ -1064,7 +1065,7 @@ __global__ void __launch_bounds__(1024) k_pack(PackArgs p) {
   const int64_t m = r == 0 ? (p.budget < p.s ? p.budget : p.s) : p.budget - r;
   const int64_t keep = m - p.recent;
   const int32_t* rp = p.rank_pos + int64_t(ul) * p.s;
-  int32_t* spos = p.slot_pos + u * p.budget;
+  int32_t* spos = p.slot_pos + u * p.stride;
   const int64_t chunk = (p.s + blockDim.x - 1) / blockDim.x;
   const int64_t lo = int64_t(threadIdx.x) * chunk, hi = lo + chunk < p.s ? lo + chunk : p.s;
   int mine = 0;
@@ -1088,17 +1089,17 @@ __global__ void __launch_bounds__(1024) k_pack(PackArgs p) {
     const int64_t pos = spos[j];
     const uint2 kw = __ldg(reinterpret_cast<const uint2*>(Ku + pos * kHeadDim) + lane);
     const uint2 vw = __ldg(reinterpret_cast<const uint2*>(Vu + pos * kHeadDim) + lane);
-    reinterpret_cast<uint2*>(p.kslots + (u * p.budget + j) * kHeadDim)[lane] = kw;
-    reinterpret_cast<uint2*>(p.vslots + (u * p.budget + j) * kHeadDim)[lane] = vw;
+    reinterpret_cast<uint2*>(p.kslots + (u * p.stride + j) * kHeadDim)[lane] = kw;
+    reinterpret_cast<uint2*>(p.vslots + (u * p.stride + j) * kHeadDim)[lane] = vw;
     if (lane == 0) {
-      p.counts[u * p.budget + j] = 0;
-      p.logc[u * p.budget + j] = 0.f;
+      p.counts[u * p.stride + j] = 0;
+      p.logc[u * p.stride + j] = 0.f;
     }
   }
   const int c = p.chosen[ul];
   for (int j = w; j < r; j += nw) {
     const int64_t e = int64_t(ul) * p.ent_stride + p.run_off[c] + j;
-    const int64_t slot = u * p.budget + m + j;
+    const int64_t slot = u * p.stride + m + j;
     reinterpret_cast<uint2*>(p.kslots + slot * kHeadDim)[lane] =
         reinterpret_cast<const uint2*>(p.kbar + e * kHeadDim)[lane];
     reinterpret_cast<uint2*>(p.vslots + slot * kHeadDim)[lane] =

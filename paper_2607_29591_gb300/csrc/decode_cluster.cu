@@ -122,23 +122,24 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   const bool hv = h < G;
   const uint32_t cs = cluster_size(), rank = cluster_rank();
 
-  // this cluster's unit, slots [ub, ub + b).  Slot indices fit in 32 bits
-  // (a cache holds fewer than 2^31 slots), so no 64-bit division is needed.
+  // this cluster's unit, slots [ub, ub + stride).  Slot indices fit in 32
+  // bits (a cache holds fewer than 2^31 slots), so no 64-bit division is needed.
   const int ul = int(blockIdx.x / cs);
   const int u = int(p.unit0) + ul;
-  const int b = p.budget;
-  const int ub = u * b;
-  // the 16-slot chunks (aligned to 16 global slots) of the unit's whole slot
-  // range, split evenly over the cluster's warps.  The fused split does not
-  // wait for n_main / n_res: the first copies are in flight before those loads
-  // return (unused tail slots, present only when s < b, are streamed and
-  // masked).  A branch pass streams only its own rows.
-  int nm = 0, nr = 0, lo = ub, hi = ub + b;
+  const int ub = u * p.stride;
+  // the 16-slot chunks (aligned to 16 global slots) of the unit's rows that
+  // may be in use, [ub, ub + span), split evenly over the cluster's warps.
+  // The fused split does not wait for n_main / n_res / n_app: the first copies
+  // are in flight before those loads return (unused rows, present only when
+  // s < b or when units of the launch hold fewer appended rows than others,
+  // are streamed and masked).  A branch pass streams only its own rows.
+  int nm = 0, nr = 0, na = 0, lo = ub, hi = ub + p.span;
   if constexpr (kMode != kFused) {
     nm = p.n_main[u];
     nr = p.n_res[u];
+    na = p.n_app ? p.n_app[u] : 0;
     lo = kMode == kMainBranch ? ub : ub + nm;
-    hi = kMode == kMainBranch ? ub + nm : ub + nm + nr;
+    hi = kMode == kMainBranch ? ub + nm + nr + na : ub + nm + nr;
   }
   const int cb = lo & ~(kCh - 1);
   const int nch = hi > lo ? (hi - cb + kCh - 1) / kCh : 0;
@@ -186,12 +187,13 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   if constexpr (kMode == kFused) {
     nm = p.n_main[u];
     nr = p.n_res[u];
+    na = p.n_app ? p.n_app[u] : 0;
   }
-  const int ue = ub + nm + nr;                             // used slots [ub, ue)
-  // rows of each branch that this launch folds in (the other branch's range
-  // is empty in a branch pass)
-  const int m_lo = kMode == kResBranch ? 0 : ub, m_hi = kMode == kResBranch ? 0 : ub + nm;
-  const int r_lo = kMode == kMainBranch ? 0 : ub + nm, r_hi = kMode == kMainBranch ? 0 : ue;
+  const int ue = ub + nm + nr + na;                        // used slots [ub, ue)
+  // main rows: [m_lo, m_hi) minus the residual rows [r_lo, r_hi) (selected
+  // tokens, then rows appended at decode time); a residual pass has none
+  const int m_lo = kMode == kResBranch ? 0 : ub, m_hi = kMode == kResBranch ? 0 : ue;
+  const int r_lo = ub + nm, r_hi = ub + nm + nr;
   uint32_t off_qk[4], off_pv[8];
   tile_offsets(lane, off_qk, off_pv);
   const float qscale = kLog2e * rsqrtf(float(kHeadDim));
@@ -216,8 +218,8 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
       break;
     }
     waited = k + 1;
-    tile_update(S, base + s * kStageBytes, logc_s + s * kCh, wcb + k * kCh, m_lo, m_hi, r_lo,
-                r_hi, qa, off_qk, off_pv, qscale, hv, qp);
+    tile_update<kMode != kMainBranch>(S, base + s * kStageBytes, logc_s + s * kCh, wcb + k * kCh,
+                                      m_lo, m_hi, r_lo, r_hi, qa, off_qk, off_pv, qscale, hv, qp);
     __syncwarp();
     if (k + kSt < nchunks) {
       if (lane == 0) {

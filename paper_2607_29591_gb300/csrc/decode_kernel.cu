@@ -113,7 +113,7 @@ __global__ void __launch_bounds__(kDecodeWarpsPerCta * 32, 1)
   uint64_t* full = reinterpret_cast<uint64_t*>(wbase + 2 * kRingBytes);
   float* logc_s = reinterpret_cast<float*>(wbase + 2 * kRingBytes + kStages * 8);
 
-  const int64_t b = p.budget;
+  const int64_t b = p.stride;
   const int64_t gbase = p.unit0 * b;                 // global slot of flat index 0
   const int64_t nchunks = (e - a + kChunk - 1) / kChunk;
 
@@ -170,11 +170,15 @@ __global__ void __launch_bounds__(kDecodeWarpsPerCta * 32, 1)
     const int64_t ubase = u * b;
     const int32_t nm = p.n_main[p.unit0 + u];
     const int32_t nr = p.n_res[p.unit0 + u];
+    const int32_t na = p.n_app ? p.n_app[p.unit0 + u] : 0;
     const int64_t main_lo = ubase > a ? ubase : a;
     const int64_t main_hi = (ubase + nm < e) ? ubase + nm : e;
     const int64_t res_lo = (ubase + nm > a) ? ubase + nm : a;
     const int64_t res_hi = (ubase + nm + nr < e) ? ubase + nm + nr : e;
-    if (main_lo >= main_hi && res_lo >= res_hi) continue;   // only unused tail slots here
+    const int64_t app_lo = (ubase + nm + nr > a) ? ubase + nm + nr : a;
+    const int64_t app_hi = (ubase + nm + nr + na < e) ? ubase + nm + nr + na : e;
+    if (main_lo >= main_hi && res_lo >= res_hi && app_lo >= app_hi)
+      continue;                                             // only unused tail slots here
 
     // queries of the G heads of this unit, over this lane's 16 dims, scaled
     // by log2(e)/sqrt(d) so that 2^{s} = e^{a}
@@ -195,9 +199,11 @@ __global__ void __launch_bounds__(kDecodeWarpsPerCta * 32, 1)
       }
     }
 
-    SegState segs[2];                 // [0] main, [1] residual: head `grp`, this lane's dims
+    // [0] main, [1] residual, [2] rows appended at decode time (main rows,
+    // folded into [0] below): head `grp`, this lane's dims
+    SegState segs[3];
 #pragma unroll
-    for (int sgi = 0; sgi < 2; ++sgi) {
+    for (int sgi = 0; sgi < 3; ++sgi) {
       segs[sgi].m = -INFINITY;
       segs[sgi].l = 0.0f;
 #pragma unroll
@@ -205,9 +211,9 @@ __global__ void __launch_bounds__(kDecodeWarpsPerCta * 32, 1)
     }
 
 #pragma unroll
-    for (int sgi = 0; sgi < 2; ++sgi) {
-      const int64_t lo = sgi == 0 ? main_lo : res_lo;
-      const int64_t hi = sgi == 0 ? main_hi : res_hi;
+    for (int sgi = 0; sgi < 3; ++sgi) {
+      const int64_t lo = sgi == 0 ? main_lo : sgi == 1 ? res_lo : app_lo;
+      const int64_t hi = sgi == 0 ? main_hi : sgi == 1 ? res_hi : app_hi;
       if (lo >= hi || failed) continue;
       const bool is_res = sgi == 1;
       release_upto(lo);
@@ -325,9 +331,18 @@ __global__ void __launch_bounds__(kDecodeWarpsPerCta * 32, 1)
       }
     }
     if (failed) break;
+    if (segs[2].l > 0.0f) {            // appended rows join the main softmax state
+      const float mx = fmaxf(segs[0].m, segs[2].m);
+      const float s0 = segs[0].l > 0.0f ? exp2f(segs[0].m - mx) : 0.0f;
+      const float s2 = exp2f(segs[2].m - mx);
+      segs[0].l = segs[0].l * s0 + segs[2].l * s2;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) segs[0].acc[i] = segs[0].acc[i] * s0 + segs[2].acc[i] * s2;
+      segs[0].m = mx;
+    }
 
     // ---- finish the unit, or leave a partial record for the last warp ----
-    const int64_t uend = ubase + nm + nr;
+    const int64_t uend = ubase + nm + nr + na;
     const bool whole = (a <= ubase) && (e >= uend);
     const int64_t orow = (u / p.n_kv_heads) * int64_t(p.n_kv_heads) * G + (u % p.n_kv_heads) * G;
     if (whole) {

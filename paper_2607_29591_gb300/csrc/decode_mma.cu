@@ -52,14 +52,15 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   const int64_t gw = int64_t(blockIdx.x) * kW + warp;
   if (gw >= p.n_warps) return;
   const int64_t T = p.total_slots, W = p.n_warps;
-  const int64_t b = p.budget;
+  const int64_t b = p.stride;
   const int64_t gbase = p.unit0 * b;
   const int64_t ga = gbase + warp_begin(gw, T, W), ge = gbase + warp_begin(gw + 1, T, W);
   if (ga >= ge) return;
   // first unit with used slots in [ga, ge): the piece may start in the unused
-  // tail slots of a unit (n_main + n_res < budget), which this warp must skip
+  // tail slots of a unit (past its n_main + n_res + n_app used rows), which
+  // this warp must skip
   int64_t u = ga / b;
-  if (u * b + p.n_main[u] + p.n_res[u] <= ga) ++u;
+  if (u * b + p.n_main[u] + p.n_res[u] + (p.n_app ? p.n_app[u] : 0) <= ga) ++u;
   if (u * b >= ge) return;
 
   // per-warp shared memory, 1024-byte aligned for the 128-byte swizzle
@@ -103,20 +104,22 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
 
   // unit cursor and its query fragments (the next unit's are loaded ahead)
   uint32_t qa[16], qn[16];
-  int32_t nm = 0, nr = 0, nm_n = 0, nr_n = 0;
-  auto load_q = [&](int64_t uu, uint32_t (&dst)[16], int32_t& m_out, int32_t& r_out) {
+  int32_t nm = 0, nr = 0, nt = 0, nm_n = 0, nr_n = 0, nt_n = 0;   // main, residual, used rows
+  auto load_q = [&](int64_t uu, uint32_t (&dst)[16], int32_t& m_out, int32_t& r_out,
+                    int32_t& t_out) {
     const int64_t ul = uu - p.unit0;
     const int64_t qrow = (ul / p.n_kv_heads) * int64_t(p.n_kv_heads) * G + (ul % p.n_kv_heads) * G + h;
     load_q_frag(p.Q, qrow, hv, qp, dst);
     m_out = p.n_main[uu];
     r_out = p.n_res[uu];
+    t_out = m_out + r_out + (p.n_app ? p.n_app[uu] : 0);
   };
   // Q, O, the partial records and the tickets only after the previous kernel
   // on the stream has completed (before: the cache alone, which no kernel
   // that may run concurrently writes)
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  load_q(u, qa, nm, nr);
-  if ((u + 1) * b < ge) load_q(u + 1, qn, nm_n, nr_n);
+  load_q(u, qa, nm, nr, nt);
+  if ((u + 1) * b < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
 
   TileState S;
   S.reset();
@@ -124,12 +127,12 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   float &mM = S.mM, &lM = S.lM, &mR = S.mR, &lR = S.lR;
 
   // Finish unit uu: write o^ (whole unit in this warp) or a partial record.
-  auto finish = [&](int64_t uu, int32_t um, int32_t ur) {
+  auto finish = [&](int64_t uu, int32_t ut) {
     float lMt = lM + __shfl_xor_sync(0xffffffffu, lM, 1);
     lMt += __shfl_xor_sync(0xffffffffu, lMt, 2);
     float lRt = lR + __shfl_xor_sync(0xffffffffu, lR, 1);
     lRt += __shfl_xor_sync(0xffffffffu, lRt, 2);
-    const int64_t ubase = uu * b, uend = ubase + um + ur;
+    const int64_t ubase = uu * b, uend = ubase + ut;
     const int64_t ul = uu - p.unit0;
     const int64_t orow = (ul / p.n_kv_heads) * int64_t(p.n_kv_heads) * G + (ul % p.n_kv_heads) * G + h;
     if (ga <= ubase && ge >= uend) {
@@ -229,7 +232,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     while (true) {
       const int64_t ubase = u * b;
       const int64_t mlo = ubase > ga ? ubase : ga;
-      const int64_t mhi = (ubase + nm < ge) ? ubase + nm : ge;
+      const int64_t mhi = (ubase + nt < ge) ? ubase + nt : ge;   // main + appended rows
       const int64_t rlo = (ubase + nm > ga) ? ubase + nm : ga;
       const int64_t rhi = (ubase + nm + nr < ge) ? ubase + nm + nr : ge;
       const bool any = (mlo < mhi && mlo < t0 + kCh && mhi > t0) ||
@@ -238,10 +241,10 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
         tile_update(S, st, lc, t0, mlo, mhi, rlo, rhi, qa, off_qk, off_pv,
                     qscale, hv, qp);
       // does unit u end inside this tile (or at the end of the piece)?
-      const int64_t uend = u * b + nm + nr;
+      const int64_t uend = u * b + nt;
       const int64_t stop = uend < ge ? uend : ge;
       if (stop > t0 + kCh) break;                        // continues in the next tile
-      finish(u, nm, nr);
+      finish(u, nt);
       S.reset();
       ++u;
       if (u * b >= ge) {
@@ -252,7 +255,8 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
       for (int i = 0; i < 16; ++i) qa[i] = qn[i];
       nm = nm_n;
       nr = nr_n;
-      if ((u + 1) * b < ge) load_q(u + 1, qn, nm_n, nr_n);
+      nt = nt_n;
+      if ((u + 1) * b < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
     }
     if (done) break;
     __syncwarp();

@@ -17,25 +17,32 @@ constexpr int kSlotRowBytes = kHeadDim * 2;
 constexpr float kLog2e = 1.4426950408889634f;
 
 // Decode split: every launch streams the concatenated slot range of its units
-// ("flat" index x = local_unit * budget + j) and cuts it into n_warps equal
+// ("flat" index x = local_unit * stride + j) and cuts it into n_warps equal
 // contiguous pieces, one per warp.  A unit covered by one warp is finished by
 // that warp; a unit cut between warps is finished by the last of them to
 // arrive, from per-(unit, warp) partial records.
+//
+// Unit u owns slots [u*stride, u*stride + stride), stride = budget + append
+// capacity: n_main exact main rows, n_res residual entries, then n_app exact
+// rows appended at decode time (main rows too); the rest is unused.
 struct DecodeParams {
   const __nv_bfloat16* kslots;  // [U, budget, d] whole cache
   const __nv_bfloat16* vslots;  // [U, budget, d]
   const float* logc;            // [U, budget]  beta*ln c at residual slots
   const int32_t* n_main;        // [U]
   const int32_t* n_res;         // [U]
+  const int32_t* n_app;         // [U] appended rows, or NULL (none)
   const __nv_bfloat16* Q;       // [n_units / H_kv, H_kv*G, d] for this launch
   float* O;                     // same shape as Q, fp32
   float* partials;              // [(n_units + n_warps) * 2 * G * (d + 2)]
   int32_t* tickets;             // [U], zero between launches
   uint32_t* status;             // device status word
   int64_t unit0;                // first unit of the launch
-  int64_t total_slots;          // n_units * budget
+  int64_t total_slots;          // n_units * stride
   int32_t n_units;
-  int32_t budget;
+  int32_t stride;               // slots per unit
+  int32_t span;                 // budget + max n_app over the launch's units: rows
+                                // from a unit's start that may be in use
   int32_t n_kv_heads;
   int32_t n_warps;              // W
   int32_t n_stages;             // ring stages per warp (tensor-core kernel)
@@ -78,6 +85,14 @@ void set_error(const std::string& msg);
 
 }  // namespace reskv
 
+struct reskv_cache;
+namespace reskv {
+// Append one K and V row to each of `n` units starting at global unit `unit0`
+// (K_new, V_new: [n, d] bf16); append.cu.
+cudaError_t launch_append(reskv_cache* c, int64_t unit0, int64_t n, const __nv_bfloat16* K_new,
+                          const __nv_bfloat16* V_new, cudaStream_t stream);
+}  // namespace reskv
+
 // The opaque handle of the C ABI.
 struct reskv_cache {
   reskv_config cfg;             // residual_override cleared
@@ -85,6 +100,9 @@ struct reskv_cache {
   int num_sms = 0;
   int64_t n_units = 0;
   int32_t budget = 0;
+  int32_t append_capacity = 0;
+  int32_t stride = 0;           // budget + append_capacity
+  std::vector<int32_t> n_app_max;   // per layer: max appended rows of its units (host copy)
   // layout (device)
   __nv_bfloat16* kslots = nullptr;
   __nv_bfloat16* vslots = nullptr;
@@ -93,6 +111,7 @@ struct reskv_cache {
   int32_t* counts = nullptr;
   int32_t* n_main = nullptr;
   int32_t* n_res = nullptr;
+  int32_t* n_app = nullptr;
   // decode workspace (device)
   float* partials = nullptr;
   int32_t* tickets = nullptr;

@@ -144,8 +144,11 @@ struct TileState {
 };
 
 // Fold the 16-slot tile staged at `st` (first global slot t0; residual
-// log-counts at lc[0..15]) into `S`.  Slots y in [mlo, mhi) are main-cache
-// slots, slots in [rlo, rhi) residual entries; every other row is masked.
+// log-counts at lc[0..15]) into `S`.  Slots y in [rlo, rhi) are residual
+// entries (folded into the residual state when kResidual; a main-only pass
+// skips them), the other slots in [mlo, mhi) are exact main rows (selected
+// tokens and rows appended at decode time); every other row is masked.
+template <bool kResidual = true>
 __device__ __forceinline__ void tile_update(TileState& S, uint32_t st, const float* lc, int64_t t0,
                                             int64_t mlo, int64_t mhi, int64_t rlo, int64_t rhi,
                                             const uint32_t (&qa)[16], const uint32_t (&off_qk)[4],
@@ -172,8 +175,9 @@ __device__ __forceinline__ void tile_update(TileState& S, uint32_t st, const flo
   for (int e = 0; e < 4; ++e) {
     const int rowi = (e >> 1) * 8 + 2 * qp + (e & 1);
     const int64_t y = t0 + rowi;
-    const bool im = hv && y >= mlo && y < mhi;
-    const bool ir = hv && y >= rlo && y < rhi;
+    const bool in_r = y >= rlo && y < rhi;
+    const bool im = hv && y >= mlo && y < mhi && !in_r;
+    const bool ir = kResidual && hv && in_r;
     sM[e] = im ? sv[e] : -INFINITY;
     sR[e] = ir ? sv[e] + lc[rowi] * kLog2e : -INFINITY;   // + beta log c_j
   }

@@ -57,7 +57,10 @@ reskv_status validate_shape(const reskv_config* cfg) {
     return fail(RESKV_ERR_INVALID_ARG, "unknown decode_kernel");
   if (cfg->softmax_mode != RESKV_SOFTMAX_SHARED && cfg->softmax_mode != RESKV_SOFTMAX_SEPARATE)
     return fail(RESKV_ERR_INVALID_ARG, "unknown softmax_mode");
-  if (double(cfg->n_layers) * cfg->batch * cfg->n_kv_heads * cfg->budget + kLogcPad >=
+  if (cfg->append_capacity < 0 || cfg->append_capacity > (1 << 20))
+    return fail(RESKV_ERR_INVALID_ARG, "append_capacity must be in [0, 2^20]");
+  if (double(cfg->n_layers) * cfg->batch * cfg->n_kv_heads *
+              (double(cfg->budget) + cfg->append_capacity) + kLogcPad >=
       double(int64_t(1) << 31))
     return fail(RESKV_ERR_UNSUPPORTED, "at most 2^31 cache slots");
   if (cfg->gate_mode != RESKV_GATE_DYNAMIC && cfg->gate_mode != RESKV_GATE_FIXED)
@@ -120,6 +123,7 @@ void free_handle(reskv_cache* c) {
   cudaFree(c->counts);
   cudaFree(c->n_main);
   cudaFree(c->n_res);
+  cudaFree(c->n_app);
   cudaFree(c->partials);
   cudaFree(c->tickets);
   cudaFree(c->status);
@@ -173,8 +177,11 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
   }
   c->n_units = int64_t(cfg.n_layers) * cfg.batch * cfg.n_kv_heads;
   c->budget = cfg.budget;
+  c->append_capacity = cfg.append_capacity;
+  c->stride = cfg.budget + cfg.append_capacity;
+  c->n_app_max.assign(size_t(cfg.n_layers), 0);
   c->max_warps = c->num_sms * kDecodeWarpsPerCta;
-  const size_t slots = size_t(c->n_units) * cfg.budget;
+  const size_t slots = size_t(c->n_units) * c->stride;
   reskv_status st = RESKV_OK;
   if ((st = dalloc(&c->kslots, slots * kHeadDim, "cache keys")) != RESKV_OK ||
       (st = dalloc(&c->vslots, slots * kHeadDim, "cache values")) != RESKV_OK ||
@@ -183,6 +190,7 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
       (st = dalloc(&c->counts, slots, "slot counts")) != RESKV_OK ||
       (st = dalloc(&c->n_main, size_t(c->n_units), "n_main")) != RESKV_OK ||
       (st = dalloc(&c->n_res, size_t(c->n_units), "n_res")) != RESKV_OK ||
+      (st = dalloc(&c->n_app, size_t(c->n_units), "n_app")) != RESKV_OK ||
       (st = dalloc(&c->partials,
                    std::max({decode_partials_floats(c->n_units, c->max_warps, cfg.group),
                              decode_mma_partials_floats(c->n_units, c->max_warps, cfg.group),
@@ -198,6 +206,7 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
   if (err == cudaSuccess) err = cudaMemsetAsync(c->logc, 0, (slots + kLogcPad) * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->slot_pos, 0xff, slots * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->counts, 0, slots * 4, stream);
+  if (err == cudaSuccess) err = cudaMemsetAsync(c->n_app, 0, size_t(c->n_units) * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->tickets, 0, size_t(c->n_units) * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->status, 0, 4, stream);
   if (err != cudaSuccess) {
@@ -281,11 +290,19 @@ reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache*
         int64_t(h->n_main[u]) + h->n_res[u] > cfg->budget)
       return fail(RESKV_ERR_INVALID_ARG,
                   "unit " + std::to_string(u) + ": need 1 <= n_main and n_main + n_res <= budget");
+    if (h->n_app && (h->n_app[u] < 0 || h->n_app[u] > cfg->append_capacity))
+      return fail(RESKV_ERR_INVALID_ARG,
+                  "unit " + std::to_string(u) + ": need 0 <= n_app <= append_capacity");
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   reskv_cache* c = nullptr;
   if ((st = alloc_handle(*cfg, s, &c)) != RESKV_OK) return st;
-  const size_t slots = size_t(U) * cfg->budget;
+  if (h->n_app) {
+    const int64_t per_layer = int64_t(cfg->batch) * cfg->n_kv_heads;
+    for (int64_t u = 0; u < U; ++u)
+      c->n_app_max[size_t(u / per_layer)] = std::max(c->n_app_max[size_t(u / per_layer)], h->n_app[u]);
+  }
+  const size_t slots = size_t(U) * c->stride;
   cudaError_t err = cudaMemcpyAsync(c->kslots, h->kslots, slots * kHeadDim * 2,
                                     cudaMemcpyHostToDevice, s);
   if (err == cudaSuccess)
@@ -296,6 +313,8 @@ reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache*
     err = cudaMemcpyAsync(c->n_main, h->n_main, size_t(U) * 4, cudaMemcpyHostToDevice, s);
   if (err == cudaSuccess)
     err = cudaMemcpyAsync(c->n_res, h->n_res, size_t(U) * 4, cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess && h->n_app)
+    err = cudaMemcpyAsync(c->n_app, h->n_app, size_t(U) * 4, cudaMemcpyHostToDevice, s);
   if (err == cudaSuccess && h->slot_pos)
     err = cudaMemcpyAsync(c->slot_pos, h->slot_pos, slots * 4, cudaMemcpyHostToDevice, s);
   if (err == cudaSuccess && h->counts)
@@ -312,10 +331,10 @@ reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache*
 reskv_status reskv_export_cache(const reskv_cache* c, reskv_host_cache* h, void* stream) {
   g_last_error.clear();
   if (!c || !h || !h->n_main || !h->n_res || !h->kslots || !h->vslots || !h->logc ||
-      !h->slot_pos || !h->counts)
+      !h->slot_pos || !h->counts || !h->n_app)
     return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const size_t U = size_t(c->n_units), slots = U * c->budget;
+  const size_t U = size_t(c->n_units), slots = U * c->stride;
   cudaError_t err = cudaMemcpyAsync(h->kslots, c->kslots, slots * kHeadDim * 2,
                                     cudaMemcpyDeviceToHost, s);
   if (err == cudaSuccess)
@@ -327,6 +346,7 @@ reskv_status reskv_export_cache(const reskv_cache* c, reskv_host_cache* h, void*
     err = cudaMemcpyAsync(h->counts, c->counts, slots * 4, cudaMemcpyDeviceToHost, s);
   if (err == cudaSuccess) err = cudaMemcpyAsync(h->n_main, c->n_main, U * 4, cudaMemcpyDeviceToHost, s);
   if (err == cudaSuccess) err = cudaMemcpyAsync(h->n_res, c->n_res, U * 4, cudaMemcpyDeviceToHost, s);
+  if (err == cudaSuccess) err = cudaMemcpyAsync(h->n_app, c->n_app, U * 4, cudaMemcpyDeviceToHost, s);
   if (err == cudaSuccess) err = cudaStreamSynchronize(s);
   if (err != cudaSuccess) return cuda_fail(err, "exporting the cache");
   return RESKV_OK;
@@ -347,6 +367,7 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   p.logc = c->logc;
   p.n_main = c->n_main;
   p.n_res = c->n_res;
+  p.n_app = c->append_capacity > 0 ? c->n_app : nullptr;
   p.Q = static_cast<const __nv_bfloat16*>(Q);
   p.O = static_cast<float*>(O);
   p.partials = c->partials;
@@ -354,9 +375,13 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   p.status = c->status;
   p.unit0 = layer < 0 ? 0 : int64_t(layer) * per_layer;
   p.n_units = int32_t(layer < 0 ? c->n_units : per_layer);
-  p.budget = c->budget;
+  p.stride = c->stride;
+  int32_t app = 0;                     // most appended rows of a unit of the launch
+  for (int l = layer < 0 ? 0 : layer; l < (layer < 0 ? cfg.n_layers : layer + 1); ++l)
+    app = std::max(app, c->n_app_max[size_t(l)]);
+  p.span = c->budget + app;
   p.n_kv_heads = cfg.n_kv_heads;
-  p.total_slots = int64_t(p.n_units) * c->budget;
+  p.total_slots = int64_t(p.n_units) * c->stride;
   p.gate_mode = cfg.gate_mode;
   p.softmax_mode = cfg.softmax_mode;
   p.tau = cfg.tau;
@@ -398,7 +423,7 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
     if (cfg.decode_warps > 0) {
       W = cfg.decode_warps;
     } else {
-      if (p.n_units >= c->num_sms && p.n_units <= 4 * int64_t(c->num_sms) && c->budget <= 256) {
+      if (p.n_units >= c->num_sms && p.n_units <= 4 * int64_t(c->num_sms) && c->stride <= 256) {
         W = p.n_units;                // one warp per unit: no partial records at all
       } else {
         wpc = int(std::min<int64_t>(8, std::max<int64_t>(1, p.total_slots / (int64_t(c->num_sms) * 200))));
@@ -424,6 +449,30 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
           : launch_decode(p, cfg.group, int((W + kDecodeWarpsPerCta - 1) / kDecodeWarpsPerCta),
                           static_cast<cudaStream_t>(stream));
   if (err != cudaSuccess) return cuda_fail(err, "decode launch");
+  return RESKV_OK;
+}
+
+reskv_status reskv_append(reskv_cache* c, int32_t layer, const void* K_new, const void* V_new,
+                          void* stream) {
+  if (!c || !K_new || !V_new) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  const reskv_config& cfg = c->cfg;
+  if (layer < -1 || layer >= cfg.n_layers)
+    return fail(RESKV_ERR_INVALID_ARG, "layer must be -1 or in [0, n_layers)");
+  if (!aligned16(K_new) || !aligned16(V_new))
+    return fail(RESKV_ERR_INVALID_ARG, "K_new and V_new must be 16-byte aligned");
+  const int l0 = layer < 0 ? 0 : layer, l1 = layer < 0 ? cfg.n_layers : layer + 1;
+  for (int l = l0; l < l1; ++l)
+    if (c->n_app_max[size_t(l)] >= c->append_capacity)
+      return fail(RESKV_ERR_UNSUPPORTED, "layer " + std::to_string(l) + ": the append region (" +
+                                             std::to_string(c->append_capacity) +
+                                             " slots per unit) is full");
+  const int64_t per_layer = int64_t(cfg.batch) * cfg.n_kv_heads;
+  cudaError_t err = launch_append(c, int64_t(l0) * per_layer, int64_t(l1 - l0) * per_layer,
+                                  static_cast<const __nv_bfloat16*>(K_new),
+                                  static_cast<const __nv_bfloat16*>(V_new),
+                                  static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return cuda_fail(err, "append launch");
+  for (int l = l0; l < l1; ++l) ++c->n_app_max[size_t(l)];
   return RESKV_OK;
 }
 
@@ -463,6 +512,11 @@ reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info) {
   info->all_cluster = auto_plan ? c->cplan_all.cluster
                                 : cluster ? std::max(1, c->cplan_all.cluster) : 0;
   for (int i = 0; i < 6; ++i) info->build_ms[i] = c->build_ms[i];
+  info->append_capacity = c->append_capacity;
+  info->stride = c->stride;
+  info->max_appended = 0;
+  for (int32_t a : c->n_app_max) info->max_appended = std::max(info->max_appended, a);
+  info->pad0 = 0;
   info->all_cluster_warps =
       info->all_cluster ? (c->cplan_all.cluster ? c->cplan_all.warps_per_cta
                                                 : cluster_warps(c->budget, 1))

@@ -17,6 +17,8 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libreskv.so")
 
 RESKV_OK = 0
+(RESKV_ERR_INVALID_ARG, RESKV_ERR_UNSUPPORTED, RESKV_ERR_OOM, RESKV_ERR_CUDA,
+ RESKV_ERR_DEVICE_STATUS) = 1, 2, 3, 4, 5
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "OOM", 4: "CUDA",
                 5: "DEVICE_STATUS"}
 RESKV_SCORE_OBS_POOL, RESKV_SCORE_KEYNORM = 0, 1
@@ -47,13 +49,13 @@ class reskv_config(ctypes.Structure):
         ("gate_mode", ctypes.c_int32), ("tau", ctypes.c_float), ("alpha", ctypes.c_float),
         ("g_min", ctypes.c_float), ("g_fixed", ctypes.c_float), ("keep_debug", ctypes.c_int32),
         ("decode_warps", ctypes.c_int32), ("decode_kernel", ctypes.c_int32),
-        ("softmax_mode", ctypes.c_int32),
+        ("softmax_mode", ctypes.c_int32), ("append_capacity", ctypes.c_int32),
     ]
 
 
 class reskv_host_cache(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
-                ("n_main", "n_res", "kslots", "vslots", "logc", "slot_pos", "counts")]
+                ("n_main", "n_res", "kslots", "vslots", "logc", "slot_pos", "counts", "n_app")]
 
 
 class reskv_cache_info(ctypes.Structure):
@@ -61,7 +63,9 @@ class reskv_cache_info(ctypes.Structure):
                 ("head_dim", ctypes.c_int32), ("slot_bytes", ctypes.c_int64),
                 ("cache_bytes", ctypes.c_int64), ("layer_cluster", ctypes.c_int32),
                 ("layer_cluster_warps", ctypes.c_int32), ("all_cluster", ctypes.c_int32),
-                ("all_cluster_warps", ctypes.c_int32), ("build_ms", ctypes.c_float * 6)]
+                ("all_cluster_warps", ctypes.c_int32), ("build_ms", ctypes.c_float * 6),
+                ("append_capacity", ctypes.c_int32), ("stride", ctypes.c_int32),
+                ("max_appended", ctypes.c_int32), ("pad0", ctypes.c_int32)]
 
 
 class reskv_device_cache(ctypes.Structure):
@@ -109,6 +113,8 @@ def load_library():
     lib.reskv_export_cache.restype = i32
     lib.reskv_export_debug.argtypes = [vp, i32, vp, sz]
     lib.reskv_export_debug.restype = i32
+    lib.reskv_append.argtypes = [vp, i32, vp, vp, vp]
+    lib.reskv_append.restype = i32
     lib.reskv_decode_attn_noalloc.argtypes = [ctypes.POINTER(reskv_device_cache), vp, vp, vp]
     lib.reskv_decode_attn_noalloc.restype = i32
     _lib = lib
@@ -224,6 +230,19 @@ def reskv_decode_attn(cache: Cache, layer: int, Q, O, stream=None) -> None:
                                             _dptr(O, "torch.float32", "O"), _stream(stream)))
 
 
+def reskv_append(cache: Cache, layer: int, K_new, V_new, stream=None) -> None:
+    """Append one token per (batch, KV head) unit: layer >= 0: K_new, V_new
+    bf16 [B, H_kv, d]; layer == -1: [L, B, H_kv, d]."""
+    c = cache.cfg
+    need = (c.n_layers if layer == -1 else 1) * c.batch * c.n_kv_heads * c.head_dim
+    for name, t in (("K_new", K_new), ("V_new", V_new)):
+        if t.numel() != need:
+            raise ValueError(f"{name} holds {t.numel()} elements; this call needs {need}")
+    _check(load_library().reskv_append(cache.handle, int(layer),
+                                       _dptr(K_new, "torch.bfloat16", "K_new"),
+                                       _dptr(V_new, "torch.bfloat16", "V_new"), _stream(stream)))
+
+
 def reskv_free(cache: Cache) -> None:
     cache.free()
 
@@ -249,21 +268,23 @@ def _host_view(arrs: dict) -> reskv_host_cache:
 
 
 def reskv_import_cache(cfg: reskv_config, n_main, n_res, kslots, vslots, logc,
-                       slot_pos=None, counts=None, stream=None) -> Cache:
+                       slot_pos=None, counts=None, n_app=None, stream=None) -> Cache:
     """Build a handle from host numpy arrays (layout as in include/reskv.h):
-    kslots/vslots uint16 bf16 bits [U, b, d], logc float32 [U, b]."""
+    kslots/vslots uint16 bf16 bits [U, S, d], logc float32 [U, S], with the
+    unit stride S = budget + append_capacity."""
     arrs = dict(n_main=np.ascontiguousarray(n_main, np.int32),
                 n_res=np.ascontiguousarray(n_res, np.int32),
                 kslots=np.ascontiguousarray(kslots, np.uint16),
                 vslots=np.ascontiguousarray(vslots, np.uint16),
                 logc=np.ascontiguousarray(logc, np.float32),
                 slot_pos=None if slot_pos is None else np.ascontiguousarray(slot_pos, np.int32),
-                counts=None if counts is None else np.ascontiguousarray(counts, np.int32))
+                counts=None if counts is None else np.ascontiguousarray(counts, np.int32),
+                n_app=None if n_app is None else np.ascontiguousarray(n_app, np.int32))
     U = cfg.n_layers * cfg.batch * cfg.n_kv_heads
-    b, d = cfg.budget, cfg.head_dim
+    b, d = cfg.budget + cfg.append_capacity, cfg.head_dim
     for k, shape in (("n_main", (U,)), ("n_res", (U,)), ("kslots", (U, b, d)),
                      ("vslots", (U, b, d)), ("logc", (U, b)), ("slot_pos", (U, b)),
-                     ("counts", (U, b))):
+                     ("counts", (U, b)), ("n_app", (U,))):
         if arrs[k] is not None and arrs[k].shape != shape:
             raise ValueError(f"{k} must have shape {shape}, got {arrs[k].shape}")
     h = _host_view(arrs)
@@ -277,11 +298,11 @@ def reskv_export_cache(cache: Cache, stream=None) -> dict:
     """Copy the cache layout to host numpy arrays."""
     cfg = cache.cfg
     U = cfg.n_layers * cfg.batch * cfg.n_kv_heads
-    b, d = cfg.budget, cfg.head_dim
+    b, d = cfg.budget + cfg.append_capacity, cfg.head_dim
     arrs = dict(n_main=np.zeros(U, np.int32), n_res=np.zeros(U, np.int32),
                 kslots=np.zeros((U, b, d), np.uint16), vslots=np.zeros((U, b, d), np.uint16),
                 logc=np.zeros((U, b), np.float32), slot_pos=np.zeros((U, b), np.int32),
-                counts=np.zeros((U, b), np.int32))
+                counts=np.zeros((U, b), np.int32), n_app=np.zeros(U, np.int32))
     h = _host_view(arrs)
     _check(load_library().reskv_export_cache(cache.handle, ctypes.byref(h), _stream(stream)))
     return arrs

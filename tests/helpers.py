@@ -29,6 +29,7 @@ def f64_to_bf16_bits(x) -> np.ndarray:
 
 
 def empty_layout(U: int, b: int, d: int = 128) -> dict:
+    """Import layout of U units with unit stride b (budget + append capacity)."""
     return dict(n_main=np.zeros(U, np.int32), n_res=np.zeros(U, np.int32),
                 kslots=np.zeros((U, b, d), np.uint16), vslots=np.zeros((U, b, d), np.uint16),
                 logc=np.zeros((U, b), np.float32), slot_pos=np.full((U, b), -1, np.int32),
@@ -50,13 +51,19 @@ def put_unit(layout: dict, u: int, cache: "orc.UnitCache"):
 
 
 def unit_from_layout(layout: dict, u: int) -> "orc.UnitCache":
-    """The oracle's view of one unit of a (host) layout."""
+    """The oracle's view of one unit of a (host) layout: main rows, residual
+    entries, then the rows appended at decode time (joined to the main cache)."""
     m, r = int(layout["n_main"][u]), int(layout["n_res"][u])
+    a = int(layout["n_app"][u]) if layout.get("n_app") is not None else 0
     k = orc.bf16_bits_to_f64(layout["kslots"][u])
     v = orc.bf16_bits_to_f64(layout["vslots"][u])
-    return orc.UnitCache(main_pos=layout["slot_pos"][u, :m].copy(), kmain=k[:m], vmain=v[:m],
+    unit = orc.UnitCache(main_pos=layout["slot_pos"][u, :m].copy(), kmain=k[:m], vmain=v[:m],
                          kbar=k[m:m + r], vbar=v[m:m + r], counts=layout["counts"][u, m:m + r],
                          logc=layout["logc"][u, m:m + r].astype(np.float64), r=r)
+    if a:
+        unit = orc.append_tokens(unit, k[m + r:m + r + a], v[m + r:m + r + a],
+                                 layout["slot_pos"][u, m + r:m + r + a].copy())
+    return unit
 
 
 def errors(out: np.ndarray, ref: np.ndarray):
