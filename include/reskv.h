@@ -115,6 +115,10 @@ typedef struct reskv_config {
   int32_t append_capacity; /* A >= 0: slots per unit reserved for tokens
                               appended at decode time (reskv_append); the
                               unit stride of the layout is budget + A        */
+  const int32_t* unit_budgets; /* host [L*B*H_kv] per-unit budgets b_u (AdaKV-
+                              style allocation across heads, App. B), or NULL
+                              for `budget` everywhere.  Unit u then owns
+                              b_u + A slots starting at sum_{v<u} (b_v + A)  */
 } reskv_config;
 
 /* Fill *cfg with the paper's defaults; shape fields are zeroed. */
@@ -183,27 +187,31 @@ typedef struct reskv_cache_info {
                               entries, validation losses + choice of r,
                               packing; zero for an imported cache          */
   int32_t append_capacity; /* A, slots per unit for appended tokens          */
-  int32_t stride;          /* b + A, slots per unit in the layout            */
+  int32_t stride;          /* b + A, slots per unit in the layout; 0 with
+                              per-unit budgets                               */
   int32_t max_appended;    /* most tokens appended to any unit so far        */
-  int32_t pad0;
+  int32_t ragged;          /* 1 with per-unit budgets                        */
+  int64_t total_slots;     /* slots of the layout (sum over units)           */
 } reskv_cache_info;
 
 reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info);
 
 /*
  * Host-side view of a cache layout, used by reskv_import_cache (read) and
- * reskv_export_cache (written).  With stride S = budget + append_capacity,
- * unit u owns slots [u*S, u*S + S): its first n_main[u] slots are main-cache
- * tokens, the next n_res[u] residual entries, the next n_app[u] tokens
- * appended at decode time (exact main rows, reskv_append); the rest is unused.
+ * reskv_export_cache (written).  Unit u owns S_u = b_u + append_capacity
+ * consecutive slots (b_u = budget, or unit_budgets[u]), starting at slot
+ * sum_{v<u} S_v (= u*S with one budget): its first n_main[u] slots are
+ * main-cache tokens, the next n_res[u] residual entries, the next n_app[u]
+ * tokens appended at decode time (exact main rows, reskv_append); the rest is
+ * unused.  With N = sum_u S_u slots:
  *   n_main, n_res : int32 [U]
- *   kslots, vslots: bf16 bit patterns, uint16 [U, S, d]
- *   logc          : fp32 [U, S]; beta*log c_j at residual slots (-inf for an
+ *   kslots, vslots: bf16 bit patterns, uint16 [N, d]
+ *   logc          : fp32 [N]; beta*log c_j at residual slots (-inf for an
  *                   empty entry), ignored at main slots
- *   slot_pos      : int32 [U, S]; original token position of main slots
+ *   slot_pos      : int32 [N]; original token position of main slots
  *                   (appended tokens: s, s+1, ...), -1 at residual slots (may
  *                   be NULL on import)
- *   counts        : int32 [U, S]; c_j at residual slots, 0 at main slots
+ *   counts        : int32 [N]; c_j at residual slots, 0 at main slots
  *                   (may be NULL on import)
  *   n_app         : int32 [U] (may be NULL on import: none appended)
  */
@@ -219,9 +227,9 @@ typedef struct reskv_host_cache {
 } reskv_host_cache;
 
 /* Build a handle from host arrays (an externally constructed cache; only the
- * shape, gate, budget and append_capacity fields of cfg are used).  Requires
- * 1 <= n_main[u], n_main[u] + n_res[u] <= budget and 0 <= n_app[u] <=
- * append_capacity. */
+ * shape, gate, budget, unit_budgets and append_capacity fields of cfg are
+ * used).  Requires 1 <= n_main[u], n_main[u] + n_res[u] <= b_u and
+ * 0 <= n_app[u] <= append_capacity. */
 reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache* h,
                                 void* stream, reskv_cache** out);
 

@@ -24,6 +24,7 @@ struct AppendArgs {
   const int32_t* n_main;
   const int32_t* n_res;
   int32_t* n_app;
+  const int32_t* offsets;       // [U+1] unit starts, or NULL (uniform stride)
   int64_t unit0;
   int32_t stride;
   int32_t capacity;
@@ -40,7 +41,8 @@ __global__ void __launch_bounds__(16) k_append(AppendArgs a) {
     if (t == 0) report_status(a.status, kStatusBadIndex);
     return;
   }
-  const int64_t row = u * a.stride + a.n_main[u] + a.n_res[u] + na;
+  const int64_t ubase = a.offsets ? int64_t(a.offsets[u]) : u * a.stride;
+  const int64_t row = ubase + a.n_main[u] + a.n_res[u] + na;
   reinterpret_cast<uint4*>(a.kslots + row * kHeadDim)[t] =
       reinterpret_cast<const uint4*>(a.K_new + i * kHeadDim)[t];
   reinterpret_cast<uint4*>(a.vslots + row * kHeadDim)[t] =
@@ -63,7 +65,8 @@ __global__ void __launch_bounds__(16) k_append(AppendArgs a) {
 cudaError_t launch_append(reskv_cache* c, int64_t unit0, int64_t n, const __nv_bfloat16* K_new,
                           const __nv_bfloat16* V_new, cudaStream_t stream) {
   AppendArgs a{K_new, V_new, c->kslots, c->vslots, c->logc, c->slot_pos, c->counts,
-               c->n_main, c->n_res, c->n_app, unit0, c->stride, c->append_capacity,
+               c->n_main, c->n_res, c->n_app, c->ragged ? c->offsets : nullptr, unit0,
+               c->stride, c->append_capacity,
                c->cfg.seq_len, c->status};
   k_append<<<unsigned(n), 16, 0, stream>>>(a);
   return cudaGetLastError();

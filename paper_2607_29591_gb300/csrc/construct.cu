@@ -107,6 +107,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
                               const int32_t* override_host, const void* const* Kl,
                               const void* const* Vl, const void* const* Ql, cudaStream_t stream) {
   // ---------------- validation ----------------
+  if (cfg.unit_budgets)
+    return fail(RESKV_ERR_UNSUPPORTED, "per-unit budgets: construction does not take them yet");
   const int64_t s = cfg.seq_len;
   const int b = cfg.budget;
   if (cfg.recent_window < 0) return fail(RESKV_ERR_INVALID_ARG, "recent_window must be >= 0");

@@ -126,14 +126,16 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   // bits (a cache holds fewer than 2^31 slots), so no 64-bit division is needed.
   const int ul = int(blockIdx.x / cs);
   const int u = int(p.unit0) + ul;
-  const int ub = u * p.stride;
+  const int ub = p.offsets ? p.offsets[u] : u * p.stride;
+  const int usize = p.offsets ? p.offsets[u + 1] - ub : p.stride;
   // the 16-slot chunks (aligned to 16 global slots) of the unit's rows that
-  // may be in use, [ub, ub + span), split evenly over the cluster's warps.
+  // may be in use, [ub, ub + usize - tail_unused), split evenly over the
+  // cluster's warps.
   // The fused split does not wait for n_main / n_res / n_app: the first copies
   // are in flight before those loads return (unused rows, present only when
   // s < b or when units of the launch hold fewer appended rows than others,
   // are streamed and masked).  A branch pass streams only its own rows.
-  int nm = 0, nr = 0, na = 0, lo = ub, hi = ub + p.span;
+  int nm = 0, nr = 0, na = 0, lo = ub, hi = ub + usize - p.tail_unused;
   if constexpr (kMode != kFused) {
     nm = p.n_main[u];
     nr = p.n_res[u];

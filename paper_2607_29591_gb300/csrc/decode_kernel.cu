@@ -2,9 +2,10 @@
 // reskv_den, reskv_num, reskv; Sec. 5.5.2 Eq. gate) on sm_103a.
 //
 // One launch covers n_units consecutive (layer, batch, KV head) units of the
-// ragged cache.  Their slots are contiguous in HBM (unit u owns slots
-// [u*b, u*b + b): n_main exact main rows, then n_res residual rows), so the
-// launch reads one flat range of K rows and one of V rows.  That range is cut
+// ragged cache.  Their slots are contiguous in HBM (unit u owns the slots from
+// u*stride, or offsets[u] with per-unit budgets: n_main exact main rows, then
+// n_res residual rows, then rows appended at decode time), so the launch
+// reads one flat range of K rows and one of V rows.  That range is cut
 // into W equal contiguous pieces, one per warp (stream-K at warp grain: every
 // warp streams the same number of bytes whatever the ragged main/residual
 // split).  Each warp
@@ -114,7 +115,11 @@ __global__ void __launch_bounds__(kDecodeWarpsPerCta * 32, 1)
   float* logc_s = reinterpret_cast<float*>(wbase + 2 * kRingBytes + kStages * 8);
 
   const int64_t b = p.stride;
-  const int64_t gbase = p.unit0 * b;                 // global slot of flat index 0
+  // global slot of flat index 0, and the flat index where local unit uu starts
+  const int64_t gbase = p.offsets ? int64_t(p.offsets[p.unit0]) : p.unit0 * b;
+  auto uflat = [&](int64_t uu) -> int64_t {
+    return p.offsets ? int64_t(p.offsets[p.unit0 + uu]) - gbase : uu * b;
+  };
   const int64_t nchunks = (e - a + kChunk - 1) / kChunk;
 
   if (lane == 0) {
@@ -166,8 +171,20 @@ __global__ void __launch_bounds__(kDecodeWarpsPerCta * 32, 1)
 
   const float qscale = kLog2e * rsqrtf(float(kHeadDim));
 
-  for (int64_t u = a / b; u * b < e && !failed; ++u) {
-    const int64_t ubase = u * b;
+  int64_t u_first = 0;                 // last unit starting at or before a
+  if (p.offsets) {
+    int64_t lo = 0, hi = p.n_units;
+    while (hi - lo > 1) {
+      const int64_t mid = (lo + hi) >> 1;
+      if (uflat(mid) <= a) lo = mid;
+      else hi = mid;
+    }
+    u_first = lo;
+  } else {
+    u_first = a / b;
+  }
+  for (int64_t u = u_first; u < p.n_units && uflat(u) < e && !failed; ++u) {
+    const int64_t ubase = uflat(u);
     const int32_t nm = p.n_main[p.unit0 + u];
     const int32_t nr = p.n_res[p.unit0 + u];
     const int32_t na = p.n_app ? p.n_app[p.unit0 + u] : 0;

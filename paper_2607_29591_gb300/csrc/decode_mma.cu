@@ -37,7 +37,8 @@ constexpr int kMaxSt = kMmaMaxSt;
 __device__ __forceinline__ int64_t warp_begin(int64_t w, int64_t T, int64_t W) { return (w * T) / W; }
 __device__ __forceinline__ int64_t warp_of(int64_t x, int64_t T, int64_t W) { return ((x + 1) * W - 1) / T; }
 
-template <int G>
+// kRagged: units at p.offsets[u] (per-unit budgets); otherwise at u * stride.
+template <int G, bool kRagged>
 __global__ void __launch_bounds__(kMaxW * 32, 1)
     reskv_decode_mma_kernel(const DecodeParams p, const __grid_constant__ CUtensorMap tmK,
                             const __grid_constant__ CUtensorMap tmV) {
@@ -53,15 +54,31 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   if (gw >= p.n_warps) return;
   const int64_t T = p.total_slots, W = p.n_warps;
   const int64_t b = p.stride;
-  const int64_t gbase = p.unit0 * b;
+  // first slot of unit uu
+  auto ustart = [&](int64_t uu) -> int64_t {
+    if constexpr (kRagged) return p.offsets[uu];
+    else return uu * b;
+  };
+  const int64_t gbase = ustart(p.unit0);
   const int64_t ga = gbase + warp_begin(gw, T, W), ge = gbase + warp_begin(gw + 1, T, W);
   if (ga >= ge) return;
   // first unit with used slots in [ga, ge): the piece may start in the unused
   // tail slots of a unit (past its n_main + n_res + n_app used rows), which
   // this warp must skip
-  int64_t u = ga / b;
-  if (u * b + p.n_main[u] + p.n_res[u] + (p.n_app ? p.n_app[u] : 0) <= ga) ++u;
-  if (u * b >= ge) return;
+  int64_t u;
+  if constexpr (kRagged) {              // last unit starting at or before ga
+    int64_t lo = p.unit0, hi = p.unit0 + p.n_units;
+    while (hi - lo > 1) {
+      const int64_t mid = (lo + hi) >> 1;
+      if (p.offsets[mid] <= ga) lo = mid;
+      else hi = mid;
+    }
+    u = lo;
+  } else {
+    u = ga / b;
+  }
+  if (ustart(u) + p.n_main[u] + p.n_res[u] + (p.n_app ? p.n_app[u] : 0) <= ga) ++u;
+  if (ustart(u) >= ge) return;
 
   // per-warp shared memory, 1024-byte aligned for the 128-byte swizzle
   const uint32_t raw = smem_u32(smem_raw);
@@ -119,7 +136,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   // that may run concurrently writes)
   asm volatile("griddepcontrol.wait;" ::: "memory");
   load_q(u, qa, nm, nr, nt);
-  if ((u + 1) * b < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
+  if (ustart(u + 1) < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
 
   TileState S;
   S.reset();
@@ -132,7 +149,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     lMt += __shfl_xor_sync(0xffffffffu, lMt, 2);
     float lRt = lR + __shfl_xor_sync(0xffffffffu, lR, 1);
     lRt += __shfl_xor_sync(0xffffffffu, lRt, 2);
-    const int64_t ubase = uu * b, uend = ubase + ut;
+    const int64_t ubase = ustart(uu), uend = ubase + ut;
     const int64_t ul = uu - p.unit0;
     const int64_t orow = (ul / p.n_kv_heads) * int64_t(p.n_kv_heads) * G + (ul % p.n_kv_heads) * G + h;
     if (ga <= ubase && ge >= uend) {
@@ -230,7 +247,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     const float* lc = logc_s + s * kCh;
     // every unit with rows in this tile
     while (true) {
-      const int64_t ubase = u * b;
+      const int64_t ubase = ustart(u);
       const int64_t mlo = ubase > ga ? ubase : ga;
       const int64_t mhi = (ubase + nt < ge) ? ubase + nt : ge;   // main + appended rows
       const int64_t rlo = (ubase + nm > ga) ? ubase + nm : ga;
@@ -241,13 +258,13 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
         tile_update(S, st, lc, t0, mlo, mhi, rlo, rhi, qa, off_qk, off_pv,
                     qscale, hv, qp);
       // does unit u end inside this tile (or at the end of the piece)?
-      const int64_t uend = u * b + nt;
+      const int64_t uend = ubase + nt;
       const int64_t stop = uend < ge ? uend : ge;
       if (stop > t0 + kCh) break;                        // continues in the next tile
       finish(u, nt);
       S.reset();
       ++u;
-      if (u * b >= ge) {
+      if (ustart(u) >= ge) {
         done = true;
         break;
       }
@@ -256,7 +273,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
       nm = nm_n;
       nr = nr_n;
       nt = nt_n;
-      if ((u + 1) * b < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
+      if (ustart(u + 1) < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
     }
     if (done) break;
     __syncwarp();
@@ -276,7 +293,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
 
 }  // namespace
 
-template <int G>
+template <int G, bool kRagged>
 static cudaError_t launch_mma_g(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
                                 int n_ctas, int warps_per_cta, cudaStream_t stream) {
   static std::atomic<unsigned long long> configured{0};
@@ -286,7 +303,7 @@ static cudaError_t launch_mma_g(const DecodeParams& p, const CUtensorMap& tk, co
   if (err != cudaSuccess) return err;
   const unsigned long long bit = 1ull << (dev & 63);
   if (!(configured.load() & bit)) {
-    err = cudaFuncSetAttribute(reskv_decode_mma_kernel<G>,
+    err = cudaFuncSetAttribute(reskv_decode_mma_kernel<G, kRagged>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit);
     if (err != cudaSuccess) return err;
     configured.fetch_or(bit);
@@ -301,17 +318,21 @@ static cudaError_t launch_mma_g(const DecodeParams& p, const CUtensorMap& tk, co
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  err = cudaLaunchKernelEx(&cfg, reskv_decode_mma_kernel<G>, p, tk, tv);
+  err = cudaLaunchKernelEx(&cfg, reskv_decode_mma_kernel<G, kRagged>, p, tk, tv);
   if (err != cudaSuccess) return err;
   return cudaGetLastError();
 }
 
 cudaError_t launch_decode_mma(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
                               int group, int n_ctas, int warps_per_cta, cudaStream_t stream) {
+  const bool ragged = p.offsets != nullptr;
   switch (group) {
-    case 1: return launch_mma_g<1>(p, tk, tv, n_ctas, warps_per_cta, stream);
-    case 2: return launch_mma_g<2>(p, tk, tv, n_ctas, warps_per_cta, stream);
-    case 4: return launch_mma_g<4>(p, tk, tv, n_ctas, warps_per_cta, stream);
+    case 1: return ragged ? launch_mma_g<1, true>(p, tk, tv, n_ctas, warps_per_cta, stream)
+                          : launch_mma_g<1, false>(p, tk, tv, n_ctas, warps_per_cta, stream);
+    case 2: return ragged ? launch_mma_g<2, true>(p, tk, tv, n_ctas, warps_per_cta, stream)
+                          : launch_mma_g<2, false>(p, tk, tv, n_ctas, warps_per_cta, stream);
+    case 4: return ragged ? launch_mma_g<4, true>(p, tk, tv, n_ctas, warps_per_cta, stream)
+                          : launch_mma_g<4, false>(p, tk, tv, n_ctas, warps_per_cta, stream);
     default: return cudaErrorInvalidValue;
   }
 }

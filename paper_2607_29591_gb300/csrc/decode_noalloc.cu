@@ -141,8 +141,9 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
   p.unit0 = 0;
   p.n_units = int32_t(c->n_units);
   p.stride = c->budget;                 // no appended rows: the stride is the budget
-  p.span = c->budget;
+  p.tail_unused = 0;
   p.n_app = nullptr;
+  p.offsets = nullptr;
   p.n_kv_heads = c->n_kv_heads;
   p.total_slots = total;
   p.n_warps = int32_t(W);

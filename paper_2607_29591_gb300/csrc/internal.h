@@ -23,8 +23,10 @@ constexpr float kLog2e = 1.4426950408889634f;
 // arrive, from per-(unit, warp) partial records.
 //
 // Unit u owns slots [u*stride, u*stride + stride), stride = budget + append
-// capacity: n_main exact main rows, n_res residual entries, then n_app exact
-// rows appended at decode time (main rows too); the rest is unused.
+// capacity, or with per-unit budgets [offsets[u], offsets[u+1]) of size
+// budget_u + append capacity: n_main exact main rows, n_res residual entries,
+// then n_app exact rows appended at decode time (main rows too); the rest is
+// unused.
 struct DecodeParams {
   const __nv_bfloat16* kslots;  // [U, budget, d] whole cache
   const __nv_bfloat16* vslots;  // [U, budget, d]
@@ -32,6 +34,7 @@ struct DecodeParams {
   const int32_t* n_main;        // [U]
   const int32_t* n_res;         // [U]
   const int32_t* n_app;         // [U] appended rows, or NULL (none)
+  const int32_t* offsets;       // [U+1] first slot of each unit, or NULL (uniform stride)
   const __nv_bfloat16* Q;       // [n_units / H_kv, H_kv*G, d] for this launch
   float* O;                     // same shape as Q, fp32
   float* partials;              // [(n_units + n_warps) * 2 * G * (d + 2)]
@@ -40,9 +43,10 @@ struct DecodeParams {
   int64_t unit0;                // first unit of the launch
   int64_t total_slots;          // n_units * stride
   int32_t n_units;
-  int32_t stride;               // slots per unit
-  int32_t span;                 // budget + max n_app over the launch's units: rows
-                                // from a unit's start that may be in use
+  int32_t stride;               // slots per unit (uniform layout)
+  int32_t tail_unused;          // append capacity - max n_app over the launch's
+                                // units: rows at the end of every unit that are
+                                // certainly unused
   int32_t n_kv_heads;
   int32_t n_warps;              // W
   int32_t n_stages;             // ring stages per warp (tensor-core kernel)
@@ -101,7 +105,11 @@ struct reskv_cache {
   int64_t n_units = 0;
   int32_t budget = 0;
   int32_t append_capacity = 0;
-  int32_t stride = 0;           // budget + append_capacity
+  int32_t stride = 0;           // budget + append_capacity (uniform layout)
+  bool ragged = false;          // per-unit budgets: units at offsets[u]
+  std::vector<int32_t> h_offsets;   // [U+1] first slot of every unit (host)
+  int64_t total_slots = 0;
+  int32_t max_unit_slots = 0;   // largest b_u + A
   std::vector<int32_t> n_app_max;   // per layer: max appended rows of its units (host copy)
   // layout (device)
   __nv_bfloat16* kslots = nullptr;
@@ -112,6 +120,7 @@ struct reskv_cache {
   int32_t* n_main = nullptr;
   int32_t* n_res = nullptr;
   int32_t* n_app = nullptr;
+  int32_t* offsets = nullptr;   // [U+1]
   // decode workspace (device)
   float* partials = nullptr;
   int32_t* tickets = nullptr;

@@ -59,9 +59,17 @@ reskv_status validate_shape(const reskv_config* cfg) {
     return fail(RESKV_ERR_INVALID_ARG, "unknown softmax_mode");
   if (cfg->append_capacity < 0 || cfg->append_capacity > (1 << 20))
     return fail(RESKV_ERR_INVALID_ARG, "append_capacity must be in [0, 2^20]");
-  if (double(cfg->n_layers) * cfg->batch * cfg->n_kv_heads *
-              (double(cfg->budget) + cfg->append_capacity) + kLogcPad >=
-      double(int64_t(1) << 31))
+  const int64_t n_units = int64_t(cfg->n_layers) * cfg->batch * cfg->n_kv_heads;
+  double slots = double(n_units) * (double(cfg->budget) + cfg->append_capacity);
+  if (cfg->unit_budgets) {
+    slots = 0;
+    for (int64_t u = 0; u < n_units; ++u) {
+      if (cfg->unit_budgets[u] < 1 || cfg->unit_budgets[u] > (1 << 20))
+        return fail(RESKV_ERR_INVALID_ARG, "unit_budgets must be in [1, 2^20]");
+      slots += double(cfg->unit_budgets[u]) + cfg->append_capacity;
+    }
+  }
+  if (slots + kLogcPad >= double(int64_t(1) << 31))
     return fail(RESKV_ERR_UNSUPPORTED, "at most 2^31 cache slots");
   if (cfg->gate_mode != RESKV_GATE_DYNAMIC && cfg->gate_mode != RESKV_GATE_FIXED)
     return fail(RESKV_ERR_INVALID_ARG, "unknown gate_mode");
@@ -124,6 +132,7 @@ void free_handle(reskv_cache* c) {
   cudaFree(c->n_main);
   cudaFree(c->n_res);
   cudaFree(c->n_app);
+  cudaFree(c->offsets);
   cudaFree(c->partials);
   cudaFree(c->tickets);
   cudaFree(c->status);
@@ -148,7 +157,7 @@ reskv_status plan_cluster(const reskv_cache* c, int64_t units, reskv_cache::Clus
   *out = reskv_cache::ClusterPlan{};
   if (units > c->num_sms) return RESKV_OK;
   for (int cs = int(std::min<int64_t>(8, c->num_sms / units)); cs >= 1; --cs) {
-    const int wpc = cluster_warps(c->budget, cs);
+    const int wpc = cluster_warps(c->max_unit_slots, cs);
     const int fit = decode_cluster_max_active(c->cfg.group, cs, wpc);
     if (fit < 0) return fail(RESKV_ERR_CUDA, "querying cluster occupancy of the decode kernel");
     if (fit >= units) {
@@ -181,7 +190,17 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
   c->stride = cfg.budget + cfg.append_capacity;
   c->n_app_max.assign(size_t(cfg.n_layers), 0);
   c->max_warps = c->num_sms * kDecodeWarpsPerCta;
-  const size_t slots = size_t(c->n_units) * c->stride;
+  c->ragged = cfg.unit_budgets != nullptr;
+  c->h_offsets.assign(size_t(c->n_units) + 1, 0);
+  c->max_unit_slots = c->stride;
+  for (int64_t u = 0; u < c->n_units; ++u) {
+    const int32_t su = (c->ragged ? cfg.unit_budgets[u] : cfg.budget) + cfg.append_capacity;
+    c->h_offsets[size_t(u) + 1] = c->h_offsets[size_t(u)] + su;
+    if (c->ragged) c->max_unit_slots = u == 0 ? su : std::max(c->max_unit_slots, su);
+  }
+  c->total_slots = c->h_offsets.back();
+  c->cfg.unit_budgets = nullptr;       // the host array is the caller's
+  const size_t slots = size_t(c->total_slots);
   reskv_status st = RESKV_OK;
   if ((st = dalloc(&c->kslots, slots * kHeadDim, "cache keys")) != RESKV_OK ||
       (st = dalloc(&c->vslots, slots * kHeadDim, "cache values")) != RESKV_OK ||
@@ -191,6 +210,8 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
       (st = dalloc(&c->n_main, size_t(c->n_units), "n_main")) != RESKV_OK ||
       (st = dalloc(&c->n_res, size_t(c->n_units), "n_res")) != RESKV_OK ||
       (st = dalloc(&c->n_app, size_t(c->n_units), "n_app")) != RESKV_OK ||
+      (c->ragged &&
+       (st = dalloc(&c->offsets, size_t(c->n_units) + 1, "unit offsets")) != RESKV_OK) ||
       (st = dalloc(&c->partials,
                    std::max({decode_partials_floats(c->n_units, c->max_warps, cfg.group),
                              decode_mma_partials_floats(c->n_units, c->max_warps, cfg.group),
@@ -207,6 +228,10 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
   if (err == cudaSuccess) err = cudaMemsetAsync(c->slot_pos, 0xff, slots * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->counts, 0, slots * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->n_app, 0, size_t(c->n_units) * 4, stream);
+  if (err == cudaSuccess && c->ragged)
+    err = cudaMemcpyAsync(c->offsets, c->h_offsets.data(), c->h_offsets.size() * 4,
+                          cudaMemcpyHostToDevice, stream);
+  if (err == cudaSuccess && c->ragged) err = cudaStreamSynchronize(stream);   // h_offsets is pageable
   if (err == cudaSuccess) err = cudaMemsetAsync(c->tickets, 0, size_t(c->n_units) * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->status, 0, 4, stream);
   if (err != cudaSuccess) {
@@ -286,8 +311,8 @@ reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache*
     return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
   const int64_t U = int64_t(cfg->n_layers) * cfg->batch * cfg->n_kv_heads;
   for (int64_t u = 0; u < U; ++u) {
-    if (h->n_main[u] < 1 || h->n_res[u] < 0 ||
-        int64_t(h->n_main[u]) + h->n_res[u] > cfg->budget)
+    const int32_t bu = cfg->unit_budgets ? cfg->unit_budgets[u] : cfg->budget;
+    if (h->n_main[u] < 1 || h->n_res[u] < 0 || int64_t(h->n_main[u]) + h->n_res[u] > bu)
       return fail(RESKV_ERR_INVALID_ARG,
                   "unit " + std::to_string(u) + ": need 1 <= n_main and n_main + n_res <= budget");
     if (h->n_app && (h->n_app[u] < 0 || h->n_app[u] > cfg->append_capacity))
@@ -302,7 +327,7 @@ reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache*
     for (int64_t u = 0; u < U; ++u)
       c->n_app_max[size_t(u / per_layer)] = std::max(c->n_app_max[size_t(u / per_layer)], h->n_app[u]);
   }
-  const size_t slots = size_t(U) * c->stride;
+  const size_t slots = size_t(c->total_slots);
   cudaError_t err = cudaMemcpyAsync(c->kslots, h->kslots, slots * kHeadDim * 2,
                                     cudaMemcpyHostToDevice, s);
   if (err == cudaSuccess)
@@ -334,7 +359,7 @@ reskv_status reskv_export_cache(const reskv_cache* c, reskv_host_cache* h, void*
       !h->slot_pos || !h->counts || !h->n_app)
     return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const size_t U = size_t(c->n_units), slots = U * c->stride;
+  const size_t U = size_t(c->n_units), slots = size_t(c->total_slots);
   cudaError_t err = cudaMemcpyAsync(h->kslots, c->kslots, slots * kHeadDim * 2,
                                     cudaMemcpyDeviceToHost, s);
   if (err == cudaSuccess)
@@ -368,6 +393,7 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   p.n_main = c->n_main;
   p.n_res = c->n_res;
   p.n_app = c->append_capacity > 0 ? c->n_app : nullptr;
+  p.offsets = c->ragged ? c->offsets : nullptr;
   p.Q = static_cast<const __nv_bfloat16*>(Q);
   p.O = static_cast<float*>(O);
   p.partials = c->partials;
@@ -379,9 +405,9 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   int32_t app = 0;                     // most appended rows of a unit of the launch
   for (int l = layer < 0 ? 0 : layer; l < (layer < 0 ? cfg.n_layers : layer + 1); ++l)
     app = std::max(app, c->n_app_max[size_t(l)]);
-  p.span = c->budget + app;
+  p.tail_unused = c->append_capacity - app;
   p.n_kv_heads = cfg.n_kv_heads;
-  p.total_slots = int64_t(p.n_units) * c->stride;
+  p.total_slots = c->h_offsets[size_t(p.unit0 + p.n_units)] - c->h_offsets[size_t(p.unit0)];
   p.gate_mode = cfg.gate_mode;
   p.softmax_mode = cfg.softmax_mode;
   p.tau = cfg.tau;
@@ -396,7 +422,7 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
     // one cluster per unit; a launch too large for one wave runs single-CTA
     // clusters in several waves
     const int cs = cp.cluster > 0 ? cp.cluster : 1;
-    const int wpc = cp.cluster > 0 ? cp.warps_per_cta : cluster_warps(c->budget, 1);
+    const int wpc = cp.cluster > 0 ? cp.warps_per_cta : cluster_warps(c->max_unit_slots, 1);
     p.n_warps = int32_t(int64_t(cs) * wpc);
     p.n_stages = decode_cluster_stages(wpc, cs);
     cudaError_t err =
@@ -423,7 +449,8 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
     if (cfg.decode_warps > 0) {
       W = cfg.decode_warps;
     } else {
-      if (p.n_units >= c->num_sms && p.n_units <= 4 * int64_t(c->num_sms) && c->stride <= 256) {
+      if (p.n_units >= c->num_sms && p.n_units <= 4 * int64_t(c->num_sms) &&
+          c->max_unit_slots <= 256 && !c->ragged) {
         W = p.n_units;                // one warp per unit: no partial records at all
       } else {
         wpc = int(std::min<int64_t>(8, std::max<int64_t>(1, p.total_slots / (int64_t(c->num_sms) * 200))));
@@ -500,26 +527,27 @@ reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info) {
   info->budget = c->budget;
   info->head_dim = kHeadDim;
   info->slot_bytes = 2 * kSlotRowBytes;
-  info->cache_bytes = c->n_units * int64_t(c->budget) * (2 * kSlotRowBytes + 4);
+  info->cache_bytes = c->total_slots * (2 * kSlotRowBytes + 4);
   const bool auto_plan = c->cfg.decode_kernel == RESKV_DECODE_AUTO && c->cfg.decode_warps == 0;
   const bool cluster = c->cfg.decode_kernel == RESKV_DECODE_CLUSTER;
   info->layer_cluster = auto_plan ? c->cplan_layer.cluster
                                   : cluster ? std::max(1, c->cplan_layer.cluster) : 0;
   info->layer_cluster_warps =
       info->layer_cluster ? (c->cplan_layer.cluster ? c->cplan_layer.warps_per_cta
-                                                    : cluster_warps(c->budget, 1))
+                                                    : cluster_warps(c->max_unit_slots, 1))
                           : 0;
   info->all_cluster = auto_plan ? c->cplan_all.cluster
                                 : cluster ? std::max(1, c->cplan_all.cluster) : 0;
   for (int i = 0; i < 6; ++i) info->build_ms[i] = c->build_ms[i];
   info->append_capacity = c->append_capacity;
-  info->stride = c->stride;
+  info->stride = c->ragged ? 0 : c->stride;
+  info->total_slots = c->total_slots;
   info->max_appended = 0;
   for (int32_t a : c->n_app_max) info->max_appended = std::max(info->max_appended, a);
-  info->pad0 = 0;
+  info->ragged = c->ragged ? 1 : 0;
   info->all_cluster_warps =
       info->all_cluster ? (c->cplan_all.cluster ? c->cplan_all.warps_per_cta
-                                                : cluster_warps(c->budget, 1))
+                                                : cluster_warps(c->max_unit_slots, 1))
                         : 0;
   return RESKV_OK;
 }

@@ -50,6 +50,7 @@ class reskv_config(ctypes.Structure):
         ("g_min", ctypes.c_float), ("g_fixed", ctypes.c_float), ("keep_debug", ctypes.c_int32),
         ("decode_warps", ctypes.c_int32), ("decode_kernel", ctypes.c_int32),
         ("softmax_mode", ctypes.c_int32), ("append_capacity", ctypes.c_int32),
+        ("unit_budgets", ctypes.POINTER(ctypes.c_int32)),
     ]
 
 
@@ -65,7 +66,8 @@ class reskv_cache_info(ctypes.Structure):
                 ("layer_cluster_warps", ctypes.c_int32), ("all_cluster", ctypes.c_int32),
                 ("all_cluster_warps", ctypes.c_int32), ("build_ms", ctypes.c_float * 6),
                 ("append_capacity", ctypes.c_int32), ("stride", ctypes.c_int32),
-                ("max_appended", ctypes.c_int32), ("pad0", ctypes.c_int32)]
+                ("max_appended", ctypes.c_int32), ("ragged", ctypes.c_int32),
+                ("total_slots", ctypes.c_int64)]
 
 
 class reskv_device_cache(ctypes.Structure):
@@ -168,8 +170,9 @@ class Cache:
 def reskv_config_default(**fields) -> reskv_config:
     """reskv_config with the paper's defaults, then ``fields`` applied.
 
-    ``grid_ratios`` may be a sequence (sets n_grid); ``residual_override`` a
-    numpy int32 array of per-unit r (kept alive on the returned struct).
+    ``grid_ratios`` may be a sequence (sets n_grid); ``residual_override`` and
+    ``unit_budgets`` numpy int32 arrays per unit (kept alive on the returned
+    struct).
     """
     cfg = reskv_config()
     load_library().reskv_config_default(ctypes.byref(cfg))
@@ -179,14 +182,14 @@ def reskv_config_default(**fields) -> reskv_config:
             cfg.n_grid = len(vals)
             for i in range(MAX_GRID):
                 cfg.grid_ratios[i] = vals[i] if i < len(vals) else 0.0
-        elif k == "residual_override":
+        elif k in ("residual_override", "unit_budgets"):
             if v is None:
-                cfg.residual_override = None
-                cfg._override_keepalive = None
+                setattr(cfg, k, None)
+                setattr(cfg, f"_{k}_keepalive", None)
             else:
                 arr = np.ascontiguousarray(v, dtype=np.int32)
-                cfg._override_keepalive = arr
-                cfg.residual_override = arr.ctypes.data_as(ctypes.POINTER(ctypes.c_int32))
+                setattr(cfg, f"_{k}_keepalive", arr)
+                setattr(cfg, k, arr.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)))
         else:
             setattr(cfg, k, v)
     return cfg
@@ -280,11 +283,14 @@ def reskv_import_cache(cfg: reskv_config, n_main, n_res, kslots, vslots, logc,
                 slot_pos=None if slot_pos is None else np.ascontiguousarray(slot_pos, np.int32),
                 counts=None if counts is None else np.ascontiguousarray(counts, np.int32),
                 n_app=None if n_app is None else np.ascontiguousarray(n_app, np.int32))
-    U = cfg.n_layers * cfg.batch * cfg.n_kv_heads
-    b, d = cfg.budget + cfg.append_capacity, cfg.head_dim
-    for k, shape in (("n_main", (U,)), ("n_res", (U,)), ("kslots", (U, b, d)),
-                     ("vslots", (U, b, d)), ("logc", (U, b)), ("slot_pos", (U, b)),
-                     ("counts", (U, b)), ("n_app", (U,))):
+    U, d = cfg.n_layers * cfg.batch * cfg.n_kv_heads, cfg.head_dim
+    N = unit_offsets(cfg)[-1]
+    for k in ("kslots", "vslots", "logc", "slot_pos", "counts"):
+        if arrs[k] is not None:                  # [U, S, ...] or flat [N, ...]
+            arrs[k] = arrs[k].reshape((N, d) if k in ("kslots", "vslots") else (N,))
+    for k, shape in (("n_main", (U,)), ("n_res", (U,)), ("kslots", (N, d)),
+                     ("vslots", (N, d)), ("logc", (N,)), ("slot_pos", (N,)),
+                     ("counts", (N,)), ("n_app", (U,))):
         if arrs[k] is not None and arrs[k].shape != shape:
             raise ValueError(f"{k} must have shape {shape}, got {arrs[k].shape}")
     h = _host_view(arrs)
@@ -297,15 +303,34 @@ def reskv_import_cache(cfg: reskv_config, n_main, n_res, kslots, vslots, logc,
 def reskv_export_cache(cache: Cache, stream=None) -> dict:
     """Copy the cache layout to host numpy arrays."""
     cfg = cache.cfg
-    U = cfg.n_layers * cfg.batch * cfg.n_kv_heads
-    b, d = cfg.budget + cfg.append_capacity, cfg.head_dim
+    U, d = cfg.n_layers * cfg.batch * cfg.n_kv_heads, cfg.head_dim
+    off = unit_offsets(cfg)
+    N = off[-1]
     arrs = dict(n_main=np.zeros(U, np.int32), n_res=np.zeros(U, np.int32),
-                kslots=np.zeros((U, b, d), np.uint16), vslots=np.zeros((U, b, d), np.uint16),
-                logc=np.zeros((U, b), np.float32), slot_pos=np.zeros((U, b), np.int32),
-                counts=np.zeros((U, b), np.int32), n_app=np.zeros(U, np.int32))
+                kslots=np.zeros((N, d), np.uint16), vslots=np.zeros((N, d), np.uint16),
+                logc=np.zeros(N, np.float32), slot_pos=np.zeros(N, np.int32),
+                counts=np.zeros(N, np.int32), n_app=np.zeros(U, np.int32))
     h = _host_view(arrs)
     _check(load_library().reskv_export_cache(cache.handle, ctypes.byref(h), _stream(stream)))
+    if cfg.unit_budgets:                         # ragged: flat arrays plus the unit offsets
+        arrs["offsets"] = off
+    else:                                        # one stride: [U, S, ...]
+        S = cfg.budget + cfg.append_capacity
+        for k in ("kslots", "vslots"):
+            arrs[k] = arrs[k].reshape(U, S, d)
+        for k in ("logc", "slot_pos", "counts"):
+            arrs[k] = arrs[k].reshape(U, S)
     return arrs
+
+
+def unit_offsets(cfg: reskv_config) -> np.ndarray:
+    """First slot of every unit (and the total) for cfg's layout: [U + 1]."""
+    U = cfg.n_layers * cfg.batch * cfg.n_kv_heads
+    if cfg.unit_budgets:
+        sizes = np.ctypeslib.as_array(cfg.unit_budgets, shape=(U,)).astype(np.int64)
+    else:
+        sizes = np.full(U, cfg.budget, np.int64)
+    return np.concatenate([[0], np.cumsum(sizes + cfg.append_capacity)]).astype(np.int64)
 
 
 def reskv_export_debug(cache: Cache, what: int, n_cand: Optional[int] = None) -> np.ndarray:

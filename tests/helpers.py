@@ -55,14 +55,19 @@ def unit_from_layout(layout: dict, u: int) -> "orc.UnitCache":
     entries, then the rows appended at decode time (joined to the main cache)."""
     m, r = int(layout["n_main"][u]), int(layout["n_res"][u])
     a = int(layout["n_app"][u]) if layout.get("n_app") is not None else 0
-    k = orc.bf16_bits_to_f64(layout["kslots"][u])
-    v = orc.bf16_bits_to_f64(layout["vslots"][u])
-    unit = orc.UnitCache(main_pos=layout["slot_pos"][u, :m].copy(), kmain=k[:m], vmain=v[:m],
-                         kbar=k[m:m + r], vbar=v[m:m + r], counts=layout["counts"][u, m:m + r],
-                         logc=layout["logc"][u, m:m + r].astype(np.float64), r=r)
+    if "offsets" in layout:                      # per-unit budgets: flat arrays
+        o0, o1 = int(layout["offsets"][u]), int(layout["offsets"][u + 1])
+        view = {k: layout[k][o0:o1] for k in ("kslots", "vslots", "logc", "slot_pos", "counts")}
+    else:
+        view = {k: layout[k][u] for k in ("kslots", "vslots", "logc", "slot_pos", "counts")}
+    k = orc.bf16_bits_to_f64(view["kslots"])
+    v = orc.bf16_bits_to_f64(view["vslots"])
+    unit = orc.UnitCache(main_pos=view["slot_pos"][:m].copy(), kmain=k[:m], vmain=v[:m],
+                         kbar=k[m:m + r], vbar=v[m:m + r], counts=view["counts"][m:m + r],
+                         logc=view["logc"][m:m + r].astype(np.float64), r=r)
     if a:
         unit = orc.append_tokens(unit, k[m + r:m + r + a], v[m + r:m + r + a],
-                                 layout["slot_pos"][u, m + r:m + r + a].copy())
+                                 view["slot_pos"][m + r:m + r + a].copy())
     return unit
 
 
