@@ -31,7 +31,13 @@ the project's design notes):
 * stored residual entries are rounded to bf16 (round-to-nearest-even); the
   validation loss is evaluated on the stored (rounded) entries;
 * the validation loss averages over validation queries and the G query heads
-  of the KV head.
+  of the KV head;
+* AdaKV budgets (App. B, "AdaKV": SnapKV scores, safeguard 0.2): the KV heads
+  of one (layer, batch element) share H*b slots; every head keeps its window
+  P and its own f = floor(safeguard * (b - |P|)) best tokens, and the other
+  H*(b - |P| - f) slots go to the best-scored remaining tokens of all heads
+  (ties: lower head, then lower position); each head is then built by Alg. 1
+  with its own budget b_h.
 
 Parity status: every function here is pinned by ``tests/test_oracle_pins.py``
 against closed forms, fixed points or hand-computed fixtures; none is
@@ -40,7 +46,7 @@ LongBench) are not reproducible here (no model weights or benchmark data).
 """
 from __future__ import annotations
 
-from dataclasses import dataclass, field
+from dataclasses import dataclass, field, replace
 from typing import Optional, Sequence
 
 import numpy as np
@@ -222,6 +228,53 @@ def candidate_budgets(budget: int, ratios: Sequence[float]) -> list:
         if r > 0:
             rs.add(r)
     return sorted(rs)
+
+
+def adakv_budgets(scores: np.ndarray, budget: int, recent: int, safeguard: float) -> np.ndarray:
+    """Per-head budgets b_h of one (layer, batch element) under AdaKV's
+    allocation across KV heads (App. B, "AdaKV": SnapKV token scores, safeguard
+    coefficient 0.2).
+
+    ``scores``: [H, s], one row per KV head.  The paper gives no formula; the
+    reading taken: the H heads share H*b slots.  Every head keeps its protected
+    window P (Eq. main_selection) and, as the safeguard, its own
+    f = floor(safeguard * (b - |P|)) highest-ranked tokens.  The remaining
+    H*(b - |P| - f) slots go to the highest scores among all heads' other
+    evictable tokens, ordered by score (descending), then head index, then
+    position.  b_h = |P| + f + (tokens of head h in that pick).  Within a head
+    the pick is a prefix of its ranking, so head h keeps exactly its top
+    b_h - |P| ranked tokens, the main selection of Alg. 1 with budget b_h.
+    With b >= s nothing is evicted and every head keeps b.
+    """
+    H, s = scores.shape
+    if budget >= s:
+        return np.full(H, budget, dtype=np.int64)
+    n_p = min(recent, s)
+    n = budget - n_p
+    if n < 0:
+        raise ValueError("budget smaller than the protected window")
+    f = int(np.floor(float(np.float32(safeguard)) * n))
+    f = min(max(f, 0), n)
+    # every head's evictable tokens beyond its safeguard, as (score, head, position)
+    sc, hd, ps = [], [], []
+    for h in range(H):
+        rest = rank_evictable(scores[h], recent)[f:]
+        sc.append(scores[h][rest])
+        hd.append(np.full(len(rest), h))
+        ps.append(rest)
+    sc, hd, ps = np.concatenate(sc), np.concatenate(hd), np.concatenate(ps)
+    order = np.lexsort((ps, hd, -sc))           # score desc, then head, then position
+    picked = hd[order[:H * (n - f)]]
+    return n_p + f + np.bincount(picked, minlength=H).astype(np.int64)
+
+
+def unit_scores(K: np.ndarray, Qobs: Optional[np.ndarray], cfg: "OracleConfig") -> np.ndarray:
+    """Token scores of one unit under cfg's score mode (Alg. 1, scoring step)."""
+    if cfg.score_mode == SCORE_OBS_POOL:
+        return scores_obs_pool(K, Qobs[:, :cfg.n_fit], cfg.pool_kernel)
+    if cfg.score_mode == SCORE_KEYNORM:
+        return scores_keynorm(K)
+    raise ValueError("unknown score mode")
 
 
 # ---------------------------------------------------------------------------
@@ -486,12 +539,7 @@ def build_unit(K: np.ndarray, V: np.ndarray, Qobs: Optional[np.ndarray],
     """
     s = K.shape[0]
     # token scores on the fit queries; recent protection P
-    if cfg.score_mode == SCORE_OBS_POOL:
-        scores = scores_obs_pool(K, Qobs[:, :cfg.n_fit], cfg.pool_kernel)
-    elif cfg.score_mode == SCORE_KEYNORM:
-        scores = scores_keynorm(K)
-    else:
-        raise ValueError("unknown score mode")
+    scores = unit_scores(K, Qobs, cfg)
     ranked = rank_evictable(scores, cfg.recent_window)
 
     if cfg.budget >= s:                        # the budget covers every token: M = S
@@ -527,3 +575,22 @@ def build_unit(K: np.ndarray, V: np.ndarray, Qobs: Optional[np.ndarray],
     out = built[r_star] if r_star > 0 else c0
     out.scores, out.ranked, out.losses = scores, ranked, losses
     return out
+
+
+def build_heads_adakv(Ks: np.ndarray, Vs: np.ndarray, Qobs: Optional[np.ndarray],
+                      cfgs: Sequence["OracleConfig"], safeguard: float):
+    """AdaKV allocation across the H KV heads of one (layer, batch element),
+    then Alg. 1 for every head with its own budget (App. B, "AdaKV" with
+    ResKV on top: Table ruler_paper, Table longbench_paper "+ResKV" rows).
+
+    ``Ks``, ``Vs``: [H, s, d]; ``Qobs``: [H, G, n_obs, d] or None; ``cfgs``: one
+    OracleConfig per head carrying the shared budget b (they may differ in
+    residual_override).  Returns (budgets [H], list of UnitCache).
+    """
+    H = Ks.shape[0]
+    scores = np.stack([unit_scores(Ks[h], None if Qobs is None else Qobs[h], cfgs[h])
+                       for h in range(H)])
+    budgets = adakv_budgets(scores, cfgs[0].budget, cfgs[0].recent_window, safeguard)
+    units = [build_unit(Ks[h], Vs[h], None if Qobs is None else Qobs[h],
+                        replace(cfgs[h], budget=int(budgets[h]))) for h in range(H)]
+    return budgets, units

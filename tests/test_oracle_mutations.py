@@ -223,6 +223,46 @@ def _attention_full_no_shift(q, K, V):
     return (w @ V) / (w.sum() + 1.0)
 
 
+
+def _adakv_generic(scores, budget, recent, safeguard, *, head_desc=False, pool_all=False,
+                   f_of=None, n_of=None):
+    """AdaKV allocation with one planted deviation (see the mutants below)."""
+    H, s = scores.shape
+    if budget >= s:
+        return np.full(H, budget, dtype=np.int64)
+    n_p = min(recent, s)
+    n = n_of(budget, n_p) if n_of else budget - n_p
+    f = f_of(safeguard, n) if f_of else int(np.floor(float(np.float32(safeguard)) * n))
+    f = min(max(f, 0), n)
+    sc, hd, ps = [], [], []
+    for h in range(H):
+        rest = core.rank_evictable(scores[h], recent)[0 if pool_all else f:]
+        sc.append(scores[h][rest])
+        hd.append(np.full(len(rest), h))
+        ps.append(rest)
+    sc, hd, ps = np.concatenate(sc), np.concatenate(hd), np.concatenate(ps)
+    order = np.lexsort((ps, -hd if head_desc else hd, -sc))
+    picked = hd[order[:H * (n - f)]]
+    return n_p + f + np.bincount(picked, minlength=H).astype(np.int64)
+
+
+def _adakv_ties_high_head(scores, budget, recent, safeguard):
+    return _adakv_generic(scores, budget, recent, safeguard, head_desc=True)
+
+
+def _adakv_pool_includes_safeguard(scores, budget, recent, safeguard):
+    return _adakv_generic(scores, budget, recent, safeguard, pool_all=True)
+
+
+def _adakv_safeguard_rounded(scores, budget, recent, safeguard):
+    return _adakv_generic(scores, budget, recent, safeguard,
+                          f_of=lambda sg, n: int(round(float(np.float32(sg)) * n)))
+
+
+def _adakv_window_not_protected(scores, budget, recent, safeguard):
+    return _adakv_generic(scores, budget, recent, safeguard, n_of=lambda b, n_p: b)
+
+
 MUTANTS = [
     ("logits", _logits_over_d),
     ("shared_softmax_decode", _decode_drop_logc),
@@ -251,6 +291,10 @@ MUTANTS = [
     ("separate_softmax_decode", _separate_drop_logc),
     ("append_tokens", _append_replaces_last_main),
     ("append_tokens", _append_as_residual),
+    ("adakv_budgets", _adakv_ties_high_head),
+    ("adakv_budgets", _adakv_pool_includes_safeguard),
+    ("adakv_budgets", _adakv_safeguard_rounded),
+    ("adakv_budgets", _adakv_window_not_protected),
 ]
 
 

@@ -573,3 +573,121 @@ def test_validation_proxy_falls_back_when_nothing_is_evicted():
     Q = bf16ish(rng, (1, 8, d))
     cache = orc.build_unit(K, V, Q, orc.OracleConfig(budget=24, recent_window=4, n_fit=6, n_val=2))
     assert cache.r == 0 and len(cache.main_pos) == s
+
+
+# ---------------------------------------------------------------------------
+# AdaKV budgets across KV heads (App. B, "AdaKV"; "+ResKV" rows of
+# Table ruler_paper and Table longbench_paper)
+# ---------------------------------------------------------------------------
+
+def test_adakv_budgets_fixture():
+    g = golden("adakv_budgets.json")
+    for case in g["cases"]:
+        got = orc.adakv_budgets(np.array(case["scores"]), g["budget"], g["recent"],
+                                case["safeguard"])
+        assert got.tolist() == case["budgets"], case["note"]
+
+
+def _best_allocation(scores, budget, recent, f):
+    """Exhaustive search: the split x_h >= f, sum x_h = H*(b - |P|), that keeps
+    the largest total score (each head keeps its top x_h evictable tokens)."""
+    H, s = scores.shape
+    n_p = min(recent, s)
+    n = budget - n_p
+    tops = [np.concatenate([[0.0], np.cumsum(np.sort(scores[h, :s - n_p])[::-1])])
+            for h in range(H)]
+    best, arg = -1.0, None
+
+    def rec(h, left, acc, xs):
+        nonlocal best, arg
+        if h == H - 1:
+            if f <= left <= s - n_p:
+                tot = acc + tops[h][left]
+                if tot > best:
+                    best, arg = tot, xs + [left]
+            return
+        for x in range(f, min(left, s - n_p) + 1):
+            rec(h + 1, left - x, acc + tops[h][x], xs + [x])
+
+    rec(0, H * n, 0.0, [])
+    return np.array(arg) + n_p
+
+
+@pytest.mark.parametrize("seed,H,s,recent,budget,safeguard",
+                         [(0, 3, 12, 2, 5, 0.2), (1, 3, 12, 2, 5, 0.5), (2, 2, 16, 3, 7, 0.2),
+                          (3, 4, 10, 1, 4, 0.34), (4, 3, 9, 0, 3, 0.0)])
+def test_adakv_budgets_maximise_kept_score(seed, H, s, recent, budget, safeguard):
+    """With distinct scores the allocation is the unique split (every head
+    above its safeguard) that keeps the largest total score: each head's
+    retained mass is concave in its budget, so the pooled pick of the best
+    remaining tokens is optimal -- checked here by enumerating every split."""
+    rng = np.random.default_rng(seed)
+    scores = rng.random((H, s))
+    n = budget - min(recent, s)
+    f = int(np.floor(float(np.float32(safeguard)) * n))
+    got = orc.adakv_budgets(scores, budget, recent, safeguard)
+    assert got.tolist() == _best_allocation(scores, budget, recent, f).tolist()
+
+
+def test_adakv_budgets_invariants_and_closed_forms():
+    rng = np.random.default_rng(7)
+    H, s, recent, b = 8, 300, 16, 64
+    scores = rng.random((H, s))
+    for sg in (0.0, 0.2, 0.5, 0.9):
+        got = orc.adakv_budgets(scores, b, recent, sg)
+        f = int(np.floor(float(np.float32(sg)) * (b - recent)))
+        assert got.sum() == H * b and np.all(got >= recent + f) and np.all(got <= s)
+    # safeguard 1: nothing is shared; identical heads: the pooled pick alternates
+    assert orc.adakv_budgets(scores, b, recent, 1.0).tolist() == [b] * H
+    assert orc.adakv_budgets(np.tile(scores[:1], (H, 1)), b, recent, 0.2).tolist() == [b] * H
+    # the budget covers every token: no allocation
+    assert orc.adakv_budgets(scores, s + 5, recent, 0.2).tolist() == [s + 5] * H
+    # one dominant head takes every shared slot, b_3 = |P| + f + H (b - |P| - f),
+    # as long as it has that many tokens; with fewer it keeps all s of them
+    dom = rng.random((H, 500))
+    dom[3] += 1000.0
+    f = int(np.floor(float(np.float32(0.2)) * (b - recent)))
+    got = orc.adakv_budgets(dom, b, recent, 0.2)
+    assert got[3] == recent + f + H * (b - recent - f)
+    assert all(got[h] == recent + f for h in range(H) if h != 3)
+    got = orc.adakv_budgets(dom[:, :300], b, recent, 0.2)
+    assert got[3] == 300 and got.sum() == H * b
+
+
+def test_adakv_safeguard_one_is_uniform_resKV():
+    """safeguard 1 leaves every head its uniform budget, so the grouped build is
+    Alg. 1 per head unchanged."""
+    rng = np.random.default_rng(3)
+    H, s, d, G = 2, 96, 128, 2
+    Ks = np.round(rng.standard_normal((H, s, d)) * 8) / 8
+    Vs = np.round(rng.standard_normal((H, s, d)) * 8) / 8
+    Qo = np.round(rng.standard_normal((H, G, 12, d)) * 8) / 8
+    cfgs = [orc.OracleConfig(budget=32, recent_window=8, n_fit=8, n_val=4)] * H
+    budgets, units = orc.build_heads_adakv(Ks, Vs, Qo, cfgs, 1.0)
+    assert budgets.tolist() == [32, 32]
+    for h in range(H):
+        ref = orc.build_unit(Ks[h], Vs[h], Qo[h], cfgs[h])
+        assert ref.r == units[h].r
+        assert np.array_equal(ref.main_pos, units[h].main_pos)
+        assert np.array_equal(ref.kbar, units[h].kbar)
+
+
+def test_adakv_grouped_build_keeps_each_heads_budget():
+    """Every head's cache fills exactly its allocated budget b_h = m_h + r_h,
+    keeps its window, and its main tokens are its top b_h - |P| ranked tokens."""
+    rng = np.random.default_rng(5)
+    H, s, d, G = 3, 160, 128, 2
+    Ks = np.round(rng.standard_normal((H, s, d)) * 8) / 8
+    Ks[1] *= 3.0                      # a sharper head attracts budget
+    Vs = np.round(rng.standard_normal((H, s, d)) * 8) / 8
+    Qo = np.concatenate([Ks[:, None, rng.integers(0, s, 12)], Ks[:, None, rng.integers(0, s, 12)]],
+                        axis=1) + 0.1
+    cfgs = [orc.OracleConfig(budget=40, recent_window=8, n_fit=8, n_val=4)] * H
+    budgets, units = orc.build_heads_adakv(Ks, Vs, Qo, cfgs, 0.2)
+    assert budgets.sum() == H * 40
+    for h in range(H):
+        u = units[h]
+        assert len(u.main_pos) + u.r == budgets[h]
+        assert set(range(s - 8, s)) <= set(u.main_pos.tolist())
+        keep = len(u.main_pos) - 8
+        assert set(u.ranked[:keep].tolist()) | set(range(s - 8, s)) == set(u.main_pos.tolist())
