@@ -57,6 +57,19 @@ enum { RESKV_GATE_DYNAMIC = 0, RESKV_GATE_FIXED = 1 };
 enum { RESKV_SOFTMAX_SHARED = 0, RESKV_SOFTMAX_SEPARATE = 1 };
 enum { RESKV_DECODE_AUTO = 0, RESKV_DECODE_FMA = 1, RESKV_DECODE_MMA = 2, RESKV_DECODE_CLUSTER = 3,
        RESKV_DECODE_LSE_MERGE = 4 };
+/* RESKV_BUDGET_UNIFORM: every (layer, batch, KV head) unit gets `budget` (or
+ * its entry of unit_budgets).  RESKV_BUDGET_ADAKV: reskv_build_cache splits the
+ * H_kv * budget slots of each (layer, batch element) between its KV heads as
+ * AdaKV does (App. B, "AdaKV": token scores as importance, safeguard
+ * coefficient 0.2), then builds every head with its own budget b_h (the
+ * "+ResKV" rows of Table ruler_paper and Table longbench_paper).  The paper
+ * prints no formula; the rule built: every head keeps its recent window P and
+ * its own f = floor(adakv_safeguard * (budget - |P|)) best-ranked tokens; the
+ * other H_kv * (budget - |P| - f) slots go to the highest scores among all
+ * heads' remaining evictable tokens (ties: lower head, then lower position);
+ * b_h = |P| + f + head h's share.  With budget >= seq_len nothing is evicted
+ * and every head keeps `budget`. */
+enum { RESKV_BUDGET_UNIFORM = 0, RESKV_BUDGET_ADAKV = 1 };
 
 #define RESKV_MAX_GRID 8
 
@@ -118,7 +131,13 @@ typedef struct reskv_config {
   const int32_t* unit_budgets; /* host [L*B*H_kv] per-unit budgets b_u (AdaKV-
                               style allocation across heads, App. B), or NULL
                               for `budget` everywhere.  Unit u then owns
-                              b_u + A slots starting at sum_{v<u} (b_v + A)  */
+                              b_u + A slots starting at sum_{v<u} (b_v + A).
+                              reskv_build_cache needs b_u >= min(|P|, s)     */
+  int32_t budget_mode;     /* RESKV_BUDGET_*; ADAKV needs unit_budgets NULL
+                              and is a construction setting (import ignores
+                              it).  The built layout is ragged: read the
+                              budgets with reskv_get_unit_budgets            */
+  float adakv_safeguard;   /* AdaKV safeguard coefficient in [0, 1] (0.2)    */
 } reskv_config;
 
 /* Fill *cfg with the paper's defaults; shape fields are zeroed. */
@@ -192,9 +211,18 @@ typedef struct reskv_cache_info {
   int32_t max_appended;    /* most tokens appended to any unit so far        */
   int32_t ragged;          /* 1 with per-unit budgets                        */
   int64_t total_slots;     /* slots of the layout (sum over units)           */
+  int32_t n_candidates;    /* candidate columns of the validation proxy (the
+                              losses array has 1 + n_candidates per unit)    */
+  int32_t ranked_width;    /* entries per unit of RESKV_DEBUG_RANKED         */
 } reskv_cache_info;
 
 reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info);
+
+/* Budget b_u of every unit of the layout (unit u owns b_u + append_capacity
+ * slots): `budget` everywhere, the caller's unit_budgets, or the allocation
+ * reskv_build_cache made with RESKV_BUDGET_ADAKV.  host_budgets: int32
+ * [n_units]; n_units must equal the handle's. */
+reskv_status reskv_get_unit_budgets(const reskv_cache* c, int32_t* host_budgets, int64_t n_units);
 
 /*
  * Host-side view of a cache layout, used by reskv_import_cache (read) and
@@ -258,9 +286,21 @@ reskv_status reskv_append(reskv_cache* c, int32_t layer, const void* K_new, cons
 
 enum {
   RESKV_DEBUG_SCORES = 0,  /* fp64 [U, s]: token scores                      */
-  RESKV_DEBUG_RANKED = 1,  /* int32 [U, b - |P|]: top of the ranking of S\P  */
-  RESKV_DEBUG_LOSSES = 2,  /* fp64 [U, 1 + n_cand]: L_0 then L_r per candidate */
-  RESKV_DEBUG_CANDIDATES = 3 /* int32 [n_cand]: candidate r values, ascending */
+  RESKV_DEBUG_RANKED = 1,  /* int32 [U, W]: top of the ranking of S\P, W =
+                              info.ranked_width (b - |P| with one budget);
+                              with per-unit budgets unit u fills its first
+                              min(b_u, s) - |P| entries, the rest is -1      */
+  RESKV_DEBUG_LOSSES = 2,  /* fp64 [U, 1 + n_cand]: L_0 then L_r per candidate
+                              column; +inf where a unit has no such candidate */
+  RESKV_DEBUG_CANDIDATES = 3, /* int32 [n_cand]: candidate r values, ascending
+                              (one budget for every unit only)               */
+  RESKV_DEBUG_UNIT_CANDIDATES = 4 /* int32 [U, n_cand]: r of every candidate
+                              column per unit, 0 where the unit has none.
+                              With per-unit budgets the columns are the
+                              positive grid ratios in ascending order and
+                              r = floor(ratio * b_u), dropped (0) when zero,
+                              equal to the previous column's r, or leaving
+                              less than |P| main slots                        */
 };
 
 /* Copy a construction intermediate (cfg.keep_debug was set) to host memory.

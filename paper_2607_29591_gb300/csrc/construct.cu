@@ -16,6 +16,7 @@ namespace reskv {
 
 reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_cache** out);
 void release_handle(reskv_cache* c);
+reskv_status finalize_ragged_layout(reskv_cache* c);
 
 namespace {
 
@@ -107,19 +108,56 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
                               const int32_t* override_host, const void* const* Kl,
                               const void* const* Vl, const void* const* Ql, cudaStream_t stream) {
   // ---------------- validation ----------------
-  if (cfg.unit_budgets)
-    return fail(RESKV_ERR_UNSUPPORTED, "per-unit budgets: construction does not take them yet");
   const int64_t s = cfg.seq_len;
   const int b = cfg.budget;
   if (cfg.recent_window < 0) return fail(RESKV_ERR_INVALID_ARG, "recent_window must be >= 0");
   const int P = int(std::min<int64_t>(cfg.recent_window, s));
-  const int n_top = int(std::min<int64_t>(b, s)) - P;
-  if (n_top > kTopMax)
-    return fail(RESKV_ERR_UNSUPPORTED, "budget - recent_window must be <= 8192");
-  const bool all_main = int64_t(b) >= s;
-  const bool proxy = override_host == nullptr && !all_main;
   const int UL = cfg.batch * cfg.n_kv_heads;
   const int G = cfg.group;
+  const int64_t U_all = int64_t(cfg.n_layers) * UL;
+  if (cfg.budget_mode != RESKV_BUDGET_UNIFORM && cfg.budget_mode != RESKV_BUDGET_ADAKV)
+    return fail(RESKV_ERR_INVALID_ARG, "unknown budget_mode");
+  // AdaKV allocation across the KV heads of each (layer, batch element); with
+  // b >= s nothing is evicted and the layout keeps one budget
+  const bool adakv = cfg.budget_mode == RESKV_BUDGET_ADAKV && int64_t(b) < s;
+  if (cfg.budget_mode == RESKV_BUDGET_ADAKV) {
+    if (cfg.unit_budgets)
+      return fail(RESKV_ERR_INVALID_ARG, "budget_mode ADAKV allocates the budgets: unit_budgets must be NULL");
+    if (!(cfg.adakv_safeguard >= 0.f && cfg.adakv_safeguard <= 1.f))
+      return fail(RESKV_ERR_INVALID_ARG, "adakv_safeguard must be in [0, 1]");
+  }
+  const bool per_unit = cfg.unit_budgets != nullptr || adakv;
+  const int n_free_head = b - P;                       // selectable slots per head (AdaKV)
+  const int ada_f = adakv ? std::min(n_free_head, std::max(0, int(std::floor(
+                                double(cfg.adakv_safeguard) * double(n_free_head))))) : 0;
+  if (adakv && double(cfg.n_kv_heads) * double(s) >= double(int64_t(1) << 31))
+    return fail(RESKV_ERR_UNSUPPORTED, "AdaKV: n_kv_heads * seq_len must be < 2^31");
+  if (adakv && n_free_head > kTopMax)
+    return fail(RESKV_ERR_UNSUPPORTED, "AdaKV: budget - recent_window must be <= 8192");
+  // the largest budget a unit can get (sizes the scratch), and whether any unit evicts
+  int64_t b_hi = b;
+  bool any_evict = int64_t(b) < s;
+  if (cfg.unit_budgets) {
+    b_hi = 0;
+    any_evict = false;
+    for (int64_t u = 0; u < U_all; ++u) {
+      const int64_t bu = cfg.unit_budgets[u];
+      if (std::min(bu, s) < P)
+        return fail(RESKV_ERR_INVALID_ARG, "unit_budgets must be >= min(recent_window, seq_len)");
+      b_hi = std::max(b_hi, bu);
+      any_evict |= bu < s;
+    }
+  } else if (int64_t(std::min<int64_t>(b, s)) < P) {
+    return fail(RESKV_ERR_INVALID_ARG, "budget must be >= min(recent_window, seq_len)");
+  }
+  if (adakv)   // |P| + f + every shared slot, within s and the ranking limit
+    b_hi = std::min<int64_t>(std::min<int64_t>(s, int64_t(P) + kTopMax),
+                             int64_t(P) + ada_f + int64_t(cfg.n_kv_heads) * (n_free_head - ada_f));
+  const int n_top = int(std::min<int64_t>(b_hi, s)) - P;   // ranking width per unit
+  if (n_top > kTopMax)
+    return fail(RESKV_ERR_UNSUPPORTED, "budget - recent_window must be <= 8192");
+  const bool all_main = !any_evict;
+  const bool proxy = override_host == nullptr && !all_main;
   if (cfg.score_mode != RESKV_SCORE_OBS_POOL && cfg.score_mode != RESKV_SCORE_KEYNORM)
     return fail(RESKV_ERR_INVALID_ARG, "unknown score_mode");
   if (cfg.pool_kernel < 1 || cfg.pool_kernel % 2 == 0)
@@ -146,42 +184,87 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   if (!(cfg.delta >= 0.f && cfg.delta < 1.f) || !std::isfinite(cfg.beta))
     return fail(RESKV_ERR_INVALID_ARG, "delta must be in [0, 1) and beta finite");
 
-  // candidate budgets r = floor(ratio * b) > 0, distinct, ascending (App. B)
-  std::vector<int32_t> cands;
-  if (proxy) {
+  // candidate budgets r = floor(ratio * b) > 0, distinct, ascending (App. B).
+  // One budget: the columns are those r.  Per-unit budgets: the columns are
+  // the distinct positive ratios, ascending; unit u's r in a column is
+  // floor(ratio * b_u), dropped (0) when zero, equal to the previous column's,
+  // or leaving less than |P| main slots (unit_cands).
+  std::vector<int32_t> cands;          // one budget: r of every column
+  std::vector<float> col_ratio;        // per-unit budgets: ratio of every column
+  std::vector<int32_t> col_rmax;       // per column: the largest r any unit can have
+  for (int i = 0; i < cfg.n_grid; ++i)
+    if (!(cfg.grid_ratios[i] >= 0.f && cfg.grid_ratios[i] <= 1.f))
+      return fail(RESKV_ERR_INVALID_ARG, "grid ratios must be in [0, 1]");
+  if (proxy && !per_unit) {
     for (int i = 0; i < cfg.n_grid; ++i) {
-      const float ratio = cfg.grid_ratios[i];
-      if (!(ratio >= 0.f && ratio <= 1.f))
-        return fail(RESKV_ERR_INVALID_ARG, "grid ratios must be in [0, 1]");
-      const int r = int(std::floor(double(ratio) * double(b)));
+      const int r = int(std::floor(double(cfg.grid_ratios[i]) * double(b)));
       if (r > 0 && b - r >= P && std::find(cands.begin(), cands.end(), r) == cands.end())
         cands.push_back(r);
     }
     std::sort(cands.begin(), cands.end());
+    col_rmax = cands;
+  } else if (proxy) {
+    for (int i = 0; i < cfg.n_grid; ++i)
+      if (cfg.grid_ratios[i] > 0.f &&
+          std::find(col_ratio.begin(), col_ratio.end(), cfg.grid_ratios[i]) == col_ratio.end())
+        col_ratio.push_back(cfg.grid_ratios[i]);
+    std::sort(col_ratio.begin(), col_ratio.end());
+    for (float ratio : col_ratio)
+      col_rmax.push_back(int(std::floor(double(ratio) * double(b_hi))));
   }
+  // r of every candidate column for the units of one layer ([ncol, UL], column 0 = 0)
+  auto unit_candidates = [&](const int32_t* bl, std::vector<int32_t>& out) {
+    const int nc = 1 + int(col_rmax.size());
+    out.assign(size_t(nc) * UL, 0);
+    for (int i = 0; i < UL; ++i) {
+      const int64_t bu = bl ? bl[i] : b;
+      int prev = 0;
+      for (int c = 1; c < nc; ++c) {
+        int r = cands.empty() ? int(std::floor(double(col_ratio[c - 1]) * double(bu))) : cands[c - 1];
+        if (r <= 0 || r == prev || bu - r < P || bu >= s) r = 0;
+        else prev = r;
+        out[size_t(c) * UL + i] = r;
+      }
+    }
+  };
   std::vector<int32_t> ovr;
   int rmax = 0;
   if (override_host) {
-    const int64_t U = int64_t(cfg.n_layers) * UL;
-    ovr.assign(override_host, override_host + U);
-    for (int64_t u = 0; u < U; ++u) {
+    ovr.assign(override_host, override_host + U_all);
+    for (int64_t u = 0; u < U_all; ++u) {
       const int r = ovr[u];
-      if (r < 0 || r >= b) return fail(RESKV_ERR_INVALID_ARG, "residual_override out of [0, budget)");
-      if (r > 0 && (all_main || b - r < P))
+      const int64_t bu = cfg.unit_budgets ? cfg.unit_budgets[u] : b;
+      if (r < 0 || r >= bu) return fail(RESKV_ERR_INVALID_ARG, "residual_override out of [0, budget)");
+      if (r > 0 && !adakv && (bu >= s || bu - r < P))
         return fail(RESKV_ERR_INVALID_ARG,
-                    "residual_override needs budget <= seq_len and budget - r >= recent_window");
+                    "residual_override needs budget < seq_len and budget - r >= recent_window");
       rmax = std::max(rmax, r);
     }
   }
-  for (int32_t r : cands) rmax = std::max(rmax, r);
+  for (int32_t r : col_rmax) rmax = std::max(rmax, r);
   if (rmax > kMaxR) return fail(RESKV_ERR_UNSUPPORTED, "residual entries per unit must be <= 8192");
 
   // ---------------- handle and scratch ----------------
   reskv_cache* c = nullptr;
-  reskv_status st = alloc_handle(cfg, stream, &c);
+  reskv_status st;
+  std::vector<int32_t> budgets_host;   // per-unit budgets (every layer)
+  if (adakv) {
+    // provisional layout with b per unit: the allocation keeps every
+    // (layer, batch element)'s total, so only offsets inside it move
+    budgets_host.assign(size_t(U_all), b);
+    reskv_config lay = cfg;
+    lay.unit_budgets = budgets_host.data();
+    st = alloc_handle(lay, stream, &c);
+  } else {
+    if (cfg.unit_budgets) budgets_host.assign(cfg.unit_budgets, cfg.unit_budgets + U_all);
+    st = alloc_handle(cfg, stream, &c);
+  }
   if (st != RESKV_OK) return st;
-  c->candidates = cands;
-  const int ncol = 1 + int(cands.size());            // run 0 = pure-main cache
+  c->candidates = per_unit ? std::vector<int32_t>() : cands;
+  c->n_candidates = int32_t(col_rmax.size());
+  c->ranked_width = std::max(n_top, 0);
+  if (proxy) c->unit_cands.assign(size_t(U_all) * col_rmax.size(), 0);
+  const int ncol = 1 + int(col_rmax.size());         // run 0 = pure-main cache
   const int ntiles = int(cdiv(s, kTile));
   const int n_fit_rows = cfg.score_mode == RESKV_SCORE_OBS_POOL ? G * cfg.n_fit : 0;
   const int n_val_rows = proxy ? G * cfg.n_val : 0;
@@ -190,9 +273,9 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   std::vector<int32_t> run_off(std::max(ncol, 2), 0);
   int64_t ent_stride = 0;
   if (proxy) {
-    for (int i = 0; i < int(cands.size()); ++i) {
+    for (int i = 0; i < int(col_rmax.size()); ++i) {
       run_off[1 + i] = int32_t(ent_stride);
-      ent_stride += cands[i];
+      ent_stride += col_rmax[i];
     }
   } else {
     ent_stride = rmax;
@@ -206,7 +289,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   int32_t *top = nullptr, *rank_pos = nullptr, *assign = nullptr, *hist = nullptr;
   int32_t *ccount = nullptr, *cbase = nullptr, *members = nullptr, *ecount = nullptr;
   int32_t *r_runs = nullptr, *r_final = nullptr, *chosen = nullptr, *run_off_d = nullptr;
-  int32_t *cand_r_d = nullptr;
+  int32_t* budgets_d = nullptr;        // [U_all] per-unit budgets (per_unit only)
   float *centersT = nullptr, *cnorm = nullptr, *vpart = nullptr, *oS = nullptr;
   double* centers64 = nullptr;
   __nv_bfloat16 *kbar = nullptr, *vbar = nullptr;
@@ -215,7 +298,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   const int nruns = proxy ? ncol : 2;
   bool ok = S.get(&scores, US) && S.get(&top, size_t(UL) * std::max(n_top, 1)) &&
             S.get(&rank_pos, US) && S.get(&r_runs, size_t(nruns) * UL) &&
-            S.get(&r_final, UL) && S.get(&chosen, UL) && S.get(&run_off_d, run_off.size());
+            S.get(&r_final, UL) && S.get(&chosen, UL) && S.get(&run_off_d, run_off.size()) &&
+            (!per_unit || S.get(&budgets_d, size_t(U_all)));
   if (ok && n_fit_rows > 0)
     ok = S.get(&A, US) && S.get(&tstats, size_t(UL) * n_fit_rows * ntiles) &&
          S.get(&rstats, size_t(UL) * n_fit_rows);
@@ -230,8 +314,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   if (ok && proxy)
     ok = S.get(&vpart, size_t(UL) * n_val_rows * nchunks * kValRec) &&
          S.get(&oS, size_t(UL) * n_val_rows * kHeadDim) &&
-         S.get(&rowerr, size_t(UL) * n_val_rows) && S.get(&losses, size_t(UL) * ncol) &&
-         S.get(&cand_r_d, ncol);
+         S.get(&rowerr, size_t(UL) * n_val_rows) && S.get(&losses, size_t(UL) * ncol);
   if (ok && cfg.keep_debug) {
     const size_t U = size_t(c->n_units);
     cudaError_t e = cudaMalloc(&c->dbg_scores, U * size_t(s) * 8);
@@ -252,17 +335,15 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     return e;
   };
 
-  // per-run r arrays (proxy: uniform per run; override: filled per layer)
-  std::vector<int32_t> hr(size_t(nruns) * UL, 0);
-  if (proxy)
-    for (int i = 0; i < int(cands.size()); ++i)
-      std::fill(hr.begin() + size_t(1 + i) * UL, hr.begin() + size_t(2 + i) * UL, cands[i]);
-  std::vector<int32_t> cand_col(ncol, 0);
-  for (int i = 0; i < int(cands.size()); ++i) cand_col[1 + i] = cands[i];
+  // per-run r arrays [nruns, UL] (proxy: per layer from the units' budgets;
+  // override: filled per layer)
+  std::vector<int32_t> hr;
+  if (proxy) unit_candidates(nullptr, hr);
   if (cudaMemcpyAsync(run_off_d, run_off.data(), run_off.size() * 4, cudaMemcpyHostToDevice,
                       stream) != cudaSuccess ||
-      (proxy && cudaMemcpyAsync(cand_r_d, cand_col.data(), ncol * 4, cudaMemcpyHostToDevice,
-                                stream) != cudaSuccess))
+      (cfg.unit_budgets && cudaMemcpyAsync(budgets_d, budgets_host.data(), size_t(U_all) * 4,
+                                           cudaMemcpyHostToDevice, stream) != cudaSuccess) ||
+      cudaStreamSynchronize(stream) != cudaSuccess)
     return cleanup_fail(fail(RESKV_ERR_CUDA, "copying run tables"));
 
   // kernel attributes
@@ -299,23 +380,74 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     }
     RESKV_LAUNCH_CHECK("scoring");
     timing_ok &= timer.mark(kStRank);
-    TopArgs ta{scores, s, P, n_top, top, rank_pos, c->status};
+    int32_t* bl_d = per_unit ? budgets_d + size_t(l) * UL : nullptr;   // this layer's budgets
+    const int32_t* bl_h = per_unit ? budgets_host.data() + size_t(l) * UL : nullptr;
+    if (adakv) {
+      // AdaKV: mark every head's safeguard (its top f), split the shared slots
+      TopArgs tf{scores, s, P, ada_f, top, rank_pos, c->status, nullptr};
+      k_topk<<<UL, kTopThreads, sm_top, stream>>>(tf);
+      AdaArgs aa{scores, rank_pos, s, P, cfg.n_kv_heads, ada_f, P + ada_f,
+                 int64_t(cfg.n_kv_heads) * (n_free_head - ada_f), bl_d};
+      k_adakv<<<cfg.batch, kTopThreads, 0, stream>>>(aa);
+      RESKV_LAUNCH_CHECK("AdaKV budgets");
+      if (cudaMemcpyAsync(budgets_host.data() + size_t(l) * UL, bl_d, size_t(UL) * 4,
+                          cudaMemcpyDeviceToHost, stream) != cudaSuccess ||
+          cudaStreamSynchronize(stream) != cudaSuccess)
+        return cleanup_fail(fail(RESKV_ERR_CUDA, "reading the AdaKV budgets"));
+      // the layer's units keep their region; place them inside it
+      const int64_t u0 = int64_t(l) * UL;
+      for (int i = 0; i < UL; ++i) {
+        const int64_t bu = bl_h[i];
+        if (bu < P + ada_f || bu > b_hi)
+          return cleanup_fail(fail(bu > b_hi ? RESKV_ERR_UNSUPPORTED : RESKV_ERR_CUDA,
+                                   "AdaKV budget " + std::to_string(bu) + " of unit " +
+                                       std::to_string(u0 + i) +
+                                       " is outside what construction covers"));
+        if (!ovr.empty() && ovr[size_t(u0 + i)] > 0 &&
+            (bu >= s || bu - ovr[size_t(u0 + i)] < P))
+          return cleanup_fail(fail(RESKV_ERR_INVALID_ARG,
+                                   "residual_override of unit " + std::to_string(u0 + i) +
+                                       " leaves less than recent_window main slots of its AdaKV budget"));
+        c->h_offsets[size_t(u0 + i) + 1] = c->h_offsets[size_t(u0 + i)] + int32_t(bu) + c->append_capacity;
+      }
+      if (cudaMemcpyAsync(c->offsets + u0, c->h_offsets.data() + u0, size_t(UL + 1) * 4,
+                          cudaMemcpyHostToDevice, stream) != cudaSuccess)
+        return cleanup_fail(fail(RESKV_ERR_CUDA, "copying unit offsets"));
+    }
+    if (per_unit && n_top > 0 &&
+        cudaMemsetAsync(top, 0xff, size_t(UL) * n_top * 4, stream) != cudaSuccess)
+      return cleanup_fail(fail(RESKV_ERR_CUDA, "clearing the ranking"));
+    TopArgs ta{scores, s, P, n_top, top, rank_pos, c->status, bl_d};
     k_topk<<<UL, kTopThreads, sm_top, stream>>>(ta);
     RESKV_LAUNCH_CHECK("ranking");
+    // candidate r per unit of this layer
+    int grid_r = rmax;
+    if (proxy) {
+      if (per_unit || l == 0) unit_candidates(bl_h, hr);
+      for (int c2 = 1; c2 < ncol; ++c2)
+        for (int i = 0; i < UL; ++i)
+          c->unit_cands[(size_t(l) * UL + i) * (ncol - 1) + (c2 - 1)] = hr[size_t(c2) * UL + i];
+      if ((per_unit || l == 0) &&
+          cudaMemcpyAsync(r_runs, hr.data(), hr.size() * 4, cudaMemcpyHostToDevice, stream) != cudaSuccess)
+        return cleanup_fail(fail(RESKV_ERR_CUDA, "copying candidate budgets"));
+      grid_r = 0;
+      for (int32_t r : hr) grid_r = std::max<int>(grid_r, r);
+    }
 
     LloydArgs la{K, V, s, P, n_top, b, ntiles, rmax, top, rank_pos, nullptr, centersT, cnorm,
                  centers64, assign, hist, ccount, cbase, members, kbar, vbar, ecount,
-                 ent_stride, 0, c->status};
-    auto lloyd_run = [&](const int32_t* r_unit, int ent_off) -> reskv_status {
+                 ent_stride, 0, c->status, bl_d};
+    auto lloyd_run = [&](const int32_t* r_unit, int ent_off, int r_hi) -> reskv_status {
       la.r_unit = r_unit;
       la.ent_off = ent_off;
       timing_ok &= timer.mark(kStLloyd);
-      k_lloyd_init<<<dim3(rmax, UL), kHeadDim, 0, stream>>>(la);
+      const unsigned gr = unsigned(std::max(r_hi, 1));
+      k_lloyd_init<<<dim3(gr, UL), kHeadDim, 0, stream>>>(la);
       for (int it = 0; it < cfg.lloyd_iters; ++it) {
         k_lloyd_assign<<<dim3(ntiles, UL), kThreads, sm_assign, stream>>>(la);
         k_lloyd_scan<<<UL, 256, 0, stream>>>(la);
         k_lloyd_scatter<<<dim3(ntiles, UL), kTile, 0, stream>>>(la);
-        k_lloyd_update<<<dim3(rmax, UL), kThreads, 0, stream>>>(la, it == cfg.lloyd_iters - 1);
+        k_lloyd_update<<<dim3(gr, UL), kThreads, 0, stream>>>(la, it == cfg.lloyd_iters - 1);
       }
       RESKV_LAUNCH_CHECK("residual entries");
       return RESKV_OK;
@@ -328,25 +460,31 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       k_val_full<<<dim3(nchunks, unsigned(cdiv(n_val_rows, kRowBlk)), UL), kThreads, sm_val, stream>>>(va);
       k_val_combine<<<dim3(n_val_rows, UL), kHeadDim, 0, stream>>>(va);
       RESKV_LAUNCH_CHECK("validation targets");
-      if (l == 0 &&
-          cudaMemcpyAsync(r_runs, hr.data(), hr.size() * 4, cudaMemcpyHostToDevice, stream) != cudaSuccess)
-        return cleanup_fail(fail(RESKV_ERR_CUDA, "copying candidate budgets"));
       for (int run = 0; run < ncol; ++run) {
         const int32_t* r_unit = r_runs + size_t(run) * UL;
         if (run > 0) {
-          st = lloyd_run(r_unit, run_off[run]);
+          int r_hi = 0;
+          for (int i = 0; i < UL; ++i) r_hi = std::max(r_hi, hr[size_t(run) * UL + i]);
+          if (r_hi == 0) {           // no unit of the layer has this candidate
+            k_loss_reduce<<<unsigned(cdiv(UL, 128)), 128, 0, stream>>>(rowerr, losses, 0, UL,
+                                                                      ncol, run, r_unit);
+            RESKV_LAUNCH_CHECK("validation loss");
+            continue;
+          }
+          st = lloyd_run(r_unit, run_off[run], r_hi);
           if (st != RESKV_OK) return cleanup_fail(st);
         }
         timing_ok &= timer.mark(kStValLoss);
         LossArgs lo{K, V, Q, s, G, cfg.n_obs, cfg.n_val, n_val_rows, P, n_top, b, top, r_unit,
                     kbar, vbar, ecount, ent_stride, run_off[run], cfg.beta, cfg.gate_mode,
-                    cfg.tau, cfg.alpha, cfg.g_min, cfg.g_fixed, oS, rowerr, cfg.softmax_mode};
+                    cfg.tau, cfg.alpha, cfg.g_min, cfg.g_fixed, oS, rowerr, cfg.softmax_mode,
+                    bl_d};
         k_val_loss<<<dim3(unsigned(cdiv(n_val_rows, 8)), UL), kThreads, 0, stream>>>(lo);
         k_loss_reduce<<<unsigned(cdiv(UL, 128)), 128, 0, stream>>>(rowerr, losses, n_val_rows, UL,
-                                                                  ncol, run);
+                                                                  ncol, run, r_unit);
         RESKV_LAUNCH_CHECK("validation loss");
       }
-      k_choose<<<unsigned(cdiv(UL, 128)), 128, 0, stream>>>(losses, ncol, cand_r_d, UL,
+      k_choose<<<unsigned(cdiv(UL, 128)), 128, 0, stream>>>(losses, ncol, r_runs, UL,
                                                            one_minus_delta, r_final, chosen);
       RESKV_LAUNCH_CHECK("choosing r");
     } else {
@@ -365,7 +503,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
           cudaStreamSynchronize(stream) != cudaSuccess)
         return cleanup_fail(fail(RESKV_ERR_CUDA, "copying residual counts"));
       if (any) {
-        st = lloyd_run(r_final, 0);
+        st = lloyd_run(r_final, 0, *std::max_element(rl.begin(), rl.end()));
         if (st != RESKV_OK) return cleanup_fail(st);
       }
     }
@@ -374,7 +512,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     timing_ok &= timer.mark(kStPack);
     PackArgs pa{K, V, s, P, b, c->stride, rank_pos, r_final, chosen, run_off_d, kbar, vbar, ecount,
                 ent_stride, cfg.beta, int64_t(l) * UL, c->kslots, c->vslots, c->logc,
-                c->slot_pos, c->counts, c->n_main, c->n_res};
+                c->slot_pos, c->counts, c->n_main, c->n_res, bl_d,
+                per_unit ? c->offsets : nullptr};
     k_pack<<<UL, 1024, 0, stream>>>(pa);
     RESKV_LAUNCH_CHECK("packing");
     timing_ok &= timer.mark(-1);
@@ -394,6 +533,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   }
   if (!timing_ok)                        // timing is reported, not needed: clear it
     for (float& t : c->build_ms) t = 0.f;
+  if (adakv && (st = finalize_ragged_layout(c)) != RESKV_OK) return cleanup_fail(st);
   // scratch is freed (cudaFree synchronises) when S leaves scope
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return cleanup_fail(fail(RESKV_ERR_CUDA, std::string("construction: ") +

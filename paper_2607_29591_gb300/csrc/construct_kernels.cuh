@@ -253,7 +253,14 @@ struct TopArgs {
   int32_t* top;           // [UL, n_top] positions in rank order
   int32_t* rank_pos;      // [UL, s]: rank, INT_MAX (never main) or -1 (protected)
   uint32_t* status;
+  const int32_t* budgets; // [UL] per-unit budgets (rank min(b_u, s) - |P| each,
+                          // at stride n_top), or NULL: rank n_top for every unit
 };
+
+// Budget of unit ul of the layer: its own, or the shared one.
+__device__ __forceinline__ int64_t unit_budget(const int32_t* budgets, int ul, int64_t b) {
+  return budgets ? int64_t(budgets[ul]) : b;
+}
 
 __device__ __forceinline__ uint64_t score_key(double v) {
   // non-negative doubles order like their bit patterns; clamp -0 and negatives to 0
@@ -298,7 +305,15 @@ __global__ void __launch_bounds__(kTopThreads, 1) k_topk(TopArgs p) {
   const int64_t n_ev = s > p.recent ? s - p.recent : 0;
   const double* sc = p.scores + int64_t(ul) * s;
   int32_t* rp = p.rank_pos + int64_t(ul) * s;
-  const int K = p.n_top;
+  int K = p.n_top;
+  if (p.budgets) {
+    const int64_t keep = (p.budgets[ul] < s ? int64_t(p.budgets[ul]) : s) - p.recent;
+    K = keep < 0 ? 0 : int(keep);
+    if (K > p.n_top) {
+      if (threadIdx.x == 0 && p.status) report_status(p.status, kStatusBadIndex);
+      K = p.n_top;
+    }
+  }
   // protected window and default ranks
   for (int64_t i = threadIdx.x; i < s; i += blockDim.x) rp[i] = (i < n_ev) ? INT_MAX : -1;
   if (K <= 0) return;
@@ -395,8 +410,104 @@ __global__ void __launch_bounds__(kTopThreads, 1) k_topk(TopArgs p) {
   }
   for (int i = threadIdx.x; i < K; i += blockDim.x) {
     const int32_t pos = sidx[i];
-    p.top[int64_t(ul) * K + i] = pos;
+    p.top[int64_t(ul) * p.n_top + i] = pos;
     rp[pos] = i;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// AdaKV budgets across the KV heads of one (layer, batch element) (App. B,
+// "AdaKV": token scores as importance, safeguard coefficient).  Every head
+// keeps |P| + f slots (its window and its f best-ranked tokens, which a
+// ranking of the top f has marked in rank_pos); the n_free other slots go to
+// the highest-scored remaining evictable tokens of all heads, ordered by
+// (score desc, head asc, position asc).  One CTA per batch element: a radix
+// select of the n_free-th largest key over the heads' remaining tokens, then
+// per-head counts above and at the threshold.
+// ---------------------------------------------------------------------------
+
+struct AdaArgs {
+  const double* scores;      // [UL, s]
+  const int32_t* rank_pos;   // [UL, s]: rank < f marks a head's safeguard tokens
+  int64_t s;
+  int32_t recent;            // |P| (clamped to s)
+  int32_t n_heads;           // H_kv; unit ul = batch * H_kv + h
+  int32_t f;                 // safeguard tokens per head
+  int32_t base;              // |P| + f
+  int64_t n_free;            // H_kv * (b - |P| - f)
+  int32_t* budgets;          // [UL] out
+};
+
+__global__ void __launch_bounds__(kTopThreads, 1) k_adakv(AdaArgs p) {
+  __shared__ int hist[256];
+  __shared__ int bcast[2];
+  __shared__ int cnt[2];
+  const int grp = blockIdx.x, H = p.n_heads;
+  const int64_t s = p.s, n_ev = s > p.recent ? s - p.recent : 0;
+  const int ul0 = grp * H;
+  if (p.n_free <= 0) {
+    for (int h = threadIdx.x; h < H; h += blockDim.x) p.budgets[ul0 + h] = p.base;
+    return;
+  }
+  // radix select: threshold key tau with count(> tau) < n_free <= count(>= tau)
+  uint64_t prefix = 0, mask = 0;
+  int64_t k_rem = p.n_free;
+  for (int shift = 56; shift >= 0; shift -= 8) {
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    for (int h = 0; h < H; ++h) {
+      const double* sc = p.scores + int64_t(ul0 + h) * s;
+      const int32_t* rp = p.rank_pos + int64_t(ul0 + h) * s;
+      for (int64_t i = threadIdx.x; i < n_ev; i += blockDim.x) {
+        if (rp[i] < p.f) continue;                       // the head's safeguard token
+        const uint64_t key = score_key(sc[i]);
+        if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 0xff], 1);
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int64_t cum = 0;
+      int digit = 0;
+      for (int d = 255; d >= 0; --d) {
+        if (cum + hist[d] >= k_rem) {
+          digit = d;
+          break;
+        }
+        cum += hist[d];
+      }
+      bcast[0] = digit;
+      bcast[1] = int(k_rem - cum);
+    }
+    __syncthreads();
+    prefix |= uint64_t(bcast[0]) << shift;
+    mask |= uint64_t(0xff) << shift;
+    k_rem = bcast[1];
+    __syncthreads();
+  }
+  const uint64_t tau = prefix;   // k_rem keys equal to tau are taken: lower heads first
+  int64_t eq_before = 0;
+  for (int h = 0; h < H; ++h) {
+    if (threadIdx.x == 0) cnt[0] = cnt[1] = 0;
+    __syncthreads();
+    const double* sc = p.scores + int64_t(ul0 + h) * s;
+    const int32_t* rp = p.rank_pos + int64_t(ul0 + h) * s;
+    int gt = 0, eq = 0;
+    for (int64_t i = threadIdx.x; i < n_ev; i += blockDim.x) {
+      if (rp[i] < p.f) continue;
+      const uint64_t key = score_key(sc[i]);
+      gt += key > tau;
+      eq += key == tau;
+    }
+    if (gt) atomicAdd(&cnt[0], gt);
+    if (eq) atomicAdd(&cnt[1], eq);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int64_t take_eq = k_rem - eq_before;
+      take_eq = take_eq < 0 ? 0 : (take_eq > cnt[1] ? cnt[1] : take_eq);
+      p.budgets[ul0 + h] = p.base + cnt[0] + int32_t(take_eq);
+    }
+    eq_before += cnt[1];
+    __syncthreads();
   }
 }
 
@@ -438,11 +549,12 @@ struct LloydArgs {
   int64_t ent_stride;
   int32_t ent_off;
   uint32_t* status;
+  const int32_t* budgets;      // [UL] per-unit budgets, or NULL (budget)
 };
 
 __device__ __forceinline__ bool in_evicted(const LloydArgs& p, int ul, int64_t pos, int r) {
   const int32_t rk = p.rank_pos[int64_t(ul) * p.s + pos];
-  const int32_t keep = p.budget - r - p.recent;           // ranked tokens kept as main
+  const int32_t keep = int32_t(unit_budget(p.budgets, ul, p.budget)) - r - p.recent;  // ranked main
   return rk >= 0 && rk >= keep;
 }
 
@@ -452,7 +564,7 @@ __global__ void k_lloyd_init(LloydArgs p) {
   const int j = blockIdx.x, ul = blockIdx.y, d = threadIdx.x;
   const int r = p.r_unit[ul];
   if (j >= r) return;
-  const int32_t keep = p.budget - r - p.recent;
+  const int32_t keep = int32_t(unit_budget(p.budgets, ul, p.budget)) - r - p.recent;
   const int32_t pos = p.top[int64_t(ul) * p.n_top + keep + j];
   const float c = __bfloat162float(p.K[(int64_t(ul) * p.s + pos) * kHeadDim + d]);
   p.centersT[(int64_t(ul) * kHeadDim + d) * p.rmax + j] = c;
@@ -915,6 +1027,7 @@ struct LossArgs {
   const float* oS;             // [UL, n_rows, d]
   double* rowerr;              // [UL, n_rows]
   int32_t softmax_mode;        // decode rule of the losses (RESKV_SOFTMAX_*)
+  const int32_t* budgets;      // [UL] per-unit budgets, or NULL (budget)
 };
 
 // ||o^(r)(q) - o_S(q)||^2 per validation query, with the decode rule of
@@ -924,7 +1037,8 @@ __global__ void __launch_bounds__(kThreads) k_val_loss(LossArgs p) {
   const int row = blockIdx.x * 8 + w, ul = blockIdx.y;
   if (row >= p.n_rows) return;
   const int r = p.r_unit[ul];
-  const int64_t m = r == 0 ? (p.budget < p.s ? p.budget : p.s) : p.budget - r;
+  const int64_t bu = unit_budget(p.budgets, ul, p.budget);
+  const int64_t m = r == 0 ? (bu < p.s ? bu : p.s) : bu - r;
   const int64_t keep = m - p.recent;
   const int g = row / p.n_val, t = row % p.n_val;
   const __nv_bfloat16* qp = p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + (p.n_obs - p.n_val) + t) * kHeadDim;
@@ -1003,27 +1117,29 @@ __global__ void __launch_bounds__(kThreads) k_val_loss(LossArgs p) {
   if (lane == 0) p.rowerr[int64_t(ul) * p.n_rows + row] = double(e);
 }
 
-// L_r = mean of the per-query errors (rows in order, fp64)
+// L_r = mean of the per-query errors (rows in order, fp64); +inf for a unit
+// without a candidate in this column (r_unit = 0 in a column c > 0)
 __global__ void k_loss_reduce(const double* rowerr, double* losses, int n_rows, int UL, int ncol,
-                              int col) {
+                              int col, const int32_t* r_unit) {
   const int ul = blockIdx.x * blockDim.x + threadIdx.x;
   if (ul >= UL) return;
   double acc = 0.0;
   for (int i = 0; i < n_rows; ++i) acc += rowerr[int64_t(ul) * n_rows + i];
-  losses[int64_t(ul) * ncol + col] = acc / double(n_rows);
+  losses[int64_t(ul) * ncol + col] = (col > 0 && r_unit[ul] == 0) ? INFINITY : acc / double(n_rows);
 }
 
-// r* = argmin_{r>0} L_r (ties -> smaller r); keep it only if L_r* < (1 - delta) L_0
-__global__ void k_choose(const double* losses, int ncol, const int32_t* cand_r, int UL,
+// r* = argmin_{r>0} L_r (ties -> smaller r: columns hold ascending r); keep it
+// only if L_r* < (1 - delta) L_0.  r_runs: [ncol, UL] r of every column.
+__global__ void k_choose(const double* losses, int ncol, const int32_t* r_runs, int UL,
                          double one_minus_delta, int32_t* r_final, int32_t* chosen) {
   const int ul = blockIdx.x * blockDim.x + threadIdx.x;
   if (ul >= UL) return;
   const double* L = losses + int64_t(ul) * ncol;
   int best = 0;
   for (int c = 1; c < ncol; ++c)
-    if (best == 0 || L[c] < L[best]) best = c;
+    if (r_runs[int64_t(c) * UL + ul] > 0 && (best == 0 || L[c] < L[best])) best = c;
   const bool use = best > 0 && L[best] < one_minus_delta * L[0];
-  r_final[ul] = use ? cand_r[best] : 0;
+  r_final[ul] = use ? r_runs[int64_t(best) * UL + ul] : 0;
   chosen[ul] = use ? best : 0;
 }
 
@@ -1055,6 +1171,8 @@ struct PackArgs {
   int32_t* counts;
   int32_t* n_main;
   int32_t* n_res;
+  const int32_t* budgets;      // [UL] per-unit budgets, or NULL (budget)
+  const int32_t* offsets;      // [U + 1] first slot of every unit, or NULL (u * stride)
 };
 
 __global__ void __launch_bounds__(1024) k_pack(PackArgs p) {
@@ -1062,10 +1180,12 @@ __global__ void __launch_bounds__(1024) k_pack(PackArgs p) {
   const int ul = blockIdx.x;
   const int64_t u = p.unit0 + ul;
   const int r = p.r_final[ul];
-  const int64_t m = r == 0 ? (p.budget < p.s ? p.budget : p.s) : p.budget - r;
+  const int64_t bu = unit_budget(p.budgets, ul, p.budget);
+  const int64_t m = r == 0 ? (bu < p.s ? bu : p.s) : bu - r;
   const int64_t keep = m - p.recent;
   const int32_t* rp = p.rank_pos + int64_t(ul) * p.s;
-  int32_t* spos = p.slot_pos + u * p.stride;
+  const int64_t base = p.offsets ? int64_t(p.offsets[u]) : u * p.stride;   // first slot of u
+  int32_t* spos = p.slot_pos + base;
   const int64_t chunk = (p.s + blockDim.x - 1) / blockDim.x;
   const int64_t lo = int64_t(threadIdx.x) * chunk, hi = lo + chunk < p.s ? lo + chunk : p.s;
   int mine = 0;
@@ -1089,17 +1209,17 @@ __global__ void __launch_bounds__(1024) k_pack(PackArgs p) {
     const int64_t pos = spos[j];
     const uint2 kw = __ldg(reinterpret_cast<const uint2*>(Ku + pos * kHeadDim) + lane);
     const uint2 vw = __ldg(reinterpret_cast<const uint2*>(Vu + pos * kHeadDim) + lane);
-    reinterpret_cast<uint2*>(p.kslots + (u * p.stride + j) * kHeadDim)[lane] = kw;
-    reinterpret_cast<uint2*>(p.vslots + (u * p.stride + j) * kHeadDim)[lane] = vw;
+    reinterpret_cast<uint2*>(p.kslots + (base + j) * kHeadDim)[lane] = kw;
+    reinterpret_cast<uint2*>(p.vslots + (base + j) * kHeadDim)[lane] = vw;
     if (lane == 0) {
-      p.counts[u * p.stride + j] = 0;
-      p.logc[u * p.stride + j] = 0.f;
+      p.counts[base + j] = 0;
+      p.logc[base + j] = 0.f;
     }
   }
   const int c = p.chosen[ul];
   for (int j = w; j < r; j += nw) {
     const int64_t e = int64_t(ul) * p.ent_stride + p.run_off[c] + j;
-    const int64_t slot = u * p.stride + m + j;
+    const int64_t slot = base + m + j;
     reinterpret_cast<uint2*>(p.kslots + slot * kHeadDim)[lane] =
         reinterpret_cast<const uint2*>(p.kbar + e * kHeadDim)[lane];
     reinterpret_cast<uint2*>(p.vslots + slot * kHeadDim)[lane] =

@@ -141,7 +141,10 @@ struct reskv_cache {
   int32_t* dbg_ranked = nullptr;
   double* dbg_losses = nullptr;
   int64_t dbg_n_top = 0;
-  std::vector<int32_t> candidates;
+  std::vector<int32_t> candidates;   // one budget: r of every candidate column
+  int32_t n_candidates = 0;          // candidate columns of the validation proxy
+  int32_t ranked_width = 0;          // entries per unit of the kept ranking
+  std::vector<int32_t> unit_cands;   // [U, n_candidates] r per column and unit (0: none)
   // device time of the construction stages (ms): scores, ranking, validation
   // targets, Lloyd, validation losses + choice of r, packing
   float build_ms[6] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f};

@@ -254,6 +254,19 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
 
 void release_handle(reskv_cache* c) { free_handle(c); }
 
+// After construction has placed units of a ragged layout (AdaKV budgets):
+// the largest unit and the cluster plans follow the final budgets.
+reskv_status finalize_ragged_layout(reskv_cache* c) {
+  c->max_unit_slots = 0;
+  for (int64_t u = 0; u < c->n_units; ++u)
+    c->max_unit_slots = std::max<int32_t>(c->max_unit_slots,
+                                          c->h_offsets[size_t(u) + 1] - c->h_offsets[size_t(u)]);
+  const int64_t per_layer = int64_t(c->cfg.batch) * c->cfg.n_kv_heads;
+  reskv_status st = plan_cluster(c, per_layer, &c->cplan_layer);
+  if (st == RESKV_OK) st = plan_cluster(c, c->n_units, &c->cplan_all);
+  return st;
+}
+
 }  // namespace reskv
 
 using namespace reskv;
@@ -284,6 +297,8 @@ void reskv_config_default(reskv_config* cfg) {
   cfg->g_min = 0.0f;
   cfg->g_fixed = 1.0f;
   cfg->keep_debug = 0;
+  cfg->budget_mode = RESKV_BUDGET_UNIFORM;
+  cfg->adakv_safeguard = 0.2f;
 }
 
 const char* reskv_last_error(void) { return g_last_error.c_str(); }
@@ -549,6 +564,16 @@ reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info) {
       info->all_cluster ? (c->cplan_all.cluster ? c->cplan_all.warps_per_cta
                                                 : cluster_warps(c->max_unit_slots, 1))
                         : 0;
+  info->n_candidates = c->n_candidates;
+  info->ranked_width = int32_t(c->dbg_ranked ? c->dbg_n_top : c->ranked_width);
+  return RESKV_OK;
+}
+
+reskv_status reskv_get_unit_budgets(const reskv_cache* c, int32_t* host_budgets, int64_t n_units) {
+  if (!c || !host_budgets) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  if (n_units != c->n_units) return fail(RESKV_ERR_INVALID_ARG, "n_units does not match the handle");
+  for (int64_t u = 0; u < n_units; ++u)
+    host_budgets[u] = c->h_offsets[size_t(u) + 1] - c->h_offsets[size_t(u)] - c->append_capacity;
   return RESKV_OK;
 }
 
@@ -569,11 +594,23 @@ reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_d
       break;
     case RESKV_DEBUG_LOSSES:
       src = c->dbg_losses;
-      need = U * (1 + ncand) * 8;
+      need = U * (1 + size_t(c->n_candidates)) * 8;
       break;
     case RESKV_DEBUG_CANDIDATES:
+      if (c->n_candidates > 0 && c->candidates.empty())
+        return fail(RESKV_ERR_INVALID_ARG,
+                    "per-unit budgets: read RESKV_DEBUG_UNIT_CANDIDATES instead");
       if (bytes != ncand * 4) return fail(RESKV_ERR_INVALID_ARG, "size mismatch");
       if (ncand) std::memcpy(host_dst, c->candidates.data(), bytes);
+      return RESKV_OK;
+    case RESKV_DEBUG_UNIT_CANDIDATES:
+      if (bytes != U * size_t(c->n_candidates) * 4)
+        return fail(RESKV_ERR_INVALID_ARG, "size mismatch: need " +
+                                               std::to_string(U * size_t(c->n_candidates) * 4) +
+                                               " bytes");
+      if (bytes && c->unit_cands.size() * 4 != bytes)
+        return fail(RESKV_ERR_INVALID_ARG, "no candidates were kept (the proxy did not run)");
+      if (bytes) std::memcpy(host_dst, c->unit_cands.data(), bytes);
       return RESKV_OK;
     default:
       return fail(RESKV_ERR_INVALID_ARG, "unknown debug array");

@@ -27,6 +27,8 @@ RESKV_DECODE_AUTO, RESKV_DECODE_FMA, RESKV_DECODE_MMA, RESKV_DECODE_CLUSTER = 0,
 RESKV_DECODE_LSE_MERGE = 4
 RESKV_SOFTMAX_SHARED, RESKV_SOFTMAX_SEPARATE = 0, 1
 RESKV_DEBUG_SCORES, RESKV_DEBUG_RANKED, RESKV_DEBUG_LOSSES, RESKV_DEBUG_CANDIDATES = 0, 1, 2, 3
+RESKV_DEBUG_UNIT_CANDIDATES = 4
+RESKV_BUDGET_UNIFORM, RESKV_BUDGET_ADAKV = 0, 1
 MAX_GRID = 8
 
 
@@ -51,6 +53,7 @@ class reskv_config(ctypes.Structure):
         ("decode_warps", ctypes.c_int32), ("decode_kernel", ctypes.c_int32),
         ("softmax_mode", ctypes.c_int32), ("append_capacity", ctypes.c_int32),
         ("unit_budgets", ctypes.POINTER(ctypes.c_int32)),
+        ("budget_mode", ctypes.c_int32), ("adakv_safeguard", ctypes.c_float),
     ]
 
 
@@ -67,7 +70,8 @@ class reskv_cache_info(ctypes.Structure):
                 ("all_cluster_warps", ctypes.c_int32), ("build_ms", ctypes.c_float * 6),
                 ("append_capacity", ctypes.c_int32), ("stride", ctypes.c_int32),
                 ("max_appended", ctypes.c_int32), ("ragged", ctypes.c_int32),
-                ("total_slots", ctypes.c_int64)]
+                ("total_slots", ctypes.c_int64), ("n_candidates", ctypes.c_int32),
+                ("ranked_width", ctypes.c_int32)]
 
 
 class reskv_device_cache(ctypes.Structure):
@@ -108,6 +112,8 @@ def load_library():
     lib.reskv_check_status.restype = i32
     lib.reskv_get_info.argtypes = [vp, ctypes.POINTER(reskv_cache_info)]
     lib.reskv_get_info.restype = i32
+    lib.reskv_get_unit_budgets.argtypes = [vp, ctypes.POINTER(ctypes.c_int32), ctypes.c_int64]
+    lib.reskv_get_unit_budgets.restype = i32
     lib.reskv_import_cache.argtypes = [cfgp, ctypes.POINTER(reskv_host_cache), vp,
                                        ctypes.POINTER(vp)]
     lib.reskv_import_cache.restype = i32
@@ -262,6 +268,16 @@ def reskv_get_info(cache: Cache) -> dict:
     return out
 
 
+def reskv_get_unit_budgets(cache: Cache) -> np.ndarray:
+    """Budget b_u of every unit of the handle's layout: int32 [U]."""
+    c = cache.cfg
+    U = c.n_layers * c.batch * c.n_kv_heads
+    out = np.zeros(U, np.int32)
+    _check(load_library().reskv_get_unit_budgets(
+        cache.handle, out.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), U))
+    return out
+
+
 def _host_view(arrs: dict) -> reskv_host_cache:
     h = reskv_host_cache()
     for k, _ in h._fields_:
@@ -304,7 +320,10 @@ def reskv_export_cache(cache: Cache, stream=None) -> dict:
     """Copy the cache layout to host numpy arrays."""
     cfg = cache.cfg
     U, d = cfg.n_layers * cfg.batch * cfg.n_kv_heads, cfg.head_dim
-    off = unit_offsets(cfg)
+    ragged = bool(reskv_get_info(cache)["ragged"])
+    off = (np.concatenate([[0], np.cumsum(reskv_get_unit_budgets(cache).astype(np.int64)
+                                          + cfg.append_capacity)])
+           if ragged else unit_offsets(cfg))
     N = off[-1]
     arrs = dict(n_main=np.zeros(U, np.int32), n_res=np.zeros(U, np.int32),
                 kslots=np.zeros((N, d), np.uint16), vslots=np.zeros((N, d), np.uint16),
@@ -312,7 +331,7 @@ def reskv_export_cache(cache: Cache, stream=None) -> dict:
                 counts=np.zeros(N, np.int32), n_app=np.zeros(U, np.int32))
     h = _host_view(arrs)
     _check(load_library().reskv_export_cache(cache.handle, ctypes.byref(h), _stream(stream)))
-    if cfg.unit_budgets:                         # ragged: flat arrays plus the unit offsets
+    if ragged:                                   # per-unit budgets: flat arrays plus offsets
         arrs["offsets"] = off
     else:                                        # one stride: [U, S, ...]
         S = cfg.budget + cfg.append_capacity
@@ -334,19 +353,23 @@ def unit_offsets(cfg: reskv_config) -> np.ndarray:
 
 
 def reskv_export_debug(cache: Cache, what: int, n_cand: Optional[int] = None) -> np.ndarray:
-    """Construction intermediates (cfg.keep_debug must have been set)."""
+    """Construction intermediates (cfg.keep_debug must have been set, except
+    for the candidate tables).  ``n_cand`` defaults to the handle's count."""
     cfg = cache.cfg
     U = cfg.n_layers * cfg.batch * cfg.n_kv_heads
-    s, b = cfg.seq_len, cfg.budget
-    n_top = max(min(b, s) - min(cfg.recent_window, s), 0)
+    s = cfg.seq_len
+    info = reskv_get_info(cache)
+    nc = info["n_candidates"] if n_cand is None else n_cand
     if what == RESKV_DEBUG_CANDIDATES:
-        out = np.zeros(n_cand if n_cand is not None else 0, np.int32)
+        out = np.zeros(nc, np.int32)
+    elif what == RESKV_DEBUG_UNIT_CANDIDATES:
+        out = np.zeros((U, nc), np.int32)
     elif what == RESKV_DEBUG_SCORES:
         out = np.zeros((U, s), np.float64)
     elif what == RESKV_DEBUG_RANKED:
-        out = np.zeros((U, n_top), np.int32)
+        out = np.zeros((U, info["ranked_width"]), np.int32)
     elif what == RESKV_DEBUG_LOSSES:
-        out = np.zeros((U, 1 + (n_cand or 0)), np.float64)
+        out = np.zeros((U, 1 + nc), np.float64)
     else:
         raise ValueError("unknown debug array")
     _check(load_library().reskv_export_debug(cache.handle, int(what),
