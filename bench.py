@@ -63,6 +63,10 @@ def parse_args():
                          "merged through log-sum-exp statistics)")
     ap.add_argument("--layers", type=int, default=0,
                     help="use only this many layers (smaller profiling case)")
+    ap.add_argument("--budget-mode", choices=["uniform", "adakv"], default="uniform",
+                    help="uniform: every (layer, batch, KV head) keeps the budget; adakv: "
+                         "construction splits each (layer, batch element)'s budget between its "
+                         "KV heads with AdaKV's rule (ragged layout)")
     return ap.parse_args()
 
 
@@ -286,7 +290,7 @@ def run_reference(args, world, rank):
 # the GPU arm
 # ---------------------------------------------------------------------------
 
-def build_workload(w: wl.Workload, n_q: int, device, decode_kernel: int):
+def build_workload(w: wl.Workload, n_q: int, device, decode_kernel: int, budget_mode: int = 0):
     """Generate inputs layer by layer; build the compressed cache (timed)."""
     from paper_2607_29591_gb300 import reskv as R
     Ks, Vs, Qs = [], [], []
@@ -303,7 +307,7 @@ def build_workload(w: wl.Workload, n_q: int, device, decode_kernel: int):
                                  recent_window=w.recent_window, n_obs=w.n_obs, n_fit=w.n_fit,
                                  n_val=w.n_val, score_mode=w.score_mode,
                                  residual_override=w.residual_override(),
-                                 decode_kernel=decode_kernel)
+                                 decode_kernel=decode_kernel, budget_mode=budget_mode)
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
@@ -338,8 +342,10 @@ def main():
     kern = {"auto": R.RESKV_DECODE_AUTO, "mma": R.RESKV_DECODE_MMA,
             "cluster": R.RESKV_DECODE_CLUSTER, "fma": R.RESKV_DECODE_FMA,
             "lse": R.RESKV_DECODE_LSE_MERGE}[args.decode_kernel]
-    cache, Qdec, build_s = build_workload(w, n_q, device, kern)
+    bmode = R.RESKV_BUDGET_ADAKV if args.budget_mode == "adakv" else R.RESKV_BUDGET_UNIFORM
+    cache, Qdec, build_s = build_workload(w, n_q, device, kern, bmode)
     info = R.reskv_get_info(cache)
+    unit_budgets = R.reskv_get_unit_budgets(cache)
 
     def plan_name(cs, wpc):
         if kern == R.RESKV_DECODE_LSE_MERGE:
@@ -416,7 +422,7 @@ def main():
             "bound": "hbm", "achieved": alg / tg / 1e9, "peak": peak, "unit": "GB/s",
             "frac": alg / tg / 1e9 / peak, "kernel": decode_plan["per_layer"],
             "traffic": (profiled_traffic(units_layer, PROFILE_LAYER, KERNEL_SOURCES_LAYER)
-                        if info["layer_cluster"] > 0 else None),
+                        if info["layer_cluster"] > 0 and not info["ragged"] else None),
             "algorithmic_bytes_per_launch": alg // w.n_layers}
         del graph
 
@@ -459,6 +465,8 @@ def main():
                        "seq_len": w.seq_len, "budget": w.budget, "residual": w.residual,
                        "mean_r": float(np.mean(r_counts)),
                        "units_with_residual": float(np.mean(r_counts > 0)),
+                       "budget_mode": args.budget_mode,
+                       "unit_budget_min_max": [int(unit_budgets.min()), int(unit_budgets.max())],
                        "launch": "one reskv_decode_attn(layer=-1) launch per step",
                        "decode_plan": decode_plan,
                        "l2": f"inputs larger than L2: {alg / 1e9:.2f} GB of cache read per step",
@@ -467,7 +475,9 @@ def main():
             "frac_of_nominal_8tbs": achieved / 8000.0,
             "us_per_layer_step": ms_step * 1e3 / w.n_layers,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": profiled_traffic(units_launch),
+                         "frac": achieved / peak,
+                         # the summaries were captured on one-budget layouts
+                         "traffic": None if info["ragged"] else profiled_traffic(units_launch),
                          "peak_kind": f"{peak_kind} (burst copy)",
                          "algorithmic_bytes_per_launch": alg},
             "per_layer_graph": per_layer,

@@ -337,3 +337,91 @@ def test_adakv_cache_on_every_decode_path(kernel):
     R.reskv_check_status(cache)
     compare_decode(O, Qd, refs, lay, w, ocfg)
     cache.free()
+
+
+def test_adakv_fullsize_bench_workload_sampled():
+    """The benchmark workload (32 layers, s = 32768, b = 1024, batch 8) built
+    with AdaKV budgets, decoded in the launch configurations bench.py times.
+    Every (layer, batch element) keeps 8 x 1024 slots; two sampled groups'
+    allocations against the oracle; one unit of each against the oracle built
+    with its budget."""
+    import gc
+    w = wl.WORKLOADS["llama8b_32l_32k_b8"]
+    L, Bt, H, G = w.n_layers, w.batch, w.n_kv_heads, w.group
+    groups = [(3, 5), (27, 1)]                      # (layer, batch element)
+    Ks, Vs, Qs, kept = [], [], [], {}
+    Qd = torch.empty((L, Bt, H * G, w.head_dim), dtype=torch.bfloat16, device="cuda")
+    for l in range(L):
+        K, V, Qo, Qdec = wl.layer_inputs(w, l, "cuda", n_dec_steps=1)
+        Ks.append(K)
+        Vs.append(V)
+        Qs.append(Qo)
+        Qd[l] = Qdec[0]
+        for (gl, gb) in groups:
+            if gl == l:
+                kept[(gl, gb)] = (K[gb].cpu(), V[gb].cpu(), Qo[gb].cpu())
+    cfg = lib_config(w, budget_mode=R.RESKV_BUDGET_ADAKV)
+    cache = R.reskv_build_cache(cfg, Ks, Vs, Qs)
+    del Ks, Vs, Qs
+    gc.collect()
+    torch.cuda.empty_cache()
+    O = torch.full(Qd.shape, float("nan"), dtype=torch.float32, device="cuda")
+    R.reskv_decode_attn(cache, -1, Qd, O)
+    O_layers = torch.full(Qd.shape, float("nan"), dtype=torch.float32, device="cuda")
+    for l in range(L):
+        R.reskv_decode_attn(cache, l, Qd[l], O_layers[l])
+    torch.cuda.synchronize()
+    R.reskv_check_status(cache)
+    On = O.cpu().numpy()
+    assert not np.isnan(On).any()
+    assert np.abs(O_layers.cpu().numpy() - On).max() <= 1e-5 * max(1.0, np.abs(On).max())
+    budgets = R.reskv_get_unit_budgets(cache)
+    P = w.recent_window
+    f = int(np.floor(float(np.float32(SAFEGUARD)) * (w.budget - P)))
+    bg = budgets.reshape(L * Bt, H)
+    assert np.all(bg.sum(axis=1) == H * w.budget) and np.all(bg >= P + f)
+    assert len(np.unique(bg)) > 16, "the allocation is not ragged"
+    info = R.reskv_get_info(cache)
+    assert info["ragged"] == 1 and info["total_slots"] == w.n_units * w.budget
+    lay = R.reskv_export_cache(cache)
+    assert np.all(lay["n_main"] + lay["n_res"] == budgets)
+    scores = R.reskv_export_debug(cache, R.RESKV_DEBUG_SCORES)
+    top = R.reskv_export_debug(cache, R.RESKV_DEBUG_RANKED)
+    qf = bf16_to_f64(Qd)
+    for (gl, gb) in groups:
+        Kg, Vg, Qg = kept[(gl, gb)]
+        u0 = (gl * Bt + gb) * H
+        sl = slice(u0, u0 + H)
+        ref_scores = np.stack([orc.unit_scores(bf16_to_f64(Kg[h]), bf16_to_f64(Qg[h * G:(h + 1) * G]),
+                                               oracle_config(w, cfg, w.budget, u0 + h))
+                               for h in range(H)])
+        own = orc.adakv_budgets(scores[sl], w.budget, P, SAFEGUARD)
+        assert np.array_equal(own, budgets[sl]), f"group {(gl, gb)}: budgets vs its own scores"
+        ref = orc.adakv_budgets(ref_scores, w.budget, P, SAFEGUARD)
+        if not np.array_equal(ref, budgets[sl]):
+            assert pooled_gap(ref_scores, w.budget, P, SAFEGUARD) < NEAR_TIE
+        h = int(np.argmax(budgets[sl]))              # the head with the largest budget
+        u = u0 + h
+        bu = int(budgets[u])
+        K, V, Q = bf16_to_f64(Kg[h]), bf16_to_f64(Vg[h]), bf16_to_f64(Qg[h * G:(h + 1) * G])
+        oc = oracle_config(w, cfg, bu, u)
+        refu = orc.build_unit(K, V, Q, oc)
+        width = bu - P
+        check_ranking(scores[u], top[u, :width], refu.scores, P, False)
+        gu = unit_from_layout(lay, u)
+        Lr = refu.losses
+        rs = sorted(k for k in Lr if k > 0)
+        best = min(rs, key=lambda r: (Lr[r], r))
+        margin = abs(Lr[best] / Lr[0] - (1 - oc.delta)) if Lr[0] > 0 else 1.0
+        vals = sorted(Lr[r] for r in rs)
+        gap = (vals[1] - vals[0]) / vals[0] if len(vals) > 1 else 1.0
+        if min(margin, gap) > 1e-3:
+            assert gu.r == refu.r
+        check_entries(gu, K, V, top[u, :width], P, w.seq_len, bu, 4)
+        q = qf[gl, gb, h * G:(h + 1) * G]
+        out = On[gl, gb, h * G:(h + 1) * G]
+        assert_output_parity(out, orc.decode_unit(refu, q, oc), f"unit {u}")
+        assert_output_parity(out, orc.decode_unit(gu, q, oc), f"unit {u} (own cache)")
+    cache.free()
+    del O, O_layers, Qd
+    torch.cuda.empty_cache()
