@@ -214,6 +214,11 @@ typedef struct reskv_cache_info {
   int32_t n_candidates;    /* candidate columns of the validation proxy (the
                               losses array has 1 + n_candidates per unit)    */
   int32_t ranked_width;    /* entries per unit of RESKV_DEBUG_RANKED         */
+  int32_t all_units_per_warp;   /* tensor-core stream-K plan of an all-layer
+                              call: k > 0 when every warp takes k whole units
+                              (short units), 0 for equal slot pieces or when
+                              that call runs another kernel                 */
+  int32_t layer_units_per_warp; /* the same for a one-layer call (layer 0)   */
 } reskv_cache_info;
 
 reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info);

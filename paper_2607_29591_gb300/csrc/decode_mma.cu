@@ -60,7 +60,17 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     else return uu * b;
   };
   const int64_t gbase = ustart(p.unit0);
-  const int64_t ga = gbase + warp_begin(gw, T, W), ge = gbase + warp_begin(gw + 1, T, W);
+  int64_t ga, ge;
+  if (p.units_per_warp > 0) {            // whole units [gw k, (gw + 1) k)
+    const int64_t k = p.units_per_warp;
+    const int64_t u_lo = gw * k, u_hi = u_lo + k < p.n_units ? u_lo + k : p.n_units;
+    if (u_lo >= u_hi) return;
+    ga = ustart(p.unit0 + u_lo);
+    ge = ustart(p.unit0 + u_hi);
+  } else {                               // equal slot pieces
+    ga = gbase + warp_begin(gw, T, W);
+    ge = gbase + warp_begin(gw + 1, T, W);
+  }
   if (ga >= ge) return;
   // first unit with used slots in [ga, ge): the piece may start in the unused
   // tail slots of a unit (past its n_main + n_res + n_app used rows), which

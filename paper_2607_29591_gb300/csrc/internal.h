@@ -53,6 +53,10 @@ struct DecodeParams {
   int32_t gate_mode;
   int32_t softmax_mode;         // RESKV_SOFTMAX_*
   float tau, alpha, g_min, g_fixed;
+  int32_t units_per_warp;       // tensor-core stream-K kernel: 0 cuts the slot
+                                // range into n_warps equal pieces; k > 0 gives
+                                // warp w the whole units [w k, (w + 1) k) of the
+                                // launch instead (short units: no unit is cut)
 };
 
 constexpr int kDecodeWarpsPerCta = 8;

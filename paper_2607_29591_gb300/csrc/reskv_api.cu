@@ -150,6 +150,45 @@ int cluster_warps(int64_t budget, int cluster) {
                                std::max<int64_t>(1, (chunks + cluster - 1) / cluster)));
 }
 
+// Split plan of the tensor-core stream-K kernel for a launch of `n_units`
+// units holding `total_slots` slots: W warps, wpc per CTA, and k > 0 when
+// every warp takes k whole units instead of an equal slot piece.
+struct MmaPlan {
+  int64_t W = 1;
+  int wpc = kDecodeWarpsPerCta;
+  int32_t k = 0;
+};
+
+MmaPlan plan_mma(const reskv_cache* c, int64_t n_units, int64_t total_slots) {
+  MmaPlan m;
+  int64_t W = 0;
+  int wpc = kDecodeWarpsPerCta;
+  if (c->cfg.decode_warps > 0) {
+    W = c->cfg.decode_warps;
+  } else if (n_units >= c->num_sms && n_units <= 4 * int64_t(c->num_sms) &&
+             c->max_unit_slots <= 256 && !c->ragged) {
+    W = n_units;                      // one warp per unit: no partial records at all
+  } else {
+    wpc = int(std::min<int64_t>(8, std::max<int64_t>(1, total_slots / (int64_t(c->num_sms) * 200))));
+    W = int64_t(c->num_sms) * wpc;
+    if (total_slots < W * 32) W = std::max<int64_t>(1, total_slots / 32);
+  }
+  if (W > total_slots) W = total_slots;
+  if (W > c->max_warps) W = c->max_warps;
+  if (W < 1) W = 1;
+  // Short units (each at most an eighth of a warp's piece): every warp takes
+  // k consecutive whole units, so no unit is cut and no partial record,
+  // ticket or merge is needed; the warps' loads differ by at most one unit.
+  if (c->cfg.decode_warps == 0 && int64_t(c->max_unit_slots) * 8 * W <= total_slots) {
+    const int64_t k = (n_units + W - 1) / W;
+    W = (n_units + k - 1) / k;
+    m.k = int32_t(k);
+  }
+  m.W = W;
+  m.wpc = int(std::min<int64_t>(8, (W + c->num_sms - 1) / c->num_sms));
+  return m;
+}
+
 // Cluster decode shape for launches of `units` units: the largest cluster
 // (at most 8 CTAs, at most SMs / units) at which all of the launch's clusters
 // are resident at once; cluster = 0 if not even single-CTA clusters are.
@@ -461,21 +500,10 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   int64_t W = 0;
   int wpc = kDecodeWarpsPerCta;
   if (mma) {
-    if (cfg.decode_warps > 0) {
-      W = cfg.decode_warps;
-    } else {
-      if (p.n_units >= c->num_sms && p.n_units <= 4 * int64_t(c->num_sms) &&
-          c->max_unit_slots <= 256 && !c->ragged) {
-        W = p.n_units;                // one warp per unit: no partial records at all
-      } else {
-        wpc = int(std::min<int64_t>(8, std::max<int64_t>(1, p.total_slots / (int64_t(c->num_sms) * 200))));
-        W = int64_t(c->num_sms) * wpc;
-        if (p.total_slots < W * 32) W = std::max<int64_t>(1, p.total_slots / 32);
-      }
-    }
-    if (W > p.total_slots) W = p.total_slots;
-    if (W > c->max_warps) W = c->max_warps;
-    wpc = int(std::min<int64_t>(8, (W + c->num_sms - 1) / c->num_sms));
+    const MmaPlan mp = plan_mma(c, p.n_units, p.total_slots);
+    W = mp.W;
+    wpc = mp.wpc;
+    p.units_per_warp = mp.k;
   } else {
     W = cfg.decode_warps > 0 ? cfg.decode_warps : p.total_slots / 32;
     if (W > p.total_slots) W = p.total_slots;
@@ -564,6 +592,14 @@ reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info) {
       info->all_cluster ? (c->cplan_all.cluster ? c->cplan_all.warps_per_cta
                                                 : cluster_warps(c->max_unit_slots, 1))
                         : 0;
+  const int64_t per_layer = int64_t(c->cfg.batch) * c->cfg.n_kv_heads;
+  const bool mma_all = c->cfg.decode_kernel == RESKV_DECODE_MMA ||
+                       (auto_plan && c->cplan_all.cluster == 0);
+  const bool mma_layer = c->cfg.decode_kernel == RESKV_DECODE_MMA ||
+                         (auto_plan && c->cplan_layer.cluster == 0);
+  info->all_units_per_warp = mma_all ? plan_mma(c, c->n_units, c->total_slots).k : 0;
+  info->layer_units_per_warp =
+      mma_layer ? plan_mma(c, per_layer, c->h_offsets[size_t(per_layer)]).k : 0;
   info->n_candidates = c->n_candidates;
   info->ranked_width = int32_t(c->dbg_ranked ? c->dbg_n_top : c->ranked_width);
   return RESKV_OK;

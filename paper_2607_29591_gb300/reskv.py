@@ -71,7 +71,8 @@ class reskv_cache_info(ctypes.Structure):
                 ("append_capacity", ctypes.c_int32), ("stride", ctypes.c_int32),
                 ("max_appended", ctypes.c_int32), ("ragged", ctypes.c_int32),
                 ("total_slots", ctypes.c_int64), ("n_candidates", ctypes.c_int32),
-                ("ranked_width", ctypes.c_int32)]
+                ("ranked_width", ctypes.c_int32), ("all_units_per_warp", ctypes.c_int32),
+                ("layer_units_per_warp", ctypes.c_int32)]
 
 
 class reskv_device_cache(ctypes.Structure):
