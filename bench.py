@@ -386,6 +386,10 @@ def main():
     launch_s = t_local / args.steps                      # one launch per step
     peak, peak_kind = measured_peak_gbs()
     achieved = alg / launch_s / 1e9
+    # Q (bf16) read and O (fp32) written by the step: necessary traffic outside
+    # the algorithmic cache bytes (1 KB + 2 KB per unit: 0.6 % of the bytes at
+    # b = 1024, 4.7 % at b = 128)
+    qo_bytes = int(w.n_units * w.group * w.head_dim * (2 + 4))
 
     # ---- per-layer calls (one launch per layer) captured in a CUDA graph ----
     per_layer = None
@@ -472,6 +476,8 @@ def main():
                        "l2": f"inputs larger than L2: {alg / 1e9:.2f} GB of cache read per step",
                        "parallelism": "replicas" if world > 1 else "single GPU"},
             "hbm_gbs": achieved, "frac_of_peak": achieved / peak,
+            "q_o_bytes_per_step": qo_bytes,
+            "hbm_gbs_with_q_o": (alg + qo_bytes) / launch_s / 1e9,
             "frac_of_nominal_8tbs": achieved / 8000.0,
             "us_per_layer_step": ms_step * 1e3 / w.n_layers,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
