@@ -291,6 +291,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   int32_t *r_runs = nullptr, *r_final = nullptr, *chosen = nullptr, *run_off_d = nullptr;
   int32_t* budgets_d = nullptr;        // [U_all] per-unit budgets (per_unit only)
   float *centersT = nullptr, *cnorm = nullptr, *vpart = nullptr, *oS = nullptr;
+  __nv_bfloat16* cplanes = nullptr;
   double* centers64 = nullptr;
   __nv_bfloat16 *kbar = nullptr, *vbar = nullptr;
   double *rowerr = nullptr, *losses = nullptr;
@@ -308,6 +309,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
          S.get(&ccount, size_t(UL) * rmax) && S.get(&cbase, size_t(UL) * rmax) &&
          S.get(&members, US) && S.get(&centersT, size_t(UL) * kHeadDim * rmax) &&
          S.get(&centers64, size_t(UL) * kHeadDim * rmax) &&
+         S.get(&cplanes, size_t(UL) * 3 * rmax * kHeadDim) &&
          S.get(&cnorm, size_t(UL) * rmax) && S.get(&kbar, size_t(UL) * ent_stride * kHeadDim) &&
          S.get(&vbar, size_t(UL) * ent_stride * kHeadDim) &&
          S.get(&ecount, size_t(UL) * ent_stride);
@@ -350,8 +352,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   const size_t sm_obs1 = size_t(kHeadDim) * (kTile + kRowBlk) * 4;
   const size_t sm_obs2 = sm_obs1 + size_t(8) * kTile * 4;
   const size_t sm_top = size_t(kTopMax) * 12 + (256 + 32 + 4) * 4;
-  const size_t sm_assign = (size_t(kHeadDim) * (kTile + kRowBlk) + kRowBlk + kTile) * 4 +
-                           size_t(8) * kTile * 3 * 4 + size_t(std::max(rmax, 1)) * 4;
+  const size_t sm_assign = lloyd_assign_smem(rmax);
   const size_t sm_val = size_t(kHeadDim) * (2 * kTile + 2 * kRowBlk) * 4;
   if (set_smem(k_obs_pass1, sm_obs1) != cudaSuccess || set_smem(k_obs_pass2, sm_obs2) != cudaSuccess ||
       set_smem(k_topk, sm_top) != cudaSuccess || set_smem(k_lloyd_assign, sm_assign) != cudaSuccess ||
@@ -436,7 +437,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
 
     LloydArgs la{K, V, s, P, n_top, b, ntiles, rmax, top, rank_pos, nullptr, centersT, cnorm,
                  centers64, assign, hist, ccount, cbase, members, kbar, vbar, ecount,
-                 ent_stride, 0, c->status, bl_d};
+                 ent_stride, 0, c->status, bl_d, cplanes};
     auto lloyd_run = [&](const int32_t* r_unit, int ent_off, int r_hi) -> reskv_status {
       la.r_unit = r_unit;
       la.ent_off = ent_off;

@@ -10,6 +10,7 @@
 
 #include "device_utils.cuh"
 #include "internal.h"
+#include "mma_tile.cuh"
 
 namespace reskv {
 namespace build {
@@ -550,12 +551,28 @@ struct LloydArgs {
   int32_t ent_off;
   uint32_t* status;
   const int32_t* budgets;      // [UL] per-unit budgets, or NULL (budget)
+  __nv_bfloat16* cplanes;      // [UL, 3, rmax, d] the fp32 centres split into
+                               // three bf16 planes c1 + c2 + c3 (tensor-core operands)
 };
 
 __device__ __forceinline__ bool in_evicted(const LloydArgs& p, int ul, int64_t pos, int r) {
   const int32_t rk = p.rank_pos[int64_t(ul) * p.s + pos];
   const int32_t keep = int32_t(unit_budget(p.budgets, ul, p.budget)) - r - p.recent;  // ranked main
   return rk >= 0 && rk >= keep;
+}
+
+// The bf16 planes of centre j, dim d: c = c1 + c2 + c3 + e, |e| <= 2^-24 |c|
+// (each remainder is exact in fp32; every plane keeps 8 significant bits).
+__device__ __forceinline__ void write_planes(const LloydArgs& p, int ul, int j, int d, float c) {
+  const __nv_bfloat16 c1 = __float2bfloat16_rn(c);
+  const float r1 = c - __bfloat162float(c1);
+  const __nv_bfloat16 c2 = __float2bfloat16_rn(r1);
+  const float r2 = r1 - __bfloat162float(c2);
+  const __nv_bfloat16 c3 = __float2bfloat16_rn(r2);
+  __nv_bfloat16* b = p.cplanes + (int64_t(ul) * 3 * p.rmax + j) * kHeadDim + d;
+  b[0] = c1;
+  b[int64_t(p.rmax) * kHeadDim] = c2;
+  b[int64_t(2) * p.rmax * kHeadDim] = c3;
 }
 
 // centre j = key of the (m - |P| + j)-th ranked token
@@ -568,6 +585,7 @@ __global__ void k_lloyd_init(LloydArgs p) {
   const int32_t pos = p.top[int64_t(ul) * p.n_top + keep + j];
   const float c = __bfloat162float(p.K[(int64_t(ul) * p.s + pos) * kHeadDim + d]);
   p.centersT[(int64_t(ul) * kHeadDim + d) * p.rmax + j] = c;
+  write_planes(p, ul, j, d, c);
   p.centers64[(int64_t(ul) * p.rmax + j) * kHeadDim + d] = double(c);
   red[d] = c * c;
   __syncthreads();
@@ -580,129 +598,211 @@ __global__ void k_lloyd_init(LloydArgs p) {
 
 // Nearest centre of every evicted token of a 128-token tile; per-tile counts.
 //
-// The choice is certified in fp64: distances are first evaluated in fp32
-// (||c||^2 - 2<c,k>, the ||k||^2 term being common) keeping the three best
-// centres per token; a rigorous bound on the fp32 error of each distance
-// (dot products of 128 terms with fused multiply-adds, fp32-rounded centres)
-// decides whether the runner-up could in truth be nearer.  Only then are the
-// candidates re-evaluated as sum_i (k_i - c_i)^2 in fp64 against the fp64
-// centres -- all centres if even the third is within the bound.  Ties go to the
-// lower centre index.
+// Distances d_j = ||c_j||^2 - 2<c_j, k> (the ||k||^2 term is common) come from
+// the tensor cores: the keys are bf16 (exact operands) and every fp32 centre
+// is split exactly into three bf16 planes, c = c1 + c2 + c3 + e with
+// |e_i| <= 2^-24 |c_i|.  <c1, k> is taken one 16-dim step at a time (a fresh
+// fp32 accumulator per mma.sync m16n8k16, added in IEEE fp32), the small
+// planes <c2 + c3, k> in one accumulator chain.  The choice is certified in
+// fp64: the four best centres per token are kept, and a bound on the error of
+// the computed distances decides whether the runner-ups could in truth be
+// nearer; only then are the candidates (all centres if even the fourth is
+// within the bound) re-evaluated as sum_i (k_i - c_i)^2 in fp64 against the
+// fp64 centres.  Ties go to the lower centre index.
+//
+// Error bound of the dot product, with P = sum_i |c_i k_i| <= ||c|| ||k|| and
+// u = 2^-24: the 16 exact products of one MMA step are summed with an error
+// of at most 16 * 2^-22 max|p| even if the accumulation truncates to 24 bits
+// (64u P over the eight steps), the result's normalisation and the fp32 adds
+// add 10u P, the chain of the small planes (|c2 + c3| <= 2^-8 |c|) at most
+// 9u P, the split u P: about 84u P, taken as 256u.
 struct Cand {
   float d;
   int j;
 };
 
-__device__ __forceinline__ void cand_insert(Cand* t, float d, int j) {
-  // keeps t[0..2] sorted by (d, j); centres arrive in increasing j per thread
-  if (d < t[2].d || (d == t[2].d && j < t[2].j)) {
-    t[2] = Cand{d, j};
-    if (t[2].d < t[1].d || (t[2].d == t[1].d && t[2].j < t[1].j)) {
-      Cand x = t[1]; t[1] = t[2]; t[2] = x;
-      if (t[1].d < t[0].d || (t[1].d == t[0].d && t[1].j < t[0].j)) {
-        x = t[0]; t[0] = t[1]; t[1] = x;
-      }
-    }
-  }
+__device__ __forceinline__ bool cand_before(float d, int j, const Cand& c) {
+  return d < c.d || (d == c.d && j < c.j);
 }
 
-__device__ __forceinline__ double dist64(const float* Kt, int tok, const double* c) {
+// keeps t[0..3] sorted by (d, j)
+__device__ __forceinline__ void cand_insert4(Cand* t, float d, int j) {
+  if (!cand_before(d, j, t[3])) return;
+  t[3] = Cand{d, j};
+#pragma unroll
+  for (int q = 3; q > 0; --q)
+    if (cand_before(t[q].d, t[q].j, t[q - 1])) {
+      const Cand x = t[q - 1];
+      t[q - 1] = t[q];
+      t[q] = x;
+    }
+}
+
+constexpr int kAsgNB = 64;                  // centres per staged block
+constexpr int kAsgRowBytes = kHeadDim * 2;  // one bf16 row (key or centre plane)
+
+// byte offset of 16-byte chunk `ch` of row `row` in a [rows][256 B] bf16 tile;
+// chunks XOR-swizzled by row so that ldmatrix reads of 8 rows are conflict free
+__device__ __forceinline__ uint32_t asg_swz(int row, int ch) {
+  return uint32_t(row) * kAsgRowBytes + uint32_t((ch ^ (row & 7)) << 4);
+}
+
+__device__ __forceinline__ float asg_key(const uint8_t* Ks, int tok, int i) {
+  const __nv_bfloat16* r =
+      reinterpret_cast<const __nv_bfloat16*>(Ks + asg_swz(tok, i >> 3));
+  return __bfloat162float(r[i & 7]);
+}
+
+__device__ __forceinline__ double dist64_bf16(const uint8_t* Ks, int tok, const double* c) {
   double acc = 0.0;
   for (int i = 0; i < kHeadDim; ++i) {
-    const double df = double(Kt[kt_index(i, tok)]) - c[i];
+    const double df = double(asg_key(Ks, tok, i)) - c[i];
     acc = fma(df, df, acc);
   }
   return acc;
 }
 
+// Shared memory of k_lloyd_assign: the key tile, one block of centre planes
+// and the tile's histogram of `rmax` centres.
+inline size_t lloyd_assign_smem(int rmax) {
+  return size_t(kTile) * kAsgRowBytes + size_t(3) * kAsgNB * kAsgRowBytes +
+         size_t(rmax > 0 ? rmax : 1) * 4;
+}
+
 __global__ void __launch_bounds__(kThreads, 2) k_lloyd_assign(LloydArgs p) {
-  extern __shared__ __align__(16) float sm[];
-  float* Kt = sm;                                   // [128][128]
-  float* Ct = Kt + kHeadDim * kTile;                // [128][32]; later candidate distances
-  float* cn = Ct + kHeadDim * kRowBlk;              // [32]
-  float* knrm = cn + kRowBlk;                       // [128] ||k|| per token
-  int* cj = reinterpret_cast<int*>(knrm + kTile);   // [8][128][3] candidate centres
-  int* cnt = cj + 8 * kTile * 3;                    // [rmax] tile histogram
-  float* cd = Ct;                                   // [8][128][3] candidate distances
-  __shared__ unsigned int cnmax_bits;               // max ||c||^2 over the unit's centres
+  extern __shared__ __align__(128) uint8_t asm_raw[];
+  uint8_t* Ks = asm_raw;                                        // [128 tok][256 B]
+  uint8_t* Cs = Ks + kTile * kAsgRowBytes;                      // [3][64 centres][256 B]
+  int* cnt = reinterpret_cast<int*>(Cs + 3 * kAsgNB * kAsgRowBytes);   // [r]
+  __shared__ float cn_s[kAsgNB];
+  __shared__ unsigned int cnmax_bits;                           // max ||c||^2 of the unit
   const int tile = blockIdx.x, ul = blockIdx.y;
   const int r = p.r_unit[ul];
   if (r == 0) return;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3;
   const int64_t tok0 = int64_t(tile) * kTile;
-  load_kt(Kt, p.K + int64_t(ul) * p.s * kHeadDim, p.s, tok0);
+  const __nv_bfloat16* Ku = p.K + int64_t(ul) * p.s * kHeadDim;
+  for (int idx = threadIdx.x; idx < kTile * 16; idx += blockDim.x) {
+    const int row = idx >> 4, ch = idx & 15;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (tok0 + row < p.s)
+      v = __ldg(reinterpret_cast<const uint4*>(Ku + (tok0 + row) * kHeadDim) + ch);
+    *reinterpret_cast<uint4*>(Ks + asg_swz(row, ch)) = v;
+  }
   for (int i = threadIdx.x; i < r; i += blockDim.x) cnt[i] = 0;
   if (threadIdx.x == 0) cnmax_bits = 0u;
-  Cand best[4][3];
+  __syncthreads();
+
+  // A fragments of this warp's 16 tokens for the eight 16-dim steps
+  const uint32_t ks_s = smem_u32(Ks), cs_s = smem_u32(Cs);
+  uint32_t A[8][4];
+  {
+    const int row = w * 16 + (mi & 1) * 8 + (lane & 7);
 #pragma unroll
-  for (int j = 0; j < 4; ++j)
+    for (int ks = 0; ks < 8; ++ks)
+      ldsm_x4(ks_s + asg_swz(row, 2 * ks + (mi >> 1)), A[ks][0], A[ks][1], A[ks][2], A[ks][3]);
+  }
+  Cand best[2][4];                      // tokens g and g + 8 of the warp's 16
 #pragma unroll
-    for (int q = 0; q < 3; ++q) best[j][q] = Cand{INFINITY, 0x7fffffff};
-  for (int cb = 0; cb < r; cb += kRowBlk) {
-    __syncthreads();
-    for (int idx = threadIdx.x; idx < kHeadDim * kRowBlk; idx += blockDim.x) {
-      const int k = idx / kRowBlk, c = idx % kRowBlk;
-      Ct[idx] = (cb + c < r) ? p.centersT[(int64_t(ul) * kHeadDim + k) * p.rmax + cb + c] : 0.f;
+  for (int a = 0; a < 2; ++a)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) best[a][q] = Cand{INFINITY, 0x7fffffff};
+
+  for (int cb = 0; cb < r; cb += kAsgNB) {
+    __syncthreads();                    // the previous block's planes are consumed
+    const int nb = r - cb < kAsgNB ? r - cb : kAsgNB;
+    for (int idx = threadIdx.x; idx < 3 * kAsgNB * 16; idx += blockDim.x) {
+      const int pl = idx / (kAsgNB * 16), rem = idx % (kAsgNB * 16);
+      const int row = rem >> 4, ch = rem & 15;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (row < nb)
+        v = *(reinterpret_cast<const uint4*>(
+                  p.cplanes + ((int64_t(ul) * 3 + pl) * p.rmax + cb + row) * kHeadDim) + ch);
+      *reinterpret_cast<uint4*>(Cs + pl * (kAsgNB * kAsgRowBytes) + asg_swz(row, ch)) = v;
     }
-    if (threadIdx.x < kRowBlk) {
-      const float v = (cb + threadIdx.x < r) ? p.cnorm[int64_t(ul) * p.rmax + cb + threadIdx.x] : 0.f;
-      cn[threadIdx.x] = v;
+    if (threadIdx.x < kAsgNB) {
+      const float v = threadIdx.x < nb ? p.cnorm[int64_t(ul) * p.rmax + cb + threadIdx.x] : 0.f;
+      cn_s[threadIdx.x] = v;
       atomicMax(&cnmax_bits, __float_as_uint(v));   // non-negative: bit order = value order
     }
     __syncthreads();
-    float S[4][4];
-    tile_logits(Ct, Kt, S);                         // <c_i, k_j> for centres 4w+i
+    for (int np = 0; np * 16 < nb; ++np) {          // 16 centres: two n-tiles of 8
+      const int crow = np * 16 + (mi >> 1) * 8 + (lane & 7);
+      float acc[2][4], lo[2][4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int c = cb + 4 * w + i;
-      if (c >= r) continue;
+      for (int e = 0; e < 4; ++e) acc[0][e] = acc[1][e] = lo[0][e] = lo[1][e] = 0.f;
 #pragma unroll
-      for (int j = 0; j < 4; ++j) cand_insert(best[j], cn[4 * w + i] - 2.0f * S[i][j], c);
-    }
-  }
-  __syncthreads();                                  // Ct is reused for the candidates
-  if (threadIdx.x < kTile) {                        // ||k|| of token threadIdx.x
-    float n = 0.f;
-    for (int i = 0; i < kHeadDim; ++i) {
-      const float x = Kt[kt_index(i, threadIdx.x)];
-      n = fmaf(x, x, n);
-    }
-    knrm[threadIdx.x] = sqrtf(n);
-  }
+      for (int ks = 0; ks < 8; ++ks) {
+        const uint32_t co = asg_swz(crow, 2 * ks + (mi & 1));
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4(cs_s + co, b0, b1, b2, b3);
+        float t0[4] = {0.f, 0.f, 0.f, 0.f}, t1[4] = {0.f, 0.f, 0.f, 0.f};
+        mma16816(t0, A[ks][0], A[ks][1], A[ks][2], A[ks][3], b0, b1);
+        mma16816(t1, A[ks][0], A[ks][1], A[ks][2], A[ks][3], b2, b3);
 #pragma unroll
-  for (int j = 0; j < 4; ++j)
-#pragma unroll
-    for (int q = 0; q < 3; ++q) {
-      const int o = (w * kTile + 4 * lane + j) * 3 + q;
-      cd[o] = best[j][q].d;
-      cj[o] = best[j][q].j;
-    }
-  __syncthreads();
-  if (threadIdx.x < kTile) {
-    const int t = threadIdx.x;
-    const int64_t pos = tok0 + t;
-    if (pos < p.s && in_evicted(p, ul, pos, r)) {
-      Cand top[3] = {{INFINITY, 0x7fffffff}, {INFINITY, 0x7fffffff}, {INFINITY, 0x7fffffff}};
-      for (int ww = 0; ww < 8; ++ww)
-        for (int q = 0; q < 3; ++q) {
-          const int o = (ww * kTile + t) * 3 + q;
-          if (cj[o] < r) cand_insert(top, cd[o], cj[o]);
+        for (int e = 0; e < 4; ++e) {
+          acc[0][e] += t0[e];
+          acc[1][e] += t1[e];
         }
-      // Bound on the fp32 error of d_j = ||c_j||^2 - 2<c_j, k> for any centre:
-      // 128-term fused dot product (gamma ~ 130 u), fp32 rounding of the fp64
-      // centre (u per coordinate), the norm sum and the final subtraction,
-      // with ||c_j|| <= max ||c||, times a safety factor 2.  A centre outside
-      // the fp32 top three lies at least d_3 - d_1 above the best in fp32.
-      const float gam = 130.0f * 5.9604645e-8f, u = 5.9604645e-8f;
-      const float kn = knrm[t];
-      const float cm = sqrtf(__uint_as_float(cnmax_bits));
-      float err[3];
+#pragma unroll
+        for (int pl = 1; pl < 3; ++pl) {
+          ldsm_x4(cs_s + pl * (kAsgNB * kAsgRowBytes) + co, b0, b1, b2, b3);
+          mma16816(lo[0], A[ks][0], A[ks][1], A[ks][2], A[ks][3], b0, b1);
+          mma16816(lo[1], A[ks][0], A[ks][1], A[ks][2], A[ks][3], b2, b3);
+        }
+      }
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int cl = np * 16 + nt * 8 + 2 * t4 + (e & 1);   // accumulator column
+          if (cl < nb)
+            cand_insert4(best[e >> 1], cn_s[cl] - 2.0f * (acc[nt][e] + lo[nt][e]), cb + cl);
+        }
+    }
+  }
+  // every lane of a quad ends with the quad's four best centres per token
+#pragma unroll
+  for (int off = 1; off <= 2; off <<= 1)
+#pragma unroll
+    for (int a = 0; a < 2; ++a) {
+      Cand o[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        o[q].d = __shfl_xor_sync(0xffffffffu, best[a][q].d, off);
+        o[q].j = __shfl_xor_sync(0xffffffffu, best[a][q].j, off);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) cand_insert4(best[a], o[q].d, o[q].j);
+    }
+
+  if (t4 < 2) {                          // lane t4 of the quad: token g + 8 t4
+    const int tt = w * 16 + g + 8 * t4;
+    const int64_t pos = tok0 + tt;
+    Cand top[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) top[q] = t4 == 0 ? best[0][q] : best[1][q];
+    if (pos < p.s && in_evicted(p, ul, pos, r)) {
+      float kn2 = 0.f;
+      for (int i = 0; i < kHeadDim; ++i) {
+        const float x = asg_key(Ks, tt, i);
+        kn2 = fmaf(x, x, kn2);
+      }
+      // err(d_q): 2 x (dot product 2 gam_tc ||c|| ||k|| + norm sum 2 gam ||c||^2
+      // + fp32 centre 4u ||k|| ||c|| + final subtraction 2u |d_q|), with
+      // ||c|| <= max ||c|| over the unit; a centre outside the four kept lies
+      // at least d_4 - d_1 above the best.
+      const float u = 5.9604645e-8f, gam = 130.0f * u, gam_tc = 256.0f * u;
+      const float kn = sqrtf(kn2), cm = sqrtf(__uint_as_float(cnmax_bits));
+      float err[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        err[q] = 2.0f * (2.0f * gam_tc * cm * kn + 2.0f * gam * cm * cm + 4.0f * u * kn * cm +
+                         2.0f * u * fabsf(top[q].d));
       int n_amb = 1;
 #pragma unroll
-      for (int q = 0; q < 3; ++q)
-        err[q] = 2.0f * (2.0f * gam * cm * kn + 2.0f * gam * cm * cm + 4.0f * u * kn * cm +
-                         2.0f * u * fabsf(top[q].d));
-      for (int q = 1; q < 3; ++q)
+      for (int q = 1; q < 4; ++q)
         if (top[q].j < r && top[q].d - top[0].d <= err[0] + err[q]) n_amb = q + 1;
       int j0 = top[0].j;
       if (j0 >= r) {                                  // only a NaN distance gets here
@@ -712,18 +812,20 @@ __global__ void __launch_bounds__(kThreads, 2) k_lloyd_assign(LloydArgs p) {
         const double* c64 = p.centers64 + int64_t(ul) * p.rmax * kHeadDim;
         double bd = INFINITY;
         int bj = j0;
-        if (n_amb < 3) {
-          for (int q = 0; q < n_amb; ++q) {
+        if (n_amb < 4) {
+#pragma unroll
+          for (int q = 0; q < 3; ++q) {
+            if (q >= n_amb) break;
             const int j = top[q].j;
-            const double dd = dist64(Kt, t, c64 + int64_t(j) * kHeadDim);
+            const double dd = dist64_bf16(Ks, tt, c64 + int64_t(j) * kHeadDim);
             if (dd < bd || (dd == bd && j < bj)) {
               bd = dd;
               bj = j;
             }
           }
-        } else {                                      // three or more within the bound
+        } else {                                      // four or more within the bound
           for (int j = 0; j < r; ++j) {
-            const double dd = dist64(Kt, t, c64 + int64_t(j) * kHeadDim);
+            const double dd = dist64_bf16(Ks, tt, c64 + int64_t(j) * kHeadDim);
             if (dd < bd) {
               bd = dd;
               bj = j;
@@ -852,6 +954,7 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_update(LloydArgs p, int fina
       mk = tk / double(cnt);
       *c64 = mk;
       *cptr = float(mk);
+      write_planes(p, ul, j, d, float(mk));
     } else {
       mk = *c64;                        // an empty cluster keeps its centre
     }
