@@ -309,7 +309,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
          S.get(&ccount, size_t(UL) * rmax) && S.get(&cbase, size_t(UL) * rmax) &&
          S.get(&members, US) && S.get(&centersT, size_t(UL) * kHeadDim * rmax) &&
          S.get(&centers64, size_t(UL) * kHeadDim * rmax) &&
-         S.get(&cplanes, size_t(UL) * 3 * rmax * kHeadDim) &&
+         S.get(&cplanes, size_t(UL) * 2 * rmax * kHeadDim) &&
          S.get(&cnorm, size_t(UL) * rmax) && S.get(&kbar, size_t(UL) * ent_stride * kHeadDim) &&
          S.get(&vbar, size_t(UL) * ent_stride * kHeadDim) &&
          S.get(&ecount, size_t(UL) * ent_stride);
