@@ -425,3 +425,56 @@ def test_adakv_fullsize_bench_workload_sampled():
     cache.free()
     del O, O_layers, Qd
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("group", [2, 4])
+def test_adakv_build_then_append(group):
+    """AdaKV construction at the wider unit stride (append capacity 6), then
+    three rounds of appended tokens: every unit's exact main cache grows
+    inside its own region and decodes (all-layer and per-layer) against the
+    oracle's cache grown by append_tokens."""
+    w = wl.scaled(wl.WORKLOADS["llama8b_layer_32k"], seq_len=1024, budget=160, batch=2,
+                  n_kv_heads=3, n_layers=2, group=group)
+    A = 6
+    (Ks, Vs, Qs), (Kd, Vd, Qdv) = make_inputs(w, sharpen_head=1)
+    cfg = lib_config(w, budget_mode=R.RESKV_BUDGET_ADAKV, append_capacity=A)
+    cache = R.reskv_build_cache(cfg, Kd, Vd, Qdv)
+    budgets = R.reskv_get_unit_budgets(cache)
+    assert budgets.reshape(-1, w.n_kv_heads).sum(axis=1).tolist() == [3 * 160] * (2 * 2)
+    lay = R.reskv_export_cache(cache)
+    assert np.array_equal(np.diff(lay["offsets"]), budgets + A)
+    units = {u: unit_from_layout(lay, u) for u in range(w.n_units)}
+    ocfg = lambda u: oracle_config(w, cfg, budgets[u], u)
+    g = torch.Generator().manual_seed(5)
+    for rnd in range(3):
+        kn = torch.randn((w.n_layers, w.batch, w.n_kv_heads, 128), generator=g).to(torch.bfloat16)
+        vn = torch.randn((w.n_layers, w.batch, w.n_kv_heads, 128), generator=g).to(torch.bfloat16)
+        if rnd == 1:
+            for l in range(w.n_layers):
+                R.reskv_append(cache, l, kn[l].cuda().contiguous(), vn[l].cuda().contiguous())
+        else:
+            R.reskv_append(cache, -1, kn.cuda().contiguous(), vn.cuda().contiguous())
+        kf, vf = bf16_to_f64(kn), bf16_to_f64(vn)
+        for u in range(w.n_units):
+            l, rem = divmod(u, w.batch * w.n_kv_heads)
+            b, h = divmod(rem, w.n_kv_heads)
+            units[u] = orc.append_tokens(units[u], kf[l, b, h][None], vf[l, b, h][None],
+                                         np.array([w.seq_len + rnd]))
+        # queries aimed at the newest token of every unit
+        Q = torch.empty((w.n_layers, w.batch, w.n_q_heads, 128), dtype=torch.bfloat16)
+        for l in range(w.n_layers):
+            for b in range(w.batch):
+                for h in range(w.n_kv_heads):
+                    Q[l, b, h * group:(h + 1) * group] = (kn[l, b, h].float() * 0.5).to(torch.bfloat16)
+        out = decode_all(cache, Q.cuda())
+        lay2 = R.reskv_export_cache(cache)
+        assert np.all(lay2["n_app"] == rnd + 1)
+        compare_decode(out, Q, units, lay2, w, ocfg)
+        O_l = np.zeros_like(out)
+        for l in range(w.n_layers):
+            Ol = torch.empty(Q.shape[1:], dtype=torch.float32, device="cuda")
+            R.reskv_decode_attn(cache, l, Q[l].cuda().contiguous(), Ol)
+            torch.cuda.synchronize()
+            O_l[l] = Ol.cpu().numpy()
+        compare_decode(O_l, Q, units, lay2, w, ocfg)
+    cache.free()

@@ -102,3 +102,39 @@ def test_whole_units_per_warp(ragged):
         assert_output_parity(Oa[l, b, h * G:(h + 1) * G], ref, f"unit {u}")
     auto.free()
     pieces.free()
+
+
+def test_whole_units_per_warp_with_appended_rows():
+    """The whole-unit split on units that also hold rows appended at decode
+    time (append capacity 4, two appends): against the equal-piece split."""
+    U = L * BT * H
+    budgets = np.full(U, 32, np.int32)
+    lay = random_layout(budgets, 21)
+    A = 4
+    S = 32 + A
+    arrs = {}
+    for k in ("kslots", "vslots"):
+        a = lay[k].reshape(U, 32, D)
+        arrs[k] = np.concatenate([a, np.zeros((U, A, D), np.uint16)], axis=1)
+    for k, fill in (("logc", 0), ("slot_pos", -1), ("counts", 0)):
+        a = lay[k].reshape(U, 32)
+        arrs[k] = np.concatenate([a, np.full((U, A), fill, a.dtype)], axis=1)
+    arrs["n_main"], arrs["n_res"] = lay["n_main"], lay["n_res"]
+    shape = dict(batch=BT, n_layers=L, n_kv_heads=H, group=G, seq_len=4096, budget=32,
+                 append_capacity=A)
+    auto = R.reskv_import_cache(R.reskv_config_default(**shape), **arrs)
+    assert R.reskv_get_info(auto)["all_units_per_warp"] > 1
+    pieces = R.reskv_import_cache(R.reskv_config_default(decode_kernel=R.RESKV_DECODE_MMA,
+                                                         decode_warps=1216, **shape), **arrs)
+    g = torch.Generator().manual_seed(9)
+    for _ in range(2):
+        kn = torch.randn((L, BT, H, D), generator=g).to(torch.bfloat16).cuda()
+        vn = torch.randn((L, BT, H, D), generator=g).to(torch.bfloat16).cuda()
+        R.reskv_append(auto, -1, kn, vn)
+        R.reskv_append(pieces, -1, kn, vn)
+    Q = torch.randn((L, BT, H * G, D), generator=g).to(torch.bfloat16).cuda()
+    Oa, Op = decode(auto, Q), decode(pieces, Q)
+    assert not np.isnan(Oa).any()
+    assert errors(Oa, Op.astype(np.float64))[1] < 1e-5
+    auto.free()
+    pieces.free()
