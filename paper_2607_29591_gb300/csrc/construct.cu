@@ -349,8 +349,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     return cleanup_fail(fail(RESKV_ERR_CUDA, "copying run tables"));
 
   // kernel attributes
-  const size_t sm_obs1 = size_t(kHeadDim) * (kTile + kRowBlk) * 4;
-  const size_t sm_obs2 = sm_obs1 + size_t(8) * kTile * 4;
+  const size_t sm_obs1 = size_t(kTile) * kAsgRowBytes;               // the key tile
+  const size_t sm_obs2 = sm_obs1 + size_t(kThreads / 32) * kTile * 4;  // + per-warp sums
   const size_t sm_top = size_t(kTopMax) * 12 + (256 + 32 + 4) * 4;
   const size_t sm_assign = lloyd_assign_smem(rmax);
   const size_t sm_val = size_t(kHeadDim) * (2 * kTile + 2 * kRowBlk) * 4;

@@ -46,6 +46,34 @@ __device__ __forceinline__ void load_kt(float* Kt, const __nv_bfloat16* K, int64
   }
 }
 
+constexpr int kAsgRowBytes = kHeadDim * 2;  // one bf16 row of 128 dims
+
+// byte offset of 16-byte chunk `ch` of row `row` in a [rows][256 B] bf16 tile;
+// chunks XOR-swizzled by row so that ldmatrix reads of 8 rows are conflict free
+__device__ __forceinline__ uint32_t asg_swz(int row, int ch) {
+  return uint32_t(row) * kAsgRowBytes + uint32_t((ch ^ (row & 7)) << 4);
+}
+
+// 16-byte asynchronous copy global -> shared; src_bytes = 0 writes zeros
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+               "r"(src_bytes)
+               : "memory");
+}
+
+// Stage the bf16 keys of tokens tok0..tok0+127 as a swizzled [128][256 B]
+// tile (zeros past s); the copies complete at the caller's wait.
+__device__ __forceinline__ void stage_key_tile(uint32_t ks_s, const __nv_bfloat16* Ku, int64_t s,
+                                               int64_t tok0) {
+  for (int idx = threadIdx.x; idx < kTile * 16; idx += blockDim.x) {
+    const int row = idx >> 4, ch = idx & 15;
+    const bool in = tok0 + row < s;
+    cp_async16(ks_s + asg_swz(row, ch), Ku + (in ? (tok0 + row) * kHeadDim : 0) + 8 * ch,
+               in ? 16u : 0u);
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
 // Load 32 query rows (scaled) into Qt[k][row]; rows >= n_rows are zero.
 // row r of the block is global row rowbase + r, read from rowptr(r).
 template <typename RowPtr>
@@ -112,40 +140,111 @@ struct ObsArgs {
   float* A;                    // [UL, s] attention summed over fit rows, averaged over G
 };
 
+// Logits of fit rows against a 128-token tile on the tensor cores: a warp
+// takes 16 query rows at a time (rows 16 rb .. 16 rb + 15, A fragments straight
+// from global memory), the keys are the B operand from the swizzled tile.
+// Products of the bf16 rows and keys are exact, accumulated in fp32, then
+// scaled by log2(e)/sqrt(d) (the logits in log2 units).  The accumulator of
+// n-tile nt holds rows g (entries 0, 1) and g + 8 (entries 2, 3) at tokens
+// 8 nt + 2 t4 (+1), with g = lane / 4, t4 = lane % 4.
+__device__ __forceinline__ const uint32_t* obs_row(const ObsArgs& p, int ul, int row) {
+  const int g = row / p.n_fit, t = row % p.n_fit;
+  return reinterpret_cast<const uint32_t*>(p.Qobs +
+                                           ((int64_t(ul) * p.G + g) * p.n_obs + t) * kHeadDim);
+}
+
+__device__ __forceinline__ void obs_afrag(const ObsArgs& p, int ul, int rb, int lane,
+                                          uint32_t (&A)[8][4]) {
+  const int g = lane >> 2, t4 = lane & 3;
+  const int r0 = rb * 16 + g, r1 = r0 + 8;
+  const uint32_t* q0 = r0 < p.n_rows ? obs_row(p, ul, r0) : nullptr;
+  const uint32_t* q1 = r1 < p.n_rows ? obs_row(p, ul, r1) : nullptr;
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    A[ks][0] = q0 ? __ldg(q0 + 8 * ks + t4) : 0u;
+    A[ks][1] = q1 ? __ldg(q1 + 8 * ks + t4) : 0u;
+    A[ks][2] = q0 ? __ldg(q0 + 8 * ks + 4 + t4) : 0u;
+    A[ks][3] = q1 ? __ldg(q1 + 8 * ks + 4 + t4) : 0u;
+  }
+}
+
+// logits of the 16 rows against tokens 64 h .. 64 h + 63 of the tile
+__device__ __forceinline__ void obs_half_logits(uint32_t ks_s, int h, int lane,
+                                                const uint32_t (&A)[8][4], float (&S)[8][4]) {
+  const int mi = lane >> 3;
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt) S[nt][0] = S[nt][1] = S[nt][2] = S[nt][3] = 0.f;
+#pragma unroll
+  for (int np = 0; np < 4; ++np) {
+    const int trow = 64 * h + 16 * np + (mi >> 1) * 8 + (lane & 7);
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4(ks_s + asg_swz(trow, 2 * ks + (mi & 1)), b0, b1, b2, b3);
+      mma16816(S[2 * np], A[ks][0], A[ks][1], A[ks][2], A[ks][3], b0, b1);
+      mma16816(S[2 * np + 1], A[ks][0], A[ks][1], A[ks][2], A[ks][3], b2, b3);
+    }
+  }
+  const float scale = kLog2e * rsqrtf(float(kHeadDim));
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) S[nt][e] *= scale;
+}
+
 // Pass 1: per (row, tile) max and sum of 2^{a log2e} over the tile's tokens.
 __global__ void __launch_bounds__(kThreads, 2) k_obs_pass1(ObsArgs p) {
-  extern __shared__ __align__(16) float sm[];
-  float* Kt = sm;
-  float* Qt = sm + kHeadDim * kTile;
+  extern __shared__ __align__(128) uint8_t obs_raw[];
   const int tile = blockIdx.x, ul = blockIdx.y;
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
   const int64_t tok0 = int64_t(tile) * kTile;
-  load_kt(Kt, p.K + int64_t(ul) * p.s * kHeadDim, p.s, tok0);
-  const float scale = kLog2e * rsqrtf(float(kHeadDim));
-  for (int rb = 0; rb < p.n_rows; rb += kRowBlk) {
-    __syncthreads();
-    load_qt(Qt, min(kRowBlk, p.n_rows - rb), scale, [&](int r) {
-      const int row = rb + r, g = row / p.n_fit, t = row % p.n_fit;
-      return p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + t) * kHeadDim;
-    });
-    __syncthreads();
-    float S[4][4];
-    tile_logits(Qt, Kt, S);
+  const uint32_t ks_s = smem_u32(obs_raw);
+  stage_key_tile(ks_s, p.K + int64_t(ul) * p.s * kHeadDim, p.s, tok0);
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  __syncthreads();
+  for (int rb = w; rb * 16 < p.n_rows; rb += kThreads / 32) {
+    uint32_t A[8][4];
+    obs_afrag(p, ul, rb, lane, A);
+    float M[2] = {-INFINITY, -INFINITY}, Lsum[2] = {0.f, 0.f};    // rows g, g + 8
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int row = rb + 4 * w + i;
-      float mx = -INFINITY;
+    for (int h = 0; h < 2; ++h) {
+      float S[8][4];
+      obs_half_logits(ks_s, h, lane, A, S);
 #pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (tok0 + 4 * lane + j < p.s) mx = fmaxf(mx, S[i][j]);
-      mx = warp_max(mx);
-      float sum = 0.f;
+      for (int a = 0; a < 2; ++a) {
+        float mx = -INFINITY;
 #pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (tok0 + 4 * lane + j < p.s) sum += exp2f(S[i][j] - mx);
-      sum = warp_sum(sum);
-      if (lane == 0 && row < p.n_rows)
-        p.tile_stats[(int64_t(ul) * p.n_rows + row) * p.ntiles + tile] = make_float2(mx, sum);
+        for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+          for (int c = 0; c < 2; ++c)
+            if (tok0 + 64 * h + 8 * nt + 2 * t4 + c < p.s) mx = fmaxf(mx, S[nt][2 * a + c]);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+        float sum = 0.f;
+        if (mx != -INFINITY) {
+#pragma unroll
+          for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+            for (int c = 0; c < 2; ++c)
+              if (tok0 + 64 * h + 8 * nt + 2 * t4 + c < p.s) sum += exp2f(S[nt][2 * a + c] - mx);
+        }
+        sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+        sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+        if (mx != -INFINITY) {                    // fold the half into the row's (max, sum)
+          const float nm = fmaxf(M[a], mx);
+          Lsum[a] = Lsum[a] * exp2f(M[a] - nm) + sum * exp2f(mx - nm);
+          M[a] = nm;
+        }
+      }
+    }
+    if (t4 == 0) {
+#pragma unroll
+      for (int a = 0; a < 2; ++a) {
+        const int row = rb * 16 + g + 8 * a;
+        if (row < p.n_rows)
+          p.tile_stats[(int64_t(ul) * p.n_rows + row) * p.ntiles + tile] =
+              make_float2(M[a], Lsum[a]);
+      }
     }
   }
 }
@@ -158,43 +257,57 @@ __global__ void k_obs_rowstats(ObsArgs p, int UL) {
   float mx = -INFINITY;
   for (int k = 0; k < p.ntiles; ++k) mx = fmaxf(mx, t[k].x);
   float sum = 0.f;
-  for (int k = 0; k < p.ntiles; ++k) sum += t[k].y * exp2f(t[k].x - mx);
+  for (int k = 0; k < p.ntiles; ++k)
+    if (t[k].y > 0.f) sum += t[k].y * exp2f(t[k].x - mx);
   p.row_stats[i] = make_float2(mx, 1.0f / sum);
 }
 
 // Pass 2: A_p = (1/G) sum over fit rows of the softmax weight of token p.
 __global__ void __launch_bounds__(kThreads, 2) k_obs_pass2(ObsArgs p) {
-  extern __shared__ __align__(16) float sm[];
-  float* Kt = sm;
-  float* Qt = sm + kHeadDim * kTile;
-  float* red = Qt + kHeadDim * kRowBlk;        // [8 warps][128 tokens]
+  extern __shared__ __align__(128) uint8_t obs_raw[];
+  float* red = reinterpret_cast<float*>(obs_raw + kTile * kAsgRowBytes);   // [8 warps][128 tokens]
   const int tile = blockIdx.x, ul = blockIdx.y;
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t4 = lane & 3;
   const int64_t tok0 = int64_t(tile) * kTile;
-  load_kt(Kt, p.K + int64_t(ul) * p.s * kHeadDim, p.s, tok0);
-  const float scale = kLog2e * rsqrtf(float(kHeadDim));
-  float col[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int rb = 0; rb < p.n_rows; rb += kRowBlk) {
-    __syncthreads();
-    load_qt(Qt, min(kRowBlk, p.n_rows - rb), scale, [&](int r) {
-      const int row = rb + r, g = row / p.n_fit, t = row % p.n_fit;
-      return p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + t) * kHeadDim;
-    });
-    __syncthreads();
-    float S[4][4];
-    tile_logits(Qt, Kt, S);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int row = rb + 4 * w + i;
-      if (row >= p.n_rows) continue;
-      const float2 st = p.row_stats[int64_t(ul) * p.n_rows + row];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) col[j] += exp2f(S[i][j] - st.x) * st.y;
-    }
-  }
+  const uint32_t ks_s = smem_u32(obs_raw);
+  stage_key_tile(ks_s, p.K + int64_t(ul) * p.s * kHeadDim, p.s, tok0);
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
   __syncthreads();
+  for (int h = 0; h < 2; ++h) {                  // tokens 64 h .. 64 h + 63
+    float col[8][2];                             // this lane's column sums
 #pragma unroll
-  for (int j = 0; j < 4; ++j) red[w * kTile + 4 * lane + j] = col[j];
+    for (int nt = 0; nt < 8; ++nt) col[nt][0] = col[nt][1] = 0.f;
+    for (int rb = w; rb * 16 < p.n_rows; rb += kThreads / 32) {
+      uint32_t A[8][4];
+      obs_afrag(p, ul, rb, lane, A);
+      float2 st[2];
+#pragma unroll
+      for (int a = 0; a < 2; ++a) {
+        const int row = rb * 16 + g + 8 * a;
+        st[a] = row < p.n_rows ? p.row_stats[int64_t(ul) * p.n_rows + row] : make_float2(0.f, 0.f);
+      }
+      float S[8][4];
+      obs_half_logits(ks_s, h, lane, A, S);
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+        for (int c = 0; c < 2; ++c)
+#pragma unroll
+          for (int a = 0; a < 2; ++a)
+            if (st[a].y > 0.f) col[nt][c] += exp2f(S[nt][2 * a + c] - st[a].x) * st[a].y;
+    }
+    // sum over the eight row groups of the warp (the warps are summed below)
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        float v = col[nt][c];
+        v += __shfl_xor_sync(0xffffffffu, v, 4);
+        v += __shfl_xor_sync(0xffffffffu, v, 8);
+        v += __shfl_xor_sync(0xffffffffu, v, 16);
+        if (g == 0) red[w * kTile + 64 * h + 8 * nt + 2 * t4 + c] = v;
+      }
+  }
   __syncthreads();
   if (threadIdx.x < kTile) {
     float a = 0.f;
@@ -632,22 +745,8 @@ __device__ __forceinline__ void top3_insert(float& d0, int& j0, float& d1, int& 
 }
 
 constexpr int kAsgNB = 32;                  // centres per staged block (double-buffered)
-constexpr int kAsgRowBytes = kHeadDim * 2;  // one bf16 row (key or centre plane)
 constexpr int kAsgPlanes = 2;               // bf16 planes per centre
 constexpr int kAsgBufBytes = kAsgPlanes * kAsgNB * kAsgRowBytes;
-
-// byte offset of 16-byte chunk `ch` of row `row` in a [rows][256 B] bf16 tile;
-// chunks XOR-swizzled by row so that ldmatrix reads of 8 rows are conflict free
-__device__ __forceinline__ uint32_t asg_swz(int row, int ch) {
-  return uint32_t(row) * kAsgRowBytes + uint32_t((ch ^ (row & 7)) << 4);
-}
-
-// 16-byte asynchronous copy global -> shared; src_bytes = 0 writes zeros
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
-               "r"(src_bytes)
-               : "memory");
-}
 
 // Shared memory of k_lloyd_assign: the key tile, two blocks of centre planes
 // and the tile's histogram of `rmax` centres.
