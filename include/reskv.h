@@ -178,6 +178,18 @@ reskv_status reskv_build_cache(const reskv_config* cfg, const void* const* K_lay
 reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* Q, void* O,
                                void* stream);
 
+/*
+ * Alg. 2 for the contiguous layers layer0 .. layer0 + n_layers - 1 in one
+ * launch (reskv_decode_attn is this call with one layer or all layers): the
+ * layers a pipeline stage owns, or a group of layers whose queries and
+ * outputs a caller moves between host and device while the next group
+ * decodes.  Q device bf16 [n_layers, B, H_kv*G, d], O device fp32, same
+ * shape, 16-byte aligned.  RESKV_ERR_INVALID_ARG unless 0 <= layer0 and
+ * 1 <= n_layers <= L - layer0.
+ */
+reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int32_t n_layers,
+                                      const void* Q, void* O, void* stream);
+
 /* Release every device buffer of the handle (synchronises the device). NULL-safe. */
 void reskv_free(reskv_cache* c);
 

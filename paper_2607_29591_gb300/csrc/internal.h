@@ -136,6 +136,9 @@ struct reskv_cache {
     int cluster = 0;
     int warps_per_cta = 0;
   } cplan_layer, cplan_all;
+  // plans of calls over other layer counts (reskv_decode_attn_layers), by
+  // count; cluster = -1 until planned
+  mutable std::vector<ClusterPlan> cplan_range;
   // 2-D TMA maps of kslots / vslots: [U * budget rows, 128 dims], boxes of
   // 16 rows x 64 dims with the 128-byte swizzle
   CUtensorMap tmap_k;

@@ -433,13 +433,23 @@ reskv_status reskv_export_cache(const reskv_cache* c, reskv_host_cache* h, void*
 
 reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* Q, void* O,
                                void* stream) {
+  if (!c) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  if (layer < -1 || layer >= c->cfg.n_layers)
+    return fail(RESKV_ERR_INVALID_ARG, "layer must be -1 or in [0, n_layers)");
+  return layer < 0 ? reskv_decode_attn_layers(c, 0, c->cfg.n_layers, Q, O, stream)
+                   : reskv_decode_attn_layers(c, layer, 1, Q, O, stream);
+}
+
+reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int32_t n_layers,
+                                      const void* Q, void* O, void* stream) {
   if (!c || !Q || !O) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
   const reskv_config& cfg = c->cfg;
-  if (layer < -1 || layer >= cfg.n_layers)
-    return fail(RESKV_ERR_INVALID_ARG, "layer must be -1 or in [0, n_layers)");
+  if (layer0 < 0 || n_layers < 1 || int64_t(layer0) + n_layers > cfg.n_layers)
+    return fail(RESKV_ERR_INVALID_ARG, "need 0 <= layer0 and 1 <= n_layers <= L - layer0");
   if (!aligned16(Q) || !aligned16(O))
     return fail(RESKV_ERR_INVALID_ARG, "Q and O must be 16-byte aligned");
   const int64_t per_layer = int64_t(cfg.batch) * cfg.n_kv_heads;
+  const int32_t l_end = layer0 + n_layers;
   DecodeParams p{};
   p.kslots = c->kslots;
   p.vslots = c->vslots;
@@ -453,12 +463,11 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   p.partials = c->partials;
   p.tickets = c->tickets;
   p.status = c->status;
-  p.unit0 = layer < 0 ? 0 : int64_t(layer) * per_layer;
-  p.n_units = int32_t(layer < 0 ? c->n_units : per_layer);
+  p.unit0 = int64_t(layer0) * per_layer;
+  p.n_units = int32_t(int64_t(n_layers) * per_layer);
   p.stride = c->stride;
   int32_t app = 0;                     // most appended rows of a unit of the launch
-  for (int l = layer < 0 ? 0 : layer; l < (layer < 0 ? cfg.n_layers : layer + 1); ++l)
-    app = std::max(app, c->n_app_max[size_t(l)]);
+  for (int l = layer0; l < l_end; ++l) app = std::max(app, c->n_app_max[size_t(l)]);
   p.tail_unused = c->append_capacity - app;
   p.n_kv_heads = cfg.n_kv_heads;
   p.total_slots = c->h_offsets[size_t(p.unit0 + p.n_units)] - c->h_offsets[size_t(p.unit0)];
@@ -468,7 +477,19 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
   p.alpha = cfg.alpha;
   p.g_min = cfg.g_min;
   p.g_fixed = cfg.g_fixed;
-  const reskv_cache::ClusterPlan& cp = layer < 0 ? c->cplan_all : c->cplan_layer;
+  reskv_cache::ClusterPlan cp;
+  if (n_layers == 1) {
+    cp = c->cplan_layer;
+  } else if (n_layers == cfg.n_layers) {
+    cp = c->cplan_all;
+  } else {                             // other layer counts: planned on first use
+    if (c->cplan_range.empty()) c->cplan_range.assign(size_t(cfg.n_layers) + 1, {-1, 0});
+    if (c->cplan_range[size_t(n_layers)].cluster < 0) {
+      reskv_status st = plan_cluster(c, p.n_units, &c->cplan_range[size_t(n_layers)]);
+      if (st != RESKV_OK) return st;
+    }
+    cp = c->cplan_range[size_t(n_layers)];
+  }
   int kernel = cfg.decode_kernel;
   if (kernel == RESKV_DECODE_AUTO)
     kernel = (cp.cluster > 0 && cfg.decode_warps == 0) ? RESKV_DECODE_CLUSTER : RESKV_DECODE_MMA;

@@ -105,6 +105,8 @@ def load_library():
     lib.reskv_build_cache.restype = i32
     lib.reskv_decode_attn.argtypes = [vp, i32, vp, vp, vp]
     lib.reskv_decode_attn.restype = i32
+    lib.reskv_decode_attn_layers.argtypes = [vp, i32, i32, vp, vp, vp]
+    lib.reskv_decode_attn_layers.restype = i32
     lib.reskv_free.argtypes = [vp]
     lib.reskv_free.restype = None
     lib.reskv_last_error.argtypes = []
@@ -238,6 +240,20 @@ def reskv_decode_attn(cache: Cache, layer: int, Q, O, stream=None) -> None:
     _check(load_library().reskv_decode_attn(cache.handle, int(layer),
                                             _dptr(Q, "torch.bfloat16", "Q"),
                                             _dptr(O, "torch.float32", "O"), _stream(stream)))
+
+
+def reskv_decode_attn_layers(cache: Cache, layer0: int, n_layers: int, Q, O, stream=None) -> None:
+    """Alg. 2 for layers layer0 .. layer0 + n_layers - 1 in one launch: Q bf16
+    [n_layers, B, H_q, d], O fp32 likewise."""
+    c = cache.cfg
+    need = int(n_layers) * c.batch * c.n_kv_heads * c.group * c.head_dim
+    for name, t in (("Q", Q), ("O", O)):
+        if t.numel() != need:
+            raise ValueError(f"{name} holds {t.numel()} elements; this call needs {need}")
+    _check(load_library().reskv_decode_attn_layers(cache.handle, int(layer0), int(n_layers),
+                                                   _dptr(Q, "torch.bfloat16", "Q"),
+                                                   _dptr(O, "torch.float32", "O"),
+                                                   _stream(stream)))
 
 
 def reskv_append(cache: Cache, layer: int, K_new, V_new, stream=None) -> None:

@@ -179,6 +179,39 @@ def test_per_layer_calls_match_all_layer_call():
         assert rel < 1e-6
 
 
+def test_layer_range_calls_match_all_layer_call():
+    """reskv_decode_attn_layers over contiguous layer ranges (one launch each)
+    gives the all-layer call's outputs; ranges outside the cache are refused."""
+    L, Bt, H, G, b = 6, 3, 2, 4, 300
+    rng = np.random.default_rng(31)
+    splits = []
+    for _ in range(L * Bt * H):
+        n = int(rng.integers(1, b + 1))
+        m = int(rng.integers(1, n + 1))
+        splits.append((m, n - m))
+    w, lay = synthetic_layout(L, Bt, H, b, splits)
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len, budget=b)
+    h = R.reskv_import_cache(cfg, **lay)
+    Q = queries_for(w, L, Bt, H, G)
+    O_all = run_decode(h, Q).cpu().numpy()
+    for l0, n in ((0, 6), (0, 2), (1, 3), (5, 1), (2, 4), (3, 2)):
+        O = torch.full((n,) + tuple(Q.shape[1:]), float("nan"), dtype=torch.float32, device="cuda")
+        R.reskv_decode_attn_layers(h, l0, n, Q[l0:l0 + n].cuda().contiguous(), O)
+        torch.cuda.synchronize()
+        assert errors(O.cpu().numpy(), O_all[l0:l0 + n].astype(np.float64))[1] < 1e-6
+    Qd = Q[:2].cuda().contiguous()
+    Od = torch.empty(Qd.shape, dtype=torch.float32, device="cuda")
+    for l0, n in ((-1, 2), (5, 2)):
+        with pytest.raises(R.ReskvError) as e:
+            R.reskv_decode_attn_layers(h, l0, n, Qd, Od)
+        assert e.value.status == R.RESKV_ERR_INVALID_ARG
+    import ctypes
+    st = R.load_library().reskv_decode_attn_layers(h.handle, 0, 0, ctypes.c_void_p(Qd.data_ptr()),
+                                                   ctypes.c_void_p(Od.data_ptr()), None)
+    assert st == R.RESKV_ERR_INVALID_ARG
+    R.reskv_check_status(h)
+
+
 def test_determinism_and_split_invariance():
     L, Bt, H, G, b = 2, 3, 2, 4, 300
     w, lay = synthetic_layout(L, Bt, H, b, SPLITS)
