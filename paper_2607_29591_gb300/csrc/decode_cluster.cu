@@ -12,7 +12,7 @@
 // chunks with the tile step of mma_tile.cuh, and the partial results never
 // leave the chip:
 //
-//   1. every warp writes its record (per query head and branch: running max,
+//   1. every warp writes its record (per query head and branch: reference max,
 //      sum, numerator) into its own, drained, ring buffer;
 //   2. after a CTA barrier, the CTA's threads merge its warps' records in
 //      warp order and store the CTA record into rank 0's shared memory
@@ -94,12 +94,6 @@ __device__ __forceinline__ void st_cluster(uint32_t local, uint32_t rank, float4
                : "memory");
 }
 
-__device__ __forceinline__ void st_cluster(uint32_t local, uint32_t rank, float2 v) {
-  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(map_rank(local, rank)), "f"(v.x),
-               "f"(v.y)
-               : "memory");
-}
-
 // What one launch computes: the fused decode (o^ of Eq. reskv, the library's
 // path), or one branch of the paper-style comparison path (Sec. 6.1, App. B:
 // main-cache attention and residual branch as separate passes merged through
@@ -115,11 +109,9 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   extern __shared__ uint8_t smem_raw[];
   const int kW = blockDim.x >> 5;       // warps per CTA of this launch
   const int kSt = p.n_stages;           // ring stages per warp of this launch
-  const int kWarpBytes = warp_bytes(kSt);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = lane >> 2;              // query head (row of the mma tile)
+  const int g = lane >> 2;              // softmax column / accumulator row of this lane
   const int qp = lane & 3;              // position in the quad
-  const bool hv = h < G;
   const uint32_t cs = cluster_size(), rank = cluster_rank();
 
   // this cluster's unit, slots [ub, ub + stride).  Slot indices fit in 32
@@ -151,16 +143,16 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   const int wcb = cb + k0 * kCh;                           // first row of this warp's run
 
   // per-warp shared memory, 1024-byte aligned for the 128-byte swizzle
-  const uint32_t raw = smem_u32(smem_raw);
-  const uint32_t abase = (raw + 1023u) & ~1023u;
-  uint8_t* abase_ptr = smem_raw + (abase - raw);
-  const uint32_t base = abase + uint32_t(warp) * kWarpBytes;
-  uint8_t* base_ptr = abase_ptr + warp * kWarpBytes;
-  float* logc_s = reinterpret_cast<float*>(base_ptr + warp_logc_offset(kSt));   // [kSt][16]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + warp_bars_offset(kSt));
+  const WarpRing ring = warp_ring(smem_raw, kW, kSt, warp);
+  uint8_t* abase_ptr = ring.cta;
+  const uint32_t abase = smem_u32(abase_ptr);
+  const uint32_t base = ring.base;
+  uint8_t* base_ptr = ring.ptr;
+  float* logc_s = ring.logc;           // [kSt][16]
+  uint64_t* bars = ring.bars;
   // CTA records [cs][2][G][kRec] after the rings (read only in rank 0)
-  float* crec = reinterpret_cast<float*>(abase_ptr + kW * kWarpBytes);
-  const uint32_t crec_s = abase + uint32_t(kW * kWarpBytes);
+  float* crec = reinterpret_cast<float*>(abase_ptr + ring_smem_bytes(kW, kSt));
+  const uint32_t crec_s = abase + uint32_t(ring_smem_bytes(kW, kSt));
 
   cluster_arrive_relaxed();             // closed by cluster_wait() before step 2
   if (lane == 0) {
@@ -196,8 +188,8 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   // tokens, then rows appended at decode time); a residual pass has none
   const int m_lo = kMode == kResBranch ? 0 : ub, m_hi = kMode == kResBranch ? 0 : ue;
   const int r_lo = ub + nm, r_hi = ub + nm + nr;
-  uint32_t off_qk[4], off_pv[8];
-  tile_offsets(lane, off_qk, off_pv);
+  uint32_t off_k[4], off_pv[8];
+  tile_offsets(lane, off_k, off_pv);
   const float qscale = kLog2e * rsqrtf(float(kHeadDim));
   const int64_t orow0 = int64_t(ul / p.n_kv_heads) * p.n_kv_heads * G + (ul % p.n_kv_heads) * G;
   uint32_t qa[16];
@@ -206,7 +198,7 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   // only the cache (K, V, log-counts, n_main, n_res), which no kernel that
   // may run concurrently writes.
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  load_q_frag(p.Q, orow0 + h, hv, qp, qa);
+  load_q_frag<G>(p.Q, orow0, lane, qa);
 
   TileState S;
   S.reset();
@@ -220,8 +212,14 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
       break;
     }
     waited = k + 1;
-    tile_update<kMode != kMainBranch>(S, base + s * kStageBytes, logc_s + s * kCh, wcb + k * kCh,
-                                      m_lo, m_hi, r_lo, r_hi, qa, off_qk, off_pv, qscale, hv, qp);
+    const int t0 = wcb + k * kCh;
+    const uint32_t st = base + s * kStageBytes;
+    if (tile_pure_main(t0, m_lo, m_hi, r_lo, r_hi))
+      tile_update<G, true>(S, st, logc_s + s * kCh, t0, m_lo, m_hi, r_lo, r_hi, qa, off_k, off_pv,
+                           qscale, lane);
+    else
+      tile_update<G, false, kMode != kMainBranch>(S, st, logc_s + s * kCh, t0, m_lo, m_hi, r_lo,
+                                                  r_hi, qa, off_k, off_pv, qscale, lane);
     __syncwarp();
     if (k + kSt < nchunks) {
       if (lane == 0) {
@@ -240,25 +238,16 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
     mbar_wait_bounded(&bars[kk % kSt], uint32_t((kk / kSt) & 1));
   __syncwarp();
 
-  // 1. this warp's record, in the first bytes of its own ring
-  float lMt = S.lM + __shfl_xor_sync(0xffffffffu, S.lM, 1);
-  lMt += __shfl_xor_sync(0xffffffffu, lMt, 2);
-  float lRt = S.lR + __shfl_xor_sync(0xffffffffu, S.lR, 1);
-  lRt += __shfl_xor_sync(0xffffffffu, lRt, 2);
-  if (hv) {
-    float* rm = reinterpret_cast<float*>(base_ptr) + (0 * G + h) * kRec;
-    float* rr = reinterpret_cast<float*>(base_ptr) + (1 * G + h) * kRec;
-    if (qp == 0) {
-      rm[0] = S.mM;
-      rm[1] = lMt;
-      rr[0] = S.mR;
-      rr[1] = lRt;
-    }
+  // 1. this warp's record, in the first bytes of its own ring: per softmax
+  //    column g < 2G (branch g / G, head g % G) its reference max, sum,
+  //    largest logit and numerator
+  const RowStats rs = tile_row_stats(S, lane);
+  if (g < 2 * G) {
+    float* r = reinterpret_cast<float*>(base_ptr) + g * kRec;
+    if (qp == 0) *reinterpret_cast<float4*>(r) = make_float4(rs.m, rs.l, rs.mt, 0.f);
 #pragma unroll
-    for (int dt = 0; dt < 16; ++dt) {
-      *reinterpret_cast<float2*>(rm + 4 + dt * 8 + 2 * qp) = make_float2(S.O[dt][0], S.O[dt][1]);
-      *reinterpret_cast<float2*>(rr + 4 + dt * 8 + 2 * qp) = make_float2(S.O[dt][2], S.O[dt][3]);
-    }
+    for (int dt = 0; dt < 16; ++dt)
+      *reinterpret_cast<float2*>(r + 4 + dt * 8 + 2 * qp) = tile_row_value(S, dt);
   }
   __syncthreads();
   cluster_wait();                        // every CTA of the cluster is running
@@ -269,19 +258,22 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   //    rank 0's CTA records (distributed shared memory).
   for (int idx = threadIdx.x; idx < 2 * G * (kHeadDim / 4); idx += blockDim.x) {
     const int rec = idx / (kHeadDim / 4), d4 = 4 * (idx % (kHeadDim / 4));
-    float2 ml[kMmaMaxW];
+    float4 ml[kMmaMaxW];
     float4 ac[kMmaMaxW];
 #pragma unroll
     for (int w = 0; w < kMmaMaxW; ++w) {
       const int ws = w < kW ? w : 0;           // in-range address; weight masked below
-      const float* r = reinterpret_cast<const float*>(abase_ptr + ws * kWarpBytes) + rec * kRec;
-      ml[w] = *reinterpret_cast<const float2*>(r);
+      const float* r = reinterpret_cast<const float*>(abase_ptr + ws * kSt * kStageBytes) + rec * kRec;
+      ml[w] = *reinterpret_cast<const float4*>(r);
       ac[w] = *reinterpret_cast<const float4*>(r + 4 + d4);
     }
-    float mx = -INFINITY;
+    float mx = -INFINITY, mt = -INFINITY;
 #pragma unroll
     for (int w = 0; w < kMmaMaxW; ++w)
-      if (w < kW && ml[w].y > 0.f) mx = fmaxf(mx, ml[w].x);
+      if (w < kW && ml[w].y > 0.f) {
+        mx = fmaxf(mx, ml[w].x);
+        mt = fmaxf(mt, ml[w].z);
+      }
     float l = 0.f;
     float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
@@ -296,7 +288,7 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
       }
     const uint32_t dst = crec_s + uint32_t(rank * kCtaRecFloats + rec * kRec) * 4u;
     st_cluster(dst + uint32_t(4 + d4) * 4u, 0, a);
-    if (d4 == 0) st_cluster(dst, 0, make_float2(mx, l));
+    if (d4 == 0) st_cluster(dst, 0, make_float4(mx, l, mt, 0.f));
   }
   cluster_sync();
   if (rank != 0) return;                 // nobody reads this CTA's shared memory
@@ -304,7 +296,7 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   // 3. rank 0: merge the CS CTA records in rank order, gate, write o^
   for (int idx = threadIdx.x; idx < G * (kHeadDim / 4); idx += blockDim.x) {
     const int hh = idx / (kHeadDim / 4), d4 = 4 * (idx % (kHeadDim / 4));
-    float2 ml[2][kMaxCluster];
+    float4 ml[2][kMaxCluster];
     float4 ac[2][kMaxCluster];
 #pragma unroll
     for (int sg = 0; sg < 2; ++sg)
@@ -312,17 +304,20 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
       for (int c = 0; c < kMaxCluster; ++c) {
         const int cc = c < int(cs) ? c : 0;
         const float* r = crec + cc * kCtaRecFloats + (sg * G + hh) * kRec;
-        ml[sg][c] = *reinterpret_cast<const float2*>(r);
+        ml[sg][c] = *reinterpret_cast<const float4*>(r);
         ac[sg][c] = *reinterpret_cast<const float4*>(r + 4 + d4);
       }
-    float Ms[2], Ls[2];
+    float Ms[2], Ls[2], Mt[2];
     float4 As[2];
 #pragma unroll
     for (int sg = 0; sg < 2; ++sg) {
-      float mx = -INFINITY;
+      float mx = -INFINITY, mt = -INFINITY;
 #pragma unroll
       for (int c = 0; c < kMaxCluster; ++c)
-        if (c < int(cs) && ml[sg][c].y > 0.f) mx = fmaxf(mx, ml[sg][c].x);
+        if (c < int(cs) && ml[sg][c].y > 0.f) {
+          mx = fmaxf(mx, ml[sg][c].x);
+          mt = fmaxf(mt, ml[sg][c].z);
+        }
       float l = 0.f;
       float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
@@ -337,10 +332,12 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
         }
       Ms[sg] = mx;
       Ls[sg] = l;
+      Mt[sg] = mt;
       As[sg] = a;
     }
     if constexpr (kMode == kFused) {
-      const float2 w = branch_coefs(p.softmax_mode, gate_of(p, Ls[0]), Ms[0], Ls[0], Ms[1], Ls[1]);
+      const float2 w = branch_coefs(p.softmax_mode, gate_of(p, sum_rel_max(Ms[0], Ls[0], Mt[0])),
+                                    Ms[0], Ls[0], Ms[1], Ls[1]);
       *reinterpret_cast<float4*>(p.O + (orow0 + hh) * kHeadDim + d4) =
           make_float4(w.x * As[0].x + w.y * As[1].x, w.x * As[0].y + w.y * As[1].y,
                       w.x * As[0].z + w.y * As[1].z, w.x * As[0].w + w.y * As[1].w);
@@ -350,7 +347,11 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
       float* br = p.partials + (orow0 + hh) * kBrRec;
       *reinterpret_cast<float4*>(br + 4 + d4) =
           make_float4(As[sg].x * inv, As[sg].y * inv, As[sg].z * inv, As[sg].w * inv);
-      if (d4 == 0) *reinterpret_cast<float2*>(br) = make_float2(Ms[sg], Ls[sg]);
+      // (m, l) relative to the branch's largest logit, as the merge's gate takes it
+      if (d4 == 0)
+        *reinterpret_cast<float2*>(br) =
+            Ls[sg] > 0.f ? make_float2(Mt[sg], sum_rel_max(Ms[sg], Ls[sg], Mt[sg]))
+                         : make_float2(Ms[sg], Ls[sg]);
     }
   }
 }
@@ -507,12 +508,11 @@ size_t decode_lse_scratch_floats(int64_t n_units, int group) {
 
 // Ring depth for `warps_per_cta` warps next to `cluster` CTA records.
 int decode_cluster_stages(int warps_per_cta, int cluster) {
-  int st = ((kSmemLimit - 1024 - cluster * kCtaRecFloats * 4) / warps_per_cta - 1024) / kStageBytes;
-  return st > kMmaMaxSt ? kMmaMaxSt : st;
+  return ring_stages(warps_per_cta, cluster * kCtaRecFloats * 4);
 }
 
 int decode_cluster_smem_bytes(int warps_per_cta, int stages, int cluster) {
-  return warps_per_cta * warp_bytes(stages) + 1024 + cluster * kCtaRecFloats * 4;
+  return 1024 + ring_smem_bytes(warps_per_cta, stages) + cluster * kCtaRecFloats * 4;
 }
 
 }  // namespace reskv

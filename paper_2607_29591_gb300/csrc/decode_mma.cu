@@ -38,6 +38,7 @@ __device__ __forceinline__ int64_t warp_begin(int64_t w, int64_t T, int64_t W) {
 __device__ __forceinline__ int64_t warp_of(int64_t x, int64_t T, int64_t W) { return ((x + 1) * W - 1) / T; }
 
 // kRagged: units at p.offsets[u] (per-unit budgets); otherwise at u * stride.
+// Slot and unit indices fit in 32 bits (a cache holds fewer than 2^31 slots).
 template <int G, bool kRagged>
 __global__ void __launch_bounds__(kMaxW * 32, 1)
     reskv_decode_mma_kernel(const DecodeParams p, const __grid_constant__ CUtensorMap tmK,
@@ -45,60 +46,57 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   extern __shared__ uint8_t smem_raw[];
   const int kW = blockDim.x >> 5;       // warps per CTA of this launch
   const int kSt = p.n_stages;           // ring stages per warp of this launch
-  const int kWarpBytes = warp_bytes(kSt);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = lane >> 2;              // query head (row of the mma tile)
+  const int g = lane >> 2;              // softmax column / accumulator row of this lane
   const int qp = lane & 3;              // position in the quad
-  const bool hv = h < G;
-  const int64_t gw = int64_t(blockIdx.x) * kW + warp;
+  const int gw = int(blockIdx.x) * kW + warp;
   if (gw >= p.n_warps) return;
   const int64_t T = p.total_slots, W = p.n_warps;
-  const int64_t b = p.stride;
+  const int unit0 = int(p.unit0);
   // first slot of unit uu
-  auto ustart = [&](int64_t uu) -> int64_t {
+  auto ustart = [&](int uu) -> int {
     if constexpr (kRagged) return p.offsets[uu];
-    else return uu * b;
+    else return uu * p.stride;
   };
-  const int64_t gbase = ustart(p.unit0);
-  int64_t ga, ge;
+  const int gbase = ustart(unit0);
+  int ga, ge;
   if (p.units_per_warp > 0) {            // whole units [gw k, (gw + 1) k)
-    const int64_t k = p.units_per_warp;
-    const int64_t u_lo = gw * k, u_hi = u_lo + k < p.n_units ? u_lo + k : p.n_units;
+    const int k = p.units_per_warp;
+    const int u_lo = gw * k, u_hi = u_lo + k < p.n_units ? u_lo + k : p.n_units;
     if (u_lo >= u_hi) return;
-    ga = ustart(p.unit0 + u_lo);
-    ge = ustart(p.unit0 + u_hi);
+    ga = ustart(unit0 + u_lo);
+    ge = ustart(unit0 + u_hi);
   } else {                               // equal slot pieces
-    ga = gbase + warp_begin(gw, T, W);
-    ge = gbase + warp_begin(gw + 1, T, W);
+    ga = gbase + int(warp_begin(gw, T, W));
+    ge = gbase + int(warp_begin(gw + 1, T, W));
   }
   if (ga >= ge) return;
   // first unit with used slots in [ga, ge): the piece may start in the unused
   // tail slots of a unit (past its n_main + n_res + n_app used rows), which
   // this warp must skip
-  int64_t u;
+  int u;
   if constexpr (kRagged) {              // last unit starting at or before ga
-    int64_t lo = p.unit0, hi = p.unit0 + p.n_units;
+    int lo = unit0, hi = unit0 + p.n_units;
     while (hi - lo > 1) {
-      const int64_t mid = (lo + hi) >> 1;
+      const int mid = (lo + hi) >> 1;
       if (p.offsets[mid] <= ga) lo = mid;
       else hi = mid;
     }
     u = lo;
   } else {
-    u = ga / b;
+    u = ga / p.stride;
   }
   if (ustart(u) + p.n_main[u] + p.n_res[u] + (p.n_app ? p.n_app[u] : 0) <= ga) ++u;
   if (ustart(u) >= ge) return;
 
-  // per-warp shared memory, 1024-byte aligned for the 128-byte swizzle
-  const uint32_t raw = smem_u32(smem_raw);
-  const uint32_t base = ((raw + 1023u) & ~1023u) + uint32_t(warp) * kWarpBytes;
-  uint8_t* base_ptr = smem_raw + (base - raw);
-  float* logc_s = reinterpret_cast<float*>(base_ptr + warp_logc_offset(kSt));   // [kSt][16]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(base_ptr + warp_bars_offset(kSt));
+  // this warp's ring, log-count copies and mbarriers
+  const WarpRing ring = warp_ring(smem_raw, kW, kSt, warp);
+  const uint32_t base = ring.base;
+  float* logc_s = ring.logc;           // [kSt][16]
+  uint64_t* bars = ring.bars;
 
-  const int64_t cb = ga & ~int64_t(kCh - 1);              // first chunk, 16-slot aligned
-  const int64_t nchunks = (ge - cb + kCh - 1) / kCh;
+  const int cb = ga & ~(kCh - 1);                        // first chunk, 16-slot aligned
+  const int nchunks = (ge - cb + kCh - 1) / kCh;
 
   if (lane == 0) {
     for (int s = 0; s < kSt; ++s) mbar_init(&bars[s], 1);
@@ -106,9 +104,8 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   }
   __syncwarp();
 
-  auto issue = [&](int64_t k) {        // lane 0
-    const int s = int(k % kSt);
-    const int row = int(cb + k * kCh);
+  auto issue = [&](int k, int s) {     // lane 0: chunk k into stage s
+    const int row = cb + k * kCh;
     const uint32_t st = base + s * kStageBytes;
     mbar_arrive_expect_tx(&bars[s], kStageBytes + kCh * 4);
     tma_load_2d(st, &tmK, 0, row, &bars[s]);
@@ -118,25 +115,28 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     bulk_g2s(logc_s + s * kCh, p.logc + row, kCh * 4, &bars[s]);
   };
   if (lane == 0)
-    for (int64_t k = 0; k < nchunks && k < kSt; ++k) issue(k);
+    for (int k = 0; k < nchunks && k < kSt; ++k) issue(k, k);
   // Programmatic dependent launch: the next kernel on the stream may start
   // now and overlap its prologue and first cache copies with this kernel.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  uint32_t off_qk[4], off_pv[8];
-  tile_offsets(lane, off_qk, off_pv);
+  uint32_t off_k[4], off_pv[8];
+  tile_offsets(lane, off_k, off_pv);
 
   const float qscale = kLog2e * rsqrtf(float(kHeadDim));
   bool failed = false;
 
-  // unit cursor and its query fragments (the next unit's are loaded ahead)
+  // unit cursor: unit u from slot ub (the next unit from ub1), its main,
+  // residual and used rows, its query fragments; the next unit's are loaded
+  // ahead
   uint32_t qa[16], qn[16];
-  int32_t nm = 0, nr = 0, nt = 0, nm_n = 0, nr_n = 0, nt_n = 0;   // main, residual, used rows
-  auto load_q = [&](int64_t uu, uint32_t (&dst)[16], int32_t& m_out, int32_t& r_out,
-                    int32_t& t_out) {
-    const int64_t ul = uu - p.unit0;
-    const int64_t qrow = (ul / p.n_kv_heads) * int64_t(p.n_kv_heads) * G + (ul % p.n_kv_heads) * G + h;
-    load_q_frag(p.Q, qrow, hv, qp, dst);
+  int nm = 0, nr = 0, nt = 0, nm_n = 0, nr_n = 0, nt_n = 0;
+  auto qrow0_of = [&](int uu) -> int64_t {
+    const int ul = uu - unit0;
+    return int64_t(ul / p.n_kv_heads) * p.n_kv_heads * G + int64_t(ul % p.n_kv_heads) * G;
+  };
+  auto load_q = [&](int uu, uint32_t (&dst)[16], int& m_out, int& r_out, int& t_out) {
+    load_q_frag<G>(p.Q, qrow0_of(uu), lane, dst);
     m_out = p.n_main[uu];
     r_out = p.n_res[uu];
     t_out = m_out + r_out + (p.n_app ? p.n_app[uu] : 0);
@@ -145,51 +145,46 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   // on the stream has completed (before: the cache alone, which no kernel
   // that may run concurrently writes)
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  int ub = ustart(u), ub1 = ustart(u + 1);
   load_q(u, qa, nm, nr, nt);
-  if (ustart(u + 1) < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
+  if (ub1 < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
 
   TileState S;
   S.reset();
-  float(&O)[16][4] = S.O;
-  float &mM = S.mM, &lM = S.lM, &mR = S.mR, &lR = S.lR;
 
-  // Finish unit uu: write o^ (whole unit in this warp) or a partial record.
-  auto finish = [&](int64_t uu, int32_t ut) {
-    float lMt = lM + __shfl_xor_sync(0xffffffffu, lM, 1);
-    lMt += __shfl_xor_sync(0xffffffffu, lMt, 2);
-    float lRt = lR + __shfl_xor_sync(0xffffffffu, lR, 1);
-    lRt += __shfl_xor_sync(0xffffffffu, lRt, 2);
-    const int64_t ubase = ustart(uu), uend = ubase + ut;
-    const int64_t ul = uu - p.unit0;
-    const int64_t orow = (ul / p.n_kv_heads) * int64_t(p.n_kv_heads) * G + (ul % p.n_kv_heads) * G + h;
+  // Finish unit uu (first slot ubase, ut used rows): write o^ (whole unit in
+  // this warp) or a partial record; the last warp of a cut unit merges them.
+  auto finish = [&](int uu, int ubase, int ut) {
+    const RowStats rs = tile_row_stats(S, lane);
+    const int uend = ubase + ut;
+    const int64_t orow0 = qrow0_of(uu);
+    const int ul = uu - unit0;
+    float* op = p.O + (orow0 + (g < G ? g : 0)) * kHeadDim + 2 * qp;
     if (ga <= ubase && ge >= uend) {
-      if (hv) {
-        const float2 w = branch_coefs(p.softmax_mode, gate_of(p, lMt), mM, lMt, mR, lRt);
-        float* op = p.O + orow * kHeadDim + 2 * qp;
+      // the residual column of head g is column g + G, 4G lanes up
+      const float mR = __shfl_down_sync(0xffffffffu, rs.m, 4 * G);
+      const float lR = __shfl_down_sync(0xffffffffu, rs.l, 4 * G);
+      const float2 w = branch_coefs(p.softmax_mode, gate_of(p, sum_rel_max(rs.m, rs.l, rs.mt)),
+                                    rs.m, rs.l, mR, lR);
 #pragma unroll
-        for (int dt = 0; dt < 16; ++dt)
+      for (int dt = 0; dt < 16; ++dt) {
+        const float2 vm = tile_row_value(S, dt);
+        const float rx = __shfl_down_sync(0xffffffffu, vm.x, 4 * G);
+        const float ry = __shfl_down_sync(0xffffffffu, vm.y, 4 * G);
+        if (g < G)
           *reinterpret_cast<float2*>(op + dt * 8) =
-              make_float2(w.x * O[dt][0] + w.y * O[dt][2], w.x * O[dt][1] + w.y * O[dt][3]);
+              make_float2(w.x * vm.x + w.y * rx, w.x * vm.y + w.y * ry);
       }
       return;
     }
-    const int64_t flat0 = ubase - gbase;
-    const int64_t w0 = warp_of(flat0, T, W), w1 = warp_of(uend - 1 - gbase, T, W);
-    float* rec = p.partials + (ul + gw) * (2 * G * kRec);
-    if (hv) {
-      float* rm = rec + (0 * G + h) * kRec;
-      float* rr = rec + (1 * G + h) * kRec;
-      if (qp == 0) {
-        rm[0] = mM;
-        rm[1] = lMt;
-        rr[0] = mR;
-        rr[1] = lRt;
-      }
+    // record of column g (< 2G): reference max, sum, largest logit, numerator
+    const int64_t w0 = warp_of(ubase - gbase, T, W), w1 = warp_of(uend - 1 - gbase, T, W);
+    if (g < 2 * G) {
+      float* r = p.partials + (int64_t(ul) + gw) * (2 * G * kRec) + g * kRec;
+      if (qp == 0) *reinterpret_cast<float4*>(r) = make_float4(rs.m, rs.l, rs.mt, 0.f);
 #pragma unroll
-      for (int dt = 0; dt < 16; ++dt) {
-        *reinterpret_cast<float2*>(rm + 4 + dt * 8 + 2 * qp) = make_float2(O[dt][0], O[dt][1]);
-        *reinterpret_cast<float2*>(rr + 4 + dt * 8 + 2 * qp) = make_float2(O[dt][2], O[dt][3]);
-      }
+      for (int dt = 0; dt < 16; ++dt)
+        *reinterpret_cast<float2*>(r + 4 + dt * 8 + 2 * qp) = tile_row_value(S, dt);
     }
     __threadfence();
     __syncwarp();
@@ -198,83 +193,81 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     ticket = __shfl_sync(0xffffffffu, ticket, 0);
     if (ticket != int(w1 - w0)) return;
     __threadfence();
-    if (hv) {
-      // one pass over the records in warp order (online log-sum-exp merge)
-      float Ms[2] = {-INFINITY, -INFINITY}, Ls[2] = {0.f, 0.f};
-      float acc[2][32];
+    // one pass over the records in warp order (online log-sum-exp merge),
+    // column g per lane, then main and residual columns combined
+    float M = kMInit, L = 0.f, MT = -INFINITY;
+    float acc[32];
 #pragma unroll
-      for (int sg = 0; sg < 2; ++sg)
-#pragma unroll
-        for (int i = 0; i < 32; ++i) acc[sg][i] = 0.f;
+    for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+    if (g < 2 * G) {
       for (int64_t w = w0; w <= w1; ++w) {
-        const float* rr = p.partials + (ul + w) * (2 * G * kRec);
+        const float* r = p.partials + (int64_t(ul) + w) * (2 * G * kRec) + g * kRec;
+        const float4 hd = __ldcg(reinterpret_cast<const float4*>(r));
+        float2 v[16];
 #pragma unroll
-        for (int sg = 0; sg < 2; ++sg) {
-          const float* r = rr + (sg * G + h) * kRec;
-          const float rm = __ldcg(r), rl = __ldcg(r + 1);
-          float2 v[16];
+        for (int dt = 0; dt < 16; ++dt)
+          v[dt] = __ldcg(reinterpret_cast<const float2*>(r + 4 + dt * 8 + 2 * qp));
+        if (hd.y > 0.f) {
+          const float mx = fmaxf(M, hd.x);
+          const float sa = exp2f(M - mx), sb = exp2f(hd.x - mx);
+          L = L * sa + hd.y * sb;
 #pragma unroll
-          for (int dt = 0; dt < 16; ++dt)
-            v[dt] = __ldcg(reinterpret_cast<const float2*>(r + 4 + dt * 8 + 2 * qp));
-          if (rl > 0.f) {
-            const float mx = fmaxf(Ms[sg], rm);
-            const float sa = exp2f(Ms[sg] - mx), sb = exp2f(rm - mx);
-            Ls[sg] = Ls[sg] * sa + rl * sb;
-#pragma unroll
-            for (int dt = 0; dt < 16; ++dt) {
-              acc[sg][2 * dt] = acc[sg][2 * dt] * sa + v[dt].x * sb;
-              acc[sg][2 * dt + 1] = acc[sg][2 * dt + 1] * sa + v[dt].y * sb;
-            }
-            Ms[sg] = mx;
+          for (int dt = 0; dt < 16; ++dt) {
+            acc[2 * dt] = acc[2 * dt] * sa + v[dt].x * sb;
+            acc[2 * dt + 1] = acc[2 * dt + 1] * sa + v[dt].y * sb;
           }
+          M = mx;
+          MT = fmaxf(MT, hd.z);
         }
       }
-      const float2 w = branch_coefs(p.softmax_mode, gate_of(p, Ls[0]), Ms[0], Ls[0], Ms[1], Ls[1]);
-      float* op = p.O + orow * kHeadDim + 2 * qp;
+    }
+    const float mR = __shfl_down_sync(0xffffffffu, M, 4 * G);
+    const float lR = __shfl_down_sync(0xffffffffu, L, 4 * G);
+    const float2 w = branch_coefs(p.softmax_mode, gate_of(p, sum_rel_max(M, L, MT)), M, L, mR, lR);
 #pragma unroll
-      for (int dt = 0; dt < 16; ++dt)
+    for (int dt = 0; dt < 16; ++dt) {
+      const float rx = __shfl_down_sync(0xffffffffu, acc[2 * dt], 4 * G);
+      const float ry = __shfl_down_sync(0xffffffffu, acc[2 * dt + 1], 4 * G);
+      if (g < G)
         *reinterpret_cast<float2*>(op + dt * 8) =
-            make_float2(w.x * acc[0][2 * dt] + w.y * acc[1][2 * dt],
-                        w.x * acc[0][2 * dt + 1] + w.y * acc[1][2 * dt + 1]);
+            make_float2(w.x * acc[2 * dt] + w.y * rx, w.x * acc[2 * dt + 1] + w.y * ry);
     }
     __syncwarp();
     if (lane == 0) p.tickets[uu] = 0;
   };
 
   bool done = false;
-  int64_t issued = nchunks < kSt ? nchunks : kSt;     // chunks [0, issued) requested
-  int64_t waited = 0;                                 // chunks [0, waited) completed
-  for (int64_t k = 0; k < nchunks && !done; ++k) {
-    const int s = int(k % kSt);
-    if (!mbar_wait_bounded(&bars[s], uint32_t((k / kSt) & 1))) {
+  int issued = nchunks < kSt ? nchunks : kSt;         // chunks [0, issued) requested
+  int waited = 0;                                     // chunks [0, waited) completed
+  int s = 0;                                          // stage of chunk k
+  uint32_t phase = 0;                                 // parity of its current use
+  for (int k = 0; k < nchunks && !done; ++k) {
+    if (!mbar_wait_bounded(&bars[s], phase)) {
       failed = true;
       if (lane == 0) report_status(p.status, kStatusWaitTimeout);
       break;
     }
     waited = k + 1;
-    const int64_t t0 = cb + k * kCh;
+    const int t0 = cb + k * kCh;
     const uint32_t st = base + s * kStageBytes;
     const float* lc = logc_s + s * kCh;
     // every unit with rows in this tile
     while (true) {
-      const int64_t ubase = ustart(u);
-      const int64_t mlo = ubase > ga ? ubase : ga;
-      const int64_t mhi = (ubase + nt < ge) ? ubase + nt : ge;   // main + appended rows
-      const int64_t rlo = (ubase + nm > ga) ? ubase + nm : ga;
-      const int64_t rhi = (ubase + nm + nr < ge) ? ubase + nm + nr : ge;
-      const bool any = (mlo < mhi && mlo < t0 + kCh && mhi > t0) ||
-                       (rlo < rhi && rlo < t0 + kCh && rhi > t0);
-      if (any)
-        tile_update(S, st, lc, t0, mlo, mhi, rlo, rhi, qa, off_qk, off_pv,
-                    qscale, hv, qp);
+      const int mlo = ub > ga ? ub : ga;
+      const int mhi = ub + nt < ge ? ub + nt : ge;              // main + appended rows
+      const int rlo = ub + nm > ga ? ub + nm : ga;
+      const int rhi = ub + nm + nr < ge ? ub + nm + nr : ge;
+      if (tile_pure_main(t0, mlo, mhi, rlo, rhi))
+        tile_update<G, true>(S, st, lc, t0, mlo, mhi, rlo, rhi, qa, off_k, off_pv, qscale, lane);
+      else if ((mlo < mhi && mlo < t0 + kCh && mhi > t0) || (rlo < rhi && rlo < t0 + kCh && rhi > t0))
+        tile_update<G, false>(S, st, lc, t0, mlo, mhi, rlo, rhi, qa, off_k, off_pv, qscale, lane);
       // does unit u end inside this tile (or at the end of the piece)?
-      const int64_t uend = ubase + nt;
-      const int64_t stop = uend < ge ? uend : ge;
-      if (stop > t0 + kCh) break;                        // continues in the next tile
-      finish(u, nt);
+      if (mhi > t0 + kCh) break;                              // continues in the next tile
+      finish(u, ub, nt);
       S.reset();
       ++u;
-      if (ustart(u) >= ge) {
+      ub = ub1;
+      if (ub >= ge) {
         done = true;
         break;
       }
@@ -283,20 +276,25 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
       nm = nm_n;
       nr = nr_n;
       nt = nt_n;
-      if (ustart(u + 1) < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
+      ub1 = ustart(u + 1);
+      if (ub1 < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
     }
     if (done) break;
     __syncwarp();
     if (k + kSt < nchunks) {
       if (lane == 0) {
         fence_proxy_async_smem();
-        issue(k + kSt);
+        issue(k + kSt, s);
       }
       issued = k + kSt + 1;
     }
+    if (++s == kSt) {
+      s = 0;
+      phase ^= 1u;
+    }
   }
   // never leave with a copy in flight into this warp's ring (bounded waits)
-  for (int64_t kk = waited; kk < issued; ++kk)
+  for (int kk = waited; kk < issued; ++kk)
     mbar_wait_bounded(&bars[kk % kSt], uint32_t((kk / kSt) & 1));
   (void)failed;
 }
@@ -307,7 +305,7 @@ template <int G, bool kRagged>
 static cudaError_t launch_mma_g(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
                                 int n_ctas, int warps_per_cta, cudaStream_t stream) {
   static std::atomic<unsigned long long> configured{0};
-  const int smem = warps_per_cta * warp_bytes(p.n_stages) + 1024;
+  const int smem = 1024 + ring_smem_bytes(warps_per_cta, p.n_stages);
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
@@ -348,10 +346,7 @@ cudaError_t launch_decode_mma(const DecodeParams& p, const CUtensorMap& tk, cons
 }
 
 // Ring depth for `warps_per_cta` warps sharing one SM's shared memory.
-int decode_mma_stages(int warps_per_cta) {
-  int st = ((kSmemLimit - 1024) / warps_per_cta - 1024) / kStageBytes;
-  return st > kMaxSt ? kMaxSt : st;
-}
+int decode_mma_stages(int warps_per_cta) { return ring_stages(warps_per_cta, 0); }
 
 size_t decode_mma_partials_floats(int64_t n_units, int n_warps, int group) {
   return size_t(n_units + n_warps) * 2 * group * kRec;

@@ -5,18 +5,20 @@
 // unit).
 //
 // One tile step covers 16 consecutive slots staged in shared memory with
-// legacy tensor-core MMAs (mma.sync m16n8k16, bf16 in, fp32 accumulate):
+// legacy tensor-core MMAs (mma.sync m16n8k16, bf16 in, fp32 accumulate), in
+// transposed form:
 //
-//   logits  S[16 x 8 slots]  = Q[16 x 128] K^T        rows 0..G-1 = query heads
-//   output  O[16 x 8 dims]  += P[16 x 16 slots] V      rows 0..G-1: main-cache
-//                                                       weights, rows 8..8+G-1:
-//                                                       residual weights
+//   logits  S^T[16 slots x 8 columns] = K[16 x 128] Q^T      8 MMAs
+//   output  O[16 rows x 8 dims]      += P[16 x 16 slots] V   16 MMAs
 //
-// The mma tile has 16 rows for G <= 4 heads; the unused rows 8..15 carry the
-// residual branch, so the main and residual numerators (which the gate scales
-// differently) accumulate side by side in one fragment with no extra MMA.
-// P is split into bf16 hi + lo parts (two MMAs) so that the weights keep
-// ~16 significant bits; logits are exact bf16 products summed in fp32.
+// Column c of S^T is query head c for c < G (main branch) and head c - G for
+// G <= c < 2G (residual branch, whose logits add beta log c_j); columns from
+// 2G on are unused.  The logits of a column are its head's, masked to the
+// branch's slots, so one MMA gives both branches.  After the softmax the
+// weights are split into bf16 hi and lo parts (~16 significant bits together)
+// and moved into the A layout with movmatrix: rows 0..7 hold the hi part of
+// columns 0..7, rows 8..15 the lo part, so accumulator row g plus row g + 8 is
+// the numerator of column g.
 //
 // A stage holds the tile's K and V rows as four 2-D TMA boxes of 64 dims x 16
 // rows with the 128-byte swizzle (K dims 0..63 | K dims 64..127 | V lo | V hi),
@@ -38,15 +40,54 @@ constexpr int kMmaMaxSt = 12;              // ring stages per warp (at most)
 constexpr int kCh = kDecodeChunk;          // slots per stage (= one MMA tile)
 constexpr int kBox = kCh * 128;            // one 64-dim half of 16 rows, bytes
 constexpr int kStageBytes = 4 * kBox;      // K lo | K hi | V lo | V hi
-constexpr int kRec = kHeadDim + 4;         // partial record: m, l, pad, pad, acc[d]
+constexpr int kRec = kHeadDim + 4;         // partial record: m, l, mt, pad, acc[d]
 constexpr int kSmemLimit = 227 * 1024;     // dynamic shared memory per CTA
 
-// A warp's ring of `stages` stages plus its 16-slot log-count copies and
-// mbarriers; each warp's region starts 1024-byte aligned (128-byte swizzle).
-__host__ __device__ constexpr int warp_bytes(int stages) { return stages * kStageBytes + 1024; }
-__host__ __device__ constexpr int warp_logc_offset(int stages) { return stages * kStageBytes; }
-__host__ __device__ constexpr int warp_bars_offset(int stages) {
-  return stages * kStageBytes + kMmaMaxSt * kCh * 4;
+// A column's reference maximum before its first logit: finite, so that
+// exponents of masked (-inf) logits stay -inf and never become NaN.
+constexpr float kMInit = -1e30f;
+// A column's reference maximum is raised only when a logit exceeds it by more
+// than kLazy (log2 units): its weights stay below 2^kLazy and most tiles skip
+// the rescale of the accumulators.  Any reference gives the same softmax; the
+// column's largest logit is kept apart for the gate's p_max.
+constexpr float kLazy = 8.0f;
+
+// Shared memory of a CTA of `warps` warps with rings of `stages` stages: from
+// a 1024-byte aligned base (128-byte swizzle), the warps' rings one after the
+// other, then the 16 log-counts of every stage, then every stage's mbarrier
+// (rounded up to 16 bytes).  Keeping the small parts out of the rings lets a
+// CTA hold 28 stages in 227 KB.
+constexpr int kStageExtra = kCh * 4 + 8;
+__host__ __device__ constexpr int ring_smem_bytes(int warps, int stages) {
+  return (warps * stages * (kStageBytes + kStageExtra) + 15) & ~15;
+}
+// Ring depth that fits `warps` warps next to `extra` more bytes.
+__host__ __device__ constexpr int ring_stages(int warps, int extra) {
+  return (kSmemLimit - 1024 - 16 - extra) / (warps * (kStageBytes + kStageExtra)) < kMmaMaxSt
+             ? (kSmemLimit - 1024 - 16 - extra) / (warps * (kStageBytes + kStageExtra))
+             : kMmaMaxSt;
+}
+
+struct WarpRing {
+  uint8_t* cta;         // the CTA's aligned base (generic)
+  uint32_t base;        // shared address of this warp's first stage
+  uint8_t* ptr;         // the same, generic
+  float* logc;          // [stages][16]
+  uint64_t* bars;       // [stages]
+};
+
+__device__ __forceinline__ WarpRing warp_ring(uint8_t* smem_raw, int warps, int stages, int warp) {
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t abase = (raw + 1023u) & ~1023u;
+  uint8_t* a = smem_raw + (abase - raw);
+  const int nst = warps * stages;
+  WarpRing r;
+  r.cta = a;
+  r.base = abase + uint32_t(warp * stages * kStageBytes);
+  r.ptr = a + warp * stages * kStageBytes;
+  r.logc = reinterpret_cast<float*>(a + nst * kStageBytes) + warp * stages * kCh;
+  r.bars = reinterpret_cast<uint64_t*>(a + nst * (kStageBytes + kCh * 4)) + warp * stages;
+  return r;
 }
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
@@ -72,6 +113,14 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t&
                : "r"(addr));
 }
 
+// The transpose of an 8x8 b16 matrix held in the m8n8 fragment layout (lane
+// l: row l / 4, columns 2 (l % 4) and 2 (l % 4) + 1).
+__device__ __forceinline__ uint32_t movm_t(uint32_t a) {
+  uint32_t d;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+  return d;
+}
+
 // D += A * B, m16n8k16, bf16 inputs, fp32 accumulators
 __device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1, uint32_t a2,
                                          uint32_t a3, uint32_t b0, uint32_t b1) {
@@ -80,6 +129,13 @@ __device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1, uin
       "{%8, %9}, {%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// 2^x with the hardware approximation (ex2.approx.ftz, PTX ISA): 2^-inf = +0.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -97,15 +153,16 @@ __device__ __forceinline__ float gate_of(const DecodeParams& p, float lM) {
   return fmaxf(p.g_min, 1.0f / (1.0f + expf(-p.alpha * (p.tau - p_max))));
 }
 
-// ldmatrix row addresses of this lane (byte offsets inside a stage): for Q K^T
-// the four 32-dim groups of K rows, for P V the eight 16-dim groups of V rows
+// ldmatrix row addresses of this lane (byte offsets inside a stage): for
+// K Q^T the A fragments of slots 0..15 x dims 16j..16j+15 (j = 0..3; dims
+// 64..127 one box further), for P V the eight 16-dim groups of V rows
 // (transposed loads).
-__device__ __forceinline__ void tile_offsets(int lane, uint32_t (&off_qk)[4], uint32_t (&off_pv)[8]) {
+__device__ __forceinline__ void tile_offsets(int lane, uint32_t (&off_k)[4], uint32_t (&off_pv)[8]) {
   const int r8 = lane & 7, mi = lane >> 3;
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {                 // dims 32j..32j+31, matrix mi = 8-dim chunk
-    const int cg = 4 * j + mi, half = cg >> 3, cc = cg & 7;
-    off_qk[j] = half * kBox + r8 * 128 + ((cc ^ r8) << 4);
+  for (int j = 0; j < 4; ++j) {                 // matrix mi: slots 8 (mi & 1).., dims 16j + 8 (mi >> 1)..
+    const int cc = 2 * j + (mi >> 1);
+    off_k[j] = (mi & 1) * 1024 + r8 * 128 + ((cc ^ r8) << 4);
   }
 #pragma unroll
   for (int q = 0; q < 8; ++q) {                 // dims 16q..16q+15
@@ -114,11 +171,15 @@ __device__ __forceinline__ void tile_offsets(int lane, uint32_t (&off_qk)[4], ui
   }
 }
 
-// A operand of Q K^T for query row `qrow` of this lane's head: the words at
-// dims 16kk + 2qp (+1) and 16kk + 8 + 2qp (+1); zero for rows >= G.
-__device__ __forceinline__ void load_q_frag(const __nv_bfloat16* Q, int64_t qrow, bool hv, int qp,
+// B operand of K Q^T for column g = lane / 4 (query head g % G; zero from
+// column 2G on): the words at dims 16kk + 2qp (+1) and 16kk + 8 + 2qp (+1) of
+// Q row `qrow0 + (g % G)`.
+template <int G>
+__device__ __forceinline__ void load_q_frag(const __nv_bfloat16* Q, int64_t qrow0, int lane,
                                             uint32_t (&dst)[16]) {
-  const uint32_t* qw = reinterpret_cast<const uint32_t*>(Q + qrow * kHeadDim);
+  const int g = lane >> 2, qp = lane & 3;
+  const bool hv = g < 2 * G;
+  const uint32_t* qw = reinterpret_cast<const uint32_t*>(Q + (qrow0 + g % G) * kHeadDim);
 #pragma unroll
   for (int kk = 0; kk < 8; ++kk) {
     dst[2 * kk] = hv ? __ldg(qw + 8 * kk + qp) : 0u;
@@ -126,111 +187,161 @@ __device__ __forceinline__ void load_q_frag(const __nv_bfloat16* Q, int64_t qrow
   }
 }
 
-// Online-softmax state of one unit in the fragment layout of the m16n8
-// accumulator: O[dt][0..1] = main numerator of head h = lane/4 at dims
-// 8dt + 2qp (+1), O[dt][2..3] = residual numerator of the same head; the
-// running maxima are in log2 units and shared by the quad, the sums are this
-// lane's share (summed over the quad when the unit finishes).
+// Online-softmax state of one unit.  O[dt][0..1] = accumulator row g (hi
+// weights of column g) and O[dt][2..3] = row g + 8 (lo weights of the same
+// column) at dims 8dt + 2qp (+1).  The lane's softmax columns are 2qp and
+// 2qp + 1: m = their reference maxima (equal in the column's 8 lanes), l and
+// mt = this lane's share of their sums and largest logits (over slots g and
+// g + 8 of every tile), reduced when the unit finishes.  Logits in log2 units.
 struct TileState {
   float O[16][4];
-  float mM, lM, mR, lR;
+  float m[2], l[2], mt[2];
 
   __device__ __forceinline__ void reset() {
 #pragma unroll
     for (int dt = 0; dt < 16; ++dt) O[dt][0] = O[dt][1] = O[dt][2] = O[dt][3] = 0.f;
-    mM = mR = -INFINITY;
-    lM = lR = 0.f;
+    m[0] = m[1] = kMInit;
+    l[0] = l[1] = 0.f;
+    mt[0] = mt[1] = -INFINITY;
   }
 };
 
 // Fold the 16-slot tile staged at `st` (first global slot t0; residual
 // log-counts at lc[0..15]) into `S`.  Slots y in [rlo, rhi) are residual
-// entries (folded into the residual state when kResidual; a main-only pass
+// entries (folded into the residual columns when kResidual; a main-only pass
 // skips them), the other slots in [mlo, mhi) are exact main rows (selected
 // tokens and rows appended at decode time); every other row is masked.
-template <bool kResidual = true>
-__device__ __forceinline__ void tile_update(TileState& S, uint32_t st, const float* lc, int64_t t0,
-                                            int64_t mlo, int64_t mhi, int64_t rlo, int64_t rhi,
-                                            const uint32_t (&qa)[16], const uint32_t (&off_qk)[4],
-                                            const uint32_t (&off_pv)[8], float qscale, bool hv,
-                                            int qp) {
-  // ---- logits S = Q K^T for the 16 slots (two 8-slot n-tiles) ----
-  float S0[4] = {0.f, 0.f, 0.f, 0.f}, S1[4] = {0.f, 0.f, 0.f, 0.f};
-  float S0b[4] = {0.f, 0.f, 0.f, 0.f}, S1b[4] = {0.f, 0.f, 0.f, 0.f};
+// kPureMain: the caller has checked that all 16 slots are main rows (no
+// bounds are read).  Slot indices fit in 32 bits (a cache holds fewer than
+// 2^31 slots).
+template <int G, bool kPureMain, bool kResidual = true>
+__device__ __forceinline__ void tile_update(TileState& S, uint32_t st, const float* lc, int t0,
+                                            int mlo, int mhi, int rlo, int rhi,
+                                            const uint32_t (&qb)[16], const uint32_t (&off_k)[4],
+                                            const uint32_t (&off_pv)[8], float qscale, int lane) {
+  const int g = lane >> 2, qp = lane & 3;
+  // ---- logits S^T = K Q^T: four accumulator chains of two 16-dim steps ----
+  float Sc[4][4];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    uint32_t b0, b1, b2, b3, c0, c1, c2, c3;
-    ldsm_x4(st + off_qk[j], b0, b1, b2, b3);             // slots 0..7
-    ldsm_x4(st + off_qk[j] + 1024, c0, c1, c2, c3);      // slots 8..15
-    mma16816(S0, qa[4 * j], 0u, qa[4 * j + 1], 0u, b0, b1);
-    mma16816(S1, qa[4 * j], 0u, qa[4 * j + 1], 0u, c0, c1);
-    mma16816(S0b, qa[4 * j + 2], 0u, qa[4 * j + 3], 0u, b2, b3);
-    mma16816(S1b, qa[4 * j + 2], 0u, qa[4 * j + 3], 0u, c2, c3);
-  }
-  // this thread's slots: t0 + 8n + 2qp + i
-  float sM[4], sR[4];
-  const float sv[4] = {(S0[0] + S0b[0]) * qscale, (S0[1] + S0b[1]) * qscale,
-                       (S1[0] + S1b[0]) * qscale, (S1[1] + S1b[1]) * qscale};
+  for (int c = 0; c < 4; ++c) Sc[c][0] = Sc[c][1] = Sc[c][2] = Sc[c][3] = 0.f;
 #pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const int rowi = (e >> 1) * 8 + 2 * qp + (e & 1);
-    const int64_t y = t0 + rowi;
-    const bool in_r = y >= rlo && y < rhi;
-    const bool im = hv && y >= mlo && y < mhi && !in_r;
-    const bool ir = kResidual && hv && in_r;
-    sM[e] = im ? sv[e] : -INFINITY;
-    sR[e] = ir ? sv[e] + lc[rowi] * kLog2e : -INFINITY;   // + beta log c_j
+  for (int kk = 0; kk < 8; ++kk) {
+    uint32_t a0, a1, a2, a3;
+    ldsm_x4(st + off_k[kk & 3] + (kk >> 2) * kBox, a0, a1, a2, a3);
+    mma16816(Sc[kk & 3], a0, a1, a2, a3, qb[2 * kk], qb[2 * kk + 1]);
   }
-  float tM = fmaxf(fmaxf(sM[0], sM[1]), fmaxf(sM[2], sM[3]));
-  float tR = fmaxf(fmaxf(sR[0], sR[1]), fmaxf(sR[2], sR[3]));
-  tM = fmaxf(tM, __shfl_xor_sync(0xffffffffu, tM, 1));
-  tM = fmaxf(tM, __shfl_xor_sync(0xffffffffu, tM, 2));
-  tR = fmaxf(tR, __shfl_xor_sync(0xffffffffu, tR, 1));
-  tR = fmaxf(tR, __shfl_xor_sync(0xffffffffu, tR, 2));
-  if (tM > S.mM) {                                   // rescale the main rows
-    const float sc = exp2f(S.mM - tM);
-    S.lM *= sc;
+  float sv[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) sv[j] = ((Sc[0][j] + Sc[1][j]) + (Sc[2][j] + Sc[3][j])) * qscale;
+  // x[i][e]: slot g + 8i, column 2qp + e
+  float x[2][2] = {{sv[0], sv[1]}, {sv[2], sv[3]}};
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const int c = 2 * qp + e;
+    const bool cM = c < G, cR = kResidual && c >= G && c < 2 * G;
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      if constexpr (kPureMain) {
+        x[i][e] = cM ? x[i][e] : -INFINITY;
+      } else {
+        const int y = t0 + g + 8 * i;
+        const bool inR = y >= rlo && y < rhi;
+        const bool sM = y >= mlo && y < mhi && !inR;
+        x[i][e] = (cM && sM) ? x[i][e]
+                  : (cR && inR) ? x[i][e] + lc[g + 8 * i] * kLog2e   // + beta log c_j
+                                : -INFINITY;
+      }
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < 2; ++e) S.mt[e] = fmaxf(S.mt[e], fmaxf(x[0][e], x[1][e]));
+  // ---- raise the reference maxima when a logit passes them by more than kLazy ----
+  const bool up = fmaxf(x[0][0], x[1][0]) > S.m[0] + kLazy || fmaxf(x[0][1], x[1][1]) > S.m[1] + kLazy;
+  if (__any_sync(0xffffffffu, up)) {
+    float sc[2];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      float t = fmaxf(x[0][e], x[1][e]);
+      t = fmaxf(t, __shfl_xor_sync(0xffffffffu, t, 4));
+      t = fmaxf(t, __shfl_xor_sync(0xffffffffu, t, 8));
+      t = fmaxf(t, __shfl_xor_sync(0xffffffffu, t, 16));
+      const float mn = fmaxf(S.m[e], t);
+      sc[e] = exp2f(S.m[e] - mn);
+      S.l[e] *= sc[e];
+      S.m[e] = mn;
+    }
+    // accumulator rows g and g + 8 belong to column g, held by lane 4g + g/2
+    const float rs = __shfl_sync(0xffffffffu, (g & 1) ? sc[1] : sc[0], 4 * g + (g >> 1));
 #pragma unroll
     for (int dt = 0; dt < 16; ++dt) {
-      S.O[dt][0] *= sc;
-      S.O[dt][1] *= sc;
+      S.O[dt][0] *= rs;
+      S.O[dt][1] *= rs;
+      S.O[dt][2] *= rs;
+      S.O[dt][3] *= rs;
     }
-    S.mM = tM;
   }
-  if (tR > S.mR) {                                   // rescale the residual rows
-    const float sc = exp2f(S.mR - tR);
-    S.lR *= sc;
+  float pr[2][2];
 #pragma unroll
-    for (int dt = 0; dt < 16; ++dt) {
-      S.O[dt][2] *= sc;
-      S.O[dt][3] *= sc;
-    }
-    S.mR = tR;
-  }
-  float pM[4], pR[4];
+  for (int i = 0; i < 2; ++i)
 #pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    pM[e] = sM[e] > -INFINITY ? exp2f(sM[e] - S.mM) : 0.f;   // masked rows weigh 0
-    pR[e] = sR[e] > -INFINITY ? exp2f(sR[e] - S.mR) : 0.f;
-    S.lM += pM[e];
-    S.lR += pR[e];
-  }
-  // A = P (rows 0..7 main, rows 8..15 residual), hi + lo bf16 parts
-  const uint32_t h0 = pack_bf16(pM[0], pM[1]), h1 = pack_bf16(pR[0], pR[1]);
-  const uint32_t h2 = pack_bf16(pM[2], pM[3]), h3 = pack_bf16(pR[2], pR[3]);
-  const float2 f0 = unpack_bf16(h0), f1 = unpack_bf16(h1), f2 = unpack_bf16(h2), f3 = unpack_bf16(h3);
-  const uint32_t l0 = pack_bf16(pM[0] - f0.x, pM[1] - f0.y), l1 = pack_bf16(pR[0] - f1.x, pR[1] - f1.y);
-  const uint32_t l2 = pack_bf16(pM[2] - f2.x, pM[3] - f2.y), l3 = pack_bf16(pR[2] - f3.x, pR[3] - f3.y);
+    for (int e = 0; e < 2; ++e) pr[i][e] = ex2_approx(x[i][e] - S.m[e]);   // masked: 0
+  S.l[0] += pr[0][0] + pr[1][0];
+  S.l[1] += pr[0][1] + pr[1][1];
+  // P^T (slots x columns) as bf16 hi + lo parts, transposed into the A layout
+  const uint32_t ha = pack_bf16(pr[0][0], pr[0][1]), hb = pack_bf16(pr[1][0], pr[1][1]);
+  const float2 fa = unpack_bf16(ha), fb = unpack_bf16(hb);
+  const uint32_t la = pack_bf16(pr[0][0] - fa.x, pr[0][1] - fa.y);
+  const uint32_t lb = pack_bf16(pr[1][0] - fb.x, pr[1][1] - fb.y);
+  const uint32_t a0 = movm_t(ha), a1 = movm_t(la), a2 = movm_t(hb), a3 = movm_t(lb);
   // ---- O += P V ----
 #pragma unroll
   for (int q = 0; q < 8; ++q) {
     uint32_t v0, v1, v2, v3;
     ldsm_x4_t(st + off_pv[q], v0, v1, v2, v3);
-    mma16816(S.O[2 * q], h0, h1, h2, h3, v0, v1);
-    mma16816(S.O[2 * q + 1], h0, h1, h2, h3, v2, v3);
-    mma16816(S.O[2 * q], l0, l1, l2, l3, v0, v1);
-    mma16816(S.O[2 * q + 1], l0, l1, l2, l3, v2, v3);
+    mma16816(S.O[2 * q], a0, a1, a2, a3, v0, v1);
+    mma16816(S.O[2 * q + 1], a0, a1, a2, a3, v2, v3);
   }
+}
+
+// Whether the 16 slots from t0 are all main rows of the given bounds.
+__device__ __forceinline__ bool tile_pure_main(int t0, int mlo, int mhi, int rlo, int rhi) {
+  return t0 >= mlo && t0 + kCh <= mhi && (rhi <= t0 || rlo >= t0 + kCh || rlo >= rhi);
+}
+
+// Statistics of the softmax column g = lane / 4 (accumulator rows g, g + 8):
+// reference max m, sum l and largest logit mt over the unit's slots so far.
+// Every lane of the warp calls it.
+struct RowStats {
+  float m, l, mt;
+};
+
+__device__ __forceinline__ RowStats tile_row_stats(const TileState& S, int lane) {
+  float l0 = S.l[0], l1 = S.l[1], t0 = S.mt[0], t1 = S.mt[1];
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) {
+    l0 += __shfl_xor_sync(0xffffffffu, l0, o);
+    l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+    t0 = fmaxf(t0, __shfl_xor_sync(0xffffffffu, t0, o));
+    t1 = fmaxf(t1, __shfl_xor_sync(0xffffffffu, t1, o));
+  }
+  const int g = lane >> 2, src = 4 * g + (g >> 1);   // lane holding column g
+  const bool odd = g & 1;
+  RowStats r;
+  r.m = __shfl_sync(0xffffffffu, odd ? S.m[1] : S.m[0], src);
+  r.l = __shfl_sync(0xffffffffu, odd ? l1 : l0, src);
+  r.mt = __shfl_sync(0xffffffffu, odd ? t1 : t0, src);
+  return r;
+}
+
+// Numerator of column g at dims 8dt + 2qp (+1): hi row plus lo row.
+__device__ __forceinline__ float2 tile_row_value(const TileState& S, int dt) {
+  return make_float2(S.O[dt][0] + S.O[dt][2], S.O[dt][1] + S.O[dt][3]);
+}
+
+// The sum relative to the largest weight (what gate_of takes for the main
+// branch), from a (reference max, sum, largest logit) triple; 0 when empty.
+__device__ __forceinline__ float sum_rel_max(float m, float l, float mt) {
+  return l > 0.f ? l * exp2f(m - mt) : 0.f;
 }
 
 }  // namespace reskv

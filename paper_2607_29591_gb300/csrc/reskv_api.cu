@@ -157,6 +157,7 @@ struct MmaPlan {
   int64_t W = 1;
   int wpc = kDecodeWarpsPerCta;
   int32_t k = 0;
+  int stages = 0;                     // ring stages per warp
 };
 
 MmaPlan plan_mma(const reskv_cache* c, int64_t n_units, int64_t total_slots) {
@@ -186,6 +187,13 @@ MmaPlan plan_mma(const reskv_cache* c, int64_t n_units, int64_t total_slots) {
   }
   m.W = W;
   m.wpc = int(std::min<int64_t>(8, (W + c->num_sms - 1) / c->num_sms));
+  // Ring depth.  Whole-unit warps take the deepest ring that fits (a unit
+  // switch needs the next unit's copies ahead).  Warps on slot pieces keep
+  // about 16 stages per SM in all: on the 32-layer 32K cache 8 warps x 2
+  // stages stream 7 % faster than 8 x 3 (and 6 x 3 than 6 x 2); more copies
+  // in flight only lengthen the loaded latency.
+  m.stages = m.k > 0 ? decode_mma_stages(m.wpc)
+                     : std::min(decode_mma_stages(m.wpc), std::max(2, (16 + m.wpc / 2) / m.wpc));
   return m;
 }
 
@@ -525,6 +533,7 @@ reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int3
     W = mp.W;
     wpc = mp.wpc;
     p.units_per_warp = mp.k;
+    p.n_stages = mp.stages;
   } else {
     W = cfg.decode_warps > 0 ? cfg.decode_warps : p.total_slots / 32;
     if (W > p.total_slots) W = p.total_slots;
@@ -533,7 +542,7 @@ reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int3
   }
   if (W < 1) W = 1;
   p.n_warps = int32_t(W);
-  p.n_stages = mma ? decode_mma_stages(wpc) : 0;
+  if (!mma) p.n_stages = 0;
   cudaError_t err =
       mma ? launch_decode_mma(p, c->tmap_k, c->tmap_v, cfg.group, int((W + wpc - 1) / wpc), wpc,
                               static_cast<cudaStream_t>(stream))

@@ -30,6 +30,10 @@ def lib():
 
 
 KERNEL = {"id": R.RESKV_DECODE_MMA}
+# Launches that cut units differently agree to fp32 rounding, not bit for bit:
+# every warp's piece raises its softmax reference maxima on its own tiles, so
+# the weights are scaled (and split into bf16 hi + lo parts) differently.
+SPLIT_REL = 1e-5
 
 
 @pytest.fixture(autouse=True, params=[R.RESKV_DECODE_FMA, R.RESKV_DECODE_MMA, R.RESKV_DECODE_CLUSTER,
@@ -176,7 +180,7 @@ def test_per_layer_calls_match_all_layer_call():
     for l in range(L):
         O_l = run_decode(h, Q[l].contiguous(), layer=l).cpu().numpy()
         mx, rel = errors(O_l, O_all[l].astype(np.float64))
-        assert rel < 1e-6
+        assert rel < SPLIT_REL
 
 
 def test_layer_range_calls_match_all_layer_call():
@@ -198,7 +202,7 @@ def test_layer_range_calls_match_all_layer_call():
         O = torch.full((n,) + tuple(Q.shape[1:]), float("nan"), dtype=torch.float32, device="cuda")
         R.reskv_decode_attn_layers(h, l0, n, Q[l0:l0 + n].cuda().contiguous(), O)
         torch.cuda.synchronize()
-        assert errors(O.cpu().numpy(), O_all[l0:l0 + n].astype(np.float64))[1] < 1e-6
+        assert errors(O.cpu().numpy(), O_all[l0:l0 + n].astype(np.float64))[1] < SPLIT_REL
     Qd = Q[:2].cuda().contiguous()
     Od = torch.empty(Qd.shape, dtype=torch.float32, device="cuda")
     for l0, n in ((-1, 2), (5, 2)):
@@ -226,7 +230,7 @@ def test_determinism_and_split_invariance():
         assert torch.equal(o1, o2), "decode must be bitwise deterministic"
         outs.append(o1.cpu().numpy().astype(np.float64))
     for o in outs[1:]:
-        assert errors(o, outs[0])[1] < 1e-6
+        assert errors(o, outs[0])[1] < SPLIT_REL
 
 
 @pytest.mark.parametrize("G", [1, 2])
