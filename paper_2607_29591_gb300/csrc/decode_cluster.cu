@@ -213,13 +213,10 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
     }
     waited = k + 1;
     const int t0 = wcb + k * kCh;
-    const uint32_t st = base + s * kStageBytes;
-    if (tile_pure_main(t0, m_lo, m_hi, r_lo, r_hi))
-      tile_update<G, true>(S, st, logc_s + s * kCh, t0, m_lo, m_hi, r_lo, r_hi, qa, off_k, off_pv,
-                           qscale, lane);
-    else
-      tile_update<G, false, kMode != kMainBranch>(S, st, logc_s + s * kCh, t0, m_lo, m_hi, r_lo,
-                                                  r_hi, qa, off_k, off_pv, qscale, lane);
+    // the tile into registers, then its stage is refilled at once (the copy
+    // overlaps this tile's softmax and P V)
+    TileFrags F;
+    tile_load(base + s * kStageBytes, logc_s + s * kCh, off_k, off_pv, lane, F);
     __syncwarp();
     if (k + kSt < nchunks) {
       if (lane == 0) {
@@ -232,6 +229,11 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
       s = 0;
       phase ^= 1u;
     }
+    if (tile_pure_main(t0, m_lo, m_hi, r_lo, r_hi))
+      tile_update<G, true>(S, F, t0, m_lo, m_hi, r_lo, r_hi, qa, qscale, lane);
+    else
+      tile_update<G, false, kMode != kMainBranch>(S, F, t0, m_lo, m_hi, r_lo, r_hi, qa, qscale,
+                                                  lane);
   }
   // never reuse the ring while a copy is in flight into it (bounded waits)
   for (int kk = waited; kk < issued; ++kk)

@@ -32,10 +32,11 @@ namespace reskv {
 namespace {
 
 constexpr int kMaxW = kMmaMaxW;
-constexpr int kMaxSt = kMmaMaxSt;
 
-__device__ __forceinline__ int64_t warp_begin(int64_t w, int64_t T, int64_t W) { return (w * T) / W; }
-__device__ __forceinline__ int64_t warp_of(int64_t x, int64_t T, int64_t W) { return ((x + 1) * W - 1) / T; }
+// Warp w of W takes chunks [w N / W, (w + 1) N / W) of N; chunk c is in the
+// piece of warp ((c + 1) W - 1) / N.
+__device__ __forceinline__ int64_t piece_begin(int64_t w, int64_t N, int64_t W) { return (w * N) / W; }
+__device__ __forceinline__ int64_t piece_of(int64_t c, int64_t N, int64_t W) { return ((c + 1) * W - 1) / N; }
 
 // kRagged: units at p.offsets[u] (per-unit budgets); otherwise at u * stride.
 // Slot and unit indices fit in 32 bits (a cache holds fewer than 2^31 slots).
@@ -59,6 +60,11 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     else return uu * p.stride;
   };
   const int gbase = ustart(unit0);
+  // the launch's 16-slot chunks, aligned to global multiples of 16 like the
+  // copies: equal pieces of whole chunks, so that no chunk is read twice
+  const int base16 = gbase & ~(kCh - 1);
+  const int64_t NC = (int64_t(gbase) + T - base16 + kCh - 1) / kCh;
+  auto warp_of_slot = [&](int y) -> int64_t { return piece_of((y - base16) / kCh, NC, W); };
   int ga, ge;
   if (p.units_per_warp > 0) {            // whole units [gw k, (gw + 1) k)
     const int k = p.units_per_warp;
@@ -66,9 +72,10 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     if (u_lo >= u_hi) return;
     ga = ustart(unit0 + u_lo);
     ge = ustart(unit0 + u_hi);
-  } else {                               // equal slot pieces
-    ga = gbase + int(warp_begin(gw, T, W));
-    ge = gbase + int(warp_begin(gw + 1, T, W));
+  } else {                               // equal pieces of whole chunks
+    const int64_t end = int64_t(gbase) + T;
+    ga = int(max(int64_t(gbase), base16 + piece_begin(gw, NC, W) * kCh));
+    ge = int(min(end, base16 + piece_begin(gw + 1, NC, W) * kCh));
   }
   if (ga >= ge) return;
   // first unit with used slots in [ga, ge): the piece may start in the unused
@@ -178,7 +185,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
       return;
     }
     // record of column g (< 2G): reference max, sum, largest logit, numerator
-    const int64_t w0 = warp_of(ubase - gbase, T, W), w1 = warp_of(uend - 1 - gbase, T, W);
+    const int64_t w0 = warp_of_slot(ubase), w1 = warp_of_slot(uend - 1);
     if (g < 2 * G) {
       float* r = p.partials + (int64_t(ul) + gw) * (2 * G * kRec) + g * kRec;
       if (qp == 0) *reinterpret_cast<float4*>(r) = make_float4(rs.m, rs.l, rs.mt, 0.f);
@@ -249,8 +256,8 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     }
     waited = k + 1;
     const int t0 = cb + k * kCh;
-    const uint32_t st = base + s * kStageBytes;
-    const float* lc = logc_s + s * kCh;
+    TileFrags F;
+    tile_load(base + s * kStageBytes, logc_s + s * kCh, off_k, off_pv, lane, F);
     // every unit with rows in this tile
     while (true) {
       const int mlo = ub > ga ? ub : ga;
@@ -258,9 +265,9 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
       const int rlo = ub + nm > ga ? ub + nm : ga;
       const int rhi = ub + nm + nr < ge ? ub + nm + nr : ge;
       if (tile_pure_main(t0, mlo, mhi, rlo, rhi))
-        tile_update<G, true>(S, st, lc, t0, mlo, mhi, rlo, rhi, qa, off_k, off_pv, qscale, lane);
+        tile_update<G, true>(S, F, t0, mlo, mhi, rlo, rhi, qa, qscale, lane);
       else if ((mlo < mhi && mlo < t0 + kCh && mhi > t0) || (rlo < rhi && rlo < t0 + kCh && rhi > t0))
-        tile_update<G, false>(S, st, lc, t0, mlo, mhi, rlo, rhi, qa, off_k, off_pv, qscale, lane);
+        tile_update<G, false>(S, F, t0, mlo, mhi, rlo, rhi, qa, qscale, lane);
       // does unit u end inside this tile (or at the end of the piece)?
       if (mhi > t0 + kCh) break;                              // continues in the next tile
       finish(u, ub, nt);
@@ -280,6 +287,8 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
       if (ub1 < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
     }
     if (done) break;
+    // refill the stage once the tile is done (measured faster here than a
+    // refill right after the register loads, which the cluster kernel uses)
     __syncwarp();
     if (k + kSt < nchunks) {
       if (lane == 0) {

@@ -206,30 +206,48 @@ struct TileState {
   }
 };
 
-// Fold the 16-slot tile staged at `st` (first global slot t0; residual
-// log-counts at lc[0..15]) into `S`.  Slots y in [rlo, rhi) are residual
-// entries (folded into the residual columns when kResidual; a main-only pass
-// skips them), the other slots in [mlo, mhi) are exact main rows (selected
-// tokens and rows appended at decode time); every other row is masked.
-// kPureMain: the caller has checked that all 16 slots are main rows (no
-// bounds are read).  Slot indices fit in 32 bits (a cache holds fewer than
-// 2^31 slots).
+// A staged 16-slot tile in registers: the A fragments of K (slots x dims
+// 16kk..16kk+15) for K Q^T, the B fragments of V (slots x dims 16q..16q+15)
+// for P V, and the log-counts of slots g and g + 8.  Once a warp holds them
+// it may refill the stage: the copy into it overlaps the tile's softmax and
+// P V.
+struct TileFrags {
+  uint32_t k[8][4];
+  uint32_t v[8][4];
+  float lc[2];
+};
+
+__device__ __forceinline__ void tile_load(uint32_t st, const float* lc, const uint32_t (&off_k)[4],
+                                          const uint32_t (&off_pv)[8], int lane, TileFrags& F) {
+#pragma unroll
+  for (int kk = 0; kk < 8; ++kk)
+    ldsm_x4(st + off_k[kk & 3] + (kk >> 2) * kBox, F.k[kk][0], F.k[kk][1], F.k[kk][2], F.k[kk][3]);
+#pragma unroll
+  for (int q = 0; q < 8; ++q) ldsm_x4_t(st + off_pv[q], F.v[q][0], F.v[q][1], F.v[q][2], F.v[q][3]);
+  const int g = lane >> 2;
+  F.lc[0] = lc[g];
+  F.lc[1] = lc[g + 8];
+}
+
+// Fold a 16-slot tile (first global slot t0) into `S`.  Slots y in
+// [rlo, rhi) are residual entries (folded into the residual columns when
+// kResidual; a main-only pass skips them), the other slots in [mlo, mhi) are
+// exact main rows (selected tokens and rows appended at decode time); every
+// other row is masked.  kPureMain: the caller has checked that all 16 slots
+// are main rows (no bounds are read).  Slot indices fit in 32 bits (a cache
+// holds fewer than 2^31 slots).
 template <int G, bool kPureMain, bool kResidual = true>
-__device__ __forceinline__ void tile_update(TileState& S, uint32_t st, const float* lc, int t0,
-                                            int mlo, int mhi, int rlo, int rhi,
-                                            const uint32_t (&qb)[16], const uint32_t (&off_k)[4],
-                                            const uint32_t (&off_pv)[8], float qscale, int lane) {
+__device__ __forceinline__ void tile_update(TileState& S, const TileFrags& F, int t0, int mlo,
+                                            int mhi, int rlo, int rhi, const uint32_t (&qb)[16],
+                                            float qscale, int lane) {
   const int g = lane >> 2, qp = lane & 3;
   // ---- logits S^T = K Q^T: four accumulator chains of two 16-dim steps ----
   float Sc[4][4];
 #pragma unroll
   for (int c = 0; c < 4; ++c) Sc[c][0] = Sc[c][1] = Sc[c][2] = Sc[c][3] = 0.f;
 #pragma unroll
-  for (int kk = 0; kk < 8; ++kk) {
-    uint32_t a0, a1, a2, a3;
-    ldsm_x4(st + off_k[kk & 3] + (kk >> 2) * kBox, a0, a1, a2, a3);
-    mma16816(Sc[kk & 3], a0, a1, a2, a3, qb[2 * kk], qb[2 * kk + 1]);
-  }
+  for (int kk = 0; kk < 8; ++kk)
+    mma16816(Sc[kk & 3], F.k[kk][0], F.k[kk][1], F.k[kk][2], F.k[kk][3], qb[2 * kk], qb[2 * kk + 1]);
   float sv[4];
 #pragma unroll
   for (int j = 0; j < 4; ++j) sv[j] = ((Sc[0][j] + Sc[1][j]) + (Sc[2][j] + Sc[3][j])) * qscale;
@@ -248,7 +266,7 @@ __device__ __forceinline__ void tile_update(TileState& S, uint32_t st, const flo
         const bool inR = y >= rlo && y < rhi;
         const bool sM = y >= mlo && y < mhi && !inR;
         x[i][e] = (cM && sM) ? x[i][e]
-                  : (cR && inR) ? x[i][e] + lc[g + 8 * i] * kLog2e   // + beta log c_j
+                  : (cR && inR) ? x[i][e] + F.lc[i] * kLog2e   // + beta log c_j
                                 : -INFINITY;
       }
     }
@@ -296,10 +314,8 @@ __device__ __forceinline__ void tile_update(TileState& S, uint32_t st, const flo
   // ---- O += P V ----
 #pragma unroll
   for (int q = 0; q < 8; ++q) {
-    uint32_t v0, v1, v2, v3;
-    ldsm_x4_t(st + off_pv[q], v0, v1, v2, v3);
-    mma16816(S.O[2 * q], a0, a1, a2, a3, v0, v1);
-    mma16816(S.O[2 * q + 1], a0, a1, a2, a3, v2, v3);
+    mma16816(S.O[2 * q], a0, a1, a2, a3, F.v[q][0], F.v[q][1]);
+    mma16816(S.O[2 * q + 1], a0, a1, a2, a3, F.v[q][2], F.v[q][3]);
   }
 }
 

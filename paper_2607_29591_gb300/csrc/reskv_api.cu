@@ -160,21 +160,27 @@ struct MmaPlan {
   int stages = 0;                     // ring stages per warp
 };
 
+// At most 7 warps per SM: 7 x 2 ring stages streamed the 32-layer 32K cache
+// 1 % faster than 8 x 2 and 8 x 3.
+constexpr int kMmaWarpsPerCta = 7;
+
 MmaPlan plan_mma(const reskv_cache* c, int64_t n_units, int64_t total_slots) {
   MmaPlan m;
   int64_t W = 0;
-  int wpc = kDecodeWarpsPerCta;
+  int wpc = kMmaWarpsPerCta;
   if (c->cfg.decode_warps > 0) {
     W = c->cfg.decode_warps;
   } else if (n_units >= c->num_sms && n_units <= 4 * int64_t(c->num_sms) &&
              c->max_unit_slots <= 256 && !c->ragged) {
     W = n_units;                      // one warp per unit: no partial records at all
   } else {
-    wpc = int(std::min<int64_t>(8, std::max<int64_t>(1, total_slots / (int64_t(c->num_sms) * 200))));
+    wpc = int(std::min<int64_t>(kMmaWarpsPerCta,
+                                std::max<int64_t>(1, total_slots / (int64_t(c->num_sms) * 200))));
     W = int64_t(c->num_sms) * wpc;
     if (total_slots < W * 32) W = std::max<int64_t>(1, total_slots / 32);
   }
-  if (W > total_slots) W = total_slots;
+  // every warp needs a 16-slot chunk of its own (pieces are whole chunks)
+  if (W > total_slots / kDecodeChunk) W = total_slots / kDecodeChunk;
   if (W > c->max_warps) W = c->max_warps;
   if (W < 1) W = 1;
   // Short units (each at most an eighth of a warp's piece): every warp takes
@@ -187,13 +193,10 @@ MmaPlan plan_mma(const reskv_cache* c, int64_t n_units, int64_t total_slots) {
   }
   m.W = W;
   m.wpc = int(std::min<int64_t>(8, (W + c->num_sms - 1) / c->num_sms));
-  // Ring depth.  Whole-unit warps take the deepest ring that fits (a unit
-  // switch needs the next unit's copies ahead).  Warps on slot pieces keep
-  // about 16 stages per SM in all: on the 32-layer 32K cache 8 warps x 2
-  // stages stream 7 % faster than 8 x 3 (and 6 x 3 than 6 x 2); more copies
-  // in flight only lengthen the loaded latency.
-  m.stages = m.k > 0 ? decode_mma_stages(m.wpc)
-                     : std::min(decode_mma_stages(m.wpc), std::max(2, (16 + m.wpc / 2) / m.wpc));
+  // Ring depth: about 16 stages per SM in all.  On the 32-layer 32K cache
+  // 8 warps x 2 stages stream faster than 8 x 3 (and 6 x 3 than 6 x 2):
+  // more copies in flight only lengthen the loaded latency.
+  m.stages = std::min(decode_mma_stages(m.wpc), std::max(2, (16 + m.wpc / 2) / m.wpc));
   return m;
 }
 
