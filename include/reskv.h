@@ -190,6 +190,25 @@ reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* 
 reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int32_t n_layers,
                                       const void* Q, void* O, void* stream);
 
+/*
+ * Alg. 2 for all layers with the queries and outputs in host memory.
+ *
+ *   Q_host : host bf16 [L, B, H_kv*G, d]
+ *   O_host : host fp32, same shape; must not overlap Q_host
+ *
+ * With page-locked buffers the device can address (cudaHostAlloc,
+ * cudaMallocHost, cudaHostRegister with mapping), the one decode launch reads
+ * Q from and writes O to host memory itself, so the transfers overlap the
+ * streaming of the cache.  Pageable buffers are staged: a copy in, the
+ * decode, a copy out on `stream` (the first such call allocates the handle's
+ * staging buffers, device Q and O of all layers, kept until reskv_free).
+ * Asynchronous on `stream`: O_host holds the result once the stream has
+ * passed the call (cudaStreamSynchronize).  Results equal reskv_decode_attn's
+ * bit for bit.
+ */
+reskv_status reskv_decode_attn_host(const reskv_cache* c, const void* Q_host, void* O_host,
+                                    void* stream);
+
 /* Release every device buffer of the handle (synchronises the device). NULL-safe. */
 void reskv_free(reskv_cache* c);
 

@@ -139,6 +139,13 @@ struct reskv_cache {
   // plans of calls over other layer counts (reskv_decode_attn_layers), by
   // count; cluster = -1 until planned
   mutable std::vector<ClusterPlan> cplan_range;
+  // reskv_decode_attn_host with pageable buffers: device staging of Q and O
+  // for all layers (made by the first such call)
+  struct HostIo {
+    void* q = nullptr;
+    void* o = nullptr;
+  };
+  mutable HostIo hio;
   // 2-D TMA maps of kslots / vslots: [U * budget rows, 128 dims], boxes of
   // 16 rows x 64 dims with the 128-byte swizzle
   CUtensorMap tmap_k;

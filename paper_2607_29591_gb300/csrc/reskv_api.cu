@@ -139,6 +139,8 @@ void free_handle(reskv_cache* c) {
   cudaFree(c->dbg_scores);
   cudaFree(c->dbg_ranked);
   cudaFree(c->dbg_losses);
+  cudaFree(c->hio.q);
+  cudaFree(c->hio.o);
   delete c;
 }
 
@@ -576,6 +578,63 @@ reskv_status reskv_append(reskv_cache* c, int32_t layer, const void* K_new, cons
                                   static_cast<cudaStream_t>(stream));
   if (err != cudaSuccess) return cuda_fail(err, "append launch");
   for (int l = l0; l < l1; ++l) ++c->n_app_max[size_t(l)];
+  return RESKV_OK;
+}
+
+// The device address of host memory the current device can access (page-locked
+// and mapped, as cudaHostAlloc / cudaMallocHost / cudaHostRegister give under
+// unified addressing), or NULL.
+static void* device_view(const void* host) {
+  cudaPointerAttributes a{};
+  if (cudaPointerGetAttributes(&a, host) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
+}
+
+reskv_status reskv_decode_attn_host(const reskv_cache* c, const void* Q_host, void* O_host,
+                                    void* stream) {
+  if (!c || !Q_host || !O_host) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  const reskv_config& cfg = c->cfg;
+  const int L = cfg.n_layers;
+  const size_t rows = size_t(cfg.batch) * cfg.n_kv_heads * cfg.group;   // query rows per layer
+  const size_t q_bytes = L * rows * kHeadDim * 2, o_bytes = L * rows * kHeadDim * 4;
+  {
+    const uint8_t* qa = static_cast<const uint8_t*>(Q_host);
+    const uint8_t* oa = static_cast<const uint8_t*>(O_host);
+    if (oa < qa + q_bytes && qa < oa + o_bytes)
+      return fail(RESKV_ERR_INVALID_ARG, "O_host overlaps Q_host");
+  }
+  // Page-locked buffers: the decode kernel reads Q from and writes O to host
+  // memory itself (over the host link), so the transfers overlap the
+  // streaming of the cache and no copy sits before or after the launch.
+  void* qv = device_view(Q_host);
+  void* ov = device_view(O_host);
+  if (qv && ov) return reskv_decode_attn_layers(c, 0, L, qv, ov, stream);
+  // Otherwise stage through device buffers owned by the handle.
+  reskv_cache::HostIo& io = c->hio;
+  if (!io.q) {
+    void* q = nullptr;
+    void* o = nullptr;
+    cudaError_t err = cudaMalloc(&q, q_bytes);
+    if (err == cudaSuccess) err = cudaMalloc(&o, o_bytes);
+    if (err != cudaSuccess) {
+      cudaGetLastError();
+      cudaFree(q);
+      return err == cudaErrorMemoryAllocation ? fail(RESKV_ERR_OOM, "staging buffers")
+                                              : cuda_fail(err, "staging buffers");
+    }
+    io.o = o;
+    io.q = q;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t err = cudaMemcpyAsync(io.q, Q_host, q_bytes, cudaMemcpyHostToDevice, s);
+  if (err != cudaSuccess) return cuda_fail(err, "copying Q in");
+  const reskv_status st = reskv_decode_attn_layers(c, 0, L, io.q, io.o, s);
+  if (st != RESKV_OK) return st;
+  err = cudaMemcpyAsync(O_host, io.o, o_bytes, cudaMemcpyDeviceToHost, s);
+  if (err != cudaSuccess) return cuda_fail(err, "copying O out");
   return RESKV_OK;
 }
 

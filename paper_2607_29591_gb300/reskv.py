@@ -107,6 +107,8 @@ def load_library():
     lib.reskv_decode_attn.restype = i32
     lib.reskv_decode_attn_layers.argtypes = [vp, i32, i32, vp, vp, vp]
     lib.reskv_decode_attn_layers.restype = i32
+    lib.reskv_decode_attn_host.argtypes = [vp, vp, vp, vp]
+    lib.reskv_decode_attn_host.restype = i32
     lib.reskv_free.argtypes = [vp]
     lib.reskv_free.restype = None
     lib.reskv_last_error.argtypes = []
@@ -254,6 +256,32 @@ def reskv_decode_attn_layers(cache: Cache, layer0: int, n_layers: int, Q, O, str
                                                    _dptr(Q, "torch.bfloat16", "Q"),
                                                    _dptr(O, "torch.float32", "O"),
                                                    _stream(stream)))
+
+
+def _hptr(t, dtype_name: str, what: str):
+    """Host pointer of a contiguous CPU tensor of the expected dtype."""
+    if t.is_cuda:
+        raise ValueError(f"{what} must be a host (CPU) tensor")
+    if str(t.dtype) != dtype_name:
+        raise ValueError(f"{what} must be {dtype_name}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{what} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def reskv_decode_attn_host(cache: Cache, Q_host, O_host, stream=None) -> None:
+    """Alg. 2 for every layer with host buffers (pinned for overlap): Q_host
+    bf16 [L, B, H_q, d], O_host fp32 likewise.  Asynchronous: O_host is
+    complete once the stream has passed the call."""
+    c = cache.cfg
+    need = c.n_layers * c.batch * c.n_kv_heads * c.group * c.head_dim
+    for name, t in (("Q_host", Q_host), ("O_host", O_host)):
+        if t.numel() != need:
+            raise ValueError(f"{name} holds {t.numel()} elements; this call needs {need}")
+    _check(load_library().reskv_decode_attn_host(cache.handle,
+                                                 _hptr(Q_host, "torch.bfloat16", "Q_host"),
+                                                 _hptr(O_host, "torch.float32", "O_host"),
+                                                 _stream(stream)))
 
 
 def reskv_append(cache: Cache, layer: int, K_new, V_new, stream=None) -> None:

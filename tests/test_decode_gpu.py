@@ -216,6 +216,45 @@ def test_layer_range_calls_match_all_layer_call():
     R.reskv_check_status(h)
 
 
+def test_host_buffer_call_matches_device_call():
+    """reskv_decode_attn_host gives the device call's outputs bit for bit and
+    matches the oracle, with page-locked buffers (the kernel reads Q and
+    writes O in host memory) and with pageable ones (staged; repeated calls
+    reuse the staging); overlapping host buffers are refused."""
+    L, Bt, H, G, b = 5, 3, 2, 4, 300          # odd layer count: uneven groups
+    rng = np.random.default_rng(37)
+    splits = []
+    for _ in range(L * Bt * H):
+        n = int(rng.integers(1, b + 1))
+        m = int(rng.integers(1, n + 1))
+        splits.append((m, n - m))
+    w, lay = synthetic_layout(L, Bt, H, b, splits)
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len, budget=b)
+    h = R.reskv_import_cache(cfg, **lay)
+    for step in (0, 1):
+        Q = queries_for(w, L, Bt, H, G, step=step)
+        O_dev = run_decode(h, Q).cpu().numpy().astype(np.float64)
+        ref = oracle_decode_all(lay, Q, cfg)
+        for pinned in (True, False):
+            Qh = Q.contiguous()
+            Oh = torch.full(Q.shape, float("nan"), dtype=torch.float32)
+            if pinned:
+                Qh, Oh = Qh.pin_memory(), Oh.pin_memory()
+            R.reskv_decode_attn_host(h, Qh, Oh)
+            torch.cuda.synchronize()
+            O = Oh.numpy().astype(np.float64)
+            assert not np.isnan(O).any()
+            assert np.array_equal(O, O_dev), f"pinned {pinned}: differs from the device call"
+            assert_output_parity(O, ref, f"host call, step {step}, pinned {pinned}")
+    buf = torch.zeros(Q.numel() * 3, dtype=torch.bfloat16)
+    Qv = buf[:Q.numel()]
+    Ov = buf.view(torch.float32)[Q.numel() // 4:Q.numel() // 4 + Q.numel()]
+    with pytest.raises(R.ReskvError) as e:
+        R.reskv_decode_attn_host(h, Qv, Ov)
+    assert e.value.status == R.RESKV_ERR_INVALID_ARG
+    R.reskv_check_status(h)
+
+
 def test_determinism_and_split_invariance():
     L, Bt, H, G, b = 2, 3, 2, 4, 300
     w, lay = synthetic_layout(L, Bt, H, b, SPLITS)
