@@ -133,28 +133,66 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   const float qscale = kLog2e * rsqrtf(float(kHeadDim));
   bool failed = false;
 
+  // this warp's staging of query rows (two buffers) and output rows
+  uint8_t* io = ring.cta + ring_smem_bytes(kW, kSt) + warp * kIoBytes;
+  const uint32_t io_s = smem_u32(io);
+  float* obuf = reinterpret_cast<float*>(io + 2 * 4 * kQRowBytes);
+
   // unit cursor: unit u from slot ub (the next unit from ub1), its main,
-  // residual and used rows, its query fragments; the next unit's are loaded
-  // ahead
-  uint32_t qa[16], qn[16];
+  // residual and used rows, its query fragments; the next unit's query rows
+  // and counts are requested ahead
+  uint32_t qa[16];
   int nm = 0, nr = 0, nt = 0, nm_n = 0, nr_n = 0, nt_n = 0;
   auto qrow0_of = [&](int uu) -> int64_t {
     const int ul = uu - unit0;
     return int64_t(ul / p.n_kv_heads) * p.n_kv_heads * G + int64_t(ul % p.n_kv_heads) * G;
   };
-  auto load_q = [&](int uu, uint32_t (&dst)[16], int& m_out, int& r_out, int& t_out) {
-    load_q_frag<G>(p.Q, qrow0_of(uu), lane, dst);
+  auto load_q = [&](int uu, int b, int& m_out, int& r_out, int& t_out) {
+    const __nv_bfloat16* src = p.Q + qrow0_of(uu) * kHeadDim;
+    for (int i = lane; i < G * 16; i += 32)    // G rows of sixteen 16-byte pieces
+      cp_async16(io_s + b * 4 * kQRowBytes + (i >> 4) * kQRowBytes + (i & 15) * 16,
+                 src + (i >> 4) * kHeadDim + (i & 15) * 8);
+    asm volatile("cp.async.commit_group;" ::: "memory");
     m_out = p.n_main[uu];
     r_out = p.n_res[uu];
     t_out = m_out + r_out + (p.n_app ? p.n_app[uu] : 0);
+  };
+  // B operand of K Q^T for column g (query head g % G; zero from 2G on),
+  // once buffer b holds the unit's rows
+  auto q_frags = [&](int b) {
+    const uint32_t* w = reinterpret_cast<const uint32_t*>(io + b * 4 * kQRowBytes + (g % G) * kQRowBytes);
+    const bool hv = g < 2 * G;
+#pragma unroll
+    for (int kk = 0; kk < 8; ++kk) {
+      qa[2 * kk] = hv ? w[8 * kk + qp] : 0u;
+      qa[2 * kk + 1] = hv ? w[8 * kk + 4 + qp] : 0u;
+    }
+  };
+  // the G output rows staged in obuf to O, whole rows per store
+  auto write_out = [&](int64_t orow0) {
+    __syncwarp();
+    for (int i = lane; i < G * 32; i += 32) {
+      const int r = i >> 5, c = i & 31;
+      *reinterpret_cast<float4*>(p.O + (orow0 + r) * kHeadDim + 4 * c) =
+          *reinterpret_cast<const float4*>(obuf + r * kORowFloats + 4 * c);
+    }
+    __syncwarp();
   };
   // Q, O, the partial records and the tickets only after the previous kernel
   // on the stream has completed (before: the cache alone, which no kernel
   // that may run concurrently writes)
   asm volatile("griddepcontrol.wait;" ::: "memory");
   int ub = ustart(u), ub1 = ustart(u + 1);
-  load_q(u, qa, nm, nr, nt);
-  if (ub1 < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
+  int qb = 0;                                       // query buffer of unit u
+  load_q(u, 0, nm, nr, nt);
+  if (ub1 < ge) {
+    load_q(u + 1, 1, nm_n, nr_n, nt_n);
+    asm volatile("cp.async.wait_group 1;" ::: "memory");   // unit u's rows
+  } else {
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+  }
+  __syncwarp();
+  q_frags(0);
 
   TileState S;
   S.reset();
@@ -166,7 +204,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     const int uend = ubase + ut;
     const int64_t orow0 = qrow0_of(uu);
     const int ul = uu - unit0;
-    float* op = p.O + (orow0 + (g < G ? g : 0)) * kHeadDim + 2 * qp;
+    float* ob = obuf + (g < G ? g : 0) * kORowFloats + 2 * qp;
     if (ga <= ubase && ge >= uend) {
       // the residual column of head g is column g + G, 4G lanes up
       const float mR = __shfl_down_sync(0xffffffffu, rs.m, 4 * G);
@@ -179,9 +217,10 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
         const float rx = __shfl_down_sync(0xffffffffu, vm.x, 4 * G);
         const float ry = __shfl_down_sync(0xffffffffu, vm.y, 4 * G);
         if (g < G)
-          *reinterpret_cast<float2*>(op + dt * 8) =
+          *reinterpret_cast<float2*>(ob + dt * 8) =
               make_float2(w.x * vm.x + w.y * rx, w.x * vm.y + w.y * ry);
       }
+      write_out(orow0);
       return;
     }
     // record of column g (< 2G): reference max, sum, largest logit, numerator
@@ -236,10 +275,10 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
       const float rx = __shfl_down_sync(0xffffffffu, acc[2 * dt], 4 * G);
       const float ry = __shfl_down_sync(0xffffffffu, acc[2 * dt + 1], 4 * G);
       if (g < G)
-        *reinterpret_cast<float2*>(op + dt * 8) =
+        *reinterpret_cast<float2*>(ob + dt * 8) =
             make_float2(w.x * acc[2 * dt] + w.y * rx, w.x * acc[2 * dt + 1] + w.y * ry);
     }
-    __syncwarp();
+    write_out(orow0);
     if (lane == 0) p.tickets[uu] = 0;
   };
 
@@ -278,13 +317,15 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
         done = true;
         break;
       }
-#pragma unroll
-      for (int i = 0; i < 16; ++i) qa[i] = qn[i];
+      qb ^= 1;
+      asm volatile("cp.async.wait_group 0;" ::: "memory");   // unit u's rows
+      __syncwarp();
+      q_frags(qb);
       nm = nm_n;
       nr = nr_n;
       nt = nt_n;
       ub1 = ustart(u + 1);
-      if (ub1 < ge) load_q(u + 1, qn, nm_n, nr_n, nt_n);
+      if (ub1 < ge) load_q(u + 1, qb ^ 1, nm_n, nr_n, nt_n);
     }
     if (done) break;
     // refill the stage once the tile is done (measured faster here than a
@@ -314,7 +355,7 @@ template <int G, bool kRagged>
 static cudaError_t launch_mma_g(const DecodeParams& p, const CUtensorMap& tk, const CUtensorMap& tv,
                                 int n_ctas, int warps_per_cta, cudaStream_t stream) {
   static std::atomic<unsigned long long> configured{0};
-  const int smem = 1024 + ring_smem_bytes(warps_per_cta, p.n_stages);
+  const int smem = 1024 + ring_smem_bytes(warps_per_cta, p.n_stages) + warps_per_cta * kIoBytes;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
@@ -355,7 +396,7 @@ cudaError_t launch_decode_mma(const DecodeParams& p, const CUtensorMap& tk, cons
 }
 
 // Ring depth for `warps_per_cta` warps sharing one SM's shared memory.
-int decode_mma_stages(int warps_per_cta) { return ring_stages(warps_per_cta, 0); }
+int decode_mma_stages(int warps_per_cta) { return ring_stages(warps_per_cta, warps_per_cta * kIoBytes); }
 
 size_t decode_mma_partials_floats(int64_t n_units, int n_warps, int group) {
   return size_t(n_units + n_warps) * 2 * group * kRec;

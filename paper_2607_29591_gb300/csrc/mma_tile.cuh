@@ -187,6 +187,20 @@ __device__ __forceinline__ void load_q_frag(const __nv_bfloat16* Q, int64_t qrow
   }
 }
 
+// Per-warp staging of a unit's query rows and output rows (stream-K kernel):
+// the G query rows arrive by 16-byte cp.async copies into one of two buffers
+// (the current unit and the next), the G output rows leave as whole 512-byte
+// rows.  Rows are padded so that the fragment reads and the output writes hit
+// distinct banks.  Whole-row transfers matter most when Q and O sit in host
+// memory and cross the host link.
+constexpr int kQRowBytes = kHeadDim * 2 + 16;                        // 272
+constexpr int kORowFloats = kHeadDim + 8;                            // 136
+constexpr int kIoBytes = 2 * 4 * kQRowBytes + 4 * kORowFloats * 4;   // G <= 4
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
 // Online-softmax state of one unit.  O[dt][0..1] = accumulator row g (hi
 // weights of column g) and O[dt][2..3] = row g + 8 (lo weights of the same
 // column) at dims 8dt + 2qp (+1).  The lane's softmax columns are 2qp and
