@@ -182,15 +182,16 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   // on the stream has completed (before: the cache alone, which no kernel
   // that may run concurrently writes)
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  // The next unit's rows are requested once the current unit has at most
+  // kQAheadSlots rows left in the piece, not at once: when Q sits in host
+  // memory, every warp asking for two units' rows at the start queues the
+  // whole of Q on the host link before the first tile.
+  constexpr int kQAheadSlots = 64;
   int ub = ustart(u), ub1 = ustart(u + 1);
   int qb = 0;                                       // query buffer of unit u
+  bool next_asked = false;                          // unit u + 1's rows requested
   load_q(u, 0, nm, nr, nt);
-  if (ub1 < ge) {
-    load_q(u + 1, 1, nm_n, nr_n, nt_n);
-    asm volatile("cp.async.wait_group 1;" ::: "memory");   // unit u's rows
-  } else {
-    asm volatile("cp.async.wait_group 0;" ::: "memory");
-  }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
   __syncwarp();
   q_frags(0);
 
@@ -317,6 +318,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
         done = true;
         break;
       }
+      if (!next_asked) load_q(u, qb ^ 1, nm_n, nr_n, nt_n);   // a short unit
       qb ^= 1;
       asm volatile("cp.async.wait_group 0;" ::: "memory");   // unit u's rows
       __syncwarp();
@@ -325,7 +327,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
       nr = nr_n;
       nt = nt_n;
       ub1 = ustart(u + 1);
-      if (ub1 < ge) load_q(u + 1, qb ^ 1, nm_n, nr_n, nt_n);
+      next_asked = false;
     }
     if (done) break;
     // refill the stage once the tile is done (measured faster here than a
@@ -341,6 +343,11 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     if (++s == kSt) {
       s = 0;
       phase ^= 1u;
+    }
+    if (!next_asked && ub1 < ge && min(ub + nt, ge) - (t0 + kCh) <= kQAheadSlots) {
+      __syncwarp();
+      load_q(u + 1, qb ^ 1, nm_n, nr_n, nt_n);
+      next_asked = true;
     }
   }
   // never leave with a copy in flight into this warp's ring (bounded waits)
