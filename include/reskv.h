@@ -359,7 +359,7 @@ reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_d
  * exits.  A call whose scratch would exceed it fails with
  * RESKV_ERR_UNSUPPORTED before launching anything; decode fewer units per call
  * (one layer at a time) in that case.  Roughly, a call needs
- * (n_units + 8 * SMs) * 2 * group * 520 bytes plus 4 bytes per unit.
+ * (n_units + 8 * SMs) * 2 * group * 528 bytes plus 4 bytes per unit.
  *
  * The first call on a device looks up the array's device address
  * (cudaGetSymbolAddress, with that device current); make that first call
@@ -374,7 +374,12 @@ reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_d
  *                    1 <= n_main[u] and n_main[u] + n_res[u] <= budget
  *   Q              : device bf16 [n_units / n_kv_heads, n_kv_heads*group, 128]
  *   O              : device fp32, same shape as Q
- * Runs the CUDA-core decode kernel, which reads only inside these arrays.
+ * When budget is a multiple of 16, logc is 16-byte aligned and the cache holds
+ * fewer than 2^31 slots, the call runs the tensor-core kernel of
+ * reskv_decode_attn (its 16-slot copies then stay inside these arrays; the
+ * copy descriptors are encoded on the host per call, which allocates
+ * nothing); otherwise the CUDA-core kernel, which reads slot by slot.  Either
+ * reads only inside these arrays.
  */
 typedef struct reskv_device_cache {
   const void* kslots;

@@ -100,20 +100,38 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
   if (err != cudaSuccess) return fail(RESKV_ERR_CUDA, cudaGetErrorString(err));
   if (dev < 0 || dev >= kMaxDevices) return fail(RESKV_ERR_UNSUPPORTED, "device ordinal >= 64");
 
-  // the same split as reskv_decode_attn chooses automatically
-  const int64_t total = c->n_units * int64_t(c->budget);
+  reskv_status st = RESKV_OK;
   void* scratch = nullptr;
   int num_sms = 0;
-  reskv_status st = setup_device(dev, &scratch, &num_sms);
+  st = setup_device(dev, &scratch, &num_sms);
   if (st != RESKV_OK) return st;
-  int64_t W = total / 32;
-  if (W > int64_t(num_sms) * kDecodeWarpsPerCta) W = int64_t(num_sms) * kDecodeWarpsPerCta;
-  if (W < 1) W = 1;
+  const int64_t total = c->n_units * int64_t(c->budget);
+  // The tensor-core stream-K kernel of reskv_decode_attn when its 16-slot
+  // copies stay inside the caller's arrays (budget a multiple of 16, so the
+  // cache ends on a chunk boundary; log-counts 16-byte aligned for their
+  // bulk copies) and slot indices fit in 32 bits; else the CUDA-core kernel,
+  // which reads slot by slot.
+  const bool mma = c->budget % kDecodeChunk == 0 && aligned16(c->logc) && total + 16 < (int64_t(1) << 31);
+  CUtensorMap tk, tv;
+  MmaPlan mp;
+  int64_t W = 0;
+  if (mma) {
+    if (!encode_rows(&tk, c->kslots, uint64_t(total)) || !encode_rows(&tv, c->vslots, uint64_t(total)))
+      return fail(RESKV_ERR_CUDA, "cuTensorMapEncodeTiled refused the cache arrays");
+    mp = plan_mma_shape(num_sms, int64_t(num_sms) * kDecodeWarpsPerCta, 0, c->budget, false,
+                        c->n_units, total);
+    W = mp.W;
+  } else {
+    W = total / 32;
+    if (W > int64_t(num_sms) * kDecodeWarpsPerCta) W = int64_t(num_sms) * kDecodeWarpsPerCta;
+    if (W < 1) W = 1;
+  }
 
   // scratch layout: [tickets: n_units int32][status word][partial records]
   const size_t ticket_bytes = align256(size_t(c->n_units) * 4);
   const size_t status_bytes = 256;
-  const size_t part_bytes = decode_partials_floats(c->n_units, int(W), c->group) * 4;
+  const size_t part_bytes = (mma ? decode_mma_partials_floats(c->n_units, int(W), c->group)
+                                 : decode_partials_floats(c->n_units, int(W), c->group)) * 4;
   const size_t need = ticket_bytes + status_bytes + part_bytes;
   if (need > kNoAllocScratchBytes)
     return fail(RESKV_ERR_UNSUPPORTED,
@@ -153,8 +171,13 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
   p.alpha = c->alpha;
   p.g_min = c->g_min;
   p.g_fixed = c->g_fixed;
-  const int n_ctas = int((W + kDecodeWarpsPerCta - 1) / kDecodeWarpsPerCta);
-  err = launch_decode(p, c->group, n_ctas, s);
+  if (mma) {
+    p.units_per_warp = mp.k;
+    p.n_stages = mp.stages;
+    err = launch_decode_mma(p, tk, tv, c->group, int((W + mp.wpc - 1) / mp.wpc), mp.wpc, s);
+  } else {
+    err = launch_decode(p, c->group, int((W + kDecodeWarpsPerCta - 1) / kDecodeWarpsPerCta), s);
+  }
   if (err != cudaSuccess) return fail(RESKV_ERR_CUDA, std::string("decode launch: ") +
                                                           cudaGetErrorString(err));
   return RESKV_OK;

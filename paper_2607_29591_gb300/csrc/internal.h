@@ -91,6 +91,22 @@ constexpr int kLogcPad = 16;
 
 void set_error(const std::string& msg);
 
+// Split plan of the tensor-core stream-K kernel for a launch of `n_units`
+// units holding `total_slots` slots (largest unit `max_unit_slots`): W warps,
+// wpc per CTA, k > 0 when every warp takes k whole units instead of an equal
+// piece of chunks, and the ring stages per warp.  user_warps > 0 fixes W.
+struct MmaPlan {
+  int64_t W = 1;
+  int wpc = kDecodeWarpsPerCta;
+  int32_t k = 0;
+  int stages = 0;
+};
+MmaPlan plan_mma_shape(int num_sms, int64_t max_warps, int32_t user_warps, int64_t max_unit_slots,
+                       bool ragged, int64_t n_units, int64_t total_slots);
+// TMA map of [rows, 128] bf16 rows: boxes of 16 rows x 64 dims, 128-byte
+// swizzle (base 16-byte aligned).  False if the driver refuses it.
+bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows);
+
 }  // namespace reskv
 
 struct reskv_cache;

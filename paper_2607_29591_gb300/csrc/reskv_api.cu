@@ -109,18 +109,6 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-// [rows, 128] bf16 row-major -> TMA map with boxes of 16 rows x 64 dims, 128B swizzle
-bool encode_rows(CUtensorMap* map, void* base, uint64_t rows) {
-  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
-  if (!enc) return false;
-  const cuuint64_t dims[2] = {cuuint64_t(kHeadDim), cuuint64_t(rows)};
-  const cuuint64_t strides[1] = {cuuint64_t(kSlotRowBytes)};
-  const cuuint32_t box[2] = {64, 16};
-  const cuuint32_t estr[2] = {1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
 
 void free_handle(reskv_cache* c) {
   if (!c) return;
@@ -152,54 +140,9 @@ int cluster_warps(int64_t budget, int cluster) {
                                std::max<int64_t>(1, (chunks + cluster - 1) / cluster)));
 }
 
-// Split plan of the tensor-core stream-K kernel for a launch of `n_units`
-// units holding `total_slots` slots: W warps, wpc per CTA, and k > 0 when
-// every warp takes k whole units instead of an equal slot piece.
-struct MmaPlan {
-  int64_t W = 1;
-  int wpc = kDecodeWarpsPerCta;
-  int32_t k = 0;
-  int stages = 0;                     // ring stages per warp
-};
-
-// At most 7 warps per SM: 7 x 2 ring stages streamed the 32-layer 32K cache
-// 1 % faster than 8 x 2 and 8 x 3.
-constexpr int kMmaWarpsPerCta = 7;
-
 MmaPlan plan_mma(const reskv_cache* c, int64_t n_units, int64_t total_slots) {
-  MmaPlan m;
-  int64_t W = 0;
-  int wpc = kMmaWarpsPerCta;
-  if (c->cfg.decode_warps > 0) {
-    W = c->cfg.decode_warps;
-  } else if (n_units >= c->num_sms && n_units <= 4 * int64_t(c->num_sms) &&
-             c->max_unit_slots <= 256 && !c->ragged) {
-    W = n_units;                      // one warp per unit: no partial records at all
-  } else {
-    wpc = int(std::min<int64_t>(kMmaWarpsPerCta,
-                                std::max<int64_t>(1, total_slots / (int64_t(c->num_sms) * 200))));
-    W = int64_t(c->num_sms) * wpc;
-    if (total_slots < W * 32) W = std::max<int64_t>(1, total_slots / 32);
-  }
-  // every warp needs a 16-slot chunk of its own (pieces are whole chunks)
-  if (W > total_slots / kDecodeChunk) W = total_slots / kDecodeChunk;
-  if (W > c->max_warps) W = c->max_warps;
-  if (W < 1) W = 1;
-  // Short units (each at most an eighth of a warp's piece): every warp takes
-  // k consecutive whole units, so no unit is cut and no partial record,
-  // ticket or merge is needed; the warps' loads differ by at most one unit.
-  if (c->cfg.decode_warps == 0 && int64_t(c->max_unit_slots) * 8 * W <= total_slots) {
-    const int64_t k = (n_units + W - 1) / W;
-    W = (n_units + k - 1) / k;
-    m.k = int32_t(k);
-  }
-  m.W = W;
-  m.wpc = int(std::min<int64_t>(8, (W + c->num_sms - 1) / c->num_sms));
-  // Ring depth: about 16 stages per SM in all.  On the 32-layer 32K cache
-  // 8 warps x 2 stages stream faster than 8 x 3 (and 6 x 3 than 6 x 2):
-  // more copies in flight only lengthen the loaded latency.
-  m.stages = std::min(decode_mma_stages(m.wpc), std::max(2, (16 + m.wpc / 2) / m.wpc));
-  return m;
+  return plan_mma_shape(c->num_sms, c->max_warps, c->cfg.decode_warps, c->max_unit_slots,
+                        c->ragged, n_units, total_slots);
 }
 
 // Cluster decode shape for launches of `units` units: the largest cluster
@@ -317,6 +260,60 @@ reskv_status finalize_ragged_layout(reskv_cache* c) {
   reskv_status st = plan_cluster(c, per_layer, &c->cplan_layer);
   if (st == RESKV_OK) st = plan_cluster(c, c->n_units, &c->cplan_all);
   return st;
+}
+
+// [rows, 128] bf16 row-major -> TMA map with boxes of 16 rows x 64 dims, 128B swizzle
+bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {cuuint64_t(kHeadDim), cuuint64_t(rows)};
+  const cuuint64_t strides[1] = {cuuint64_t(kSlotRowBytes)};
+  const cuuint32_t box[2] = {64, 16};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// At most 7 warps per SM: 7 x 2 ring stages streamed the 32-layer 32K cache
+// 1 % faster than 8 x 2 and 8 x 3.
+constexpr int kMmaWarpsPerCta = 7;
+
+MmaPlan plan_mma_shape(int num_sms, int64_t max_warps, int32_t user_warps, int64_t max_unit_slots,
+                       bool ragged, int64_t n_units, int64_t total_slots) {
+  MmaPlan m;
+  int64_t W = 0;
+  int wpc = kMmaWarpsPerCta;
+  if (user_warps > 0) {
+    W = user_warps;
+  } else if (n_units >= num_sms && n_units <= 4 * int64_t(num_sms) &&
+             max_unit_slots <= 256 && !ragged) {
+    W = n_units;                      // one warp per unit: no partial records at all
+  } else {
+    wpc = int(std::min<int64_t>(kMmaWarpsPerCta,
+                                std::max<int64_t>(1, total_slots / (int64_t(num_sms) * 200))));
+    W = int64_t(num_sms) * wpc;
+    if (total_slots < W * 32) W = std::max<int64_t>(1, total_slots / 32);
+  }
+  // every warp needs a 16-slot chunk of its own (pieces are whole chunks)
+  if (W > total_slots / kDecodeChunk) W = total_slots / kDecodeChunk;
+  if (W > max_warps) W = max_warps;
+  if (W < 1) W = 1;
+  // Short units (each at most an eighth of a warp's piece): every warp takes
+  // k consecutive whole units, so no unit is cut and no partial record,
+  // ticket or merge is needed; the warps' loads differ by at most one unit.
+  if (user_warps == 0 && int64_t(max_unit_slots) * 8 * W <= total_slots) {
+    const int64_t k = (n_units + W - 1) / W;
+    W = (n_units + k - 1) / k;
+    m.k = int32_t(k);
+  }
+  m.W = W;
+  m.wpc = int(std::min<int64_t>(8, (W + num_sms - 1) / num_sms));
+  // Ring depth: about 16 stages per SM in all.  On the 32-layer 32K cache
+  // 8 warps x 2 stages stream faster than 8 x 3 (and 6 x 3 than 6 x 2):
+  // more copies in flight only lengthen the loaded latency.
+  m.stages = std::min(decode_mma_stages(m.wpc), std::max(2, (16 + m.wpc / 2) / m.wpc));
+  return m;
 }
 
 }  // namespace reskv

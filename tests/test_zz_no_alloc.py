@@ -52,10 +52,13 @@ def _layout(L, Bt, H, b, seed=7):
     return lay, Q
 
 
-def test_noalloc_matches_regular_entry_point_on_repeated_calls():
+@pytest.mark.parametrize("b", [400, 300])
+def test_noalloc_matches_regular_entry_point_on_repeated_calls(b):
+    """b = 400 (a multiple of 16) runs the tensor-core kernel, b = 300 the
+    CUDA-core one; both agree with the regular entry point."""
     assert torch.cuda.is_available(), "GPU tests need a CUDA device"
     B.build()
-    L, Bt, H, b = 3, 2, 4, 400
+    L, Bt, H = 3, 2, 4
     lay, Q = _layout(L, Bt, H, b)
     cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=4, seq_len=b + 32,
                                  budget=b)
