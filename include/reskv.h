@@ -250,6 +250,11 @@ typedef struct reskv_cache_info {
                               (short units), 0 for equal slot pieces or when
                               that call runs another kernel                 */
   int32_t layer_units_per_warp; /* the same for a one-layer call (layer 0)   */
+  int32_t kv_copy_rank;    /* rank of the TMA copies of the tensor-core
+                              kernels: 3 (one copy per 16-row K or V chunk)
+                              or 2 (two 64-dim copies, when the driver
+                              refuses the 3-D map)                           */
+  int32_t reserved0;
 } reskv_cache_info;
 
 reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info);

@@ -162,14 +162,8 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   __syncwarp();
 
   auto issue = [&](int k, int s) {     // lane 0: chunk k into stage s
-    const int row = wcb + k * kCh;
-    const uint32_t st = base + s * kStageBytes;
-    mbar_arrive_expect_tx(&bars[s], kStageBytes + kCh * 4);
-    tma_load_2d(st, &tmK, 0, row, &bars[s]);
-    tma_load_2d(st + kBox, &tmK, 64, row, &bars[s]);
-    tma_load_2d(st + 2 * kBox, &tmV, 0, row, &bars[s]);
-    tma_load_2d(st + 3 * kBox, &tmV, 64, row, &bars[s]);
-    bulk_g2s(logc_s + s * kCh, p.logc + row, kCh * 4, &bars[s]);
+    issue_stage(base + s * kStageBytes, logc_s + s * kCh, &tmK, &tmV, p.logc, wcb + k * kCh, p.kv_rank,
+                &bars[s]);
   };
   const int issued0 = nchunks < kSt ? nchunks : kSt;
   if (lane == 0)

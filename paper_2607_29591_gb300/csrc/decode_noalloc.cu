@@ -113,10 +113,16 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
   // which reads slot by slot.
   const bool mma = c->budget % kDecodeChunk == 0 && aligned16(c->logc) && total + 16 < (int64_t(1) << 31);
   CUtensorMap tk, tv;
+  int kv_rank = 2;
   MmaPlan mp;
   int64_t W = 0;
   if (mma) {
-    if (!encode_rows(&tk, c->kslots, uint64_t(total)) || !encode_rows(&tv, c->vslots, uint64_t(total)))
+    kv_rank = 3;                        // one copy per chunk, else two
+    if (!encode_rows(&tk, c->kslots, uint64_t(total), 3) ||
+        !encode_rows(&tv, c->vslots, uint64_t(total), 3))
+      kv_rank = 2;
+    if (kv_rank == 2 && (!encode_rows(&tk, c->kslots, uint64_t(total), 2) ||
+                         !encode_rows(&tv, c->vslots, uint64_t(total), 2)))
       return fail(RESKV_ERR_CUDA, "cuTensorMapEncodeTiled refused the cache arrays");
     mp = plan_mma_shape(num_sms, int64_t(num_sms) * kDecodeWarpsPerCta, 0, c->budget, false,
                         c->n_units, total);
@@ -162,6 +168,7 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
   p.tail_unused = 0;
   p.n_app = nullptr;
   p.offsets = nullptr;
+  p.kv_rank = kv_rank;
   p.n_kv_heads = c->n_kv_heads;
   p.total_slots = total;
   p.n_warps = int32_t(W);

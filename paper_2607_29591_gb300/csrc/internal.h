@@ -53,6 +53,8 @@ struct DecodeParams {
   int32_t gate_mode;
   int32_t softmax_mode;         // RESKV_SOFTMAX_*
   float tau, alpha, g_min, g_fixed;
+  int32_t kv_rank;              // rank of the K and V TMA maps: 3 (one copy per
+                                // 16-row chunk) or 2 (two copies)
   int32_t units_per_warp;       // tensor-core stream-K kernel: 0 cuts the slot
                                 // range into n_warps equal pieces; k > 0 gives
                                 // warp w the whole units [w k, (w + 1) k) of the
@@ -103,9 +105,13 @@ struct MmaPlan {
 };
 MmaPlan plan_mma_shape(int num_sms, int64_t max_warps, int32_t user_warps, int64_t max_unit_slots,
                        bool ragged, int64_t n_units, int64_t total_slots);
-// TMA map of [rows, 128] bf16 rows: boxes of 16 rows x 64 dims, 128-byte
-// swizzle (base 16-byte aligned).  False if the driver refuses it.
-bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows);
+// TMA map of [rows, 128] bf16 rows (base 16-byte aligned) for 16-row chunk
+// copies into the 128-byte swizzled stage layout [dims 0..63 of the 16 rows |
+// dims 64..127 of the 16 rows].  rank 3: one copy per chunk, box {64 dims,
+// 16 rows, 2 halves} over dims {64, rows, 2} whose halves lie 128 bytes apart;
+// rank 2: two copies, box {64 dims, 16 rows} at dims 0 and 64.  False if the
+// driver refuses the map.
+bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, int rank);
 
 }  // namespace reskv
 
@@ -166,6 +172,7 @@ struct reskv_cache {
   // 16 rows x 64 dims with the 128-byte swizzle
   CUtensorMap tmap_k;
   CUtensorMap tmap_v;
+  int32_t kv_rank = 2;          // rank of both maps (encode_rows)
   // construction intermediates kept for reskv_export_debug (device)
   double* dbg_scores = nullptr;
   int32_t* dbg_ranked = nullptr;

@@ -99,6 +99,34 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map, int x, int y, int z,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::
+          "r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// The copies of one stage (one thread): K and V rows [row, row + 16) into st
+// (K dims 0..63 | K dims 64..127 | V dims 0..63 | V dims 64..127) and their
+// 16 log-counts into lc, all completing on bar.  kv_rank: that of the maps.
+__device__ __forceinline__ void issue_stage(uint32_t st, float* lc, const CUtensorMap* tmK,
+                                            const CUtensorMap* tmV, const float* logc, int row,
+                                            int kv_rank, uint64_t* bar) {
+  mbar_arrive_expect_tx(bar, kStageBytes + kCh * 4);
+  if (kv_rank == 3) {
+    tma_load_3d(st, tmK, 0, row, 0, bar);
+    tma_load_3d(st + 2 * kBox, tmV, 0, row, 0, bar);
+  } else {
+    tma_load_2d(st, tmK, 0, row, bar);
+    tma_load_2d(st + kBox, tmK, 64, row, bar);
+    tma_load_2d(st + 2 * kBox, tmV, 0, row, bar);
+    tma_load_2d(st + 3 * kBox, tmV, 64, row, bar);
+  }
+  bulk_g2s(lc, logc + row, kCh * 4, bar);
+}
+
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
                                         uint32_t& r3) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"

@@ -233,7 +233,11 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
     free_handle(c);
     return cuda_fail(err, "initialising the cache");
   }
-  if (!encode_rows(&c->tmap_k, c->kslots, slots) || !encode_rows(&c->tmap_v, c->vslots, slots)) {
+  c->kv_rank = 3;                       // one copy per chunk, else two
+  if (!encode_rows(&c->tmap_k, c->kslots, slots, 3) || !encode_rows(&c->tmap_v, c->vslots, slots, 3))
+    c->kv_rank = 2;
+  if (c->kv_rank == 2 &&
+      (!encode_rows(&c->tmap_k, c->kslots, slots, 2) || !encode_rows(&c->tmap_v, c->vslots, slots, 2))) {
     free_handle(c);
     return fail(RESKV_ERR_CUDA, "creating the TMA tensor maps of the cache");
   }
@@ -262,16 +266,23 @@ reskv_status finalize_ragged_layout(reskv_cache* c) {
   return st;
 }
 
-// [rows, 128] bf16 row-major -> TMA map with boxes of 16 rows x 64 dims, 128B swizzle
-bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows) {
+bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, int rank) {
   PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
   if (!enc) return false;
+  const cuuint32_t estr[3] = {1, 1, 1};
+  if (rank == 3) {
+    const cuuint64_t dims[3] = {64, cuuint64_t(rows), 2};
+    const cuuint64_t strides[2] = {cuuint64_t(kSlotRowBytes), 128};
+    const cuuint32_t box[3] = {64, 16, 2};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  }
   const cuuint64_t dims[2] = {cuuint64_t(kHeadDim), cuuint64_t(rows)};
   const cuuint64_t strides[1] = {cuuint64_t(kSlotRowBytes)};
   const cuuint32_t box[2] = {64, 16};
-  const cuuint32_t estr[2] = {1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -468,6 +479,7 @@ reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int3
   p.n_res = c->n_res;
   p.n_app = c->append_capacity > 0 ? c->n_app : nullptr;
   p.offsets = c->ragged ? c->offsets : nullptr;
+  p.kv_rank = c->kv_rank;
   p.Q = static_cast<const __nv_bfloat16*>(Q);
   p.O = static_cast<float*>(O);
   p.partials = c->partials;
@@ -691,6 +703,8 @@ reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info) {
       mma_layer ? plan_mma(c, per_layer, c->h_offsets[size_t(per_layer)]).k : 0;
   info->n_candidates = c->n_candidates;
   info->ranked_width = int32_t(c->dbg_ranked ? c->dbg_n_top : c->ranked_width);
+  info->kv_copy_rank = c->kv_rank;
+  info->reserved0 = 0;
   return RESKV_OK;
 }
 

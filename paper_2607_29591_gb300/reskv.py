@@ -72,7 +72,8 @@ class reskv_cache_info(ctypes.Structure):
                 ("max_appended", ctypes.c_int32), ("ragged", ctypes.c_int32),
                 ("total_slots", ctypes.c_int64), ("n_candidates", ctypes.c_int32),
                 ("ranked_width", ctypes.c_int32), ("all_units_per_warp", ctypes.c_int32),
-                ("layer_units_per_warp", ctypes.c_int32)]
+                ("layer_units_per_warp", ctypes.c_int32), ("kv_copy_rank", ctypes.c_int32),
+                ("reserved0", ctypes.c_int32)]
 
 
 class reskv_device_cache(ctypes.Structure):

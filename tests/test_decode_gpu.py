@@ -216,6 +216,17 @@ def test_layer_range_calls_match_all_layer_call():
     R.reskv_check_status(h)
 
 
+def test_kv_chunks_are_single_3d_copies():
+    """On this part the driver takes the 3-D K/V maps: one TMA copy per
+    16-row chunk of K or of V (the 2-D form, two copies each, is the
+    fallback).  The decode results are those the other tests check."""
+    L, Bt, H, G, b = 1, 1, 2, 4, 64
+    w, lay = synthetic_layout(L, Bt, H, b, [(60, 4), (64, 0)])
+    cfg = mkcfg(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len, budget=b)
+    h = R.reskv_import_cache(cfg, **lay)
+    assert R.reskv_get_info(h)["kv_copy_rank"] == 3
+
+
 def test_host_buffer_call_matches_device_call():
     """reskv_decode_attn_host gives the device call's outputs bit for bit and
     matches the oracle, with page-locked buffers (the kernel reads Q and
