@@ -5,17 +5,19 @@
 // Launches are programmatic dependent launches (a kernel streams its first
 // ring of cache chunks while the previous kernel on the stream finishes).
 //
-// Same split of work as the CUDA-core kernel (decode_kernel.cu): a launch
-// streams the flat slot range of its units, cut into W equal contiguous
-// pieces, one per warp; units cut between warps are merged by the last warp
-// to arrive.  What changes is the inner loop, which is instruction-bound on
-// CUDA cores (about 50 warp instructions per 512-byte slot).  Here one warp
-// step covers a 16-slot tile with legacy tensor-core MMAs (mma_tile.cuh).
+// A launch streams the flat slot range of its units as 16-slot chunks
+// (aligned to 16 global slots), cut into W equal pieces of whole chunks, one
+// per warp (or, for short units, k whole units per warp); units cut between
+// warps are merged by the last warp to arrive.  The CUDA-core kernel
+// (decode_kernel.cu) splits the same range by slots and is instruction-bound
+// (about 50 warp instructions per 512-byte slot); here one warp step covers a
+// 16-slot tile with legacy tensor-core MMAs (mma_tile.cuh).
 //
-// K and V rows reach shared memory through 2-D TMA tensor copies with the
-// 128-byte swizzle; the residual log-counts of each 16-slot chunk ride along
-// as a 64-byte bulk copy.  Chunks are aligned to 16 global slots; rows outside
-// the warp's piece are masked.
+// K and V rows reach shared memory through TMA tensor copies with the
+// 128-byte swizzle; the residual log-counts of each chunk ride along as a
+// 64-byte bulk copy.  Rows of a chunk outside the warp's units are masked.
+// Each warp stages its units' query rows and output rows through shared
+// memory as whole rows, which matters when Q and O sit in host memory.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -125,7 +127,6 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   tile_offsets(lane, off_k, off_pv);
 
   const float qscale = kLog2e * rsqrtf(float(kHeadDim));
-  bool failed = false;
 
   // this warp's staging of query rows (two buffers) and output rows
   uint8_t* io = ring.cta + ring_smem_bytes(kW, kSt) + warp * kIoBytes;
@@ -284,7 +285,6 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   uint32_t phase = 0;                                 // parity of its current use
   for (int k = 0; k < nchunks && !done; ++k) {
     if (!mbar_wait_bounded(&bars[s], phase)) {
-      failed = true;
       if (lane == 0) report_status(p.status, kStatusWaitTimeout);
       break;
     }
@@ -347,7 +347,6 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   // never leave with a copy in flight into this warp's ring (bounded waits)
   for (int kk = waited; kk < issued; ++kk)
     mbar_wait_bounded(&bars[kk % kSt], uint32_t((kk / kSt) & 1));
-  (void)failed;
 }
 
 }  // namespace

@@ -17,10 +17,12 @@ constexpr int kSlotRowBytes = kHeadDim * 2;
 constexpr float kLog2e = 1.4426950408889634f;
 
 // Decode split: every launch streams the concatenated slot range of its units
-// ("flat" index x = local_unit * stride + j) and cuts it into n_warps equal
-// contiguous pieces, one per warp.  A unit covered by one warp is finished by
-// that warp; a unit cut between warps is finished by the last of them to
-// arrive, from per-(unit, warp) partial records.
+// ("flat" index x = local_unit * stride + j) and cuts it into n_warps pieces,
+// one per warp (equal slot pieces in the CUDA-core kernel, equal pieces of
+// whole 16-slot chunks or whole units in the tensor-core stream-K kernel).  A
+// unit covered by one warp is finished by that warp; a unit cut between warps
+// is finished by the last of them to arrive, from per-(unit, warp) partial
+// records.
 //
 // Unit u owns slots [u*stride, u*stride + stride), stride = budget + append
 // capacity, or with per-unit budgets [offsets[u], offsets[u+1]) of size
