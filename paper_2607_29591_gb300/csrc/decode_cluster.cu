@@ -161,13 +161,13 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   }
   __syncwarp();
 
-  auto issue = [&](int k, int s) {     // lane 0: chunk k into stage s
+  auto issue = [&](int k, int s, bool with_logc) {   // lane 0: chunk k into stage s
     issue_stage(base + s * kStageBytes, logc_s + s * kCh, &tmK, &tmV, p.logc, wcb + k * kCh, p.kv_rank,
-                &bars[s]);
+                with_logc, &bars[s]);
   };
   const int issued0 = nchunks < kSt ? nchunks : kSt;
   if (lane == 0)
-    for (int k = 0; k < issued0; ++k) issue(k, k);
+    for (int k = 0; k < issued0; ++k) issue(k, k, true);   // before the counts are read
   // Programmatic dependent launch: the next kernel on the stream may start
   // now (its own prologue and cache copies overlap this kernel's tail) ...
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -215,7 +215,10 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
     if (k + kSt < nchunks) {
       if (lane == 0) {
         fence_proxy_async_smem();
-        issue(k + kSt, s);
+        // a main-only pass never reads log-counts; otherwise only chunks
+        // with residual rows need them
+        issue(k + kSt, s,
+              kMode != kMainBranch && !chunk_main_only(wcb + (k + kSt) * kCh, ub, nm, nr, nm + nr + na));
       }
       issued = k + kSt + 1;
     }

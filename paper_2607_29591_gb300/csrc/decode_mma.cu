@@ -113,12 +113,13 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   }
   __syncwarp();
 
-  auto issue = [&](int k, int s) {     // lane 0: chunk k into stage s
+  auto issue = [&](int k, int s, bool with_logc) {   // lane 0: chunk k into stage s
     issue_stage(base + s * kStageBytes, logc_s + s * kCh, &tmK, &tmV, p.logc, cb + k * kCh, p.kv_rank,
-                &bars[s]);
+                with_logc, &bars[s]);
   };
+  // the first ring goes out before the unit's counts are read: with log-counts
   if (lane == 0)
-    for (int k = 0; k < nchunks && k < kSt; ++k) issue(k, k);
+    for (int k = 0; k < nchunks && k < kSt; ++k) issue(k, k, true);
   // Programmatic dependent launch: the next kernel on the stream may start
   // now and overlap its prologue and first cache copies with this kernel.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -330,7 +331,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     if (k + kSt < nchunks) {
       if (lane == 0) {
         fence_proxy_async_smem();
-        issue(k + kSt, s);
+        issue(k + kSt, s, !chunk_main_only(cb + (k + kSt) * kCh, ub, nm, nr, nt));
       }
       issued = k + kSt + 1;
     }

@@ -109,12 +109,14 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* map
 }
 
 // The copies of one stage (one thread): K and V rows [row, row + 16) into st
-// (K dims 0..63 | K dims 64..127 | V dims 0..63 | V dims 64..127) and their
-// 16 log-counts into lc, all completing on bar.  kv_rank: that of the maps.
+// (K dims 0..63 | K dims 64..127 | V dims 0..63 | V dims 64..127) and, with
+// with_logc, their 16 log-counts into lc, all completing on bar.  kv_rank:
+// that of the maps.  A chunk known to hold no residual rows skips the
+// log-counts (the tile step reads them only at residual rows).
 __device__ __forceinline__ void issue_stage(uint32_t st, float* lc, const CUtensorMap* tmK,
                                             const CUtensorMap* tmV, const float* logc, int row,
-                                            int kv_rank, uint64_t* bar) {
-  mbar_arrive_expect_tx(bar, kStageBytes + kCh * 4);
+                                            int kv_rank, bool with_logc, uint64_t* bar) {
+  mbar_arrive_expect_tx(bar, kStageBytes + (with_logc ? kCh * 4 : 0));
   if (kv_rank == 3) {
     tma_load_3d(st, tmK, 0, row, 0, bar);
     tma_load_3d(st + 2 * kBox, tmV, 0, row, 0, bar);
@@ -124,7 +126,13 @@ __device__ __forceinline__ void issue_stage(uint32_t st, float* lc, const CUtens
     tma_load_2d(st + 2 * kBox, tmV, 0, row, bar);
     tma_load_2d(st + 3 * kBox, tmV, 64, row, bar);
   }
-  bulk_g2s(lc, logc + row, kCh * 4, bar);
+  if (with_logc) bulk_g2s(lc, logc + row, kCh * 4, bar);
+}
+
+// Whether the 16 rows from r0 are all main or appended rows of a unit whose
+// used rows are [ub, ub + nt) with residual rows [ub + nm, ub + nm + nr).
+__device__ __forceinline__ bool chunk_main_only(int r0, int ub, int nm, int nr, int nt) {
+  return r0 >= ub && r0 + kCh <= ub + nt && (r0 + kCh <= ub + nm || r0 >= ub + nm + nr);
 }
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
