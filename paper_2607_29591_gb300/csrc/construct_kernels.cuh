@@ -976,7 +976,8 @@ __global__ void __launch_bounds__(kThreads, 2) k_lloyd_assign(LloydArgs p) {
       double a[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const double4 c = *reinterpret_cast<const double4*>(c64 + int64_t(jq[q] < 0 ? 0 : jq[q]) * kHeadDim);
+        const double4_32a c =
+            *reinterpret_cast<const double4_32a*>(c64 + int64_t(jq[q] < 0 ? 0 : jq[q]) * kHeadDim);
         double s = (kx[0] - c.x) * (kx[0] - c.x);
         s = fma(kx[1] - c.y, kx[1] - c.y, s);
         s = fma(kx[2] - c.z, kx[2] - c.z, s);
