@@ -542,8 +542,10 @@ def main():
     # waits for every step.
     Qh = Qdec[:min(n_q, 64)].cpu().pin_memory()
     Oh = torch.empty(O.shape, dtype=torch.float32).pin_memory()
-    e2e_steps = args.steps                  # every step synchronises the host: time as many
-    stream = torch.cuda.current_stream()    # as the device leg so that a host hiccup weighs little
+    # every step synchronises the host: time as many steps as the device leg,
+    # so that one host hiccup weighs little
+    e2e_steps = args.steps
+    stream = torch.cuda.current_stream()
     for i in range(max(3, args.warmup)):
         R.reskv_decode_attn_host(cache, Qh[i % Qh.shape[0]], Oh, stream=stream)
         stream.synchronize()
