@@ -95,6 +95,40 @@ def test_noalloc_matches_regular_entry_point_on_repeated_calls(b):
     handle.free()
 
 
+def test_noalloc_misaligned_logcounts_take_the_cuda_core_kernel():
+    """Log-counts that are not 16-byte aligned rule out the tensor-core
+    kernel's bulk copies; the call takes the CUDA-core kernel and still agrees
+    with the regular entry point."""
+    B.build()
+    L, Bt, H, b = 2, 2, 4, 400
+    lay, Q = _layout(L, Bt, H, b, seed=11)
+    cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=4, seq_len=b + 32,
+                                 budget=b)
+    handle = R.reskv_import_cache(cfg, **lay)
+    Qd = Q.cuda()
+    O_ref = torch.empty(Qd.shape, dtype=torch.float32, device="cuda")
+    R.reskv_decode_attn(handle, -1, Qd, O_ref)
+    dev = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a)).cuda().view(dt)
+    ks = dev(lay["kslots"].view(np.int16), torch.bfloat16)
+    vs = dev(lay["vslots"].view(np.int16), torch.bfloat16)
+    U = L * Bt * H
+    lc_buf = torch.zeros(U * b + 4, dtype=torch.float32, device="cuda")
+    lc = lc_buf[1:1 + U * b].view(U, b)                 # 4 bytes past a 16-byte boundary
+    lc.copy_(dev(lay["logc"], torch.float32))
+    assert lc.data_ptr() % 16 == 4
+    nm = dev(lay["n_main"], torch.int32)
+    nr = dev(lay["n_res"], torch.int32)
+    O = torch.full(Qd.shape, float("nan"), dtype=torch.float32, device="cuda")
+    R.reskv_decode_attn_noalloc(ks, vs, lc, nm, nr, H, 4, Qd, O)
+    torch.cuda.synchronize()
+    out = O.cpu().numpy()
+    ref = O_ref.cpu().numpy().astype(np.float64)
+    assert not np.isnan(out).any()
+    assert_output_parity(out, ref, "misaligned log-counts")
+    assert errors(out, ref)[1] < 1e-5
+    handle.free()
+
+
 def test_noalloc_rejects_calls_beyond_its_scratch():
     """A call whose scratch would exceed the 16 MiB array fails on the host
     with a clear message, before anything is launched."""
