@@ -204,7 +204,9 @@ reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int3
  * staging buffers, device Q and O of all layers, kept until reskv_free).
  * Asynchronous on `stream`: O_host holds the result once the stream has
  * passed the call (cudaStreamSynchronize).  Results equal reskv_decode_attn's
- * bit for bit.
+ * bit for bit.  The caller keeps both buffers.  RESKV_ERR_INVALID_ARG for a
+ * NULL pointer or overlapping buffers, RESKV_ERR_OOM when the staging buffers
+ * cannot be allocated, RESKV_ERR_CUDA when a copy or the launch fails.
  */
 reskv_status reskv_decode_attn_host(const reskv_cache* c, const void* Q_host, void* O_host,
                                     void* stream);
