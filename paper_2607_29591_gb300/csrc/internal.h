@@ -170,8 +170,9 @@ struct reskv_cache {
     void* o = nullptr;
   };
   mutable HostIo hio;
-  // 2-D TMA maps of kslots / vslots: [U * budget rows, 128 dims], boxes of
-  // 16 rows x 64 dims with the 128-byte swizzle
+  // TMA maps of kslots / vslots over [U * budget rows, 128 dims] for 16-row
+  // chunk copies with the 128-byte swizzle: rank 3 (one copy per chunk) or 2
+  // (two 64-dim copies), see encode_rows
   CUtensorMap tmap_k;
   CUtensorMap tmap_v;
   int32_t kv_rank = 2;          // rank of both maps (encode_rows)

@@ -20,9 +20,10 @@
 // columns 0..7, rows 8..15 the lo part, so accumulator row g plus row g + 8 is
 // the numerator of column g.
 //
-// A stage holds the tile's K and V rows as four 2-D TMA boxes of 64 dims x 16
-// rows with the 128-byte swizzle (K dims 0..63 | K dims 64..127 | V lo | V hi),
-// so that ldmatrix reads of eight rows at one column are bank-conflict free.
+// A stage holds the tile's K and V rows as four 2 KB blocks of 16 rows x 64
+// dims with the 128-byte swizzle (K dims 0..63 | K dims 64..127 | V lo | V hi;
+// one 3-D TMA copy fills both blocks of K, one both of V), so that ldmatrix
+// reads of eight rows at one column are bank-conflict free.
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
