@@ -21,7 +21,8 @@ the project's design notes):
   are averaged over the GQA group and summed over fit queries, then average
   pooled with a zero-padded window of ``pool`` (5) tokens (App. B.2);
 * query-free scoring (no observation window): ``s_p = ||k_p||^2`` -- a build
-  choice, the paper defines no such rule;
+  choice, the paper defines no such rule -- as the exact sum of the squares
+  rounded once to float64 (independent of summation order);
 * ranking ties go to the lower token index; Lloyd assignment ties go to the
   lower centre index; an empty cluster keeps its centre and ends with count 0
   (log-count ``-inf``: the slot contributes nothing);
@@ -46,6 +47,7 @@ LongBench) are not reproducible here (no model weights or benchmark data).
 """
 from __future__ import annotations
 
+import math
 from dataclasses import dataclass, field, replace
 from typing import Optional, Sequence
 
@@ -177,12 +179,13 @@ def scores_obs_pool(K: np.ndarray, Qfit: np.ndarray, pool: int) -> np.ndarray:
 
 
 def scores_keynorm(K: np.ndarray) -> np.ndarray:
-    """Query-free score s_p = ||k_p||^2 (a build choice; the paper has none),
-    summed over the dimensions in order (k_1^2 + k_2^2 + ...)."""
-    acc = np.zeros(K.shape[0], dtype=np.float64)
-    for i in range(K.shape[1]):
-        acc = acc + K[:, i] * K[:, i]
-    return acc
+    """Query-free score s_p = ||k_p||^2 (a build choice; the paper has none):
+    the exact sum of the squares, rounded once to float64.
+
+    Every square of a bf16 value is exact in float64 (8 significant bits
+    squared), so math.fsum, which returns the correctly rounded sum of its
+    exact inputs, gives the exact score whatever the order of the dims."""
+    return np.array([math.fsum(row) for row in K * K], dtype=np.float64)
 
 
 # ---------------------------------------------------------------------------

@@ -181,6 +181,13 @@ def _keynorm_abs(K):
     return np.sum(np.abs(K), axis=1)
 
 
+def _keynorm_in_dim_order(K):
+    acc = np.zeros(K.shape[0])
+    for i in range(K.shape[1]):
+        acc = acc + K[:, i] * K[:, i]
+    return acc
+
+
 def _val_loss_no_mean(cache, Qval, O_full, cfg):
     return _orig["validation_loss"](cache, Qval, O_full, cfg) * Qval.shape[0] * Qval.shape[1]
 
@@ -285,6 +292,7 @@ MUTANTS = [
     ("round_to_bf16", _round_truncate),
     ("log_counts", _logc_plus_one),
     ("scores_keynorm", _keynorm_abs),
+    ("scores_keynorm", _keynorm_in_dim_order),
     ("validation_loss", _val_loss_no_mean),
     ("attention_full", _attention_full_no_shift),
     ("separate_softmax_decode", _separate_additive),

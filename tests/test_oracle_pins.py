@@ -16,6 +16,7 @@ import pytest
 from scipy.special import softmax
 
 import oracle as orc
+from paper_2607_29591_gb300 import workloads as wl
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
 
@@ -506,6 +507,45 @@ def test_build_uses_only_fit_rows_for_scores():
 def test_keynorm_scores():
     K = np.array([[1.0, 2.0], [3.0, -1.0], [0.0, 0.5]])
     np.testing.assert_array_equal(orc.scores_keynorm(K), [5.0, 10.0, 0.25])
+
+
+def test_keynorm_score_is_the_exact_sum_rounded_once():
+    """A row of bf16 values whose squares span more than 53 bits: 2^14 in the
+    first dim (square 2^28, ulp 2^-24) and 2^-13 in the other 127 (squares
+    2^-26, a quarter ulp each).  Summed in dim order, every small square is
+    rounded away and the sum stays 2^28; the exact sum 2^28 + 127 * 2^-26
+    rounds to 2^28 + 32 * 2^-24 = 2^28 + 2^-19.  The score must be the
+    latter in every dim order."""
+    row = np.full(128, 2.0 ** -13)
+    row[0] = 2.0 ** 14
+    in_order = 0.0
+    for x in row:
+        in_order += x * x
+    assert in_order == 2.0 ** 28                      # what in-order summation gives
+    want = 2.0 ** 28 + 2.0 ** -19
+    K = np.stack([row, row[::-1], np.roll(row, 37)])
+    np.testing.assert_array_equal(orc.scores_keynorm(K), [want, want, want])
+    # exact integer arithmetic on the same squares agrees (every square of a
+    # bf16 value is a dyadic rational: scale by 2^26 to integers)
+    exact = sum(int(x * x * 2.0 ** 26) for x in row)
+    assert exact == 2 ** 54 + 127 and float(exact) * 2.0 ** -26 == want
+
+
+def test_keynorm_score_independent_of_dim_order_on_generator_rows():
+    """On rows drawn like the workloads' keys (with outlier channels), any
+    permutation of the dims gives the same score bit for bit, and the score
+    equals the exact rational sum rounded once."""
+    from fractions import Fraction
+    w = wl.scaled(wl.WORKLOADS["small_budget_b64"], seq_len=64)
+    K, _ = wl.unit_kv(w, 3, 1, 5)
+    Kf = K.double().numpy()
+    base = orc.scores_keynorm(Kf)
+    rng = np.random.default_rng(8)
+    for _ in range(3):
+        np.testing.assert_array_equal(orc.scores_keynorm(Kf[:, rng.permutation(128)]), base)
+    for p in range(0, 64, 9):
+        exact = sum(Fraction(float(x)) ** 2 for x in Kf[p])
+        assert float(exact) == base[p]
 
 
 # ---------------------------------------------------------------------------
