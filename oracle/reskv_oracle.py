@@ -33,6 +33,11 @@ the project's design notes):
   validation loss is evaluated on the stored (rounded) entries;
 * the validation loss averages over validation queries and the G query heads
   of the KV head;
+* decode-time growth into a bounded region of appended tokens: once it is
+  full, the oldest appended token leaves the exact window and is dropped or
+  folded into its nearest residual entry (exact squared distance, ties to the
+  lower entry) as a running mean (c k_bar + k) / (c + 1) in float64, stored as
+  bf16, count + 1;
 * AdaKV budgets (App. B, "AdaKV": SnapKV scores, safeguard 0.2): the KV heads
   of one (layer, batch element) share H*b slots; every head keeps its window
   P and its own f = floor(safeguard * (b - |P|)) best tokens, and the other
@@ -498,6 +503,80 @@ def append_tokens(cache: UnitCache, k_new: np.ndarray, v_new: np.ndarray,
                      kmain=np.vstack([cache.kmain, k_new]), vmain=np.vstack([cache.vmain, v_new]),
                      kbar=cache.kbar, vbar=cache.vbar, counts=cache.counts, logc=cache.logc,
                      r=cache.r, losses=cache.losses, scores=cache.scores)
+
+
+# policies for a token leaving a full append region (decode-time growth)
+APPEND_FAIL = 0          # no room: the append is refused
+APPEND_RING_DROP = 1     # the oldest appended token leaves the cache
+APPEND_RING_FOLD = 2     # the oldest appended token joins its nearest residual entry
+
+
+def nearest_entry(k: np.ndarray, kbar: np.ndarray) -> int:
+    """argmin_j ||k - kbar_j||^2 over the stored entries, ties -> lowest j
+    (the assignment rule of Eq. residual_partition), decided exactly.
+
+    Every bf16 value is an integer multiple of 2^-133 (the smallest bf16
+    subnormal), so the squared distances are compared as exact integers after
+    scaling by 2^133 (the scaling is a power of two: exact in float64)."""
+    scale = 2.0 ** 133
+    ki = [int(x * scale) for x in k]
+    best, best_d = -1, None
+    for j in range(kbar.shape[0]):
+        d = sum((a - int(b * scale)) ** 2 for a, b in zip(ki, kbar[j]))
+        if best_d is None or d < best_d:
+            best, best_d = j, d
+    return best
+
+
+def fold_into_entry(kbar_j, vbar_j, c_j: int, k, v, beta: float):
+    """One more member for entry j (Eq. summary as a running mean): with c_j
+    members summarised by the stored means, the new means are
+    (c_j kbar_j + k) / (c_j + 1) and (c_j vbar_j + v) / (c_j + 1), evaluated in
+    float64 in that order and stored as bf16 (round to nearest even); the
+    count becomes c_j + 1 and the logit term beta * log(c_j + 1).  An empty
+    entry (c_j = 0) becomes the token itself."""
+    c = float(c_j)
+    kb = round_to_bf16((c * kbar_j + k) / (c + 1.0))
+    vb = round_to_bf16((c * vbar_j + v) / (c + 1.0))
+    return kb, vb, c_j + 1, beta * np.log(c + 1.0)
+
+
+def append_ring(cache: UnitCache, k_new: np.ndarray, v_new: np.ndarray, positions: np.ndarray,
+                n_app: int, capacity: int, policy: int, beta: float = 1.0):
+    """Decode-time growth (Sec. 3.1: each decode step appends the new token)
+    into a bounded region of `capacity` appended tokens; n_app of them are the
+    last rows of the unit's main cache now.
+
+    While the region has room the token is appended (append_tokens).  When it
+    is full the oldest appended token leaves the exact window first: with
+    APPEND_RING_DROP it leaves the cache; with APPEND_RING_FOLD it becomes a
+    member of its nearest residual entry (nearest_entry, fold_into_entry) --
+    the residual refresh that the paper leaves to future work (App. E), in the
+    running-mean form of Eq. summary -- or leaves the cache when the unit has no
+    residual entries.  APPEND_FAIL refuses (ValueError).  Returns the grown
+    cache and its count of appended tokens."""
+    out = UnitCache(main_pos=cache.main_pos.copy(), kmain=cache.kmain.copy(),
+                    vmain=cache.vmain.copy(), kbar=cache.kbar.copy(), vbar=cache.vbar.copy(),
+                    counts=cache.counts.copy(), logc=cache.logc.copy(), r=cache.r,
+                    losses=cache.losses, scores=cache.scores)
+    for t in range(len(positions)):
+        if n_app == capacity:
+            if policy == APPEND_FAIL or capacity == 0:
+                raise ValueError("the append region is full")
+            o = out.kmain.shape[0] - n_app            # the oldest appended row
+            k_old, v_old = out.kmain[o].copy(), out.vmain[o].copy()
+            keep = np.arange(out.kmain.shape[0]) != o
+            out.kmain, out.vmain, out.main_pos = out.kmain[keep], out.vmain[keep], out.main_pos[keep]
+            n_app -= 1
+            if policy == APPEND_RING_FOLD and out.r > 0:
+                j = nearest_entry(k_old, out.kbar)
+                out.kbar[j], out.vbar[j], out.counts[j], out.logc[j] = fold_into_entry(
+                    out.kbar[j], out.vbar[j], int(out.counts[j]), k_old, v_old, beta)
+        out.kmain = np.vstack([out.kmain, k_new[t][None]])
+        out.vmain = np.vstack([out.vmain, v_new[t][None]])
+        out.main_pos = np.concatenate([out.main_pos, positions[t:t + 1]])
+        n_app += 1
+    return out, n_app
 
 
 def decode_unit(cache: UnitCache, Q: np.ndarray, cfg: OracleConfig) -> np.ndarray:

@@ -181,6 +181,44 @@ def _keynorm_abs(K):
     return np.sum(np.abs(K), axis=1)
 
 
+def _nearest_fp64(k, kbar):
+    return int(np.argmin(np.sum((kbar - k) ** 2, axis=1)))
+
+
+def _nearest_ties_high(k, kbar):
+    d = [float(np.sum((kbar[j] - k) ** 2)) for j in range(kbar.shape[0])]
+    return int(len(d) - 1 - np.argmin(d[::-1]))
+
+
+def _fold_halfway(kbar_j, vbar_j, c_j, k, v, beta):
+    return (orc_round((kbar_j + k) / 2), orc_round((vbar_j + v) / 2), c_j + 1,
+            beta * np.log(c_j + 1.0))
+
+
+def _fold_count_stays(kbar_j, vbar_j, c_j, k, v, beta):
+    kb, vb, c, lc = _orig["fold_into_entry"](kbar_j, vbar_j, c_j, k, v, beta)
+    return kb, vb, c_j, beta * np.log(max(c_j, 1))
+
+
+def _ring_evicts_newest(cache, k_new, v_new, positions, n_app, capacity, policy, beta=1.0):
+    out, na = cache, n_app
+    for t in range(len(positions)):
+        if na == capacity:
+            if policy == core.APPEND_FAIL:
+                raise ValueError("full")
+            out = core.UnitCache(main_pos=out.main_pos[:-1], kmain=out.kmain[:-1],
+                                 vmain=out.vmain[:-1], kbar=out.kbar, vbar=out.vbar,
+                                 counts=out.counts, logc=out.logc, r=out.r)
+            na -= 1
+        out = core.append_tokens(out, k_new[t:t + 1], v_new[t:t + 1], positions[t:t + 1])
+        na += 1
+    return out, na
+
+
+def orc_round(x):
+    return _orig["round_to_bf16"](x)
+
+
 def _keynorm_in_dim_order(K):
     acc = np.zeros(K.shape[0])
     for i in range(K.shape[1]):
@@ -293,6 +331,11 @@ MUTANTS = [
     ("log_counts", _logc_plus_one),
     ("scores_keynorm", _keynorm_abs),
     ("scores_keynorm", _keynorm_in_dim_order),
+    ("nearest_entry", _nearest_fp64),
+    ("nearest_entry", _nearest_ties_high),
+    ("fold_into_entry", _fold_halfway),
+    ("fold_into_entry", _fold_count_stays),
+    ("append_ring", _ring_evicts_newest),
     ("validation_loss", _val_loss_no_mean),
     ("attention_full", _attention_full_no_shift),
     ("separate_softmax_decode", _separate_additive),

@@ -731,3 +731,101 @@ def test_adakv_grouped_build_keeps_each_heads_budget():
         assert set(range(s - 8, s)) <= set(u.main_pos.tolist())
         keep = len(u.main_pos) - 8
         assert set(u.ranked[:keep].tolist()) | set(range(s - 8, s)) == set(u.main_pos.tolist())
+
+
+# ---------------------------------------------------------------------------
+# Decode-time growth into a bounded region (Sec. 3.1; App. E refresh)
+# ---------------------------------------------------------------------------
+
+def test_nearest_entry_is_exact_with_ties_to_the_lower_entry():
+    d = 128
+    k = np.zeros(d)
+    # squared distances 2^54 + 1 and 2^54 + 1/4: equal once rounded to float64
+    # (ulp 4 at 2^54), so only the exact comparison finds entry 1
+    kbar = np.zeros((2, d))
+    kbar[:, 0] = 2.0 ** 27
+    kbar[0, 1], kbar[1, 1] = 1.0, 0.5
+    fp64 = np.sum((kbar - k) ** 2, axis=1)
+    assert fp64[0] == fp64[1]
+    assert orc.nearest_entry(k, kbar) == 1
+    # exact ties go to the lower entry; k midway between two entries
+    kbar = np.zeros((3, d))
+    kbar[0, 3], kbar[1, 3], kbar[2, 3] = 1.0, -1.0, 1.0
+    assert orc.nearest_entry(k, kbar) == 0
+    assert orc.nearest_entry(k, kbar[[1, 0, 2]]) == 0
+    # brute force on separated random entries agrees with a float64 argmin
+    rng = np.random.default_rng(21)
+    for _ in range(20):
+        kb = orc.round_to_bf16(rng.normal(size=(7, d)) * 3)
+        kk = orc.round_to_bf16(kb[rng.integers(7)] + rng.normal(size=d) * 0.1)
+        assert orc.nearest_entry(kk, kb) == int(np.argmin(np.sum((kb - kk) ** 2, axis=1)))
+    # bf16 subnormals take part exactly
+    kbar = np.zeros((2, d))
+    kbar[0, 0], kbar[1, 0] = 3 * 2.0 ** -133, 2.0 ** -133
+    assert orc.nearest_entry(np.zeros(d), kbar) == 1
+
+
+def test_fold_is_the_running_mean_stored_in_bf16():
+    d = 128
+    z = np.zeros(d)
+    k = np.full(d, 0.75)
+    kb, vb, c, lc = orc.fold_into_entry(z, z, 0, k, -k, 1.0)      # empty entry: the token
+    assert np.array_equal(kb, k) and np.array_equal(vb, -k) and c == 1 and lc == 0.0
+    kb, vb, c, lc = orc.fold_into_entry(np.ones(d), np.full(d, 2.0), 3, np.full(d, 5.0),
+                                        np.full(d, -6.0), 1.0)
+    assert np.all(kb == 2.0) and np.all(vb == 0.0) and c == 4       # (3+5)/4, (6-6)/4
+    assert lc == pytest.approx(np.log(4.0), rel=0, abs=0)
+    # (2 * 1 + 2) / 3 = 4/3 = 1.0101010101...b: bf16 keeps 1.0101011b = 1.3359375
+    kb, _, _, lc = orc.fold_into_entry(np.ones(d), z, 2, np.full(d, 2.0), z, 0.5)
+    assert np.all(kb == 1.3359375) and lc == 0.5 * np.log(3.0)
+
+
+def _small_unit(rng, m, r, d=16, s_tokens=None):
+    K = bf16ish(rng, (m + r, d))
+    V = bf16ish(rng, (m + r, d))
+    counts = rng.integers(1, 9, r)
+    return orc.UnitCache(main_pos=np.arange(m), kmain=K[:m], vmain=V[:m], kbar=K[m:],
+                         vbar=V[m:], counts=counts, logc=np.log(counts.astype(np.float64)), r=r)
+
+
+def test_ring_append_keeps_the_most_recent_tokens():
+    rng = np.random.default_rng(22)
+    base = _small_unit(rng, 10, 0)
+    A, n = 3, 8
+    Kn, Vn = bf16ish(rng, (n, 16)), bf16ish(rng, (n, 16))
+    pos = np.arange(100, 100 + n)
+    # with room the ring is plain growth
+    grown, na = orc.append_ring(base, Kn[:A], Vn[:A], pos[:A], 0, A, orc.APPEND_RING_DROP)
+    ref = orc.append_tokens(base, Kn[:A], Vn[:A], pos[:A])
+    assert na == A and np.array_equal(grown.kmain, ref.kmain)
+    for policy in (orc.APPEND_RING_DROP, orc.APPEND_RING_FOLD):   # no entries: both drop
+        out, na = orc.append_ring(base, Kn, Vn, pos, 0, A, policy)
+        assert na == A
+        assert np.array_equal(out.main_pos, np.concatenate([np.arange(10), pos[-A:]]))
+        assert np.array_equal(out.kmain[-A:], Kn[-A:]) and np.array_equal(out.vmain[-A:], Vn[-A:])
+        q = bf16ish(rng, 16)
+        np.testing.assert_allclose(orc.decode_unit(out, q[None], orc.OracleConfig(budget=1))[0],
+                                   textbook_attention(q, out.kmain, out.vmain), rtol=1e-12)
+    with pytest.raises(ValueError):
+        orc.append_ring(base, Kn, Vn, pos, 0, A, orc.APPEND_FAIL)
+
+
+def test_ring_fold_loses_no_token_and_updates_the_nearest_entry():
+    rng = np.random.default_rng(23)
+    m, r, A = 12, 4, 5
+    base = _small_unit(rng, m, r)
+    before = base.counts.sum() + m
+    Kn, Vn = bf16ish(rng, (3 * A, 16)), bf16ish(rng, (3 * A, 16))
+    out, na = orc.append_ring(base, Kn, Vn, np.arange(50, 50 + 3 * A), 0, A,
+                              orc.APPEND_RING_FOLD)
+    assert na == A and out.kmain.shape[0] == m + A
+    assert out.counts.sum() + out.kmain.shape[0] == before + 3 * A       # every token kept
+    # the first token to leave (appended first) went to its nearest entry
+    one, _ = orc.append_ring(base, Kn[:A + 1], Vn[:A + 1], np.arange(A + 1), 0, A,
+                             orc.APPEND_RING_FOLD)
+    j = orc.nearest_entry(Kn[0], base.kbar)
+    assert one.counts[j] == base.counts[j] + 1
+    assert np.array_equal(np.delete(one.counts, j), np.delete(base.counts, j))
+    want = orc.round_to_bf16((base.counts[j] * base.kbar[j] + Kn[0]) / (base.counts[j] + 1))
+    assert np.array_equal(one.kbar[j], want)
+    assert one.logc[j] == np.log(base.counts[j] + 1.0)
