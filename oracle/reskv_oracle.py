@@ -112,16 +112,16 @@ def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
 def round_to_bf16(x: np.ndarray) -> np.ndarray:
     """Round float64 values to the nearest bf16 value, ties to even.
 
-    Direct rounding from float64 (8 significant bits kept), written with
-    frexp/ldexp so that no float32 double rounding occurs.  Zero stays zero;
-    the values rounded here (cluster means of bf16 inputs) lie far inside the
-    bf16 normal range.
+    bf16 keeps 8 significant bits down to 2^-126; below that (subnormals) its
+    spacing stays 2^-133.  Each value is divided by the spacing at its
+    magnitude (a power of two: exact), rounded to an integer (numpy rint:
+    half to even) and scaled back, so no float32 double rounding occurs.
+    Zero stays zero; values beyond the bf16 range are not expected here.
     """
     x = np.asarray(x, dtype=np.float64)
-    mant, expo = np.frexp(x)                 # x = mant * 2**expo, 0.5 <= |mant| < 1
-    scaled = np.ldexp(mant, 8)               # 8 significant bits in the integer part
-    rounded = np.rint(scaled)                # numpy rint: round half to even
-    return np.ldexp(rounded, expo - 8)
+    _, expo = np.frexp(x)                    # |x| in [2^(expo-1), 2^expo)
+    quantum = np.maximum(expo - 8, -133)     # exponent of the spacing at |x|
+    return np.ldexp(np.rint(np.ldexp(x, -quantum)), quantum)
 
 
 # ---------------------------------------------------------------------------

@@ -829,3 +829,21 @@ def test_ring_fold_loses_no_token_and_updates_the_nearest_entry():
     want = orc.round_to_bf16((base.counts[j] * base.kbar[j] + Kn[0]) / (base.counts[j] + 1))
     assert np.array_equal(one.kbar[j], want)
     assert one.logc[j] == np.log(base.counts[j] + 1.0)
+
+
+def test_bf16_rounding_in_the_subnormal_range():
+    """Below 2^-126 bf16 values are multiples of 2^-133: 2^-134 is a tie
+    between 0 and 2^-133 (to even: 0), 3 * 2^-134 a tie between 2^-133 and
+    2 * 2^-133 (to even: 2^-132), 1.25 * 2^-133 rounds down to 2^-133; the
+    smallest normal 2^-126 and its neighbours keep 8 significant bits."""
+    t = 2.0 ** -133
+    got = orc.round_to_bf16(np.array([2.0 ** -134, 3 * 2.0 ** -134, 1.25 * t, -1.75 * t,
+                                      2.0 ** -126, 2.0 ** -126 * (1 + 2.0 ** -8),
+                                      2.0 ** -126 * (1 + 3 * 2.0 ** -8), 127.5 * t]))
+    want = [0.0, 2.0 ** -132, t, -2 * t, 2.0 ** -126, 2.0 ** -126,
+            2.0 ** -126 * (1 + 2 * 2.0 ** -7), 128 * t]
+    assert got.tolist() == want
+    # every value the bf16 format holds is left alone
+    bits = np.arange(0, 0x7f80, 7, dtype=np.uint16)
+    vals = orc.bf16_bits_to_f64(bits)
+    assert np.array_equal(orc.round_to_bf16(vals), vals)
