@@ -2,9 +2,12 @@
 
 One step = one shared-softmax decode (Alg. 2) of every (layer, batch, KV head)
 unit of the workload for one fresh decode query per query head, through the
-C ABI (reskv_decode_attn with layer = -1: one launch covers all layers).  The
-compressed cache is built first by reskv_build_cache (Alg. 1, timed on its
-own).  Prints one JSON line.
+C ABI as a decoder issues it: one reskv_decode_attn call per layer (layer 0 ..
+L-1), the L launches captured in one CUDA graph.  Also reported: all layers
+in one launch (a ceiling: it needs every layer's query up front),
+end to end with host buffers, and a second workload measured the same way.
+The compressed cache is built first by reskv_build_cache (Alg. 1, timed on
+its own).  Prints one JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   (the fp64 CPU oracle on host cores)
@@ -54,7 +57,10 @@ def parse_args():
     ap.add_argument("--impl", choices=["reskv", "reference"], default="reskv")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(wl.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--no-per-layer", action="store_true")
+    ap.add_argument("--second-workload", default="long_128k_b4",
+                    choices=["none"] + sorted(wl.WORKLOADS),
+                    help="a second workload measured the same way (no e2e leg), reported "
+                         "under second_workload")
     ap.add_argument("--decode-kernel", choices=["auto", "mma", "cluster", "fma", "lse"],
                     default="auto",
                     help="automatic plan (default: cluster kernel for launches whose units "
@@ -259,24 +265,37 @@ def _oracle_decode(args):
 
 class OraclePool:
     """The fp64 oracle decode on the host cores: one spawned process per core,
-    each holding the seeded sample; work is split by units."""
+    each holding its part of the seeded sample.  Both CPU legs (the GPU arm's
+    cpu_baseline and the reference arm) time it the same way: one dispatch =
+    every worker decodes its units `reps` times, wall clock around the
+    dispatch, with reps chosen so that a dispatch takes about a second and its
+    inter-process cost (measured alone: a dispatch with reps = 0) is small."""
 
     def __init__(self, w: wl.Workload, n_sample: int, procs: int):
         import concurrent.futures
         import multiprocessing
         self.idx = oracle_sample(w, n_sample)
         self.procs = max(1, min(procs, len(self.idx)))
+        self.chunks = [c.tolist() for c in np.array_split(np.array(self.idx), self.procs) if len(c)]
         self.ex = concurrent.futures.ProcessPoolExecutor(
             self.procs, mp_context=multiprocessing.get_context("spawn"),
             initializer=_oracle_init, initargs=(w, self.idx))
         self.run(1)                                  # every worker up and warm
+        _, self.dispatch_s = self.run(0)
+        _, t1 = self.run(1)
+        self.reps = max(1, int(round(1.0 / max(t1, 1e-3))))
 
     def run(self, reps: int) -> tuple:
-        """(unit decodes, wall seconds) of `reps` passes over the sample."""
-        chunks = [c.tolist() for c in np.array_split(np.array(self.idx), self.procs) if len(c)]
+        """(unit decodes, wall seconds) of one dispatch of `reps` passes."""
         t0 = time.perf_counter()
-        n = sum(self.ex.map(_oracle_decode, [(c, reps) for c in chunks]))
+        n = sum(self.ex.map(_oracle_decode, [(c, reps) for c in self.chunks]))
         return n, time.perf_counter() - t0
+
+    def describe(self) -> str:
+        return (f"fp64 oracle decode of {len(self.idx)} seeded units split over {self.procs} "
+                f"spawned processes; one dispatch = {self.reps} passes over the sample "
+                f"(inter-process cost of a dispatch alone {self.dispatch_s * 1e3:.1f} ms), "
+                f"wall clock, extrapolated to all units of one step")
 
     def close(self):
         self.ex.shutdown()
@@ -334,12 +353,16 @@ def cpu_construction(w: wl.Workload, budget_s: float = 10.0):
                    f"figure assumes the {w.n_units} independent units spread over {cores} cores"}
 
 
-def cpu_baseline(w: wl.Workload, target_s: float = 12.0):
+def cpu_baseline(w: wl.Workload, dispatches: int = 8):
+    """The oracle as it stands on the host cores (same method as the
+    reference arm), a single-thread figure, and the oracle's construction."""
     cores = os.cpu_count() or 1
     pool = OraclePool(w, 64, cores)
-    n1, t1 = pool.run(1)
-    reps = max(1, int(target_s / max(t1, 1e-3)))
-    n, t = pool.run(reps)
+    n, t = 0, 0.0
+    for _ in range(dispatches):
+        dn, dt = pool.run(pool.reps)
+        n += dn
+        t += dt
     pool.close()
     step_s = t * w.n_units / n
     # one thread: the same units in this process
@@ -351,26 +374,25 @@ def cpu_baseline(w: wl.Workload, target_s: float = 12.0):
         orc.decode_unit(un, q, cfg)
     step_s1 = (time.perf_counter() - t0) * w.n_units / len(one)
     return {"value": w.batch / step_s, "unit": "tokens/s", "cores": pool.procs, "kind": "oracle",
-            "sample": f"fp64 oracle decode of {len(pool.idx)} seeded units x {reps} passes "
-                      f"(G={w.group} heads each, b={w.budget}) split over {pool.procs} processes, "
-                      f"wall clock, extrapolated to all {w.n_units} units of one step",
+            "sample": pool.describe() + f"; {dispatches} dispatches",
             "single_thread_value": w.batch / step_s1,
             "single_thread_sample": f"{len(one)} of those units in one process, one thread",
             "construction": cpu_construction(w)}
 
 
 def run_reference(args, world, rank):
-    """The reference arm: the fp64 oracle, as it stands, on the host cores."""
+    """The reference arm: the fp64 oracle, as it stands, on the host cores;
+    every step is one dispatch (cpu_baseline's method)."""
     if rank != 0:
         return
     w = wl.WORKLOADS[args.workload]
     cores = os.cpu_count() or 1
-    pool = OraclePool(w, 4 * cores, cores)
+    pool = OraclePool(w, 64, cores)
     for _ in range(args.warmup):
-        pool.run(1)
+        pool.run(pool.reps)
     n_tot, t = 0, 0.0
     for _ in range(args.steps):
-        n, dt = pool.run(1)
+        n, dt = pool.run(pool.reps)
         n_tot += n
         t += dt
     pool.close()
@@ -380,15 +402,20 @@ def run_reference(args, world, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name},
+            "config": workload_config(w),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": pool.procs,
                              "kind": "oracle",
-                             "sample": f"each step: fp64 oracle decode of {len(pool.idx)} seeded "
-                                       f"units over {pool.procs} processes (wall clock), "
-                                       f"extrapolated to {w.n_units} units"},
+                             "sample": pool.describe() + "; one dispatch per step"},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def workload_config(w: wl.Workload) -> dict:
+    """The workload's shape, named as in the JSON line's config."""
+    return {"workload": w.name, "layers": w.n_layers, "batch": w.batch,
+            "kv_heads": w.n_kv_heads, "q_heads": w.n_q_heads, "head_dim": w.head_dim,
+            "seq_len": w.seq_len, "budget": w.budget, "residual": w.residual}
 
 
 # ---------------------------------------------------------------------------
@@ -426,6 +453,182 @@ def build_workload(w: wl.Workload, n_q: int, device, decode_kernel: int, budget_
     return cache, Qdec, build_s
 
 
+def roofline(alg_bytes: int, launch_s: float, peak: float, peak_kind: str, kernel: str,
+             traffic) -> dict:
+    achieved = alg_bytes / launch_s / 1e9
+    return {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+            "frac": achieved / peak, "traffic": traffic, "kernel": kernel,
+            "peak_kind": f"{peak_kind} (burst copy)", "algorithmic_bytes_per_launch": alg_bytes,
+            "launch_us": launch_s * 1e6}
+
+
+def time_per_layer(R, cache, w, Qdec, O, warmup: int, steps: int, device,
+                   clk=None, world: int = 1):
+    """Seconds of `steps` decode steps of one-layer calls: the L launches of a
+    step (layer 0 .. L-1, reskv_decode_attn) captured in one CUDA graph; every
+    step copies its fresh queries into the graph's query buffer, then replays
+    it.  CUDA events on the launching stream."""
+    s = torch.cuda.Stream(device)
+    s.wait_stream(torch.cuda.current_stream(device))
+    Qs = torch.empty_like(Qdec[0])                    # [L, B, H_q, d]
+
+    def launches():
+        for l in range(w.n_layers):
+            R.reskv_decode_attn(cache, l, Qs[l], O[l], stream=s)
+
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(s):
+        Qs.copy_(Qdec[0])
+        launches()                                    # warm, outside capture
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=s):
+            launches()
+        for i in range(warmup):
+            Qs.copy_(Qdec[i % Qdec.shape[0]])
+            graph.replay()
+        s.synchronize()
+        with clk if clk is not None else _nullctx():
+            barrier(world)
+            torch.cuda.synchronize()
+            e0.record(s)
+            for i in range(steps):
+                Qs.copy_(Qdec[(warmup + i) % Qdec.shape[0]])
+                graph.replay()
+            e1.record(s)
+            torch.cuda.synchronize()
+            barrier(world)
+    del graph
+    return e0.elapsed_time(e1) / 1e3
+
+
+class _nullctx:
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        return False
+
+
+def time_all_layer(R, cache, w, Qdec, O, warmup: int, steps: int):
+    """Seconds of `steps` steps of one reskv_decode_attn(layer = -1) launch
+    each (every layer in one launch), fresh queries per step."""
+    stream = torch.cuda.current_stream()
+    for i in range(warmup):
+        R.reskv_decode_attn(cache, -1, Qdec[i % Qdec.shape[0]], O)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(steps):
+        R.reskv_decode_attn(cache, -1, Qdec[(warmup + i) % Qdec.shape[0]], O)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / 1e3
+
+
+def time_e2e(R, cache, Qdec, O, warmup: int, steps: int, world: int, device) -> tuple:
+    """reskv_decode_attn_host on page-locked host Q and O: the one decode
+    launch reads each unit's queries from host memory and writes its outputs
+    there (over the host link, overlapped with streaming the cache); the host
+    waits for every step."""
+    Qh = Qdec[:min(Qdec.shape[0], 64)].cpu().pin_memory()
+    Oh = torch.empty(O.shape, dtype=torch.float32).pin_memory()
+    stream = torch.cuda.current_stream()
+    for i in range(max(3, warmup)):
+        R.reskv_decode_attn_host(cache, Qh[i % Qh.shape[0]], Oh, stream=stream)
+        stream.synchronize()
+    barrier(world)
+    t0 = time.perf_counter()
+    for i in range(steps):
+        R.reskv_decode_attn_host(cache, Qh[i % Qh.shape[0]], Oh, stream=stream)
+        stream.synchronize()
+    te = reduce_max(time.perf_counter() - t0, world, device)
+    return te, int(Qh[0].numel() * 2), int(Oh.numel() * 4)
+
+
+def measure(args, w: wl.Workload, R, kern: int, bmode: int, device, world: int, peak: float,
+            peak_kind: str, clk=None, with_e2e: bool = True) -> dict:
+    """Build the workload's cache, then time its decode step: one-layer calls
+    in a CUDA graph, one
+    all-layer launch, and end to end with host buffers."""
+    n_q = args.steps + args.warmup
+    cache, Qdec, build_s = build_workload(w, n_q, device, kern, bmode)
+    info = R.reskv_get_info(cache)
+    unit_budgets = R.reskv_get_unit_budgets(cache)
+
+    def plan_name(cs, wpc):
+        if kern == R.RESKV_DECODE_LSE_MERGE:
+            return "paper-style: main pass + residual pass + log-sum-exp merge (3 launches)"
+        if cs == 0:
+            return "fma" if kern == R.RESKV_DECODE_FMA else "tensor-core stream-K"
+        return f"tensor-core cluster: {cs} CTA(s) x {wpc} warps per unit"
+
+    plan = {"all_layer": plan_name(info["all_cluster"], info["all_cluster_warps"]),
+            "per_layer": plan_name(info["layer_cluster"], info["layer_cluster_warps"])}
+    meta = R.reskv_export_cache(cache)
+    alg = algorithmic_bytes(meta["n_main"], meta["n_res"])
+    r_counts = meta["n_res"]
+    del meta
+    O = torch.empty((w.n_layers, w.batch, w.n_q_heads, w.head_dim), dtype=torch.float32,
+                    device=device)
+    L = w.n_layers
+    alg_layer = alg // L
+    launches_per_step = 3 * L if kern == R.RESKV_DECODE_LSE_MERGE else L
+    units_layer = w.batch * w.n_kv_heads
+    traffic_layer = None
+    if info["layer_cluster"] > 0 and not info["ragged"] and w.name == DEFAULT_WORKLOAD:
+        traffic_layer = profiled_traffic(units_layer, PROFILE_LAYER, KERNEL_SOURCES_LAYER)
+
+    # ---- the step: one-layer calls ----
+    t_local = time_per_layer(R, cache, w, Qdec, O, args.warmup, args.steps, device, clk, world)
+    t = reduce_max(t_local, world, device)
+    R.reskv_check_status(cache)
+    per_layer = {"s": t, "us_per_step": t / args.steps * 1e6,
+                 "us_per_layer_step": t / args.steps / L * 1e6,
+                 "tokens_per_s": aggregate(w.batch * args.steps, t, world),
+                 "roofline": roofline(alg_layer, t_local / args.steps / L, peak, peak_kind,
+                                      plan["per_layer"], traffic_layer),
+                 "how": f"{L} one-layer reskv_decode_attn launches per step replayed as one CUDA "
+                        f"graph; each step copies fresh queries into the graph's buffer"}
+    # ---- every layer in one launch ----
+    t_all = time_all_layer(R, cache, w, Qdec, O, args.warmup, args.steps)
+    R.reskv_check_status(cache)
+    all_layer = {"us_per_step": t_all / args.steps * 1e6,
+                 "us_per_layer_step": t_all / args.steps / L * 1e6,
+                 "tokens_per_s": w.batch * args.steps / t_all,
+                 "roofline": roofline(alg, t_all / args.steps, peak, peak_kind, plan["all_layer"],
+                                      None if info["ragged"] or w.name != DEFAULT_WORKLOAD
+                                      else profiled_traffic(w.n_units)),
+                 "q_o_bytes_per_step": int(w.n_units * w.group * w.head_dim * (2 + 4)),
+                 "how": "one reskv_decode_attn(layer=-1) launch per step (needs every layer's "
+                        "query up front: a ceiling, not a decoder's step)"}
+    out = {"config": dict(workload_config(w), **{
+               "mean_r": float(np.mean(r_counts)),
+               "units_with_residual": float(np.mean(r_counts > 0)),
+               "unit_budget_min_max": [int(unit_budgets.min()), int(unit_budgets.max())],
+               "decode_plan": plan,
+               "l2": f"inputs larger than L2: {alg / 1e9:.2f} GB of cache read per step"}),
+           "per_layer": per_layer, "all_layer": all_layer,
+           "launches_per_step": launches_per_step, "construction_s": build_s,
+           "construction_stages_ms": dict(zip(
+               ["scores", "ranking", "validation_targets", "lloyd", "validation_loss_and_choice",
+                "pack"], [round(x, 3) for x in info["build_ms"]])),
+           "construction_tflops": {
+               k: round(f / (info["build_ms"][i] * 1e-3) / 1e12, 2)
+               for k, i in (("scores", 0), ("validation_targets", 2), ("lloyd", 3))
+               for f in [construction_flops(w).get(k)] if f and info["build_ms"][i] > 0}}
+    if with_e2e:
+        te, bi, bo = time_e2e(R, cache, Qdec, O, args.warmup, args.steps, world, device)
+        out["e2e"] = {"value": aggregate(w.batch * args.steps, te, world), "unit": "tokens/s",
+                      "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo,
+                      "how": "reskv_decode_attn_host on pinned host Q and O: the decode launch "
+                             "reads Q from and writes O to host memory (NVLink-C2C), host waits "
+                             "every step"}
+    cache.free()
+    del Qdec, O
+    torch.cuda.empty_cache()
+    return out
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -443,173 +646,58 @@ def main():
     w = wl.WORKLOADS[args.workload]
     if args.layers:
         w = wl.scaled(w, n_layers=args.layers, name=f"{w.name}_{args.layers}l")
-    n_q = args.steps + args.warmup
     kern = {"auto": R.RESKV_DECODE_AUTO, "mma": R.RESKV_DECODE_MMA,
             "cluster": R.RESKV_DECODE_CLUSTER, "fma": R.RESKV_DECODE_FMA,
             "lse": R.RESKV_DECODE_LSE_MERGE}[args.decode_kernel]
     bmode = R.RESKV_BUDGET_ADAKV if args.budget_mode == "adakv" else R.RESKV_BUDGET_UNIFORM
-    cache, Qdec, build_s = build_workload(w, n_q, device, kern, bmode)
-    info = R.reskv_get_info(cache)
-    unit_budgets = R.reskv_get_unit_budgets(cache)
-
-    def plan_name(cs, wpc):
-        if kern == R.RESKV_DECODE_LSE_MERGE:
-            return "paper-style: main pass + residual pass + log-sum-exp merge (3 launches)"
-        if cs == 0:
-            return "fma" if kern == R.RESKV_DECODE_FMA else "tensor-core stream-K"
-        return f"tensor-core cluster: {cs} CTA(s) x {wpc} warps per unit"
-
-    decode_plan = {"all_layer": plan_name(info["all_cluster"], info["all_cluster_warps"]),
-                   "per_layer": plan_name(info["layer_cluster"], info["layer_cluster_warps"])}
-    lay_meta = R.reskv_export_cache(cache)
-    alg = algorithmic_bytes(lay_meta["n_main"], lay_meta["n_res"])
-    r_counts = lay_meta["n_res"]
-    del lay_meta
-    O = torch.empty((w.n_layers, w.batch, w.n_q_heads, w.head_dim), dtype=torch.float32,
-                    device=device)
-    stream = torch.cuda.current_stream(device)
-
-    # ---- device-resident timing: K steps, one launch each ----
-    for i in range(args.warmup):
-        R.reskv_decode_attn(cache, -1, Qdec[i], O)
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with ClockSampler(local) as clk:
-        barrier(world)
-        torch.cuda.synchronize()
-        e0.record(stream)
-        for i in range(args.steps):
-            R.reskv_decode_attn(cache, -1, Qdec[args.warmup + i], O)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        barrier(world)
-    t_local = e0.elapsed_time(e1) / 1e3
-    t = reduce_max(t_local, world, device)
-    R.reskv_check_status(cache)
-    ms_step = t * 1e3 / args.steps
-    value = aggregate(w.batch * args.steps, t, world)
-    launch_s = t_local / args.steps                      # one launch per step
     peak, peak_kind = measured_peak_gbs()
-    achieved = alg / launch_s / 1e9
-    # Q (bf16) read and O (fp32) written by the step: necessary traffic outside
-    # the algorithmic cache bytes (1 KB + 2 KB per unit: 0.6 % of the bytes at
-    # b = 1024, 4.7 % at b = 128)
-    qo_bytes = int(w.n_units * w.group * w.head_dim * (2 + 4))
 
-    # ---- per-layer calls (one launch per layer) captured in a CUDA graph ----
-    per_layer = None
-    if not args.no_per_layer:
-        Ql = [Qdec[0, l].contiguous() for l in range(w.n_layers)]
-        Ol = [O[l] for l in range(w.n_layers)]
-        g_stream = torch.cuda.Stream(device)
-        g_stream.wait_stream(stream)
-        with torch.cuda.stream(g_stream):
-            for l in range(w.n_layers):                      # warm, outside capture
-                R.reskv_decode_attn(cache, l, Ql[l], Ol[l], stream=g_stream)
-            graph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(graph, stream=g_stream):
-                for l in range(w.n_layers):
-                    R.reskv_decode_attn(cache, l, Ql[l], Ol[l], stream=g_stream)
-        stream.wait_stream(g_stream)
-        for _ in range(args.warmup):
-            graph.replay()
-        torch.cuda.synchronize()
-        reps = max(10, args.steps // 4)
-        e0.record(stream)
-        for _ in range(reps):
-            graph.replay()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        tg = e0.elapsed_time(e1) / 1e3 / reps
-        per_layer = {"us_per_step": tg * 1e6, "us_per_layer_step": tg * 1e6 / w.n_layers,
-                     "tokens_per_s": w.batch / tg, "gbs": alg / tg / 1e9,
-                     "frac_of_peak": alg / tg / 1e9 / peak,
-                     "how": f"{w.n_layers} per-layer reskv_decode_attn launches replayed as one "
-                            f"CUDA graph, {reps} replays"}
-        units_layer = w.batch * w.n_kv_heads
-        per_layer["roofline"] = {
-            "bound": "hbm", "achieved": alg / tg / 1e9, "peak": peak, "unit": "GB/s",
-            "frac": alg / tg / 1e9 / peak, "kernel": decode_plan["per_layer"],
-            "traffic": (profiled_traffic(units_layer, PROFILE_LAYER, KERNEL_SOURCES_LAYER)
-                        if info["layer_cluster"] > 0 and not info["ragged"] else None),
-            "algorithmic_bytes_per_launch": alg // w.n_layers}
-        del graph
-
-    # ---- end to end through the C ABI with host buffers ----
-    # reskv_decode_attn_host with page-locked host Q and O: the decode kernel
-    # reads each unit's queries from host memory and writes its outputs there
-    # (over the host link, overlapped with streaming the cache); the host
-    # waits for every step.
-    Qh = Qdec[:min(n_q, 64)].cpu().pin_memory()
-    Oh = torch.empty(O.shape, dtype=torch.float32).pin_memory()
-    # every step synchronises the host: time as many steps as the device leg,
-    # so that one host hiccup weighs little
-    e2e_steps = args.steps
-    stream = torch.cuda.current_stream()
-    for i in range(max(3, args.warmup)):
-        R.reskv_decode_attn_host(cache, Qh[i % Qh.shape[0]], Oh, stream=stream)
-        stream.synchronize()
-    stream.synchronize()
-    barrier(world)
-    t0 = time.perf_counter()
-    for i in range(e2e_steps):
-        R.reskv_decode_attn_host(cache, Qh[i % Qh.shape[0]], Oh, stream=stream)
-        stream.synchronize()
-    te = reduce_max(time.perf_counter() - t0, world, device)
-    e2e = {"value": aggregate(w.batch * e2e_steps, te, world), "unit": "tokens/s",
-           "h2d_bytes_per_step": int(Qh[0].numel() * 2), "d2h_bytes_per_step": int(Oh.numel() * 4),
-           "how": "reskv_decode_attn_host on pinned host Q and O: the decode launch reads Q "
-                  "from and writes O to host memory (NVLink-C2C), host waits every step"}
+    # clocks are sampled around the timed region of the step
+    clk = ClockSampler(local)
+    main_rec = measure(args, w, R, kern, bmode, device, world, peak, peak_kind, clk=clk)
+    clocks = clk.summary()
+    second = None
+    if args.second_workload != "none" and not args.layers:
+        w2 = wl.WORKLOADS[args.second_workload]
+        clk2 = ClockSampler(local)
+        second = measure(args, w2, R, kern, bmode, device, world, peak, peak_kind, clk=clk2,
+                         with_e2e=False)
+        second["clocks"] = clk2.summary()
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w)
 
     if rank == 0:
-        units_launch = w.n_units
+        pl = main_rec["per_layer"]
         line = {
-            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+            "metric": METRIC, "value": pl["tokens_per_s"], "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": pl["us_per_step"] / 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
-            "config": {"workload": w.name, "layers": w.n_layers, "batch": w.batch,
-                       "kv_heads": w.n_kv_heads, "q_heads": w.n_q_heads, "head_dim": w.head_dim,
-                       "seq_len": w.seq_len, "budget": w.budget, "residual": w.residual,
-                       "mean_r": float(np.mean(r_counts)),
-                       "units_with_residual": float(np.mean(r_counts > 0)),
-                       "budget_mode": args.budget_mode,
-                       "unit_budget_min_max": [int(unit_budgets.min()), int(unit_budgets.max())],
-                       "launch": "one reskv_decode_attn(layer=-1) launch per step",
-                       "decode_plan": decode_plan,
-                       "l2": f"inputs larger than L2: {alg / 1e9:.2f} GB of cache read per step",
-                       "parallelism": "replicas" if world > 1 else "single GPU"},
-            "hbm_gbs": achieved, "frac_of_peak": achieved / peak,
-            "q_o_bytes_per_step": qo_bytes,
-            "hbm_gbs_with_q_o": (alg + qo_bytes) / launch_s / 1e9,
-            "frac_of_nominal_8tbs": achieved / 8000.0,
-            "us_per_layer_step": ms_step * 1e3 / w.n_layers,
-            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak,
-                         # the summaries were captured on one-budget layouts
-                         "traffic": None if info["ragged"] else profiled_traffic(units_launch),
-                         "peak_kind": f"{peak_kind} (burst copy)",
-                         "algorithmic_bytes_per_launch": alg},
-            "per_layer_graph": per_layer,
-            "construction_s": build_s,
-            "construction_stages_ms": dict(zip(
-                ["scores", "ranking", "validation_targets", "lloyd", "validation_loss_and_choice",
-                 "pack"], [round(x, 3) for x in info["build_ms"]])),
-            "construction_tflops": {
-                k: round(f / (info["build_ms"][i] * 1e-3) / 1e12, 2)
-                for k, i in (("scores", 0), ("validation_targets", 2), ("lloyd", 3))
-                for f in [construction_flops(w).get(k)] if f and info["build_ms"][i] > 0},
-            "e2e": e2e,
-            "clocks": clk.summary(),
-            "gpu_launches": args.steps * (3 if kern == R.RESKV_DECODE_LSE_MERGE else 1),
+            "config": dict(main_rec["config"], **{
+                "budget_mode": args.budget_mode,
+                "launch": f"one reskv_decode_attn(layer) launch per layer, {w.n_layers} per step, "
+                          f"in one CUDA graph",
+                "parallelism": "replicas" if world > 1 else "single GPU"}),
+            "us_per_layer_step": pl["us_per_layer_step"],
+            "roofline": pl["roofline"],
+            "all_layer_launch": main_rec["all_layer"],
+            "construction_s": main_rec["construction_s"],
+            "construction_stages_ms": main_rec["construction_stages_ms"],
+            "construction_tflops": main_rec["construction_tflops"],
+            "e2e": main_rec["e2e"],
+            "clocks": clocks,
+            "gpu_launches": args.steps * main_rec["launches_per_step"],
             "cpu_baseline": cpu,
         }
+        if second is not None:
+            line["second_workload"] = {
+                "config": second["config"], "per_layer": second["per_layer"],
+                "all_layer_launch": second["all_layer"], "construction_s": second["construction_s"],
+                "construction_stages_ms": second["construction_stages_ms"],
+                "clocks": second["clocks"], "steps": args.steps, "warmup": args.warmup}
         print(json.dumps(line), flush=True)
-    cache.free()
 
 
 if __name__ == "__main__":

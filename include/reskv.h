@@ -71,6 +71,21 @@ enum { RESKV_DECODE_AUTO = 0, RESKV_DECODE_FMA = 1, RESKV_DECODE_MMA = 2, RESKV_
  * and every head keeps `budget`. */
 enum { RESKV_BUDGET_UNIFORM = 0, RESKV_BUDGET_ADAKV = 1 };
 
+/* What reskv_append does when a unit's append_capacity slots are taken.
+ * RESKV_APPEND_FAIL: the call fails (RESKV_ERR_UNSUPPORTED, nothing written).
+ * RESKV_APPEND_RING_DROP, RESKV_APPEND_RING_FOLD: the A appended slots are a
+ * ring of the unit's A most recent tokens; the oldest leaves the exact window
+ * to make room.  DROP: it leaves the cache.  FOLD: it becomes a member of its
+ * nearest residual entry (least squared distance between keys, decided
+ * exactly, ties to the lower entry; the nearest-centre rule of Eq.
+ * residual_partition) whose stored means and count are updated as a running
+ * mean (Eq. summary): k_bar <- (c k_bar + k) / (c + 1) and v_bar likewise,
+ * evaluated in fp64 and stored in bf16 (round to nearest even), c <- c + 1,
+ * log-count beta ln(c + 1); a unit without residual entries drops it.  The
+ * paper leaves refreshing residual entries during generation to future work
+ * (App. E); this is the reading built. */
+enum { RESKV_APPEND_FAIL = 0, RESKV_APPEND_RING_DROP = 1, RESKV_APPEND_RING_FOLD = 2 };
+
 #define RESKV_MAX_GRID 8
 
 /*
@@ -138,6 +153,8 @@ typedef struct reskv_config {
                               it).  The built layout is ragged: read the
                               budgets with reskv_get_unit_budgets            */
   float adakv_safeguard;   /* AdaKV safeguard coefficient in [0, 1] (0.2)    */
+  int32_t append_policy;   /* RESKV_APPEND_* (reskv_config_default:
+                              RESKV_APPEND_RING_FOLD)                        */
 } reskv_config;
 
 /* Fill *cfg with the paper's defaults; shape fields are zeroed. */
@@ -310,19 +327,24 @@ reskv_status reskv_export_cache(const reskv_cache* c, reskv_host_cache* h, void*
 
 /*
  * Append the newest decoded token to the cache: one exact K row and V row per
- * (batch, KV head) unit of `layer`, after the unit's main and residual slots
- * (Sec. 3.1: each decode step appends the new token's key and value; Alg. 2
- * attends over the cache as it stands).  Appended tokens are main-cache tokens
- * for every later decode: exact rows in the shared softmax, counted in p_max of
- * the gate.  Residual entries are not refreshed (the paper leaves residual
- * updates during generation to future work, App. E).
+ * (batch, KV head) unit of `layer`, into the unit's append_capacity slots after
+ * its main and residual slots (Sec. 3.1: each decode step appends the new
+ * token's key and value; Alg. 2 attends over the cache as it stands).
+ * Appended tokens are main-cache tokens for every later decode: exact rows in
+ * the shared softmax, counted in p_max of the gate.  When the slots are taken,
+ * cfg.append_policy decides (RESKV_APPEND_*): refuse, or drop the oldest
+ * appended token, or fold it into its nearest residual entry.  The slots then
+ * hold the A most recent tokens in ring order (reskv_export_cache gives each
+ * its position; an imported cache's appended rows count as appended in slot
+ * order).
  *
  *   layer in [0, L) : K_new, V_new device bf16 [B, H_kv, d]
  *   layer == -1     : every layer, K_new, V_new [L, B, H_kv, d]
  *
- * RESKV_ERR_UNSUPPORTED (nothing written) when a unit of the call has
- * append_capacity tokens already.  The rows are complete when the stream
- * reaches the next call on it.
+ * RESKV_ERR_UNSUPPORTED (nothing written) when append_capacity is 0, or when a
+ * unit of the call has append_capacity tokens already under
+ * RESKV_APPEND_FAIL.  The rows are complete when the stream reaches the next
+ * call on it.
  */
 reskv_status reskv_append(reskv_cache* c, int32_t layer, const void* K_new, const void* V_new,
                           void* stream);
@@ -352,6 +374,24 @@ reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_d
                                 size_t bytes);
 
 /*
+ * Fault injection, for testing the failure paths without faulting a GPU (no
+ * counterpart in the paper).  Process-wide; takes effect on the next calls:
+ *   RESKV_TEST_FAIL_FIRST_WAIT, n >= 0: the next n decode launches (any decode
+ *     entry point) run with every warp giving up its first ring wait as if
+ *     the wait's bound had run out: the kernel sets its status word (code 1),
+ *     waits for its own copies in flight and returns with the output
+ *     incomplete.  The handle's partial-result tickets are then not reset:
+ *     free the handle after reskv_check_status reports the fault.
+ *   RESKV_TEST_FAIL_ALLOC, n >= 1: the n-th device allocation of the library
+ *     from now on fails as cudaMalloc out of memory would (nothing is
+ *     allocated for it; the call returns RESKV_ERR_OOM and frees what it had
+ *     allocated).  n = 0 cancels.
+ * RESKV_ERR_INVALID_ARG for another `what` or n < 0.
+ */
+enum { RESKV_TEST_FAIL_FIRST_WAIT = 1, RESKV_TEST_FAIL_ALLOC = 2 };
+reskv_status reskv_test_inject(int32_t what, int64_t n);
+
+/*
  * Decode that allocates nothing.  The paper has no counterpart: this entry
  * point exists for callers that cannot allocate device memory at decode time
  * -- code running inside a host application whose memory manager owns every
@@ -368,11 +408,14 @@ reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_d
  * (one layer at a time) in that case.  Roughly, a call needs
  * (n_units + 8 * SMs) * 2 * group * 528 bytes plus 4 bytes per unit.
  *
- * The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress, with that device current); make that first call
- * before any stream capture.  Every call shares the array and clears the
- * parts that must start at zero, so calls that overlap on the GPU race: order
- * them on one stream (or synchronise between them).
+ * Every call looks up the array's device address (cudaGetSymbolAddress, with
+ * the caller's device current; it allocates nothing).  The first call on a
+ * device may also load the library's device code, so make it before any
+ * stream capture.  Every call shares the array and clears the parts that must
+ * start at zero, so calls that overlap on the GPU race: order them on one
+ * stream (or synchronise between them).  A kernel fault (a bounded wait that
+ * gave up, leaving O partly unwritten, or an index out of range) is ORed into
+ * a device status word that only reskv_noalloc_check_status reads and clears.
  *
  * The cache has no appended tokens (budget here is the unit stride).
  *   kslots, vslots : device bf16 [n_units, budget, 128], 16-byte aligned
@@ -404,6 +447,21 @@ typedef struct reskv_device_cache {
 
 reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, const void* Q, void* O,
                                        void* stream);
+
+/*
+ * Status of the no-allocation decode (no counterpart in the paper; it
+ * allocates nothing either).  Synchronises `stream`, reads the current
+ * device's status word of reskv_decode_attn_noalloc -- the codes of every
+ * kernel fault since the last check, ORed together -- and clears it.
+ * RESKV_ERR_DEVICE_STATUS when a fault was recorded (the message names the
+ * codes: 1 = bounded wait timed out, 2 = index out of range), else RESKV_OK.
+ * last_kernel (may be NULL) receives the kernel that the calling thread's
+ * last successful reskv_decode_attn_noalloc launched: RESKV_DECODE_MMA (the
+ * tensor-core stream-K kernel) or RESKV_DECODE_FMA (the CUDA-core kernel,
+ * taken when budget is not a multiple of 16 or logc is not 16-byte aligned);
+ * 0 before the first call.
+ */
+reskv_status reskv_noalloc_check_status(void* stream, int32_t* last_kernel);
 
 #ifdef __cplusplus
 }

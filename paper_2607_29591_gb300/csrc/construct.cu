@@ -36,7 +36,7 @@ struct Scratch {
   bool get(T** p, size_t count) {
     *p = nullptr;
     if (count == 0) count = 1;
-    if (cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T)) != cudaSuccess) {
+    if (device_alloc(reinterpret_cast<void**>(p), count * sizeof(T)) != cudaSuccess) {
       cudaGetLastError();
       *p = nullptr;
       return false;
@@ -319,9 +319,10 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
          S.get(&rowerr, size_t(UL) * n_val_rows) && S.get(&losses, size_t(UL) * ncol);
   if (ok && cfg.keep_debug) {
     const size_t U = size_t(c->n_units);
-    cudaError_t e = cudaMalloc(&c->dbg_scores, U * size_t(s) * 8);
-    if (e == cudaSuccess) e = cudaMalloc(&c->dbg_ranked, U * std::max(n_top, 1) * 4);
-    if (e == cudaSuccess) e = cudaMalloc(&c->dbg_losses, U * ncol * 8);
+    cudaError_t e = device_alloc(reinterpret_cast<void**>(&c->dbg_scores), U * size_t(s) * 8);
+    if (e == cudaSuccess)
+      e = device_alloc(reinterpret_cast<void**>(&c->dbg_ranked), U * std::max(n_top, 1) * 4);
+    if (e == cudaSuccess) e = device_alloc(reinterpret_cast<void**>(&c->dbg_losses), U * ncol * 8);
     if (e == cudaSuccess) e = cudaMemsetAsync(c->dbg_losses, 0, U * ncol * 8, stream);
     ok = e == cudaSuccess;
     c->dbg_n_top = n_top;
@@ -377,7 +378,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       k_obs_pass2<<<dim3(ntiles, UL), kThreads, sm_obs2, stream>>>(oa);
       k_pool<<<unsigned(cdiv(int64_t(US), 256)), 256, 0, stream>>>(A, scores, s, UL, cfg.pool_kernel);
     } else {
-      k_score_keynorm<<<unsigned(cdiv(int64_t(US), 256)), 256, 0, stream>>>(K, scores, int64_t(US));
+      k_score_keynorm<<<unsigned(cdiv(int64_t(US), 8)), 256, 0, stream>>>(K, scores, int64_t(US));
     }
     RESKV_LAUNCH_CHECK("scoring");
     timing_ok &= timer.mark(kStRank);

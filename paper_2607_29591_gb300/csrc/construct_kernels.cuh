@@ -331,23 +331,130 @@ __global__ void k_pool(const float* A, double* scores, int64_t s, int UL, int po
   scores[i] = acc / double(pool);
 }
 
-// Query-free score ||k_p||^2, summed in fp64 over dims in order (no FMA).
+// Query-free score ||k_p||^2 (a build choice; the paper defines none): the
+// exact sum of the squares, rounded once to the nearest fp64 value (ties to
+// even), so it does not depend on any summation order.
+//
+// A bf16 value is M 2^e with an integer M < 2^8 (M = 128 + mantissa field for
+// normal values, the mantissa field for subnormals), so its square is
+// M^2 2^t with M^2 < 2^16 and t = 2e even, t in [-266, 242].  One warp per
+// row, four dims per lane.  With tmax the largest t of the row's nonzero
+// squares, every square with t >= tmax - 104 is an exact integer multiple of
+// 2^(tmax - 104) below 2^120, and 128 of them sum below 2^127: the warp adds
+// them as 128-bit integers and one lane rounds the sum.  A row with a
+// nonzero square below that window (its values span more than 52 binades)
+// goes to an exact 576-bit accumulator in one lane.
+
+using u128 = unsigned __int128;
+
+// Correctly rounded fp64 value of a 2^base, a > 0; `sticky`: a positive
+// amount below a's last bit is to be added as well.
+__device__ inline double round_u128(u128 a, int base, bool sticky) {
+  const uint64_t hi = uint64_t(a >> 64), lo = uint64_t(a);
+  const int p = hi ? 127 - __clzll((long long)hi) : 63 - __clzll((long long)lo);
+  if (p <= 52) return ldexp(double(lo), base);            // exact (sticky never set here)
+  const int sh = p - 52;
+  uint64_t mant = uint64_t(a >> sh);
+  const u128 one = 1;
+  const u128 rem = a & ((one << sh) - 1), half = one << (sh - 1);
+  if (rem > half || (rem == half && (sticky || (mant & 1u)))) ++mant;
+  return ldexp(double(mant), base + sh);
+}
+
+// The square of one bf16 value as (M^2, t); M^2 = 0 for zero.
+__device__ inline void bf16_square(uint32_t b, uint32_t& m2, int& t, bool& finite) {
+  const uint32_t ef = (b >> 7) & 0xffu, mf = b & 0x7fu;
+  const uint32_t M = ef ? 128u + mf : mf;
+  m2 = M * M;
+  t = 2 * (int(ef ? ef : 1u) - 134);
+  finite = ef != 0xffu;
+}
+
+// Exact sum of a row's squares in 32-bit digits (bit q = t + 266 of the sum
+// in digit q / 32), then the correctly rounded fp64 value.  One thread.
+__device__ double keynorm_wide(const __nv_bfloat16* rowp) {
+  const uint16_t* bits = reinterpret_cast<const uint16_t*>(rowp);
+  uint64_t dig[18];
+#pragma unroll
+  for (int j = 0; j < 18; ++j) dig[j] = 0;
+  for (int i = 0; i < kHeadDim; ++i) {
+    uint32_t m2;
+    int t;
+    bool fin;
+    bf16_square(bits[i], m2, t, fin);
+    if (!m2) continue;
+    const int q = t + 266;
+    const uint64_t v = uint64_t(m2) << (q & 31);
+    dig[q >> 5] += v & 0xffffffffu;
+    dig[(q >> 5) + 1] += v >> 32;
+  }
+  for (int j = 0; j < 17; ++j) {
+    dig[j + 1] += dig[j] >> 32;
+    dig[j] &= 0xffffffffu;
+  }
+  int top = 17;
+  while (top > 0 && dig[top] == 0) --top;
+  u128 a = 0;
+  for (int j = top; j > top - 4; --j) a = (a << 32) | (j >= 0 ? dig[j] : 0u);
+  bool sticky = false;
+  for (int j = 0; j < top - 3; ++j) sticky |= dig[j] != 0;
+  return a ? round_u128(a, (top - 3) * 32 - 266, sticky) : 0.0;
+}
+
+// One warp per row; the grid covers n_rows warps (blockDim a multiple of 32).
 __global__ void k_score_keynorm(const __nv_bfloat16* K, double* scores, int64_t n_rows) {
-  const int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (i >= n_rows) return;
-  const uint4* row = reinterpret_cast<const uint4*>(K + i * kHeadDim);
-  double acc = 0.0;
-  for (int c = 0; c < 16; ++c) {
-    const uint4 w = __ldg(row + c);
-    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+  const int64_t row = (int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= n_rows) return;                              // whole warps leave together
+  const uint2 w = __ldg(reinterpret_cast<const uint2*>(K + row * kHeadDim) + lane);
+  const uint32_t b[4] = {w.x & 0xffffu, w.x >> 16, w.y & 0xffffu, w.y >> 16};
+  uint32_t m2[4];
+  int t[4];
+  bool finite = true;
+  int tmax = INT_MIN;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    bool f;
+    bf16_square(b[j], m2[j], t[j], f);
+    finite &= f;
+    if (m2[j]) tmax = max(tmax, t[j]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) tmax = max(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
+  if (!__all_sync(0xffffffffu, finite)) {                 // inf or NaN: the fp64 sum is too
+    double acc = 0.0;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const float2 f = bf16x2_to_float2(ws[j]);
-      acc = __dadd_rn(acc, __dmul_rn(double(f.x), double(f.x)));
-      acc = __dadd_rn(acc, __dmul_rn(double(f.y), double(f.y)));
+      const double x = double(__uint_as_float(b[j] << 16));
+      acc += x * x;
     }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) scores[row] = acc;
+    return;
   }
-  scores[i] = acc;
+  if (tmax == INT_MIN) {                                  // every value is zero
+    if (lane == 0) scores[row] = 0.0;
+    return;
+  }
+  bool wide = false;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) wide |= m2[j] != 0 && t[j] < tmax - 104;
+  if (__any_sync(0xffffffffu, wide)) {
+    if (lane == 0) scores[row] = keynorm_wide(K + row * kHeadDim);
+    return;
+  }
+  u128 a = 0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    if (m2[j]) a += u128(m2[j]) << (t[j] - tmax + 104);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint64_t hi = __shfl_xor_sync(0xffffffffu, uint64_t(a >> 64), o);
+    const uint64_t lo = __shfl_xor_sync(0xffffffffu, uint64_t(a), o);
+    a += (u128(hi) << 64) | lo;
+  }
+  if (lane == 0) scores[row] = round_u128(a, tmax - 104, false);
 }
 
 // ---------------------------------------------------------------------------

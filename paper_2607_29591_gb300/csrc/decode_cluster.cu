@@ -102,6 +102,72 @@ __device__ __forceinline__ void st_cluster(uint32_t local, uint32_t rank, float4
 enum : int { kFused = 0, kMainBranch = 1, kResBranch = 2 };
 constexpr int kBrRec = kHeadDim + 4;    // branch record: m, l, pad, pad, o[d]
 
+// Step 3 of the cluster kernel, in rank 0: merge the n <= CS CTA records
+// (crec, [CS][2 branches][G heads][kRec]) in rank order, apply the gate and
+// write o^ (or, on a branch pass, the branch record).  One thread per two dims
+// of one head: every thread of the CTA takes part, and with CS equal to the
+// cluster size no record is read twice.
+template <int G, int kMode, int CS>
+__device__ __forceinline__ void rank0_merge(const DecodeParams& p, const float* crec,
+                                            int64_t orow0, int n) {
+  for (int idx = threadIdx.x; idx < G * (kHeadDim / 2); idx += blockDim.x) {
+    const int hh = idx / (kHeadDim / 2), d2 = 2 * (idx % (kHeadDim / 2));
+    float4 ml[2][CS];
+    float2 ac[2][CS];
+#pragma unroll
+    for (int sg = 0; sg < 2; ++sg)
+#pragma unroll
+      for (int c = 0; c < CS; ++c) {
+        const int cc = c < n ? c : 0;
+        const float* r = crec + cc * kCtaRecFloats + (sg * G + hh) * kRec;
+        ml[sg][c] = *reinterpret_cast<const float4*>(r);
+        ac[sg][c] = *reinterpret_cast<const float2*>(r + 4 + d2);
+      }
+    float Ms[2], Ls[2], Mt[2];
+    float2 As[2];
+#pragma unroll
+    for (int sg = 0; sg < 2; ++sg) {
+      float mx = -INFINITY, mt = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < CS; ++c)
+        if (c < n && ml[sg][c].y > 0.f) {
+          mx = fmaxf(mx, ml[sg][c].x);
+          mt = fmaxf(mt, ml[sg][c].z);
+        }
+      float l = 0.f;
+      float2 a = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int c = 0; c < CS; ++c)
+        if (c < n && ml[sg][c].y > 0.f) {
+          const float sc = exp2f(ml[sg][c].x - mx);
+          l += ml[sg][c].y * sc;
+          a.x += ac[sg][c].x * sc;
+          a.y += ac[sg][c].y * sc;
+        }
+      Ms[sg] = mx;
+      Ls[sg] = l;
+      Mt[sg] = mt;
+      As[sg] = a;
+    }
+    if constexpr (kMode == kFused) {
+      const float2 w = branch_coefs(p.softmax_mode, gate_of(p, sum_rel_max(Ms[0], Ls[0], Mt[0])),
+                                    Ms[0], Ls[0], Ms[1], Ls[1]);
+      *reinterpret_cast<float2*>(p.O + (orow0 + hh) * kHeadDim + d2) =
+          make_float2(w.x * As[0].x + w.y * As[1].x, w.x * As[0].y + w.y * As[1].y);
+    } else {
+      constexpr int sg = kMode == kMainBranch ? 0 : 1;
+      const float inv = Ls[sg] > 0.f ? 1.0f / Ls[sg] : 0.f;
+      float* br = p.partials + (orow0 + hh) * kBrRec;
+      *reinterpret_cast<float2*>(br + 4 + d2) = make_float2(As[sg].x * inv, As[sg].y * inv);
+      // (m, l) relative to the branch's largest logit, as the merge's gate takes it
+      if (d2 == 0)
+        *reinterpret_cast<float2*>(br) =
+            Ls[sg] > 0.f ? make_float2(Mt[sg], sum_rel_max(Ms[sg], Ls[sg], Mt[sg]))
+                         : make_float2(Ms[sg], Ls[sg]);
+    }
+  }
+}
+
 template <int G, int kMode>
 __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
     reskv_decode_cluster_kernel(const DecodeParams p, const __grid_constant__ CUtensorMap tmK,
@@ -161,9 +227,10 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   }
   __syncwarp();
 
+  const uint64_t pol = l2_evict_first_policy();
   auto issue = [&](int k, int s, bool with_logc) {   // lane 0: chunk k into stage s
     issue_stage(base + s * kStageBytes, logc_s + s * kCh, &tmK, &tmV, p.logc, wcb + k * kCh, p.kv_rank,
-                with_logc, &bars[s]);
+                with_logc, &bars[s], pol);
   };
   const int issued0 = nchunks < kSt ? nchunks : kSt;
   if (lane == 0)
@@ -201,7 +268,7 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   int s = 0;                            // stage of chunk k
   uint32_t phase = 0;                   // parity of its current use
   for (int k = 0; k < nchunks; ++k) {
-    if (!mbar_wait_bounded(&bars[s], phase)) {
+    if ((k == 0 && p.test_fault) || !mbar_wait_bounded(&bars[s], phase)) {
       if (lane == 0) report_status(p.status, kStatusWaitTimeout);
       break;
     }
@@ -293,65 +360,11 @@ __global__ void __launch_bounds__(kMmaMaxW * 32, 1)
   if (rank != 0) return;                 // nobody reads this CTA's shared memory
 
   // 3. rank 0: merge the CS CTA records in rank order, gate, write o^
-  for (int idx = threadIdx.x; idx < G * (kHeadDim / 4); idx += blockDim.x) {
-    const int hh = idx / (kHeadDim / 4), d4 = 4 * (idx % (kHeadDim / 4));
-    float4 ml[2][kMaxCluster];
-    float4 ac[2][kMaxCluster];
-#pragma unroll
-    for (int sg = 0; sg < 2; ++sg)
-#pragma unroll
-      for (int c = 0; c < kMaxCluster; ++c) {
-        const int cc = c < int(cs) ? c : 0;
-        const float* r = crec + cc * kCtaRecFloats + (sg * G + hh) * kRec;
-        ml[sg][c] = *reinterpret_cast<const float4*>(r);
-        ac[sg][c] = *reinterpret_cast<const float4*>(r + 4 + d4);
-      }
-    float Ms[2], Ls[2], Mt[2];
-    float4 As[2];
-#pragma unroll
-    for (int sg = 0; sg < 2; ++sg) {
-      float mx = -INFINITY, mt = -INFINITY;
-#pragma unroll
-      for (int c = 0; c < kMaxCluster; ++c)
-        if (c < int(cs) && ml[sg][c].y > 0.f) {
-          mx = fmaxf(mx, ml[sg][c].x);
-          mt = fmaxf(mt, ml[sg][c].z);
-        }
-      float l = 0.f;
-      float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int c = 0; c < kMaxCluster; ++c)
-        if (c < int(cs) && ml[sg][c].y > 0.f) {
-          const float sc = exp2f(ml[sg][c].x - mx);
-          l += ml[sg][c].y * sc;
-          a.x += ac[sg][c].x * sc;
-          a.y += ac[sg][c].y * sc;
-          a.z += ac[sg][c].z * sc;
-          a.w += ac[sg][c].w * sc;
-        }
-      Ms[sg] = mx;
-      Ls[sg] = l;
-      Mt[sg] = mt;
-      As[sg] = a;
-    }
-    if constexpr (kMode == kFused) {
-      const float2 w = branch_coefs(p.softmax_mode, gate_of(p, sum_rel_max(Ms[0], Ls[0], Mt[0])),
-                                    Ms[0], Ls[0], Ms[1], Ls[1]);
-      *reinterpret_cast<float4*>(p.O + (orow0 + hh) * kHeadDim + d4) =
-          make_float4(w.x * As[0].x + w.y * As[1].x, w.x * As[0].y + w.y * As[1].y,
-                      w.x * As[0].z + w.y * As[1].z, w.x * As[0].w + w.y * As[1].w);
-    } else {
-      constexpr int sg = kMode == kMainBranch ? 0 : 1;
-      const float inv = Ls[sg] > 0.f ? 1.0f / Ls[sg] : 0.f;
-      float* br = p.partials + (orow0 + hh) * kBrRec;
-      *reinterpret_cast<float4*>(br + 4 + d4) =
-          make_float4(As[sg].x * inv, As[sg].y * inv, As[sg].z * inv, As[sg].w * inv);
-      // (m, l) relative to the branch's largest logit, as the merge's gate takes it
-      if (d4 == 0)
-        *reinterpret_cast<float2*>(br) =
-            Ls[sg] > 0.f ? make_float2(Mt[sg], sum_rel_max(Ms[sg], Ls[sg], Mt[sg]))
-                         : make_float2(Ms[sg], Ls[sg]);
-    }
+  switch (cs) {
+    case 1: rank0_merge<G, kMode, 1>(p, crec, orow0, 1); break;
+    case 2: rank0_merge<G, kMode, 2>(p, crec, orow0, 2); break;
+    case 4: rank0_merge<G, kMode, 4>(p, crec, orow0, 4); break;
+    default: rank0_merge<G, kMode, kMaxCluster>(p, crec, orow0, int(cs)); break;
   }
 }
 

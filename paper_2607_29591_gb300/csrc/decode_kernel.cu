@@ -150,7 +150,8 @@ __global__ void __launch_bounds__(kDecodeWarpsPerCta * 32, 1)
   auto wait_upto = [&](int64_t k) {
     while (ready < k && !failed) {
       ++ready;
-      if (!mbar_wait_bounded(&full[ready % kStages], uint32_t((ready / kStages) & 1))) {
+      if ((ready == 0 && p.test_fault) ||
+          !mbar_wait_bounded(&full[ready % kStages], uint32_t((ready / kStages) & 1))) {
         failed = true;
         if (lane == 0) report_status(p.status, kStatusWaitTimeout);
       }

@@ -113,9 +113,10 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   }
   __syncwarp();
 
+  const uint64_t pol = l2_evict_first_policy();
   auto issue = [&](int k, int s, bool with_logc) {   // lane 0: chunk k into stage s
     issue_stage(base + s * kStageBytes, logc_s + s * kCh, &tmK, &tmV, p.logc, cb + k * kCh, p.kv_rank,
-                with_logc, &bars[s]);
+                with_logc, &bars[s], pol);
   };
   // the first ring goes out before the unit's counts are read: with log-counts
   if (lane == 0)
@@ -285,7 +286,7 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
   int s = 0;                                          // stage of chunk k
   uint32_t phase = 0;                                 // parity of its current use
   for (int k = 0; k < nchunks && !done; ++k) {
-    if (!mbar_wait_bounded(&bars[s], phase)) {
+    if ((k == 0 && p.test_fault) || !mbar_wait_bounded(&bars[s], phase)) {
       if (lane == 0) report_status(p.status, kStatusWaitTimeout);
       break;
     }
@@ -346,8 +347,10 @@ __global__ void __launch_bounds__(kMaxW * 32, 1)
     }
   }
   // never leave with a copy in flight into this warp's ring (bounded waits)
+  // or with query rows still arriving (after a timed-out wait)
   for (int kk = waited; kk < issued; ++kk)
     mbar_wait_bounded(&bars[kk % kSt], uint32_t((kk / kSt) & 1));
+  asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
 }  // namespace

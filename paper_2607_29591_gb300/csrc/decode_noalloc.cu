@@ -14,13 +14,19 @@
 // The array is file-scope device memory: every GPU on which the library's
 // code is loaded holds its 16 MiB until the process exits.  Host code cannot
 // use the array's name as a device address (on the host it names a stand-in
-// object), so the address is looked up with cudaGetSymbolAddress once per
-// device, with that device current, and handed to the kernel.
+// object), so every call looks the address up with cudaGetSymbolAddress, with
+// the caller's device current, and hands it to the kernel.  The lookup
+// allocates nothing; looking it up per call (rather than caching it) keeps it
+// right after a cudaDeviceReset, which reloads the module at a new address.
+//
+// The kernels' status word (a bounded wait that gave up, an index out of
+// range) is a separate device word that calls only OR into; it is read and
+// cleared by reskv_noalloc_check_status, so a fault of any call since the
+// last check is reported, not overwritten by the next call.
 #include <cuda_runtime.h>
 
 #include <cmath>
 #include <cstdint>
-#include <mutex>
 #include <string>
 
 #include "internal.h"
@@ -30,15 +36,18 @@ namespace reskv {
 namespace {
 
 constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;   // 16 MiB
-constexpr int kMaxDevices = 64;
 
 // Shared by every call of reskv_decode_attn_noalloc in the process; keeps the
 // contents of the last call.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-std::mutex g_setup_mutex;
-void* g_scratch_addr[kMaxDevices] = {};
-int g_num_sms[kMaxDevices] = {};
+// Kernel status of every call since the last reskv_noalloc_check_status on
+// this device (codes ORed together).
+static __device__ uint32_t g_noalloc_status;
+
+// The kernel the last successful call on this thread launched
+// (RESKV_DECODE_MMA or RESKV_DECODE_FMA; 0 before the first call).
+thread_local int32_t g_last_kernel = 0;
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
@@ -47,25 +56,26 @@ reskv_status fail(reskv_status st, const std::string& msg) {
   return st;
 }
 
-// Device address of the scratch array and the SM count of device `dev`
-// (current), looked up on the first call on that device.
-reskv_status setup_device(int dev, void** addr, int* num_sms) {
-  std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    cudaError_t err = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (err != cudaSuccess || !p)
-      return fail(RESKV_ERR_CUDA, std::string("cudaGetSymbolAddress of the static scratch: ") +
-                                      cudaGetErrorString(err));
-    int sms = 0;
-    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (err != cudaSuccess || sms < 1)
-      return fail(RESKV_ERR_CUDA, std::string("reading the SM count: ") + cudaGetErrorString(err));
-    g_num_sms[dev] = sms;
-    g_scratch_addr[dev] = p;
-  }
-  *addr = g_scratch_addr[dev];
-  *num_sms = g_num_sms[dev];
+// Device addresses of the scratch array and the status word and the SM count
+// of the current device `dev`.
+reskv_status setup_device(int dev, void** addr, uint32_t** status, int* num_sms) {
+  void* p = nullptr;
+  cudaError_t err = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (err != cudaSuccess || !p)
+    return fail(RESKV_ERR_CUDA, std::string("cudaGetSymbolAddress of the static scratch: ") +
+                                    cudaGetErrorString(err));
+  void* w = nullptr;
+  err = cudaGetSymbolAddress(&w, g_noalloc_status);
+  if (err != cudaSuccess || !w)
+    return fail(RESKV_ERR_CUDA, std::string("cudaGetSymbolAddress of the status word: ") +
+                                    cudaGetErrorString(err));
+  int sms = 0;
+  err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (err != cudaSuccess || sms < 1)
+    return fail(RESKV_ERR_CUDA, std::string("reading the SM count: ") + cudaGetErrorString(err));
+  *addr = p;
+  *status = static_cast<uint32_t*>(w);
+  *num_sms = sms;
   return RESKV_OK;
 }
 
@@ -98,12 +108,12 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return fail(RESKV_ERR_CUDA, cudaGetErrorString(err));
-  if (dev < 0 || dev >= kMaxDevices) return fail(RESKV_ERR_UNSUPPORTED, "device ordinal >= 64");
 
   reskv_status st = RESKV_OK;
   void* scratch = nullptr;
+  uint32_t* status = nullptr;
   int num_sms = 0;
-  st = setup_device(dev, &scratch, &num_sms);
+  st = setup_device(dev, &scratch, &status, &num_sms);
   if (st != RESKV_OK) return st;
   const int64_t total = c->n_units * int64_t(c->budget);
   // The tensor-core stream-K kernel of reskv_decode_attn when its 16-slot
@@ -133,12 +143,11 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
     if (W < 1) W = 1;
   }
 
-  // scratch layout: [tickets: n_units int32][status word][partial records]
+  // scratch layout: [tickets: n_units int32][partial records]
   const size_t ticket_bytes = align256(size_t(c->n_units) * 4);
-  const size_t status_bytes = 256;
   const size_t part_bytes = (mma ? decode_mma_partials_floats(c->n_units, int(W), c->group)
                                  : decode_partials_floats(c->n_units, int(W), c->group)) * 4;
-  const size_t need = ticket_bytes + status_bytes + part_bytes;
+  const size_t need = ticket_bytes + part_bytes;
   if (need > kNoAllocScratchBytes)
     return fail(RESKV_ERR_UNSUPPORTED,
                 "this call needs " + std::to_string(need) + " bytes of scratch but the static "
@@ -147,8 +156,8 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
 
   unsigned char* base = static_cast<unsigned char*>(scratch);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // tickets and the status word must start at zero; the rest is overwritten
-  err = cudaMemsetAsync(base, 0, ticket_bytes + status_bytes, s);
+  // the tickets must start at zero; the partial records are overwritten
+  err = cudaMemsetAsync(base, 0, ticket_bytes, s);
   if (err != cudaSuccess) return fail(RESKV_ERR_CUDA, cudaGetErrorString(err));
 
   DecodeParams p{};
@@ -160,8 +169,9 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
   p.Q = static_cast<const __nv_bfloat16*>(Q);
   p.O = static_cast<float*>(O);
   p.tickets = reinterpret_cast<int32_t*>(base);
-  p.status = reinterpret_cast<uint32_t*>(base + ticket_bytes);
-  p.partials = reinterpret_cast<float*>(base + ticket_bytes + status_bytes);
+  p.status = status;
+  p.partials = reinterpret_cast<float*>(base + ticket_bytes);
+  p.test_fault = take_test_wait_fault() ? 1 : 0;
   p.unit0 = 0;
   p.n_units = int32_t(c->n_units);
   p.stride = c->budget;                 // no appended rows: the stride is the budget
@@ -187,5 +197,26 @@ extern "C" reskv_status reskv_decode_attn_noalloc(const reskv_device_cache* c, c
   }
   if (err != cudaSuccess) return fail(RESKV_ERR_CUDA, std::string("decode launch: ") +
                                                           cudaGetErrorString(err));
+  g_last_kernel = mma ? RESKV_DECODE_MMA : RESKV_DECODE_FMA;
   return RESKV_OK;
+}
+
+extern "C" reskv_status reskv_noalloc_check_status(void* stream, int32_t* last_kernel) {
+  if (last_kernel) *last_kernel = g_last_kernel;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint32_t word = 0;
+  cudaError_t err = cudaStreamSynchronize(s);
+  if (err == cudaSuccess) err = cudaMemcpyFromSymbolAsync(&word, g_noalloc_status, 4, 0,
+                                                          cudaMemcpyDeviceToHost, s);
+  if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+  if (err != cudaSuccess)
+    return fail(RESKV_ERR_CUDA, std::string("reading the status word: ") + cudaGetErrorString(err));
+  if (word == 0) return RESKV_OK;
+  const uint32_t zero = 0;
+  err = cudaMemcpyToSymbolAsync(g_noalloc_status, &zero, 4, 0, cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess) err = cudaStreamSynchronize(s);
+  if (err != cudaSuccess)
+    return fail(RESKV_ERR_CUDA, std::string("clearing the status word: ") + cudaGetErrorString(err));
+  return fail(RESKV_ERR_DEVICE_STATUS, "no-allocation decode status word " + std::to_string(word) +
+                                           " (1 = bounded wait timed out, 2 = index out of range)");
 }

@@ -61,6 +61,10 @@ struct DecodeParams {
                                 // range into n_warps equal pieces; k > 0 gives
                                 // warp w the whole units [w k, (w + 1) k) of the
                                 // launch instead (short units: no unit is cut)
+  // testing only (reskv_test_inject): nonzero makes every warp of the launch
+  // give up its first ring wait as if its bound had run out (status word
+  // set, copies in flight drained, output incomplete)
+  int32_t test_fault;
 };
 
 constexpr int kDecodeWarpsPerCta = 8;
@@ -94,6 +98,13 @@ constexpr int kDecodeChunk = 16;
 constexpr int kLogcPad = 16;
 
 void set_error(const std::string& msg);
+
+// Fault injection for tests (reskv_test_inject): whether the next decode
+// launch is to report a timed-out first wait (consumes one pending launch),
+// and every device allocation of the library, which fails as cudaMalloc out
+// of memory when an injected failure is due.
+bool take_test_wait_fault();
+cudaError_t device_alloc(void** p, size_t bytes);
 
 // Split plan of the tensor-core stream-K kernel for a launch of `n_units`
 // units holding `total_slots` slots (largest unit `max_unit_slots`): W warps,
@@ -148,6 +159,7 @@ struct reskv_cache {
   int32_t* n_main = nullptr;
   int32_t* n_res = nullptr;
   int32_t* n_app = nullptr;
+  int32_t* n_total = nullptr;   // [U] tokens appended since construction (ring order)
   int32_t* offsets = nullptr;   // [U+1]
   // decode workspace (device)
   float* partials = nullptr;

@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -19,6 +20,29 @@ namespace reskv {
 static thread_local std::string g_last_error;
 
 void set_error(const std::string& msg) { g_last_error = msg; }
+
+// reskv_test_inject state: decode launches still to fail their first wait;
+// allocations until the injected failure (0: none pending)
+static std::atomic<int64_t> g_wait_faults{0};
+static std::atomic<int64_t> g_alloc_countdown{0};
+
+bool take_test_wait_fault() {
+  int64_t n = g_wait_faults.load();
+  while (n > 0 && !g_wait_faults.compare_exchange_weak(n, n - 1)) {
+  }
+  return n > 0;
+}
+
+cudaError_t device_alloc(void** p, size_t bytes) {
+  int64_t n = g_alloc_countdown.load();
+  while (n > 0 && !g_alloc_countdown.compare_exchange_weak(n, n - 1)) {
+  }
+  if (n == 1) {                        // the injected failure: nothing allocated
+    *p = nullptr;
+    return cudaErrorMemoryAllocation;
+  }
+  return cudaMalloc(p, bytes);
+}
 
 // construction (construct.cu)
 reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
@@ -57,6 +81,9 @@ reskv_status validate_shape(const reskv_config* cfg) {
     return fail(RESKV_ERR_INVALID_ARG, "unknown decode_kernel");
   if (cfg->softmax_mode != RESKV_SOFTMAX_SHARED && cfg->softmax_mode != RESKV_SOFTMAX_SEPARATE)
     return fail(RESKV_ERR_INVALID_ARG, "unknown softmax_mode");
+  if (cfg->append_policy != RESKV_APPEND_FAIL && cfg->append_policy != RESKV_APPEND_RING_DROP &&
+      cfg->append_policy != RESKV_APPEND_RING_FOLD)
+    return fail(RESKV_ERR_INVALID_ARG, "unknown append_policy");
   if (cfg->append_capacity < 0 || cfg->append_capacity > (1 << 20))
     return fail(RESKV_ERR_INVALID_ARG, "append_capacity must be in [0, 2^20]");
   const int64_t n_units = int64_t(cfg->n_layers) * cfg->batch * cfg->n_kv_heads;
@@ -86,7 +113,7 @@ template <typename T>
 reskv_status dalloc(T** p, size_t count, const char* what) {
   *p = nullptr;
   if (count == 0) count = 1;
-  cudaError_t err = cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T));
+  cudaError_t err = device_alloc(reinterpret_cast<void**>(p), count * sizeof(T));
   if (err != cudaSuccess) {
     *p = nullptr;
     cudaGetLastError();
@@ -120,6 +147,7 @@ void free_handle(reskv_cache* c) {
   cudaFree(c->n_main);
   cudaFree(c->n_res);
   cudaFree(c->n_app);
+  cudaFree(c->n_total);
   cudaFree(c->offsets);
   cudaFree(c->partials);
   cudaFree(c->tickets);
@@ -205,6 +233,7 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
       (st = dalloc(&c->n_main, size_t(c->n_units), "n_main")) != RESKV_OK ||
       (st = dalloc(&c->n_res, size_t(c->n_units), "n_res")) != RESKV_OK ||
       (st = dalloc(&c->n_app, size_t(c->n_units), "n_app")) != RESKV_OK ||
+      (st = dalloc(&c->n_total, size_t(c->n_units), "appended token counts")) != RESKV_OK ||
       (c->ragged &&
        (st = dalloc(&c->offsets, size_t(c->n_units) + 1, "unit offsets")) != RESKV_OK) ||
       (st = dalloc(&c->partials,
@@ -223,6 +252,7 @@ reskv_status alloc_handle(const reskv_config& cfg, cudaStream_t stream, reskv_ca
   if (err == cudaSuccess) err = cudaMemsetAsync(c->slot_pos, 0xff, slots * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->counts, 0, slots * 4, stream);
   if (err == cudaSuccess) err = cudaMemsetAsync(c->n_app, 0, size_t(c->n_units) * 4, stream);
+  if (err == cudaSuccess) err = cudaMemsetAsync(c->n_total, 0, size_t(c->n_units) * 4, stream);
   if (err == cudaSuccess && c->ragged)
     err = cudaMemcpyAsync(c->offsets, c->h_offsets.data(), c->h_offsets.size() * 4,
                           cudaMemcpyHostToDevice, stream);
@@ -359,6 +389,7 @@ void reskv_config_default(reskv_config* cfg) {
   cfg->keep_debug = 0;
   cfg->budget_mode = RESKV_BUDGET_UNIFORM;
   cfg->adakv_safeguard = 0.2f;
+  cfg->append_policy = RESKV_APPEND_RING_FOLD;
 }
 
 const char* reskv_last_error(void) { return g_last_error.c_str(); }
@@ -415,6 +446,8 @@ reskv_status reskv_import_cache(const reskv_config* cfg, const reskv_host_cache*
     err = cudaMemcpyAsync(c->n_res, h->n_res, size_t(U) * 4, cudaMemcpyHostToDevice, s);
   if (err == cudaSuccess && h->n_app)
     err = cudaMemcpyAsync(c->n_app, h->n_app, size_t(U) * 4, cudaMemcpyHostToDevice, s);
+  if (err == cudaSuccess && h->n_app)      // imported appended rows: appended in slot order
+    err = cudaMemcpyAsync(c->n_total, c->n_app, size_t(U) * 4, cudaMemcpyDeviceToDevice, s);
   if (err == cudaSuccess && h->slot_pos)
     err = cudaMemcpyAsync(c->slot_pos, h->slot_pos, slots * 4, cudaMemcpyHostToDevice, s);
   if (err == cudaSuccess && h->counts)
@@ -452,17 +485,14 @@ reskv_status reskv_export_cache(const reskv_cache* c, reskv_host_cache* h, void*
   return RESKV_OK;
 }
 
-reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* Q, void* O,
-                               void* stream) {
-  if (!c) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
-  if (layer < -1 || layer >= c->cfg.n_layers)
-    return fail(RESKV_ERR_INVALID_ARG, "layer must be -1 or in [0, n_layers)");
-  return layer < 0 ? reskv_decode_attn_layers(c, 0, c->cfg.n_layers, Q, O, stream)
-                   : reskv_decode_attn_layers(c, layer, 1, Q, O, stream);
-}
+}  // extern "C"
 
-reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int32_t n_layers,
-                                      const void* Q, void* O, void* stream) {
+namespace reskv {
+namespace {
+
+// Alg. 2 for layers [layer0, layer0 + n_layers) in one launch.
+reskv_status decode_layers(const reskv_cache* c, int32_t layer0, int32_t n_layers,
+                           const void* Q, void* O, void* stream) {
   if (!c || !Q || !O) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
   const reskv_config& cfg = c->cfg;
   if (layer0 < 0 || n_layers < 1 || int64_t(layer0) + n_layers > cfg.n_layers)
@@ -499,6 +529,7 @@ reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int3
   p.alpha = cfg.alpha;
   p.g_min = cfg.g_min;
   p.g_fixed = cfg.g_fixed;
+  p.test_fault = take_test_wait_fault() ? 1 : 0;
   reskv_cache::ClusterPlan cp;
   if (n_layers == 1) {
     cp = c->cplan_layer;
@@ -566,6 +597,25 @@ reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int3
   return RESKV_OK;
 }
 
+}  // namespace
+}  // namespace reskv
+
+extern "C" {
+
+reskv_status reskv_decode_attn(const reskv_cache* c, int32_t layer, const void* Q, void* O,
+                               void* stream) {
+  if (!c) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
+  if (layer < -1 || layer >= c->cfg.n_layers)
+    return fail(RESKV_ERR_INVALID_ARG, "layer must be -1 or in [0, n_layers)");
+  return layer < 0 ? decode_layers(c, 0, c->cfg.n_layers, Q, O, stream)
+                   : decode_layers(c, layer, 1, Q, O, stream);
+}
+
+reskv_status reskv_decode_attn_layers(const reskv_cache* c, int32_t layer0, int32_t n_layers,
+                                      const void* Q, void* O, void* stream) {
+  return decode_layers(c, layer0, n_layers, Q, O, stream);
+}
+
 reskv_status reskv_append(reskv_cache* c, int32_t layer, const void* K_new, const void* V_new,
                           void* stream) {
   if (!c || !K_new || !V_new) return fail(RESKV_ERR_INVALID_ARG, "NULL argument");
@@ -575,18 +625,22 @@ reskv_status reskv_append(reskv_cache* c, int32_t layer, const void* K_new, cons
   if (!aligned16(K_new) || !aligned16(V_new))
     return fail(RESKV_ERR_INVALID_ARG, "K_new and V_new must be 16-byte aligned");
   const int l0 = layer < 0 ? 0 : layer, l1 = layer < 0 ? cfg.n_layers : layer + 1;
-  for (int l = l0; l < l1; ++l)
-    if (c->n_app_max[size_t(l)] >= c->append_capacity)
-      return fail(RESKV_ERR_UNSUPPORTED, "layer " + std::to_string(l) + ": the append region (" +
-                                             std::to_string(c->append_capacity) +
-                                             " slots per unit) is full");
+  if (c->append_capacity == 0)
+    return fail(RESKV_ERR_UNSUPPORTED, "the cache has no append region (append_capacity 0)");
+  if (cfg.append_policy == RESKV_APPEND_FAIL)
+    for (int l = l0; l < l1; ++l)
+      if (c->n_app_max[size_t(l)] >= c->append_capacity)
+        return fail(RESKV_ERR_UNSUPPORTED, "layer " + std::to_string(l) + ": the append region (" +
+                                               std::to_string(c->append_capacity) +
+                                               " slots per unit) is full");
   const int64_t per_layer = int64_t(cfg.batch) * cfg.n_kv_heads;
   cudaError_t err = launch_append(c, int64_t(l0) * per_layer, int64_t(l1 - l0) * per_layer,
                                   static_cast<const __nv_bfloat16*>(K_new),
                                   static_cast<const __nv_bfloat16*>(V_new),
                                   static_cast<cudaStream_t>(stream));
   if (err != cudaSuccess) return cuda_fail(err, "append launch");
-  for (int l = l0; l < l1; ++l) ++c->n_app_max[size_t(l)];
+  for (int l = l0; l < l1; ++l)
+    c->n_app_max[size_t(l)] = std::min(c->n_app_max[size_t(l)] + 1, c->append_capacity);
   return RESKV_OK;
 }
 
@@ -626,8 +680,8 @@ reskv_status reskv_decode_attn_host(const reskv_cache* c, const void* Q_host, vo
   if (!io.q) {
     void* q = nullptr;
     void* o = nullptr;
-    cudaError_t err = cudaMalloc(&q, q_bytes);
-    if (err == cudaSuccess) err = cudaMalloc(&o, o_bytes);
+    cudaError_t err = device_alloc(&q, q_bytes);
+    if (err == cudaSuccess) err = device_alloc(&o, o_bytes);
     if (err != cudaSuccess) {
       cudaGetLastError();
       cudaFree(q);
@@ -706,6 +760,15 @@ reskv_status reskv_get_info(const reskv_cache* c, reskv_cache_info* info) {
   info->kv_copy_rank = c->kv_rank;
   info->reserved0 = 0;
   return RESKV_OK;
+}
+
+reskv_status reskv_test_inject(int32_t what, int64_t n) {
+  if (n < 0) return fail(RESKV_ERR_INVALID_ARG, "n must be >= 0");
+  switch (what) {
+    case RESKV_TEST_FAIL_FIRST_WAIT: g_wait_faults.store(n); return RESKV_OK;
+    case RESKV_TEST_FAIL_ALLOC: g_alloc_countdown.store(n); return RESKV_OK;
+    default: return fail(RESKV_ERR_INVALID_ARG, "unknown fault to inject");
+  }
 }
 
 reskv_status reskv_get_unit_budgets(const reskv_cache* c, int32_t* host_budgets, int64_t n_units) {

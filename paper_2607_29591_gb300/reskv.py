@@ -29,6 +29,8 @@ RESKV_SOFTMAX_SHARED, RESKV_SOFTMAX_SEPARATE = 0, 1
 RESKV_DEBUG_SCORES, RESKV_DEBUG_RANKED, RESKV_DEBUG_LOSSES, RESKV_DEBUG_CANDIDATES = 0, 1, 2, 3
 RESKV_DEBUG_UNIT_CANDIDATES = 4
 RESKV_BUDGET_UNIFORM, RESKV_BUDGET_ADAKV = 0, 1
+RESKV_TEST_FAIL_FIRST_WAIT, RESKV_TEST_FAIL_ALLOC = 1, 2
+RESKV_APPEND_FAIL, RESKV_APPEND_RING_DROP, RESKV_APPEND_RING_FOLD = 0, 1, 2
 MAX_GRID = 8
 
 
@@ -54,6 +56,7 @@ class reskv_config(ctypes.Structure):
         ("softmax_mode", ctypes.c_int32), ("append_capacity", ctypes.c_int32),
         ("unit_budgets", ctypes.POINTER(ctypes.c_int32)),
         ("budget_mode", ctypes.c_int32), ("adakv_safeguard", ctypes.c_float),
+        ("append_policy", ctypes.c_int32),
     ]
 
 
@@ -131,6 +134,10 @@ def load_library():
     lib.reskv_append.restype = i32
     lib.reskv_decode_attn_noalloc.argtypes = [ctypes.POINTER(reskv_device_cache), vp, vp, vp]
     lib.reskv_decode_attn_noalloc.restype = i32
+    lib.reskv_noalloc_check_status.argtypes = [vp, ctypes.POINTER(ctypes.c_int32)]
+    lib.reskv_noalloc_check_status.restype = i32
+    lib.reskv_test_inject.argtypes = [i32, ctypes.c_int64]
+    lib.reskv_test_inject.restype = i32
     _lib = lib
     return lib
 
@@ -298,6 +305,12 @@ def reskv_append(cache: Cache, layer: int, K_new, V_new, stream=None) -> None:
                                        _dptr(V_new, "torch.bfloat16", "V_new"), _stream(stream)))
 
 
+def reskv_test_inject(what: int, n: int) -> None:
+    """Testing only: inject a decode wait timeout or an allocation failure
+    (see include/reskv.h)."""
+    _check(load_library().reskv_test_inject(int(what), int(n)))
+
+
 def reskv_free(cache: Cache) -> None:
     cache.free()
 
@@ -431,18 +444,42 @@ def reskv_decode_attn_noalloc(kslots, vslots, logc, n_main, n_res, n_kv_heads: i
     device allocation by the library (see include/reskv.h).
 
     kslots, vslots: bf16 [U, b, 128]; logc: float32 [U, b]; n_main, n_res:
-    int32 [U]; Q: bf16 [U / n_kv_heads, n_kv_heads * group, 128]; O: float32.
+    int32 [U]; Q: bf16 [U / n_kv_heads, n_kv_heads * group, 128]; O: float32,
+    Q's shape.  Every shape is checked here, before the call: the kernel reads
+    and writes inside these arrays by their sizes alone.
     """
+    if kslots.dim() != 3 or int(kslots.shape[2]) != 128:
+        raise ValueError(f"kslots must be [U, b, 128], got {tuple(kslots.shape)}")
     U, b = int(kslots.shape[0]), int(kslots.shape[1])
+    H, G = int(n_kv_heads), int(group)
+    if H < 1 or U % H != 0:
+        raise ValueError(f"n_units {U} is not a multiple of n_kv_heads {H}")
+    # row-major arrays of these many elements (any leading shape)
+    for name, t, n in (("vslots", vslots, U * b * 128), ("logc", logc, U * b),
+                       ("n_main", n_main, U), ("n_res", n_res, U),
+                       ("Q", Q, U * G * 128), ("O", O, U * G * 128)):
+        if t.numel() != n or (name in ("vslots", "Q", "O") and int(t.shape[-1]) != 128):
+            raise ValueError(f"{name} must hold {n} elements (rows of 128 for vslots, Q, O), "
+                             f"got shape {tuple(t.shape)}")
     d = reskv_device_cache(
         kslots=_dptr(kslots, "torch.bfloat16", "kslots").value,
         vslots=_dptr(vslots, "torch.bfloat16", "vslots").value,
         logc=_dptr(logc, "torch.float32", "logc").value,
         n_main=_dptr(n_main, "torch.int32", "n_main").value,
         n_res=_dptr(n_res, "torch.int32", "n_res").value,
-        n_units=U, budget=b, n_kv_heads=int(n_kv_heads), group=int(group),
+        n_units=U, budget=b, n_kv_heads=H, group=G,
         gate_mode=int(gate_mode), tau=tau, alpha=alpha, g_min=g_min, g_fixed=g_fixed)
     _check(load_library().reskv_decode_attn_noalloc(ctypes.byref(d),
                                                     _dptr(Q, "torch.bfloat16", "Q"),
                                                     _dptr(O, "torch.float32", "O"),
                                                     _stream(stream)))
+
+
+def reskv_noalloc_check_status(stream=None) -> int:
+    """Read and clear the no-allocation decode's device status word; raises
+    ReskvError (RESKV_ERR_DEVICE_STATUS) if a kernel fault was recorded.
+    Returns the kernel the thread's last call launched (RESKV_DECODE_MMA or
+    RESKV_DECODE_FMA, 0 before the first call)."""
+    k = ctypes.c_int32(0)
+    _check(load_library().reskv_noalloc_check_status(_stream(stream), ctypes.byref(k)))
+    return int(k.value)

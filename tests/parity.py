@@ -90,3 +90,86 @@ def decode_parity(cache, lay, ref_units, Ks, Qd, w, ocfg_of):
     return worst
 
 
+
+
+# ---------------------------------------------------------------------------
+# oracle construction in worker processes (full-size tests)
+# ---------------------------------------------------------------------------
+
+def stratified_units(w, n):
+    """n units spread over layers, batch elements and KV heads (all units if
+    the workload has at most n)."""
+    if n >= w.n_units:
+        return list(range(w.n_units))
+    out = []
+    for i in range(n):
+        l = (i * w.n_layers) // n
+        b = (i * 5 + i // 3) % w.batch
+        h = (i * 3 + i // w.n_kv_heads) % w.n_kv_heads
+        out.append((l * w.batch + b) * w.n_kv_heads + h)
+    return sorted(set(out))
+
+
+def input_digest(*tensors):
+    import hashlib
+    h = hashlib.sha256()
+    for t in tensors:
+        if t is not None:
+            h.update(t.contiguous().view(torch.int16).numpy().tobytes())
+    return h.hexdigest()
+
+
+def oracle_build_job(args):
+    """Worker: regenerate one unit's inputs on the CPU and run the oracle's
+    Alg. 1 on them.  Returns (unit, oracle cache, digest of the inputs)."""
+    from paper_2607_29591_gb300 import workloads as wl
+    name, u, delta, r_override = args
+    w = wl.WORKLOADS[name]
+    l, rem = divmod(u, w.batch * w.n_kv_heads)
+    b, h = divmod(rem, w.n_kv_heads)
+    Kc, Vc = wl.unit_kv(w, l, b, h, "cpu")
+    Qc = wl.unit_obs_queries(w, l, b, h, Kc, "cpu") if w.n_obs > 0 else None
+    oc = orc.OracleConfig(budget=w.budget, recent_window=w.recent_window, n_fit=w.n_fit,
+                          n_val=w.n_val, score_mode=w.score_mode, residual_override=r_override,
+                          delta=delta)
+    ref = orc.build_unit(bf16_to_f64(Kc), bf16_to_f64(Vc),
+                         None if Qc is None else bf16_to_f64(Qc), oc)
+    return u, ref, input_digest(Kc, Vc, Qc)
+
+
+def _single_thread():
+    torch.set_num_threads(1)
+
+
+def oracle_pool(n_jobs):
+    """Spawned worker processes (one BLAS thread each) for oracle builds."""
+    import concurrent.futures
+    import multiprocessing
+    import os
+    procs = max(1, min(n_jobs, os.cpu_count() or 1))
+    old = {k: os.environ.get(k) for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS",
+                                          "MKL_NUM_THREADS")}
+    for k in old:
+        os.environ[k] = "1"
+    try:
+        return concurrent.futures.ProcessPoolExecutor(
+            procs, mp_context=multiprocessing.get_context("spawn"), initializer=_single_thread)
+    finally:
+        for k, v in old.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+
+
+def r_margin(losses, delta):
+    """The oracle's deciding margin for r: the distance of L_r*/L_0 from the
+    threshold 1 - delta, and the relative gap between the two best L_r."""
+    rs = sorted(k for k in losses if k > 0)
+    if not rs:
+        return 1.0
+    best = min(rs, key=lambda r: (losses[r], r))
+    margin = abs(losses[best] / losses[0] - (1 - delta)) if losses[0] > 0 else 1.0
+    vals = sorted(losses[r] for r in rs)
+    gap = (vals[1] - vals[0]) / vals[0] if len(vals) > 1 and vals[0] > 0 else 1.0
+    return min(margin, gap)

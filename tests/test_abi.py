@@ -104,3 +104,53 @@ def test_host_validation_errors(lib):
         assert st == 1 and word in R.reskv_last_error() and out.value is None, field
         setattr(cfg, field, 0)
     lib.reskv_free(None)                       # NULL-safe
+
+
+def test_noalloc_binding_checks_every_shape(lib):
+    """The no-allocation decode's binding checks every array against the
+    shape the kernel will read and write, before any CUDA call: a short
+    vslots, logc, n_main, n_res, Q or O raises ValueError naming it."""
+    import torch
+    U, b, H, G = 16, 32, 4, 4
+    good = dict(kslots=torch.zeros((U, b, 128), dtype=torch.bfloat16),
+                vslots=torch.zeros((U, b, 128), dtype=torch.bfloat16),
+                logc=torch.zeros((U, b), dtype=torch.float32),
+                n_main=torch.ones(U, dtype=torch.int32), n_res=torch.zeros(U, dtype=torch.int32),
+                Q=torch.zeros((U // H, H * G, 128), dtype=torch.bfloat16),
+                O=torch.zeros((U // H, H * G, 128), dtype=torch.float32))
+
+    def call(**over):
+        a = dict(good, **over)
+        R.reskv_decode_attn_noalloc(a["kslots"], a["vslots"], a["logc"], a["n_main"], a["n_res"],
+                                    H, G, a["Q"], a["O"])
+
+    bad = {"vslots": torch.zeros((U, b - 1, 128), dtype=torch.bfloat16),
+           "logc": torch.zeros((U - 1, b), dtype=torch.float32),
+           "n_main": torch.ones(U - 1, dtype=torch.int32),
+           "n_res": torch.zeros(U + 1, dtype=torch.int32),
+           "Q": torch.zeros((U // H, H * G - 1, 128), dtype=torch.bfloat16),
+           "O": torch.zeros((U // H - 1, H * G, 128), dtype=torch.float32)}
+    for name, t in bad.items():
+        with pytest.raises(ValueError, match=name):
+            call(**{name: t})
+    with pytest.raises(ValueError, match="kslots"):
+        call(kslots=torch.zeros((U, b, 64), dtype=torch.bfloat16))
+    with pytest.raises(ValueError, match="multiple of n_kv_heads"):
+        R.reskv_decode_attn_noalloc(*(torch.zeros((U + 1, b, 128), dtype=torch.bfloat16),) * 2,
+                                    good["logc"], good["n_main"], good["n_res"], H, G, good["Q"],
+                                    good["O"])
+    # shapes right: only now the device check (these are host tensors)
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        call()
+
+
+def test_fault_injection_arguments_are_checked(lib):
+    """reskv_test_inject validates its arguments on the host (no GPU needed)."""
+    with pytest.raises(R.ReskvError) as e:
+        R.reskv_test_inject(7, 1)
+    assert e.value.status == R.RESKV_ERR_INVALID_ARG
+    with pytest.raises(R.ReskvError) as e:
+        R.reskv_test_inject(R.RESKV_TEST_FAIL_ALLOC, -1)
+    assert e.value.status == R.RESKV_ERR_INVALID_ARG
+    R.reskv_test_inject(R.RESKV_TEST_FAIL_ALLOC, 0)
+    R.reskv_test_inject(R.RESKV_TEST_FAIL_FIRST_WAIT, 0)

@@ -5,8 +5,8 @@ Stage-wise protocol (float32 on the GPU, float64 in the oracle):
   ranking    bit-exact when the oracle ranks the GPU's own scores; against the
              oracle's fp64 scores, two positions may only trade places if their
              fp64 scores differ by < 1e-5 relative (a near tie);
-  key-norm   scores and selection bit-exact (both sides sum the same bf16 squares
-             in fp64 in the same order);
+  key-norm   scores and selection bit-exact (both sides give the exact sum of
+             the squares rounded once to fp64, in any summation order);
   entries    given the GPU's evicted set in the GPU's rank order, the oracle's
              Lloyd gives the same counts and the same bf16 entries (up to one
              bf16 ulp where the fp32 centres left a near tie);
@@ -182,3 +182,72 @@ def test_budget_covering_every_token():
                   n_kv_heads=2)
     out = run_case(w)
     assert out["swaps"] == 0
+
+
+def _keynorm_rows():
+    """Rows (bf16-exact float64 values) where the order or the rounding of the
+    sum of squares matters, one per list entry."""
+    d = 128
+    rows = []
+    r = np.full(d, 2.0 ** -13)
+    r[0] = 2.0 ** 14                       # in dim order: 2^28; exact: 2^28 + 2^-19
+    rows += [r, r[::-1].copy()]
+    # a tie at half an ulp of 2^-40 (two squares 2^-94), broken upwards by
+    # squares far below the 128-bit window (the wide accumulator) ...
+    r = np.full(d, 2.0 ** -126)
+    r[:3] = [2.0 ** -20, 2.0 ** -47, 2.0 ** -47]
+    rows.append(r)
+    # ... by a square inside the window, and not at all (ties to even)
+    r = np.zeros(d)
+    r[:4] = [2.0 ** -20, 2.0 ** -47, 2.0 ** -47, 2.0 ** -70]
+    rows.append(r)
+    r = np.zeros(d)
+    r[5:8] = [2.0 ** -47, 2.0 ** -20, 2.0 ** -47]
+    rows.append(r)
+    r = np.zeros(d)                        # bf16 subnormals only
+    r[::3] = 2.0 ** -133
+    r[1] = 3 * 2.0 ** -130
+    rows.append(r)
+    rows.append(np.zeros(d))
+    r = np.full(d, -(2.0 ** -8))           # signs do not matter
+    r[9] = 255 * 2.0 ** -10
+    rows.append(r)
+    return rows
+
+
+def test_keynorm_scores_exact_on_crafted_rows():
+    """Key-norm scores (a build choice: the exact sum of squares rounded once)
+    bit for bit with the oracle on crafted rows and on generator rows, and the
+    ranking on them bit-exact; r = 0 so that no other stage sees the rows."""
+    s, b, P = 1024, 256, 64
+    w = wl.scaled(wl.WORKLOADS["small_budget_b64"], seq_len=s, budget=b, batch=1, n_layers=1,
+                  n_kv_heads=2)
+    K, V, _, _ = wl.layer_inputs(w, 0, "cpu")
+    rows = _keynorm_rows()
+    for h in range(2):
+        for i, row in enumerate(rows):
+            t = torch.from_numpy(row.astype(np.float32)).to(torch.bfloat16)
+            assert np.array_equal(t.double().numpy(), row)          # exact in bf16
+            K[0, h, 100 * h + 37 * i] = t
+    cfg = R.reskv_config_default(batch=1, n_layers=1, n_kv_heads=2, group=w.group, seq_len=s,
+                                 budget=b, recent_window=P, n_obs=0, n_fit=0, n_val=0,
+                                 score_mode=R.RESKV_SCORE_KEYNORM,
+                                 residual_override=np.zeros(2, np.int32), keep_debug=1)
+    cache = R.reskv_build_cache(cfg, [K.cuda()], [V.cuda()], None)
+    torch.cuda.synchronize()
+    R.reskv_check_status(cache)
+    scores = R.reskv_export_debug(cache, R.RESKV_DEBUG_SCORES).reshape(2, s)
+    top = R.reskv_export_debug(cache, R.RESKV_DEBUG_RANKED).reshape(2, -1)
+    for h in range(2):
+        Kf = K[0, h].double().numpy()
+        ref = orc.scores_keynorm(Kf)
+        bad = np.nonzero(scores[h] != ref)[0]
+        assert bad.size == 0, (h, bad[:5], scores[h][bad[:5]], ref[bad[:5]])
+        check_ranking(scores[h], top[h], ref, P, keynorm=True)
+    p0 = 37 * 0
+    assert scores[0][p0] == 2.0 ** 28 + 2.0 ** -19
+    assert scores[0][37 * 2] == 2.0 ** -40 + 2.0 ** -92
+    assert scores[0][37 * 3] == 2.0 ** -40 + 2.0 ** -92
+    assert scores[0][37 * 4] == 2.0 ** -40
+    assert scores[0][37 * 6] == 0.0
+    cache.free()

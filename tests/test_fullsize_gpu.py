@@ -2,12 +2,16 @@
 bench.py times (one all-layer reskv_decode_attn launch after reskv_build_cache,
 and one launch per layer).
 
-The inputs are generated on the GPU by the same generator as the benchmark;
-for a seeded sample of units they are regenerated on the CPU (and checked to be
-bit-identical), built and decoded by the fp64 oracle, and compared with the
-GPU's cache and outputs under the stage-wise protocol of tests/parity.py.
-Properties that hold at any size are checked on every unit: per-unit budgets,
-the protected window, residual counts, and finite outputs.
+The inputs are generated on the GPU by the same generator as the benchmark.
+Every unit's output is compared with the fp64 oracle's decode (Alg. 2) of the
+GPU-built cache.  For at least 16 units spread over layers, batch elements and
+KV heads the inputs are regenerated on the CPU (and checked to be
+bit-identical), built by the oracle's Alg. 1 in worker processes, and compared
+with the GPU's cache and outputs under the stage-wise protocol of
+tests/parity.py; the units whose choice of r lies inside the oracle's margin
+band are counted and bounded.  Properties that hold at any size are checked
+on every unit: per-unit budgets, the protected window, residual counts, and
+finite outputs.
 """
 import gc
 
@@ -21,7 +25,8 @@ from paper_2607_29591_gb300 import reskv as R
 from paper_2607_29591_gb300 import workloads as wl
 
 from helpers import assert_output_parity, bf16_to_f64, errors, unit_from_layout
-from parity import check_entries, check_ranking
+from parity import (check_entries, check_ranking, input_digest, oracle_build_job, oracle_pool,
+                    r_margin, stratified_units)
 
 pytestmark = pytest.mark.gpu
 
@@ -33,17 +38,19 @@ def lib():
     return R.load_library()
 
 
-def _units(w, n_sample):
-    rng = np.random.default_rng(42)
-    if n_sample >= w.n_units:
-        return list(range(w.n_units))
-    return sorted(int(u) for u in rng.choice(w.n_units, size=n_sample, replace=False))
+MARGIN = 1e-3          # r is compared where the oracle's deciding margin exceeds this
 
 
 def run_full(name, n_sample):
     w = wl.WORKLOADS[name]
     L, Bt, H, G = w.n_layers, w.batch, w.n_kv_heads, w.group
-    sample = _units(w, n_sample)
+    sample = stratified_units(w, n_sample)
+    ovr = w.residual_override()
+    delta = float(np.float32(R.reskv_config_default().delta))
+    # the oracle's Alg. 1 on the sample runs in worker processes meanwhile
+    pool = oracle_pool(len(sample))
+    jobs = [pool.submit(oracle_build_job, (name, u, delta, None if ovr is None else int(ovr[u])))
+            for u in sample]
     Ks, Vs, Qs = [], [], []
     Qd = torch.empty((L, Bt, H * G, w.head_dim), dtype=torch.bfloat16, device="cuda")
     kept = {}
@@ -57,12 +64,12 @@ def run_full(name, n_sample):
             ul, rem = divmod(u, Bt * H)
             if ul == l:
                 b, h = divmod(rem, H)
-                kept[u] = (K[b, h].cpu(), V[b, h].cpu(),
-                           None if Qo is None else Qo[b, h * G:(h + 1) * G].cpu())
+                kept[u] = input_digest(K[b, h].cpu(), V[b, h].cpu(),
+                                       None if Qo is None else Qo[b, h * G:(h + 1) * G].cpu())
     cfg = R.reskv_config_default(batch=Bt, n_layers=L, n_kv_heads=H, group=G, seq_len=w.seq_len,
                                  budget=w.budget, recent_window=w.recent_window, n_obs=w.n_obs,
                                  n_fit=w.n_fit, n_val=w.n_val, score_mode=w.score_mode,
-                                 residual_override=w.residual_override(), keep_debug=1)
+                                 residual_override=ovr, keep_debug=1)
     cache = R.reskv_build_cache(cfg, Ks, Vs, Qs if w.n_obs > 0 else None)
     del Ks, Vs, Qs
     gc.collect()
@@ -84,82 +91,85 @@ def run_full(name, n_sample):
     top = R.reskv_export_debug(cache, R.RESKV_DEBUG_RANKED)
     On = O.cpu().numpy()
     qf = bf16_to_f64(Qd)
+    cache.free()
+    del O, Qd
+    torch.cuda.empty_cache()
 
     # properties of every unit
     P = min(w.recent_window, w.seq_len)
     assert not np.isnan(On).any()
     assert np.all(lay["n_main"] + lay["n_res"] == min(w.budget, w.seq_len))
     assert np.all(lay["n_main"] >= P)
-    ovr = w.residual_override()
     if ovr is not None:
         assert np.array_equal(lay["n_res"], ovr)
-    for u in range(0, w.n_units, max(1, w.n_units // 64)):
+    for u in range(w.n_units):
         m, r = lay["n_main"][u], lay["n_res"][u]
         pos = lay["slot_pos"][u, :m]
         assert np.all(np.diff(pos) > 0) and np.all(pos[m - P:] == np.arange(w.seq_len - P, w.seq_len))
         if r > 0:                             # every evicted token sits in one entry
             assert lay["counts"][u, m:m + r].sum() == w.seq_len - m
 
-    # sampled units against the oracle
-    swaps, worst = 0, 0.0
-    proxy = w.residual == "proxy"
-    for u in sample:
+    # Alg. 2 on every unit: the oracle's decode of the GPU-built cache against
+    # the kernel's output of the benchmark's launch (the kernel alone), at the
+    # target's bar and at 1e-4 relative
+    oc_dec = orc.OracleConfig(budget=w.budget)
+    worst_own = 0.0
+    for u in range(w.n_units):
         l, rem = divmod(u, Bt * H)
         b, h = divmod(rem, H)
-        Kg, Vg, Qg = kept[u]
-        Kc, Vc = wl.unit_kv(w, l, b, h, "cpu")
-        assert torch.equal(Kc, Kg) and torch.equal(Vc, Vg), "GPU and CPU generators differ"
-        Qc = wl.unit_obs_queries(w, l, b, h, Kc, "cpu") if w.n_obs > 0 else None
-        if Qc is not None:
-            assert torch.equal(Qc, Qg)
-        K, V = bf16_to_f64(Kc), bf16_to_f64(Vc)
-        Qo = None if Qc is None else bf16_to_f64(Qc)
-        oc = orc.OracleConfig(budget=w.budget, recent_window=w.recent_window, n_fit=w.n_fit,
-                              n_val=w.n_val, score_mode=w.score_mode,
-                              residual_override=None if ovr is None else int(ovr[u]),
-                              delta=float(np.float32(cfg.delta)))
-        ref = orc.build_unit(K, V, Qo, oc)
+        q = qf[l, b, h * G:(h + 1) * G]
+        out = On[l, b, h * G:(h + 1) * G]
+        own = orc.decode_unit(unit_from_layout(lay, u), q, oc_dec)
+        assert_output_parity(out, own, f"unit {u} (GPU-built cache)")
+        rel = errors(out, own)[1]
+        assert rel < 1e-4, f"unit {u}: kernel vs oracle on the GPU's cache, rel {rel:.3g}"
+        worst_own = max(worst_own, rel)
+
+    # the sample's construction against the oracle's Alg. 1 (stage-wise)
+    swaps, worst, skipped = 0, 0.0, []
+    proxy = w.residual == "proxy"
+    for fut in jobs:
+        u, ref, digest = fut.result()
+        assert digest == kept[u], f"unit {u}: GPU and CPU generators differ"
+        l, rem = divmod(u, Bt * H)
+        b, h = divmod(rem, H)
         swaps += check_ranking(scores[u], top[u], ref.scores, P, w.score_mode == 1)
         gu = unit_from_layout(lay, u)
-        if proxy:
-            L_ = ref.losses
-            rs = sorted(k for k in L_ if k > 0)
-            best = min(rs, key=lambda r: (L_[r], r))
-            margin = abs(L_[best] / L_[0] - (1 - oc.delta)) if L_[0] > 0 else 1.0
-            vals = sorted(L_[r] for r in rs)
-            gap = (vals[1] - vals[0]) / vals[0] if len(vals) > 1 else 1.0
-            if min(margin, gap) > 1e-3:
-                assert gu.r == ref.r, f"unit {u}: r {gu.r} vs oracle {ref.r}"
+        if proxy and r_margin(ref.losses, delta) <= MARGIN:
+            skipped.append(u)
         else:
-            assert gu.r == ref.r
+            assert gu.r == ref.r, f"unit {u}: r {gu.r} vs oracle {ref.r}"
+        K, V = (bf16_to_f64(t) for t in wl.unit_kv(w, l, b, h, "cpu"))
         check_entries(gu, K, V, top[u], P, w.seq_len, w.budget, 4)
         q = qf[l, b, h * G:(h + 1) * G]
         out = On[l, b, h * G:(h + 1) * G]
+        oc = orc.OracleConfig(budget=w.budget)
         mx, rel = assert_output_parity(out, orc.decode_unit(ref, q, oc), f"unit {u}")
         worst = max(worst, rel)
-        own = orc.decode_unit(gu, q, oc)
-        assert errors(out, own)[1] < 1e-4, f"unit {u}: kernel vs oracle on the GPU's cache"
-    cache.free()
-    del O, Qd
-    torch.cuda.empty_cache()
+    pool.shutdown()
+    print(f"{name}: {w.n_units} units decoded against the oracle (worst rel {worst_own:.2e}); "
+          f"{len(sample)} built by the oracle, r compared on {len(sample) - len(skipped)}, "
+          f"skipped inside the {MARGIN:g} margin band: {skipped}")
+    assert len(skipped) <= max(1, int(np.ceil(0.05 * len(sample)))), skipped
     return worst, swaps
 
 
 def test_llama8b_layer_32k_all_units():
-    """One Llama-3.1-8B-shaped layer, s = 32768, b = 512, every unit checked."""
+    """One Llama-3.1-8B-shaped layer, s = 32768, b = 512: every unit built by
+    the oracle too."""
     run_full("llama8b_layer_32k", 8)
 
 
-def test_llama8b_32l_32k_b8_sampled():
+def test_llama8b_32l_32k_b8():
     """The benchmark workload: 32 layers, s = 32768, b = 1024, batch 8."""
-    run_full("llama8b_32l_32k_b8", 4)
+    run_full("llama8b_32l_32k_b8", 16)
 
 
-def test_long_128k_b4_sampled():
+def test_long_128k_b4():
     """Long-context stress: 32 layers, s = 131072, b = 2048, batch 4, drift + needles."""
-    run_full("long_128k_b4", 2)
+    run_full("long_128k_b4", 16)
 
 
-def test_small_budget_b64_sampled():
+def test_small_budget_b64():
     """Small budget, batch 64: 32 layers, s = 16384, b = 128, key-norm scores, drawn r."""
-    run_full("small_budget_b64", 8)
+    run_full("small_budget_b64", 16)
