@@ -173,3 +173,20 @@ def r_margin(losses, delta):
     vals = sorted(losses[r] for r in rs)
     gap = (vals[1] - vals[0]) / vals[0] if len(vals) > 1 and vals[0] > 0 else 1.0
     return min(margin, gap)
+
+
+def check_r(gu_r, ref, delta, u, skipped, margin_band=1e-3):
+    """r of the GPU's unit against the oracle's, unless the oracle's deciding
+    margin lies inside the band (then the unit is recorded in `skipped`)."""
+    if r_margin(ref.losses, delta) <= margin_band:
+        skipped.append(u)
+    else:
+        assert gu_r == ref.r, f"unit {u}: r {gu_r} vs oracle {ref.r}"
+
+
+def assert_few_skipped(skipped, n_checked, what=""):
+    """At most 5 % of the checked units (at least one allowed) may fall inside
+    the margin band; the count is printed with -s / -rA."""
+    print(f"{what}: r compared on {n_checked - len(skipped)} of {n_checked} units; "
+          f"inside the margin band: {skipped}")
+    assert len(skipped) <= max(1, int(np.ceil(0.05 * n_checked))), (what, skipped)
