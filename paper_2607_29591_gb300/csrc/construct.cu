@@ -10,6 +10,7 @@
 #include <vector>
 
 #include "construct_kernels.cuh"
+#include "lloyd_tc.cuh"
 #include "internal.h"
 
 namespace reskv {
@@ -353,10 +354,10 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   const size_t sm_obs1 = size_t(kTile) * kAsgRowBytes;               // the key tile
   const size_t sm_obs2 = sm_obs1 + size_t(kThreads / 32) * kTile * 4;  // + per-warp sums
   const size_t sm_top = size_t(kTopMax) * 12 + (256 + 32 + 4) * 4;
-  const size_t sm_assign = lloyd_assign_smem(rmax);
+  const size_t sm_assign = lloyd_tc_smem(rmax);
   const size_t sm_val = size_t(kHeadDim) * (2 * kTile + 2 * kRowBlk) * 4;
   if (set_smem(k_obs_pass1, sm_obs1) != cudaSuccess || set_smem(k_obs_pass2, sm_obs2) != cudaSuccess ||
-      set_smem(k_topk, sm_top) != cudaSuccess || set_smem(k_lloyd_assign, sm_assign) != cudaSuccess ||
+      set_smem(k_topk, sm_top) != cudaSuccess || set_smem(k_lloyd_assign_tc, sm_assign) != cudaSuccess ||
       set_smem(k_val_full, sm_val) != cudaSuccess)
     return cleanup_fail(fail(RESKV_ERR_CUDA, "setting kernel shared-memory limits"));
 
@@ -446,7 +447,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       const unsigned gr = unsigned(std::max(r_hi, 1));
       k_lloyd_init<<<dim3(gr, UL), kHeadDim, 0, stream>>>(la);
       for (int it = 0; it < cfg.lloyd_iters; ++it) {
-        k_lloyd_assign<<<dim3(ntiles, UL), kThreads, sm_assign, stream>>>(la);
+        k_lloyd_assign_tc<<<dim3(ntiles, UL), kTcThreads, sm_assign, stream>>>(la);
         k_lloyd_scan<<<UL, 256, 0, stream>>>(la);
         k_lloyd_scatter<<<dim3(ntiles, UL), kTile, 0, stream>>>(la);
         k_lloyd_update<<<dim3(gr, UL), kThreads, 0, stream>>>(la, it == cfg.lloyd_iters - 1);

@@ -812,35 +812,10 @@ __global__ void k_lloyd_init(LloydArgs p) {
   }
 }
 
-// Nearest centre of every evicted token of a 128-token tile; per-tile counts.
-//
-// Distances d_j = ||c_j||^2 - 2<c_j, k> (the ||k||^2 term is common) come from
-// the tensor cores: the keys are bf16 (exact operands) and every fp32 centre
-// is split exactly into two bf16 planes, c = c1 + c2 + e with
-// |e_i| <= 2^-16 |c_i|.  <c1, k> is taken 32 dims at a time (two chained
-// mma.sync m16n8k16 into a fresh accumulator, added in IEEE fp32), the small
-// plane <c2, k> in one accumulator chain.  The choice is certified in fp64.
-// Each of the four lanes that share a token keeps the best and second-best
-// of the centres it computes and the third-best distance (branch-free); every
-// centre a lane did not keep lies at or above that lane's third best, so L =
-// the least of the four third bests bounds all of them from below.  A bound on the error of the
-// computed distances then decides: if L is beyond the bound of the best, only
-// the kept candidates within it can in truth be nearest, and those are
-// re-evaluated as sum_i (k_i - c_i)^2 in fp64 against the fp64 centres; if not,
-// every centre is.  The whole warp does the fp64 work, one token at a time
-// (fp64 is scarce on this part: one lane's serial 128-term chain would hold
-// its CTA for long).  Ties go to the lower centre index.
-//
-// Error bound of the dot product, with P = sum_i |c_i k_i| <= ||c|| ||k|| and
-// u = 2^-24: one MMA step adds 16 exact products to its accumulator with an
-// error of at most 17 * 2^-22 times the largest magnitude involved, even if
-// the accumulation truncates to 24 bits, so a two-step chain errs by at most
-// 136u of its products' P (136u P over the four chains); the fp32 adds of the
-// chains add 4u P, the chain of the small plane (|c2| <= 2^-8 |c|) at most
-// 5u P, the split 256u P: about 400u P, taken as 1024u.
-// best (d0, j0), second best (d1, j1) and third-best distance d2 of a lane's
-// centres for one token; centres arrive in increasing index, so strict
-// comparisons keep the lower index on ties
+// Lloyd assignment (k_lloyd_assign_tc, lloyd_tc.cuh): best (d0, j0), second
+// best (d1, j1) and third-best distance d2 of the centres seen so far for one
+// token; centres arrive in increasing index, so strict comparisons keep the
+// lower index on ties
 __device__ __forceinline__ void top3_insert(float& d0, int& j0, float& d1, int& j1, float& d2,
                                             float x, int jx) {
   const bool c0 = x < d0, c1 = x < d1, c2 = x < d2;
@@ -849,286 +824,6 @@ __device__ __forceinline__ void top3_insert(float& d0, int& j0, float& d1, int& 
   j1 = c0 ? j0 : (c1 ? jx : j1);
   d0 = c0 ? x : d0;
   j0 = c0 ? jx : j0;
-}
-
-constexpr int kAsgNB = 32;                  // centres per staged block (double-buffered)
-constexpr int kAsgPlanes = 2;               // bf16 planes per centre
-constexpr int kAsgBufBytes = kAsgPlanes * kAsgNB * kAsgRowBytes;
-
-// Shared memory of k_lloyd_assign: the key tile, two blocks of centre planes
-// and the tile's histogram of `rmax` centres.
-inline size_t lloyd_assign_smem(int rmax) {
-  return size_t(kTile) * kAsgRowBytes + size_t(2) * kAsgBufBytes + size_t(rmax > 0 ? rmax : 1) * 4;
-}
-
-__global__ void __launch_bounds__(kThreads, 2) k_lloyd_assign(LloydArgs p) {
-  extern __shared__ __align__(128) uint8_t asm_raw[];
-  uint8_t* Ks = asm_raw;                                        // [128 tok][256 B]
-  uint8_t* Cs = Ks + kTile * kAsgRowBytes;                      // [2][2 planes][32 centres][256 B]
-  int* cnt = reinterpret_cast<int*>(Cs + 2 * kAsgBufBytes);     // [r]
-  __shared__ float cn_s[2][kAsgNB];
-  __shared__ float kn2_s[kTile];                                // ||k||^2 per token
-  __shared__ unsigned int cnmax_bits;                           // max ||c||^2 of the unit
-  const int tile = blockIdx.x, ul = blockIdx.y;
-  const int r = p.r_unit[ul];
-  if (r == 0) return;
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int g = lane >> 2, t4 = lane & 3, mi = lane >> 3;
-  const int64_t tok0 = int64_t(tile) * kTile;
-  const uint32_t ks_s = smem_u32(Ks), cs_s = smem_u32(Cs);
-  const __nv_bfloat16* Ku = p.K + int64_t(ul) * p.s * kHeadDim;
-  const __nv_bfloat16* planes = p.cplanes + int64_t(ul) * kAsgPlanes * p.rmax * kHeadDim;
-  const float* cnorm = p.cnorm + int64_t(ul) * p.rmax;
-
-  // block `b` of centre planes and norms into buffer b & 1
-  auto stage = [&](int b) {
-    const int cb = b * kAsgNB, nb = r - cb < kAsgNB ? r - cb : kAsgNB;
-    const uint32_t dst0 = cs_s + uint32_t(b & 1) * kAsgBufBytes;
-    for (int idx = threadIdx.x; idx < kAsgPlanes * kAsgNB * 16; idx += blockDim.x) {
-      const int pl = idx / (kAsgNB * 16), rem = idx % (kAsgNB * 16);
-      const int row = rem >> 4, ch = rem & 15;
-      const bool in = row < nb;
-      const __nv_bfloat16* src = planes + (int64_t(pl) * p.rmax + (in ? cb + row : 0)) * kHeadDim + 8 * ch;
-      cp_async16(dst0 + uint32_t(pl) * (kAsgNB * kAsgRowBytes) + asg_swz(row, ch), src, in ? 16u : 0u);
-    }
-    if (threadIdx.x < kAsgNB) cn_s[b & 1][threadIdx.x] = threadIdx.x < nb ? cnorm[cb + threadIdx.x] : 0.f;
-    asm volatile("cp.async.commit_group;" ::: "memory");
-  };
-  stage(0);
-  for (int idx = threadIdx.x; idx < kTile * 16; idx += blockDim.x) {
-    const int row = idx >> 4, ch = idx & 15;
-    const bool in = tok0 + row < p.s;
-    cp_async16(ks_s + asg_swz(row, ch), Ku + (in ? (tok0 + row) * kHeadDim : 0) + 8 * ch, in ? 16u : 0u);
-  }
-  asm volatile("cp.async.commit_group;" ::: "memory");
-  for (int i = threadIdx.x; i < r; i += blockDim.x) cnt[i] = 0;
-  if (threadIdx.x == 0) cnmax_bits = 0u;
-  __syncthreads();
-  float cmx = 0.f;
-  for (int i = threadIdx.x; i < r; i += blockDim.x) cmx = fmaxf(cmx, cnorm[i]);
-  atomicMax(&cnmax_bits, __float_as_uint(cmx));     // non-negative: bit order = value order
-  asm volatile("cp.async.wait_group 0;" ::: "memory");
-  __syncthreads();
-
-  // ||k||^2 of this warp's 16 tokens (two lanes per token) and the A fragments
-  {
-    const int tt = w * 16 + (lane >> 1), h0 = 8 * (lane & 1);
-    float s2 = 0.f;
-#pragma unroll
-    for (int ch = 0; ch < 8; ++ch) {
-      const uint4 v = *reinterpret_cast<const uint4*>(Ks + asg_swz(tt, h0 + ch));
-      const uint32_t wd[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float2 f = bf16x2_to_float2(wd[q]);
-        s2 = fmaf(f.x, f.x, s2);
-        s2 = fmaf(f.y, f.y, s2);
-      }
-    }
-    s2 += __shfl_xor_sync(0xffffffffu, s2, 1);
-    if ((lane & 1) == 0) kn2_s[tt] = s2;
-  }
-  // this lane's ldmatrix chunk offsets for the centre rows, per 16-dim step
-  // (every row it addresses has the same row & 7 = lane & 7)
-  uint32_t swz_b[8];
-#pragma unroll
-  for (int ks = 0; ks < 8; ++ks) swz_b[ks] = uint32_t(((2 * ks + (mi & 1)) ^ (lane & 7)) << 4);
-  uint32_t A[8][4];
-  {
-    const int row = w * 16 + (mi & 1) * 8 + (lane & 7);
-#pragma unroll
-    for (int ks = 0; ks < 8; ++ks)
-      ldsm_x4(ks_s + asg_swz(row, 2 * ks + (mi >> 1)), A[ks][0], A[ks][1], A[ks][2], A[ks][3]);
-  }
-  // per token slot a (tokens g and g + 8 of the warp's 16): this lane's best
-  // and second-best centre
-  float bd0[2] = {INFINITY, INFINITY}, bd1[2] = {INFINITY, INFINITY}, bd2[2] = {INFINITY, INFINITY};
-  int bj0[2] = {INT_MAX, INT_MAX}, bj1[2] = {INT_MAX, INT_MAX};
-
-  const int nblk = (r + kAsgNB - 1) / kAsgNB;
-  for (int b = 0; b < nblk; ++b) {
-    __syncthreads();                    // block b - 1 is consumed: its buffer is free
-    if (b + 1 < nblk) {
-      stage(b + 1);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-    }
-    __syncthreads();                    // block b is in shared memory
-    const int cb = b * kAsgNB, nb = r - cb < kAsgNB ? r - cb : kAsgNB;
-    const uint32_t buf = cs_s + uint32_t(b & 1) * kAsgBufBytes;
-    for (int np = 0; np * 16 < nb; ++np) {          // 16 centres: two n-tiles of 8
-      const uint32_t rowb = buf + uint32_t(np * 16 + (mi >> 1) * 8 + (lane & 7)) * kAsgRowBytes;
-      float acc[2][4], lo[2][4];
-#pragma unroll
-      for (int e = 0; e < 4; ++e) acc[0][e] = acc[1][e] = lo[0][e] = lo[1][e] = 0.f;
-#pragma unroll
-      for (int k2 = 0; k2 < 4; ++k2) {             // 32 dims: two chained steps
-        float t0[4] = {0.f, 0.f, 0.f, 0.f}, t1[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int kk = 0; kk < 2; ++kk) {
-          const int ks = 2 * k2 + kk;
-          const uint32_t co = rowb + swz_b[ks];
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4(co, b0, b1, b2, b3);
-          mma16816(t0, A[ks][0], A[ks][1], A[ks][2], A[ks][3], b0, b1);
-          mma16816(t1, A[ks][0], A[ks][1], A[ks][2], A[ks][3], b2, b3);
-          ldsm_x4(co + kAsgNB * kAsgRowBytes, b0, b1, b2, b3);
-          mma16816(lo[0], A[ks][0], A[ks][1], A[ks][2], A[ks][3], b0, b1);
-          mma16816(lo[1], A[ks][0], A[ks][1], A[ks][2], A[ks][3], b2, b3);
-        }
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          acc[0][e] += t0[e];
-          acc[1][e] += t1[e];
-        }
-      }
-      // this lane's four new distances per token, in increasing centre index
-#pragma unroll
-      for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          const int cl = np * 16 + nt * 8 + 2 * t4 + q;         // accumulator column
-#pragma unroll
-          for (int a = 0; a < 2; ++a) {
-            const int e = 2 * a + q;
-            const float dd = cl < nb ? cn_s[b & 1][cl] - 2.0f * (acc[nt][e] + lo[nt][e]) : INFINITY;
-            top3_insert(bd0[a], bj0[a], bd1[a], bj1[a], bd2[a], dd, cb + cl);
-          }
-        }
-    }
-  }
-  // lane t4 < 2 of a quad decides token g + 8 t4 of the warp's 16 from the
-  // quad's eight kept candidates (lane i: best, second best)
-  const int tt = w * 16 + g + 8 * (t4 & 1);
-  const int64_t pos = tok0 + tt;
-  const bool mine = t4 < 2 && pos < p.s;
-  float cd[8];
-  int cj[8];
-  float L = INFINITY;           // least third best: bounds every centre not kept
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float t0 = __shfl_sync(0xffffffffu, bd2[0], (lane & ~3) | i);
-    const float t1 = __shfl_sync(0xffffffffu, bd2[1], (lane & ~3) | i);
-    L = fminf(L, (t4 & 1) ? t1 : t0);
-  }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int srcl = (lane & ~3) | i;
-    const float a0 = __shfl_sync(0xffffffffu, bd0[0], srcl), a1 = __shfl_sync(0xffffffffu, bd0[1], srcl);
-    const float s0 = __shfl_sync(0xffffffffu, bd1[0], srcl), s1 = __shfl_sync(0xffffffffu, bd1[1], srcl);
-    const int ja0 = __shfl_sync(0xffffffffu, bj0[0], srcl), ja1 = __shfl_sync(0xffffffffu, bj0[1], srcl);
-    const int js0 = __shfl_sync(0xffffffffu, bj1[0], srcl), js1 = __shfl_sync(0xffffffffu, bj1[1], srcl);
-    cd[2 * i] = (t4 & 1) ? a1 : a0;
-    cj[2 * i] = (t4 & 1) ? ja1 : ja0;
-    cd[2 * i + 1] = (t4 & 1) ? s1 : s0;
-    cj[2 * i + 1] = (t4 & 1) ? js1 : js0;
-  }
-  const bool ev = mine && in_evicted(p, ul, pos, r);
-  int ib = 0;                                       // the best of the eight: (d, j) order
-  float d0 = cd[0];
-  int j0 = cj[0];
-#pragma unroll
-  for (int c = 1; c < 8; ++c)
-    if (cd[c] < d0 || (cd[c] == d0 && cj[c] < j0)) {
-      ib = c;
-      d0 = cd[c];
-      j0 = cj[c];
-    }
-  unsigned cmask = 0u;                              // kept candidates to re-evaluate
-  bool full = false;                                // ... or every centre
-  if (ev) {
-    // err(d): 2 x (dot product 2 gam_tc ||c|| ||k|| + norm sum 2 gam ||c||^2
-    // + fp32 centre 4u ||k|| ||c|| + final subtraction 2u |d|), with
-    // ||c|| <= max ||c|| over the unit
-    const float u = 5.9604645e-8f, gam = 130.0f * u, gam_tc = 1024.0f * u;
-    const float kn = sqrtf(kn2_s[tt]) * (1.0f + gam), cm = sqrtf(__uint_as_float(cnmax_bits));
-    const float e0 = 2.0f * (2.0f * gam_tc * cm * kn + 2.0f * gam * cm * cm + 4.0f * u * kn * cm);
-    const float err0 = e0 + 4.0f * u * fabsf(d0);
-    full = L - d0 <= err0 + e0 + 4.0f * u * fabsf(L);
-#pragma unroll
-    for (int c = 0; c < 8; ++c)
-      if (c != ib && cj[c] < r && cd[c] - d0 <= err0 + e0 + 4.0f * u * fabsf(cd[c]))
-        cmask |= 1u << c;
-    if (j0 >= r) {                                  // only a NaN distance gets here
-      report_status(p.status, kStatusBadIndex);
-      j0 = 0;
-      cmask = 0u;
-      full = false;
-    } else if (cmask) {
-      cmask |= 1u << ib;
-    }
-  }
-  // fp64 re-evaluation, one ambiguous token at a time by the whole warp: lane
-  // i holds dims 4i..4i+3, the distance is reduced over the warp (lane 0's sum
-  // decides); ties -> lower index
-  unsigned amb = __ballot_sync(0xffffffffu, ev && (full || cmask != 0u));
-  const double* c64 = p.centers64 + int64_t(ul) * p.rmax * kHeadDim + 4 * lane;
-  while (amb) {
-    const int src = __ffs(amb) - 1;
-    amb &= amb - 1;
-    const int ts = __shfl_sync(0xffffffffu, tt, src);
-    const bool fs = __shfl_sync(0xffffffffu, full ? 1 : 0, src) != 0;
-    const unsigned ms = __shfl_sync(0xffffffffu, cmask, src);
-    int js[8];
-#pragma unroll
-    for (int c = 0; c < 8; ++c) js[c] = __shfl_sync(0xffffffffu, cj[c], src);
-    const uint2 kw = *reinterpret_cast<const uint2*>(Ks + asg_swz(ts, lane >> 1) + 8 * (lane & 1));
-    const float2 k01 = bf16x2_to_float2(kw.x), k23 = bf16x2_to_float2(kw.y);
-    const double kx[4] = {k01.x, k01.y, k23.x, k23.y};
-    double bd = INFINITY;
-    int bj = INT_MAX;
-    // fp64 distances of four centres (index < 0: none), reduced over the warp
-    auto eval4 = [&](const int (&jq)[4]) {
-      double a[4];
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const double4_32a c =
-            *reinterpret_cast<const double4_32a*>(c64 + int64_t(jq[q] < 0 ? 0 : jq[q]) * kHeadDim);
-        double s = (kx[0] - c.x) * (kx[0] - c.x);
-        s = fma(kx[1] - c.y, kx[1] - c.y, s);
-        s = fma(kx[2] - c.z, kx[2] - c.z, s);
-        a[q] = fma(kx[3] - c.w, kx[3] - c.w, s);
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-        for (int q = 0; q < 4; ++q) a[q] += __shfl_xor_sync(0xffffffffu, a[q], o);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const double dd = __shfl_sync(0xffffffffu, a[q], 0);
-        if (jq[q] >= 0 && (dd < bd || (dd == bd && jq[q] < bj))) {
-          bd = dd;
-          bj = jq[q];
-        }
-      }
-    };
-    if (fs) {                                       // every centre
-      for (int jb = 0; jb < r; jb += 4) {
-        const int jq[4] = {jb, jb + 1 < r ? jb + 1 : -1, jb + 2 < r ? jb + 2 : -1,
-                           jb + 3 < r ? jb + 3 : -1};
-        eval4(jq);
-      }
-    } else {                                        // the flagged kept candidates
-#pragma unroll
-      for (int h4 = 0; h4 < 2; ++h4) {
-        int jq[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) jq[q] = (ms >> (4 * h4 + q)) & 1u ? js[4 * h4 + q] : -1;
-        eval4(jq);
-      }
-    }
-    if (lane == src) j0 = bj;
-  }
-  if (ev) {
-    p.assign[int64_t(ul) * p.s + pos] = j0;
-    atomicAdd(&cnt[j0], 1);
-  } else if (mine) {
-    p.assign[int64_t(ul) * p.s + pos] = -1;
-  }
-  __syncthreads();
-  int32_t* h = p.hist + (int64_t(ul) * p.ntiles + tile) * p.rmax;
-  for (int i = threadIdx.x; i < r; i += blockDim.x) h[i] = cnt[i];
 }
 
 // per centre: counts, per-tile offsets (in place) and member bases
