@@ -385,6 +385,7 @@ def run_reference(args, world, rank):
     every step is one dispatch (cpu_baseline's method)."""
     if rank != 0:
         return
+    world = 1 if world < 1 else world
     w = wl.WORKLOADS[args.workload]
     cores = os.cpu_count() or 1
     pool = OraclePool(w, 64, cores)
@@ -402,7 +403,7 @@ def run_reference(args, world, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": step_s * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(w),
+            "config": workload_config(w, args.budget_mode, world),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": pool.procs,
                              "kind": "oracle",
                              "sample": pool.describe() + "; one dispatch per step"},
@@ -411,11 +412,16 @@ def run_reference(args, world, rank):
     print(json.dumps(line), flush=True)
 
 
-def workload_config(w: wl.Workload) -> dict:
-    """The workload's shape, named as in the JSON line's config."""
+def workload_config(w: wl.Workload, budget_mode: str = "uniform", world: int = 1) -> dict:
+    """The JSON line's config, the same in both arms: the workload's shape,
+    its budget mode, the parallelism, and why no L2 flush is needed."""
+    slots = w.n_units * min(w.budget, w.seq_len) * SLOT_BYTES
     return {"workload": w.name, "layers": w.n_layers, "batch": w.batch,
             "kv_heads": w.n_kv_heads, "q_heads": w.n_q_heads, "head_dim": w.head_dim,
-            "seq_len": w.seq_len, "budget": w.budget, "residual": w.residual}
+            "seq_len": w.seq_len, "budget": w.budget, "residual": w.residual,
+            "budget_mode": budget_mode,
+            "parallelism": "replicas" if world > 1 else "single GPU",
+            "l2": f"inputs larger than L2: {slots / 1e9:.2f} GB of K/V slots read per step"}
 
 
 # ---------------------------------------------------------------------------
@@ -601,12 +607,12 @@ def measure(args, w: wl.Workload, R, kern: int, bmode: int, device, world: int, 
                  "q_o_bytes_per_step": int(w.n_units * w.group * w.head_dim * (2 + 4)),
                  "how": "one reskv_decode_attn(layer=-1) launch per step (needs every layer's "
                         "query up front: a ceiling, not a decoder's step)"}
-    out = {"config": dict(workload_config(w), **{
-               "mean_r": float(np.mean(r_counts)),
-               "units_with_residual": float(np.mean(r_counts > 0)),
-               "unit_budget_min_max": [int(unit_budgets.min()), int(unit_budgets.max())],
-               "decode_plan": plan,
-               "l2": f"inputs larger than L2: {alg / 1e9:.2f} GB of cache read per step"}),
+    out = {"config": workload_config(w, args.budget_mode, world),
+           "run": {"mean_r": float(np.mean(r_counts)),
+                   "units_with_residual": float(np.mean(r_counts > 0)),
+                   "unit_budget_min_max": [int(unit_budgets.min()), int(unit_budgets.max())],
+                   "decode_plan": plan,
+                   "algorithmic_bytes_per_step": alg},
            "per_layer": per_layer, "all_layer": all_layer,
            "launches_per_step": launches_per_step, "construction_s": build_s,
            "construction_stages_ms": dict(zip(
@@ -675,11 +681,9 @@ def main():
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": pl["us_per_step"] / 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
-            "config": dict(main_rec["config"], **{
-                "budget_mode": args.budget_mode,
-                "launch": f"one reskv_decode_attn(layer) launch per layer, {w.n_layers} per step, "
-                          f"in one CUDA graph",
-                "parallelism": "replicas" if world > 1 else "single GPU"}),
+            "config": main_rec["config"],
+            "run": dict(main_rec["run"], launch=f"one reskv_decode_attn(layer) launch per layer, "
+                                                f"{w.n_layers} per step, in one CUDA graph"),
             "us_per_layer_step": pl["us_per_layer_step"],
             "roofline": pl["roofline"],
             "all_layer_launch": main_rec["all_layer"],
@@ -693,7 +697,7 @@ def main():
         }
         if second is not None:
             line["second_workload"] = {
-                "config": second["config"], "per_layer": second["per_layer"],
+                "config": second["config"], "run": second["run"], "per_layer": second["per_layer"],
                 "all_layer_launch": second["all_layer"], "construction_s": second["construction_s"],
                 "construction_stages_ms": second["construction_stages_ms"],
                 "clocks": second["clocks"], "steps": args.steps, "warmup": args.warmup}
