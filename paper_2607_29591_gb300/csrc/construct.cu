@@ -10,6 +10,7 @@
 #include <vector>
 
 #include "construct_kernels.cuh"
+#include "lloyd_pt.cuh"
 #include "lloyd_tc.cuh"
 #include "internal.h"
 
@@ -294,6 +295,12 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   float *centersT = nullptr, *cnorm = nullptr, *vpart = nullptr, *oS = nullptr;
   __nv_bfloat16* cplanes = nullptr;
   double* centers64 = nullptr;
+  long long* msum = nullptr;
+  uint32_t* mflag = nullptr;
+  float* knorm2 = nullptr;
+  int4* amb = nullptr;
+  int* amb_count = nullptr;
+  float* centers32 = nullptr;
   __nv_bfloat16 *kbar = nullptr, *vbar = nullptr;
   double *rowerr = nullptr, *losses = nullptr;
   const size_t US = size_t(UL) * size_t(s);
@@ -313,7 +320,15 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
          S.get(&cplanes, size_t(UL) * 2 * rmax * kHeadDim) &&
          S.get(&cnorm, size_t(UL) * rmax) && S.get(&kbar, size_t(UL) * ent_stride * kHeadDim) &&
          S.get(&vbar, size_t(UL) * ent_stride * kHeadDim) &&
-         S.get(&ecount, size_t(UL) * ent_stride);
+         S.get(&ecount, size_t(UL) * ent_stride) &&
+         S.get(&msum, size_t(UL) * rmax * 2 * kHeadDim) && S.get(&mflag, size_t(UL) * rmax) &&
+         S.get(&knorm2, US) && S.get(&amb, US) && S.get(&amb_count, 1) &&
+         S.get(&centers32, size_t(UL) * rmax * kHeadDim);
+  // the member sums start at zero; each pass's k_lloyd_finish clears what it read
+  if (ok && rmax > 0)
+    ok = cudaMemsetAsync(msum, 0, size_t(UL) * rmax * 2 * kHeadDim * sizeof(long long), stream) ==
+             cudaSuccess &&
+         cudaMemsetAsync(mflag, 0, size_t(UL) * rmax * sizeof(uint32_t), stream) == cudaSuccess;
   if (ok && proxy)
     ok = S.get(&vpart, size_t(UL) * n_val_rows * nchunks * kValRec) &&
          S.get(&oS, size_t(UL) * n_val_rows * kHeadDim) &&
@@ -358,6 +373,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   const size_t sm_val = size_t(kHeadDim) * (2 * kTile + 2 * kRowBlk) * 4;
   if (set_smem(k_obs_pass1, sm_obs1) != cudaSuccess || set_smem(k_obs_pass2, sm_obs2) != cudaSuccess ||
       set_smem(k_topk, sm_top) != cudaSuccess || set_smem(k_lloyd_assign_tc, sm_assign) != cudaSuccess ||
+      set_smem(k_lloyd_assign_pt, lloyd_pt_smem()) != cudaSuccess ||
       set_smem(k_val_full, sm_val) != cudaSuccess)
     return cleanup_fail(fail(RESKV_ERR_CUDA, "setting kernel shared-memory limits"));
 
@@ -439,18 +455,34 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
 
     LloydArgs la{K, V, s, P, n_top, b, ntiles, rmax, top, rank_pos, nullptr, centersT, cnorm,
                  centers64, assign, hist, ccount, cbase, members, kbar, vbar, ecount,
-                 ent_stride, 0, c->status, bl_d, cplanes};
+                 ent_stride, 0, c->status, bl_d, cplanes, msum, mflag, knorm2, amb, amb_count, centers32};
+    if (rmax > 0)
+      k_key_norm2<<<unsigned(cdiv(int64_t(US), 8)), 256, 0, stream>>>(K, knorm2, int64_t(US));
     auto lloyd_run = [&](const int32_t* r_unit, int ent_off, int r_hi) -> reskv_status {
       la.r_unit = r_unit;
       la.ent_off = ent_off;
       timing_ok &= timer.mark(kStLloyd);
       const unsigned gr = unsigned(std::max(r_hi, 1));
+      const unsigned pt_grid = unsigned(std::min<int64_t>(c->num_sms, int64_t(UL) * ntiles));
       k_lloyd_init<<<dim3(gr, UL), kHeadDim, 0, stream>>>(la);
       for (int it = 0; it < cfg.lloyd_iters; ++it) {
-        k_lloyd_assign_tc<<<dim3(ntiles, UL), kTcThreads, sm_assign, stream>>>(la);
+        if (r_hi <= kPtRmax) {        // the centres fit in shared memory: persistent form
+          if (cudaMemsetAsync(amb_count, 0, sizeof(int), stream) != cudaSuccess)
+            return fail(RESKV_ERR_CUDA, "clearing the ambiguous-token count");
+          k_lloyd_assign_pt<<<pt_grid, kPtThreads, lloyd_pt_smem(), stream>>>(la, UL);
+          k_lloyd_resolve<<<unsigned(4 * c->num_sms), kResWarps * 32, 0, stream>>>(la);
+        } else {
+          k_lloyd_assign_tc<<<dim3(ntiles, UL), kTcThreads, sm_assign, stream>>>(la);
+        }
         k_lloyd_scan<<<UL, 256, 0, stream>>>(la);
         k_lloyd_scatter<<<dim3(ntiles, UL), kTile, 0, stream>>>(la);
-        k_lloyd_update<<<dim3(gr, UL), kThreads, 0, stream>>>(la, it == cfg.lloyd_iters - 1);
+        const int last = it == cfg.lloyd_iters - 1;
+        const dim3 ga(unsigned(cdiv(s, int64_t(kAccRows))), UL);
+        if (last)
+          k_lloyd_accum<true><<<ga, kThreads, 0, stream>>>(la);
+        else
+          k_lloyd_accum<false><<<ga, kThreads, 0, stream>>>(la);
+        k_lloyd_finish<<<dim3(gr, UL), kHeadDim, 0, stream>>>(la, last);
       }
       RESKV_LAUNCH_CHECK("residual entries");
       return RESKV_OK;

@@ -773,6 +773,12 @@ struct LloydArgs {
   const int32_t* budgets;      // [UL] per-unit budgets, or NULL (budget)
   __nv_bfloat16* cplanes;      // [UL, 2, rmax, d] the fp32 centres split into
                                // two bf16 planes c1 + c2 (tensor-core operands)
+  long long* msum;             // [UL, rmax, 2, d] fixed-point member sums (K, V); zero between passes
+  uint32_t* mflag;             // [UL, rmax] set when a member value is outside the fixed-point range
+  float* knorm2;               // [UL, s] fp32 ||k||^2 of every key (the persistent assignment's bound)
+  int4* amb;                   // [UL * s] tokens the persistent assignment leaves to k_lloyd_resolve
+  int* amb_count;              // their number (zeroed before each assignment)
+  float* centers32;            // [UL, rmax, d] row-major fp32 copy of the centres
 };
 
 __device__ __forceinline__ bool in_evicted(const LloydArgs& p, int ul, int64_t pos, int r) {
@@ -803,6 +809,7 @@ __global__ void k_lloyd_init(LloydArgs p) {
   p.centersT[(int64_t(ul) * kHeadDim + d) * p.rmax + j] = c;
   write_planes(p, ul, j, d, c);
   p.centers64[(int64_t(ul) * p.rmax + j) * kHeadDim + d] = double(c);
+  p.centers32[(int64_t(ul) * p.rmax + j) * kHeadDim + d] = c;
   red[d] = c * c;
   __syncthreads();
   if (d == 0) {
@@ -838,10 +845,21 @@ __global__ void k_lloyd_scan(LloydArgs p) {
     const int j = threadIdx.x * per + q;
     if (j >= r) break;
     int run = 0;
-    for (int t = 0; t < p.ntiles; ++t) {
-      int32_t* h = p.hist + (int64_t(ul) * p.ntiles + t) * p.rmax + j;
-      const int c = *h;
-      *h = run;
+    int32_t* h = p.hist + int64_t(ul) * p.ntiles * p.rmax + j;
+    int t = 0;
+    for (; t + 16 <= p.ntiles; t += 16) {     // 16 independent loads in flight
+      int c[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) c[u] = h[int64_t(t + u) * p.rmax];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        h[int64_t(t + u) * p.rmax] = run;
+        run += c[u];
+      }
+    }
+    for (; t < p.ntiles; ++t) {
+      const int c = h[int64_t(t) * p.rmax];
+      h[int64_t(t) * p.rmax] = run;
       run += c;
     }
     p.ccount[int64_t(ul) * p.rmax + j] = run;
@@ -875,143 +893,205 @@ __global__ void k_lloyd_scatter(LloydArgs p) {
   p.members[int64_t(ul) * p.s + off] = int32_t(pos);
 }
 
-// A bf16 value as a 64-bit fixed-point integer with 32 fractional bits:
-// value = sign * M * 2^(e - 134) with the 8-bit significand M, so v = M << (e - 102).
-// `ok` is cleared when the value is not represented exactly (|x| < 2^-25 with
-// low bits set, a subnormal, |x| >= 2^14, inf or NaN); below 2^14 a sum of
-// 2^17 terms stays under 2^63.
-__device__ __forceinline__ long long bf16_fixed32(uint32_t b, bool& ok) {
-  const int e = int((b >> 7) & 0xffu);
-  const uint32_t m7 = b & 0x7fu;
-  if (e == 0) {                                   // +-0 exact, subnormals not
-    ok = ok && m7 == 0u;
-    return 0;
-  }
-  const long long M = (long long)(m7 | 0x80u);
-  const int sh = e - 102;
-  long long v;
-  if (sh >= 0) {
-    ok = ok && sh <= 38;
-    v = M << (sh <= 38 ? sh : 38);
-  } else {
-    const int rs = -sh;
-    ok = ok && rs <= 7 && (M & ((1LL << (rs <= 7 ? rs : 7)) - 1)) == 0;
-    v = rs <= 7 ? (M >> rs) : 0;
-  }
-  return (b & 0x8000u) ? -v : v;
+// New centre = mean key of its members; on the last iteration also the mean
+// value, and the stored bf16 entry (Eq. summary).  The member sums are exact
+// fixed-point integers, so they are free of summation order, and the
+// conversion of the total to fp64 is the exact sum rounded once; mean = that
+// sum / count.  If a member value is outside the fixed-point range the centre
+// is summed in fp64 in member order instead.
+//
+// Two kernels.  k_lloyd_accum sweeps the member list (grouped by centre)
+// token-parallel: each warp takes kAccRowsPerWarp consecutive member slots,
+// gathers their rows, keeps running sums for the centre it is in, and adds
+// them into msum[ul][j] with 64-bit integer atomics when the centre changes.
+// Integer addition is associative, so the totals do not depend on the order
+// the atomics land in.  k_lloyd_finish then forms the means, one CTA per
+// centre, and clears msum / mflag for the next pass.
+//
+// The running sums split every member value on the FP32 pipe, with two
+// magic-number roundings (no integer shifts, which would bound the kernel on
+// the integer ALU).  For |x| < 128 and x a multiple of 2^-32:
+//   s = x + C1 (C1 = 1.5 * 2^8; s lies in [256, 512), whose ulp is 2^-15),
+//   h = s - C1 (x rounded to a multiple of 2^-15; exact), l = x - h (exact,
+//   |l| <= 2^-16), t = l + C2 (C2 = 1.5 * 2^-9; t lies in [2^-9, 2^-8), ulp
+//   2^-32, so t is exact).
+// Then bits(s) - bits(C1) = h * 2^15 and bits(t) - bits(C2) = l * 2^32 as
+// integers, so a lane adds bits(s) and bits(t) into 32-bit sums (mod 2^32)
+// and the flush subtracts n * bits(C) for the n rows added: the exact
+// |sum h * 2^15| < 2^28 and |sum l * 2^32| <= 2^22 for n <= 64.  The flush
+// joins them into the 64-bit total (sum h * 2^15) * 2^17 + sum l * 2^32
+// (unit 2^-32).  A value outside the window shows as t - C2 != l (inexact:
+// a subnormal, a tail below 2^-32, inf, NaN) or as |x| >= 128; the centre is
+// then summed in fp64 instead.  Below 128 a sum of 2^17 terms stays under 2^63.
+constexpr int kAccRowsPerWarp = 64;
+constexpr int kAccRows = kAccRowsPerWarp * (kThreads / 32);   // member slots per CTA
+static_assert(kAccRowsPerWarp <= 64, "the mod-2^32 lane sums must stay below 2^31");
+constexpr float kFixC1 = 384.0f;
+constexpr float kFixC2 = 0x1.8p-9f;
+
+struct FixSum {
+  uint32_t hi[4], lo[4];
+};
+
+struct FixState {
+  float err, mx;                 // sum of |t - C2 - l|, max |x|: exact iff 0 and < 128
+};
+
+__device__ __forceinline__ void fix_add(float x, uint32_t& hi, uint32_t& lo, FixState& st) {
+  const float s = __fadd_rn(x, kFixC1);
+  const float h = __fadd_rn(s, -kFixC1);
+  const float l = __fadd_rn(x, -h);
+  const float t = __fadd_rn(l, kFixC2);
+  st.err = __fadd_rn(st.err, fabsf(__fadd_rn(__fadd_rn(t, -kFixC2), -l)));
+  st.mx = fmaxf(st.mx, fabsf(x));
+  hi += __float_as_uint(s);
+  lo += __float_as_uint(t);
 }
 
-// new centre = mean key of its members; on the last iteration also the mean
-// value, and the stored bf16 entry.  The member sums are exact: 64-bit
-// fixed-point integers (order-free), converted to fp64 once -- exactly, as a
-// sum of at most 2^17 terms in [2^-25, 2^14) needs fewer than 53 bits -- so
-// mean = sum / count is the fp64 mean of the exact sum.  If a term falls
-// outside that range the centre is summed in fp64 in member order instead.
-__global__ void __launch_bounds__(kThreads) k_lloyd_update(LloydArgs p, int final_pass) {
-  __shared__ long long redk[8][kHeadDim];
-  __shared__ long long redv[8][kHeadDim];
-  __shared__ double dk[kHeadDim], dv[kHeadDim];
-  __shared__ float nrm[kHeadDim];
-  const int j = blockIdx.x, ul = blockIdx.y;
+// four consecutive bf16 (two words, low half first) into the lane sums
+__device__ __forceinline__ void acc_row(uint2 w, FixSum& a, FixState& st) {
+  fix_add(__uint_as_float(w.x << 16), a.hi[0], a.lo[0], st);
+  fix_add(__uint_as_float(w.x & 0xffff0000u), a.hi[1], a.lo[1], st);
+  fix_add(__uint_as_float(w.y << 16), a.hi[2], a.lo[2], st);
+  fix_add(__uint_as_float(w.y & 0xffff0000u), a.hi[3], a.lo[3], st);
+}
+
+// dim q's 64-bit fixed-point total of n added rows; the lane sums are cleared
+__device__ __forceinline__ unsigned long long fix_total(FixSum& a, int q, uint32_t n) {
+  const int32_t h = int32_t(a.hi[q] - n * __float_as_uint(kFixC1));
+  const int32_t l = int32_t(a.lo[q] - n * __float_as_uint(kFixC2));
+  a.hi[q] = 0u;
+  a.lo[q] = 0u;
+  return static_cast<unsigned long long>(((long long)h << 17) + (long long)l);
+}
+
+template <bool final_pass>
+__global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
+  const int ul = blockIdx.y;
   const int r = p.r_unit[ul];
-  if (j >= r) return;
+  if (r <= 0) return;
+  const int32_t* cb = p.cbase + int64_t(ul) * p.rmax;
+  const int32_t* cc = p.ccount + int64_t(ul) * p.rmax;
+  const int n_mem = cb[r - 1] + cc[r - 1];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int cnt = p.ccount[int64_t(ul) * p.rmax + j];
-  const int base = p.cbase[int64_t(ul) * p.rmax + j];
-  const int per = (cnt + 7) / 8;
-  const int lo = w * per, hi = min(cnt, lo + per);
-  const int32_t* mem = p.members + int64_t(ul) * p.s + base;
+  const int lo = blockIdx.x * kAccRows + w * kAccRowsPerWarp;
+  if (lo >= n_mem) return;
+  const int hi = min(n_mem, lo + kAccRowsPerWarp);
+  // the centre holding slot lo: the last j with cbase[j] <= lo (it is never
+  // empty: an empty centre shares its cbase with the next one)
+  int j = 0;
+  for (int step = 1 << (31 - __clz(max(r - 1, 1))); step > 0; step >>= 1)
+    if (j + step < r && cb[j + step] <= lo) j += step;
+  int bnd = cb[j] + cc[j];
+  const int32_t* mem = p.members + int64_t(ul) * p.s;
   const __nv_bfloat16* Kb = p.K + int64_t(ul) * p.s * kHeadDim + 4 * lane;
   const __nv_bfloat16* Vb = p.V + int64_t(ul) * p.s * kHeadDim + 4 * lane;
-  long long sk[4] = {0, 0, 0, 0}, sv[4] = {0, 0, 0, 0};
-  bool ok = true;
-  for (int i = lo; i < hi; i += 4) {
-    uint2 kw[4], vw[4];
+  unsigned long long* ms = reinterpret_cast<unsigned long long*>(p.msum) +
+                           int64_t(ul) * p.rmax * 2 * kHeadDim + 4 * lane;
+  FixSum sk = {}, sv = {};
+  FixState st = {0.0f, 0.0f};
+  uint32_t n = 0;                 // rows in the lane sums
+  auto flush = [&](int jj) {
+    unsigned long long* m = ms + int64_t(jj) * 2 * kHeadDim;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      if (i + q < hi) {
-        const int64_t pos = mem[i + q];
-        kw[q] = __ldg(reinterpret_cast<const uint2*>(Kb + pos * kHeadDim));
-        if (final_pass) vw[q] = __ldg(reinterpret_cast<const uint2*>(Vb + pos * kHeadDim));
-      }
+    for (int q = 0; q < 4; ++q) atomicAdd(m + q, fix_total(sk, q, n));
+    if constexpr (final_pass) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) atomicAdd(m + kHeadDim + q, fix_total(sv, q, n));
     }
+    const bool ok = st.err == 0.0f && st.mx < 128.0f;
+    if (__any_sync(0xffffffffu, !ok) && lane == 0) atomicOr(p.mflag + int64_t(ul) * p.rmax + jj, 1u);
+    st = FixState{0.0f, 0.0f};
+    n = 0;
+  };
+  for (int i32 = lo; i32 < hi; i32 += 32) {
+    const int my = i32 + lane < hi ? mem[i32 + lane] : 0;
+#pragma unroll 1
+    for (int i8 = 0; i8 < 32 && i32 + i8 < hi; i8 += 8) {
+      uint2 kw[8], vw[8];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      if (i + q < hi) {
-        sk[0] += bf16_fixed32(kw[q].x & 0xffffu, ok);
-        sk[1] += bf16_fixed32(kw[q].x >> 16, ok);
-        sk[2] += bf16_fixed32(kw[q].y & 0xffffu, ok);
-        sk[3] += bf16_fixed32(kw[q].y >> 16, ok);
-        if (final_pass) {
-          sv[0] += bf16_fixed32(vw[q].x & 0xffffu, ok);
-          sv[1] += bf16_fixed32(vw[q].x >> 16, ok);
-          sv[2] += bf16_fixed32(vw[q].y & 0xffffu, ok);
-          sv[3] += bf16_fixed32(vw[q].y >> 16, ok);
+      for (int q = 0; q < 8; ++q) {
+        const int64_t pos = __shfl_sync(0xffffffffu, my, i8 + q);
+        if (i32 + i8 + q < hi) {
+          kw[q] = __ldg(reinterpret_cast<const uint2*>(Kb + pos * kHeadDim));
+          if constexpr (final_pass) vw[q] = __ldg(reinterpret_cast<const uint2*>(Vb + pos * kHeadDim));
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int i = i32 + i8 + q;
+        if (i < hi) {
+          while (i >= bnd) {            // warp-uniform: the next centre starts here
+            flush(j);
+            ++j;
+            bnd = cb[j] + cc[j];
+          }
+          acc_row(kw[q], sk, st);
+          if constexpr (final_pass) acc_row(vw[q], sv, st);
+          ++n;
         }
       }
     }
   }
-#pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    redk[w][4 * lane + q] = sk[q];
-    redv[w][4 * lane + q] = sv[q];
-  }
-  const bool exact = __syncthreads_and(ok) != 0;
+  flush(j);
+}
+
+__global__ void __launch_bounds__(kHeadDim) k_lloyd_finish(LloydArgs p, int final_pass) {
+  __shared__ float nrm[kHeadDim];
+  const int j = blockIdx.x, ul = blockIdx.y;
+  const int r = p.r_unit[ul];
+  if (j >= r) return;
+  const int d = threadIdx.x;
+  const int64_t uj = int64_t(ul) * p.rmax + j;
+  const int cnt = p.ccount[uj];
+  const bool exact = p.mflag[uj] == 0u;
+  long long* ms = p.msum + uj * 2 * kHeadDim;
+  const long long tki = ms[d], tvi = ms[kHeadDim + d];
+  ms[d] = 0;
+  ms[kHeadDim + d] = 0;
+  double tk, tv;
   if (exact) {
-    if (threadIdx.x < kHeadDim) {
-      const int d = threadIdx.x;
-      long long tk = 0, tv = 0;
-      for (int ww = 0; ww < 8; ++ww) {
-        tk += redk[ww][d];
-        tv += redv[ww][d];
-      }
-      dk[d] = double(tk) * 0x1p-32;
-      dv[d] = double(tv) * 0x1p-32;
-    }
+    tk = double(tki) * 0x1p-32;
+    tv = double(tvi) * 0x1p-32;
   } else {
-    // fp64 sums in member order (one thread per dim)
-    if (threadIdx.x < kHeadDim) {
-      const int d = threadIdx.x;
-      double tk = 0.0, tv = 0.0;
-      const __nv_bfloat16* Kd = p.K + int64_t(ul) * p.s * kHeadDim + d;
-      const __nv_bfloat16* Vd = p.V + int64_t(ul) * p.s * kHeadDim + d;
-      for (int i = 0; i < cnt; ++i) {
-        const int64_t pos = mem[i];
-        tk += double(__bfloat162float(Kd[pos * kHeadDim]));
-        if (final_pass) tv += double(__bfloat162float(Vd[pos * kHeadDim]));
-      }
-      dk[d] = tk;
-      dv[d] = tv;
+    // fp64 sums in member order
+    tk = 0.0;
+    tv = 0.0;
+    const int32_t* mem = p.members + int64_t(ul) * p.s + p.cbase[uj];
+    const __nv_bfloat16* Kd = p.K + int64_t(ul) * p.s * kHeadDim + d;
+    const __nv_bfloat16* Vd = p.V + int64_t(ul) * p.s * kHeadDim + d;
+    for (int i = 0; i < cnt; ++i) {
+      const int64_t pos = mem[i];
+      tk += double(__bfloat162float(Kd[pos * kHeadDim]));
+      if (final_pass) tv += double(__bfloat162float(Vd[pos * kHeadDim]));
     }
   }
-  if (threadIdx.x < kHeadDim) {
-    const int d = threadIdx.x;
-    const double tk = dk[d], tv = dv[d];
-    float* cptr = p.centersT + (int64_t(ul) * kHeadDim + d) * p.rmax + j;
-    double* c64 = p.centers64 + (int64_t(ul) * p.rmax + j) * kHeadDim + d;
-    double mk;
-    if (cnt > 0) {
-      mk = tk / double(cnt);
-      *c64 = mk;
-      *cptr = float(mk);
-      write_planes(p, ul, j, d, float(mk));
-    } else {
-      mk = *c64;                        // an empty cluster keeps its centre
-    }
-    const float c = *cptr;
-    nrm[d] = c * c;
-    if (final_pass) {
-      const int64_t e = int64_t(ul) * p.ent_stride + p.ent_off + j;
-      p.kbar[e * kHeadDim + d] = __double2bfloat16(mk);
-      p.vbar[e * kHeadDim + d] = __double2bfloat16(cnt > 0 ? tv / double(cnt) : 0.0);
-      if (d == 0) p.ecount[e] = cnt;
-    }
+  float* cptr = p.centersT + (int64_t(ul) * kHeadDim + d) * p.rmax + j;
+  double* c64 = p.centers64 + uj * kHeadDim + d;
+  double mk;
+  if (cnt > 0) {
+    mk = tk / double(cnt);
+    *c64 = mk;
+    *cptr = float(mk);
+    p.centers32[uj * kHeadDim + d] = float(mk);
+    write_planes(p, ul, j, d, float(mk));
+  } else {
+    mk = *c64;                        // an empty centre keeps its place
+  }
+  const float c = *cptr;
+  nrm[d] = c * c;
+  if (final_pass) {
+    const int64_t e = int64_t(ul) * p.ent_stride + p.ent_off + j;
+    p.kbar[e * kHeadDim + d] = __double2bfloat16(mk);
+    p.vbar[e * kHeadDim + d] = __double2bfloat16(cnt > 0 ? tv / double(cnt) : 0.0);
+    if (d == 0) p.ecount[e] = cnt;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
+  if (d == 0) {
     float n = 0.f;
     for (int i = 0; i < kHeadDim; ++i) n += nrm[i];
-    p.cnorm[int64_t(ul) * p.rmax + j] = n;
+    p.cnorm[uj] = n;
+    p.mflag[uj] = 0u;
   }
 }
 

@@ -1,0 +1,634 @@
+// Lloyd assignment (Sec. 5.3, Eq. residual_partition), persistent form for
+// units with at most 256 centres: one CTA per SM walks a contiguous range of
+// (unit, 128-token tile) pairs, with the unit's centre planes resident in
+// shared memory, so a tile costs one key-tile load and one tcgen05.mma chain.
+// Three roles run decoupled, linked by mbarrier rings:
+//
+//   producer warp    loads key tile t into buffer t & 1 (cp.async, 128-byte
+//                    swizzle) one tile ahead, and issues the MMA chain of
+//                    tile t - 1 (2 planes x 8 K-steps, M = 128 tokens, N = r
+//                    rounded up to 16) into TMEM columns 256 ((t - 1) & 1) ..,
+//                    committed to full[].  At a change of unit it waits for
+//                    every earlier MMA and for the column warps to be done with
+//                    the old centre norms, then stages the new planes.
+//   8 column warps   warp w reads TMEM lanes 32 (w % 4).. (its tokens) and the
+//                    16-column chunks w / 4, w / 4 + 2, .. of the distances,
+//                    keeping two top-3 lists per thread (even and odd columns:
+//                    independent dependency chains), frees the TMEM buffer
+//                    (tmem_empty[]), merges the two column halves and posts the
+//                    tile's lists in a ring of kPtRing slots (list_full[]).
+//   4 certifier      certify each token's choice and re-evaluate ambiguous
+//   warps            tokens in fp64 as the streaming kernel does (keys from
+//                    global memory, key norms precomputed per layer), write
+//                    assign, count members per centre and write the tile's
+//                    counts, then free the slot (list_empty[]).
+//
+// fp64 is slow on this part; with its own warps and a ring in between, a
+// tile whose tokens need many fp64 distances delays the column warps only
+// once the ring is full.  Every wait is bounded; a wait that gives up raises
+// kStatusWaitTimeout and an abort flag, and each role leaves its loop at a
+// tile boundary agreed by a barrier reduction over the role's threads.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "lloyd_tc.cuh"
+
+namespace reskv {
+namespace build {
+
+constexpr int kPtColWarps = 8;
+constexpr int kPtColThreads = kPtColWarps * 32;
+constexpr int kPtCertWarps = 4;
+constexpr int kPtCertThreads = kPtCertWarps * 32;
+constexpr int kPtProducer = kPtColWarps + kPtCertWarps;        // the producer warp's index
+constexpr int kPtThreads = (kPtProducer + 1) * 32;
+constexpr int kPtRmax = 256;                                    // centres held resident
+constexpr int kPtRing = 4;                                      // list slots
+constexpr int kPtPlaneHalf = kPtRmax * 128;                     // one 64-dim half of a plane, bytes
+constexpr int kPtPlanes = 2 * 2 * kPtPlaneHalf;                 // both planes
+constexpr int kPtKeys = 2 * kTcHalf;                            // one key tile
+constexpr uint32_t kPtBufCols = 256;                            // TMEM columns per buffer
+constexpr uint32_t kPtCols = 2 * kPtBufCols;
+constexpr int kPtXch = kTile * 5;                               // floats: d0, j0, d1, j1, d2 per token
+constexpr int kPtList = kTile * 7;                              // the same, + rank, ||k||^2
+
+// Shared memory (from a 1024-aligned base): planes, 2 key tiles, centre
+// norms, 2 x the column halves' exchange lists, the ring (lists, counts,
+// info), 2 x TMEM tile info, the abort flag, mbarriers, the TMEM address.
+constexpr size_t kPtOffKeys = kPtPlanes;
+constexpr size_t kPtOffNorm = kPtOffKeys + 2 * size_t(kPtKeys);
+constexpr size_t kPtOffXch = kPtOffNorm + kPtRmax * 4;
+constexpr size_t kPtOffList = kPtOffXch + 2 * kPtXch * 4;
+constexpr size_t kPtOffCnt = kPtOffList + kPtRing * kPtList * 4;
+constexpr size_t kPtOffRInfo = kPtOffCnt + kPtRing * kPtRmax * 4;
+constexpr size_t kPtOffTInfo = kPtOffRInfo + kPtRing * 8 * 4;
+constexpr size_t kPtOffAbort = kPtOffTInfo + 2 * 4 * 4;
+constexpr size_t kPtOffBars = kPtOffAbort + 8;
+constexpr int kPtNumBars = 2 + 2 + 2 * kPtRing;                  // full, tmem_empty, list_full, list_empty
+constexpr size_t kPtOffSlot = kPtOffBars + kPtNumBars * 8;
+constexpr size_t kPtSmemUsed = kPtOffSlot + 16;
+static_assert(kPtOffBars % 8 == 0, "mbarriers need 8-byte alignment");
+
+inline size_t lloyd_pt_smem() { return 1024 + kPtSmemUsed; }
+
+// Instruction descriptor of kind::f16 for N = n (a multiple of 16, <= 256).
+__device__ __forceinline__ uint32_t pt_idesc(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (uint32_t(n >> 3) << 17) | (uint32_t(kTile >> 4) << 24);
+}
+
+__device__ __forceinline__ void pt_mma(uint32_t tmem_d, uint64_t ad, uint64_t bd, uint32_t idesc,
+                                       bool accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(ad), "l"(bd), "r"(idesc), "r"(accumulate ? 1 : 0));
+}
+
+// 16 consecutive fp32 columns of this thread's TMEM lane from column address ta
+__device__ __forceinline__ void tc_ld16(uint32_t ta, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, "
+      "%13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+        "=r"(r[15])
+      : "r"(ta));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void pt_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+// named barrier `id` over `n` threads
+__device__ __forceinline__ void pt_bar(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+// named barrier `id` over `n` threads, returning whether any of them passed true
+__device__ __forceinline__ bool pt_bar_or(int id, int n, bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 q, %1, 0;\n\t"
+      "bar.red.or.pred p, %2, %3, q;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(r)
+      : "r"(v ? 1u : 0u), "r"(id), "r"(n)
+      : "memory");
+  return r != 0u;
+}
+
+// Wait for phase `parity` of bar; false after the bound or once the abort
+// flag is up.
+__device__ __forceinline__ bool pt_wait(uint64_t* bar, uint32_t parity, const volatile uint32_t* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (*abort != 0u || clock64() - t0 > kTcWaitCycles) return false;
+  }
+  return true;
+}
+
+__device__ __forceinline__ void pt_raise(volatile uint32_t* abort, uint32_t* status) {
+  if (*abort == 0u) {
+    *abort = 1u;
+    report_status(status, kStatusWaitTimeout);
+  }
+}
+
+// (x, jx) into a best-two list ordered by (distance, index) with the
+// third-best distance alongside (the lists of different column sets meet here)
+__device__ __forceinline__ void top3_insert_lex(float& d0, int& j0, float& d1, int& j1, float& d2,
+                                                float x, int jx) {
+  const bool c0 = x < d0 || (x == d0 && jx < j0);
+  const bool c1 = x < d1 || (x == d1 && jx < j1);
+  const bool c2 = x < d2;
+  d2 = c1 ? d1 : (c2 ? x : d2);
+  d1 = c0 ? d0 : (c1 ? x : d1);
+  j1 = c0 ? j0 : (c1 ? jx : j1);
+  d0 = c0 ? x : d0;
+  j0 = c0 ? jx : j0;
+}
+
+// another list's best two and third-best distance into (d0, j0, d1, j1, d2)
+__device__ __forceinline__ void top3_merge(float& d0, int& j0, float& d1, int& j1, float& d2,
+                                           float e0, int k0, float e1, int k1, float e2) {
+  top3_insert_lex(d0, j0, d1, j1, d2, e0, k0);
+  top3_insert_lex(d0, j0, d1, j1, d2, e1, k1);
+  d2 = fminf(d2, e2);
+}
+
+// fp32 ||k||^2 of every key row (a warp per row), for the certification
+// bound: 128 products summed in any order stay within 130 u of the sum.
+__global__ void k_key_norm2(const __nv_bfloat16* __restrict__ K, float* __restrict__ out, int64_t rows) {
+  const int64_t row = int64_t(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (row >= rows) return;
+  const int lane = threadIdx.x & 31;
+  const uint2 w = *reinterpret_cast<const uint2*>(K + row * kHeadDim + 4 * lane);
+  const float2 a = bf16x2_to_float2(w.x), b = bf16x2_to_float2(w.y);
+  float s = fmaf(a.x, a.x, fmaf(a.y, a.y, fmaf(b.x, b.x, b.y * b.y)));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if (lane == 0) out[row] = s;
+}
+
+// Nearest centre of every evicted token of the tiles [g0, g1) of the flat
+// (unit, tile) order, g = unit * ntiles + tile (assign: centre index, -1 for
+// tokens outside E), and each tile's member count per centre (hist).  Units
+// with r = 0 are skipped; every unit must have r <= 256; p.knorm2 holds the
+// layer's key norms (k_key_norm2).
+__global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, int n_units) {
+  extern __shared__ uint8_t pt_raw[];
+  uint8_t* base = pt_raw + ((1024u - (smem_u32(pt_raw) & 1023u)) & 1023u);
+  float* cn_s = reinterpret_cast<float*>(base + kPtOffNorm);
+  float* xch = reinterpret_cast<float*>(base + kPtOffXch);        // [2][kPtList]
+  float* lists = reinterpret_cast<float*>(base + kPtOffList);     // [kPtRing][kPtList]
+  int* cnts = reinterpret_cast<int*>(base + kPtOffCnt);           // [kPtRing][kPtRmax]
+  int* rinfo = reinterpret_cast<int*>(base + kPtOffRInfo);        // [kPtRing]: u, tile, r, max ||c||^2
+  int* tinfo = reinterpret_cast<int*>(base + kPtOffTInfo);        // [2]: the same per TMEM buffer
+  volatile uint32_t* abort_s = reinterpret_cast<volatile uint32_t*>(base + kPtOffAbort);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + kPtOffBars);
+  uint64_t* full = bars;                                           // [2] MMA commit + producer lanes
+  uint64_t* tmem_empty = bars + 2;                                 // [2] column threads
+  uint64_t* list_full = bars + 4;                                  // [kPtRing] column half 0
+  uint64_t* list_empty = bars + 4 + kPtRing;                       // [kPtRing] certifier threads
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(base + kPtOffSlot);
+  const uint32_t planes_s = smem_u32(base), keys_s = smem_u32(base + kPtOffKeys);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int64_t n_all = int64_t(n_units) * p.ntiles;
+  const int64_t g0 = n_all * blockIdx.x / gridDim.x, g1 = n_all * (blockIdx.x + 1) / gridDim.x;
+
+  for (int i = tid; i < kPtRing * kPtRmax; i += kPtThreads) cnts[i] = 0;
+  if (tid == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&full[i], 33);
+      mbar_init(&tmem_empty[i], kPtColThreads);
+    }
+    for (int i = 0; i < kPtRing; ++i) {
+      mbar_init(&list_full[i], kPtColThreads / 2);
+      mbar_init(&list_empty[i], kPtCertThreads);
+    }
+    *abort_s = 0u;
+    fence_mbar_init();
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tslot)),
+                 "r"(kPtCols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+
+  if (warp == kPtProducer) {
+    // ---------------- producer ----------------
+    int t = 0, cur_u = -1, n_issued = 0;
+    int pu = 0, ptile = 0, pr = 0;                  // tile t - 1, loaded, MMA not yet issued
+    bool pend = false;
+    float cmx = 0.f;                                 // max ||c||^2 of the staged unit
+    // the MMA chain of tile tt = t - 1 from key buffer tt & 1 (its copies complete)
+    auto issue = [&](int tt) -> bool {
+      const int bb = tt & 1;
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      bool w = tt < 2 || pt_wait(&tmem_empty[bb], uint32_t(((tt - 2) >> 1) & 1), abort_s);
+      if (__any_sync(0xffffffffu, !w)) return false;
+      __syncwarp();
+      if (lane == 0) {
+        tinfo[4 * bb + 0] = pu;
+        tinfo[4 * bb + 1] = ptile;
+        tinfo[4 * bb + 2] = pr;
+        tinfo[4 * bb + 3] = __float_as_int(cmx);
+        tc_fence_after();
+        const uint32_t idesc = pt_idesc((pr + 15) & ~15);
+        const uint32_t d_tmem = tmem + uint32_t(bb) * kPtBufCols;
+        const uint32_t kb = keys_s + uint32_t(bb * kPtKeys);
+#pragma unroll
+        for (int pl = 0; pl < 2; ++pl)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t half = uint32_t(k >> 2), kk = uint32_t(k & 3) * 32u;
+            pt_mma(d_tmem, tc_desc(kb + half * kTcHalf + kk),
+                   tc_desc(planes_s + uint32_t(pl * 2 * kPtPlaneHalf) + half * kPtPlaneHalf + kk), idesc,
+                   pl + k > 0);
+          }
+        tc_commit(&full[bb]);
+      }
+      __syncwarp();
+      pt_arrive(&full[bb]);
+      ++n_issued;
+      return true;
+    };
+    bool ok = true;
+    for (int64_t g = g0; g < g1 && ok; ++g) {
+      const int u = int(g / p.ntiles), tile = int(g % p.ntiles);
+      const int r = p.r_unit[u];
+      if (r <= 0) continue;
+      if (__any_sync(0xffffffffu, *abort_s != 0u)) {
+        ok = false;
+        break;
+      }
+      if (u != cur_u) {
+        // finish the pending tile on the old planes; then wait for its MMAs
+        // (the planes are free) and for the column warps (the norms are free)
+        if (pend) {
+          asm volatile("cp.async.wait_group 0;" ::: "memory");
+          pend = false;
+          if (!(ok = issue(t - 1))) break;
+        }
+        if (t >= 1) {
+          bool w = pt_wait(&full[(t - 1) & 1], uint32_t(((t - 1) >> 1) & 1), abort_s) &&
+                   pt_wait(&tmem_empty[(t - 1) & 1], uint32_t(((t - 1) >> 1) & 1), abort_s);
+          if (__any_sync(0xffffffffu, !w)) {
+            ok = false;
+            break;
+          }
+        }
+        const int rpad = (r + 15) & ~15;
+        const __nv_bfloat16* planes = p.cplanes + int64_t(u) * 2 * p.rmax * kHeadDim;
+        for (int i = lane; i < 2 * rpad * 16; i += 32) {
+          const int pl = i / (rpad * 16), rem = i - pl * (rpad * 16), row = rem >> 4, ch = rem & 15;
+          const bool in = row < r;
+          cp_async16(planes_s + uint32_t(pl * 2 * kPtPlaneHalf + (ch >> 3) * kPtPlaneHalf) + tc_sw128(row, ch & 7),
+                     planes + (int64_t(pl) * p.rmax + (in ? row : 0)) * kHeadDim + 8 * ch, in ? 16u : 0u);
+        }
+        const float* cnorm = p.cnorm + int64_t(u) * p.rmax;
+        cmx = 0.f;
+        for (int i = lane; i < kPtRmax; i += 32) {
+          const float c = i < r ? cnorm[i] : INFINITY;
+          cn_s[i] = c;
+          if (i < r) cmx = fmaxf(cmx, c);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) cmx = fmaxf(cmx, __shfl_xor_sync(0xffffffffu, cmx, o));
+        cur_u = u;
+      }
+      const int b = t & 1;
+      if (t >= 2) {                                  // MMA(t - 2) done: key buffer b is free
+        bool w = pt_wait(&full[b], uint32_t(((t - 2) >> 1) & 1), abort_s);
+        if (__any_sync(0xffffffffu, !w)) {
+          ok = false;
+          break;
+        }
+      }
+      const __nv_bfloat16* Ku = p.K + int64_t(u) * p.s * kHeadDim;
+      const int64_t tok0 = int64_t(tile) * kTile;
+      const uint32_t kb = keys_s + uint32_t(b * kPtKeys);
+      for (int i = lane; i < kTile * 16; i += 32) {
+        const int row = i >> 4, ch = i & 15;
+        const bool in = tok0 + row < p.s;
+        cp_async16(kb + uint32_t((ch >> 3) * kTcHalf) + tc_sw128(row, ch & 7),
+                   Ku + (in ? (tok0 + row) * kHeadDim : 0) + 8 * ch, in ? 16u : 0u);
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+      if (pend) {                                    // tile t - 1's keys have landed
+        asm volatile("cp.async.wait_group 1;" ::: "memory");
+        if (!(ok = issue(t - 1))) break;
+      }
+      pend = true;
+      pu = u;
+      ptile = tile;
+      pr = r;
+      ++t;
+    }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    if (ok && pend) ok = issue(t - 1);
+    if (!ok && lane == 0) pt_raise(abort_s, p.status);
+    // every issued MMA completes before TMEM is freed
+    if (n_issued >= 1) {
+      const int lt = n_issued - 1;
+      const long long t0 = clock64();
+      while (!mbar_try_wait(&full[lt & 1], uint32_t((lt >> 1) & 1)) && clock64() - t0 < kTcWaitCycles) {
+      }
+    }
+  } else if (warp < kPtColWarps) {
+    // ---------------- column warps ----------------
+    const int q = warp & 3, half = warp >> 2, tok = 32 * q + lane;
+    int t = 0;
+    for (int64_t g = g0; g < g1; ++g) {
+      if (p.r_unit[int(g / p.ntiles)] <= 0) continue;
+      const int b = t & 1, slot = t % kPtRing;
+      const bool ok = *abort_s == 0u && pt_wait(&full[b], uint32_t((t >> 1) & 1), abort_s);
+      if (!ok) pt_raise(abort_s, p.status);
+      if (pt_bar_or(1, kPtColThreads, !ok)) break;        // all column threads leave together
+      tc_fence_after();
+      const int r = tinfo[4 * b + 2], rpad = (r + 15) & ~15;
+      const int tu = tinfo[4 * b + 0], ttile = tinfo[4 * b + 1], tcm = tinfo[4 * b + 3];
+      // the token's rank and key norm, loaded now and used after the column loop
+      const int64_t pos = int64_t(ttile) * kTile + tok;
+      int rk = -1;
+      float kn2 = 0.f;
+      if (half == 0 && pos < p.s) {
+        rk = p.rank_pos[int64_t(tu) * p.s + pos];
+        kn2 = p.knorm2[int64_t(tu) * p.s + pos];
+      }
+      // token tok's distances over this half's chunks: lists A (even) and B (odd)
+      float a0 = INFINITY, a1 = INFINITY, a2 = INFINITY, e0 = INFINITY, e1 = INFINITY, e2 = INFINITY;
+      int ja0 = INT_MAX, ja1 = INT_MAX, je0 = INT_MAX, je1 = INT_MAX;
+      const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(b) * kPtBufCols;
+      for (int k = half; k < (rpad >> 4); k += 2) {
+        float v[16];
+        tc_ld16(tb + uint32_t(16 * k), v);
+#pragma unroll
+        for (int i = 0; i < 16; i += 2) {
+          const int col = 16 * k + i;
+          top3_insert(a0, ja0, a1, ja1, a2, fmaf(-2.0f, v[i], cn_s[col]), col);
+          top3_insert(e0, je0, e1, je1, e2, fmaf(-2.0f, v[i + 1], cn_s[col + 1]), col + 1);
+        }
+      }
+      top3_merge(a0, ja0, a1, ja1, a2, e0, je0, e1, je1, e2);
+      tc_fence_before();
+      pt_arrive(&tmem_empty[b]);                          // TMEM buffer b and its tile info are free
+      float* xb = xch + b * kPtXch + tok * 5;
+      if (half == 1) {
+        xb[0] = a0;
+        xb[1] = __int_as_float(ja0);
+        xb[2] = a1;
+        xb[3] = __int_as_float(ja1);
+        xb[4] = a2;
+      }
+      pt_bar(1, kPtColThreads);
+      if (half == 0) {
+        const bool ok2 = t < kPtRing ||
+                         pt_wait(&list_empty[slot], uint32_t(((t / kPtRing) - 1) & 1), abort_s);
+        if (!ok2) {
+          pt_raise(abort_s, p.status);                    // the next tile's vote ends the loop
+        } else {
+          top3_merge(a0, ja0, a1, ja1, a2, xb[0], __float_as_int(xb[1]), xb[2], __float_as_int(xb[3]), xb[4]);
+          float* ls = lists + slot * kPtList + tok * 7;
+          ls[0] = a0;
+          ls[1] = __int_as_float(ja0);
+          ls[2] = a1;
+          ls[3] = __int_as_float(ja1);
+          ls[4] = a2;
+          ls[5] = __int_as_float(rk);
+          ls[6] = kn2;
+          if (tok == 0) {
+            rinfo[8 * slot + 0] = tu;
+            rinfo[8 * slot + 1] = ttile;
+            rinfo[8 * slot + 2] = r;
+            rinfo[8 * slot + 3] = tcm;
+            // ranked main slots of the unit: evicted tokens rank at or past it
+            rinfo[8 * slot + 4] = int(unit_budget(p.budgets, tu, p.budget)) - r - p.recent;
+          }
+          pt_arrive(&list_full[slot]);
+        }
+      }
+      ++t;
+    }
+  } else {
+    // ---------------- certifier warps ----------------
+    const int ct = tid - kPtColThreads;                   // the token of the tile this thread certifies
+    int t = 0;
+    for (int64_t g = g0; g < g1; ++g) {
+      if (p.r_unit[int(g / p.ntiles)] <= 0) continue;
+      const int slot = t % kPtRing;
+      const bool ok = *abort_s == 0u && pt_wait(&list_full[slot], uint32_t((t / kPtRing) & 1), abort_s);
+      if (!ok) pt_raise(abort_s, p.status);
+      if (pt_bar_or(2, kPtCertThreads, !ok)) break;
+      const int u = rinfo[8 * slot + 0], tile = rinfo[8 * slot + 1], r = rinfo[8 * slot + 2];
+      const float cnmax = __int_as_float(rinfo[8 * slot + 3]);
+      const int keep = rinfo[8 * slot + 4];
+      const float* ls = lists + slot * kPtList + ct * 7;
+      const float d0 = ls[0], d1 = ls[2], d2 = ls[4], s2 = ls[6];
+      int j0 = __float_as_int(ls[1]);
+      const int j1 = __float_as_int(ls[3]), rk = __float_as_int(ls[5]);
+      int* cnt = cnts + slot * kPtRmax;
+      const int64_t pos = int64_t(tile) * kTile + ct;
+      const bool mine = pos < p.s;
+      const bool ev = mine && rk >= 0 && rk >= keep;     // in E (in_evicted)
+      bool amb = false, fullscan = false;
+      if (ev) {
+        // the bound of k_lloyd_assign_tc on the computed distances' error
+        const float uu = 5.9604645e-8f, gam = 130.0f * uu, gam_tc = 2048.0f * uu;
+        const float kn = sqrtf(s2) * (1.0f + gam), cm = sqrtf(cnmax);
+        const float ee = 2.0f * (2.0f * gam_tc * cm * kn + 2.0f * gam * cm * cm + 4.0f * uu * kn * cm);
+        const float err0 = ee + 4.0f * uu * fabsf(d0);
+        fullscan = d2 - d0 <= err0 + ee + 4.0f * uu * fabsf(d2);
+        amb = fullscan || (j1 < r && d1 - d0 <= err0 + ee + 4.0f * uu * fabsf(d1));
+        if (j0 >= r) {                                    // only a NaN distance gets here
+          report_status(p.status, kStatusBadIndex);
+          j0 = 0;
+          amb = false;
+        }
+      }
+      if (amb) {
+        // decided by k_lloyd_resolve in fp64; it also counts the token
+        const int i = atomicAdd(p.amb_count, 1);
+        p.amb[i] = make_int4(u, int(pos), j0 | (fullscan ? int(0x80000000u) : 0), j1);
+      } else if (ev) {
+        p.assign[int64_t(u) * p.s + pos] = j0;
+        atomicAdd(&cnt[j0], 1);
+      } else if (mine) {
+        p.assign[int64_t(u) * p.s + pos] = -1;
+      }
+      pt_bar(2, kPtCertThreads);
+      int32_t* h = p.hist + (int64_t(u) * p.ntiles + tile) * p.rmax;
+      for (int i = ct; i < r; i += kPtCertThreads) {
+        h[i] = cnt[i];
+        cnt[i] = 0;
+      }
+      pt_arrive(&list_empty[slot]);
+      ++t;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kPtCols));
+  }
+}
+
+// The decision of the tokens k_lloyd_assign_pt left ambiguous, a warp per
+// token (lane l holds dims 4l..4l+3).  Candidates: the two kept centres, or
+// every centre when the third best was within the tensor-core bound.
+//
+// First their distances are taken directly in fp32, d32_j = sum_i (k_i -
+// c32_i)^2 against the fp32 centres: no cancellation, so the error is small
+// relative to the distance itself.  With u = 2^-24, |d32_j - D_j| <= b_j =
+// 16 u d32_j + 3 u ||c_j|| (sqrt(d32_j) + u ||c_j||) bounds the difference to
+// the exact distance D_j to the fp64 centre (12 u for the rounded differences,
+// the 4-term chain and the 5 butterfly levels; 2 u ||c|| (2 sqrt(D) + u ||c||)
+// for |c32 - c64| <= u ||c||; the rest is slack for using d32 in place of D).
+// The fp32 best decides unless another candidate's interval
+// [d32_j - b_j, d32_j + b_j] reaches the best's; those few are re-evaluated in
+// fp64 as the streaming kernel does, ties to the lower index.  Writes assign
+// and adds the token to its tile's member count.
+constexpr int kResWarps = 8;
+
+__global__ void __launch_bounds__(kResWarps * 32) k_lloyd_resolve(LloydArgs p) {
+  __shared__ float dsm[kResWarps][kPtRmax];       // candidate distances (fp32)
+  __shared__ int jsm[kResWarps][kPtRmax];         // centres left for fp64
+  const int lane = threadIdx.x & 31, wb = threadIdx.x >> 5;
+  float* dl = dsm[wb];
+  int* jl = jsm[wb];
+  const int n = *p.amb_count;
+  const int nw = int((int64_t(gridDim.x) * blockDim.x) >> 5);
+  const float uu = 5.9604645e-8f;
+  for (int i = int((int64_t(blockIdx.x) * blockDim.x + threadIdx.x) >> 5); i < n; i += nw) {
+    const int4 e = p.amb[i];
+    const int u = e.x, r = p.r_unit[u];
+    const int64_t pos = e.y;
+    const bool fs = e.z < 0;
+    const int js0 = e.z & 0x7fffffff, js1 = e.w;
+    const int nc = fs ? r : 2;
+    auto cand = [&](int k) { return fs ? k : (k == 0 ? js0 : js1); };
+    const uint2 kw = *reinterpret_cast<const uint2*>(p.K + (int64_t(u) * p.s + pos) * kHeadDim + 4 * lane);
+    const float2 k01 = bf16x2_to_float2(kw.x), k23 = bf16x2_to_float2(kw.y);
+    const float* c32 = p.centers32 + int64_t(u) * p.rmax * kHeadDim + 4 * lane;
+    const float* cnu = p.cnorm + int64_t(u) * p.rmax;
+    // fp32 distances, four centres at a time
+    for (int k0 = 0; k0 < nc; k0 += 4) {
+      float a[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int k = k0 + q < nc ? k0 + q : k0;
+        const float4 c = *reinterpret_cast<const float4*>(c32 + int64_t(cand(k)) * kHeadDim);
+        const float x0 = k01.x - c.x, x1 = k01.y - c.y, x2 = k23.x - c.z, x3 = k23.y - c.w;
+        a[q] = fmaf(x3, x3, fmaf(x2, x2, fmaf(x1, x1, x0 * x0)));
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) a[q] += __shfl_xor_sync(0xffffffffu, a[q], o);
+      if (lane < 4 && k0 + lane < nc) dl[k0 + lane] = lane == 0 ? a[0] : lane == 1 ? a[1] : lane == 2 ? a[2] : a[3];
+    }
+    __syncwarp();
+    // the fp32 best (distance, index)
+    float bd = INFINITY;
+    int bj = INT_MAX;
+    for (int k = lane; k < nc; k += 32) {
+      const float d = dl[k];
+      const int j = cand(k);
+      if (d < bd || (d == bd && j < bj)) {
+        bd = d;
+        bj = j;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float od = __shfl_xor_sync(0xffffffffu, bd, o);
+      const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+      if (od < bd || (od == bd && oj < bj)) {
+        bd = od;
+        bj = oj;
+      }
+    }
+    auto bound = [&](float d, int j) {
+      const float cn = sqrtf(cnu[j]) * 1.001f;
+      return 16.0f * uu * d + 3.0f * uu * cn * (sqrtf(d) + uu * cn);
+    };
+    int res = bj;
+    if (bj < r) {
+      // centres whose interval reaches the best's: fp64 decides among them
+      const float hi = bd + bound(bd, bj);
+      int na = 0;
+      for (int k0 = 0; k0 < nc; k0 += 32) {
+        const int k = k0 + lane;
+        bool m = false;
+        if (k < nc) {
+          const float d = dl[k];
+          const int j = cand(k);
+          m = j != bj && !(d - bound(d, j) > hi);
+        }
+        const unsigned bal = __ballot_sync(0xffffffffu, m);
+        if (m) jl[na + __popc(bal & ((1u << lane) - 1u))] = cand(k);
+        na += __popc(bal);
+      }
+      __syncwarp();
+      if (na > 0) {
+        const double kx[4] = {k01.x, k01.y, k23.x, k23.y};
+        const double* c64 = p.centers64 + int64_t(u) * p.rmax * kHeadDim + 4 * lane;
+        double bd64 = INFINITY;
+        int bj64 = INT_MAX;
+        // the best first, then the others, four at a time
+        for (int k0 = -1; k0 < na; k0 += 4) {
+          int jq[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) jq[q] = k0 + q < 0 ? bj : (k0 + q < na ? jl[k0 + q] : -1);
+          double a[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const double4_32a c =
+                *reinterpret_cast<const double4_32a*>(c64 + int64_t(jq[q] < 0 ? 0 : jq[q]) * kHeadDim);
+            double tt = (kx[0] - c.x) * (kx[0] - c.x);
+            tt = fma(kx[1] - c.y, kx[1] - c.y, tt);
+            tt = fma(kx[2] - c.z, kx[2] - c.z, tt);
+            a[q] = fma(kx[3] - c.w, kx[3] - c.w, tt);
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) a[q] += __shfl_xor_sync(0xffffffffu, a[q], o);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const double dd = __shfl_sync(0xffffffffu, a[q], 0);
+            if (jq[q] >= 0 && (dd < bd64 || (dd == bd64 && jq[q] < bj64))) {
+              bd64 = dd;
+              bj64 = jq[q];
+            }
+          }
+        }
+        res = bj64;
+      }
+    }
+    if (lane == 0) {
+      if (res >= r) {                                   // only NaN distances get here
+        report_status(p.status, kStatusBadIndex);
+        res = 0;
+      }
+      p.assign[int64_t(u) * p.s + pos] = res;
+      atomicAdd(&p.hist[(int64_t(u) * p.ntiles + pos / kTile) * p.rmax + res], 1);
+    }
+    __syncwarp();                                       // dl / jl are reused by the next token
+  }
+}
+
+}  // namespace build
+}  // namespace reskv

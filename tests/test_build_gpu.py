@@ -250,3 +250,41 @@ def test_keynorm_scores_exact_on_crafted_rows():
     assert scores[0][37 * 4] == 2.0 ** -40
     assert scores[0][37 * 6] == 0.0
     cache.free()
+
+
+def test_lloyd_sums_outside_the_fixed_point_range():
+    """Centre means (Eq. summary) when member values leave the exact
+    fixed-point range of the member sums (multiples of 2^-32 below 128): every
+    key carries a dim of values 2^-40 m (m up to 255), some keys a bf16
+    subnormal, and some values 2^40.  Those centres take the fp64 member-order
+    sums; counts and bf16 entries must match the oracle's Lloyd on the same
+    evicted set, and a missed range check (a truncated or saturated sum) would
+    not."""
+    s, b, P, r = 1024, 256, 64, 8
+    w = wl.scaled(wl.WORKLOADS["small_budget_b64"], seq_len=s, budget=b, batch=1, n_layers=1,
+                  n_kv_heads=2)
+    K, V, _, _ = wl.layer_inputs(w, 0, "cpu")
+    g = np.random.default_rng(7)
+    for h in range(2):
+        m = g.integers(1, 256, size=s) * g.choice([-1.0, 1.0], size=s)
+        K[0, h, :, 5] = torch.from_numpy(m * 2.0 ** -40).to(torch.bfloat16)
+        K[0, h, ::97, 9] = 2.0 ** -133
+        V[0, h, 3::41, 7] = 2.0 ** 40
+        assert torch.all(K[0, h, :, 5].double() == torch.from_numpy(m * 2.0 ** -40))
+    cfg = R.reskv_config_default(batch=1, n_layers=1, n_kv_heads=2, group=w.group, seq_len=s,
+                                 budget=b, recent_window=P, n_obs=0, n_fit=0, n_val=0,
+                                 score_mode=R.RESKV_SCORE_KEYNORM,
+                                 residual_override=np.full(2, r, np.int32), keep_debug=1)
+    cache = R.reskv_build_cache(cfg, [K.cuda()], [V.cuda()], None)
+    torch.cuda.synchronize()
+    R.reskv_check_status(cache)
+    lay = R.reskv_export_cache(cache)
+    top = R.reskv_export_debug(cache, R.RESKV_DEBUG_RANKED)
+    big = 0
+    for h in range(2):
+        gu = unit_from_layout(lay, h)
+        assert gu.r == r
+        check_entries(gu, bf16_to_f64(K[0, h]), bf16_to_f64(V[0, h]), top[h], P, s, b, 4)
+        big += int(np.sum(np.abs(gu.vbar[:, 7]) > 2.0 ** 20))
+    assert big > 0                       # some centre holds a 2^40 value
+    cache.free()
