@@ -373,7 +373,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   const size_t sm_val = size_t(kHeadDim) * (2 * kTile + 2 * kRowBlk) * 4;
   if (set_smem(k_obs_pass1, sm_obs1) != cudaSuccess || set_smem(k_obs_pass2, sm_obs2) != cudaSuccess ||
       set_smem(k_topk, sm_top) != cudaSuccess || set_smem(k_lloyd_assign_tc, sm_assign) != cudaSuccess ||
-      set_smem(k_lloyd_assign_pt, lloyd_pt_smem()) != cudaSuccess ||
+      set_smem(k_lloyd_assign_pt, kPtSmemMax) != cudaSuccess ||
       set_smem(k_val_full, sm_val) != cudaSuccess)
     return cleanup_fail(fail(RESKV_ERR_CUDA, "setting kernel shared-memory limits"));
 
@@ -458,6 +458,10 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
                  ent_stride, 0, c->status, bl_d, cplanes, msum, mflag, knorm2, amb, amb_count, centers32};
     if (rmax > 0)
       k_key_norm2<<<unsigned(cdiv(int64_t(US), 8)), 256, 0, stream>>>(K, knorm2, int64_t(US));
+    // the persistent assignment loads key tiles by TMA (a 16-byte aligned
+    // base and at least one whole tile of rows); otherwise the streaming form
+    CUtensorMap tmK;
+    const bool pt_keys = rmax > 0 && US >= size_t(kTile) && encode_key_tiles(&tmK, K, uint64_t(US));
     auto lloyd_run = [&](const int32_t* r_unit, int ent_off, int r_hi) -> reskv_status {
       la.r_unit = r_unit;
       la.ent_off = ent_off;
@@ -466,10 +470,12 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       const unsigned pt_grid = unsigned(std::min<int64_t>(c->num_sms, int64_t(UL) * ntiles));
       k_lloyd_init<<<dim3(gr, UL), kHeadDim, 0, stream>>>(la);
       for (int it = 0; it < cfg.lloyd_iters; ++it) {
-        if (r_hi <= kPtRmax) {        // the centres fit in shared memory: persistent form
+        if (pt_keys && r_hi <= kPtRmax) {   // the centres fit in shared memory: persistent form
           if (cudaMemsetAsync(amb_count, 0, sizeof(int), stream) != cudaSuccess)
             return fail(RESKV_ERR_CUDA, "clearing the ambiguous-token count");
-          k_lloyd_assign_pt<<<pt_grid, kPtThreads, lloyd_pt_smem(), stream>>>(la, UL);
+          const int rp = (r_hi + 15) & ~15;
+          k_lloyd_assign_pt<<<pt_grid, kPtThreads, lloyd_pt_smem(rp), stream>>>(la, UL, rp,
+                                                                                 lloyd_pt_key_bufs(rp), tmK);
           k_lloyd_resolve<<<unsigned(4 * c->num_sms), kResWarps * 32, 0, stream>>>(la);
         } else {
           k_lloyd_assign_tc<<<dim3(ntiles, UL), kTcThreads, sm_assign, stream>>>(la);

@@ -125,6 +125,9 @@ MmaPlan plan_mma_shape(int num_sms, int64_t max_warps, int32_t user_warps, int64
 // rank 2: two copies, box {64 dims, 16 rows} at dims 0 and 64.  False if the
 // driver refuses the map.
 bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, int rank);
+// 128-row tiles of a [rows, 128] bf16 key array, both 64-dim halves in one
+// copy, 128-byte swizzle (the Lloyd assignment's key tiles)
+bool encode_key_tiles(CUtensorMap* map, const void* keys, uint64_t rows);
 
 }  // namespace reskv
 

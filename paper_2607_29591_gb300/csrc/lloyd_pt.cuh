@@ -4,13 +4,16 @@
 // shared memory, so a tile costs one key-tile load and one tcgen05.mma chain.
 // Three roles run decoupled, linked by mbarrier rings:
 //
-//   producer warp    loads key tile t into buffer t & 1 (cp.async, 128-byte
-//                    swizzle) one tile ahead, and issues the MMA chain of
-//                    tile t - 1 (2 planes x 8 K-steps, M = 128 tokens, N = r
-//                    rounded up to 16) into TMEM columns 256 ((t - 1) & 1) ..,
-//                    committed to full[].  At a change of unit it waits for
-//                    every earlier MMA and for the column warps to be done with
-//                    the old centre norms, then stages the new planes.
+//   producer warp    loads key tiles by TMA (both 64-dim halves, 128-byte
+//                    swizzle, one 32 KB copy) into a ring of nk buffers, up to
+//                    nk tiles ahead and across unit changes (key_full[]); for
+//                    each tile it issues the MMA chain of all the unit's
+//                    centres (2 planes x 8 K-steps, M = 128 tokens, N = r
+//                    rounded up to 16) into TMEM columns 256 (t & 1) ..,
+//                    committed to full[] and to the key buffer's key_free[].
+//                    At a change of unit it waits for every earlier MMA and
+//                    for the column warps to be done with the old centre
+//                    norms, then stages the new planes (cp.async).
 //   8 column warps   warp w reads TMEM lanes 32 (w % 4).. (its tokens) and the
 //                    16-column chunks w / 4, w / 4 + 2, .. of the distances,
 //                    keeping two top-3 lists per thread (even and odd columns:
@@ -29,9 +32,12 @@
 // kStatusWaitTimeout and an abort flag, and each role leaves its loop at a
 // tile boundary agreed by a barrier reduction over the role's threads.
 #pragma once
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
+#include <cfloat>
 #include <cstdint>
 
 #include "lloyd_tc.cuh"
@@ -47,19 +53,19 @@ constexpr int kPtProducer = kPtColWarps + kPtCertWarps;        // the producer w
 constexpr int kPtThreads = (kPtProducer + 1) * 32;
 constexpr int kPtRmax = 256;                                    // centres held resident
 constexpr int kPtRing = 4;                                      // list slots
-constexpr int kPtPlaneHalf = kPtRmax * 128;                     // one 64-dim half of a plane, bytes
-constexpr int kPtPlanes = 2 * 2 * kPtPlaneHalf;                 // both planes
 constexpr int kPtKeys = 2 * kTcHalf;                            // one key tile
 constexpr uint32_t kPtBufCols = 256;                            // TMEM columns per buffer
 constexpr uint32_t kPtCols = 2 * kPtBufCols;
-constexpr int kPtXch = kTile * 5;                               // floats: d0, j0, d1, j1, d2 per token
-constexpr int kPtList = kTile * 7;                              // the same, + rank, ||k||^2
+constexpr int kPtXch = kTile * 3;                               // a token's three best keys
+constexpr int kPtList = kTile * 5;                              // the same, + rank, ||k||^2
 
-// Shared memory (from a 1024-aligned base): planes, 2 key tiles, centre
-// norms, 2 x the column halves' exchange lists, the ring (lists, counts,
-// info), 2 x TMEM tile info, the abort flag, mbarriers, the TMEM address.
-constexpr size_t kPtOffKeys = kPtPlanes;
-constexpr size_t kPtOffNorm = kPtOffKeys + 2 * size_t(kPtKeys);
+// Shared memory, from a 1024-aligned base: the planes of rp = r rounded up
+// to 16 centres ([plane][64-dim half][rp rows][128 B], 512 rp bytes), nk key
+// tiles of 32 KB, then a tail of fixed size: centre norms, 2 x the column
+// halves' exchange keys, the ring (lists, counts, info), 2 x TMEM tile info,
+// the abort flag, the mbarriers and the TMEM address.
+constexpr int kPtMaxKeyBufs = 4;
+constexpr size_t kPtOffNorm = 0;
 constexpr size_t kPtOffXch = kPtOffNorm + kPtRmax * 4;
 constexpr size_t kPtOffList = kPtOffXch + 2 * kPtXch * 4;
 constexpr size_t kPtOffCnt = kPtOffList + kPtRing * kPtList * 4;
@@ -67,12 +73,22 @@ constexpr size_t kPtOffRInfo = kPtOffCnt + kPtRing * kPtRmax * 4;
 constexpr size_t kPtOffTInfo = kPtOffRInfo + kPtRing * 8 * 4;
 constexpr size_t kPtOffAbort = kPtOffTInfo + 2 * 4 * 4;
 constexpr size_t kPtOffBars = kPtOffAbort + 8;
-constexpr int kPtNumBars = 2 + 2 + 2 * kPtRing;                  // full, tmem_empty, list_full, list_empty
+// full, tmem_empty (2 each), list_full, list_empty (ring), key_full, key_free (key buffers)
+constexpr int kPtNumBars = 2 + 2 + 2 * kPtRing + 2 * kPtMaxKeyBufs;
 constexpr size_t kPtOffSlot = kPtOffBars + kPtNumBars * 8;
-constexpr size_t kPtSmemUsed = kPtOffSlot + 16;
+constexpr size_t kPtTail = kPtOffSlot + 16;
 static_assert(kPtOffBars % 8 == 0, "mbarriers need 8-byte alignment");
+constexpr size_t kPtSmemMax = 232448;                  // 227 KB of opt-in shared memory per CTA
 
-inline size_t lloyd_pt_smem() { return 1024 + kPtSmemUsed; }
+__host__ __device__ inline size_t lloyd_pt_planes(int rp) { return size_t(rp) * 512; }
+// key buffers that fit beside the planes of rp centres (>= 2 for rp <= 256)
+inline int lloyd_pt_key_bufs(int rp) {
+  const size_t room = kPtSmemMax - 1024 - kPtTail - lloyd_pt_planes(rp);
+  return int(std::min<size_t>(kPtMaxKeyBufs, room / kPtKeys));
+}
+inline size_t lloyd_pt_smem(int rp) {
+  return 1024 + lloyd_pt_planes(rp) + size_t(lloyd_pt_key_bufs(rp)) * kPtKeys + kPtTail;
+}
 
 // Instruction descriptor of kind::f16 for N = n (a multiple of 16, <= 256).
 __device__ __forceinline__ uint32_t pt_idesc(int n) {
@@ -100,6 +116,16 @@ __device__ __forceinline__ void tc_ld16(uint32_t ta, float (&v)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// one 128-token key tile (both 64-dim halves, 128-byte swizzle) from row y
+// of the layer's keys, completing on bar
+__device__ __forceinline__ void tma_keys(uint32_t dst, const CUtensorMap* map, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::
+          "r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(y), "r"(0), "r"(smem_u32(bar))
+      : "memory");
 }
 
 __device__ __forceinline__ void pt_arrive(uint64_t* bar) {
@@ -163,6 +189,23 @@ __device__ __forceinline__ void top3_merge(float& d0, int& j0, float& d1, int& j
   d2 = fminf(d2, e2);
 }
 
+// A distance with the centre index in its 8 low significand bits (r <= 256):
+// keys order like the distances up to |key - d| <= 2^-15 |d|, and distinct
+// centres never tie, so three fminf / fmaxf pairs keep a token's best three.
+__device__ __forceinline__ float pt_key(float d, int col) {
+  return __int_as_float((__float_as_int(d) & ~0xFF) | col);
+}
+__device__ __forceinline__ int pt_key_index(float key) { return __float_as_int(key) & 0xFF; }
+
+// key into the ascending best three (x0, x1, x2)
+__device__ __forceinline__ void pt_ins3(float& x0, float& x1, float& x2, float key) {
+  const float t0 = fmaxf(x0, key);
+  x0 = fminf(x0, key);
+  const float t1 = fmaxf(x1, t0);
+  x1 = fminf(x1, t0);
+  x2 = fminf(x2, t1);
+}
+
 // fp32 ||k||^2 of every key row (a warp per row), for the certification
 // bound: 128 products summed in any order stay within 130 u of the sum.
 __global__ void k_key_norm2(const __nv_bfloat16* __restrict__ K, float* __restrict__ out, int64_t rows) {
@@ -182,23 +225,28 @@ __global__ void k_key_norm2(const __nv_bfloat16* __restrict__ K, float* __restri
 // tokens outside E), and each tile's member count per centre (hist).  Units
 // with r = 0 are skipped; every unit must have r <= 256; p.knorm2 holds the
 // layer's key norms (k_key_norm2).
-__global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, int n_units) {
+__global__ void __launch_bounds__(kPtThreads, 1)
+    k_lloyd_assign_pt(LloydArgs p, int n_units, int rp_max, int nk, const __grid_constant__ CUtensorMap tmK) {
   extern __shared__ uint8_t pt_raw[];
   uint8_t* base = pt_raw + ((1024u - (smem_u32(pt_raw) & 1023u)) & 1023u);
-  float* cn_s = reinterpret_cast<float*>(base + kPtOffNorm);
-  float* xch = reinterpret_cast<float*>(base + kPtOffXch);        // [2][kPtList]
-  float* lists = reinterpret_cast<float*>(base + kPtOffList);     // [kPtRing][kPtList]
-  int* cnts = reinterpret_cast<int*>(base + kPtOffCnt);           // [kPtRing][kPtRmax]
-  int* rinfo = reinterpret_cast<int*>(base + kPtOffRInfo);        // [kPtRing]: u, tile, r, max ||c||^2
-  int* tinfo = reinterpret_cast<int*>(base + kPtOffTInfo);        // [2]: the same per TMEM buffer
-  volatile uint32_t* abort_s = reinterpret_cast<volatile uint32_t*>(base + kPtOffAbort);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(base + kPtOffBars);
+  const uint32_t plane_half = uint32_t(rp_max) * 128u;           // one plane's 64-dim half, bytes
+  uint8_t* tail = base + lloyd_pt_planes(rp_max) + size_t(nk) * kPtKeys;
+  float* cn_s = reinterpret_cast<float*>(tail + kPtOffNorm);
+  float* xch = reinterpret_cast<float*>(tail + kPtOffXch);        // [2][kPtXch]
+  float* lists = reinterpret_cast<float*>(tail + kPtOffList);     // [kPtRing][kPtList]
+  int* cnts = reinterpret_cast<int*>(tail + kPtOffCnt);           // [kPtRing][kPtRmax]
+  int* rinfo = reinterpret_cast<int*>(tail + kPtOffRInfo);        // [kPtRing]: u, tile, r, max ||c||^2, keep
+  int* tinfo = reinterpret_cast<int*>(tail + kPtOffTInfo);        // [2]: u, tile, r, max ||c||^2
+  volatile uint32_t* abort_s = reinterpret_cast<volatile uint32_t*>(tail + kPtOffAbort);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(tail + kPtOffBars);
   uint64_t* full = bars;                                           // [2] MMA commit + producer lanes
   uint64_t* tmem_empty = bars + 2;                                 // [2] column threads
   uint64_t* list_full = bars + 4;                                  // [kPtRing] column half 0
   uint64_t* list_empty = bars + 4 + kPtRing;                       // [kPtRing] certifier threads
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(base + kPtOffSlot);
-  const uint32_t planes_s = smem_u32(base), keys_s = smem_u32(base + kPtOffKeys);
+  uint64_t* key_full = bars + 4 + 2 * kPtRing;                     // [nk] the key tile's TMA bytes
+  uint64_t* key_free = key_full + kPtMaxKeyBufs;                   // [nk] MMA commit: buffer read
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(tail + kPtOffSlot);
+  const uint32_t planes_s = smem_u32(base), keys_s = planes_s + uint32_t(lloyd_pt_planes(rp_max));
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int64_t n_all = int64_t(n_units) * p.ntiles;
   const int64_t g0 = n_all * blockIdx.x / gridDim.x, g1 = n_all * (blockIdx.x + 1) / gridDim.x;
@@ -212,6 +260,10 @@ __global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, 
     for (int i = 0; i < kPtRing; ++i) {
       mbar_init(&list_full[i], kPtColThreads / 2);
       mbar_init(&list_empty[i], kPtCertThreads);
+    }
+    for (int i = 0; i < nk; ++i) {
+      mbar_init(&key_full[i], 1);
+      mbar_init(&key_free[i], 1);
     }
     *abort_s = 0u;
     fence_mbar_init();
@@ -228,62 +280,47 @@ __global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, 
 
   if (warp == kPtProducer) {
     // ---------------- producer ----------------
-    int t = 0, cur_u = -1, n_issued = 0;
-    int pu = 0, ptile = 0, pr = 0;                  // tile t - 1, loaded, MMA not yet issued
-    bool pend = false;
+    // Two cursors over the tiles: gl, the next key tile to load (up to nk
+    // ahead, across unit changes too), and gm, the next tile to compute.
+    int64_t gl = g0, gm = g0;
+    int nl = 0, nm = 0, cur_u = -1;
     float cmx = 0.f;                                 // max ||c||^2 of the staged unit
-    // the MMA chain of tile tt = t - 1 from key buffer tt & 1 (its copies complete)
-    auto issue = [&](int tt) -> bool {
-      const int bb = tt & 1;
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      bool w = tt < 2 || pt_wait(&tmem_empty[bb], uint32_t(((tt - 2) >> 1) & 1), abort_s);
-      if (__any_sync(0xffffffffu, !w)) return false;
-      __syncwarp();
-      if (lane == 0) {
-        tinfo[4 * bb + 0] = pu;
-        tinfo[4 * bb + 1] = ptile;
-        tinfo[4 * bb + 2] = pr;
-        tinfo[4 * bb + 3] = __float_as_int(cmx);
-        tc_fence_after();
-        const uint32_t idesc = pt_idesc((pr + 15) & ~15);
-        const uint32_t d_tmem = tmem + uint32_t(bb) * kPtBufCols;
-        const uint32_t kb = keys_s + uint32_t(bb * kPtKeys);
-#pragma unroll
-        for (int pl = 0; pl < 2; ++pl)
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const uint32_t half = uint32_t(k >> 2), kk = uint32_t(k & 3) * 32u;
-            pt_mma(d_tmem, tc_desc(kb + half * kTcHalf + kk),
-                   tc_desc(planes_s + uint32_t(pl * 2 * kPtPlaneHalf) + half * kPtPlaneHalf + kk), idesc,
-                   pl + k > 0);
-          }
-        tc_commit(&full[bb]);
-      }
-      __syncwarp();
-      pt_arrive(&full[bb]);
-      ++n_issued;
-      return true;
-    };
     bool ok = true;
-    for (int64_t g = g0; g < g1 && ok; ++g) {
-      const int u = int(g / p.ntiles), tile = int(g % p.ntiles);
-      const int r = p.r_unit[u];
-      if (r <= 0) continue;
-      if (__any_sync(0xffffffffu, *abort_s != 0u)) {
-        ok = false;
-        break;
-      }
-      if (u != cur_u) {
-        // finish the pending tile on the old planes; then wait for its MMAs
-        // (the planes are free) and for the column warps (the norms are free)
-        if (pend) {
-          asm volatile("cp.async.wait_group 0;" ::: "memory");
-          pend = false;
-          if (!(ok = issue(t - 1))) break;
+    auto next_live = [&](int64_t g) {                // the first tile at or after g with r > 0
+      while (g < g1 && p.r_unit[int(g / p.ntiles)] <= 0) ++g;
+      return g;
+    };
+    gl = next_live(gl);
+    gm = next_live(gm);
+    while (gm < g1 && ok) {
+      // key tiles ahead, while a buffer is free
+      while (gl < g1 && nl - nm < nk) {
+        const int slot = nl % nk;
+        if (nl >= nk) {                              // MMA(nl - nk) has read the buffer
+          bool w = pt_wait(&key_free[slot], uint32_t(((nl / nk) - 1) & 1), abort_s);
+          if (__any_sync(0xffffffffu, !w)) {
+            ok = false;
+            break;
+          }
         }
-        if (t >= 1) {
-          bool w = pt_wait(&full[(t - 1) & 1], uint32_t(((t - 1) >> 1) & 1), abort_s) &&
-                   pt_wait(&tmem_empty[(t - 1) & 1], uint32_t(((t - 1) >> 1) & 1), abort_s);
+        if (lane == 0) {
+          const int u = int(gl / p.ntiles), tile = int(gl % p.ntiles);
+          mbar_arrive_expect_tx(&key_full[slot], uint32_t(kPtKeys));
+          tma_keys(keys_s + uint32_t(slot * kPtKeys), &tmK, int(int64_t(u) * p.s + int64_t(tile) * kTile),
+                   &key_full[slot]);
+        }
+        ++nl;
+        gl = next_live(gl + 1);
+      }
+      if (!ok) break;
+      const int u = int(gm / p.ntiles), tile = int(gm % p.ntiles);
+      const int r = p.r_unit[u];
+      if (u != cur_u) {
+        // the planes and norms of the old unit are in use until its last
+        // tile's MMAs are done and the column warps have read that tile
+        if (nm >= 1) {
+          bool w = pt_wait(&full[(nm - 1) & 1], uint32_t(((nm - 1) >> 1) & 1), abort_s) &&
+                   pt_wait(&tmem_empty[(nm - 1) & 1], uint32_t(((nm - 1) >> 1) & 1), abort_s);
           if (__any_sync(0xffffffffu, !w)) {
             ok = false;
             break;
@@ -294,55 +331,66 @@ __global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, 
         for (int i = lane; i < 2 * rpad * 16; i += 32) {
           const int pl = i / (rpad * 16), rem = i - pl * (rpad * 16), row = rem >> 4, ch = rem & 15;
           const bool in = row < r;
-          cp_async16(planes_s + uint32_t(pl * 2 * kPtPlaneHalf + (ch >> 3) * kPtPlaneHalf) + tc_sw128(row, ch & 7),
+          cp_async16(planes_s + uint32_t(pl * 2) * plane_half + uint32_t(ch >> 3) * plane_half + tc_sw128(row, ch & 7),
                      planes + (int64_t(pl) * p.rmax + (in ? row : 0)) * kHeadDim + 8 * ch, in ? 16u : 0u);
         }
+        asm volatile("cp.async.commit_group;" ::: "memory");
         const float* cnorm = p.cnorm + int64_t(u) * p.rmax;
         cmx = 0.f;
         for (int i = lane; i < kPtRmax; i += 32) {
-          const float c = i < r ? cnorm[i] : INFINITY;
+          const float c = i < r ? cnorm[i] : FLT_MAX;    // finite: padded keys stay ordered
           cn_s[i] = c;
           if (i < r) cmx = fmaxf(cmx, c);
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) cmx = fmaxf(cmx, __shfl_xor_sync(0xffffffffu, cmx, o));
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         cur_u = u;
       }
-      const int b = t & 1;
-      if (t >= 2) {                                  // MMA(t - 2) done: key buffer b is free
-        bool w = pt_wait(&full[b], uint32_t(((t - 2) >> 1) & 1), abort_s);
-        if (__any_sync(0xffffffffu, !w)) {
-          ok = false;
-          break;
-        }
+      // tile nm: its keys, a free TMEM buffer, then the MMA chain
+      const int slot = nm % nk, bb = nm & 1;
+      bool w = pt_wait(&key_full[slot], uint32_t((nm / nk) & 1), abort_s) &&
+               (nm < 2 || pt_wait(&tmem_empty[bb], uint32_t(((nm - 2) >> 1) & 1), abort_s));
+      if (__any_sync(0xffffffffu, !w)) {
+        ok = false;
+        break;
       }
-      const __nv_bfloat16* Ku = p.K + int64_t(u) * p.s * kHeadDim;
-      const int64_t tok0 = int64_t(tile) * kTile;
-      const uint32_t kb = keys_s + uint32_t(b * kPtKeys);
-      for (int i = lane; i < kTile * 16; i += 32) {
-        const int row = i >> 4, ch = i & 15;
-        const bool in = tok0 + row < p.s;
-        cp_async16(kb + uint32_t((ch >> 3) * kTcHalf) + tc_sw128(row, ch & 7),
-                   Ku + (in ? (tok0 + row) * kHeadDim : 0) + 8 * ch, in ? 16u : 0u);
+      __syncwarp();
+      if (lane == 0) {
+        tinfo[4 * bb + 0] = u;
+        tinfo[4 * bb + 1] = tile;
+        tinfo[4 * bb + 2] = r;
+        tinfo[4 * bb + 3] = __float_as_int(cmx);
+        tc_fence_after();
+        const uint32_t idesc = pt_idesc((r + 15) & ~15);
+        const uint32_t d_tmem = tmem + uint32_t(bb) * kPtBufCols;
+        const uint32_t kb = keys_s + uint32_t(slot * kPtKeys);
+#pragma unroll
+        for (int pl = 0; pl < 2; ++pl)
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t half = uint32_t(k >> 2), kk = uint32_t(k & 3) * 32u;
+            pt_mma(d_tmem, tc_desc(kb + half * kTcHalf + kk),
+                   tc_desc(planes_s + uint32_t(pl * 2 + half) * plane_half + kk), idesc, pl + k > 0);
+          }
+        tc_commit(&full[bb]);
+        tc_commit(&key_free[slot]);
       }
-      asm volatile("cp.async.commit_group;" ::: "memory");
-      if (pend) {                                    // tile t - 1's keys have landed
-        asm volatile("cp.async.wait_group 1;" ::: "memory");
-        if (!(ok = issue(t - 1))) break;
-      }
-      pend = true;
-      pu = u;
-      ptile = tile;
-      pr = r;
-      ++t;
+      __syncwarp();
+      pt_arrive(&full[bb]);
+      ++nm;
+      gm = next_live(gm + 1);
     }
-    asm volatile("cp.async.wait_group 0;" ::: "memory");
-    if (ok && pend) ok = issue(t - 1);
     if (!ok && lane == 0) pt_raise(abort_s, p.status);
-    // every issued MMA completes before TMEM is freed
-    if (n_issued >= 1) {
-      const int lt = n_issued - 1;
-      const long long t0 = clock64();
+    // every issued copy and MMA completes before the CTA exits
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    const long long t0 = clock64();
+    for (int i = nm; i < nl; ++i)                    // key tiles loaded but never computed
+      while (!mbar_try_wait(&key_full[i % nk], uint32_t((i / nk) & 1)) && clock64() - t0 < kTcWaitCycles) {
+      }
+    if (nm >= 1) {
+      const int lt = nm - 1;
       while (!mbar_try_wait(&full[lt & 1], uint32_t((lt >> 1) & 1)) && clock64() - t0 < kTcWaitCycles) {
       }
     }
@@ -369,7 +417,6 @@ __global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, 
       }
       // token tok's distances over this half's chunks: lists A (even) and B (odd)
       float a0 = INFINITY, a1 = INFINITY, a2 = INFINITY, e0 = INFINITY, e1 = INFINITY, e2 = INFINITY;
-      int ja0 = INT_MAX, ja1 = INT_MAX, je0 = INT_MAX, je1 = INT_MAX;
       const uint32_t tb = tmem + (uint32_t(32 * q) << 16) + uint32_t(b) * kPtBufCols;
       for (int k = half; k < (rpad >> 4); k += 2) {
         float v[16];
@@ -377,20 +424,20 @@ __global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, 
 #pragma unroll
         for (int i = 0; i < 16; i += 2) {
           const int col = 16 * k + i;
-          top3_insert(a0, ja0, a1, ja1, a2, fmaf(-2.0f, v[i], cn_s[col]), col);
-          top3_insert(e0, je0, e1, je1, e2, fmaf(-2.0f, v[i + 1], cn_s[col + 1]), col + 1);
+          pt_ins3(a0, a1, a2, pt_key(fmaf(-2.0f, v[i], cn_s[col]), col));
+          pt_ins3(e0, e1, e2, pt_key(fmaf(-2.0f, v[i + 1], cn_s[col + 1]), col + 1));
         }
       }
-      top3_merge(a0, ja0, a1, ja1, a2, e0, je0, e1, je1, e2);
+      pt_ins3(a0, a1, a2, e0);
+      pt_ins3(a0, a1, a2, e1);
+      pt_ins3(a0, a1, a2, e2);
       tc_fence_before();
       pt_arrive(&tmem_empty[b]);                          // TMEM buffer b and its tile info are free
-      float* xb = xch + b * kPtXch + tok * 5;
+      float* xb = xch + b * kPtXch + tok * 3;
       if (half == 1) {
         xb[0] = a0;
-        xb[1] = __int_as_float(ja0);
-        xb[2] = a1;
-        xb[3] = __int_as_float(ja1);
-        xb[4] = a2;
+        xb[1] = a1;
+        xb[2] = a2;
       }
       pt_bar(1, kPtColThreads);
       if (half == 0) {
@@ -399,15 +446,15 @@ __global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, 
         if (!ok2) {
           pt_raise(abort_s, p.status);                    // the next tile's vote ends the loop
         } else {
-          top3_merge(a0, ja0, a1, ja1, a2, xb[0], __float_as_int(xb[1]), xb[2], __float_as_int(xb[3]), xb[4]);
-          float* ls = lists + slot * kPtList + tok * 7;
+          pt_ins3(a0, a1, a2, xb[0]);
+          pt_ins3(a0, a1, a2, xb[1]);
+          pt_ins3(a0, a1, a2, xb[2]);
+          float* ls = lists + slot * kPtList + tok * 5;
           ls[0] = a0;
-          ls[1] = __int_as_float(ja0);
-          ls[2] = a1;
-          ls[3] = __int_as_float(ja1);
-          ls[4] = a2;
-          ls[5] = __int_as_float(rk);
-          ls[6] = kn2;
+          ls[1] = a1;
+          ls[2] = a2;
+          ls[3] = __int_as_float(rk);
+          ls[4] = kn2;
           if (tok == 0) {
             rinfo[8 * slot + 0] = tu;
             rinfo[8 * slot + 1] = ttile;
@@ -434,10 +481,10 @@ __global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, 
       const int u = rinfo[8 * slot + 0], tile = rinfo[8 * slot + 1], r = rinfo[8 * slot + 2];
       const float cnmax = __int_as_float(rinfo[8 * slot + 3]);
       const int keep = rinfo[8 * slot + 4];
-      const float* ls = lists + slot * kPtList + ct * 7;
-      const float d0 = ls[0], d1 = ls[2], d2 = ls[4], s2 = ls[6];
-      int j0 = __float_as_int(ls[1]);
-      const int j1 = __float_as_int(ls[3]), rk = __float_as_int(ls[5]);
+      const float* ls = lists + slot * kPtList + ct * 5;
+      const float d0 = ls[0], d1 = ls[1], d2 = ls[2], s2 = ls[4];
+      int j0 = pt_key_index(d0);
+      const int j1 = pt_key_index(d1), rk = __float_as_int(ls[3]);
       int* cnt = cnts + slot * kPtRmax;
       const int64_t pos = int64_t(tile) * kTile + ct;
       const bool mine = pos < p.s;
@@ -448,10 +495,12 @@ __global__ void __launch_bounds__(kPtThreads, 1) k_lloyd_assign_pt(LloydArgs p, 
         const float uu = 5.9604645e-8f, gam = 130.0f * uu, gam_tc = 2048.0f * uu;
         const float kn = sqrtf(s2) * (1.0f + gam), cm = sqrtf(cnmax);
         const float ee = 2.0f * (2.0f * gam_tc * cm * kn + 2.0f * gam * cm * cm + 4.0f * uu * kn * cm);
-        const float err0 = ee + 4.0f * uu * fabsf(d0);
-        fullscan = d2 - d0 <= err0 + ee + 4.0f * uu * fabsf(d2);
-        amb = fullscan || (j1 < r && d1 - d0 <= err0 + ee + 4.0f * uu * fabsf(d1));
-        if (j0 >= r) {                                    // only a NaN distance gets here
+        // + the key packing: |key - d| <= 2^-15 |d|
+        const float pk = 0x1p-15f;
+        const float err0 = ee + (4.0f * uu + pk) * fabsf(d0);
+        fullscan = d2 - d0 <= err0 + ee + (4.0f * uu + pk) * fabsf(d2);
+        amb = fullscan || (j1 < r && d1 - d0 <= err0 + ee + (4.0f * uu + pk) * fabsf(d1));
+        if (j0 >= r || !(d0 < INFINITY)) {                // only NaN or infinite distances get here
           report_status(p.status, kStatusBadIndex);
           j0 = 0;
           amb = false;

@@ -316,6 +316,18 @@ bool encode_rows(CUtensorMap* map, const void* base, uint64_t rows, int rank) {
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool encode_key_tiles(CUtensorMap* map, const void* keys, uint64_t rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint32_t estr[3] = {1, 1, 1};
+  const cuuint64_t dims[3] = {64, cuuint64_t(rows), 2};
+  const cuuint64_t strides[2] = {cuuint64_t(kHeadDim) * 2, 128};
+  const cuuint32_t box[3] = {64, 128, 2};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(keys), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // At most 7 warps per SM: 7 x 2 ring stages streamed the 32-layer 32K cache
 // 1 % faster than 8 x 2 and 8 x 3.
 constexpr int kMmaWarpsPerCta = 7;
