@@ -484,11 +484,9 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
         k_lloyd_scatter<<<dim3(ntiles, UL), kTile, 0, stream>>>(la);
         const int last = it == cfg.lloyd_iters - 1;
         const dim3 ga(unsigned(cdiv(s, int64_t(kAccRows))), UL);
-        if (last)
-          k_lloyd_accum<true><<<ga, kThreads, 0, stream>>>(la);
-        else
-          k_lloyd_accum<false><<<ga, kThreads, 0, stream>>>(la);
-        k_lloyd_finish<<<dim3(gr, UL), kHeadDim, 0, stream>>>(la, last);
+        k_lloyd_accum<false><<<ga, kThreads, 0, stream>>>(la);
+        if (last) k_lloyd_accum<true><<<ga, kThreads, 0, stream>>>(la);
+        k_lloyd_finish<<<dim3(unsigned(cdiv(int64_t(gr), kFinWarps)), UL), kFinWarps * 32, 0, stream>>>(la, last);
       }
       RESKV_LAUNCH_CHECK("residual entries");
       return RESKV_OK;

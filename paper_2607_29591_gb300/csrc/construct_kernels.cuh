@@ -965,7 +965,10 @@ __device__ __forceinline__ unsigned long long fix_total(FixSum& a, int q, uint32
   return static_cast<unsigned long long>(((long long)h << 17) + (long long)l);
 }
 
-template <bool final_pass>
+// values = false: the key sums (every pass); values = true: the value sums
+// (the last pass), a launch of their own so each keeps 8 rows in flight per
+// warp at full occupancy
+template <bool values>
 __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
   const int ul = blockIdx.y;
   const int r = p.r_unit[ul];
@@ -984,21 +987,16 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
     if (j + step < r && cb[j + step] <= lo) j += step;
   int bnd = cb[j] + cc[j];
   const int32_t* mem = p.members + int64_t(ul) * p.s;
-  const __nv_bfloat16* Kb = p.K + int64_t(ul) * p.s * kHeadDim + 4 * lane;
-  const __nv_bfloat16* Vb = p.V + int64_t(ul) * p.s * kHeadDim + 4 * lane;
+  const __nv_bfloat16* Xb = (values ? p.V : p.K) + int64_t(ul) * p.s * kHeadDim + 4 * lane;
   unsigned long long* ms = reinterpret_cast<unsigned long long*>(p.msum) +
-                           int64_t(ul) * p.rmax * 2 * kHeadDim + 4 * lane;
-  FixSum sk = {}, sv = {};
+                           int64_t(ul) * p.rmax * 2 * kHeadDim + (values ? kHeadDim : 0) + 4 * lane;
+  FixSum sk = {};
   FixState st = {0.0f, 0.0f};
   uint32_t n = 0;                 // rows in the lane sums
   auto flush = [&](int jj) {
     unsigned long long* m = ms + int64_t(jj) * 2 * kHeadDim;
 #pragma unroll
     for (int q = 0; q < 4; ++q) atomicAdd(m + q, fix_total(sk, q, n));
-    if constexpr (final_pass) {
-#pragma unroll
-      for (int q = 0; q < 4; ++q) atomicAdd(m + kHeadDim + q, fix_total(sv, q, n));
-    }
     const bool ok = st.err == 0.0f && st.mx < 128.0f;
     if (__any_sync(0xffffffffu, !ok) && lane == 0) atomicOr(p.mflag + int64_t(ul) * p.rmax + jj, 1u);
     st = FixState{0.0f, 0.0f};
@@ -1008,14 +1006,11 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
     const int my = i32 + lane < hi ? mem[i32 + lane] : 0;
 #pragma unroll 1
     for (int i8 = 0; i8 < 32 && i32 + i8 < hi; i8 += 8) {
-      uint2 kw[8], vw[8];
+      uint2 kw[8];
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
         const int64_t pos = __shfl_sync(0xffffffffu, my, i8 + q);
-        if (i32 + i8 + q < hi) {
-          kw[q] = __ldg(reinterpret_cast<const uint2*>(Kb + pos * kHeadDim));
-          if constexpr (final_pass) vw[q] = __ldg(reinterpret_cast<const uint2*>(Vb + pos * kHeadDim));
-        }
+        if (i32 + i8 + q < hi) kw[q] = __ldg(reinterpret_cast<const uint2*>(Xb + pos * kHeadDim));
       }
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
@@ -1027,7 +1022,6 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
             bnd = cb[j] + cc[j];
           }
           acc_row(kw[q], sk, st);
-          if constexpr (final_pass) acc_row(vw[q], sv, st);
           ++n;
         }
       }
@@ -1036,60 +1030,90 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
   flush(j);
 }
 
-__global__ void __launch_bounds__(kHeadDim) k_lloyd_finish(LloydArgs p, int final_pass) {
-  __shared__ float nrm[kHeadDim];
-  const int j = blockIdx.x, ul = blockIdx.y;
+// One warp per centre, lane l on dims 4l..4l+3 (coalesced sums, centres and
+// entries); ||c||^2 of the fp32 centre by a butterfly (the certification
+// bounds its rounding for any summation order).
+constexpr int kFinWarps = 8;
+
+__global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, int final_pass) {
+  const int lane = threadIdx.x & 31;
+  const int j = blockIdx.x * kFinWarps + (threadIdx.x >> 5), ul = blockIdx.y;
   const int r = p.r_unit[ul];
   if (j >= r) return;
-  const int d = threadIdx.x;
   const int64_t uj = int64_t(ul) * p.rmax + j;
   const int cnt = p.ccount[uj];
   const bool exact = p.mflag[uj] == 0u;
-  long long* ms = p.msum + uj * 2 * kHeadDim;
-  const long long tki = ms[d], tvi = ms[kHeadDim + d];
-  ms[d] = 0;
-  ms[kHeadDim + d] = 0;
-  double tk, tv;
+  long long* ms = p.msum + uj * 2 * kHeadDim + 4 * lane;
+  double tk[4], tv[4];
   if (exact) {
-    tk = double(tki) * 0x1p-32;
-    tv = double(tvi) * 0x1p-32;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      tk[q] = double(ms[q]) * 0x1p-32;
+      tv[q] = double(ms[kHeadDim + q]) * 0x1p-32;
+    }
   } else {
     // fp64 sums in member order
-    tk = 0.0;
-    tv = 0.0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) tk[q] = tv[q] = 0.0;
     const int32_t* mem = p.members + int64_t(ul) * p.s + p.cbase[uj];
-    const __nv_bfloat16* Kd = p.K + int64_t(ul) * p.s * kHeadDim + d;
-    const __nv_bfloat16* Vd = p.V + int64_t(ul) * p.s * kHeadDim + d;
+    const __nv_bfloat16* Kd = p.K + int64_t(ul) * p.s * kHeadDim + 4 * lane;
+    const __nv_bfloat16* Vd = p.V + int64_t(ul) * p.s * kHeadDim + 4 * lane;
     for (int i = 0; i < cnt; ++i) {
       const int64_t pos = mem[i];
-      tk += double(__bfloat162float(Kd[pos * kHeadDim]));
-      if (final_pass) tv += double(__bfloat162float(Vd[pos * kHeadDim]));
+      const uint2 kw = *reinterpret_cast<const uint2*>(Kd + pos * kHeadDim);
+      const float2 k01 = bf16x2_to_float2(kw.x), k23 = bf16x2_to_float2(kw.y);
+      tk[0] += double(k01.x);
+      tk[1] += double(k01.y);
+      tk[2] += double(k23.x);
+      tk[3] += double(k23.y);
+      if (final_pass) {
+        const uint2 vw = *reinterpret_cast<const uint2*>(Vd + pos * kHeadDim);
+        const float2 v01 = bf16x2_to_float2(vw.x), v23 = bf16x2_to_float2(vw.y);
+        tv[0] += double(v01.x);
+        tv[1] += double(v01.y);
+        tv[2] += double(v23.x);
+        tv[3] += double(v23.y);
+      }
     }
   }
-  float* cptr = p.centersT + (int64_t(ul) * kHeadDim + d) * p.rmax + j;
-  double* c64 = p.centers64 + uj * kHeadDim + d;
-  double mk;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) ms[q] = ms[kHeadDim + q] = 0;
+  double* c64 = p.centers64 + uj * kHeadDim + 4 * lane;
+  float* c32 = p.centers32 + uj * kHeadDim + 4 * lane;
+  double mk[4];
+  float cf[4];
   if (cnt > 0) {
-    mk = tk / double(cnt);
-    *c64 = mk;
-    *cptr = float(mk);
-    p.centers32[uj * kHeadDim + d] = float(mk);
-    write_planes(p, ul, j, d, float(mk));
-  } else {
-    mk = *c64;                        // an empty centre keeps its place
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int d = 4 * lane + q;
+      mk[q] = tk[q] / double(cnt);
+      cf[q] = float(mk[q]);
+      c64[q] = mk[q];
+      c32[q] = cf[q];
+      p.centersT[(int64_t(ul) * kHeadDim + d) * p.rmax + j] = cf[q];
+      write_planes(p, ul, j, d, cf[q]);
+    }
+  } else {                            // an empty centre keeps its place
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      mk[q] = c64[q];
+      cf[q] = c32[q];
+    }
   }
-  const float c = *cptr;
-  nrm[d] = c * c;
+  float n = fmaf(cf[3], cf[3], fmaf(cf[2], cf[2], fmaf(cf[1], cf[1], cf[0] * cf[0])));
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) n += __shfl_xor_sync(0xffffffffu, n, o);
   if (final_pass) {
     const int64_t e = int64_t(ul) * p.ent_stride + p.ent_off + j;
-    p.kbar[e * kHeadDim + d] = __double2bfloat16(mk);
-    p.vbar[e * kHeadDim + d] = __double2bfloat16(cnt > 0 ? tv / double(cnt) : 0.0);
-    if (d == 0) p.ecount[e] = cnt;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      p.kbar[e * kHeadDim + 4 * lane + q] = __double2bfloat16(mk[q]);
+      p.vbar[e * kHeadDim + 4 * lane + q] = __double2bfloat16(cnt > 0 ? tv[q] / double(cnt) : 0.0);
+    }
+    if (lane == 0) p.ecount[e] = cnt;
   }
-  __syncthreads();
-  if (d == 0) {
-    float n = 0.f;
-    for (int i = 0; i < kHeadDim; ++i) n += nrm[i];
+  __syncwarp();                       // every lane has read mflag
+  if (lane == 0) {
     p.cnorm[uj] = n;
     p.mflag[uj] = 0u;
   }
