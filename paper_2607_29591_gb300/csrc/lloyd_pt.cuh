@@ -220,6 +220,36 @@ __global__ void k_key_norm2(const __nv_bfloat16* __restrict__ K, float* __restri
   if (lane == 0) out[row] = s;
 }
 
+// (unit, tile) of the flat tile order g = unit * ntiles + tile, stepped
+// without divisions, skipping units with r = 0; r is read once per unit
+struct PtCursor {
+  int64_t g, g1;
+  int u, tile, r;
+  __device__ PtCursor(const LloydArgs& p, int64_t g0_, int64_t g1_) : g(g0_), g1(g1_) {
+    u = int(g0_ / p.ntiles);
+    tile = int(g0_ % p.ntiles);
+    r = g < g1 ? p.r_unit[u] : 0;
+    skip(p);
+  }
+  __device__ void skip(const LloydArgs& p) {
+    while (g < g1 && r <= 0) {
+      g += p.ntiles - tile;
+      tile = 0;
+      ++u;
+      r = g < g1 ? p.r_unit[u] : 0;
+    }
+  }
+  __device__ void next(const LloydArgs& p) {
+    ++g;
+    if (++tile == p.ntiles) {
+      tile = 0;
+      ++u;
+      r = g < g1 ? p.r_unit[u] : 0;
+    }
+    skip(p);
+  }
+};
+
 // Nearest centre of every evicted token of the tiles [g0, g1) of the flat
 // (unit, tile) order, g = unit * ntiles + tile (assign: centre index, -1 for
 // tokens outside E), and each tile's member count per centre (hist).  Units
@@ -280,41 +310,40 @@ __global__ void __launch_bounds__(kPtThreads, 1)
 
   if (warp == kPtProducer) {
     // ---------------- producer ----------------
-    // Two cursors over the tiles: gl, the next key tile to load (up to nk
-    // ahead, across unit changes too), and gm, the next tile to compute.
-    int64_t gl = g0, gm = g0;
+    // Two cursors over the tiles: cl, the next key tile to load (up to nk
+    // ahead, across unit changes too), and cm, the next tile to compute.
+    PtCursor cl(p, g0, g1), cm(p, g0, g1);
     int nl = 0, nm = 0, cur_u = -1;
     float cmx = 0.f;                                 // max ||c||^2 of the staged unit
     bool ok = true;
-    auto next_live = [&](int64_t g) {                // the first tile at or after g with r > 0
-      while (g < g1 && p.r_unit[int(g / p.ntiles)] <= 0) ++g;
-      return g;
-    };
-    gl = next_live(gl);
-    gm = next_live(gm);
-    while (gm < g1 && ok) {
-      // key tiles ahead, while a buffer is free
-      while (gl < g1 && nl - nm < nk) {
+    while (cm.g < g1 && ok) {
+      // key tiles ahead into the buffers already free; wait for one only
+      // when no tile is loaded ahead of the next MMA
+      while (cl.g < g1 && nl - nm < nk) {
         const int slot = nl % nk;
         if (nl >= nk) {                              // MMA(nl - nk) has read the buffer
-          bool w = pt_wait(&key_free[slot], uint32_t(((nl / nk) - 1) & 1), abort_s);
-          if (__any_sync(0xffffffffu, !w)) {
-            ok = false;
-            break;
+          const uint32_t par = uint32_t(((nl / nk) - 1) & 1);
+          if (nl > nm) {
+            if (!__all_sync(0xffffffffu, mbar_try_wait(&key_free[slot], par))) break;
+          } else {
+            bool w = pt_wait(&key_free[slot], par, abort_s);
+            if (__any_sync(0xffffffffu, !w)) {
+              ok = false;
+              break;
+            }
           }
         }
         if (lane == 0) {
-          const int u = int(gl / p.ntiles), tile = int(gl % p.ntiles);
+          const int u = cl.u, tile = cl.tile;
           mbar_arrive_expect_tx(&key_full[slot], uint32_t(kPtKeys));
           tma_keys(keys_s + uint32_t(slot * kPtKeys), &tmK, int(int64_t(u) * p.s + int64_t(tile) * kTile),
                    &key_full[slot]);
         }
         ++nl;
-        gl = next_live(gl + 1);
+        cl.next(p);
       }
       if (!ok) break;
-      const int u = int(gm / p.ntiles), tile = int(gm % p.ntiles);
-      const int r = p.r_unit[u];
+      const int u = cm.u, tile = cm.tile, r = cm.r;
       if (u != cur_u) {
         // the planes and norms of the old unit are in use until its last
         // tile's MMAs are done and the column warps have read that tile
@@ -380,7 +409,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
       __syncwarp();
       pt_arrive(&full[bb]);
       ++nm;
-      gm = next_live(gm + 1);
+      cm.next(p);
     }
     if (!ok && lane == 0) pt_raise(abort_s, p.status);
     // every issued copy and MMA completes before the CTA exits
@@ -398,8 +427,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
     // ---------------- column warps ----------------
     const int q = warp & 3, half = warp >> 2, tok = 32 * q + lane;
     int t = 0;
-    for (int64_t g = g0; g < g1; ++g) {
-      if (p.r_unit[int(g / p.ntiles)] <= 0) continue;
+    for (PtCursor cc(p, g0, g1); cc.g < g1; cc.next(p)) {
       const int b = t & 1, slot = t % kPtRing;
       const bool ok = *abort_s == 0u && pt_wait(&full[b], uint32_t((t >> 1) & 1), abort_s);
       if (!ok) pt_raise(abort_s, p.status);
@@ -472,8 +500,7 @@ __global__ void __launch_bounds__(kPtThreads, 1)
     // ---------------- certifier warps ----------------
     const int ct = tid - kPtColThreads;                   // the token of the tile this thread certifies
     int t = 0;
-    for (int64_t g = g0; g < g1; ++g) {
-      if (p.r_unit[int(g / p.ntiles)] <= 0) continue;
+    for (PtCursor cc(p, g0, g1); cc.g < g1; cc.next(p)) {
       const int slot = t % kPtRing;
       const bool ok = *abort_s == 0u && pt_wait(&list_full[slot], uint32_t((t / kPtRing) & 1), abort_s);
       if (!ok) pt_raise(abort_s, p.status);
