@@ -480,7 +480,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
         } else {
           k_lloyd_assign_tc<<<dim3(ntiles, UL), kTcThreads, sm_assign, stream>>>(la);
         }
-        k_lloyd_scan<<<UL, 256, 0, stream>>>(la);
+        k_lloyd_scan<<<dim3(UL, unsigned(cdiv(int64_t(gr), kScanCentres))), kScanCentres * kScanSegs, 0, stream>>>(la);
+        k_lloyd_bases<<<UL, 256, 0, stream>>>(la);
         k_lloyd_scatter<<<dim3(ntiles, UL), kTile, 0, stream>>>(la);
         const int last = it == cfg.lloyd_iters - 1;
         const dim3 ga(unsigned(cdiv(s, int64_t(kAccRows))), UL);

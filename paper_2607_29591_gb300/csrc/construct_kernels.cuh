@@ -833,44 +833,82 @@ __device__ __forceinline__ void top3_insert(float& d0, int& j0, float& d1, int& 
   j0 = c0 ? jx : j0;
 }
 
-// per centre: counts, per-tile offsets (in place) and member bases
-__global__ void k_lloyd_scan(LloydArgs p) {
+// Per centre: the member count of each tile becomes the tile's offset within
+// the centre's members (an exclusive prefix over tiles, in place), and the
+// total its count.  A CTA takes 32 centres of a unit; its 8 warps split the
+// tiles into 8 segments (coalesced over the 32 centres), sum them, and
+// rewrite their segment from the prefix of the segments before.
+constexpr int kScanCentres = 32;
+constexpr int kScanSegs = 8;
+
+__global__ void __launch_bounds__(kScanCentres * kScanSegs) k_lloyd_scan(LloydArgs p) {
+  __shared__ int seg[kScanSegs][kScanCentres];
+  const int ul = blockIdx.x;
+  const int r = p.r_unit[ul];
+  if (int(blockIdx.y) * kScanCentres >= r) return;
+  const int lane = threadIdx.x & 31, sg = threadIdx.x >> 5;
+  const int c = blockIdx.y * kScanCentres + lane;
+  const bool live = c < r;
+  const int T = p.ntiles, t0 = T * sg / kScanSegs, t1 = T * (sg + 1) / kScanSegs;
+  int32_t* h = p.hist + int64_t(ul) * T * p.rmax + c;
+  int sum = 0;
+  if (live) {
+    int t = t0;
+    for (; t + 16 <= t1; t += 16) {            // 16 independent loads in flight
+      int v[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) v[u] = h[int64_t(t + u) * p.rmax];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) sum += v[u];
+    }
+    for (; t < t1; ++t) sum += h[int64_t(t) * p.rmax];
+  }
+  seg[sg][lane] = sum;
+  __syncthreads();
+  int run = 0;
+  for (int k = 0; k < sg; ++k) run += seg[k][lane];
+  if (live) {
+    int t = t0;
+    for (; t + 16 <= t1; t += 16) {
+      int v[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) v[u] = h[int64_t(t + u) * p.rmax];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        h[int64_t(t + u) * p.rmax] = run;
+        run += v[u];
+      }
+    }
+    for (; t < t1; ++t) {
+      const int v = h[int64_t(t) * p.rmax];
+      h[int64_t(t) * p.rmax] = run;
+      run += v;
+    }
+    if (sg == kScanSegs - 1) p.ccount[int64_t(ul) * p.rmax + c] = run;
+  }
+}
+
+// Per unit: centre j's members start at cbase[j], the exclusive prefix of
+// the counts.
+__global__ void k_lloyd_bases(LloydArgs p) {
   __shared__ int warp_sums[32];
   const int ul = blockIdx.x;
   const int r = p.r_unit[ul];
   if (r == 0) return;
   const int per = (r + blockDim.x - 1) / blockDim.x;      // centres per thread (contiguous)
-  int total_mine = 0;
+  const int32_t* cc = p.ccount + int64_t(ul) * p.rmax;
+  int mine = 0;
   for (int q = 0; q < per; ++q) {
     const int j = threadIdx.x * per + q;
-    if (j >= r) break;
-    int run = 0;
-    int32_t* h = p.hist + int64_t(ul) * p.ntiles * p.rmax + j;
-    int t = 0;
-    for (; t + 16 <= p.ntiles; t += 16) {     // 16 independent loads in flight
-      int c[16];
-#pragma unroll
-      for (int u = 0; u < 16; ++u) c[u] = h[int64_t(t + u) * p.rmax];
-#pragma unroll
-      for (int u = 0; u < 16; ++u) {
-        h[int64_t(t + u) * p.rmax] = run;
-        run += c[u];
-      }
-    }
-    for (; t < p.ntiles; ++t) {
-      const int c = h[int64_t(t) * p.rmax];
-      h[int64_t(t) * p.rmax] = run;
-      run += c;
-    }
-    p.ccount[int64_t(ul) * p.rmax + j] = run;
-    total_mine += run;
+    if (j < r) mine += cc[j];
   }
-  int base = block_exclusive_scan(total_mine, warp_sums, nullptr);
+  int base = block_exclusive_scan(mine, warp_sums, nullptr);
   for (int q = 0; q < per; ++q) {
     const int j = threadIdx.x * per + q;
-    if (j >= r) break;
-    p.cbase[int64_t(ul) * p.rmax + j] = base;
-    base += p.ccount[int64_t(ul) * p.rmax + j];
+    if (j < r) {
+      p.cbase[int64_t(ul) * p.rmax + j] = base;
+      base += cc[j];
+    }
   }
 }
 
