@@ -2,12 +2,14 @@
 // units with at most 256 centres: one CTA per SM walks a contiguous range of
 // (unit, 128-token tile) pairs, with the unit's centre planes resident in
 // shared memory, so a tile costs one key-tile load and one tcgen05.mma chain.
-// Three roles run decoupled, linked by mbarrier rings:
+// Four roles run decoupled, linked by mbarrier rings:
 //
-//   producer warp    loads key tiles by TMA (both 64-dim halves, 128-byte
-//                    swizzle, one 32 KB copy) into a ring of nk buffers, up to
-//                    nk tiles ahead and across unit changes (key_full[]); for
-//                    each tile it issues the MMA chain of all the unit's
+//   loader warp      loads key tiles by TMA (both 64-dim halves, 128-byte
+//                    swizzle, one 32 KB copy) into a ring of nk buffers, as far
+//                    ahead as the buffers allow, across unit changes too
+//                    (key_full[]; a buffer is refilled once key_free[] says
+//                    its MMAs are done).
+//   MMA warp         for each tile issues the MMA chain of all the unit's
 //                    centres (2 planes x 8 K-steps, M = 128 tokens, N = r
 //                    rounded up to 16) into TMEM columns 256 (t & 1) ..,
 //                    committed to full[] and to the key buffer's key_free[].
@@ -49,8 +51,9 @@ constexpr int kPtColWarps = 8;
 constexpr int kPtColThreads = kPtColWarps * 32;
 constexpr int kPtCertWarps = 4;
 constexpr int kPtCertThreads = kPtCertWarps * 32;
-constexpr int kPtProducer = kPtColWarps + kPtCertWarps;        // the producer warp's index
-constexpr int kPtThreads = (kPtProducer + 1) * 32;
+constexpr int kPtProducer = kPtColWarps + kPtCertWarps;        // the MMA-issuing warp's index
+constexpr int kPtLoader = kPtProducer + 1;                      // the key-loading warp's index
+constexpr int kPtThreads = (kPtLoader + 1) * 32;
 constexpr int kPtRmax = 256;                                    // centres held resident
 constexpr int kPtRing = 4;                                      // list slots
 constexpr int kPtKeys = 2 * kTcHalf;                            // one key tile
@@ -126,6 +129,26 @@ __device__ __forceinline__ void tma_keys(uint32_t dst, const CUtensorMap* map, i
           "r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(y), "r"(0), "r"(smem_u32(bar))
       : "memory");
+}
+
+// A shared-memory descriptor advanced by `bytes` (a multiple of 16): the start
+// address sits in bits 0..13 as address / 16, and stays below 2^14 for the
+// 227 KB of shared memory, so the low word takes the addition without carry.
+__device__ __forceinline__ uint64_t desc_plus(uint64_t d, uint32_t bytes) {
+  return d + uint64_t(bytes >> 4);
+}
+
+// a probe of phase `parity` of bar that never blocks
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
 }
 
 __device__ __forceinline__ void pt_arrive(uint64_t* bar) {
@@ -308,41 +331,41 @@ __global__ void __launch_bounds__(kPtThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
-  if (warp == kPtProducer) {
-    // ---------------- producer ----------------
-    // Two cursors over the tiles: cl, the next key tile to load (up to nk
-    // ahead, across unit changes too), and cm, the next tile to compute.
-    PtCursor cl(p, g0, g1), cm(p, g0, g1);
-    int nl = 0, nm = 0, cur_u = -1;
+  if (warp == kPtLoader) {
+    // ---------------- loader ----------------
+    // Key tiles by TMA into the ring of nk buffers, as far ahead of the MMAs
+    // as the buffers allow (across unit changes too).
+    int nl = 0;
+    bool ok = true;
+    for (PtCursor cl(p, g0, g1); cl.g < g1; cl.next(p), ++nl) {
+      const int slot = nl % nk;
+      if (nl >= nk) {                                // MMA(nl - nk) has read the buffer
+        const bool w = pt_wait(&key_free[slot], uint32_t(((nl / nk) - 1) & 1), abort_s);
+        if (__any_sync(0xffffffffu, !w)) {
+          ok = false;
+          break;
+        }
+      }
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&key_full[slot], uint32_t(kPtKeys));
+        tma_keys(keys_s + uint32_t(slot * kPtKeys), &tmK,
+                 int(int64_t(cl.u) * p.s + int64_t(cl.tile) * kTile), &key_full[slot]);
+      }
+    }
+    if (!ok && lane == 0) pt_raise(abort_s, p.status);
+    // the copies in flight land before the CTA exits (the latest phase of
+    // each buffer: no older one can alias it)
+    const long long t0 = clock64();
+    for (int i = nl > nk ? nl - nk : 0; i < nl; ++i)
+      while (!mbar_try_wait(&key_full[i % nk], uint32_t((i / nk) & 1)) && clock64() - t0 < kTcWaitCycles) {
+      }
+  } else if (warp == kPtProducer) {
+    // ---------------- MMA issue ----------------
+    int nm = 0, cur_u = -1;
     float cmx = 0.f;                                 // max ||c||^2 of the staged unit
     bool ok = true;
-    while (cm.g < g1 && ok) {
-      // key tiles ahead into the buffers already free; wait for one only
-      // when no tile is loaded ahead of the next MMA
-      while (cl.g < g1 && nl - nm < nk) {
-        const int slot = nl % nk;
-        if (nl >= nk) {                              // MMA(nl - nk) has read the buffer
-          const uint32_t par = uint32_t(((nl / nk) - 1) & 1);
-          if (nl > nm) {
-            if (!__all_sync(0xffffffffu, mbar_try_wait(&key_free[slot], par))) break;
-          } else {
-            bool w = pt_wait(&key_free[slot], par, abort_s);
-            if (__any_sync(0xffffffffu, !w)) {
-              ok = false;
-              break;
-            }
-          }
-        }
-        if (lane == 0) {
-          const int u = cl.u, tile = cl.tile;
-          mbar_arrive_expect_tx(&key_full[slot], uint32_t(kPtKeys));
-          tma_keys(keys_s + uint32_t(slot * kPtKeys), &tmK, int(int64_t(u) * p.s + int64_t(tile) * kTile),
-                   &key_full[slot]);
-        }
-        ++nl;
-        cl.next(p);
-      }
-      if (!ok) break;
+    const uint64_t da0 = tc_desc(keys_s), db0 = tc_desc(planes_s);   // descriptors of the bases
+    for (PtCursor cm(p, g0, g1); cm.g < g1; cm.next(p), ++nm) {
       const int u = cm.u, tile = cm.tile, r = cm.r;
       if (u != cur_u) {
         // the planes and norms of the old unit are in use until its last
@@ -394,32 +417,27 @@ __global__ void __launch_bounds__(kPtThreads, 1)
         tc_fence_after();
         const uint32_t idesc = pt_idesc((r + 15) & ~15);
         const uint32_t d_tmem = tmem + uint32_t(bb) * kPtBufCols;
-        const uint32_t kb = keys_s + uint32_t(slot * kPtKeys);
+        const uint64_t da = desc_plus(da0, uint32_t(slot * kPtKeys));
 #pragma unroll
         for (int pl = 0; pl < 2; ++pl)
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             const uint32_t half = uint32_t(k >> 2), kk = uint32_t(k & 3) * 32u;
-            pt_mma(d_tmem, tc_desc(kb + half * kTcHalf + kk),
-                   tc_desc(planes_s + uint32_t(pl * 2 + half) * plane_half + kk), idesc, pl + k > 0);
+            pt_mma(d_tmem, desc_plus(da, half * kTcHalf + kk),
+                   desc_plus(db0, uint32_t(pl * 2 + half) * plane_half + kk), idesc, pl + k > 0);
           }
         tc_commit(&full[bb]);
         tc_commit(&key_free[slot]);
       }
       __syncwarp();
       pt_arrive(&full[bb]);
-      ++nm;
-      cm.next(p);
     }
     if (!ok && lane == 0) pt_raise(abort_s, p.status);
-    // every issued copy and MMA completes before the CTA exits
+    // every issued MMA completes before TMEM is freed
     asm volatile("cp.async.wait_group 0;" ::: "memory");
-    const long long t0 = clock64();
-    for (int i = nm; i < nl; ++i)                    // key tiles loaded but never computed
-      while (!mbar_try_wait(&key_full[i % nk], uint32_t((i / nk) & 1)) && clock64() - t0 < kTcWaitCycles) {
-      }
     if (nm >= 1) {
       const int lt = nm - 1;
+      const long long t0 = clock64();
       while (!mbar_try_wait(&full[lt & 1], uint32_t((lt >> 1) & 1)) && clock64() - t0 < kTcWaitCycles) {
       }
     }
