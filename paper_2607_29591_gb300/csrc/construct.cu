@@ -301,6 +301,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   int4* amb = nullptr;
   int* amb_count = nullptr;
   float* centers32 = nullptr;
+  // the previous Lloyd iteration's assignment and member lists
+  int32_t *assign2 = nullptr, *members2 = nullptr, *cbase2 = nullptr, *ccount2 = nullptr;
   __nv_bfloat16 *kbar = nullptr, *vbar = nullptr;
   double *rowerr = nullptr, *losses = nullptr;
   const size_t US = size_t(UL) * size_t(s);
@@ -323,7 +325,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
          S.get(&ecount, size_t(UL) * ent_stride) &&
          S.get(&msum, size_t(UL) * rmax * 2 * kHeadDim) && S.get(&mflag, size_t(UL) * rmax) &&
          S.get(&knorm2, US) && S.get(&amb, US) && S.get(&amb_count, 1) &&
-         S.get(&centers32, size_t(UL) * rmax * kHeadDim);
+         S.get(&centers32, size_t(UL) * rmax * kHeadDim) && S.get(&assign2, US) &&
+         S.get(&members2, US) && S.get(&cbase2, size_t(UL) * rmax) && S.get(&ccount2, size_t(UL) * rmax);
   // the member sums start at zero; each pass's k_lloyd_finish clears what it read
   if (ok && rmax > 0)
     ok = cudaMemsetAsync(msum, 0, size_t(UL) * rmax * 2 * kHeadDim * sizeof(long long), stream) ==
@@ -455,7 +458,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
 
     LloydArgs la{K, V, s, P, n_top, b, ntiles, rmax, top, rank_pos, nullptr, centersT, cnorm,
                  centers64, assign, hist, ccount, cbase, members, kbar, vbar, ecount,
-                 ent_stride, 0, c->status, bl_d, cplanes, msum, mflag, knorm2, amb, amb_count, centers32};
+                 ent_stride, 0, c->status, bl_d, cplanes, msum, mflag, knorm2, amb, amb_count, centers32,
+                 assign2, members2, cbase2, ccount2};
     if (rmax > 0)
       k_key_norm2<<<unsigned(cdiv(int64_t(US), 8)), 256, 0, stream>>>(K, knorm2, int64_t(US));
     // the persistent assignment loads key tiles by TMA (a 16-byte aligned
@@ -469,7 +473,22 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       const unsigned gr = unsigned(std::max(r_hi, 1));
       const unsigned pt_grid = unsigned(std::min<int64_t>(c->num_sms, int64_t(UL) * ntiles));
       k_lloyd_init<<<dim3(gr, UL), kHeadDim, 0, stream>>>(la);
+      // key sums in full for the first kDeltaFrom iterations, then updated
+      // from the previous iteration's by the tokens that moved (a third of
+      // the tokens move in the second iteration, about a tenth later)
+      constexpr int kDeltaFrom = 2;
+      int32_t* const abuf[2][4] = {{assign, members, cbase, ccount}, {assign2, members2, cbase2, ccount2}};
       for (int it = 0; it < cfg.lloyd_iters; ++it) {
+        int32_t* const* cur = abuf[it & 1];
+        int32_t* const* prv = abuf[(it + 1) & 1];
+        la.assign = cur[0];
+        la.members = cur[1];
+        la.cbase = cur[2];
+        la.ccount = cur[3];
+        la.assign_prev = prv[0];
+        la.members_prev = prv[1];
+        la.cbase_prev = prv[2];
+        la.ccount_prev = prv[3];
         if (pt_keys && r_hi <= kPtRmax) {   // the centres fit in shared memory: persistent form
           if (cudaMemsetAsync(amb_count, 0, sizeof(int), stream) != cudaSuccess)
             return fail(RESKV_ERR_CUDA, "clearing the ambiguous-token count");
@@ -485,9 +504,16 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
         k_lloyd_scatter<<<dim3(ntiles, UL), kTile, 0, stream>>>(la);
         const int last = it == cfg.lloyd_iters - 1;
         const dim3 ga(unsigned(cdiv(s, int64_t(kAccRows))), UL);
-        k_lloyd_accum<false><<<ga, kThreads, 0, stream>>>(la);
-        if (last) k_lloyd_accum<true><<<ga, kThreads, 0, stream>>>(la);
-        k_lloyd_finish<<<dim3(unsigned(cdiv(int64_t(gr), kFinWarps)), UL), kFinWarps * 32, 0, stream>>>(la, last);
+        if (it >= kDeltaFrom) {
+          k_lloyd_accum<false, 1><<<ga, kThreads, 0, stream>>>(la);
+          k_lloyd_accum<false, -1><<<ga, kThreads, 0, stream>>>(la);
+        } else {
+          k_lloyd_accum<false, 0><<<ga, kThreads, 0, stream>>>(la);
+        }
+        if (last) k_lloyd_accum<true, 0><<<ga, kThreads, 0, stream>>>(la);
+        const int keep = !last && it + 1 >= kDeltaFrom;     // the next pass updates these sums
+        k_lloyd_finish<<<dim3(unsigned(cdiv(int64_t(gr), kFinWarps)), UL), kFinWarps * 32, 0, stream>>>(
+            la, last, keep);
       }
       RESKV_LAUNCH_CHECK("residual entries");
       return RESKV_OK;

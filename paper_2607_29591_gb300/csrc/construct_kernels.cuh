@@ -779,6 +779,11 @@ struct LloydArgs {
   int4* amb;                   // [UL * s] tokens the persistent assignment leaves to k_lloyd_resolve
   int* amb_count;              // their number (zeroed before each assignment)
   float* centers32;            // [UL, rmax, d] row-major fp32 copy of the centres
+  // the previous iteration's assignment and member lists (delta accumulation)
+  const int32_t* assign_prev;
+  const int32_t* members_prev;
+  const int32_t* cbase_prev;
+  const int32_t* ccount_prev;
 };
 
 __device__ __forceinline__ bool in_evicted(const LloydArgs& p, int ul, int64_t pos, int r) {
@@ -1005,14 +1010,22 @@ __device__ __forceinline__ unsigned long long fix_total(FixSum& a, int q, uint32
 
 // values = false: the key sums (every pass); values = true: the value sums
 // (the last pass), a launch of their own so each keeps 8 rows in flight per
-// warp at full occupancy
-template <bool values>
+// warp at full occupancy.
+// delta = 0: every member of the current lists.  Once few tokens move, the
+// key sums are updated instead (integer sums: the update is exact):
+// delta = +1 adds the members of the current lists whose centre changed, and
+// delta = -1 subtracts the members of the previous lists whose centre changed
+// (a 4-byte test of both assignments per member; rows of movers only).  An
+// inexact value that joins raises the centre's flag; flags are kept while the
+// sums are (a flagged centre is summed again in fp64 from its members).
+template <bool values, int delta>
 __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
+  static_assert(delta == 0 || !values, "value sums are taken in full");
   const int ul = blockIdx.y;
   const int r = p.r_unit[ul];
   if (r <= 0) return;
-  const int32_t* cb = p.cbase + int64_t(ul) * p.rmax;
-  const int32_t* cc = p.ccount + int64_t(ul) * p.rmax;
+  const int32_t* cb = (delta < 0 ? p.cbase_prev : p.cbase) + int64_t(ul) * p.rmax;
+  const int32_t* cc = (delta < 0 ? p.ccount_prev : p.ccount) + int64_t(ul) * p.rmax;
   const int n_mem = cb[r - 1] + cc[r - 1];
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int lo = blockIdx.x * kAccRows + w * kAccRowsPerWarp;
@@ -1024,7 +1037,7 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
   for (int step = 1 << (31 - __clz(max(r - 1, 1))); step > 0; step >>= 1)
     if (j + step < r && cb[j + step] <= lo) j += step;
   int bnd = cb[j] + cc[j];
-  const int32_t* mem = p.members + int64_t(ul) * p.s;
+  const int32_t* mem = (delta < 0 ? p.members_prev : p.members) + int64_t(ul) * p.s;
   const __nv_bfloat16* Xb = (values ? p.V : p.K) + int64_t(ul) * p.s * kHeadDim + 4 * lane;
   unsigned long long* ms = reinterpret_cast<unsigned long long*>(p.msum) +
                            int64_t(ul) * p.rmax * 2 * kHeadDim + (values ? kHeadDim : 0) + 4 * lane;
@@ -1034,14 +1047,53 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
   auto flush = [&](int jj) {
     unsigned long long* m = ms + int64_t(jj) * 2 * kHeadDim;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) atomicAdd(m + q, fix_total(sk, q, n));
+    for (int q = 0; q < 4; ++q) {
+      const unsigned long long v = fix_total(sk, q, n);
+      atomicAdd(m + q, delta < 0 ? 0ull - v : v);
+    }
     const bool ok = st.err == 0.0f && st.mx < 128.0f;
-    if (__any_sync(0xffffffffu, !ok) && lane == 0) atomicOr(p.mflag + int64_t(ul) * p.rmax + jj, 1u);
+    if (delta >= 0 && __any_sync(0xffffffffu, !ok) && lane == 0)
+      atomicOr(p.mflag + int64_t(ul) * p.rmax + jj, 1u);
     st = FixState{0.0f, 0.0f};
     n = 0;
   };
   for (int i32 = lo; i32 < hi; i32 += 32) {
     const int my = i32 + lane < hi ? mem[i32 + lane] : 0;
+    if constexpr (delta != 0) {
+      // the block's movers, in list order, 8 rows at a time
+      bool mv = false;
+      if (i32 + lane < hi)
+        mv = p.assign[int64_t(ul) * p.s + my] != p.assign_prev[int64_t(ul) * p.s + my];
+      unsigned take = __ballot_sync(0xffffffffu, mv);
+      while (take) {
+        int idx[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          idx[q] = take ? __ffs(take) - 1 : -1;
+          take &= take - 1;
+        }
+        uint2 kw[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const int64_t pos = __shfl_sync(0xffffffffu, my, idx[q] < 0 ? 0 : idx[q]);
+          if (idx[q] >= 0) kw[q] = __ldg(reinterpret_cast<const uint2*>(Xb + pos * kHeadDim));
+        }
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          if (idx[q] >= 0) {
+            const int i = i32 + idx[q];
+            while (i >= bnd) {          // warp-uniform: the next centre starts here
+              flush(j);
+              ++j;
+              bnd = cb[j] + cc[j];
+            }
+            acc_row(kw[q], sk, st);
+            ++n;
+          }
+        }
+      }
+      continue;
+    }
 #pragma unroll 1
     for (int i8 = 0; i8 < 32 && i32 + i8 < hi; i8 += 8) {
       uint2 kw[8];
@@ -1073,7 +1125,9 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
 // bounds its rounding for any summation order).
 constexpr int kFinWarps = 8;
 
-__global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, int final_pass) {
+// keep: the key sums and flags stay for the next pass's update (delta
+// accumulation); otherwise both halves of the sums and the flag are cleared.
+__global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, int final_pass, int keep) {
   const int lane = threadIdx.x & 31;
   const int j = blockIdx.x * kFinWarps + (threadIdx.x >> 5), ul = blockIdx.y;
   const int r = p.r_unit[ul];
@@ -1114,8 +1168,10 @@ __global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, in
       }
     }
   }
+  if (!keep) {
 #pragma unroll
-  for (int q = 0; q < 4; ++q) ms[q] = ms[kHeadDim + q] = 0;
+    for (int q = 0; q < 4; ++q) ms[q] = ms[kHeadDim + q] = 0;
+  }
   double* c64 = p.centers64 + uj * kHeadDim + 4 * lane;
   float* c32 = p.centers32 + uj * kHeadDim + 4 * lane;
   double mk[4];
@@ -1153,7 +1209,7 @@ __global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, in
   __syncwarp();                       // every lane has read mflag
   if (lane == 0) {
     p.cnorm[uj] = n;
-    p.mflag[uj] = 0u;
+    if (!keep) p.mflag[uj] = 0u;
   }
 }
 
