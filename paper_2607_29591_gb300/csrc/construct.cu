@@ -303,6 +303,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   float* centers32 = nullptr;
   // the previous Lloyd iteration's assignment and member lists
   int32_t *assign2 = nullptr, *members2 = nullptr, *cbase2 = nullptr, *ccount2 = nullptr;
+  uint32_t* moved = nullptr;
   __nv_bfloat16 *kbar = nullptr, *vbar = nullptr;
   double *rowerr = nullptr, *losses = nullptr;
   const size_t US = size_t(UL) * size_t(s);
@@ -326,7 +327,8 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
          S.get(&msum, size_t(UL) * rmax * 2 * kHeadDim) && S.get(&mflag, size_t(UL) * rmax) &&
          S.get(&knorm2, US) && S.get(&amb, US) && S.get(&amb_count, 1) &&
          S.get(&centers32, size_t(UL) * rmax * kHeadDim) && S.get(&assign2, US) &&
-         S.get(&members2, US) && S.get(&cbase2, size_t(UL) * rmax) && S.get(&ccount2, size_t(UL) * rmax);
+         S.get(&members2, US) && S.get(&cbase2, size_t(UL) * rmax) && S.get(&ccount2, size_t(UL) * rmax) &&
+         S.get(&moved, (US + 31) / 32);
   // the member sums start at zero; each pass's k_lloyd_finish clears what it read
   if (ok && rmax > 0)
     ok = cudaMemsetAsync(msum, 0, size_t(UL) * rmax * 2 * kHeadDim * sizeof(long long), stream) ==
@@ -459,7 +461,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     LloydArgs la{K, V, s, P, n_top, b, ntiles, rmax, top, rank_pos, nullptr, centersT, cnorm,
                  centers64, assign, hist, ccount, cbase, members, kbar, vbar, ecount,
                  ent_stride, 0, c->status, bl_d, cplanes, msum, mflag, knorm2, amb, amb_count, centers32,
-                 assign2, members2, cbase2, ccount2};
+                 assign2, members2, cbase2, ccount2, moved};
     if (rmax > 0)
       k_key_norm2<<<unsigned(cdiv(int64_t(US), 8)), 256, 0, stream>>>(K, knorm2, int64_t(US));
     // the persistent assignment loads key tiles by TMA (a 16-byte aligned
@@ -505,6 +507,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
         const int last = it == cfg.lloyd_iters - 1;
         const dim3 ga(unsigned(cdiv(s, int64_t(kAccRows))), UL);
         if (it >= kDeltaFrom) {
+          k_lloyd_moved<<<unsigned(cdiv(int64_t(US), 256)), 256, 0, stream>>>(la, int64_t(US));
           k_lloyd_accum<false, 1><<<ga, kThreads, 0, stream>>>(la);
           k_lloyd_accum<false, -1><<<ga, kThreads, 0, stream>>>(la);
         } else {

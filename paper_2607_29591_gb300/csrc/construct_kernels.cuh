@@ -784,6 +784,7 @@ struct LloydArgs {
   const int32_t* members_prev;
   const int32_t* cbase_prev;
   const int32_t* ccount_prev;
+  uint32_t* moved;             // [UL * s / 32] bit per token: its centre changed (delta accumulation)
 };
 
 __device__ __forceinline__ bool in_evicted(const LloydArgs& p, int ul, int64_t pos, int r) {
@@ -1015,9 +1016,17 @@ __device__ __forceinline__ unsigned long long fix_total(FixSum& a, int q, uint32
 // key sums are updated instead (integer sums: the update is exact):
 // delta = +1 adds the members of the current lists whose centre changed, and
 // delta = -1 subtracts the members of the previous lists whose centre changed
-// (a 4-byte test of both assignments per member; rows of movers only).  An
+// (a bit of the moved-token bitmap per member; rows of movers only).  An
 // inexact value that joins raises the centre's flag; flags are kept while the
 // sums are (a flagged centre is summed again in fp64 from its members).
+// the moved-token bitmap of the iteration: token t's bit in word t / 32
+__global__ void k_lloyd_moved(LloydArgs p, int64_t n_tok) {
+  const int64_t t = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  const bool mv = t < n_tok && p.assign[t] != p.assign_prev[t];
+  const unsigned b = __ballot_sync(0xffffffffu, mv);
+  if ((threadIdx.x & 31) == 0 && t < n_tok) p.moved[t >> 5] = b;
+}
+
 template <bool values, int delta>
 __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
   static_assert(delta == 0 || !values, "value sums are taken in full");
@@ -1062,8 +1071,10 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
     if constexpr (delta != 0) {
       // the block's movers, in list order, 8 rows at a time
       bool mv = false;
-      if (i32 + lane < hi)
-        mv = p.assign[int64_t(ul) * p.s + my] != p.assign_prev[int64_t(ul) * p.s + my];
+      if (i32 + lane < hi) {
+        const int64_t t = int64_t(ul) * p.s + my;
+        mv = (p.moved[t >> 5] >> (t & 31)) & 1u;
+      }
       unsigned take = __ballot_sync(0xffffffffu, mv);
       while (take) {
         int idx[8];
@@ -1136,12 +1147,27 @@ __global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, in
   const int cnt = p.ccount[uj];
   const bool exact = p.mflag[uj] == 0u;
   long long* ms = p.msum + uj * 2 * kHeadDim + 4 * lane;
-  double tk[4], tv[4];
+  // mean = RN(sum / cnt) with sum = RN(S * 2^-32) for the integer sum S: by
+  // Markstein's correction with the rounded reciprocal y = RN(1 / (cnt 2^32)),
+  // q0 = RN(S y), r = S - q0 cnt 2^32 (exact in one fma), q = RN(q0 + r y) is
+  // the correctly rounded quotient -- two fp64 fmas and a product per
+  // dimension instead of a division (fp64 is scarce on this part)
+  double tk[4], tv[4], mk[4], mv[4];
+  const double cd = double(cnt);
   if (exact) {
+    const double y = cnt > 0 ? (1.0 / cd) * 0x1p-32 : 0.0;
+    const double bd = cd * 0x1p32;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      tk[q] = double(ms[q]) * 0x1p-32;
-      tv[q] = double(ms[kHeadDim + q]) * 0x1p-32;
+      const double sk = double(ms[q]);
+      const double qk = sk * y;
+      mk[q] = fma(fma(-qk, bd, sk), y, qk);
+      mv[q] = 0.0;
+      if (final_pass) {
+        const double sv = double(ms[kHeadDim + q]);
+        const double qv = sv * y;
+        mv[q] = fma(fma(-qv, bd, sv), y, qv);
+      }
     }
   } else {
     // fp64 sums in member order
@@ -1167,6 +1193,11 @@ __global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, in
         tv[3] += double(v23.y);
       }
     }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      mk[q] = tk[q] / cd;
+      mv[q] = final_pass ? tv[q] / cd : 0.0;
+    }
   }
   if (!keep) {
 #pragma unroll
@@ -1174,13 +1205,11 @@ __global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, in
   }
   double* c64 = p.centers64 + uj * kHeadDim + 4 * lane;
   float* c32 = p.centers32 + uj * kHeadDim + 4 * lane;
-  double mk[4];
   float cf[4];
   if (cnt > 0) {
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const int d = 4 * lane + q;
-      mk[q] = tk[q] / double(cnt);
       cf[q] = float(mk[q]);
       c64[q] = mk[q];
       c32[q] = cf[q];
@@ -1202,7 +1231,7 @@ __global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, in
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       p.kbar[e * kHeadDim + 4 * lane + q] = __double2bfloat16(mk[q]);
-      p.vbar[e * kHeadDim + 4 * lane + q] = __double2bfloat16(cnt > 0 ? tv[q] / double(cnt) : 0.0);
+      p.vbar[e * kHeadDim + 4 * lane + q] = __double2bfloat16(cnt > 0 ? mv[q] : 0.0);
     }
     if (lane == 0) p.ecount[e] = cnt;
   }

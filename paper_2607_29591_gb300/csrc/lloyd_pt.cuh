@@ -220,6 +220,13 @@ __device__ __forceinline__ float pt_key(float d, int col) {
 }
 __device__ __forceinline__ int pt_key_index(float key) { return __float_as_int(key) & 0xFF; }
 
+// pt_key by one byte permute: byte 0 from byte b of `cols`, which holds
+// four consecutive centre indices (one per byte)
+template <int b>
+__device__ __forceinline__ float pt_key4(float d, uint32_t cols) {
+  return __int_as_float(int(__byte_perm(uint32_t(__float_as_int(d)), cols, 0x3214u + b)));
+}
+
 // key into the ascending best three (x0, x1, x2)
 __device__ __forceinline__ void pt_ins3(float& x0, float& x1, float& x2, float key) {
   const float t0 = fmaxf(x0, key);
@@ -467,11 +474,15 @@ __global__ void __launch_bounds__(kPtThreads, 1)
       for (int k = half; k < (rpad >> 4); k += 2) {
         float v[16];
         tc_ld16(tb + uint32_t(16 * k), v);
+        const uint32_t c0 = uint32_t(16 * k) * 0x01010101u + 0x03020100u;   // columns 16k .. 16k + 3
 #pragma unroll
-        for (int i = 0; i < 16; i += 2) {
-          const int col = 16 * k + i;
-          pt_ins3(a0, a1, a2, pt_key(fmaf(-2.0f, v[i], cn_s[col]), col));
-          pt_ins3(e0, e1, e2, pt_key(fmaf(-2.0f, v[i + 1], cn_s[col + 1]), col + 1));
+        for (int m = 0; m < 4; ++m) {
+          const uint32_t cols = c0 + uint32_t(4 * m) * 0x01010101u;
+          const int col = 16 * k + 4 * m;
+          pt_ins3(a0, a1, a2, pt_key4<0>(fmaf(-2.0f, v[4 * m], cn_s[col]), cols));
+          pt_ins3(e0, e1, e2, pt_key4<1>(fmaf(-2.0f, v[4 * m + 1], cn_s[col + 1]), cols));
+          pt_ins3(a0, a1, a2, pt_key4<2>(fmaf(-2.0f, v[4 * m + 2], cn_s[col + 2]), cols));
+          pt_ins3(e0, e1, e2, pt_key4<3>(fmaf(-2.0f, v[4 * m + 3], cn_s[col + 3]), cols));
         }
       }
       pt_ins3(a0, a1, a2, e0);
