@@ -381,7 +381,12 @@ reskv_status reskv_export_debug(const reskv_cache* c, int32_t what, void* host_d
  *     the wait's bound had run out: the kernel sets its status word (code 1),
  *     waits for its own copies in flight and returns with the output
  *     incomplete.  The handle's partial-result tickets are then not reset:
- *     free the handle after reskv_check_status reports the fault.
+ *     free the handle after reskv_check_status reports the fault.  A
+ *     reskv_build_cache call takes one of the n instead: in its first
+ *     persistent Lloyd assignment, CTA 0's certifier gives up its first
+ *     wait; that CTA stops at a tile boundary, the build completes with the
+ *     entries of that run incomplete, and the new handle's status word
+ *     reports code 1.
  *   RESKV_TEST_FAIL_ALLOC, n >= 1: the n-th device allocation of the library
  *     from now on fails as cudaMalloc out of memory would (nothing is
  *     allocated for it; the call returns RESKV_ERR_OOM and frees what it had

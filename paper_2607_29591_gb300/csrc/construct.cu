@@ -329,7 +329,13 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
          S.get(&centers32, size_t(UL) * rmax * kHeadDim) && S.get(&assign2, US) &&
          S.get(&members2, US) && S.get(&cbase2, size_t(UL) * rmax) && S.get(&ccount2, size_t(UL) * rmax) &&
          S.get(&moved, (US + 31) / 32);
-  // the member sums start at zero; each pass's k_lloyd_finish clears what it read
+  // the member sums start at zero; each pass's k_lloyd_finish clears what it
+  // read.  Assignments start at -1 (no centre) and per-tile counts at 0, so
+  // that a tile a failed assignment never reached holds no index and no count
+  if (ok && rmax > 0)
+    ok = cudaMemsetAsync(assign, 0xff, US * sizeof(int32_t), stream) == cudaSuccess &&
+         cudaMemsetAsync(assign2, 0xff, US * sizeof(int32_t), stream) == cudaSuccess &&
+         cudaMemsetAsync(hist, 0, size_t(UL) * ntiles * rmax * sizeof(int32_t), stream) == cudaSuccess;
   if (ok && rmax > 0)
     ok = cudaMemsetAsync(msum, 0, size_t(UL) * rmax * 2 * kHeadDim * sizeof(long long), stream) ==
              cudaSuccess &&
@@ -386,6 +392,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   StageTimer timer(stream);
   bool timing_ok = true;
 
+  int test_fault = take_test_wait_fault() ? 1 : 0;   // test hook (reskv_test_inject)
   for (int l = 0; l < cfg.n_layers; ++l) {
     const __nv_bfloat16* K = static_cast<const __nv_bfloat16*>(Kl[l]);
     const __nv_bfloat16* V = static_cast<const __nv_bfloat16*>(Vl[l]);
@@ -461,7 +468,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
     LloydArgs la{K, V, s, P, n_top, b, ntiles, rmax, top, rank_pos, nullptr, centersT, cnorm,
                  centers64, assign, hist, ccount, cbase, members, kbar, vbar, ecount,
                  ent_stride, 0, c->status, bl_d, cplanes, msum, mflag, knorm2, amb, amb_count, centers32,
-                 assign2, members2, cbase2, ccount2, moved};
+                 assign2, members2, cbase2, ccount2, moved, 0};
     if (rmax > 0)
       k_key_norm2<<<unsigned(cdiv(int64_t(US), 8)), 256, 0, stream>>>(K, knorm2, int64_t(US));
     // the persistent assignment loads key tiles by TMA (a 16-byte aligned
@@ -495,8 +502,11 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
           if (cudaMemsetAsync(amb_count, 0, sizeof(int), stream) != cudaSuccess)
             return fail(RESKV_ERR_CUDA, "clearing the ambiguous-token count");
           const int rp = (r_hi + 15) & ~15;
+          la.test_fault = test_fault;     // an injected fault is taken by the first launch only
+          test_fault = 0;
           k_lloyd_assign_pt<<<pt_grid, kPtThreads, lloyd_pt_smem(rp), stream>>>(la, UL, rp,
                                                                                  lloyd_pt_key_bufs(rp), tmK);
+          la.test_fault = 0;
           k_lloyd_resolve<<<unsigned(4 * c->num_sms), kResWarps * 32, 0, stream>>>(la);
         } else {
           k_lloyd_assign_tc<<<dim3(ntiles, UL), kTcThreads, sm_assign, stream>>>(la);

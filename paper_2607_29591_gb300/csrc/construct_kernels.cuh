@@ -785,6 +785,7 @@ struct LloydArgs {
   const int32_t* cbase_prev;
   const int32_t* ccount_prev;
   uint32_t* moved;             // [UL * s / 32] bit per token: its centre changed (delta accumulation)
+  int32_t test_fault;          // test hook: CTA 0's certifier gives up its first wait
 };
 
 __device__ __forceinline__ bool in_evicted(const LloydArgs& p, int ul, int64_t pos, int r) {
@@ -930,10 +931,18 @@ __global__ void k_lloyd_scatter(LloydArgs p) {
   a_s[t] = a;
   __syncthreads();
   if (a < 0) return;
+  if (a >= r) {                        // only after a failed assignment
+    report_status(p.status, kStatusBadIndex);
+    return;
+  }
   int rank = 0;
   for (int i = 0; i < t; ++i) rank += (a_s[i] == a);
   const int64_t off = p.cbase[int64_t(ul) * p.rmax + a] +
                       p.hist[(int64_t(ul) * p.ntiles + tile) * p.rmax + a] + rank;
+  if (off < 0 || off >= p.s) {         // counts inconsistent with the assignment: the same
+    report_status(p.status, kStatusBadIndex);
+    return;
+  }
   p.members[int64_t(ul) * p.s + off] = int32_t(pos);
 }
 
@@ -1035,7 +1044,8 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
   if (r <= 0) return;
   const int32_t* cb = (delta < 0 ? p.cbase_prev : p.cbase) + int64_t(ul) * p.rmax;
   const int32_t* cc = (delta < 0 ? p.ccount_prev : p.ccount) + int64_t(ul) * p.rmax;
-  const int n_mem = cb[r - 1] + cc[r - 1];
+  // (the clamps below only act after a failed assignment, whose status is raised)
+  const int n_mem = min(cb[r - 1] + cc[r - 1], int(p.s));
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int lo = blockIdx.x * kAccRows + w * kAccRowsPerWarp;
   if (lo >= n_mem) return;
@@ -1067,7 +1077,10 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
     n = 0;
   };
   for (int i32 = lo; i32 < hi; i32 += 32) {
-    const int my = i32 + lane < hi ? mem[i32 + lane] : 0;
+    // a member position outside the unit only follows a failed assignment
+    // (its status is raised): read row 0 instead of leaving the array
+    int my = i32 + lane < hi ? mem[i32 + lane] : 0;
+    my = uint32_t(my) < uint32_t(p.s) ? my : 0;
     if constexpr (delta != 0) {
       // the block's movers, in list order, 8 rows at a time
       bool mv = false;
@@ -1093,7 +1106,7 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
         for (int q = 0; q < 8; ++q) {
           if (idx[q] >= 0) {
             const int i = i32 + idx[q];
-            while (i >= bnd) {          // warp-uniform: the next centre starts here
+            while (i >= bnd && j < r - 1) {   // warp-uniform: the next centre starts here
               flush(j);
               ++j;
               bnd = cb[j] + cc[j];
@@ -1103,27 +1116,27 @@ __global__ void __launch_bounds__(kThreads) k_lloyd_accum(LloydArgs p) {
           }
         }
       }
-      continue;
-    }
+    } else {
 #pragma unroll 1
-    for (int i8 = 0; i8 < 32 && i32 + i8 < hi; i8 += 8) {
-      uint2 kw[8];
+      for (int i8 = 0; i8 < 32 && i32 + i8 < hi; i8 += 8) {
+        uint2 kw[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const int64_t pos = __shfl_sync(0xffffffffu, my, i8 + q);
-        if (i32 + i8 + q < hi) kw[q] = __ldg(reinterpret_cast<const uint2*>(Xb + pos * kHeadDim));
-      }
+        for (int q = 0; q < 8; ++q) {
+          const int64_t pos = __shfl_sync(0xffffffffu, my, i8 + q);
+          if (i32 + i8 + q < hi) kw[q] = __ldg(reinterpret_cast<const uint2*>(Xb + pos * kHeadDim));
+        }
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const int i = i32 + i8 + q;
-        if (i < hi) {
-          while (i >= bnd) {            // warp-uniform: the next centre starts here
-            flush(j);
-            ++j;
-            bnd = cb[j] + cc[j];
+        for (int q = 0; q < 8; ++q) {
+          const int i = i32 + i8 + q;
+          if (i < hi) {
+            while (i >= bnd && j < r - 1) {   // warp-uniform: the next centre starts here
+              flush(j);
+              ++j;
+              bnd = cb[j] + cc[j];
+            }
+            acc_row(kw[q], sk, st);
+            ++n;
           }
-          acc_row(kw[q], sk, st);
-          ++n;
         }
       }
     }
@@ -1173,11 +1186,13 @@ __global__ void __launch_bounds__(kFinWarps * 32) k_lloyd_finish(LloydArgs p, in
     // fp64 sums in member order
 #pragma unroll
     for (int q = 0; q < 4; ++q) tk[q] = tv[q] = 0.0;
-    const int32_t* mem = p.members + int64_t(ul) * p.s + p.cbase[uj];
+    const int64_t mb = p.cbase[uj];
+    const int cnt_in = (mb >= 0 && mb + cnt <= p.s) ? cnt : 0;   // see k_lloyd_accum
+    const int32_t* mem = p.members + int64_t(ul) * p.s + (cnt_in > 0 ? mb : 0);
     const __nv_bfloat16* Kd = p.K + int64_t(ul) * p.s * kHeadDim + 4 * lane;
     const __nv_bfloat16* Vd = p.V + int64_t(ul) * p.s * kHeadDim + 4 * lane;
-    for (int i = 0; i < cnt; ++i) {
-      const int64_t pos = mem[i];
+    for (int i = 0; i < cnt_in; ++i) {
+      const int64_t pos = uint32_t(mem[i]) < uint32_t(p.s) ? mem[i] : 0;   // see k_lloyd_accum
       const uint2 kw = *reinterpret_cast<const uint2*>(Kd + pos * kHeadDim);
       const float2 k01 = bf16x2_to_float2(kw.x), k23 = bf16x2_to_float2(kw.y);
       tk[0] += double(k01.x);

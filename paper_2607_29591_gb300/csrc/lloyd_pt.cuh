@@ -531,7 +531,8 @@ __global__ void __launch_bounds__(kPtThreads, 1)
     int t = 0;
     for (PtCursor cc(p, g0, g1); cc.g < g1; cc.next(p)) {
       const int slot = t % kPtRing;
-      const bool ok = *abort_s == 0u && pt_wait(&list_full[slot], uint32_t((t / kPtRing) & 1), abort_s);
+      bool ok = *abort_s == 0u && pt_wait(&list_full[slot], uint32_t((t / kPtRing) & 1), abort_s);
+      if (p.test_fault && blockIdx.x == 0 && t == 0) ok = false;   // a timed-out wait, injected
       if (!ok) pt_raise(abort_s, p.status);
       if (pt_bar_or(2, kPtCertThreads, !ok)) break;
       const int u = rinfo[8 * slot + 0], tile = rinfo[8 * slot + 1], r = rinfo[8 * slot + 2];

@@ -1,8 +1,9 @@
 """Failure paths, exercised without faulting or hanging a GPU.
 
-reskv_test_inject makes (a) the next decode launch's warps give up their first
-ring wait as a timed-out bounded wait would -- the kernel sets its status word,
-waits for its own copies in flight and returns -- and (b) the n-th device
+reskv_test_inject makes (a) the next decode launch's warps (or, in a build,
+the persistent Lloyd assignment's CTA 0 certifier) give up their first wait
+as a timed-out bounded wait would -- the kernel sets its status word, waits
+for its own copies in flight and returns -- and (b) the n-th device
 allocation fail as cudaMalloc out of memory would.  The host must see the
 fault (reskv_check_status: RESKV_ERR_DEVICE_STATUS; the call: RESKV_ERR_OOM),
 leave the output handle untouched, leak no device memory, and a fresh handle
@@ -72,6 +73,32 @@ def test_timed_out_wait_is_reported_and_a_fresh_handle_decodes(kernel, layer):
     ref = oracle_decode_all(lay, Q, cfg)
     assert_output_parity(O2.cpu().numpy(), ref if layer < 0 else ref[layer], kernel)
     h2.free()
+
+
+def test_timed_out_wait_in_construction_is_reported_and_a_fresh_build_matches():
+    """The persistent Lloyd assignment (Alg. 1): CTA 0's certifier gives up its
+    first wait as a timed-out bounded wait would.  Every role of that CTA
+    leaves at a tile boundary, its copies and MMAs finish, the build returns
+    with the timeout in the status word, the later construction kernels stay
+    inside their arrays, and a fresh build matches the oracle."""
+    import re
+
+    from test_build_gpu import lib_config, make_inputs, run_case
+
+    w = wl.WORKLOADS["tiny"]                      # one unit, r = 32: the persistent form
+    _, (Kd, Vd, Qdv) = make_inputs(w)
+    cfg = lib_config(w)
+    R.reskv_test_inject(R.RESKV_TEST_FAIL_FIRST_WAIT, 1)
+    cache = R.reskv_build_cache(cfg, Kd, Vd, Qdv if w.n_obs > 0 else None)
+    torch.cuda.synchronize()
+    with pytest.raises(R.ReskvError) as e:
+        R.reskv_check_status(cache)
+    assert e.value.status == R.RESKV_ERR_DEVICE_STATUS
+    m = re.search(r"word (\d+)", str(e.value))
+    assert m and int(m.group(1)) & 1                 # kStatusWaitTimeout
+    cache.free()
+    out = run_case(w)                                  # a fresh build: full parity
+    assert out["worst_rel"] < 2e-3
 
 
 def _raw_build(cfg, Ks, Vs, Qs):
