@@ -288,3 +288,40 @@ def test_lloyd_sums_outside_the_fixed_point_range():
         big += int(np.sum(np.abs(gu.vbar[:, 7]) > 2.0 ** 20))
     assert big > 0                       # some centre holds a 2^40 value
     cache.free()
+
+
+def test_lloyd_at_the_persistent_assignment_edges():
+    """Lloyd (Sec. 5.3) with r at the edges of the persistent assignment:
+    r = 1 (one centre among padded keys), 16 and 17 (one and two 16-column
+    MMA blocks), 255 and 256 (the most centres held in shared memory), and
+    r = 0 units between them, in one layer; in the other layer 257 and 300
+    switch that layer's runs to the streaming form.  Counts bit-exact and
+    entries within one bf16 ulp of the oracle's Lloyd on the GPU's evicted
+    set, for every unit."""
+    s, b, P = 2048, 512, 64
+    w = wl.scaled(wl.WORKLOADS["small_budget_b64"], seq_len=s, budget=b, batch=4, n_layers=2,
+                  n_kv_heads=2)
+    ovr = np.array([1, 16, 17, 0, 255, 256, 0, 40,            # layer 0: persistent
+                    257, 300, 0, 33, 1, 256, 128, 2], np.int32)  # layer 1: streaming
+    assert ovr.size == w.n_units
+    Ks, Vs = [], []
+    for l in range(w.n_layers):
+        K, V, _, _ = wl.layer_inputs(w, l, "cpu")
+        Ks.append(K)
+        Vs.append(V)
+    cfg = R.reskv_config_default(batch=w.batch, n_layers=w.n_layers, n_kv_heads=w.n_kv_heads,
+                                 group=w.group, seq_len=s, budget=b, recent_window=P, n_obs=0,
+                                 n_fit=0, n_val=0, score_mode=R.RESKV_SCORE_KEYNORM,
+                                 residual_override=ovr, keep_debug=1)
+    cache = R.reskv_build_cache(cfg, [k.cuda() for k in Ks], [v.cuda() for v in Vs], None)
+    torch.cuda.synchronize()
+    R.reskv_check_status(cache)
+    lay = R.reskv_export_cache(cache)
+    top = R.reskv_export_debug(cache, R.RESKV_DEBUG_RANKED)
+    for u in range(w.n_units):
+        l, rem = divmod(u, w.batch * w.n_kv_heads)
+        bb, h = divmod(rem, w.n_kv_heads)
+        gu = unit_from_layout(lay, u)
+        assert gu.r == ovr[u], (u, gu.r, ovr[u])
+        check_entries(gu, bf16_to_f64(Ks[l][bb, h]), bf16_to_f64(Vs[l][bb, h]), top[u], P, s, b, 4)
+    cache.free()
