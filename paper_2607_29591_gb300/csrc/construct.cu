@@ -385,6 +385,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   if (set_smem(k_obs_pass1, sm_obs1) != cudaSuccess || set_smem(k_obs_pass2, sm_obs2) != cudaSuccess ||
       set_smem(k_topk, sm_top) != cudaSuccess || set_smem(k_lloyd_assign_tc, sm_assign) != cudaSuccess ||
       set_smem(k_lloyd_assign_pt, kPtSmemMax) != cudaSuccess ||
+      set_smem(k_val_loss, sm_val) != cudaSuccess ||
       set_smem(k_val_full, sm_val) != cudaSuccess)
     return cleanup_fail(fail(RESKV_ERR_CUDA, "setting kernel shared-memory limits"));
 
@@ -558,7 +559,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
                     kbar, vbar, ecount, ent_stride, run_off[run], cfg.beta, cfg.gate_mode,
                     cfg.tau, cfg.alpha, cfg.g_min, cfg.g_fixed, oS, rowerr, cfg.softmax_mode,
                     bl_d};
-        k_val_loss<<<dim3(unsigned(cdiv(n_val_rows, 8)), UL), kThreads, 0, stream>>>(lo);
+        k_val_loss<<<dim3(unsigned(cdiv(n_val_rows, kRowBlk)), UL), kThreads, sm_val, stream>>>(lo);
         k_loss_reduce<<<unsigned(cdiv(UL, 128)), 128, 0, stream>>>(rowerr, losses, n_val_rows, UL,
                                                                   ncol, run, r_unit);
         RESKV_LAUNCH_CHECK("validation loss");

@@ -1416,90 +1416,192 @@ struct LossArgs {
 };
 
 // ||o^(r)(q) - o_S(q)||^2 per validation query, with the decode rule of
-// Sec. 5.4 and the gate (one warp per query, 4 dims per lane)
-__global__ void __launch_bounds__(kThreads) k_val_loss(LossArgs p) {
+// Sec. 5.4 and the gate.  Tiled like k_val_full: a CTA takes 32 query rows of
+// a unit (warp w: rows 4w..4w+3; lane l: tokens 4l..4l+3 of a 128-token tile
+// for the logits, dims 4l..4l+3 for the outputs) and walks the candidate's
+// main slots (the kept ranked tokens, then the recent window), then its
+// residual entries (logit + beta ln c), each gathered into shared memory
+// once for all 32 rows, with one online-softmax state per branch.
+// Dynamic shared memory: that of k_val_full.
+struct LossState {
+  float m[4], l[4], acc[4][4];
+};
+
+template <class RowPtr>
+__device__ __forceinline__ void load_rows_kt(float* Kt, RowPtr rowptr) {
+  for (int it = 0; it < 8; ++it) {
+    const int idx = it * kThreads + threadIdx.x;
+    const int tok = idx >> 4, dc = idx & 15;
+    const __nv_bfloat16* src = rowptr(tok);
+    uint4 w = make_uint4(0, 0, 0, 0);
+    if (src) w = __ldg(reinterpret_cast<const uint4*>(src) + dc);
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = bf16x2_to_float2(ws[j]);
+      Kt[kt_index(8 * dc + 2 * j, tok)] = f.x;
+      Kt[kt_index(8 * dc + 2 * j + 1, tok)] = f.y;
+    }
+  }
+}
+
+template <class RowPtr>
+__device__ __forceinline__ void load_rows_v(float* Vs, RowPtr rowptr) {
+  for (int it = 0; it < 8; ++it) {
+    const int idx = it * kThreads + threadIdx.x;
+    const int tok = idx >> 4, dc = idx & 15;
+    const __nv_bfloat16* src = rowptr(tok);
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (src) v = __ldg(reinterpret_cast<const uint4*>(src) + dc);
+    const float2 a = bf16x2_to_float2(v.x), b = bf16x2_to_float2(v.y);
+    const float2 c = bf16x2_to_float2(v.z), d = bf16x2_to_float2(v.w);
+    *reinterpret_cast<float4*>(Vs + tok * kHeadDim + 8 * dc) = make_float4(a.x, a.y, b.x, b.y);
+    *reinterpret_cast<float4*>(Vs + tok * kHeadDim + 8 * dc + 4) = make_float4(c.x, c.y, d.x, d.y);
+  }
+}
+
+// One 128-token tile (K in Kt, V in Vs) into state st: logits + bias[j] for
+// this lane's tokens 4l + j (-inf: no token)
+__device__ __forceinline__ void loss_tile(const float* Qt, const float* Kt, const float* Vs, float* Pt,
+                                          const float (&bias)[4], LossState& st) {
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int row = blockIdx.x * 8 + w, ul = blockIdx.y;
-  if (row >= p.n_rows) return;
+  float S[4][4];
+  tile_logits(Qt, Kt, S);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float tmax = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      S[i][j] += bias[j];
+      tmax = fmaxf(tmax, S[i][j]);
+    }
+    tmax = warp_max(tmax);
+    const float mn = fmaxf(st.m[i], tmax);
+    // a tile with no token leaves the state as it is (mn = -inf)
+    const float sc = mn == -INFINITY ? 1.0f : exp2f(st.m[i] - mn);
+    st.l[i] *= sc;
+#pragma unroll
+    for (int d = 0; d < 4; ++d) st.acc[i][d] *= sc;
+    st.m[i] = mn;
+    float ps = 0.f;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      S[i][j] = mn == -INFINITY ? 0.f : exp2f(S[i][j] - mn);
+      ps += S[i][j];
+    }
+    st.l[i] += warp_sum(ps);
+  }
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int tok = 4 * lane + j;
+    *reinterpret_cast<float4*>(Pt + tok * kRowBlk + ((w ^ (lane & 7)) << 2)) =
+        make_float4(S[0][j], S[1][j], S[2][j], S[3][j]);
+  }
+  __syncthreads();
+#pragma unroll 4
+  for (int tok = 0; tok < kTile; ++tok) {
+    const float4 pp = *reinterpret_cast<const float4*>(Pt + tok * kRowBlk + ((w ^ ((tok >> 2) & 7)) << 2));
+    const float4 vv = *reinterpret_cast<const float4*>(Vs + tok * kHeadDim + 4 * lane);
+    const float pa[4] = {pp.x, pp.y, pp.z, pp.w};
+    const float va[4] = {vv.x, vv.y, vv.z, vv.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int d = 0; d < 4; ++d) st.acc[i][d] = fmaf(pa[i], va[d], st.acc[i][d]);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 1) k_val_loss(LossArgs p) {
+  extern __shared__ __align__(16) float sm[];
+  float* Kt = sm;                               // [128][128] swizzled
+  float* Vs = Kt + kHeadDim * kTile;            // [128 tok][128 d]
+  float* Qt = Vs + kHeadDim * kTile;            // [128][32]
+  float* Pt = Qt + kHeadDim * kRowBlk;          // [128 tok][32 rows] swizzled
+  const int rb = blockIdx.x * kRowBlk, ul = blockIdx.y;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = p.r_unit[ul];
   const int64_t bu = unit_budget(p.budgets, ul, p.budget);
   const int64_t m = r == 0 ? (bu < p.s ? bu : p.s) : bu - r;
   const int64_t keep = m - p.recent;
-  const int g = row / p.n_val, t = row % p.n_val;
-  const __nv_bfloat16* qp = p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + (p.n_obs - p.n_val) + t) * kHeadDim;
   const float scale = kLog2e * rsqrtf(float(kHeadDim));
-  const uint2 qw = __ldg(reinterpret_cast<const uint2*>(qp + 4 * lane));
-  const float2 q01 = bf16x2_to_float2(qw.x), q23 = bf16x2_to_float2(qw.y);
-  const float q[4] = {q01.x * scale, q01.y * scale, q23.x * scale, q23.y * scale};
-  const __nv_bfloat16* Ku = p.K + int64_t(ul) * p.s * kHeadDim + 4 * lane;
-  const __nv_bfloat16* Vu = p.V + int64_t(ul) * p.s * kHeadDim + 4 * lane;
-  const int32_t* top = p.top + int64_t(ul) * p.n_top;
-  // main cache
-  float mM = -INFINITY, lM = 0.f, aM[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int64_t j0 = 0; j0 < m; j0 += 4) {
-    uint2 kw[4], vw[4];
+  load_qt(Qt, min(kRowBlk, p.n_rows - rb), scale, [&](int row) {
+    const int g = (rb + row) / p.n_val, t = (rb + row) % p.n_val;
+    return p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + (p.n_obs - p.n_val) + t) * kHeadDim;
+  });
+  LossState sM, sR;
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int64_t j = j0 + u;
-      if (j < m) {
-        const int64_t pos = j < keep ? top[j] : (p.s - p.recent) + (j - keep);
-        kw[u] = __ldg(reinterpret_cast<const uint2*>(Ku + pos * kHeadDim));
-        vw[u] = __ldg(reinterpret_cast<const uint2*>(Vu + pos * kHeadDim));
+  for (int i = 0; i < 4; ++i) {
+    sM.m[i] = sR.m[i] = -INFINITY;
+    sM.l[i] = sR.l[i] = 0.f;
+#pragma unroll
+    for (int d = 0; d < 4; ++d) sM.acc[i][d] = sR.acc[i][d] = 0.f;
+  }
+  const __nv_bfloat16* Ku = p.K + int64_t(ul) * p.s * kHeadDim;
+  const __nv_bfloat16* Vu = p.V + int64_t(ul) * p.s * kHeadDim;
+  const int32_t* top = p.top + int64_t(ul) * p.n_top;
+  // main slots: the ranked tokens kept, then the recent window
+  for (int64_t j0 = 0; j0 < m; j0 += kTile) {
+    auto pos = [&](int tok) -> int64_t {
+      const int64_t j = j0 + tok;
+      return j >= m ? -1 : (j < keep ? top[j] : (p.s - p.recent) + (j - keep));
+    };
+    __syncthreads();
+    load_rows_kt(Kt, [&](int tok) {
+      const int64_t q = pos(tok);
+      return q < 0 ? static_cast<const __nv_bfloat16*>(nullptr) : Ku + q * kHeadDim;
+    });
+    load_rows_v(Vs, [&](int tok) {
+      const int64_t q = pos(tok);
+      return q < 0 ? static_cast<const __nv_bfloat16*>(nullptr) : Vu + q * kHeadDim;
+    });
+    __syncthreads();
+    float bias[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) bias[j] = j0 + 4 * lane + j < m ? 0.f : -INFINITY;
+    loss_tile(Qt, Kt, Vs, Pt, bias, sM);
+  }
+  // residual entries: logit + beta ln c (log2 units); an empty entry is inert
+  const int64_t e0 = int64_t(ul) * p.ent_stride + p.ent_off;
+  for (int j0 = 0; j0 < r; j0 += kTile) {
+    __syncthreads();
+    load_rows_kt(Kt, [&](int tok) {
+      return j0 + tok < r ? p.kbar + (e0 + j0 + tok) * kHeadDim : static_cast<const __nv_bfloat16*>(nullptr);
+    });
+    load_rows_v(Vs, [&](int tok) {
+      return j0 + tok < r ? p.vbar + (e0 + j0 + tok) * kHeadDim : static_cast<const __nv_bfloat16*>(nullptr);
+    });
+    __syncthreads();
+    float bias[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int e = j0 + 4 * lane + j;
+      const int c = e < r ? p.ecount[e0 + e] : 0;
+      bias[j] = c > 0 ? p.beta * logf(float(c)) * kLog2e : -INFINITY;
+    }
+    loss_tile(Qt, Kt, Vs, Pt, bias, sR);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int row = rb + 4 * w + i;
+    float g_val = p.g_fixed;
+    if (p.gate_mode == RESKV_GATE_DYNAMIC) {
+      const float pmax = 1.0f / sM.l[i];
+      g_val = fmaxf(p.g_min, 1.0f / (1.0f + expf(-p.alpha * (p.tau - pmax))));
+    }
+    const float2 coef = branch_coefs(p.softmax_mode, g_val, sM.m[i], sM.l[i], sR.m[i], sR.l[i]);
+    float e = 0.f;
+    if (row < p.n_rows) {
+      const float* os = p.oS + (int64_t(ul) * p.n_rows + row) * kHeadDim + 4 * lane;
+#pragma unroll
+      for (int d = 0; d < 4; ++d) {
+        const float o = coef.x * sM.acc[i][d] + coef.y * sR.acc[i][d];
+        const float df = o - os[d];
+        e += df * df;
       }
     }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      if (j0 + u >= m) break;
-      const float2 k01 = bf16x2_to_float2(kw[u].x), k23 = bf16x2_to_float2(kw[u].y);
-      const float a = warp_sum(q[0] * k01.x + q[1] * k01.y + q[2] * k23.x + q[3] * k23.y);
-      const float mn = fmaxf(mM, a);
-      const float sc = exp2f(mM - mn), pr = exp2f(a - mn);
-      const float2 v01 = bf16x2_to_float2(vw[u].x), v23 = bf16x2_to_float2(vw[u].y);
-      lM = lM * sc + pr;
-      aM[0] = aM[0] * sc + pr * v01.x;
-      aM[1] = aM[1] * sc + pr * v01.y;
-      aM[2] = aM[2] * sc + pr * v23.x;
-      aM[3] = aM[3] * sc + pr * v23.y;
-      mM = mn;
-    }
+    e = warp_sum(e);
+    if (lane == 0 && row < p.n_rows) p.rowerr[int64_t(ul) * p.n_rows + row] = double(e);
   }
-  // residual entries: logit + beta*log c (log2 units); gate applied below
-  float mR = -INFINITY, lR = 0.f, aR[4] = {0.f, 0.f, 0.f, 0.f};
-  const int64_t e0 = int64_t(ul) * p.ent_stride + p.ent_off;
-  for (int j = 0; j < r; ++j) {
-    const int c = p.ecount[e0 + j];
-    if (c <= 0) continue;
-    const uint2 kw = *reinterpret_cast<const uint2*>(p.kbar + (e0 + j) * kHeadDim + 4 * lane);
-    const uint2 vw = *reinterpret_cast<const uint2*>(p.vbar + (e0 + j) * kHeadDim + 4 * lane);
-    const float2 k01 = bf16x2_to_float2(kw.x), k23 = bf16x2_to_float2(kw.y);
-    const float a = warp_sum(q[0] * k01.x + q[1] * k01.y + q[2] * k23.x + q[3] * k23.y) +
-                    p.beta * logf(float(c)) * kLog2e;
-    const float mn = fmaxf(mR, a);
-    const float sc = exp2f(mR - mn), pr = exp2f(a - mn);
-    const float2 v01 = bf16x2_to_float2(vw.x), v23 = bf16x2_to_float2(vw.y);
-    lR = lR * sc + pr;
-    aR[0] = aR[0] * sc + pr * v01.x;
-    aR[1] = aR[1] * sc + pr * v01.y;
-    aR[2] = aR[2] * sc + pr * v23.x;
-    aR[3] = aR[3] * sc + pr * v23.y;
-    mR = mn;
-  }
-  float g_val = p.g_fixed;
-  if (p.gate_mode == RESKV_GATE_DYNAMIC) {
-    const float pmax = 1.0f / lM;
-    g_val = fmaxf(p.g_min, 1.0f / (1.0f + expf(-p.alpha * (p.tau - pmax))));
-  }
-  const float2 coef = branch_coefs(p.softmax_mode, g_val, mM, lM, mR, lR);
-  const float* os = p.oS + (int64_t(ul) * p.n_rows + row) * kHeadDim + 4 * lane;
-  float e = 0.f;
-#pragma unroll
-  for (int d = 0; d < 4; ++d) {
-    const float o = coef.x * aM[d] + coef.y * aR[d];
-    const float df = o - os[d];
-    e += df * df;
-  }
-  e = warp_sum(e);
-  if (lane == 0) p.rowerr[int64_t(ul) * p.n_rows + row] = double(e);
 }
 
 // L_r = mean of the per-query errors (rows in order, fp64); +inf for a unit
