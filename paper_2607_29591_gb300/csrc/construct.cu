@@ -381,12 +381,11 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
   const size_t sm_obs2 = sm_obs1 + size_t(kThreads / 32) * kTile * 4;  // + per-warp sums
   const size_t sm_top = size_t(kTopMax) * 12 + (256 + 32 + 4) * 4;
   const size_t sm_assign = lloyd_tc_smem(rmax);
-  const size_t sm_val = size_t(kHeadDim) * (2 * kTile + 2 * kRowBlk) * 4;
   if (set_smem(k_obs_pass1, sm_obs1) != cudaSuccess || set_smem(k_obs_pass2, sm_obs2) != cudaSuccess ||
       set_smem(k_topk, sm_top) != cudaSuccess || set_smem(k_lloyd_assign_tc, sm_assign) != cudaSuccess ||
       set_smem(k_lloyd_assign_pt, kPtSmemMax) != cudaSuccess ||
-      set_smem(k_val_loss, sm_val) != cudaSuccess ||
-      set_smem(k_val_full, sm_val) != cudaSuccess)
+      set_smem(k_val_loss, kValSmem) != cudaSuccess ||
+      set_smem(k_val_full, kValSmem) != cudaSuccess)
     return cleanup_fail(fail(RESKV_ERR_CUDA, "setting kernel shared-memory limits"));
 
   const double one_minus_delta = 1.0 - double(cfg.delta);
@@ -537,7 +536,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
       // ---- validation targets, candidates, choice of r ----
       timing_ok &= timer.mark(kStValTargets);
       ValArgs va{K, V, Q, s, G, cfg.n_obs, cfg.n_val, n_val_rows, nchunks, vpart, oS};
-      k_val_full<<<dim3(nchunks, unsigned(cdiv(n_val_rows, kRowBlk)), UL), kThreads, sm_val, stream>>>(va);
+      k_val_full<<<dim3(nchunks, unsigned(cdiv(n_val_rows, kRowBlk)), UL), kThreads, kValSmem, stream>>>(va);
       k_val_combine<<<dim3(n_val_rows, UL), kHeadDim, 0, stream>>>(va);
       RESKV_LAUNCH_CHECK("validation targets");
       for (int run = 0; run < ncol; ++run) {
@@ -559,7 +558,7 @@ reskv_status build_all_layers(reskv_cache** out, const reskv_config& cfg,
                     kbar, vbar, ecount, ent_stride, run_off[run], cfg.beta, cfg.gate_mode,
                     cfg.tau, cfg.alpha, cfg.g_min, cfg.g_fixed, oS, rowerr, cfg.softmax_mode,
                     bl_d};
-        k_val_loss<<<dim3(unsigned(cdiv(n_val_rows, kRowBlk)), UL), kThreads, sm_val, stream>>>(lo);
+        k_val_loss<<<dim3(unsigned(cdiv(n_val_rows, kRowBlk)), UL), kThreads, kValSmem, stream>>>(lo);
         k_loss_reduce<<<unsigned(cdiv(UL, 128)), 128, 0, stream>>>(rowerr, losses, n_val_rows, UL,
                                                                   ncol, run, r_unit);
         RESKV_LAUNCH_CHECK("validation loss");

@@ -1280,17 +1280,107 @@ __device__ __forceinline__ const __nv_bfloat16* val_row(const ValArgs& p, int ul
   return p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + (p.n_obs - p.n_val) + t) * kHeadDim;
 }
 
+// Shared memory of the validation kernels (k_val_full, k_val_loss): the key
+// tile (bf16, 256-byte rows with the 16-byte chunks XOR-swizzled for
+// ldmatrix), the value tile (bf16 rows), the logits of the CTA's 32 query rows
+// (fp32, rows padded to 136 floats: the fragment stores are conflict free)
+// and P^T (fp32, swizzled).  Under 113 KB: two CTAs per SM.
+constexpr int kValSRow = kTile + 8;
+constexpr size_t kValOffV = size_t(kTile) * kAsgRowBytes;
+constexpr size_t kValOffS = kValOffV + size_t(kTile) * kAsgRowBytes;
+constexpr size_t kValOffP = kValOffS + size_t(kRowBlk) * kValSRow * 4;
+constexpr size_t kValSmem = kValOffP + size_t(kTile) * kRowBlk * 4;
+
+// A fragments (m16n8k16) of 16 query rows: row g and g + 8 of lane g = lane / 4
+// from rowptr(i) (nullptr: a zero row), unscaled bf16
+template <typename RowPtr>
+__device__ __forceinline__ void val_afrag(RowPtr rowptr, int lane, uint32_t (&A)[8][4]) {
+  const int g = lane >> 2, t4 = lane & 3;
+  const uint32_t* q0 = reinterpret_cast<const uint32_t*>(rowptr(g));
+  const uint32_t* q1 = reinterpret_cast<const uint32_t*>(rowptr(g + 8));
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    A[ks][0] = q0 ? __ldg(q0 + 8 * ks + t4) : 0u;
+    A[ks][1] = q1 ? __ldg(q1 + 8 * ks + t4) : 0u;
+    A[ks][2] = q0 ? __ldg(q0 + 8 * ks + 4 + t4) : 0u;
+    A[ks][3] = q1 ? __ldg(q1 + 8 * ks + 4 + t4) : 0u;
+  }
+}
+
+// The scaled logits (log2 domain) of the CTA's 32 rows against the staged key
+// tile into St: warp w < 4 takes rows 16 (w / 2).. and tokens 64 (w % 2)..
+// (tensor cores: exact bf16 products, fp32 sums); the other warps wait.
+__device__ __forceinline__ void val_tile_logits(uint32_t ks_s, const uint32_t (&A)[8][4], float* St) {
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (w >= 4) return;
+  float S[8][4];
+  obs_half_logits(ks_s, w & 1, lane, A, S);
+  const int g = lane >> 2, t4 = lane & 3, r0 = 16 * (w >> 1) + g;
+#pragma unroll
+  for (int nt = 0; nt < 8; ++nt) {
+    const int tk = 64 * (w & 1) + 8 * nt + 2 * t4;
+    *reinterpret_cast<float2*>(St + r0 * kValSRow + tk) = make_float2(S[nt][0], S[nt][1]);
+    *reinterpret_cast<float2*>(St + (r0 + 8) * kValSRow + tk) = make_float2(S[nt][2], S[nt][3]);
+  }
+}
+
+// this thread's logits: rows 4w..4w+3, tokens 4l..4l+3
+__device__ __forceinline__ void val_read_logits(const float* St, float (&S)[4][4]) {
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float4 v = *reinterpret_cast<const float4*>(St + (4 * w + i) * kValSRow + 4 * lane);
+    S[i][0] = v.x;
+    S[i][1] = v.y;
+    S[i][2] = v.z;
+    S[i][3] = v.w;
+  }
+}
+
+// 128 rows of 256 bytes into a bf16 tile (rows swizzled for ldmatrix or
+// plain) by cp.async, one 16-byte chunk per copy; rowptr(i) = nullptr: zeros
+// (the copy then reads nothing from `any`, a valid global address)
+template <bool swz, typename RowPtr>
+__device__ __forceinline__ void val_stage_rows(uint32_t dst, RowPtr rowptr, const __nv_bfloat16* any) {
+  for (int idx = threadIdx.x; idx < kTile * 16; idx += blockDim.x) {
+    const int row = idx >> 4, ch = idx & 15;
+    const __nv_bfloat16* src = rowptr(row);
+    cp_async16(dst + (swz ? asg_swz(row, ch) : uint32_t(row * kAsgRowBytes + ch * 16)),
+               src ? src + 8 * ch : any, src ? 16u : 0u);
+  }
+}
+
+// acc[i][d] += P^T[tok][row 4w + i] * V[tok][dim 4l + d] over the tile
+__device__ __forceinline__ void val_pv(const float* Pt, const __nv_bfloat16* Vb, float (&acc)[4][4]) {
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+#pragma unroll 4
+  for (int tok = 0; tok < kTile; ++tok) {
+    const float4 pp = *reinterpret_cast<const float4*>(Pt + tok * kRowBlk + ((w ^ ((tok >> 2) & 7)) << 2));
+    const uint2 vw = *reinterpret_cast<const uint2*>(Vb + tok * kHeadDim + 4 * lane);
+    const float2 v01 = bf16x2_to_float2(vw.x), v23 = bf16x2_to_float2(vw.y);
+    const float pa[4] = {pp.x, pp.y, pp.z, pp.w};
+    const float va[4] = {v01.x, v01.y, v23.x, v23.y};
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int d = 0; d < 4; ++d) acc[i][d] = fmaf(pa[i], va[d], acc[i][d]);
+  }
+}
+
 // o_S(q) over all s tokens for the validation queries (Eq. attn), per chunk
-__global__ void __launch_bounds__(kThreads, 1) k_val_full(ValArgs p) {
-  extern __shared__ __align__(16) float sm[];
-  float* Kt = sm;                               // [128][128] swizzled
-  float* Vs = Kt + kHeadDim * kTile;            // [128 tok][128 d]
-  float* Qt = Vs + kHeadDim * kTile;            // [128][32]
-  float* Pt = Qt + kHeadDim * kRowBlk;          // [128 tok][32 rows] swizzled
+__global__ void __launch_bounds__(kThreads, 2) k_val_full(ValArgs p) {
+  extern __shared__ __align__(1024) uint8_t vraw[];
+  const uint32_t ks_s = smem_u32(vraw), vb_s = ks_s + uint32_t(kValOffV);
+  const __nv_bfloat16* Vb = reinterpret_cast<const __nv_bfloat16*>(vraw + kValOffV);
+  float* St = reinterpret_cast<float*>(vraw + kValOffS);
+  float* Pt = reinterpret_cast<float*>(vraw + kValOffP);
   const int chunk = blockIdx.x, rb = blockIdx.y * kRowBlk, ul = blockIdx.z;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const float scale = kLog2e * rsqrtf(float(kHeadDim));
-  load_qt(Qt, min(kRowBlk, p.n_rows - rb), scale, [&](int r) { return val_row(p, ul, rb + r); });
+  uint32_t A[8][4];
+  if (w < 4) {
+    const int r16 = rb + 16 * (w >> 1);
+    val_afrag([&](int i) { return r16 + i < p.n_rows ? val_row(p, ul, r16 + i) : nullptr; }, lane, A);
+  }
   float m[4], l[4], acc[4][4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
@@ -1305,20 +1395,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_val_full(ValArgs p) {
     const int64_t tok0 = (int64_t(chunk) * kValChunkTiles + tt) * kTile;
     if (tok0 >= p.s) break;
     __syncthreads();
-    load_kt(Kt, Ku, p.s, tok0);
-    for (int it = 0; it < 8; ++it) {
-      const int idx = it * kThreads + threadIdx.x;
-      const int tok = idx >> 4, dc = idx & 15;
-      uint4 v = make_uint4(0, 0, 0, 0);
-      if (tok0 + tok < p.s) v = __ldg(reinterpret_cast<const uint4*>(Vu + (tok0 + tok) * kHeadDim) + dc);
-      const float2 a = bf16x2_to_float2(v.x), b = bf16x2_to_float2(v.y);
-      const float2 c = bf16x2_to_float2(v.z), d = bf16x2_to_float2(v.w);
-      *reinterpret_cast<float4*>(Vs + tok * kHeadDim + 8 * dc) = make_float4(a.x, a.y, b.x, b.y);
-      *reinterpret_cast<float4*>(Vs + tok * kHeadDim + 8 * dc + 4) = make_float4(c.x, c.y, d.x, d.y);
-    }
+    auto krow = [&](int i) { return tok0 + i < p.s ? Ku + (tok0 + i) * kHeadDim : nullptr; };
+    auto vrow = [&](int i) { return tok0 + i < p.s ? Vu + (tok0 + i) * kHeadDim : nullptr; };
+    val_stage_rows<true>(ks_s, krow, Ku);
+    val_stage_rows<false>(vb_s, vrow, Vu);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    val_tile_logits(ks_s, A, St);
     __syncthreads();
     float S[4][4];
-    tile_logits(Qt, Kt, S);
+    val_read_logits(St, S);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       float tmax = -INFINITY;
@@ -1350,17 +1437,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_val_full(ValArgs p) {
           make_float4(S[0][j], S[1][j], S[2][j], S[3][j]);
     }
     __syncthreads();
-#pragma unroll 4
-    for (int tok = 0; tok < kTile; ++tok) {
-      const float4 pp = *reinterpret_cast<const float4*>(Pt + tok * kRowBlk + ((w ^ ((tok >> 2) & 7)) << 2));
-      const float4 vv = *reinterpret_cast<const float4*>(Vs + tok * kHeadDim + 4 * lane);
-      const float pa[4] = {pp.x, pp.y, pp.z, pp.w};
-      const float va[4] = {vv.x, vv.y, vv.z, vv.w};
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int d = 0; d < 4; ++d) acc[i][d] = fmaf(pa[i], va[d], acc[i][d]);
-    }
+    val_pv(Pt, Vb, acc);
   }
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
@@ -1417,56 +1494,22 @@ struct LossArgs {
 
 // ||o^(r)(q) - o_S(q)||^2 per validation query, with the decode rule of
 // Sec. 5.4 and the gate.  Tiled like k_val_full: a CTA takes 32 query rows of
-// a unit (warp w: rows 4w..4w+3; lane l: tokens 4l..4l+3 of a 128-token tile
-// for the logits, dims 4l..4l+3 for the outputs) and walks the candidate's
-// main slots (the kept ranked tokens, then the recent window), then its
-// residual entries (logit + beta ln c), each gathered into shared memory
-// once for all 32 rows, with one online-softmax state per branch.
-// Dynamic shared memory: that of k_val_full.
+// a unit and walks the candidate's main slots (the kept ranked tokens, then
+// the recent window), then its residual entries (logit + beta ln c), each
+// gathered into shared memory once for all 32 rows (logits on the tensor
+// cores), with one online-softmax state per branch.  Dynamic shared memory:
+// kValSmem.
 struct LossState {
   float m[4], l[4], acc[4][4];
 };
 
-template <class RowPtr>
-__device__ __forceinline__ void load_rows_kt(float* Kt, RowPtr rowptr) {
-  for (int it = 0; it < 8; ++it) {
-    const int idx = it * kThreads + threadIdx.x;
-    const int tok = idx >> 4, dc = idx & 15;
-    const __nv_bfloat16* src = rowptr(tok);
-    uint4 w = make_uint4(0, 0, 0, 0);
-    if (src) w = __ldg(reinterpret_cast<const uint4*>(src) + dc);
-    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float2 f = bf16x2_to_float2(ws[j]);
-      Kt[kt_index(8 * dc + 2 * j, tok)] = f.x;
-      Kt[kt_index(8 * dc + 2 * j + 1, tok)] = f.y;
-    }
-  }
-}
-
-template <class RowPtr>
-__device__ __forceinline__ void load_rows_v(float* Vs, RowPtr rowptr) {
-  for (int it = 0; it < 8; ++it) {
-    const int idx = it * kThreads + threadIdx.x;
-    const int tok = idx >> 4, dc = idx & 15;
-    const __nv_bfloat16* src = rowptr(tok);
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (src) v = __ldg(reinterpret_cast<const uint4*>(src) + dc);
-    const float2 a = bf16x2_to_float2(v.x), b = bf16x2_to_float2(v.y);
-    const float2 c = bf16x2_to_float2(v.z), d = bf16x2_to_float2(v.w);
-    *reinterpret_cast<float4*>(Vs + tok * kHeadDim + 8 * dc) = make_float4(a.x, a.y, b.x, b.y);
-    *reinterpret_cast<float4*>(Vs + tok * kHeadDim + 8 * dc + 4) = make_float4(c.x, c.y, d.x, d.y);
-  }
-}
-
-// One 128-token tile (K in Kt, V in Vs) into state st: logits + bias[j] for
-// this lane's tokens 4l + j (-inf: no token)
-__device__ __forceinline__ void loss_tile(const float* Qt, const float* Kt, const float* Vs, float* Pt,
+// One 128-token tile (logits in St, V in Vb) into state st: logits + bias[j]
+// for this lane's tokens 4l + j (-inf: no token)
+__device__ __forceinline__ void loss_tile(const float* St, float* Pt, const __nv_bfloat16* Vb,
                                           const float (&bias)[4], LossState& st) {
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   float S[4][4];
-  tile_logits(Qt, Kt, S);
+  val_read_logits(St, S);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     float tmax = -INFINITY;
@@ -1498,36 +1541,31 @@ __device__ __forceinline__ void loss_tile(const float* Qt, const float* Kt, cons
         make_float4(S[0][j], S[1][j], S[2][j], S[3][j]);
   }
   __syncthreads();
-#pragma unroll 4
-  for (int tok = 0; tok < kTile; ++tok) {
-    const float4 pp = *reinterpret_cast<const float4*>(Pt + tok * kRowBlk + ((w ^ ((tok >> 2) & 7)) << 2));
-    const float4 vv = *reinterpret_cast<const float4*>(Vs + tok * kHeadDim + 4 * lane);
-    const float pa[4] = {pp.x, pp.y, pp.z, pp.w};
-    const float va[4] = {vv.x, vv.y, vv.z, vv.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-      for (int d = 0; d < 4; ++d) st.acc[i][d] = fmaf(pa[i], va[d], st.acc[i][d]);
-  }
+  val_pv(Pt, Vb, st.acc);
 }
 
 __global__ void __launch_bounds__(kThreads, 1) k_val_loss(LossArgs p) {
-  extern __shared__ __align__(16) float sm[];
-  float* Kt = sm;                               // [128][128] swizzled
-  float* Vs = Kt + kHeadDim * kTile;            // [128 tok][128 d]
-  float* Qt = Vs + kHeadDim * kTile;            // [128][32]
-  float* Pt = Qt + kHeadDim * kRowBlk;          // [128 tok][32 rows] swizzled
+  extern __shared__ __align__(1024) uint8_t vraw[];
+  const uint32_t ks_s = smem_u32(vraw), vb_s = ks_s + uint32_t(kValOffV);
+  const __nv_bfloat16* Vb = reinterpret_cast<const __nv_bfloat16*>(vraw + kValOffV);
+  float* St = reinterpret_cast<float*>(vraw + kValOffS);
+  float* Pt = reinterpret_cast<float*>(vraw + kValOffP);
   const int rb = blockIdx.x * kRowBlk, ul = blockIdx.y;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = p.r_unit[ul];
   const int64_t bu = unit_budget(p.budgets, ul, p.budget);
   const int64_t m = r == 0 ? (bu < p.s ? bu : p.s) : bu - r;
   const int64_t keep = m - p.recent;
-  const float scale = kLog2e * rsqrtf(float(kHeadDim));
-  load_qt(Qt, min(kRowBlk, p.n_rows - rb), scale, [&](int row) {
-    const int g = (rb + row) / p.n_val, t = (rb + row) % p.n_val;
-    return p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + (p.n_obs - p.n_val) + t) * kHeadDim;
-  });
+  uint32_t A[8][4];
+  if (w < 4) {
+    const int r16 = rb + 16 * (w >> 1);
+    val_afrag([&](int i) -> const __nv_bfloat16* {
+      const int row = r16 + i;
+      if (row >= p.n_rows) return nullptr;
+      const int g = row / p.n_val, t = row % p.n_val;
+      return p.Qobs + ((int64_t(ul) * p.G + g) * p.n_obs + (p.n_obs - p.n_val) + t) * kHeadDim;
+    }, lane, A);
+  }
   LossState sM, sR;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
@@ -1546,30 +1584,38 @@ __global__ void __launch_bounds__(kThreads, 1) k_val_loss(LossArgs p) {
       return j >= m ? -1 : (j < keep ? top[j] : (p.s - p.recent) + (j - keep));
     };
     __syncthreads();
-    load_rows_kt(Kt, [&](int tok) {
+    val_stage_rows<true>(ks_s, [&](int tok) {
       const int64_t q = pos(tok);
       return q < 0 ? static_cast<const __nv_bfloat16*>(nullptr) : Ku + q * kHeadDim;
-    });
-    load_rows_v(Vs, [&](int tok) {
+    }, Ku);
+    val_stage_rows<false>(vb_s, [&](int tok) {
       const int64_t q = pos(tok);
       return q < 0 ? static_cast<const __nv_bfloat16*>(nullptr) : Vu + q * kHeadDim;
-    });
+    }, Vu);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    val_tile_logits(ks_s, A, St);
     __syncthreads();
     float bias[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) bias[j] = j0 + 4 * lane + j < m ? 0.f : -INFINITY;
-    loss_tile(Qt, Kt, Vs, Pt, bias, sM);
+    loss_tile(St, Pt, Vb, bias, sM);
   }
   // residual entries: logit + beta ln c (log2 units); an empty entry is inert
   const int64_t e0 = int64_t(ul) * p.ent_stride + p.ent_off;
   for (int j0 = 0; j0 < r; j0 += kTile) {
     __syncthreads();
-    load_rows_kt(Kt, [&](int tok) {
+    val_stage_rows<true>(ks_s, [&](int tok) {
       return j0 + tok < r ? p.kbar + (e0 + j0 + tok) * kHeadDim : static_cast<const __nv_bfloat16*>(nullptr);
-    });
-    load_rows_v(Vs, [&](int tok) {
+    }, Ku);
+    val_stage_rows<false>(vb_s, [&](int tok) {
       return j0 + tok < r ? p.vbar + (e0 + j0 + tok) * kHeadDim : static_cast<const __nv_bfloat16*>(nullptr);
-    });
+    }, Vu);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    val_tile_logits(ks_s, A, St);
     __syncthreads();
     float bias[4];
 #pragma unroll
@@ -1578,7 +1624,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_val_loss(LossArgs p) {
       const int c = e < r ? p.ecount[e0 + e] : 0;
       bias[j] = c > 0 ? p.beta * logf(float(c)) * kLog2e : -INFINITY;
     }
-    loss_tile(Qt, Kt, Vs, Pt, bias, sR);
+    loss_tile(St, Pt, Vb, bias, sR);
   }
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
