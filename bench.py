@@ -61,6 +61,9 @@ def parse_args():
                     choices=["none"] + sorted(wl.WORKLOADS),
                     help="a second workload measured the same way (no e2e leg), reported "
                          "under second_workload")
+    ap.add_argument("--comparison", default="lse", choices=["lse", "none"],
+                    help="also time the paper's decode structure (main pass, residual pass, "
+                         "log-sum-exp merge) on the main workload, reported under comparison")
     ap.add_argument("--decode-kernel", choices=["auto", "mma", "cluster", "fma", "lse"],
                     default="auto",
                     help="automatic plan (default: cluster kernel for launches whose units "
@@ -670,6 +673,19 @@ def main():
                          with_e2e=False)
         second["clocks"] = clk2.summary()
 
+    comparison = None
+    if args.comparison == "lse" and not args.layers and kern != R.RESKV_DECODE_LSE_MERGE:
+        # the same cache built again, decoded the paper's way (3 launches per call)
+        cmp = measure(args, w, R, R.RESKV_DECODE_LSE_MERGE, bmode, device, world, peak, peak_kind,
+                      clk=None, with_e2e=False)
+        comparison = {
+            "what": "paper-style decode: main-cache pass, residual pass and a log-sum-exp merge "
+                    "kernel per call (Sec. 6.1; App. B), same workload, same roofline bytes",
+            "per_layer": {k: cmp["per_layer"][k] for k in ("us_per_layer_step", "tokens_per_s")},
+            "per_layer_frac": cmp["per_layer"]["roofline"]["frac"],
+            "all_layer": {k: cmp["all_layer"][k] for k in ("us_per_layer_step", "tokens_per_s")},
+            "all_layer_frac": cmp["all_layer"]["roofline"]["frac"]}
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w)
@@ -701,6 +717,8 @@ def main():
                 "all_layer_launch": second["all_layer"], "construction_s": second["construction_s"],
                 "construction_stages_ms": second["construction_stages_ms"],
                 "clocks": second["clocks"], "steps": args.steps, "warmup": args.warmup}
+        if comparison is not None:
+            line["comparison"] = comparison
         print(json.dumps(line), flush=True)
 
 
