@@ -18,21 +18,26 @@
 //                    norms, then stages the new planes (cp.async).
 //   8 column warps   warp w reads TMEM lanes 32 (w % 4).. (its tokens) and the
 //                    16-column chunks w / 4, w / 4 + 2, .. of the distances,
-//                    keeping two top-3 lists per thread (even and odd columns:
-//                    independent dependency chains), frees the TMEM buffer
-//                    (tmem_empty[]), merges the two column halves and posts the
-//                    tile's lists in a ring of kPtRing slots (list_full[]).
-//   4 certifier      certify each token's choice and re-evaluate ambiguous
-//   warps            tokens in fp64 as the streaming kernel does (keys from
-//                    global memory, key norms precomputed per layer), write
-//                    assign, count members per centre and write the tile's
-//                    counts, then free the slot (list_empty[]).
+//                    keeping each token's best three as fp32 keys with the
+//                    centre index in the low 8 significand bits (two lists
+//                    per thread, even and odd columns, each a fminf/fmaxf
+//                    network), frees the TMEM buffer (tmem_empty[]), merges
+//                    the two column halves and posts the tile's lists, with
+//                    each token's rank and key norm, in a ring of kPtRing
+//                    slots (list_full[]).
+//   4 certifier      decide each evicted token from a rigorous bound on the
+//   warps            tensor-core distance error: the best centre is certified,
+//                    or the token joins a list that k_lloyd_resolve decides
+//                    (direct fp32 distances, then fp64 where those still
+//                    overlap).  They write assign, count the certified members
+//                    per centre, write the tile's counts and free the slot
+//                    (list_empty[]).
 //
-// fp64 is slow on this part; with its own warps and a ring in between, a
-// tile whose tokens need many fp64 distances delays the column warps only
-// once the ring is full.  Every wait is bounded; a wait that gives up raises
-// kStatusWaitTimeout and an abort flag, and each role leaves its loop at a
-// tile boundary agreed by a barrier reduction over the role's threads.
+// Certification needs no global memory and no fp64 (scarce on this part),
+// so the certifiers keep pace with the column warps.  Every wait is bounded;
+// a wait that gives up raises kStatusWaitTimeout and an abort flag, and each
+// role leaves its loop at a tile boundary agreed by a barrier reduction over
+// the role's threads.
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
