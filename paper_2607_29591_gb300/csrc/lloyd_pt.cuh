@@ -634,21 +634,36 @@ __global__ void __launch_bounds__(kResWarps * 32) k_lloyd_resolve(LloydArgs p) {
     const float2 k01 = bf16x2_to_float2(kw.x), k23 = bf16x2_to_float2(kw.y);
     const float* c32 = p.centers32 + int64_t(u) * p.rmax * kHeadDim + 4 * lane;
     const float* cnu = p.cnorm + int64_t(u) * p.rmax;
-    // fp32 distances, four centres at a time
-    for (int k0 = 0; k0 < nc; k0 += 4) {
-      float a[4];
+    // fp32 distances, eight centres at a time: a 4-term chain per lane, then
+    // a transposed butterfly (9 shuffles) that leaves centre 4 b4 + 2 b3 + b2
+    // (b_i: bit i of the lane) summed over all lanes -- five levels of adds,
+    // as the bound assumes
+    const int b4 = (lane >> 4) & 1, b3 = (lane >> 3) & 1, b2 = (lane >> 2) & 1;
+    for (int k0 = 0; k0 < nc; k0 += 8) {
+      float a[8];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
+      for (int q = 0; q < 8; ++q) {
         const int k = k0 + q < nc ? k0 + q : k0;
         const float4 c = *reinterpret_cast<const float4*>(c32 + int64_t(cand(k)) * kHeadDim);
         const float x0 = k01.x - c.x, x1 = k01.y - c.y, x2 = k23.x - c.z, x3 = k23.y - c.w;
         a[q] = fmaf(x3, x3, fmaf(x2, x2, fmaf(x1, x1, x0 * x0)));
       }
+      float bq[4], cq[2];
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1)
+      for (int i = 0; i < 4; ++i) {
+        const float send = b4 ? a[i] : a[i + 4];
+        bq[i] = (b4 ? a[i + 4] : a[i]) + __shfl_xor_sync(0xffffffffu, send, 16);
+      }
 #pragma unroll
-        for (int q = 0; q < 4; ++q) a[q] += __shfl_xor_sync(0xffffffffu, a[q], o);
-      if (lane < 4 && k0 + lane < nc) dl[k0 + lane] = lane == 0 ? a[0] : lane == 1 ? a[1] : lane == 2 ? a[2] : a[3];
+      for (int i = 0; i < 2; ++i) {
+        const float send = b3 ? bq[i] : bq[i + 2];
+        cq[i] = (b3 ? bq[i + 2] : bq[i]) + __shfl_xor_sync(0xffffffffu, send, 8);
+      }
+      float dq = (b2 ? cq[1] : cq[0]) + __shfl_xor_sync(0xffffffffu, b2 ? cq[0] : cq[1], 4);
+      dq += __shfl_xor_sync(0xffffffffu, dq, 2);
+      dq += __shfl_xor_sync(0xffffffffu, dq, 1);
+      const int v = 4 * b4 + 2 * b3 + b2;
+      if ((lane & 3) == 0 && k0 + v < nc) dl[k0 + v] = dq;
     }
     __syncwarp();
     // the fp32 best (distance, index)
