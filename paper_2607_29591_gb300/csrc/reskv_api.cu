@@ -565,11 +565,12 @@ reskv_status decode_layers(const reskv_cache* c, int32_t layer0, int32_t n_layer
     const int wpc = cp.cluster > 0 ? cp.warps_per_cta : cluster_warps(c->max_unit_slots, 1);
     p.n_warps = int32_t(int64_t(cs) * wpc);
     // ring depth: as deep as shared memory allows, but 2 stages per warp in
-    // clusters of 4 or more CTAs (measured on one-layer launches of 32 units,
-    // b = 2048: 7.55 us against 7.64 with 3 stages; 2-CTA clusters at
-    // b = 1024 are fastest with 3)
+    // clusters of 2 or more CTAs (one-layer launches of 32 units, b = 2048,
+    // 4-CTA clusters: 7.55 us against 7.64 with 3 stages; of 64 units,
+    // b = 1024, 2-CTA clusters, alternating on one GPU: 7.70-7.73 us against
+    // 7.74-7.76)
     p.n_stages = decode_cluster_stages(wpc, cs);
-    if (cs >= 4) p.n_stages = std::min(p.n_stages, 2);
+    if (cs >= 2) p.n_stages = std::min(p.n_stages, 2);
     cudaError_t err =
         kernel == RESKV_DECODE_CLUSTER
             ? launch_decode_cluster(p, c->tmap_k, c->tmap_v, cfg.group, cs, wpc,
